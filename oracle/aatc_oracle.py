@@ -1,0 +1,375 @@
+"""AATC oracle: a plain, slow, fp64 CPU restatement of the paper's method.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / reference leg of ``bench.py`` may import this module.  It shares
+no code with the CUDA library (``paper_2608_14191_gb300``) and imports nothing
+from it; the only shared module is ``workloads`` (seeded inputs, no method
+arithmetic).
+
+Every function cites the passage of arxiv 2608.14191 ("KV Cache Compression
+Through the Lens of Transform Coding") that it follows.  Floating point is fp64
+except :func:`dequantize_f32`, which spells out the two fp32 multiplies that
+define the stored-code reconstruction so that the GPU's can be checked bit for
+bit.
+
+Pins (tests/test_oracle_pins.py) tie each function to something other than
+itself: the transform round trip (Sec. 3.1), the reverse water-filling closed
+form (Eq. bit-allocation, Sec. 3.1), brute force over integer allocations at d=4
+(Eq. waterfilling-keys), a Monte Carlo check of Theorem 1, the whitening-SVD /
+PCA equivalence (Appendix, Proposition), the quantizer error bound
+(Def. uniform-quant), library SDPA for decode, hand-computed small cases and
+the compression ratio the paper prints (Sec. 6.1).
+
+parity unpinned: the packed record bit layout (:func:`pack_records`,
+:func:`cache_records`) is defined by this build, not by the paper, which prints
+no worked encoding.  It is pinned only by the round trip unpack(pack(c)) == c,
+the record-size identity (352 code bits per token and stream at 2.75 bits,
+i.e. the paper's 16/2.75 = 5.82x) and a hand-computed packed word.
+"""
+from __future__ import annotations
+
+import math
+import numpy as np
+
+D = 128
+TILE = 128          # tokens per word-planar tile of the packed cache
+
+
+# ----------------------------------------------------------------------------
+# Offline calibration (Sec. 5, Algorithm 1 calibration half, Appendix A.x)
+# ----------------------------------------------------------------------------
+
+def second_moment(x: np.ndarray) -> np.ndarray:
+    """Uncentered empirical second moment C = X^T X / N (Sec. 5 Step 1, Sigma_X = X^T X / T)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x.T @ x / x.shape[0]
+
+
+def canonical_sign(vectors: np.ndarray) -> np.ndarray:
+    """Flip each column so that its largest-magnitude entry (lowest index on ties) is positive.
+
+    The paper leaves eigenvector signs open; this is the build's convention.
+    """
+    v = np.array(vectors, dtype=np.float64, copy=True)
+    for j in range(v.shape[1]):
+        i = int(np.argmax(np.abs(v[:, j])))
+        if v[i, j] < 0:
+            v[:, j] = -v[:, j]
+    return v
+
+
+def eigenbasis(c: np.ndarray):
+    """Eigen-decomposition C = U diag(lam) U^T, eigenvalues descending (Sec. 3.1, KLT;
+    Appendix Proposition: the PCA of K = XW equals the whitening-SVD transform)."""
+    lam, vec = np.linalg.eigh(np.asarray(c, dtype=np.float64))
+    order = np.argsort(-lam, kind="stable")
+    return lam[order], canonical_sign(vec[:, order])
+
+
+def channel_variance(encode_basis: np.ndarray, x: np.ndarray) -> np.ndarray:
+    """sigma_c^2 = mean over calibration of h_c^2 with h = x A (Alg. 1 calibration, 'record latent
+    variance'; uncentered because the source is zero-mean, Sec. 3.1)."""
+    h = np.asarray(x, np.float64) @ encode_basis
+    return np.mean(h * h, axis=0)
+
+
+def key_weights(recon_rows: np.ndarray, queries_by_head) -> np.ndarray:
+    """w^K_c = sum over the query heads of the GQA group of (1/T) sum_i (B_c . q_i)^2
+    (Eq. waterfilling-keys; GQA remark in the appendix derivation).  ``recon_rows`` is B
+    (channel c reconstructs along row B_c); for an orthonormal basis B = U^T."""
+    b = np.asarray(recon_rows, np.float64)
+    w = np.zeros(b.shape[0])
+    for q in queries_by_head:
+        proj = np.asarray(q, np.float64) @ b.T          # (T, channels)
+        w += np.mean(proj * proj, axis=0)
+    return w
+
+
+def value_weights(recon_rows: np.ndarray, w_o: np.ndarray | None = None) -> np.ndarray:
+    """w^V_c = ||(B^V W_O)_c||^2 (Sec. 5 Step 2, values).  The decode path has no output
+    projection (Alg. 1 output line), so W_O = I by default and w^V_c = ||B_c||^2."""
+    b = np.asarray(recon_rows, np.float64)
+    m = b if w_o is None else b @ np.asarray(w_o, np.float64)
+    return np.sum(m * m, axis=1)
+
+
+def allocation_objective(g: np.ndarray, bits: np.ndarray) -> float:
+    """Weighted distortion surrogate sum_c g_c 2^(-2 b_c) (Eq. waterfilling-keys objective with
+    g_c = w_c sigma_c^2; the common constant gamma of Eq. noise-model drops out)."""
+    return float(np.sum(np.asarray(g, np.float64) * np.exp2(-2.0 * np.asarray(bits, np.float64))))
+
+
+def greedy_allocation(g: np.ndarray, budget: int, b_max: int) -> np.ndarray:
+    """Integer reverse water-filling: minimise sum_c g_c 4^(-b_c) s.t. sum b_c <= budget,
+    b_c in {0..b_max} (Eq. waterfilling-keys; Remark 'Zero-bit dimensions').
+
+    The objective is separable with convex, decreasing per-channel terms, so handing out
+    one bit at a time to the channel whose term drops the most is exactly optimal.  The
+    drop for channel c at b_c bits is (3/4) g_c 4^(-b_c); the 3/4 is common and omitted.
+    Ties go to the lowest channel index.
+    """
+    g = np.asarray(g, np.float64)
+    bits = np.zeros(len(g), dtype=np.int64)
+    for _ in range(int(budget)):
+        gain = np.where(bits < b_max, g * np.exp2(-2.0 * bits), -np.inf)
+        c = int(np.argmax(gain))
+        if not np.isfinite(gain[c]):
+            break
+        bits[c] += 1
+    return bits
+
+
+def continuous_allocation(g: np.ndarray, budget: float, b_max: float = np.inf):
+    """Continuous reverse water-filling (Eq. bit-allocation, weighted form of Sec. 5 Step 2):
+    b_c = clip(1/2 log2(g_c / theta), 0, b_max) with the water level theta chosen so that
+    sum_c b_c = budget.  Returns (bits, theta)."""
+    g = np.asarray(g, np.float64)
+
+    def total(log_theta):
+        return float(np.sum(np.clip(0.5 * (np.log2(g) - log_theta), 0.0, b_max)))
+
+    lo, hi = math.log2(g.min()) - 2 * 64, math.log2(g.max())
+    for _ in range(400):
+        mid = 0.5 * (lo + hi)
+        if total(mid) > budget:
+            lo = mid
+        else:
+            hi = mid
+    theta_log = 0.5 * (lo + hi)
+    return np.clip(0.5 * (np.log2(g) - theta_log), 0.0, b_max), 2.0 ** theta_log
+
+
+def percentile_linear(values: np.ndarray, p: float) -> float:
+    """Percentile with linear interpolation at rank (p/100)(N-1) of the sorted sample."""
+    a = np.sort(np.asarray(values, np.float64))
+    pos = (p / 100.0) * (len(a) - 1)
+    lo = int(math.floor(pos))
+    hi = min(lo + 1, len(a) - 1)
+    return float(a[lo] + (pos - lo) * (a[hi] - a[lo]))
+
+
+def channel_scales(encode_basis: np.ndarray, x: np.ndarray, p: float = 99.0) -> np.ndarray:
+    """s_c = 99th percentile of |h_c| over the calibration tokens (Sec. 5, 'The right scaling')."""
+    h = np.abs(np.asarray(x, np.float64) @ encode_basis)
+    return np.array([percentile_linear(h[:, c], p) for c in range(h.shape[1])])
+
+
+def plan_stream(x_calib: np.ndarray, avg_bits: float, b_max: int = 8, queries_by_head=None,
+                weights: str = "aatc"):
+    """Calibrate one stream (one layer, kv-head and K|V): Algorithm 1 calibration half with the
+    PCA eigenbasis standing in for the whitening-SVD transform (Appendix Proposition).
+
+    weights: 'aatc' (keys: query weights if queries_by_head is given; values: W_O = I) or
+    'var' (AATC var-only: w = 1, Sec. 6).
+    Channels are stored in descending order of g_c = w_c sigma_c^2 (stable), which makes the
+    bit widths non-increasing along storage order.
+    """
+    c = second_moment(x_calib)
+    lam, u = eigenbasis(c)
+    if weights == "var":
+        w = np.ones(D)
+    elif queries_by_head is not None:
+        w = key_weights(u.T, queries_by_head)
+    else:
+        w = value_weights(u.T)
+    g = w * lam
+    order = np.argsort(-g, kind="stable")
+    u, lam, w, g = u[:, order], lam[order], w[order], g[order]
+    budget = int(round(avg_bits * D))
+    bits = greedy_allocation(g, budget, b_max)
+    scales = channel_scales(u, x_calib)
+    return {"basis": u, "bits": bits, "scales": scales, "sigma2": lam, "weights": w, "g": g}
+
+
+# ----------------------------------------------------------------------------
+# Online encode (Algorithm 1 inference half: project, quantize, append)
+# ----------------------------------------------------------------------------
+
+def token_scale(h: np.ndarray, scales: np.ndarray, bits: np.ndarray) -> np.ndarray:
+    """alpha_t = max_c |h_c / s_c| over the retained channels (b_c >= 1) (Sec. 5, token scale)."""
+    keep = np.asarray(bits) > 0
+    return np.max(np.abs(h[:, keep]) / np.asarray(scales, np.float64)[keep], axis=1)
+
+
+def quantize(h: np.ndarray, alpha: np.ndarray, scales: np.ndarray, bits: np.ndarray):
+    """Symmetric uniform quantizer of Sec. 5: Delta = 2 alpha s_c / 2^b_c,
+    code = clamp(floor(h/Delta + 1/2), -2^(b-1), 2^(b-1) - 1).  Channels with b_c = 0 are
+    dropped (code 0).  Returns (codes, t = h/Delta) with t = 0 where alpha = 0."""
+    h = np.asarray(h, np.float64)
+    b = np.asarray(bits, np.int64)
+    s = np.asarray(scales, np.float64)
+    keep = b > 0
+    codes = np.zeros(h.shape, dtype=np.int64)
+    t = np.zeros(h.shape)
+    delta = 2.0 * alpha[:, None] * s[None, keep] / np.exp2(b[keep])[None, :]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        tk = np.where(delta > 0, h[:, keep] / np.where(delta > 0, delta, 1.0), 0.0)
+    lo = -np.exp2(b[keep] - 1)
+    hi = np.exp2(b[keep] - 1) - 1
+    codes[:, keep] = np.clip(np.floor(tk + 0.5), lo, hi).astype(np.int64)
+    t[:, keep] = tk
+    return codes, t
+
+
+def dequantize(codes: np.ndarray, alpha: np.ndarray, scales: np.ndarray, bits: np.ndarray):
+    """dqtz(c) = Delta c (Sec. 5), fp64."""
+    b = np.asarray(bits, np.int64)
+    delta = 2.0 * alpha[:, None] * np.asarray(scales, np.float64)[None, :] / np.exp2(b)[None, :]
+    return np.where(b[None, :] > 0, codes * delta, 0.0)
+
+
+def encode_stream(x: np.ndarray, encode_basis: np.ndarray, bits: np.ndarray, scales: np.ndarray):
+    """Project h = x A (Alg. 1 'Project'), per-token scale, quantize (Alg. 1 'Append qtz(h)').
+
+    Returns (codes (n,128) int, alpha (n,) fp64, t (n,128) = h/Delta)."""
+    h = np.asarray(x, np.float64) @ np.asarray(encode_basis, np.float64)
+    alpha = token_scale(h, scales, bits)
+    codes, t = quantize(h, alpha, scales, bits)
+    return codes, alpha, t
+
+
+def dequantize_f32(codes: np.ndarray, alpha_f32: np.ndarray, scales_f32: np.ndarray,
+                   bits: np.ndarray) -> np.ndarray:
+    """Stored-code reconstruction in fp32, two correctly rounded multiplies in this order:
+    f_c = s_c 2^(1-b_c) (exact), Delta = fl32(alpha f_c), h_hat = fl32(code Delta)
+    (Sec. 5 dqtz with Delta = 2 alpha s_c / 2^b_c)."""
+    b = np.asarray(bits, np.int64)
+    f = (np.asarray(scales_f32, np.float32) * np.exp2(1 - b).astype(np.float32)).astype(np.float32)
+    delta = (np.asarray(alpha_f32, np.float32)[:, None] * f[None, :]).astype(np.float32)
+    out = (np.asarray(codes).astype(np.float32) * delta).astype(np.float32)
+    return np.where(b[None, :] > 0, out, np.float32(0.0)).astype(np.float32)
+
+
+# ----------------------------------------------------------------------------
+# Packed layout (build-defined; the paper prints none)
+# ----------------------------------------------------------------------------
+
+def record_words(bits_per_stream) -> int:
+    """Words per record: W = ceil(max over streams of sum_c b_c / 32), at least 1."""
+    mx = max(int(np.sum(b)) for b in bits_per_stream)
+    return max(1, (mx + 31) // 32)
+
+
+def pack_records(codes: np.ndarray, bits: np.ndarray, n_words: int) -> np.ndarray:
+    """Offset-binary fields u_c = code_c + 2^(b_c - 1), LSB-first, in storage channel order,
+    allowed to straddle 32-bit words; unused bits zero.  Returns (n, n_words) uint32."""
+    b = np.asarray(bits, np.int64)
+    n = codes.shape[0]
+    acc = np.zeros((n, n_words + 1), dtype=np.uint64)
+    off = 0
+    for c in range(len(b)):
+        if b[c] == 0:
+            continue
+        u = (codes[:, c] + (1 << (b[c] - 1))).astype(np.uint64)
+        assert np.all(u < (1 << b[c]))
+        w, sh = off // 32, off % 32
+        acc[:, w] |= (u << np.uint64(sh)) & np.uint64(0xFFFFFFFF)
+        if sh + b[c] > 32:
+            acc[:, w + 1] |= u >> np.uint64(32 - sh)
+        off += int(b[c])
+    assert off <= 32 * n_words
+    return acc[:, :n_words].astype(np.uint32)
+
+
+def unpack_records(words: np.ndarray, bits: np.ndarray) -> np.ndarray:
+    """Inverse of :func:`pack_records`: (n, W) uint32 -> (n, 128) signed codes."""
+    b = np.asarray(bits, np.int64)
+    w64 = np.asarray(words).astype(np.uint64)
+    w64 = np.concatenate([w64, np.zeros((w64.shape[0], 1), np.uint64)], axis=1)
+    codes = np.zeros((w64.shape[0], len(b)), dtype=np.int64)
+    off = 0
+    for c in range(len(b)):
+        if b[c] == 0:
+            continue
+        w, sh = off // 32, off % 32
+        both = w64[:, w] | (w64[:, w + 1] << np.uint64(32))
+        u = (both >> np.uint64(sh)) & np.uint64((1 << b[c]) - 1)
+        codes[:, c] = u.astype(np.int64) - (1 << (b[c] - 1))
+        off += int(b[c])
+    return codes
+
+
+def cache_geometry(batch: int, n_kv_heads: int, max_tokens: int, n_words: int) -> dict:
+    """Per-layer packed cache: uint32 words [batch][H_kv][2][n_tiles][W][128], then fp32 alpha
+    [batch][H_kv][2][n_tiles*128].  Token t of a sequence sits in tile t // 128, lane t % 128."""
+    n_tiles = (max_tokens + TILE - 1) // TILE
+    n_word_elems = batch * n_kv_heads * 2 * n_tiles * n_words * TILE
+    n_alpha = batch * n_kv_heads * 2 * n_tiles * TILE
+    return {"n_tiles": n_tiles, "words": n_word_elems, "alpha": n_alpha,
+            "bytes": 4 * (n_word_elems + n_alpha)}
+
+
+def cache_records(cache_u32: np.ndarray, batch: int, n_kv_heads: int, max_tokens: int,
+                  n_words: int, b: int, head: int, kind: int, t0: int, n: int):
+    """Read (records (n, W) uint32, alpha (n,) float32) of one stream back out of a cache image."""
+    geo = cache_geometry(batch, n_kv_heads, max_tokens, n_words)
+    nt = geo["n_tiles"]
+    words = np.asarray(cache_u32[: geo["words"]]).reshape(batch, n_kv_heads, 2, nt, n_words, TILE)
+    alpha = np.asarray(cache_u32[geo["words"]: geo["words"] + geo["alpha"]]).view(np.float32)
+    alpha = alpha.reshape(batch, n_kv_heads, 2, nt * TILE)
+    t = np.arange(t0, t0 + n)
+    rec = words[b, head, kind][t // TILE, :, t % TILE]        # (n, W)
+    return rec, alpha[b, head, kind, t0:t0 + n]
+
+
+# ----------------------------------------------------------------------------
+# Decode attention (Def. sdpa with one query row; Algorithm 1 inference lines)
+# ----------------------------------------------------------------------------
+
+def softmax(s: np.ndarray) -> np.ndarray:
+    s = np.asarray(s, np.float64)
+    e = np.exp(s - np.max(s))
+    return e / np.sum(e)
+
+
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, w_o: np.ndarray | None = None):
+    """Single decode-step SDPA: s_i = q.k_i / sqrt(d_k), a = softmax(s), o = sum_i a_i v_i W_O
+    (Def. sdpa, Eq. singleheadattoutput)."""
+    q = np.asarray(q, np.float64)
+    a = softmax(np.asarray(k, np.float64) @ q / math.sqrt(q.shape[-1]))
+    o = a @ np.asarray(v, np.float64)
+    return o if w_o is None else o @ np.asarray(w_o, np.float64)
+
+
+def decode_attention(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_k: np.ndarray,
+                     basis_v: np.ndarray, group: int) -> np.ndarray:
+    """Decode over coded coefficients of one sequence and layer (Alg. 1 reconstruct/attend lines).
+
+    q_heads: (H_q, 128); hk, hv: (H_kv, n, 128) dequantized coefficients in storage order;
+    basis_k, basis_v: (H_kv, 128, 128) reconstruction bases (K_hat = h_hat U^T).
+    The keys are never rebuilt: q . (U h) = (U^T q) . h, and the value transform is applied
+    once to the weighted sum.  Query head j reads kv-head j // group.
+    """
+    out = np.zeros((q_heads.shape[0], D))
+    for j in range(q_heads.shape[0]):
+        h = j // group
+        qt = np.asarray(basis_k[h], np.float64).T @ np.asarray(q_heads[j], np.float64)
+        a = softmax(np.asarray(hk[h], np.float64) @ qt / math.sqrt(D))
+        out[j] = np.asarray(basis_v[h], np.float64) @ (a @ np.asarray(hv[h], np.float64))
+    return out
+
+
+# ----------------------------------------------------------------------------
+# Theorem 1 (attention-output distortion decomposition)
+# ----------------------------------------------------------------------------
+
+def distortion_decomposition(q, k, v, var_k, var_v, w_o=None):
+    """D_K and D_V of Theorem 1 for one decode step.
+
+    D_K = sum_{i,c} a_i^2 ||v_i W_O - o||^2 q_c^2 E[dk_ic^2] and
+    D_V = sum_{i,c} a_i^2 E[dv_ic^2] ||W_O,c||^2, where q_c is read as the c-th component of
+    q / sqrt(d_k), the sensitivity of the score s_i to k_ic under Def. sdpa's scaling.
+    """
+    q = np.asarray(q, np.float64)
+    k = np.asarray(k, np.float64)
+    v = np.asarray(v, np.float64)
+    d = q.shape[-1]
+    wo = np.eye(v.shape[1]) if w_o is None else np.asarray(w_o, np.float64)
+    a = softmax(k @ q / math.sqrt(d))
+    vw = v @ wo
+    o = a @ vw
+    qe = q / math.sqrt(d)
+    resid = np.sum((vw - o) ** 2, axis=1)
+    dk = float(np.sum(a ** 2 * resid * (np.asarray(var_k) @ (qe ** 2))))
+    dv = float(np.sum(a ** 2 * (np.asarray(var_v) @ np.sum(wo ** 2, axis=1))))
+    return dk, dv
