@@ -1,0 +1,195 @@
+/*
+ * aatc.h -- C ABI of the GB300 (sm_103a) hot path of Attention-Aware Transform Coding
+ * (AATC, arxiv 2608.14191, "KV Cache Compression Through the Lens of Transform Coding").
+ *
+ * The problem the library solves (Sec. 3.2 KV cache, Sec. 5, Algorithm 1): calibrate a
+ * per-layer, per-kv-head orthonormal transform and a per-channel bit allocation offline,
+ * then, online, append each new key/value head-vector to a packed cache in transform
+ * coordinates and run single-token decode attention directly over that packed cache.
+ *
+ * Conventions shared by every call:
+ *   - head_dim d is 128.  A *stream* is one (layer, kv-head, K|V) triple; streams are
+ *     indexed s = (layer * n_kv_heads + kv_head) * 2 + kind with kind 0 = keys, 1 = values.
+ *   - Pointers documented as "device" must be CUDA device memory of the current device;
+ *     "host" pointers are ordinary host memory.  The library never takes ownership of
+ *     caller memory and never frees it.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  All
+ *     device work is enqueued on it asynchronously; only aatc_plan_create,
+ *     aatc_plan_destroy and aatc_get_device_error synchronize.
+ *   - Argument errors are detected on the host before any launch; the call then returns a
+ *     non-zero status and leaves all outputs untouched.  A failed launch returns
+ *     AATC_ERR_CUDA (see aatc_last_cuda_error).
+ *   - No call allocates device memory except aatc_plan_create.
+ */
+#ifndef AATC_H
+#define AATC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AATC_HEAD_DIM 128
+#define AATC_MAX_BITS 8      /* widest channel code (bits); widths are 0..AATC_MAX_BITS */
+
+typedef struct aatc_plan_s* aatc_plan_t;   /* opaque; immutable after creation */
+
+typedef enum {
+  AATC_OK = 0,
+  AATC_ERR_INVALID_ARG = 1,   /* null pointer, bad shape, out-of-range index            */
+  AATC_ERR_BUDGET = 2,        /* bit budget not representable (e.g. > b_max * d)        */
+  AATC_ERR_CAPACITY = 3,      /* token range exceeds the cache capacity                  */
+  AATC_ERR_WORKSPACE = 4,     /* caller workspace smaller than the required size         */
+  AATC_ERR_UNSUPPORTED = 5,   /* shape the kernels do not implement (e.g. GQA group > 8) */
+  AATC_ERR_CUDA = 6,          /* a CUDA runtime call or kernel launch failed             */
+  AATC_ERR_NOMEM = 7,         /* host or device allocation failed                        */
+  AATC_ERR_DEVICE_FLAG = 8    /* reserved for callers that turn device flags into status */
+} aatc_status_t;
+
+/* Model dimensions.  d must be 128; n_q_heads % n_kv_heads == 0; b_max in 1..8. */
+typedef struct {
+  int32_t d;
+  int32_t n_layers;
+  int32_t n_kv_heads;
+  int32_t n_q_heads;
+  int32_t b_max;
+} aatc_dims_t;
+
+/* Human-readable name of a status code (static string). */
+const char* aatc_status_string(aatc_status_t status);
+
+/* cudaError_t value of the most recent AATC_ERR_CUDA on this thread (0 if none). */
+int32_t aatc_last_cuda_error(void);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int32_t aatc_version(void);
+
+/*
+ * Offline calibration (host only, no GPU needed) -- Sec. 5 Steps 1-2 and the calibration
+ * half of Algorithm 1, with the PCA eigenbasis of the calibration keys/values standing in
+ * for the whitening-SVD transform (equivalent by the appendix Proposition).  Per stream:
+ *   C = X^T X / N (uncentered second moment); C = U diag(sigma^2) U^T by cyclic Jacobi in
+ *   fp64 (eigenvalues descending; each eigenvector's largest |entry| made positive, lowest
+ *   index on ties); weights w^K_c = sum over the group's query heads of mean_i (u_c . q_i)^2
+ *   (Eq. waterfilling-keys and its GQA remark), w^V_c = 1 (W_O = I);  g_c = w_c sigma_c^2;
+ *   channels re-sorted by g descending (stable); integer reverse water-filling
+ *   min sum_c g_c 4^-b_c s.t. sum_c b_c = round(avg_bits * d), b_c in 0..b_max (exact greedy;
+ *   ties to the lower index); s_c = 99th percentile of |u_c . x| (linear interpolation at
+ *   rank 0.99 (N - 1)).
+ *
+ *   calib_k, calib_v : host fp32 [n_layers][n_kv_heads][n_calib][128]
+ *   calib_q          : host fp32 [n_layers][n_q_heads][n_calib_q][128], or NULL (then w^K = 1)
+ *   avg_bits_k/v     : average code bits per channel; avg * 128 must be an integer
+ *   weights_mode     : 0 = attention-aware (AATC), 1 = variance only (AATC var-only, Sec. 6)
+ *   basis_out        : host fp32 [L][H_kv][2][128 (input dim)][128 (channel, storage order)]
+ *   bits_out         : host uint8 [L][H_kv][2][128], non-increasing along storage order
+ *   scales_out       : host fp32 [L][H_kv][2][128]
+ *   sigma2_out, weights_out : host fp64 [L][H_kv][2][128] or NULL (diagnostics)
+ *   n_threads        : host worker threads (0 = hardware concurrency)
+ * Errors: AATC_ERR_INVALID_ARG (null/shape), AATC_ERR_BUDGET (avg*128 not integral or >
+ * b_max*128 or < 0).
+ */
+aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k, const float* calib_v,
+                             int32_t n_calib, const float* calib_q, int32_t n_calib_q,
+                             double avg_bits_k, double avg_bits_v, int32_t weights_mode,
+                             float* basis_out, uint8_t* bits_out, float* scales_out,
+                             double* sigma2_out, double* weights_out, int32_t n_threads);
+
+/*
+ * Build an immutable device plan from basis / bits / scales in the layouts aatc_calibrate
+ * writes (Algorithm 1 outputs).  Derives per stream: R = #{b_c >= 1}, bit offsets, the
+ * record length W = ceil(max_s sum_c b_c / 32) words (plan-wide), f_c = s_c 2^(1-b_c), the
+ * bf16 encode basis (round-to-nearest-even of `basis`), and uploads everything with one
+ * copy on `stream`, then synchronizes it.  Host inputs are copied; the caller keeps them.
+ * Errors: AATC_ERR_INVALID_ARG (null, bits > b_max, bits not non-increasing, scale <= 0 or
+ * non-finite where bits > 0, non-finite basis), AATC_ERR_CUDA, AATC_ERR_NOMEM.
+ */
+aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
+                               const float* scales, void* stream, aatc_plan_t* plan_out);
+
+/* Free the plan and its device tables (synchronizes the device).  NULL is a no-op. */
+aatc_status_t aatc_plan_destroy(aatc_plan_t plan);
+
+/* Words per packed record (W) and per-stream retained channel counts R (host int32
+ * [L][H_kv][2], may be NULL). */
+aatc_status_t aatc_plan_info(aatc_plan_t plan, int32_t* n_words, int32_t* retained);
+
+/*
+ * Bytes of one layer's packed cache for `batch` sequences of capacity max_tokens:
+ *   uint32 words [batch][H_kv][2][n_tiles][W][128], then fp32 alpha [batch][H_kv][2][n_tiles*128],
+ *   n_tiles = ceil(max_tokens / 128).  Token t of a sequence lives in tile t/128, lane t%128
+ *   (build-defined layout: the paper leaves the storage format open).
+ */
+aatc_status_t aatc_cache_bytes(aatc_plan_t plan, int32_t batch, int32_t max_tokens, size_t* bytes);
+
+/*
+ * Encode (Algorithm 1: "Project", "Append qtz(h)"; quantizer of Sec. 5): for every token and
+ * stream, h = U_bf16^T x (bf16 x bf16 -> fp32 on tcgen05 tensor cores), alpha = max over
+ * retained channels of |h_c| / s_c (fp32), code_c = clamp(floor(h_c / (alpha f_c) + 1/2),
+ * -2^(b-1), 2^(b-1)-1), stored as u = code + 2^(b-1) in b_c-bit fields, LSB first in storage
+ * channel order (fields may straddle words; unused bits are written as zero).
+ *   K, V   : device bf16 [batch][n_tokens][n_kv_heads][128], contiguous
+ *   cache  : device, one layer, sized by aatc_cache_bytes(batch, max_tokens); tokens are written
+ *            at positions [start, start + n_tokens) of every sequence; other positions untouched.
+ * A non-finite alpha sets device error flag bit 0 (aatc_get_device_error).
+ * Errors: AATC_ERR_INVALID_ARG, AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_CUDA.
+ * n_tokens == 0 is a no-op.
+ */
+aatc_status_t aatc_encode(aatc_plan_t plan, int32_t layer, const void* K, const void* V,
+                          int32_t batch, int32_t start, int32_t n_tokens, void* cache,
+                          int32_t max_tokens, void* stream);
+
+/* Device workspace bytes aatc_decode_attention needs for (batch, n_ctx). */
+aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t plan, int32_t batch, int32_t n_ctx,
+                                          size_t* bytes);
+
+/*
+ * Decode attention over the packed cache (Def. sdpa with one query row; Algorithm 1
+ * reconstruct/attend lines computed without rebuilding K): per query head j (kv-head
+ * j / group), q~ = U_K^T q, s_t = q~ . h_hat^K_t / sqrt(128), a = softmax(s),
+ * o_hat = sum_t a_t h_hat^V_t, out = U_V o_hat, with h_hat_c = code_c * (alpha_t f_c).
+ * Attends to tokens [0, n_ctx) of each sequence (no mask).  Split-K over the context with a
+ * log-sum-exp combine; fp32 accumulation; fp32 output.
+ *   q         : device bf16 [batch][n_q_heads][128]
+ *   out       : device fp32 [batch][n_q_heads][128]
+ *   workspace : device, >= aatc_decode_workspace_bytes(batch, n_ctx), contents ignored
+ * Errors: AATC_ERR_INVALID_ARG (n_ctx < 1 ...), AATC_ERR_CAPACITY (n_ctx > max_tokens),
+ * AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (group > 8), AATC_ERR_CUDA.
+ */
+aatc_status_t aatc_decode_attention(aatc_plan_t plan, int32_t layer, const void* q,
+                                    const void* cache, int32_t batch, int32_t n_ctx,
+                                    int32_t max_tokens, float* out, void* workspace,
+                                    size_t workspace_bytes, void* stream);
+
+/*
+ * Test hook: dequantized coefficients h_hat_c = fl32(code_c * fl32(alpha_t * f_c)) (zero for
+ * dropped channels) of tokens [t0, t0 + n) of every sequence.
+ *   coeffs_out : device fp32 [batch][n][n_kv_heads][2][128]
+ */
+aatc_status_t aatc_dequantize(aatc_plan_t plan, int32_t layer, const void* cache, int32_t batch,
+                              int32_t t0, int32_t n, int32_t max_tokens, float* coeffs_out,
+                              void* stream);
+
+/* Sticky device error flags of the plan (bit 0: non-finite token scale seen by encode;
+ * bit 1: a bounded wait inside a kernel timed out).  Synchronizes; clear != 0 resets them. */
+aatc_status_t aatc_get_device_error(aatc_plan_t plan, int32_t* flags, int32_t clear);
+
+/*
+ * Reference point: uncompressed bf16 decode attention (Def. sdpa), split-K with the same
+ * combine.  K, V: device bf16 [batch][max_tokens][n_kv_heads][128]; attends to [0, n_ctx).
+ * q: device bf16 [batch][n_q_heads][128]; out: device fp32 [batch][n_q_heads][128].
+ */
+aatc_status_t aatc_bf16_decode_workspace_bytes(int32_t batch, int32_t n_kv_heads,
+                                               int32_t n_q_heads, int32_t n_ctx, size_t* bytes);
+aatc_status_t aatc_bf16_decode_attention(const void* K, const void* V, const void* q,
+                                         int32_t batch, int32_t n_ctx, int32_t max_tokens,
+                                         int32_t n_kv_heads, int32_t n_q_heads, float* out,
+                                         void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AATC_H */

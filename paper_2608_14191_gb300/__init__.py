@@ -1,0 +1,243 @@
+"""GB300 (sm_103a) hot path of Attention-Aware Transform Coding (AATC), arxiv 2608.14191.
+
+Thin Python binding over the C ABI in ``include/aatc.h`` (library ``libaatc.so`` built in-tree
+by :mod:`paper_2608_14191_gb300.build`).  The binding only marshals arguments: PyTorch
+tensors provide device memory and the current CUDA stream; every step of the path runs in
+the library.  There is no fallback: if the shared object is missing the import of
+:data:`lib` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+HEAD_DIM = 128
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libaatc.so")
+
+_STATUS = {
+    0: "ok", 1: "invalid argument", 2: "bit budget not representable", 3: "token range exceeds cache capacity",
+    4: "workspace too small", 5: "unsupported shape", 6: "CUDA error", 7: "out of memory", 8: "device error flag set",
+}
+
+
+class AatcError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = f"{where}: {_STATUS.get(status, 'unknown')} (status {status})"
+        if status == 6 and _lib is not None:
+            msg += f", cudaError {_lib.aatc_last_cuda_error()}"
+        super().__init__(msg)
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int32), ("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("b_max", ctypes.c_int32)]
+
+
+_lib = None
+_P, _I32, _SZ, _F64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t, ctypes.c_double
+
+# name -> (restype, argtypes); mirrors include/aatc.h
+SIGNATURES = {
+    "aatc_status_string": (ctypes.c_char_p, [_I32]),
+    "aatc_last_cuda_error": (_I32, []),
+    "aatc_version": (_I32, []),
+    "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
+    "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
+    "aatc_plan_destroy": (_I32, [_P]),
+    "aatc_plan_info": (_I32, [_P, ctypes.POINTER(_I32), _P]),
+    "aatc_cache_bytes": (_I32, [_P, _I32, _I32, ctypes.POINTER(_SZ)]),
+    "aatc_encode": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _P, _I32, _P]),
+    "aatc_decode_workspace_bytes": (_I32, [_P, _I32, _I32, ctypes.POINTER(_SZ)]),
+    "aatc_decode_attention": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _P, _P, _SZ, _P]),
+    "aatc_dequantize": (_I32, [_P, _I32, _P, _I32, _I32, _I32, _I32, _P, _P]),
+    "aatc_get_device_error": (_I32, [_P, ctypes.POINTER(_I32), _I32]),
+    "aatc_bf16_decode_workspace_bytes": (_I32, [_I32, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
+    "aatc_bf16_decode_attention": (_I32, [_P, _P, _P, _I32, _I32, _I32, _I32, _I32, _P, _P, _SZ, _P]),
+}
+
+
+def load(path: str = LIB_PATH):
+    """Load libaatc.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise AatcError(status, where)
+
+
+def _ptr(a) -> int:
+    """Address of a torch tensor or numpy array (must be contiguous)."""
+    if hasattr(a, "data_ptr"):
+        if not a.is_contiguous():
+            raise ValueError("tensor must be contiguous")
+        return a.data_ptr()
+    if not a.flags["C_CONTIGUOUS"]:
+        raise ValueError("array must be C-contiguous")
+    return a.ctypes.data
+
+
+def _stream(stream=None) -> int:
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def dims(n_layers: int, n_kv_heads: int, n_q_heads: int, b_max: int = 8) -> Dims:
+    return Dims(HEAD_DIM, n_layers, n_kv_heads, n_q_heads, b_max)
+
+
+def calibrate(dm: Dims, calib_k: np.ndarray, calib_v: np.ndarray, calib_q: np.ndarray | None,
+              avg_bits_k: float, avg_bits_v: float | None = None, var_only: bool = False,
+              n_threads: int = 0):
+    """Host planner (Sec. 5 Steps 1-2).  calib_k/v: fp32 [L][H_kv][N][128]; calib_q: fp32
+    [L][H_q][Nq][128] or None.  Returns dict(basis, bits, scales, sigma2, weights)."""
+    lib = load()
+    ck = np.ascontiguousarray(calib_k, dtype=np.float32)
+    cv = np.ascontiguousarray(calib_v, dtype=np.float32)
+    cq = None if calib_q is None else np.ascontiguousarray(calib_q, dtype=np.float32)
+    L, H = dm.n_layers, dm.n_kv_heads
+    if ck.shape[:2] != (L, H) or ck.shape[3] != HEAD_DIM or cv.shape != ck.shape:
+        raise ValueError("calibration arrays must be [L][H_kv][N][128]")
+    if cq is not None and (cq.shape[:2] != (L, dm.n_q_heads) or cq.shape[3] != HEAD_DIM):
+        raise ValueError("calibration queries must be [L][H_q][Nq][128]")
+    S = L * H * 2
+    basis = np.empty((L, H, 2, HEAD_DIM, HEAD_DIM), np.float32)
+    bits = np.empty((L, H, 2, HEAD_DIM), np.uint8)
+    scales = np.empty((L, H, 2, HEAD_DIM), np.float32)
+    sigma2 = np.empty((L, H, 2, HEAD_DIM), np.float64)
+    weights = np.empty((L, H, 2, HEAD_DIM), np.float64)
+    st = lib.aatc_calibrate(ctypes.byref(dm), _ptr(ck), _ptr(cv), ck.shape[2], None if cq is None else _ptr(cq),
+                            0 if cq is None else cq.shape[2], float(avg_bits_k),
+                            float(avg_bits_k if avg_bits_v is None else avg_bits_v), 1 if var_only else 0,
+                            _ptr(basis), _ptr(bits), _ptr(scales), _ptr(sigma2), _ptr(weights), int(n_threads))
+    _check(st, "aatc_calibrate")
+    assert S == basis.shape[0] * H * 2
+    return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
+
+
+class Plan:
+    """Device plan (aatc_plan_t).  Create from the planner outputs; destroyed on close()."""
+
+    def __init__(self, dm: Dims, basis: np.ndarray, bits: np.ndarray, scales: np.ndarray, stream=None):
+        lib = load()
+        self.dims = dm
+        self._basis = np.ascontiguousarray(basis, dtype=np.float32)
+        self._bits = np.ascontiguousarray(bits, dtype=np.uint8)
+        self._scales = np.ascontiguousarray(scales, dtype=np.float32)
+        h = ctypes.c_void_p()
+        st = lib.aatc_plan_create(ctypes.byref(dm), _ptr(self._basis), _ptr(self._bits), _ptr(self._scales),
+                                  _stream(stream), ctypes.byref(h))
+        _check(st, "aatc_plan_create")
+        self.handle = h.value
+        w = _I32()
+        ret = np.empty((dm.n_layers, dm.n_kv_heads, 2), np.int32)
+        _check(lib.aatc_plan_info(self.handle, ctypes.byref(w), _ptr(ret)), "aatc_plan_info")
+        self.n_words = w.value
+        self.retained = ret
+
+    @property
+    def group(self) -> int:
+        return self.dims.n_q_heads // self.dims.n_kv_heads
+
+    def cache_bytes(self, batch: int, max_tokens: int) -> int:
+        n = _SZ()
+        _check(load().aatc_cache_bytes(self.handle, batch, max_tokens, ctypes.byref(n)), "aatc_cache_bytes")
+        return n.value
+
+    def new_cache(self, batch: int, max_tokens: int, device="cuda"):
+        import torch
+        return torch.empty(self.cache_bytes(batch, max_tokens) // 4, dtype=torch.int32, device=device)
+
+    def workspace_bytes(self, batch: int, n_ctx: int) -> int:
+        n = _SZ()
+        _check(load().aatc_decode_workspace_bytes(self.handle, batch, n_ctx, ctypes.byref(n)),
+               "aatc_decode_workspace_bytes")
+        return n.value
+
+    def device_error(self, clear: bool = False) -> int:
+        f = _I32()
+        _check(load().aatc_get_device_error(self.handle, ctypes.byref(f), int(clear)), "aatc_get_device_error")
+        return f.value
+
+    def close(self):
+        if getattr(self, "handle", None):
+            _check(load().aatc_plan_destroy(self.handle), "aatc_plan_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def encode(plan: Plan, layer: int, K, V, cache, start: int, max_tokens: int, stream=None):
+    """aatc_encode: K, V bf16 [batch][n_tokens][H_kv][128] (device); writes positions
+    [start, start + n_tokens) of the packed cache."""
+    batch, n_tokens = K.shape[0], K.shape[1]
+    _check(load().aatc_encode(plan.handle, layer, _ptr(K), _ptr(V), batch, start, n_tokens, _ptr(cache),
+                              max_tokens, _stream(stream)), "aatc_encode")
+
+
+def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: int, out=None, workspace=None,
+                     stream=None):
+    """aatc_decode_attention: q bf16 [batch][H_q][128] -> fp32 [batch][H_q][128]."""
+    import torch
+    batch = q.shape[0]
+    if out is None:
+        out = torch.empty((batch, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    nbytes = plan.workspace_bytes(batch, n_ctx)
+    if workspace is None:
+        workspace = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device=q.device)
+    _check(load().aatc_decode_attention(plan.handle, layer, _ptr(q), _ptr(cache), batch, n_ctx, max_tokens,
+                                        _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                        _stream(stream)), "aatc_decode_attention")
+    return out
+
+
+def dequantize(plan: Plan, layer: int, cache, batch: int, t0: int, n: int, max_tokens: int, stream=None):
+    """aatc_dequantize test hook -> fp32 [batch][n][H_kv][2][128]."""
+    import torch
+    out = torch.empty((batch, n, plan.dims.n_kv_heads, 2, HEAD_DIM), dtype=torch.float32, device=cache.device)
+    _check(load().aatc_dequantize(plan.handle, layer, _ptr(cache), batch, t0, n, max_tokens, _ptr(out),
+                                  _stream(stream)), "aatc_dequantize")
+    return out
+
+
+def bf16_workspace_bytes(batch: int, n_kv: int, n_q: int, n_ctx: int) -> int:
+    n = _SZ()
+    _check(load().aatc_bf16_decode_workspace_bytes(batch, n_kv, n_q, n_ctx, ctypes.byref(n)),
+           "aatc_bf16_decode_workspace_bytes")
+    return n.value
+
+
+def bf16_decode_attention(K, V, q, n_ctx: int, out=None, workspace=None, stream=None):
+    """Uncompressed reference decode: K, V bf16 [batch][max_tokens][H_kv][128]; q bf16 [batch][H_q][128]."""
+    import torch
+    batch, max_tokens, n_kv = K.shape[0], K.shape[1], K.shape[2]
+    n_q = q.shape[1]
+    if out is None:
+        out = torch.empty((batch, n_q, HEAD_DIM), dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = torch.empty(max(1, bf16_workspace_bytes(batch, n_kv, n_q, n_ctx) // 4), dtype=torch.float32,
+                                device=q.device)
+    _check(load().aatc_bf16_decode_attention(_ptr(K), _ptr(V), _ptr(q), batch, n_ctx, max_tokens, n_kv, n_q,
+                                             _ptr(out), _ptr(workspace), workspace.numel() * 4, _stream(stream)),
+           "aatc_bf16_decode_attention")
+    return out

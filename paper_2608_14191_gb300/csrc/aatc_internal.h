@@ -1,0 +1,110 @@
+// Internal declarations shared by the C ABI (capi.cpp), the planner and the CUDA kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "aatc.h"
+
+#if defined(__CUDACC__)
+#define AATC_HD __host__ __device__
+#else
+#define AATC_HD
+#endif
+
+namespace aatc {
+
+constexpr int D = 128;              // head_dim
+constexpr int TILE = 128;           // tokens per word-planar cache tile
+constexpr int MAX_GROUP = 8;        // query heads per kv-head supported by the decode kernels
+constexpr uint32_t PLAN_MAGIC = 0xAA7C0DE1u;
+constexpr uint32_t PLAN_DEAD = 0xDEADDEADu;
+
+// Packing schedule word of one channel (encode epilogue): bit offset inside its first word,
+// whether the field completes that word, and the width.
+AATC_HD constexpr int sched_shift(int s) { return s & 31; }
+AATC_HD constexpr bool sched_flush(int s) { return (s >> 8) & 1; }
+AATC_HD constexpr int sched_bits(int s) { return (s >> 16) & 15; }
+
+struct ChanEnc {          // per-channel encode constants (one 16-byte load)
+  float inv_f;            // 1 / f_c, f_c = s_c 2^(1-b_c); 0 for dropped channels
+  float lo;               // -2^(b_c-1) as float (0 for dropped)
+  float hi;               // 2^(b_c-1) - 1 as float (0 for dropped)
+  float magic;            // 1.5 * 2^23 + 2^(b_c-1): floor to offset-binary u via round-down add
+};
+
+struct PlanDevice {
+  const void* ubf16_t;    // bf16 [S][128 channel][128 dim]   encode basis (MMA B operand, K-major)
+  const float* u32;       // fp32 [S][128 dim][128 channel]   decode query rotation / value inverse
+  const ChanEnc* enc;     // [S][128]
+  const int* sched;       // [S][128]
+  const float* inv_s;     // [S][128] 1/s_c (0 for dropped)
+  const float* f;         // [S][128] f_c (0 for dropped)
+  const int* ext;         // [S][128] decode extraction word: (offset in record) | (b << 16)
+  const int* nret;        // [S] retained channels R
+  int* err;               // [4] sticky device flags
+};
+
+struct Plan {
+  uint32_t magic = PLAN_MAGIC;
+  aatc_dims_t dims{};
+  int n_streams = 0;
+  int n_words = 0;        // W, words per record (plan-wide)
+  int num_sms = 0;
+  int device = 0;
+  std::vector<int> retained;
+  std::vector<int> nbits;
+  PlanDevice dev{};
+  void* block = nullptr;  // single device allocation holding every table
+  size_t block_bytes = 0;
+  alignas(64) unsigned char tmap_u[128];   // CUtensorMap over ubf16_t (2D: 128 dims x S*128 rows)
+  bool tmap_ok = false;
+};
+
+inline bool valid_dims(const aatc_dims_t* d) {
+  return d && d->d == D && d->n_layers >= 1 && d->n_kv_heads >= 1 && d->n_q_heads >= d->n_kv_heads &&
+         d->n_q_heads % d->n_kv_heads == 0 && d->b_max >= 1 && d->b_max <= AATC_MAX_BITS &&
+         d->n_layers <= 4096 && d->n_q_heads <= 4096;
+}
+
+struct CacheGeom {
+  int n_tiles;
+  size_t words_elems;     // uint32 elements of the word region
+  size_t alpha_elems;     // fp32 elements of the alpha region
+  size_t bytes;
+};
+
+inline CacheGeom cache_geom(int batch, int n_kv, int max_tokens, int n_words) {
+  CacheGeom g;
+  g.n_tiles = (max_tokens + TILE - 1) / TILE;
+  g.words_elems = static_cast<size_t>(batch) * n_kv * 2 * g.n_tiles * n_words * TILE;
+  g.alpha_elems = static_cast<size_t>(batch) * n_kv * 2 * g.n_tiles * TILE;
+  g.bytes = 4 * (g.words_elems + g.alpha_elems);
+  return g;
+}
+
+struct DecodeSplit {
+  int n_splits;
+  int split_len;          // tokens per split, a multiple of TILE
+};
+
+DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
+size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp);
+
+// Kernel launchers (defined in the .cu files); return the CUDA error of the launch.
+cudaError_t encode_tensor_maps_u(Plan& plan);
+cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch,
+                          int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st);
+cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch,
+                          int n_ctx, int max_tokens, float* out, void* ws, const DecodeSplit& sp,
+                          cudaStream_t st);
+cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n,
+                           int max_tokens, float* out, cudaStream_t st);
+cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx,
+                               int max_tokens, int n_kv, int n_q, float* out, void* ws,
+                               const DecodeSplit& sp, cudaStream_t st);
+
+}  // namespace aatc

@@ -1,0 +1,329 @@
+// C ABI of the AATC library: argument validation, plan construction (packed-layout
+// descriptor and per-channel constants) and dispatch to the CUDA kernels.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "aatc.h"
+#include "aatc_internal.h"
+
+namespace {
+
+thread_local int32_t g_last_cuda_error = 0;
+
+aatc_status_t cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return AATC_OK;
+  g_last_cuda_error = static_cast<int32_t>(e);
+  return AATC_ERR_CUDA;
+}
+
+aatc::Plan* as_plan(aatc_plan_t p) {
+  auto* plan = reinterpret_cast<aatc::Plan*>(p);
+  if (!plan || plan->magic != aatc::PLAN_MAGIC) return nullptr;
+  return plan;
+}
+
+// fp32 -> bf16 bits, round to nearest even (inputs are finite; validated by the caller).
+uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  const uint32_t round = 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>((u + round) >> 16);
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+namespace aatc {
+
+DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
+  const int tiles = (n_ctx + TILE - 1) / TILE;
+  const long units = static_cast<long>(batch) * n_kv;
+  const long target = 2L * std::max(1, num_sms);                 // ~2 CTAs per SM
+  long per = (static_cast<long>(tiles) * units + target - 1) / target;
+  per = std::max(1L, std::min(per, 16L));                           // <= 2048 tokens per split
+  DecodeSplit sp;
+  sp.n_splits = static_cast<int>((tiles + per - 1) / per);
+  sp.split_len = static_cast<int>(per) * TILE;
+  return sp;
+}
+
+size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp) {
+  return static_cast<size_t>(batch) * n_q * sp.n_splits * (D + 2) * sizeof(float);
+}
+
+}  // namespace aatc
+
+extern "C" {
+
+const char* aatc_status_string(aatc_status_t s) {
+  switch (s) {
+    case AATC_OK: return "ok";
+    case AATC_ERR_INVALID_ARG: return "invalid argument";
+    case AATC_ERR_BUDGET: return "bit budget not representable";
+    case AATC_ERR_CAPACITY: return "token range exceeds cache capacity";
+    case AATC_ERR_WORKSPACE: return "workspace too small";
+    case AATC_ERR_UNSUPPORTED: return "unsupported shape";
+    case AATC_ERR_CUDA: return "CUDA error";
+    case AATC_ERR_NOMEM: return "out of memory";
+    case AATC_ERR_DEVICE_FLAG: return "device error flag set";
+  }
+  return "unknown status";
+}
+
+int32_t aatc_last_cuda_error(void) { return g_last_cuda_error; }
+
+int32_t aatc_version(void) { return 100; }
+
+aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
+                               const float* scales, void* stream, aatc_plan_t* plan_out) {
+  using namespace aatc;
+  if (!valid_dims(dims) || !basis || !bits || !scales || !plan_out) return AATC_ERR_INVALID_ARG;
+  const int S = dims->n_layers * dims->n_kv_heads * 2;
+  const size_t SD = static_cast<size_t>(S) * D;
+  // validate
+  std::vector<int> retained(S), nbits(S);
+  for (int s = 0; s < S; ++s) {
+    int r = 0, nb = 0;
+    for (int c = 0; c < D; ++c) {
+      const int b = bits[s * D + c];
+      if (b > dims->b_max) return AATC_ERR_INVALID_ARG;
+      if (c > 0 && b > bits[s * D + c - 1]) return AATC_ERR_INVALID_ARG;   // non-increasing
+      if (b > 0) {
+        const float sc = scales[s * D + c];
+        if (!(std::isfinite(sc) && sc > 0.0f)) return AATC_ERR_INVALID_ARG;
+        ++r;
+      }
+      nb += b;
+    }
+    retained[s] = r;
+    nbits[s] = nb;
+  }
+  for (size_t i = 0; i < SD * D; ++i)
+    if (!std::isfinite(basis[i])) return AATC_ERR_INVALID_ARG;
+  const int max_nb = *std::max_element(nbits.begin(), nbits.end());
+  const int W = std::max(1, (max_nb + 31) / 32);
+
+  // host staging of every table, in one block
+  size_t off = 0;
+  const size_t o_ubf = off;  off = align_up(off + SD * D * 2, 256);
+  const size_t o_u32 = off;  off = align_up(off + SD * D * 4, 256);
+  const size_t o_enc = off;  off = align_up(off + SD * sizeof(ChanEnc), 256);
+  const size_t o_sch = off;  off = align_up(off + SD * 4, 256);
+  const size_t o_invs = off; off = align_up(off + SD * 4, 256);
+  const size_t o_f = off;    off = align_up(off + SD * 4, 256);
+  const size_t o_ext = off;  off = align_up(off + SD * 4, 256);
+  const size_t o_nret = off; off = align_up(off + static_cast<size_t>(S) * 4, 256);
+  const size_t o_err = off;  off = align_up(off + 16, 256);
+  const size_t total = off;
+  std::vector<unsigned char> host;
+  try {
+    host.assign(total, 0);
+  } catch (const std::bad_alloc&) {
+    return AATC_ERR_NOMEM;
+  }
+  auto* ubf = reinterpret_cast<uint16_t*>(host.data() + o_ubf);
+  auto* u32 = reinterpret_cast<float*>(host.data() + o_u32);
+  auto* enc = reinterpret_cast<ChanEnc*>(host.data() + o_enc);
+  auto* sch = reinterpret_cast<int*>(host.data() + o_sch);
+  auto* invs = reinterpret_cast<float*>(host.data() + o_invs);
+  auto* fc = reinterpret_cast<float*>(host.data() + o_f);
+  auto* ext = reinterpret_cast<int*>(host.data() + o_ext);
+  auto* nret = reinterpret_cast<int*>(host.data() + o_nret);
+  for (int s = 0; s < S; ++s) {
+    const float* bs = basis + static_cast<size_t>(s) * D * D;     // [dim][channel]
+    for (int d = 0; d < D; ++d)
+      for (int c = 0; c < D; ++c) {
+        ubf[(static_cast<size_t>(s) * D + c) * D + d] = f32_to_bf16_rne(bs[d * D + c]);
+        u32[(static_cast<size_t>(s) * D + d) * D + c] = bs[d * D + c];
+      }
+    int o = 0;
+    for (int c = 0; c < D; ++c) {
+      const size_t i = static_cast<size_t>(s) * D + c;
+      const int b = bits[i];
+      ChanEnc e{0.0f, 0.0f, 0.0f, 12582912.0f};
+      if (b > 0) {
+        const float f = std::ldexp(scales[i], 1 - b);            // exact power-of-two scaling
+        e.inv_f = 1.0f / f;
+        e.lo = -std::ldexp(1.0f, b - 1);
+        e.hi = std::ldexp(1.0f, b - 1) - 1.0f;
+        e.magic = 12582912.0f + std::ldexp(1.0f, b - 1);
+        fc[i] = f;
+        invs[i] = 1.0f / scales[i];
+      }
+      enc[i] = e;
+      const int sh = o & 31;
+      const int flush = (b > 0 && sh + b >= 32) ? 1 : 0;
+      sch[i] = sh | (flush << 8) | (b << 16);
+      ext[i] = o | (b << 16);
+      o += b;
+    }
+    nret[s] = retained[s];
+  }
+
+  auto* plan = new (std::nothrow) Plan();
+  if (!plan) return AATC_ERR_NOMEM;
+  plan->dims = *dims;
+  plan->n_streams = S;
+  plan->n_words = W;
+  plan->retained = retained;
+  plan->nbits = nbits;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaGetDevice(&plan->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&plan->num_sms, cudaDevAttrMultiProcessorCount, plan->device);
+  if (e == cudaSuccess) e = cudaMalloc(&plan->block, total);
+  if (e != cudaSuccess) {
+    delete plan;
+    return e == cudaErrorMemoryAllocation ? AATC_ERR_NOMEM : cuda_status(e);
+  }
+  plan->block_bytes = total;
+  e = cudaMemcpyAsync(plan->block, host.data(), total, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  auto* base = static_cast<unsigned char*>(plan->block);
+  plan->dev.ubf16_t = base + o_ubf;
+  plan->dev.u32 = reinterpret_cast<const float*>(base + o_u32);
+  plan->dev.enc = reinterpret_cast<const ChanEnc*>(base + o_enc);
+  plan->dev.sched = reinterpret_cast<const int*>(base + o_sch);
+  plan->dev.inv_s = reinterpret_cast<const float*>(base + o_invs);
+  plan->dev.f = reinterpret_cast<const float*>(base + o_f);
+  plan->dev.ext = reinterpret_cast<const int*>(base + o_ext);
+  plan->dev.nret = reinterpret_cast<const int*>(base + o_nret);
+  plan->dev.err = reinterpret_cast<int*>(base + o_err);
+  if (e == cudaSuccess) e = encode_tensor_maps_u(*plan);
+  if (e != cudaSuccess) {
+    cudaFree(plan->block);
+    delete plan;
+    return cuda_status(e);
+  }
+  *plan_out = reinterpret_cast<aatc_plan_t>(plan);
+  return AATC_OK;
+}
+
+aatc_status_t aatc_plan_destroy(aatc_plan_t p) {
+  if (!p) return AATC_OK;
+  aatc::Plan* plan = as_plan(p);
+  if (!plan) return AATC_ERR_INVALID_ARG;
+  cudaError_t e = cudaDeviceSynchronize();
+  cudaError_t e2 = cudaFree(plan->block);
+  plan->magic = aatc::PLAN_DEAD;
+  delete plan;
+  if (e != cudaSuccess) return cuda_status(e);
+  return cuda_status(e2);
+}
+
+aatc_status_t aatc_plan_info(aatc_plan_t p, int32_t* n_words, int32_t* retained) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !n_words) return AATC_ERR_INVALID_ARG;
+  *n_words = plan->n_words;
+  if (retained)
+    for (int s = 0; s < plan->n_streams; ++s) retained[s] = plan->retained[s];
+  return AATC_OK;
+}
+
+aatc_status_t aatc_cache_bytes(aatc_plan_t p, int32_t batch, int32_t max_tokens, size_t* bytes) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !bytes || batch < 1 || max_tokens < 1) return AATC_ERR_INVALID_ARG;
+  *bytes = aatc::cache_geom(batch, plan->dims.n_kv_heads, max_tokens, plan->n_words).bytes;
+  return AATC_OK;
+}
+
+aatc_status_t aatc_encode(aatc_plan_t p, int32_t layer, const void* K, const void* V, int32_t batch,
+                          int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
+                          void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !K || !V || !cache || layer < 0 || layer >= plan->dims.n_layers || batch < 1 ||
+      start < 0 || n_tokens < 0 || max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(start) + n_tokens > max_tokens) return AATC_ERR_CAPACITY;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
+  if (n_tokens == 0) return AATC_OK;
+  return cuda_status(aatc::launch_encode(*plan, layer, K, V, batch, start, n_tokens, cache,
+                                         max_tokens, static_cast<cudaStream_t>(stream)));
+}
+
+aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
+  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
+  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, sp);
+  return AATC_OK;
+}
+
+aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q, const void* cache,
+                                    int32_t batch, int32_t n_ctx, int32_t max_tokens, float* out,
+                                    void* workspace, size_t workspace_bytes, void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !q || !cache || !out || !workspace || layer < 0 || layer >= plan->dims.n_layers ||
+      batch < 1 || n_ctx < 1 || max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
+  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if (!aligned16(cache) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
+  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
+  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, sp)) return AATC_ERR_WORKSPACE;
+  return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
+                                         workspace, sp, static_cast<cudaStream_t>(stream)));
+}
+
+aatc_status_t aatc_dequantize(aatc_plan_t p, int32_t layer, const void* cache, int32_t batch,
+                              int32_t t0, int32_t n, int32_t max_tokens, float* coeffs_out,
+                              void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !cache || !coeffs_out || layer < 0 || layer >= plan->dims.n_layers || batch < 1 ||
+      t0 < 0 || n < 0 || max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(t0) + n > max_tokens) return AATC_ERR_CAPACITY;
+  if (n == 0) return AATC_OK;
+  return cuda_status(aatc::launch_dequant(*plan, layer, cache, batch, t0, n, max_tokens, coeffs_out,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
+aatc_status_t aatc_get_device_error(aatc_plan_t p, int32_t* flags, int32_t clear) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !flags) return AATC_ERR_INVALID_ARG;
+  int32_t h[4] = {0, 0, 0, 0};
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(h, plan->dev.err, sizeof(h), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && clear) e = cudaMemset(plan->dev.err, 0, sizeof(h));
+  if (e != cudaSuccess) return cuda_status(e);
+  *flags = h[0];
+  return AATC_OK;
+}
+
+aatc_status_t aatc_bf16_decode_workspace_bytes(int32_t batch, int32_t n_kv, int32_t n_q, int32_t n_ctx,
+                                               size_t* bytes) {
+  if (!bytes || batch < 1 || n_kv < 1 || n_q < n_kv || n_q % n_kv || n_ctx < 1) return AATC_ERR_INVALID_ARG;
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    sms = 1;
+  *bytes = aatc::decode_workspace(batch, n_q, aatc::decode_split(batch, n_kv, n_ctx, sms));
+  return AATC_OK;
+}
+
+aatc_status_t aatc_bf16_decode_attention(const void* K, const void* V, const void* q, int32_t batch,
+                                         int32_t n_ctx, int32_t max_tokens, int32_t n_kv, int32_t n_q,
+                                         float* out, void* workspace, size_t workspace_bytes,
+                                         void* stream) {
+  if (!K || !V || !q || !out || !workspace || batch < 1 || n_ctx < 1 || n_kv < 1 || n_q < n_kv ||
+      n_q % n_kv || max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
+  if (n_q / n_kv > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if (!aligned16(K) || !aligned16(V) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_status(e);
+  const auto sp = aatc::decode_split(batch, n_kv, n_ctx, sms);
+  if (workspace_bytes < aatc::decode_workspace(batch, n_q, sp)) return AATC_ERR_WORKSPACE;
+  return cuda_status(aatc::launch_bf16_decode(K, V, q, batch, n_ctx, max_tokens, n_kv, n_q, out,
+                                              workspace, sp, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

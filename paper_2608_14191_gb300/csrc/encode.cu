@@ -1,0 +1,314 @@
+// AATC encode on sm_103a (Algorithm 1 "Project" + "Append qtz(h)"; quantizer of Sec. 5).
+//
+// One persistent CTA per (basis, slice of work): a basis is one (layer, kv-head, K|V) stream,
+// an item is 128 consecutive new tokens of one sequence.  Warp roles:
+//   warp 4  : TMA producer -- 128 x 128 bf16 token tiles into a 3-stage SW128 ring,
+//   warp 5  : MMA issuer   -- tcgen05.mma (M=128 tokens, N=128 channels, K=128) into one of
+//                             two TMEM accumulators,
+//   warps 0-3: epilogue    -- thread = token = TMEM lane: token scale alpha, quantize, pack the
+//                             offset-binary fields and store the word-planar record.
+// The projection uses the plan's bf16 basis; accumulation is fp32.
+#include <cudaTypedefs.h>
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "aatc_internal.h"
+#include "ptx.cuh"
+
+namespace aatc {
+namespace {
+
+constexpr int kStages = 3;
+constexpr int kTileBytes = TILE * D * 2;          // 32 KB of bf16
+constexpr int kThreads = 192;
+constexpr int kAccCols = 128;                     // fp32 columns per accumulator
+constexpr uint32_t kTmemCols = 256;               // two accumulators
+
+struct EncodeArgs {
+  const ChanEnc* enc;     // plan tables (whole plan)
+  const int* sched;
+  const float* inv_s;
+  const int* nret;
+  int* err;
+  uint32_t* words;        // cache word region (this layer)
+  float* alpha;           // cache alpha region
+  int layer, n_kv, batch, start, n_tokens, n_chunks, n_words, n_tiles, ctas_per_basis;
+};
+
+struct EncodeSmem {
+  // 1024-aligned tiles first
+  alignas(1024) unsigned char u_tile[kTileBytes];
+  alignas(1024) unsigned char x_tile[kStages][kTileBytes];
+  ChanEnc enc[D];
+  float inv_s[D];
+  int sched[D];
+  uint64_t full[kStages], empty[kStages], tfull[2], tempty[2], ubar;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__device__ __forceinline__ void raise_abort(EncodeSmem& sm, int* err) {
+  sm.abort_flag = 1;
+  atomicOr(err, 2);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    aatc_encode_kernel(const __grid_constant__ CUtensorMap tmap_k, const __grid_constant__ CUtensorMap tmap_v,
+                       const __grid_constant__ CUtensorMap tmap_u, const EncodeArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  EncodeSmem& sm = *reinterpret_cast<EncodeSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+
+  const int basis = blockIdx.x / a.ctas_per_basis;           // (kv-head, kind) inside the layer
+  const int sub = blockIdx.x % a.ctas_per_basis;
+  const int head = basis >> 1, kind = basis & 1;
+  const int stream = (a.layer * a.n_kv + head) * 2 + kind;
+  const long n_items = static_cast<long>(a.batch) * a.n_chunks;
+  const long it0 = n_items * sub / a.ctas_per_basis;
+  const long it1 = n_items * (sub + 1) / a.ctas_per_basis;
+  const int my_items = static_cast<int>(it1 - it0);
+  const CUtensorMap* tmap_x = kind == 0 ? &tmap_k : &tmap_v;
+
+  // per-channel tables of this stream
+  for (int c = tid; c < D; c += kThreads) {
+    sm.enc[c] = a.enc[stream * D + c];
+    sm.inv_s[c] = a.inv_s[stream * D + c];
+    sm.sched[c] = a.sched[stream * D + c];
+  }
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      ptx::mbar_init(&sm.full[s], 1);
+      ptx::mbar_init(&sm.empty[s], 1);
+    }
+    for (int j = 0; j < 2; ++j) {
+      ptx::mbar_init(&sm.tfull[j], 1);
+      ptx::mbar_init(&sm.tempty[j], 128);
+    }
+    ptx::mbar_init(&sm.ubar, 1);
+    sm.abort_flag = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 5) {
+    ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && my_items > 0) {
+      ptx::prefetch_tmap(tmap_x);
+      ptx::prefetch_tmap(&tmap_u);
+      ptx::mbar_arrive_expect_tx(&sm.ubar, kTileBytes);
+      ptx::tma_load_2d(sm.u_tile, &tmap_u, &sm.ubar, 0, stream * D);
+      ptx::tma_load_2d(sm.u_tile + kTileBytes / 2, &tmap_u, &sm.ubar, 64, stream * D);
+      for (int it = 0; it < my_items; ++it) {
+        const int s = it % kStages;
+        const uint32_t ph = (it / kStages) & 1;
+        if (!ptx::mbar_wait_bounded(&sm.empty[s], ph ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
+        const long item = it0 + it;
+        const int b = static_cast<int>(item / a.n_chunks);
+        const int i0 = static_cast<int>(item % a.n_chunks) * TILE;
+        ptx::mbar_arrive_expect_tx(&sm.full[s], kTileBytes);
+        ptx::tma_load_4d(sm.x_tile[s], tmap_x, &sm.full[s], 0, head, i0, b);
+        ptx::tma_load_4d(sm.x_tile[s] + kTileBytes / 2, tmap_x, &sm.full[s], 64, head, i0, b);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && my_items > 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128);
+      const uint32_t u_base = ptx::smem_u32(sm.u_tile);
+      bool ok = ptx::mbar_wait_bounded(&sm.ubar, 0, abort_flag);
+      if (!ok) raise_abort(sm, a.err);
+      for (int it = 0; ok && it < my_items; ++it) {
+        const int s = it % kStages;
+        const uint32_t ph = (it / kStages) & 1;
+        const int acc = it & 1;
+        const uint32_t aph = (it >> 1) & 1;
+        if (!ptx::mbar_wait_bounded(&sm.tempty[acc], aph ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
+        ptx::tc_fence_after();
+        if (!ptx::mbar_wait_bounded(&sm.full[s], ph, abort_flag)) { raise_abort(sm, a.err); break; }
+        ptx::tc_fence_after();
+        const uint32_t x_base = ptx::smem_u32(sm.x_tile[s]);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t koff = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          ptx::umma_bf16(tmem + acc * kAccCols, ptx::sdesc_kmajor_sw128(x_base + koff),
+                         ptx::sdesc_kmajor_sw128(u_base + koff), idesc, kk > 0 ? 1u : 0u);
+        }
+        ptx::umma_commit(&sm.empty[s]);
+        ptx::umma_commit(&sm.tfull[acc]);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue: thread = token
+    const int R = a.nret[stream];
+    const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
+    for (int it = 0; it < my_items; ++it) {
+      const int acc = it & 1;
+      const uint32_t aph = (it >> 1) & 1;
+      if (!ptx::mbar_wait_bounded(&sm.tfull[acc], aph, abort_flag)) { raise_abort(sm, a.err); break; }
+      ptx::tc_fence_after();
+      float h[D];
+      const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(warp * 32) << 16);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) ptx::tmem_ld_32cols(taddr + 32 * j, h + 32 * j);
+      ptx::tmem_ld_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&sm.tempty[acc]);
+
+      const long item = it0 + it;
+      const int b = static_cast<int>(item / a.n_chunks);
+      const int i = static_cast<int>(item % a.n_chunks) * TILE + tid;     // input token index
+      if (i >= a.n_tokens) continue;
+      const int pos = a.start + i;
+      const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
+      uint32_t* wout = a.words + sidx * stream_words + static_cast<size_t>(pos / TILE) * a.n_words * TILE + (pos % TILE);
+
+      // alpha = max_c |h_c| / s_c over retained channels (inv_s = 0 for dropped ones)
+      float amax = 0.0f;
+#pragma unroll
+      for (int c = 0; c < D; c += 4) {
+        const float4 is = *reinterpret_cast<const float4*>(&sm.inv_s[c]);
+        amax = fmaxf(amax, fabsf(h[c]) * is.x);
+        amax = fmaxf(amax, fabsf(h[c + 1]) * is.y);
+        amax = fmaxf(amax, fabsf(h[c + 2]) * is.z);
+        amax = fmaxf(amax, fabsf(h[c + 3]) * is.w);
+      }
+      if (!isfinite(amax)) atomicOr(a.err, 1);
+      a.alpha[sidx * a.n_tiles * TILE + pos] = amax;
+      const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+
+      // quantize + pack, channels in storage order
+      uint32_t word = 0;
+      int wi = 0;
+#pragma unroll
+      for (int c = 0; c < D; ++c) {
+        if (c < R) {
+        const ChanEnc e = sm.enc[c];
+        const int sc = sm.sched[c];
+        float x = fmaf(h[c], e.inv_f * ia, 0.5f);                 // h / Delta + 1/2
+        x = fminf(fmaxf(x, e.lo), e.hi);                           // clamp (bounds are integers)
+        const float y = __fadd_rd(x, e.magic);                     // floor, offset binary in the mantissa
+        const uint32_t u = __float_as_uint(y) - 0x4B400000u;
+        const int sh = sched_shift(sc);
+        word |= u << sh;
+        if (sched_flush(sc)) {
+          wout[static_cast<size_t>(wi) * TILE] = word;
+          ++wi;
+          word = u >> (32 - sh);
+        }
+        }
+      }
+      for (; wi < a.n_words; ++wi) {
+        wout[static_cast<size_t>(wi) * TILE] = word;
+        word = 0;
+      }
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// K or V: bf16 [batch][n_tokens][n_kv][128]; box = 64 dims x 1 head x 128 tokens x 1 sequence.
+cudaError_t make_kv_map(CUtensorMap* map, const void* base, int batch, int n_tokens, int n_kv) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(n_kv),
+                              static_cast<cuuint64_t>(n_tokens), static_cast<cuuint64_t>(batch)};
+  const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(n_kv) * D * 2,
+                                 static_cast<cuuint64_t>(n_tokens) * n_kv * D * 2};
+  const cuuint32_t box[4] = {64, 1, TILE, 1};
+  const cuuint32_t es[4] = {1, 1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t encode_tensor_maps_u(Plan& plan) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  auto* map = reinterpret_cast<CUtensorMap*>(plan.tmap_u);
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(plan.n_streams) * D};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(D) * 2};
+  const cuuint32_t box[2] = {64, TILE};
+  const cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(plan.dev.ubf16_t), dims, strides,
+                   box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  plan.tmap_ok = r == CUDA_SUCCESS;
+  return plan.tmap_ok ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch, int start,
+                          int n_tokens, void* cache, int max_tokens, cudaStream_t st) {
+  static_assert(sizeof(CUtensorMap) == 128, "CUtensorMap size");
+  CUtensorMap mk, mv;
+  cudaError_t e = make_kv_map(&mk, K, batch, n_tokens, plan.dims.n_kv_heads);
+  if (e == cudaSuccess) e = make_kv_map(&mv, V, batch, n_tokens, plan.dims.n_kv_heads);
+  if (e != cudaSuccess) return e;
+  const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
+  EncodeArgs a;
+  a.enc = plan.dev.enc;
+  a.sched = plan.dev.sched;
+  a.inv_s = plan.dev.inv_s;
+  a.nret = plan.dev.nret;
+  a.err = plan.dev.err;
+  a.words = static_cast<uint32_t*>(cache);
+  a.alpha = reinterpret_cast<float*>(static_cast<uint32_t*>(cache) + g.words_elems);
+  a.layer = layer;
+  a.n_kv = plan.dims.n_kv_heads;
+  a.batch = batch;
+  a.start = start;
+  a.n_tokens = n_tokens;
+  a.n_chunks = (n_tokens + TILE - 1) / TILE;
+  a.n_words = plan.n_words;
+  a.n_tiles = g.n_tiles;
+  const int n_basis = 2 * plan.dims.n_kv_heads;
+  const long items_per_basis = static_cast<long>(batch) * a.n_chunks;
+  int k = std::max(1, plan.num_sms / n_basis);
+  if (k > items_per_basis) k = static_cast<int>(items_per_basis);
+  a.ctas_per_basis = k;
+  const size_t smem = sizeof(EncodeSmem) + 1024;
+  static bool attr_done = false;
+  if (!attr_done) {
+    e = cudaFuncSetAttribute(aatc_encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  const auto* mu = reinterpret_cast<const CUtensorMap*>(plan.tmap_u);
+  aatc_encode_kernel<<<n_basis * k, kThreads, smem, st>>>(mk, mv, *mu, a);
+  return cudaGetLastError();
+}
+
+}  // namespace aatc

@@ -1,0 +1,262 @@
+// Host-side AATC planner: calibration statistics, eigenbasis, attention-aware weights,
+// integer reverse water-filling and per-channel scales (Sec. 5 Steps 1-2; Algorithm 1,
+// calibration half).  Plain C++17, fp64, no LAPACK: the eigenbasis comes from a cyclic
+// Jacobi iteration on the 128x128 second-moment matrix.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <numeric>
+#include <thread>
+#include <vector>
+
+#include "aatc.h"
+#include "aatc_internal.h"
+
+namespace aatc {
+namespace {
+
+constexpr int kD = 128;
+
+// C = (1/N) sum_n x_n x_n^T over fp32 rows, accumulated in fp64 (Sec. 5 Step 1: Sigma = X^T X / T).
+void second_moment(const float* x, int n, std::vector<double>& c) {
+  c.assign(kD * kD, 0.0);
+  std::vector<double> row(kD);
+  for (int t = 0; t < n; ++t) {
+    const float* xt = x + static_cast<size_t>(t) * kD;
+    for (int i = 0; i < kD; ++i) row[i] = xt[i];
+    for (int i = 0; i < kD; ++i) {
+      const double xi = row[i];
+      double* ci = c.data() + i * kD;
+      for (int j = i; j < kD; ++j) ci[j] += xi * row[j];
+    }
+  }
+  const double inv = 1.0 / n;
+  for (int i = 0; i < kD; ++i)
+    for (int j = i; j < kD; ++j) {
+      c[i * kD + j] *= inv;
+      c[j * kD + i] = c[i * kD + j];
+    }
+}
+
+// Cyclic Jacobi: rotate away each off-diagonal element in turn until the off-diagonal mass is
+// negligible.  a is overwritten (its diagonal converges to the eigenvalues); v accumulates the
+// rotations, so columns of v are the eigenvectors.
+void jacobi_eigen(std::vector<double>& a, std::vector<double>& v) {
+  v.assign(kD * kD, 0.0);
+  for (int i = 0; i < kD; ++i) v[i * kD + i] = 1.0;
+  double frob = 0.0;
+  for (double e : a) frob += e * e;
+  const double tiny = 1e-300;
+  for (int sweep = 0; sweep < 100; ++sweep) {
+    double off = 0.0;
+    for (int p = 0; p < kD; ++p)
+      for (int q = p + 1; q < kD; ++q) off += a[p * kD + q] * a[p * kD + q];
+    if (off <= 1e-30 * frob || off < tiny) break;
+    for (int p = 0; p < kD - 1; ++p) {
+      for (int q = p + 1; q < kD; ++q) {
+        const double apq = a[p * kD + q];
+        if (std::fabs(apq) < tiny) continue;
+        const double app = a[p * kD + p], aqq = a[q * kD + q];
+        // Choose the rotation angle that zeroes a_pq: tan(2 phi) = 2 a_pq / (a_qq - a_pp),
+        // taking the smaller root t = tan(phi) for stability.
+        const double theta = (aqq - app) / (2.0 * apq);
+        const double t = (theta >= 0 ? 1.0 : -1.0) / (std::fabs(theta) + std::sqrt(theta * theta + 1.0));
+        const double c = 1.0 / std::sqrt(t * t + 1.0);
+        const double s = t * c;
+        for (int k = 0; k < kD; ++k) {          // A <- A J (columns p, q)
+          const double akp = a[k * kD + p], akq = a[k * kD + q];
+          a[k * kD + p] = c * akp - s * akq;
+          a[k * kD + q] = s * akp + c * akq;
+        }
+        for (int k = 0; k < kD; ++k) {          // A <- J^T A (rows p, q)
+          const double apk = a[p * kD + k], aqk = a[q * kD + k];
+          a[p * kD + k] = c * apk - s * aqk;
+          a[q * kD + k] = s * apk + c * aqk;
+        }
+        a[p * kD + q] = a[q * kD + p] = 0.0;
+        for (int k = 0; k < kD; ++k) {          // V <- V J
+          const double vkp = v[k * kD + p], vkq = v[k * kD + q];
+          v[k * kD + p] = c * vkp - s * vkq;
+          v[k * kD + q] = s * vkp + c * vkq;
+        }
+      }
+    }
+  }
+}
+
+double percentile99(std::vector<double>& vals) {
+  std::sort(vals.begin(), vals.end());
+  const double pos = 0.99 * static_cast<double>(vals.size() - 1);
+  const size_t lo = static_cast<size_t>(std::floor(pos));
+  const size_t hi = std::min(lo + 1, vals.size() - 1);
+  return vals[lo] + (pos - static_cast<double>(lo)) * (vals[hi] - vals[lo]);
+}
+
+struct StreamJob {
+  const float* x;              // calibration vectors [n][128]
+  int n;
+  const float* const* q_heads; // query heads of the group (keys only) or nullptr
+  int n_q_heads_in_group;
+  int n_q;
+  int budget;
+  int b_max;
+  bool var_only;
+  float* basis_out;            // [128][128]
+  uint8_t* bits_out;           // [128]
+  float* scales_out;           // [128]
+  double* sigma2_out;          // [128] or null
+  double* weights_out;         // [128] or null
+};
+
+void plan_one_stream(const StreamJob& job) {
+  std::vector<double> c, v;
+  second_moment(job.x, job.n, c);
+  jacobi_eigen(c, v);
+  // eigenvalues descending (stable on the Jacobi index order), canonical signs
+  std::vector<int> ord(kD);
+  std::iota(ord.begin(), ord.end(), 0);
+  std::stable_sort(ord.begin(), ord.end(), [&](int i, int j) { return c[i * kD + i] > c[j * kD + j]; });
+  std::vector<double> lam(kD), u(kD * kD);   // u[d][k]
+  for (int k = 0; k < kD; ++k) {
+    const int src = ord[k];
+    lam[k] = c[src * kD + src];
+    int imax = 0;
+    double amax = -1.0;
+    for (int d = 0; d < kD; ++d) {
+      const double a = std::fabs(v[d * kD + src]);
+      if (a > amax) { amax = a; imax = d; }
+    }
+    const double sgn = v[imax * kD + src] < 0 ? -1.0 : 1.0;
+    for (int d = 0; d < kD; ++d) u[d * kD + k] = sgn * v[d * kD + src];
+  }
+  // weights: w^K_c = sum_heads u_c^T M_j u_c with M_j = mean_i q_i q_i^T; w^V_c = 1
+  std::vector<double> w(kD, 1.0);
+  if (!job.var_only && job.q_heads != nullptr) {
+    std::vector<double> m(kD * kD, 0.0), mj;
+    for (int j = 0; j < job.n_q_heads_in_group; ++j) {
+      second_moment(job.q_heads[j], job.n_q, mj);
+      for (int i = 0; i < kD * kD; ++i) m[i] += mj[i];
+    }
+    for (int k = 0; k < kD; ++k) {
+      double acc = 0.0;
+      for (int i = 0; i < kD; ++i) {
+        double row = 0.0;
+        for (int j2 = 0; j2 < kD; ++j2) row += m[i * kD + j2] * u[j2 * kD + k];
+        acc += u[i * kD + k] * row;
+      }
+      w[k] = acc;
+    }
+  }
+  // storage order: g = w * sigma^2 descending, stable
+  std::vector<double> g(kD);
+  for (int k = 0; k < kD; ++k) g[k] = w[k] * lam[k];
+  std::vector<int> so(kD);
+  std::iota(so.begin(), so.end(), 0);
+  std::stable_sort(so.begin(), so.end(), [&](int i, int j) { return g[i] > g[j]; });
+  std::vector<double> gs(kD);
+  for (int c2 = 0; c2 < kD; ++c2) gs[c2] = g[so[c2]];
+  // exact integer reverse water-filling by marginal gains (gain of one more bit on channel c at
+  // b_c bits is (3/4) g_c 4^-b_c; the 3/4 is common), ties to the lower storage index
+  std::vector<int> bits(kD, 0);
+  for (int it = 0; it < job.budget; ++it) {
+    int best = -1;
+    double bg = -1.0;
+    for (int c2 = 0; c2 < kD; ++c2) {
+      if (bits[c2] >= job.b_max) continue;
+      const double gain = std::ldexp(gs[c2], -2 * bits[c2]);
+      if (best < 0 || gain > bg) { best = c2; bg = gain; }
+    }
+    if (best < 0) break;
+    ++bits[best];
+  }
+  // scales: 99th percentile of |u_c . x| over the calibration vectors
+  std::vector<double> h(static_cast<size_t>(job.n) * kD, 0.0);
+  for (int t = 0; t < job.n; ++t) {
+    const float* xt = job.x + static_cast<size_t>(t) * kD;
+    double* ht = h.data() + static_cast<size_t>(t) * kD;
+    for (int d = 0; d < kD; ++d) {
+      const double xd = xt[d];
+      const double* ud = u.data() + d * kD;
+      for (int k = 0; k < kD; ++k) ht[k] += xd * ud[k];
+    }
+  }
+  std::vector<double> col(job.n);
+  for (int c2 = 0; c2 < kD; ++c2) {
+    const int k = so[c2];
+    for (int t = 0; t < job.n; ++t) col[t] = std::fabs(h[static_cast<size_t>(t) * kD + k]);
+    job.scales_out[c2] = static_cast<float>(percentile99(col));
+    job.bits_out[c2] = static_cast<uint8_t>(bits[c2]);
+    for (int d = 0; d < kD; ++d) job.basis_out[d * kD + c2] = static_cast<float>(u[d * kD + k]);
+    if (job.sigma2_out) job.sigma2_out[c2] = lam[k];
+    if (job.weights_out) job.weights_out[c2] = w[k];
+  }
+}
+
+bool budget_from_avg(double avg, int b_max, int* budget) {
+  const double b = avg * kD;
+  const double r = std::nearbyint(b);
+  if (!std::isfinite(b) || std::fabs(b - r) > 1e-9 || r < 0 || r > static_cast<double>(b_max) * kD) return false;
+  *budget = static_cast<int>(r);
+  return true;
+}
+
+}  // namespace
+}  // namespace aatc
+
+extern "C" aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k,
+                                        const float* calib_v, int32_t n_calib, const float* calib_q,
+                                        int32_t n_calib_q, double avg_bits_k, double avg_bits_v,
+                                        int32_t weights_mode, float* basis_out, uint8_t* bits_out,
+                                        float* scales_out, double* sigma2_out, double* weights_out,
+                                        int32_t n_threads) {
+  using namespace aatc;
+  if (!valid_dims(dims) || !calib_k || !calib_v || !basis_out || !bits_out || !scales_out)
+    return AATC_ERR_INVALID_ARG;
+  if (n_calib < 2 || (calib_q && n_calib_q < 1) || (weights_mode != 0 && weights_mode != 1))
+    return AATC_ERR_INVALID_ARG;
+  int bk = 0, bv = 0;
+  if (!budget_from_avg(avg_bits_k, dims->b_max, &bk) || !budget_from_avg(avg_bits_v, dims->b_max, &bv))
+    return AATC_ERR_BUDGET;
+  const int L = dims->n_layers, H = dims->n_kv_heads, HQ = dims->n_q_heads, G = HQ / H;
+  const size_t cal = static_cast<size_t>(n_calib) * kD;
+  const size_t qsz = static_cast<size_t>(n_calib_q) * kD;
+  std::vector<const float*> qptr(static_cast<size_t>(L) * HQ, nullptr);
+  if (calib_q)
+    for (int l = 0; l < L; ++l)
+      for (int j = 0; j < HQ; ++j) qptr[static_cast<size_t>(l) * HQ + j] = calib_q + (static_cast<size_t>(l) * HQ + j) * qsz;
+  std::vector<StreamJob> jobs;
+  for (int l = 0; l < L; ++l)
+    for (int h = 0; h < H; ++h)
+      for (int kind = 0; kind < 2; ++kind) {
+        const size_t s = (static_cast<size_t>(l) * H + h) * 2 + kind;
+        const size_t lh = static_cast<size_t>(l) * H + h;
+        StreamJob j;
+        j.x = (kind == 0 ? calib_k : calib_v) + lh * cal;
+        j.n = n_calib;
+        j.q_heads = (kind == 0 && calib_q) ? qptr.data() + static_cast<size_t>(l) * HQ + static_cast<size_t>(h) * G : nullptr;
+        j.n_q_heads_in_group = G;
+        j.n_q = n_calib_q;
+        j.budget = kind == 0 ? bk : bv;
+        j.b_max = dims->b_max;
+        j.var_only = weights_mode == 1;
+        j.basis_out = basis_out + s * kD * kD;
+        j.bits_out = bits_out + s * kD;
+        j.scales_out = scales_out + s * kD;
+        j.sigma2_out = sigma2_out ? sigma2_out + s * kD : nullptr;
+        j.weights_out = weights_out ? weights_out + s * kD : nullptr;
+        jobs.push_back(j);
+      }
+  int nt = n_threads > 0 ? n_threads : static_cast<int>(std::thread::hardware_concurrency());
+  nt = std::max(1, std::min<int>(nt, static_cast<int>(jobs.size())));
+  std::atomic<size_t> next{0};
+  auto worker = [&]() {
+    for (size_t i = next++; i < jobs.size(); i = next++) plan_one_stream(jobs[i]);
+  };
+  std::vector<std::thread> pool;
+  for (int t = 1; t < nt; ++t) pool.emplace_back(worker);
+  worker();
+  for (auto& th : pool) th.join();
+  return AATC_OK;
+}

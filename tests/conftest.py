@@ -25,3 +25,13 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def aatc():
+    """The built library's Python binding (builds libaatc.so in-tree if it is missing)."""
+    from paper_2608_14191_gb300 import build as b
+    b.build()
+    import paper_2608_14191_gb300 as m
+    m.load()
+    return m
