@@ -1,0 +1,451 @@
+"""Benchmark of the AATC hot path on GB300: encode + decode attention over the packed cache.
+
+Workload (default): the Llama-3.1-8B-shaped single layer -- 32 query heads, 8 kv-heads,
+head_dim 128, batch 1, context 32768, 2.75 average bits.  One *step* = encode the full context
+(32768 tokens x 8 kv-heads, K and V) into the packed cache, then 256 decode-attention steps with
+random bf16 queries.  Inputs are synthetic (workloads/: seeded anisotropic Gaussian KV).
+
+Reported metric (one JSON line): decode-attention GB/s on algorithmic packed-cache bytes
+(codes + per-token scales, 96 B per token and kv-head at 2.75 bits) and its fraction of the
+measured HBM copy bandwidth; encode Mtok/s alongside.  The packed cache is 25 MB, smaller than
+L2, so the decodes rotate over 16 cache copies (403 MB > 129 MB L2).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun (N > 1) every rank runs the same workload on its own GPU (weak scaling; the
+path has no data exchange); rank 0 prints the line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+METRIC = "compressed-KV decode attn GB/s & % of HBM peak; encode Mtok/s (1 GB300)"
+N_COPIES = 16
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
+DECODE_SRC = os.path.join(ROOT, "paper_2608_14191_gb300", "csrc", "decode.cu")
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    return ws, rank
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.out,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _source_hash(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def _traffic_per_launch():
+    """DRAM bytes per decode launch from the committed ncu summary, if it was taken on this source."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    with open(TRAFFIC_FILE) as f:
+        d = json.load(f)
+    if d.get("decode_cu_sha256_16") != _source_hash(DECODE_SRC):
+        return None
+    return d.get("bytes_per_decode_call")
+
+
+def build_case(aatc, cfg, avg_bits, device):
+    ck, cv, cq = W.layer_calibration(cfg, 0)
+    dm = aatc.dims(1, cfg.n_kv_heads, cfg.n_q_heads)
+    p = aatc.calibrate(dm, ck[None], cv[None], cq[None], avg_bits)
+    plan = aatc.Plan(dm, p["basis"], p["bits"], p["scales"])
+    return plan, p
+
+
+def decode_bytes(plan, cfg, batch, n_ctx):
+    """Algorithmic bytes one decode reads: packed codes (sum of widths) + fp32 alpha, K and V."""
+    bits = plan._bits.reshape(-1, 2, 128).astype(np.int64).sum(axis=2)      # (H_kv, 2) code bits per token
+    per_token = float(np.sum(bits) / 8.0 + 4 * bits.size)
+    return batch * n_ctx * per_token
+
+
+# ------------------------------------------------------------------------------------ our arm
+
+def run_ours(args):
+    import torch
+    import paper_2608_14191_gb300 as aatc
+    from paper_2608_14191_gb300 import build as bld
+
+    ws_, rank = _dist()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws_ > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0 or not os.path.exists(bld.LIB):
+        bld.build()
+    if ws_ > 1:
+        torch.distributed.barrier()
+    aatc.load()
+
+    cfg = W.CONFIGS[args.config]
+    avg_bits = cfg.avg_bits[-1] if args.bits is None else args.bits
+    B, T, steps_dec = cfg.batch, cfg.n_ctx, cfg.decode_steps
+    plan, _ = build_case(aatc, cfg, avg_bits, dev)
+    kd, vd = W.kv_device(cfg, 0, B, T, dev)
+    qs = W.queries_device(cfg, 0, B, steps_dec, dev)
+    caches = [plan.new_cache(B, T, dev) for _ in range(N_COPIES)]
+    for c in caches:
+        aatc.encode(plan, 0, kd, vd, c, 0, T)
+    out = torch.empty((steps_dec, B, cfg.n_q_heads, 128), dtype=torch.float32, device=dev)
+    wsb = plan.workspace_bytes(B, T)
+    wspace = torch.empty(wsb // 4, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+
+    def decodes(step):
+        for i in range(steps_dec):
+            aatc.decode_attention(plan, 0, qs[i], caches[(step * steps_dec + i) % N_COPIES], T, T, out=out[i],
+                                  workspace=wspace)
+
+    # CUDA graphs of the 256 decode calls, one per rotation offset (a step's decodes start at
+    # copy (step * 256) % 16 = 0, so one graph serves every step)
+    for _ in range(2):
+        decodes(0)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        decodes(0)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+
+    def step_dev(s, e3=None):
+        if e3:
+            e3[0].record(stream)
+        aatc.encode(plan, 0, kd, vd, caches[s % N_COPIES], 0, T)
+        if e3:
+            e3[1].record(stream)
+        graph.replay()
+        if e3:
+            e3[2].record(stream)
+
+    for s in range(args.warmup):
+        step_dev(s)
+    torch.cuda.synchronize()
+    if ws_ > 1:
+        torch.distributed.barrier()
+    with ClockSampler(local) as clk:
+        torch.cuda.synchronize()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for s in range(args.steps):
+            step_dev(s, ev[s])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if ws_ > 1:
+        torch.distributed.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    enc_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    clocks = clk.summary()
+
+    # end to end through the public API from pinned host buffers (no graphs)
+    kh = torch.empty(kd.shape, dtype=torch.bfloat16, pin_memory=True)
+    vh = torch.empty(vd.shape, dtype=torch.bfloat16, pin_memory=True)
+    qh = torch.empty(qs.shape, dtype=torch.bfloat16, pin_memory=True)
+    oh = torch.empty(out.shape, dtype=torch.float32, pin_memory=True)
+    kh.copy_(kd)
+    vh.copy_(vd)
+    qh.copy_(qs)
+    kd2, vd2, qs2 = torch.empty_like(kd), torch.empty_like(vd), torch.empty_like(qs)
+
+    def step_e2e(s):
+        kd2.copy_(kh, non_blocking=True)
+        vd2.copy_(vh, non_blocking=True)
+        qs2.copy_(qh, non_blocking=True)
+        aatc.encode(plan, 0, kd2, vd2, caches[s % N_COPIES], 0, T)
+        for i in range(steps_dec):
+            aatc.decode_attention(plan, 0, qs2[i], caches[(s * steps_dec + i) % N_COPIES], T, T, out=out[i],
+                                  workspace=wspace)
+        oh.copy_(out, non_blocking=True)
+
+    e2e_steps = max(1, min(args.steps, 10))
+    for s in range(2):
+        step_e2e(s)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(e2e_steps):
+        step_e2e(s)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    h2d = kd.numel() * 2 + vd.numel() * 2 + qs.numel() * 2
+    d2h = out.numel() * 4
+    assert plan.device_error() == 0
+
+    # max over ranks
+    vals = torch.tensor([total_ms, float(np.mean(dec_ms)), float(np.mean(enc_ms)), e2e_ms], device=dev)
+    if ws_ > 1:
+        torch.distributed.all_reduce(vals, op=torch.distributed.ReduceOp.MAX)
+    total_ms, dec_mean, enc_mean, e2e_ms = [float(x) for x in vals.cpu()]
+    if rank != 0:
+        if ws_ > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    peak, peak_kind = _peaks()
+    dbytes = decode_bytes(plan, cfg, B, T)
+    per_decode_ms = dec_mean / steps_dec
+    gbs = ws_ * dbytes / (per_decode_ms * 1e-3) / 1e9           # whole job
+    achieved = dbytes / (per_decode_ms * 1e-3) / 1e9              # per launch (one GPU)
+    enc_tokens = B * T
+    enc_in_bytes = B * T * cfg.n_kv_heads * 2 * 128 * 2
+    line = {
+        "metric": METRIC,
+        "value": round(gbs, 2),
+        "unit": "GB/s",
+        "n_gpus": ws_,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(total_ms / args.steps, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic (seeded anisotropic Gaussian KV, power-law spectrum, key outliers; bf16)",
+        "config": {"workload": cfg.workload, "avg_bits": avg_bits, "batch": B, "n_ctx": T,
+                   "n_kv_heads": cfg.n_kv_heads, "n_q_heads": cfg.n_q_heads, "decode_steps_per_step": steps_dec,
+                   "l2": f"decodes rotate over {N_COPIES} packed-cache copies "
+                         f"({N_COPIES * dbytes / 1e6:.0f} MB > 129 MB L2); encode input {enc_in_bytes / 1e6:.0f} MB",
+                   "parallelism": f"replica x{ws_}", "decode_graph": "256 decode calls replayed as one CUDA graph"},
+        "decode": {"gbs": round(achieved, 2), "us_per_call": round(per_decode_ms * 1e3, 3),
+                   "bytes_per_call": dbytes, "frac_of_measured_hbm": round(achieved / peak, 4),
+                   "frac_of_nominal_8tbs": round(achieved / 8000.0, 4)},
+        "encode": {"mtok_s": round(ws_ * enc_tokens / (enc_mean * 1e-3) / 1e6, 2),
+                   "us_per_call": round(enc_mean * 1e3, 2),
+                   "input_gbs": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9, 2),
+                   "frac_of_measured_hbm_on_input": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9 / peak, 4)},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": _traffic_per_launch(),
+                     "kernel": "aatc_decode_split_kernel + aatc_decode_combine_kernel (one decode call)",
+                     "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"},
+        "e2e": {"value": round(ws_ * steps_dec * dbytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                "ms_per_step": round(e2e_ms, 4),
+                "what": "per step: H2D of K, V and queries from pinned host memory, encode, 256 decode calls "
+                        "through the public API, D2H of all outputs"},
+        "gpu_launches": args.steps * (1 + 2 * steps_dec),
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+    if ws_ > 1:
+        torch.distributed.destroy_process_group()
+
+
+# ------------------------------------------------------------------------------ oracle baseline
+
+_ORACLE_CHILD = r"""
+import json, os, sys, time
+import numpy as np
+sys.path.insert(0, sys.argv[1])
+from oracle import aatc_oracle as O
+d = np.load(sys.argv[2])
+budget = float(sys.argv[3])
+g = int(d["group"]); hkv = int(d["hkv"])
+t0 = time.perf_counter(); n_done = 0; bytes_done = 0.0
+while True:
+    for h in range(hkv):
+        hh = []
+        for kind in (0, 1):
+            bits = d["bits"][h, kind].astype(np.int64)
+            codes = O.unpack_records(d["records"][h, kind], bits)
+            hh.append(O.dequantize_f32(codes, d["alpha"][h, kind], d["scales"][h, kind], bits))
+        O.decode_attention(d["q"][h * g:(h + 1) * g], hh[0][None], hh[1][None], d["basis"][h, 0][None],
+                           d["basis"][h, 1][None], g)
+    n_done += 1
+    bytes_done += float(d["bytes"])
+    if time.perf_counter() - t0 > budget:
+        break
+el = time.perf_counter() - t0
+print(json.dumps({"seconds": el, "decodes": n_done, "bytes": bytes_done}))
+"""
+
+
+def oracle_sample(cfg, avg_bits, n_tokens):
+    """CPU-only input for the oracle: its own plan (from the library's numpy twin: the oracle
+    planner) and its own encode of n_tokens per stream."""
+    from oracle import aatc_oracle as O
+    ck, cv, cq = W.layer_calibration(cfg, 0)
+    k, v = W.kv_host(cfg, 0, 1, n_tokens)
+    g = cfg.group
+    H = cfg.n_kv_heads
+    recs, alphas, bits_all, scales_all, basis_all = [], [], [], [], []
+    for h in range(H):
+        rr, aa, bb, ss, uu = [], [], [], [], []
+        for kind, x, cal in ((0, k, ck), (1, v, cv)):
+            qsh = [cq[j].astype(np.float64) for j in range(h * g, (h + 1) * g)] if kind == 0 else None
+            p = O.plan_stream(cal[h].astype(np.float64), avg_bits, queries_by_head=qsh)
+            ub = W.to_bf16(p["basis"]).astype(np.float64)
+            codes, alpha, _ = O.encode_stream(x[0, :, h, :].astype(np.float64), ub, p["bits"], p["scales"])
+            nw = O.record_words([p["bits"]])
+            rr.append(O.pack_records(codes, p["bits"], nw))
+            aa.append(alpha.astype(np.float32))
+            bb.append(p["bits"])
+            ss.append(p["scales"].astype(np.float32))
+            uu.append(p["basis"].astype(np.float32))
+        nw = max(r.shape[1] for r in rr)
+        rr = [np.pad(r, ((0, 0), (0, nw - r.shape[1]))) for r in rr]
+        recs.append(rr)
+        alphas.append(aa)
+        bits_all.append(bb)
+        scales_all.append(ss)
+        basis_all.append(uu)
+    q = W.queries_host(cfg, 0, 1, 1)[0, 0]
+    bits_arr = np.array(bits_all)
+    per_token = float(np.sum(bits_arr) / 8.0 + 4 * H * 2)
+    return {"records": np.array(recs), "alpha": np.array(alphas), "bits": bits_arr,
+            "scales": np.array(scales_all), "basis": np.array(basis_all), "q": q, "group": g, "hkv": H,
+            "bytes": per_token * n_tokens}
+
+
+def cpu_baseline(cfg, avg_bits, budget_s=15.0, n_tokens=4096):
+    """Oracle decode (unpack + fp32 dequant + fp64 attention) timed on one host thread over a
+    bounded sample: all 32 q-heads over the first n_tokens tokens, repeated for ~budget_s s."""
+    sample = oracle_sample(cfg, avg_bits, n_tokens)
+    with tempfile.TemporaryDirectory() as td:
+        path = os.path.join(td, "sample.npz")
+        np.savez(path, **sample)
+        env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, "-c", _ORACLE_CHILD, ROOT, path, str(budget_s)], capture_output=True,
+                           text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        return {"value": None, "unit": "GB/s", "cores": 1, "kind": "oracle", "error": r.stderr[-300:]}
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": round(res["bytes"] / res["seconds"] / 1e9, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"oracle decode of all {cfg.n_q_heads} q-heads over the first {n_tokens} tokens "
+                      f"(numpy fp64, 1 thread), {res['decodes']} repetitions in {res['seconds']:.1f} s"}
+
+
+def run_reference(args):
+    ws_, rank = _dist()
+    if rank != 0:
+        return
+    cfg = W.CONFIGS[args.config]
+    avg_bits = cfg.avg_bits[-1] if args.bits is None else args.bits
+    per_step = max(1.0, min(10.0, 120.0 / max(1, args.steps + args.warmup)))
+    times = []
+    res = None
+    for s in range(args.warmup + args.steps):
+        res = cpu_baseline(cfg, avg_bits, budget_s=per_step, n_tokens=2048)
+        if s >= args.warmup:
+            times.append(res)
+    vals = [r["value"] for r in times if r.get("value")]
+    value = float(np.mean(vals)) if vals else None
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": ws_, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(per_step * 1e3, 1), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.workload, "avg_bits": avg_bits, "batch": cfg.batch, "n_ctx": cfg.n_ctx},
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": (res or {}).get("sample", "")},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="llama_layer", choices=sorted(W.CONFIGS))
+    ap.add_argument("--bits", type=float, default=None)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -541,9 +541,13 @@ size_t split_smem_bytes(int split_len, int n_words) {
 template <int GP>
 cudaError_t launch_split(const DecodeArgs& a, int batch, int n_kv, cudaStream_t st) {
   const size_t smem = split_smem_bytes<GP>(a.split_len, a.n_words);
-  cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
+  static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
   aatc_decode_split_kernel<GP><<<dim3(a.n_splits, n_kv, batch), kThreads, smem, st>>>(a);
   return cudaGetLastError();
 }
@@ -552,9 +556,13 @@ template <int GP>
 cudaError_t launch_bf16_split(const Bf16Args& a, int batch, cudaStream_t st) {
   const size_t smem = 4 * (static_cast<size_t>(D) * GP + 32 + static_cast<size_t>(a.split_len) * GP + 4 * GP * D) +
                       2 * static_cast<size_t>(TILE) * (D + 8) * 2;
-  cudaError_t e = cudaFuncSetAttribute(aatc_bf16_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
+  static size_t smem_set = 0;
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(aatc_bf16_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
   aatc_bf16_split_kernel<GP><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
   return cudaGetLastError();
 }
