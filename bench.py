@@ -428,6 +428,30 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_profile_once(args):
+    """Minimal launch sequence for ncu captures: one encode, two decodes, one bf16 decode."""
+    import torch
+    import paper_2608_14191_gb300 as aatc
+    from paper_2608_14191_gb300 import build as bld
+    bld.build()
+    aatc.load()
+    dev = torch.device("cuda", 0)
+    cfg = W.CONFIGS[args.config]
+    avg_bits = cfg.avg_bits[-1] if args.bits is None else args.bits
+    B, T = cfg.batch, cfg.n_ctx
+    plan, _ = build_case(aatc, cfg, avg_bits, dev)
+    kd, vd = W.kv_device(cfg, 0, B, T, dev)
+    qs = W.queries_device(cfg, 0, B, 2, dev)
+    cache = plan.new_cache(B, T, dev)
+    aatc.encode(plan, 0, kd, vd, cache, 0, T)
+    for i in range(2):
+        aatc.decode_attention(plan, 0, qs[i], cache, T, T)
+    aatc.bf16_decode_attention(kd, vd, qs[0], T)
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    print(json.dumps({"profile_once": cfg.name, "decode_bytes": decode_bytes(plan, cfg, B, T)}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -438,10 +462,13 @@ def main():
     ap.add_argument("--bits", type=float, default=None)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-once", action="store_true", help="one encode + two decodes, for ncu")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.profile_once:
+        run_profile_once(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
