@@ -177,6 +177,33 @@ aatc_status_t aatc_dequantize(aatc_plan_t plan, int32_t layer, const void* cache
 aatc_status_t aatc_get_device_error(aatc_plan_t plan, int32_t* flags, int32_t clear);
 
 /*
+ * Size of the fixed scratch array behind aatc_decode_attention_noalloc (split partials).
+ */
+#define AATC_NOALLOC_SCRATCH_BYTES (4u << 20)
+
+/*
+ * aatc_decode_attention without a caller workspace.  The paper has no counterpart: this entry
+ * point exists for callers that cannot allocate device memory when they call -- for example a
+ * serving runtime that carves up all device memory once at start-up with its own pool and may
+ * not call cudaMalloc on the request path (it would synchronize the device and stall other
+ * streams), or plugin code running inside a framework that does not expose its allocator.
+ * Same arguments, math and outputs as aatc_decode_attention; the split partials go to a fixed
+ * scratch array of AATC_NOALLOC_SCRATCH_BYTES that the library keeps in device memory on every
+ * GPU that loads it, until the process exits.  Nothing is allocated or freed by this call.
+ *   - The first call on a device looks up that device's scratch address (with the device
+ *     current); make that first call before any stream capture.
+ *   - Every call on a device shares the one array, and it keeps the previous call's contents.
+ *     Nothing in it has to start at zero (each partial is written before it is read), but
+ *     calls that overlap on the GPU (different streams, or concurrent host threads) race on it:
+ *     serialize them.
+ * Errors: as aatc_decode_attention, plus AATC_ERR_WORKSPACE when (batch, n_ctx) needs more
+ * than AATC_NOALLOC_SCRATCH_BYTES of partials (see aatc_decode_workspace_bytes).
+ */
+aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t plan, int32_t layer, const void* q,
+                                            const void* cache, int32_t batch, int32_t n_ctx,
+                                            int32_t max_tokens, float* out, void* stream);
+
+/*
  * Reference point: uncompressed bf16 decode attention (Def. sdpa), split-K with the same
  * combine.  K, V: device bf16 [batch][max_tokens][n_kv_heads][128]; attends to [0, n_ctx).
  * q: device bf16 [batch][n_q_heads][128]; out: device fp32 [batch][n_q_heads][128].

@@ -53,6 +53,7 @@ SIGNATURES = {
     "aatc_encode": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _P, _I32, _P]),
     "aatc_decode_workspace_bytes": (_I32, [_P, _I32, _I32, ctypes.POINTER(_SZ)]),
     "aatc_decode_attention": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _P, _P, _SZ, _P]),
+    "aatc_decode_attention_noalloc": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _P, _P]),
     "aatc_dequantize": (_I32, [_P, _I32, _P, _I32, _I32, _I32, _I32, _P, _P]),
     "aatc_get_device_error": (_I32, [_P, ctypes.POINTER(_I32), _I32]),
     "aatc_bf16_decode_workspace_bytes": (_I32, [_I32, _I32, _I32, _I32, ctypes.POINTER(_SZ)]),
@@ -208,6 +209,15 @@ def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: i
     _check(load().aatc_decode_attention(plan.handle, layer, _ptr(q), _ptr(cache), batch, n_ctx, max_tokens,
                                         _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                         _stream(stream)), "aatc_decode_attention")
+    return out
+
+
+def decode_attention_noalloc(plan: Plan, layer: int, q, out, cache, n_ctx: int, max_tokens: int, stream=None):
+    """aatc_decode_attention_noalloc: as decode_attention, but with no workspace and no allocation
+    (the caller passes `out`; the library's fixed scratch holds the split partials)."""
+    _check(load().aatc_decode_attention_noalloc(plan.handle, layer, _ptr(q), _ptr(cache), q.shape[0], n_ctx,
+                                                max_tokens, _ptr(out), _stream(stream)),
+           "aatc_decode_attention_noalloc")
     return out
 
 

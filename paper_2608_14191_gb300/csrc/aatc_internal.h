@@ -94,6 +94,10 @@ struct DecodeSplit {
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
 size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp);
 
+// Handle check and CUDA-status mapping shared by every C entry point (defined in capi.cpp).
+Plan* plan_from_handle(aatc_plan_t p);
+aatc_status_t status_from_cuda(cudaError_t e);
+
 // Kernel launchers (defined in the .cu files); return the CUDA error of the launch.
 cudaError_t encode_tensor_maps_u(Plan& plan);
 cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch,

@@ -53,6 +53,10 @@ DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
   return sp;
 }
 
+Plan* plan_from_handle(aatc_plan_t p) { return as_plan(p); }
+
+aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
+
 size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp) {
   return static_cast<size_t>(batch) * n_q * sp.n_splits * (D + 2) * sizeof(float);
 }

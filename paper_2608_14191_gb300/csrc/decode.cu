@@ -13,6 +13,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "aatc_internal.h"
 
@@ -631,3 +632,51 @@ cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int 
 }
 
 }  // namespace aatc
+
+// ------------------------------------------------------------------ decode without a workspace
+// For callers that cannot allocate device memory at call time (see aatc_decode_attention_noalloc
+// in aatc.h): the split partials live in one fixed array of this file, reserved on every device
+// that loads the library.  Host code must not use the array's name as an address; the device
+// address is looked up once per device with cudaGetSymbolAddress.
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[AATC_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_address[kMaxDevices] = {};
+
+}  // namespace
+
+extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t layer, const void* q,
+                                                       const void* cache, int32_t batch, int32_t n_ctx,
+                                                       int32_t max_tokens, float* out, void* stream) {
+  using namespace aatc;
+  Plan* plan = plan_from_handle(p);
+  if (!plan || !q || !cache || !out || layer < 0 || layer >= plan->dims.n_layers || batch < 1 || n_ctx < 1 ||
+      max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
+  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(cache) & 15u) != 0) return AATC_ERR_INVALID_ARG;
+  const DecodeSplit sp = decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
+  if (decode_workspace(batch, plan->dims.n_q_heads, sp) > AATC_NOALLOC_SCRATCH_BYTES) return AATC_ERR_WORKSPACE;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return status_from_cuda(e);
+  if (dev < 0 || dev >= kMaxDevices) return AATC_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_address[dev]) {
+      e = cudaGetSymbolAddress(&g_noalloc_address[dev], g_noalloc_scratch);
+      if (e != cudaSuccess) {
+        g_noalloc_address[dev] = nullptr;
+        return status_from_cuda(e);
+      }
+    }
+    scratch = g_noalloc_address[dev];
+  }
+  return status_from_cuda(launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out, scratch, sp,
+                                        static_cast<cudaStream_t>(stream)));
+}
