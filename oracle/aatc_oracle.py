@@ -20,11 +20,12 @@ PCA equivalence (Appendix, Proposition), the quantizer error bound
 (Def. uniform-quant), library SDPA for decode, hand-computed small cases and
 the compression ratio the paper prints (Sec. 6.1).
 
-parity unpinned: the packed record bit layout (:func:`pack_records`,
-:func:`cache_records`) is defined by this build, not by the paper, which prints
-no worked encoding.  It is pinned only by the round trip unpack(pack(c)) == c,
-the record-size identity (352 code bits per token and stream at 2.75 bits,
-i.e. the paper's 16/2.75 = 5.82x) and a hand-computed packed word.
+parity unpinned: the packed record bit layout (:func:`record_entries`,
+:func:`pack_records`, :func:`cache_records`) is defined by this build, not by the
+paper, which prints no worked encoding.  It is pinned only by the round trip
+unpack(pack(c)) == c, the record-size identity (352 code bits per token and stream
+at 2.75 bits, i.e. the paper's 16/2.75 = 5.82x, in exactly 11 words) and
+hand-computed packed words.
 """
 from __future__ import annotations
 
@@ -242,56 +243,90 @@ def dequantize_f32(codes: np.ndarray, alpha_f32: np.ndarray, scales_f32: np.ndar
 
 # ----------------------------------------------------------------------------
 # Packed layout (build-defined; the paper prints none)
+#
+# Each stored code is u = code + 2^(b-1) (offset binary, b bits).  The record of one token
+# and stream splits u into base-4 digits and single top bits, grouped by significance:
+#   D2 = for k = 0..3: digit k (bits 2k, 2k+1) of every channel with b >= 2k+2
+#   D1 = the top bit (bit b-1) of every odd-width channel, in channel order
+# Channels are in storage order (widths non-increasing), so each D2 layer is a prefix.  If |D2| is not a multiple of 16, its last |D2| mod 16
+# entries move to the end of D1 as two single bits each.  Record words: the D2 entries at
+# 16 per word (entry i at bits 2(i mod 16)), then the D1 entries at 32 per word (entry j at
+# bit j mod 32), then zero words up to W.
 # ----------------------------------------------------------------------------
 
+def record_entries(bits: np.ndarray):
+    """(D2, D1): lists of (channel, bit shift) entries of one stream's record."""
+    b = [int(x) for x in bits]
+    d2 = []
+    for k in range(4):
+        d2 += [(c, 2 * k) for c in range(len(b)) if b[c] >= 2 * k + 2]
+    d1 = [(c, b[c] - 1) for c in range(len(b)) if b[c] % 2 == 1]
+    r = len(d2) % 16
+    if r:
+        moved = d2[len(d2) - r:]
+        d2 = d2[:len(d2) - r]
+        for (c, sh) in moved:
+            d1 += [(c, sh), (c, sh + 1)]
+    return d2, d1
+
+
+def stream_words(bits: np.ndarray) -> int:
+    d2, d1 = record_entries(bits)
+    return len(d2) // 16 + (len(d1) + 31) // 32
+
+
 def record_words(bits_per_stream) -> int:
-    """Words per record: W = ceil(max over streams of sum_c b_c / 32), at least 1."""
-    mx = max(int(np.sum(b)) for b in bits_per_stream)
-    return max(1, (mx + 31) // 32)
+    """Words per record: W = max over streams, at least 1."""
+    return max(1, max(stream_words(b) for b in bits_per_stream))
 
 
 def pack_records(codes: np.ndarray, bits: np.ndarray, n_words: int) -> np.ndarray:
-    """Offset-binary fields u_c = code_c + 2^(b_c - 1), LSB-first, in storage channel order,
-    allowed to straddle 32-bit words; unused bits zero.  Returns (n, n_words) uint32."""
+    """codes (n, 128) signed -> (n, n_words) uint32 records (token-major, before any interleave)."""
     b = np.asarray(bits, np.int64)
-    n = codes.shape[0]
-    acc = np.zeros((n, n_words + 1), dtype=np.uint64)
-    off = 0
-    for c in range(len(b)):
-        if b[c] == 0:
-            continue
-        u = (codes[:, c] + (1 << (b[c] - 1))).astype(np.uint64)
-        assert np.all(u < (1 << b[c]))
-        w, sh = off // 32, off % 32
-        acc[:, w] |= (u << np.uint64(sh)) & np.uint64(0xFFFFFFFF)
-        if sh + b[c] > 32:
-            acc[:, w + 1] |= u >> np.uint64(32 - sh)
-        off += int(b[c])
-    assert off <= 32 * n_words
-    return acc[:, :n_words].astype(np.uint32)
+    u = np.where(b[None, :] > 0, codes + np.where(b > 0, 2 ** np.maximum(b - 1, 0), 0)[None, :], 0).astype(np.uint64)
+    assert np.all(u < np.where(b > 0, 2 ** b, 1)[None, :])
+    d2, d1 = record_entries(b)
+    words = np.zeros((codes.shape[0], n_words), dtype=np.uint64)
+    for i, (c, sh) in enumerate(d2):
+        words[:, i // 16] |= ((u[:, c] >> np.uint64(sh)) & np.uint64(3)) << np.uint64(2 * (i % 16))
+    base = len(d2) // 16
+    for j, (c, sh) in enumerate(d1):
+        words[:, base + j // 32] |= ((u[:, c] >> np.uint64(sh)) & np.uint64(1)) << np.uint64(j % 32)
+    assert base + (len(d1) + 31) // 32 <= n_words
+    return words.astype(np.uint32)
 
 
 def unpack_records(words: np.ndarray, bits: np.ndarray) -> np.ndarray:
     """Inverse of :func:`pack_records`: (n, W) uint32 -> (n, 128) signed codes."""
     b = np.asarray(bits, np.int64)
     w64 = np.asarray(words).astype(np.uint64)
-    w64 = np.concatenate([w64, np.zeros((w64.shape[0], 1), np.uint64)], axis=1)
-    codes = np.zeros((w64.shape[0], len(b)), dtype=np.int64)
-    off = 0
-    for c in range(len(b)):
-        if b[c] == 0:
-            continue
-        w, sh = off // 32, off % 32
-        both = w64[:, w] | (w64[:, w + 1] << np.uint64(32))
-        u = (both >> np.uint64(sh)) & np.uint64((1 << b[c]) - 1)
-        codes[:, c] = u.astype(np.int64) - (1 << (b[c] - 1))
-        off += int(b[c])
-    return codes
+    u = np.zeros((w64.shape[0], len(b)), dtype=np.uint64)
+    d2, d1 = record_entries(b)
+    for i, (c, sh) in enumerate(d2):
+        u[:, c] |= ((w64[:, i // 16] >> np.uint64(2 * (i % 16))) & np.uint64(3)) << np.uint64(sh)
+    base = len(d2) // 16
+    for j, (c, sh) in enumerate(d1):
+        u[:, c] |= ((w64[:, base + j // 32] >> np.uint64(j % 32)) & np.uint64(1)) << np.uint64(sh)
+    off = np.where(b > 0, 2 ** np.maximum(b - 1, 0), 0)
+    return np.where(b[None, :] > 0, u.astype(np.int64) - off[None, :], 0)
+
+
+def value_lane_of(token_in_tile: int) -> tuple:
+    """Values are stored pair-interleaved.  In each 16-token group, tokens i and i+8 form a
+    pair; the pair's two records are stored as two words per record word: (low halves of
+    both) and (high halves of both), the first token's half in the low 16 bits.  Returns
+    (lane holding this token's low halves, lane holding its high halves, half index 0/1)."""
+    g, j = divmod(token_in_tile, 16)
+    i, second = j % 8, j >= 8
+    q, r = i % 4, i // 4                 # pairs i and i+4 share a 4-lane block
+    base = 16 * g + 4 * q + 2 * r
+    return base, base + 1, int(second)
 
 
 def cache_geometry(batch: int, n_kv_heads: int, max_tokens: int, n_words: int) -> dict:
     """Per-layer packed cache: uint32 words [batch][H_kv][2][n_tiles][W][128], then fp32 alpha
-    [batch][H_kv][2][n_tiles*128].  Token t of a sequence sits in tile t // 128, lane t % 128."""
+    [batch][H_kv][2][n_tiles*128].  Keys: token t of a sequence sits in tile t // 128, lane
+    t % 128.  Values: lanes as :func:`value_lane_of` says."""
     n_tiles = (max_tokens + TILE - 1) // TILE
     n_word_elems = batch * n_kv_heads * 2 * n_tiles * n_words * TILE
     n_alpha = batch * n_kv_heads * 2 * n_tiles * TILE
@@ -308,8 +343,42 @@ def cache_records(cache_u32: np.ndarray, batch: int, n_kv_heads: int, max_tokens
     alpha = np.asarray(cache_u32[geo["words"]: geo["words"] + geo["alpha"]]).view(np.float32)
     alpha = alpha.reshape(batch, n_kv_heads, 2, nt * TILE)
     t = np.arange(t0, t0 + n)
-    rec = words[b, head, kind][t // TILE, :, t % TILE]        # (n, W)
+    if kind == 0:
+        rec = words[b, head, kind][t // TILE, :, t % TILE]        # (n, W)
+    else:
+        lanes = np.array([value_lane_of(int(x)) for x in t % TILE])
+        lo = words[b, head, kind][t // TILE, :, lanes[:, 0]].astype(np.uint64)
+        hi = words[b, head, kind][t // TILE, :, lanes[:, 1]].astype(np.uint64)
+        sel = lanes[:, 2][:, None].astype(np.uint64) * np.uint64(16)
+        m16 = np.uint64(0xFFFF)
+        rec = (((lo >> sel) & m16) | (((hi >> sel) & m16) << np.uint64(16))).astype(np.uint32)
     return rec, alpha[b, head, kind, t0:t0 + n]
+
+
+def cache_image(records_k, records_v, alpha_k, alpha_v, batch, n_kv_heads, max_tokens, n_words):
+    """Build a whole-layer cache image (uint32) from per-stream records (for tests): records_x
+    [batch][H_kv] -> (max_tokens, W) uint32 arrays; alpha_x [batch][H_kv] -> (max_tokens,)."""
+    geo = cache_geometry(batch, n_kv_heads, max_tokens, n_words)
+    nt = geo["n_tiles"]
+    words = np.zeros((batch, n_kv_heads, 2, nt, n_words, TILE), np.uint32)
+    alpha = np.zeros((batch, n_kv_heads, 2, nt * TILE), np.float32)
+    for b in range(batch):
+        for h in range(n_kv_heads):
+            rk = records_k[b][h]
+            for t in range(rk.shape[0]):
+                words[b, h, 0, t // TILE, :, t % TILE] = rk[t]
+            rv = records_v[b][h]
+            for t in range(rv.shape[0]):
+                lo, hi, half = value_lane_of(t % TILE)
+                for w in range(n_words):
+                    x = int(rv[t, w])
+                    for lane, part in ((lo, x & 0xFFFF), (hi, x >> 16)):
+                        cur = int(words[b, h, 1, t // TILE, w, lane])
+                        cur &= ~(0xFFFF << (16 * half)) & 0xFFFFFFFF
+                        words[b, h, 1, t // TILE, w, lane] = cur | (part << (16 * half))
+            alpha[b, h, 0, :rk.shape[0]] = alpha_k[b][h]
+            alpha[b, h, 1, :rv.shape[0]] = alpha_v[b][h]
+    return np.concatenate([words.reshape(-1), alpha.reshape(-1).view(np.uint32)])
 
 
 # ----------------------------------------------------------------------------

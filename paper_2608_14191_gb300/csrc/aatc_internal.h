@@ -23,28 +23,40 @@ constexpr int MAX_GROUP = 8;        // query heads per kv-head supported by the 
 constexpr uint32_t PLAN_MAGIC = 0xAA7C0DE1u;
 constexpr uint32_t PLAN_DEAD = 0xDEADDEADu;
 
-// Packing schedule word of one channel (encode epilogue): bit offset inside its first word,
-// whether the field completes that word, and the width.
-AATC_HD constexpr int sched_shift(int s) { return s & 31; }
-AATC_HD constexpr bool sched_flush(int s) { return (s >> 8) & 1; }
-AATC_HD constexpr int sched_bits(int s) { return (s >> 16) & 15; }
-
-struct ChanEnc {          // per-channel encode constants (one 16-byte load)
+// Per-channel encode constants (one 16-byte load in the encode epilogue).
+struct ChanEnc {
   float inv_f;            // 1 / f_c, f_c = s_c 2^(1-b_c); 0 for dropped channels
-  float lo;               // -2^(b_c-1) as float (0 for dropped)
-  float hi;               // 2^(b_c-1) - 1 as float (0 for dropped)
-  float magic;            // 1.5 * 2^23 + 2^(b_c-1): floor to offset-binary u via round-down add
+  float hi;               // 2^(b_c-1) - 1 as float: upper clamp of h/Delta + 1/2 (0 for dropped)
+  float magic;            // 1.5 * 2^23 + 2^(b_c-1): round-down add leaves u = code + 2^(b-1) in the mantissa
+  float off;              // 2^(b_c-1) (offset of the stored code), 0 for dropped
+};
+
+// Record layout of one stream.  The stored value u = code + 2^(b-1) of every retained channel
+// is split into base-4 digits and single top bits:
+//   D2: for k = 0..3, digit k (bits 2k, 2k+1) of channels 0..l2[k]-1  (16 two-bit fields/word)
+//   D1: the top bit of every odd-width channel (channel order), then the digits that did not
+//       fill the last D2 word, each as two single bits (32 one-bit fields/word)
+// Record words: n2/16 D2 words, then ceil(n1/32) D1 words, then zeros up to the plan's W.
+// `entry[e]` (int16, per stream) lists the D2 entries then the D1 entries as
+// (channel | bit shift << 8); padding entries are -1.
+struct StreamLayout {
+  int n2;                 // D2 entries (a multiple of 16)
+  int n1;                 // D1 entries
+  int words;              // record words this stream uses
+  int nret;               // retained channels R
+  int l2[4];              // D2 digit-layer lengths
 };
 
 struct PlanDevice {
   const void* ubf16_t;    // bf16 [S][128 channel][128 dim]   encode basis (MMA B operand, K-major)
-  const float* u32;       // fp32 [S][128 dim][128 channel]   decode query rotation / value inverse
+  const float* u32;       // fp32 [S][128 dim][128 channel]   decode query rotation
+  const float* u32t;      // fp32 [S][128 channel][128 dim]   decode inverse value transform
   const ChanEnc* enc;     // [S][128]
-  const int* sched;       // [S][128]
   const float* inv_s;     // [S][128] 1/s_c (0 for dropped)
   const float* f;         // [S][128] f_c (0 for dropped)
-  const int* ext;         // [S][128] decode extraction word: (offset in record) | (b << 16)
-  const int* nret;        // [S] retained channels R
+  const StreamLayout* lay;  // [S]
+  const short* entry;     // [S][n_entries]
+  const short* chan_ent;  // [S][128][8]: entries of each channel (-1 padded)
   int* err;               // [4] sticky device flags
 };
 
@@ -53,10 +65,12 @@ struct Plan {
   aatc_dims_t dims{};
   int n_streams = 0;
   int n_words = 0;        // W, words per record (plan-wide)
+  int n_entries = 0;      // entries per stream in `entry` (32 * W)
   int num_sms = 0;
   int device = 0;
   std::vector<int> retained;
   std::vector<int> nbits;
+  std::vector<StreamLayout> layout;
   PlanDevice dev{};
   void* block = nullptr;  // single device allocation holding every table
   size_t block_bytes = 0;
@@ -92,7 +106,8 @@ struct DecodeSplit {
 };
 
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
-size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp);
+// Split partials: per (sequence, query head, split) n_entries value sums, then m, l, S'.
+size_t decode_workspace(int batch, int n_q, int n_entries, const DecodeSplit& sp);
 
 // Handle check and CUDA-status mapping shared by every C entry point (defined in capi.cpp).
 Plan* plan_from_handle(aatc_plan_t p);

@@ -57,8 +57,42 @@ Plan* plan_from_handle(aatc_plan_t p) { return as_plan(p); }
 
 aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
 
-size_t decode_workspace(int batch, int n_q, const DecodeSplit& sp) {
-  return static_cast<size_t>(batch) * n_q * sp.n_splits * (D + 2) * sizeof(float);
+size_t decode_workspace(int batch, int n_q, int n_entries, const DecodeSplit& sp) {
+  return static_cast<size_t>(batch) * n_q * sp.n_splits * (n_entries + 3) * sizeof(float);
+}
+
+// D2 / D1 record layout of one stream from its (non-increasing) widths; see StreamLayout.
+void build_layout(const uint8_t* bits, StreamLayout* lay, std::vector<short>& entries) {
+  std::vector<short> d2, d1;
+  auto ent = [](int c, int sh) { return static_cast<short>(c | (sh << 8)); };
+  for (int k = 0; k < 4; ++k) {
+    int n = 0;
+    for (int c = 0; c < D; ++c)
+      if (bits[c] >= 2 * k + 2) {
+        d2.push_back(ent(c, 2 * k));
+        ++n;
+      }
+    lay->l2[k] = n;
+  }
+  for (int c = 0; c < D; ++c)
+    if (bits[c] & 1) d1.push_back(ent(c, bits[c] - 1));
+  const int r = static_cast<int>(d2.size()) % 16;
+  for (int i = static_cast<int>(d2.size()) - r; i < static_cast<int>(d2.size()); ++i) {
+    const int c = d2[i] & 0xFF, sh = d2[i] >> 8;
+    d1.push_back(ent(c, sh));
+    d1.push_back(ent(c, sh + 1));
+  }
+  d2.resize(d2.size() - r);
+  for (int k = 3, left = r; k >= 0 && left > 0; --k) {      // the moved digits came off the last layers
+    const int take = std::min(left, lay->l2[k]);
+    lay->l2[k] -= take;
+    left -= take;
+  }
+  lay->n2 = static_cast<int>(d2.size());
+  lay->n1 = static_cast<int>(d1.size());
+  lay->words = lay->n2 / 16 + (lay->n1 + 31) / 32;
+  entries = d2;
+  entries.insert(entries.end(), d1.begin(), d1.end());
 }
 
 }  // namespace aatc
@@ -110,19 +144,27 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   }
   for (size_t i = 0; i < SD * D; ++i)
     if (!std::isfinite(basis[i])) return AATC_ERR_INVALID_ARG;
-  const int max_nb = *std::max_element(nbits.begin(), nbits.end());
-  const int W = std::max(1, (max_nb + 31) / 32);
+  std::vector<StreamLayout> layout(S);
+  std::vector<std::vector<short>> entries(S);
+  int W = 1;
+  for (int s = 0; s < S; ++s) {
+    build_layout(bits + static_cast<size_t>(s) * D, &layout[s], entries[s]);
+    layout[s].nret = retained[s];
+    W = std::max(W, layout[s].words);
+  }
+  const int E = 32 * W;                                             // entries per stream (padded)
 
   // host staging of every table, in one block
   size_t off = 0;
   const size_t o_ubf = off;  off = align_up(off + SD * D * 2, 256);
   const size_t o_u32 = off;  off = align_up(off + SD * D * 4, 256);
+  const size_t o_u32t = off; off = align_up(off + SD * D * 4, 256);
   const size_t o_enc = off;  off = align_up(off + SD * sizeof(ChanEnc), 256);
-  const size_t o_sch = off;  off = align_up(off + SD * 4, 256);
   const size_t o_invs = off; off = align_up(off + SD * 4, 256);
   const size_t o_f = off;    off = align_up(off + SD * 4, 256);
-  const size_t o_ext = off;  off = align_up(off + SD * 4, 256);
-  const size_t o_nret = off; off = align_up(off + static_cast<size_t>(S) * 4, 256);
+  const size_t o_lay = off;  off = align_up(off + static_cast<size_t>(S) * sizeof(StreamLayout), 256);
+  const size_t o_ent = off;  off = align_up(off + static_cast<size_t>(S) * E * sizeof(short), 256);
+  const size_t o_che = off;  off = align_up(off + SD * 8 * sizeof(short), 256);
   const size_t o_err = off;  off = align_up(off + 16, 256);
   const size_t total = off;
   std::vector<unsigned char> host;
@@ -133,41 +175,46 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   }
   auto* ubf = reinterpret_cast<uint16_t*>(host.data() + o_ubf);
   auto* u32 = reinterpret_cast<float*>(host.data() + o_u32);
+  auto* u32t = reinterpret_cast<float*>(host.data() + o_u32t);
   auto* enc = reinterpret_cast<ChanEnc*>(host.data() + o_enc);
-  auto* sch = reinterpret_cast<int*>(host.data() + o_sch);
   auto* invs = reinterpret_cast<float*>(host.data() + o_invs);
   auto* fc = reinterpret_cast<float*>(host.data() + o_f);
-  auto* ext = reinterpret_cast<int*>(host.data() + o_ext);
-  auto* nret = reinterpret_cast<int*>(host.data() + o_nret);
+  auto* lay = reinterpret_cast<StreamLayout*>(host.data() + o_lay);
+  auto* ent = reinterpret_cast<short*>(host.data() + o_ent);
+  auto* che = reinterpret_cast<short*>(host.data() + o_che);
   for (int s = 0; s < S; ++s) {
     const float* bs = basis + static_cast<size_t>(s) * D * D;     // [dim][channel]
     for (int d = 0; d < D; ++d)
       for (int c = 0; c < D; ++c) {
         ubf[(static_cast<size_t>(s) * D + c) * D + d] = f32_to_bf16_rne(bs[d * D + c]);
         u32[(static_cast<size_t>(s) * D + d) * D + c] = bs[d * D + c];
+        u32t[(static_cast<size_t>(s) * D + c) * D + d] = bs[d * D + c];
       }
-    int o = 0;
     for (int c = 0; c < D; ++c) {
       const size_t i = static_cast<size_t>(s) * D + c;
       const int b = bits[i];
-      ChanEnc e{0.0f, 0.0f, 0.0f, 12582912.0f};
+      ChanEnc e{0.0f, 0.0f, 12582912.0f, 0.0f};
       if (b > 0) {
         const float f = std::ldexp(scales[i], 1 - b);            // exact power-of-two scaling
         e.inv_f = 1.0f / f;
-        e.lo = -std::ldexp(1.0f, b - 1);
         e.hi = std::ldexp(1.0f, b - 1) - 1.0f;
         e.magic = 12582912.0f + std::ldexp(1.0f, b - 1);
+        e.off = std::ldexp(1.0f, b - 1);
         fc[i] = f;
         invs[i] = 1.0f / scales[i];
       }
       enc[i] = e;
-      const int sh = o & 31;
-      const int flush = (b > 0 && sh + b >= 32) ? 1 : 0;
-      sch[i] = sh | (flush << 8) | (b << 16);
-      ext[i] = o | (b << 16);
-      o += b;
     }
-    nret[s] = retained[s];
+    lay[s] = layout[s];
+    for (int e = 0; e < E; ++e)
+      ent[static_cast<size_t>(s) * E + e] = e < static_cast<int>(entries[s].size()) ? entries[s][e] : short(-1);
+    short* ce = che + static_cast<size_t>(s) * D * 8;
+    for (int i = 0; i < D * 8; ++i) ce[i] = -1;
+    int fill[D] = {0};
+    for (int e = 0; e < static_cast<int>(entries[s].size()); ++e) {
+      const int c = entries[s][e] & 0xFF;
+      if (fill[c] < 8) ce[c * 8 + fill[c]++] = static_cast<short>(e);
+    }
   }
 
   auto* plan = new (std::nothrow) Plan();
@@ -175,8 +222,10 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   plan->dims = *dims;
   plan->n_streams = S;
   plan->n_words = W;
+  plan->n_entries = E;
   plan->retained = retained;
   plan->nbits = nbits;
+  plan->layout = layout;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaGetDevice(&plan->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&plan->num_sms, cudaDevAttrMultiProcessorCount, plan->device);
@@ -191,12 +240,13 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   auto* base = static_cast<unsigned char*>(plan->block);
   plan->dev.ubf16_t = base + o_ubf;
   plan->dev.u32 = reinterpret_cast<const float*>(base + o_u32);
+  plan->dev.u32t = reinterpret_cast<const float*>(base + o_u32t);
   plan->dev.enc = reinterpret_cast<const ChanEnc*>(base + o_enc);
-  plan->dev.sched = reinterpret_cast<const int*>(base + o_sch);
   plan->dev.inv_s = reinterpret_cast<const float*>(base + o_invs);
   plan->dev.f = reinterpret_cast<const float*>(base + o_f);
-  plan->dev.ext = reinterpret_cast<const int*>(base + o_ext);
-  plan->dev.nret = reinterpret_cast<const int*>(base + o_nret);
+  plan->dev.lay = reinterpret_cast<const StreamLayout*>(base + o_lay);
+  plan->dev.entry = reinterpret_cast<const short*>(base + o_ent);
+  plan->dev.chan_ent = reinterpret_cast<const short*>(base + o_che);
   plan->dev.err = reinterpret_cast<int*>(base + o_err);
   if (e == cudaSuccess) e = encode_tensor_maps_u(*plan);
   if (e != cudaSuccess) {
@@ -254,7 +304,7 @@ aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t 
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
   const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, sp);
+  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp);
   return AATC_OK;
 }
 
@@ -269,7 +319,8 @@ aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q,
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if (!aligned16(cache) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
   const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, sp)) return AATC_ERR_WORKSPACE;
+  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp))
+    return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
                                          workspace, sp, static_cast<cudaStream_t>(stream)));
 }
@@ -306,7 +357,7 @@ aatc_status_t aatc_bf16_decode_workspace_bytes(int32_t batch, int32_t n_kv, int3
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     sms = 1;
-  *bytes = aatc::decode_workspace(batch, n_q, aatc::decode_split(batch, n_kv, n_ctx, sms));
+  *bytes = aatc::decode_workspace(batch, n_q, aatc::D, aatc::decode_split(batch, n_kv, n_ctx, sms));
   return AATC_OK;
 }
 
@@ -325,7 +376,7 @@ aatc_status_t aatc_bf16_decode_attention(const void* K, const void* V, const voi
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return cuda_status(e);
   const auto sp = aatc::decode_split(batch, n_kv, n_ctx, sms);
-  if (workspace_bytes < aatc::decode_workspace(batch, n_q, sp)) return AATC_ERR_WORKSPACE;
+  if (workspace_bytes < aatc::decode_workspace(batch, n_q, aatc::D, sp)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_bf16_decode(K, V, q, batch, n_ctx, max_tokens, n_kv, n_q, out,
                                               workspace, sp, static_cast<cudaStream_t>(stream)));
 }

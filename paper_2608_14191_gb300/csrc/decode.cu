@@ -57,329 +57,443 @@ __device__ __forceinline__ void block_reduce(float (&v)[GP], float* scratch /* [
   __syncthreads();
 }
 
+// ---------------------------------------------------------------- packed-cache decode
+//
+// Tensor-core formulation (mma.sync m16n8k16, fp16 operands, fp32 accumulate):
+//   scores:  A = folded query q'_c 2^shift per record entry, split hi (rows g) / lo (rows g+8),
+//            B = record digits / bits of 8 tokens (each fragment register: one shift + mask of a
+//            packed word, then subtracting the 1024 magic), accumulated over the record words.
+//   values:  A = probabilities P' = p alpha^V split hi / lo, B = value digits / bits of 16 tokens
+//            from the pair-interleaved value words, one n-tile per 8 record entries.
+// Token order inside a 16-token group g16 (both products): k = 2i <-> token i, k = 2i+1 <->
+// token i+8 for i < 8.  Score n-tile A holds k 0..7, n-tile B k 8..15.
+
 struct DecodeArgs {
   const uint32_t* words;   // cache word region (this layer)
   const float* alpha;      // cache alpha region
   const __nv_bfloat16* q;  // [batch][HQ][128]
-  float* ws;               // [batch][HQ][n_splits][130]
+  float* ws;               // [batch][HQ][n_splits][n_entries + 3]
+  float* out;              // [batch][HQ][128]
   const float* u32;        // plan: [S][128 dim][128 ch]
+  const float* u32t;       // plan: [S][128 ch][128 dim]
   const float* f;          // plan: [S][128]
-  const int* ext;          // plan: [S][128]
-  const int* nret;         // plan: [S]
-  int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_splits, split_len;
+  const ChanEnc* enc;      // plan: [S][128] (offsets 2^(b-1))
+  const StreamLayout* lay; // plan: [S]
+  const short* entry;      // plan: [S][n_entries]
+  const short* chan_ent;   // plan: [S][128][8]
+  int* err;
+  int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len;
 };
 
-// Shared-memory plan of the split kernel (floats unless noted).
-template <int GP>
-struct SplitSmem {
-  static constexpr int kQt = 0;                                 // [128][GP] folded query
-  static constexpr int kQf = kQt + D * GP;                      // [GP][128] query (fp32)
-  static constexpr int kCg = kQf + GP * D;                      // [GP] offset corrections
-  static constexpr int kRed = kCg + 8;                          // [4][8] reductions
-  static constexpr int kExtK = kRed + 32;                       // int [128] (offset | b << 16)
-  static constexpr int kAlpha = kExtK + D;                      // [2][128] alpha of the staged tile
-  static constexpr int kScores = kAlpha + 2 * TILE;             // [split_len][GP]
-  // followed by the word tiles: [2][(W + 2) * 132] u32, then acc scratch [4][GP][128]
+__device__ __forceinline__ uint32_t hsub_magic(uint32_t x) {
+  // x holds two 16-bit fields (1024 + v) as fp16 bit patterns; returns the fp16 pair (v_lo, v_hi)
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__device__ __forceinline__ void mma_16816(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
+}
+
+// fp32 -> (hi, lo) fp16 pair with hi + lo = v to ~2^-22 relative
+__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
+  hi = __half2float(__float2half_rn(v));
+  lo = v - hi;
+}
+
+constexpr int kGroups = TILE / 16;        // 16-token groups per tile
+constexpr int kWarps = kThreads / 32;
+
+// shared-memory carve-up of the split kernel (32-bit words)
+struct SplitLayout {
+  int qc, cg, afrag, stile, pfrag, corr, red, kw, vw, ak, av, n_words_total;
+  __host__ __device__ SplitLayout(int n_ks, int W) {
+    int o = 0;
+    qc = o;    o += MAX_GROUP * D;             // folded query per channel
+    cg = o;    o += MAX_GROUP;                 // offset corrections
+    red = o;   o += 4 * MAX_GROUP * 2;         // reductions
+    corr = o;  o += 4 * MAX_GROUP;             // corr, m, l, S' of the running softmax
+    o = (o + 3) & ~3;
+    afrag = o; o += n_ks * 32 * 4;             // uint4 per (k-step, lane)
+    stile = o; o += MAX_GROUP * TILE;          // scores of the current tile
+    pfrag = o; o += kGroups * MAX_GROUP * 16;  // half2 (hi, lo) of P' per (group, query, slot)
+    kw = o;    o += 2 * W * TILE;              // two stages of key words
+    vw = o;    o += 2 * W * TILE;              // two stages of value words
+    ak = o;    o += 2 * TILE;
+    av = o;    o += 2 * TILE;
+    n_words_total = o;
+  }
 };
 
-template <int GP>
+template <int NTW>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
-  extern __shared__ __align__(16) float sm[];
+  extern __shared__ __align__(16) uint32_t smw[];
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t = lane & 3;                       // mma fragment coordinates
   const int G = a.group;
-  const int sk = (a.layer * a.n_kv + head) * 2;                 // key stream; value = sk + 1
-  const int RK = a.nret[sk], RV = a.nret[sk + 1];
-  using L = SplitSmem<GP>;
-  float* qt = sm + L::kQt;
-  float* qf = sm + L::kQf;
-  float* cg = sm + L::kCg;
-  float* red = sm + L::kRed;
-  int* extk = reinterpret_cast<int*>(sm + L::kExtK);
-  float* al = sm + L::kAlpha;
-  float* sc = sm + L::kScores;
-  const int stride = 132;                                       // padded word-plane stride (u32)
-  uint32_t* wt = reinterpret_cast<uint32_t*>(sc + a.split_len * GP);   // [2][(W+2)*132]
-  const int wt_elems = (a.n_words + 2) * stride;
-  float* accs = reinterpret_cast<float*>(wt + 2 * wt_elems);    // [4][GP][128]
+  const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;   // key / value streams
+  const StreamLayout lk = a.lay[sk], lv = a.lay[sv];
+  const int W = a.n_words;
+  const int n2w_k = lk.n2 / 16, n1w_k = (lk.n1 + 31) / 32;
+  const int n_ks = n2w_k + 2 * n1w_k;
+  const int n2w_v = lv.n2 / 16, n1w_v = (lv.n1 + 31) / 32;
+  const int n_nt = 2 * n2w_v + 4 * n1w_v;
+  const SplitLayout L(n_ks, W);
+  float* qc = reinterpret_cast<float*>(smw + L.qc);
+  float* cg = reinterpret_cast<float*>(smw + L.cg);
+  float* red = reinterpret_cast<float*>(smw + L.red);
+  float* run = reinterpret_cast<float*>(smw + L.corr);         // [0..7] corr, [8..15] m, [16..23] l, [24..31] S'
+  uint4* afrag = reinterpret_cast<uint4*>(smw + L.afrag);
+  float* stile = reinterpret_cast<float*>(smw + L.stile);
+  uint32_t* pfrag = smw + L.pfrag;
+  uint32_t* kw = smw + L.kw;
+  uint32_t* vw = smw + L.vw;
+  float* ak = reinterpret_cast<float*>(smw + L.ak);
+  float* av = reinterpret_cast<float*>(smw + L.av);
 
   const int t_begin = split * a.split_len;
   const int t_end = min(a.n_ctx, t_begin + a.split_len);
   const int n_tiles_split = (t_end - t_begin + TILE - 1) / TILE;
-  const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-  const size_t bk = (static_cast<size_t>(b) * a.n_kv + head) * 2;   // cache stream index of K
+  const int tile0 = t_begin / TILE;
+  const size_t stream_words = static_cast<size_t>(a.n_tiles) * W * TILE;
+  const size_t bk = (static_cast<size_t>(b) * a.n_kv + head) * 2;   // cache stream of the keys
   const uint32_t* kwords = a.words + bk * stream_words;
   const uint32_t* vwords = a.words + (bk + 1) * stream_words;
   const float* kalpha = a.alpha + bk * a.n_tiles * TILE;
   const float* valpha = a.alpha + (bk + 1) * a.n_tiles * TILE;
 
-  // ---- prologue: folded query q'_{g,c} = (U_K^T q_g)_c f_c log2e / sqrt(128)
-  for (int i = tid; i < GP * D; i += kThreads) {
-    const int g = i / D, d = i % D;
-    qf[i] = g < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + g) * D + d]) : 0.0f;
-  }
-  extk[tid] = a.ext[sk * D + tid];
-  __syncthreads();
+  auto stage = [&](int tile, int buf) {
+    const int chunks = W * (TILE / 4);
+    const uint32_t* sk_ = kwords + static_cast<size_t>(tile) * W * TILE;
+    const uint32_t* sv_ = vwords + static_cast<size_t>(tile) * W * TILE;
+    for (int i = tid; i < chunks; i += kThreads) {
+      cp_async16(kw + buf * W * TILE + 4 * i, sk_ + 4 * i);
+      cp_async16(vw + buf * W * TILE + 4 * i, sv_ + 4 * i);
+    }
+    if (tid < TILE / 4) cp_async16(ak + buf * TILE + 4 * tid, kalpha + tile * TILE + 4 * tid);
+    else if (tid < TILE / 2) cp_async16(av + buf * TILE + 4 * (tid - TILE / 4), valpha + tile * TILE + 4 * (tid - TILE / 4));
+    cp_async_commit();
+  };
+  stage(tile0, 0);
+
+  // ---- prologue: folded query q'_{g,c} = (U_K^T q_g)_c f_c log2(e) / sqrt(128)
   {
+    float* qf = stile;                                      // scratch: fp32 query [8][128]
+    for (int i = tid; i < MAX_GROUP * D; i += kThreads) {
+      const int gq = i / D, d = i % D;
+      qf[i] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + d]) : 0.0f;
+    }
+    __syncthreads();
     const int c = tid;
-    float accq[GP];
+    float accq[MAX_GROUP];
 #pragma unroll
-    for (int g = 0; g < GP; ++g) accq[g] = 0.0f;
+    for (int gq = 0; gq < MAX_GROUP; ++gq) accq[gq] = 0.0f;
     const float* uk = a.u32 + static_cast<size_t>(sk) * D * D;
     for (int d = 0; d < D; ++d) {
       const float u = uk[d * D + c];
 #pragma unroll
-      for (int g = 0; g < GP; ++g) accq[g] = fmaf(u, qf[g * D + d], accq[g]);
+      for (int gq = 0; gq < MAX_GROUP; ++gq) accq[gq] = fmaf(u, qf[gq * D + d], accq[gq]);
     }
     const float fk = a.f[sk * D + c] * (kLog2e * 0.08838834764831845f);   // 1/sqrt(128)
-    const int bits = extk[c] >> 16;
-    const float off = bits > 0 ? static_cast<float>(1 << (bits - 1)) : 0.0f;
-    float corr[GP];
+    const float off = a.enc[sk * D + c].off;
+    float corr8[MAX_GROUP];
 #pragma unroll
-    for (int g = 0; g < GP; ++g) {
-      const float v = c < RK ? accq[g] * fk : 0.0f;
-      qt[c * GP + g] = v;
-      corr[g] = v * off;
+    for (int gq = 0; gq < MAX_GROUP; ++gq) {
+      const float v = accq[gq] * fk;
+      qc[gq * D + c] = v;
+      corr8[gq] = v * off;
     }
-    block_reduce<GP, false>(corr, red);
-    if (tid < GP) cg[tid] = corr[tid];
+    block_reduce<MAX_GROUP, false>(corr8, red);
+    if (tid < MAX_GROUP) cg[tid] = corr8[tid];
+    if (tid < MAX_GROUP) {
+      run[tid] = 0.0f;                 // corr
+      run[8 + tid] = -INFINITY;        // m
+      run[16 + tid] = 0.0f;            // l
+      run[24 + tid] = 0.0f;            // S'
+    }
   }
   __syncthreads();
-
-  // ---- phase 1: scores, thread = token
-  auto stage_tile = [&](const uint32_t* src_words, const float* src_alpha, int tile, int buf) {
-    uint32_t* dst = wt + buf * wt_elems;
-    const uint32_t* src = src_words + static_cast<size_t>(tile) * a.n_words * TILE;
-    const int chunks = a.n_words * (TILE / 4);
-    for (int i = tid; i < chunks; i += kThreads) {
-      const int w = i / (TILE / 4), q4 = i % (TILE / 4);
-      cp_async16(dst + w * stride + q4 * 4, src + w * TILE + q4 * 4);
-    }
-    if (tid < TILE / 4) cp_async16(al + buf * TILE + tid * 4, src_alpha + tile * TILE + tid * 4);
-    cp_async_commit();
-  };
-  // zero the two guard planes once (read past the record by the sliding window)
-  for (int i = tid; i < 2 * stride; i += kThreads) {
-    wt[a.n_words * stride + i] = 0u;
-    wt[wt_elems + a.n_words * stride + i] = 0u;
-  }
-  const int tile0 = t_begin / TILE;
-  stage_tile(kwords, kalpha, tile0, 0);
-  float mloc[GP];
+  // score A fragments: slot k of k-step ks -> record entry -> coefficient q'_c 2^shift
+  {
+    const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
+    for (int i = tid; i < n_ks * 32; i += kThreads) {
+      const int ks = i >> 5, ln = i & 31, gq = ln >> 2, tq = ln & 3;
+      int fld[4];                                   // fields for k = 2t, 2t+1, 2t+8, 2t+9
+      int ebase;
+      if (ks < n2w_k) {
+        ebase = 16 * ks;
+        fld[0] = tq; fld[1] = tq + 8; fld[2] = tq + 4; fld[3] = tq + 12;
+      } else {
+        const int r = ks - n2w_k, h8 = 8 * (r & 1);
+        ebase = lk.n2 + 32 * (r >> 1);
+        fld[0] = tq + h8; fld[1] = tq + 16 + h8; fld[2] = tq + 4 + h8; fld[3] = tq + 20 + h8;
+      }
+      float hi[4], lo[4];
 #pragma unroll
-  for (int g = 0; g < GP; ++g) mloc[g] = -INFINITY;
+      for (int j = 0; j < 4; ++j) {
+        const int e = ebase + fld[j];
+        const int ce = (e < lk.n2 + lk.n1) ? ent[e] : -1;
+        const float coef = (ce >= 0 && gq < G) ? ldexpf(qc[gq * D + (ce & 0xFF)], ce >> 8) : 0.0f;
+        split_hi_lo(coef, hi[j], lo[j]);
+      }
+      afrag[i] = make_uint4(pack_half2(hi[0], hi[1]), pack_half2(lo[0], lo[1]), pack_half2(hi[2], hi[3]),
+                            pack_half2(lo[2], lo[3]));
+    }
+  }
+
+  // value n-tiles of this warp and their accumulators (rows g: P' hi part, g+8: lo part)
+  const int j0 = warp * n_nt / kWarps, j1 = (warp + 1) * n_nt / kWarps;
+  float acc[NTW][4];
+#pragma unroll
+  for (int jj = 0; jj < NTW; ++jj)
+#pragma unroll
+    for (int r = 0; r < 4; ++r) acc[jj][r] = 0.0f;
+
   for (int ti = 0; ti < n_tiles_split; ++ti) {
     const int buf = ti & 1;
     cp_async_wait_all();
     __syncthreads();
-    if (ti + 1 < n_tiles_split) stage_tile(kwords, kalpha, tile0 + ti + 1, buf ^ 1);
-    const uint32_t* w = wt + buf * wt_elems;
-    float s[GP];
+    if (ti + 1 < n_tiles_split) stage(tile0 + ti + 1, buf ^ 1);
+    const uint32_t* kt = kw + buf * W * TILE;
+    const uint32_t* vt = vw + buf * W * TILE;
+    const int tbase = (tile0 + ti) * TILE;
+
+    // ---- phase S: warp handles groups 2 warp, 2 warp + 1 (4 score n-tiles of 8 tokens)
+    {
+      float sc[4][4];
+      int tok[4];
 #pragma unroll
-    for (int g = 0; g < GP; ++g) s[g] = 0.0f;
-    uint32_t lo = w[tid], hi = w[stride + tid];
-    int cw = 0;
-    for (int c = 0; c < RK; ++c) {
-      const int e = extk[c];
-      const int o = e & 0xFFFF;
-      const int nb = e >> 16;
-      if ((o >> 5) != cw) {                     // uniform: advance the two-word window
-        cw = o >> 5;
-        lo = hi;
-        hi = w[(cw + 1) * stride + tid];
+      for (int n = 0; n < 4; ++n) {
+        const int g16 = 2 * warp + (n >> 1);
+        const int half8 = n & 1;                               // n-tile A (0) or B (1)
+        tok[n] = 16 * g16 + (g & 1 ? 8 : 0) + (g >> 1) + 4 * half8;   // token of column n = g
+#pragma unroll
+        for (int r = 0; r < 4; ++r) sc[n][r] = 0.0f;
       }
-      const uint32_t x = __funnelshift_r(lo, hi, o & 31);
-      const uint32_t u = (x & ((1u << nb) - 1u)) | 0x4B000000u;
-      const float cf = __uint_as_float(u) - 8388608.0f;
-      if constexpr (GP == 4) {
-        const float4 qv = *reinterpret_cast<const float4*>(qt + c * 4);
-        s[0] = fmaf(qv.x, cf, s[0]);
-        s[1] = fmaf(qv.y, cf, s[1]);
-        s[2] = fmaf(qv.z, cf, s[2]);
-        s[3] = fmaf(qv.w, cf, s[3]);
-      } else {
+      for (int wd = 0; wd < n2w_k; ++wd) {
+        const uint4 af = afrag[wd * 32 + lane];
 #pragma unroll
-        for (int g4 = 0; g4 < GP; g4 += 4) {
-          const float4 qv = *reinterpret_cast<const float4*>(qt + c * GP + g4);
-          s[g4] = fmaf(qv.x, cf, s[g4]);
-          s[g4 + 1] = fmaf(qv.y, cf, s[g4 + 1]);
-          s[g4 + 2] = fmaf(qv.z, cf, s[g4 + 2]);
-          s[g4 + 3] = fmaf(qv.w, cf, s[g4 + 3]);
+        for (int n = 0; n < 4; ++n) {
+          const uint32_t x = kt[wd * TILE + tok[n]];
+          const uint32_t b0 = hsub_magic(((x >> (2 * t)) & 0x00030003u) | 0x64006400u);
+          const uint32_t b1 = hsub_magic(((x >> (2 * t + 8)) & 0x00030003u) | 0x64006400u);
+          mma_16816(sc[n], af, b0, b1);
+        }
+      }
+      for (int w1 = 0; w1 < n1w_k; ++w1) {
+        const int wd = n2w_k + w1;
+        const uint4 af0 = afrag[(n2w_k + 2 * w1) * 32 + lane];
+        const uint4 af1 = afrag[(n2w_k + 2 * w1 + 1) * 32 + lane];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) {
+          const uint32_t x = kt[wd * TILE + tok[n]];
+          mma_16816(sc[n], af0, hsub_magic(((x >> t) & 0x00010001u) | 0x64006400u),
+                    hsub_magic(((x >> (t + 4)) & 0x00010001u) | 0x64006400u));
+          mma_16816(sc[n], af1, hsub_magic(((x >> (t + 8)) & 0x00010001u) | 0x64006400u),
+                    hsub_magic(((x >> (t + 12)) & 0x00010001u) | 0x64006400u));
+        }
+      }
+      // lane holds query g, columns 2t, 2t+1 of each n-tile
+      if (g < G) {
+        const float c0 = cg[g];
+#pragma unroll
+        for (int n = 0; n < 4; ++n) {
+          const int g16 = 2 * warp + (n >> 1);
+          const int half8 = n & 1;
+          const int ta = 16 * g16 + t + 4 * half8;             // column 2t
+          const int tb = ta + 8;                                // column 2t+1
+          const float sa = ak[buf * TILE + ta] * (sc[n][0] + sc[n][2] - c0);
+          const float sb = ak[buf * TILE + tb] * (sc[n][1] + sc[n][3] - c0);
+          stile[g * TILE + ta] = tbase + ta < t_end ? sa : -INFINITY;
+          stile[g * TILE + tb] = tbase + tb < t_end ? sb : -INFINITY;
         }
       }
     }
-    const int t = (tile0 + ti) * TILE + tid;
-    const float ak = al[buf * TILE + tid];
-    const bool valid = t < t_end;
-    float* out = sc + (ti * TILE + tid) * GP;
-#pragma unroll
-    for (int g = 0; g < GP; ++g) {
-      const float v = valid ? ak * (s[g] - cg[g]) : -INFINITY;
-      out[g] = v;
-      mloc[g] = fmaxf(mloc[g], v);
-    }
-  }
-  cp_async_wait_all();
-  __syncthreads();
-
-  // ---- phase 2: split max, probabilities (scaled by alpha^V), split sum
-  block_reduce<GP, true>(mloc, red);
-  stage_tile(vwords, valpha, tile0, 0);
-  float lsum[GP];
-#pragma unroll
-  for (int g = 0; g < GP; ++g) lsum[g] = 0.0f;
-  for (int ti = 0; ti < n_tiles_split; ++ti) {
-    float* p = sc + (ti * TILE + tid) * GP;
-    const int t = (tile0 + ti) * TILE + tid;
-    const float av = t < t_end ? valpha[t] : 0.0f;
-#pragma unroll
-    for (int g = 0; g < GP; ++g) {
-      const float e = exp2f(p[g] - mloc[g]);     // exp2(-inf) = 0 for padding tokens
-      lsum[g] += e;
-      p[g] = e * av;
-    }
-  }
-  block_reduce<GP, false>(lsum, red);
-
-  // ---- phase 3: value accumulation, thread = (4 channels, token quarter)
-  const int cgp = tid & 31, tq = tid >> 5;
-  const int c0 = cgp * 4;
-  int ws_ = 0, sh0 = 0, rel[4], msk[4];
-  float kof[4];
-  {
-    const int* ev = a.ext + (sk + 1) * D;
-    const int o0 = ev[c0] & 0xFFFF;
-    ws_ = o0 >> 5;
-    sh0 = o0 & 31;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int c = c0 + i;
-      const int e = ev[c];
-      const int nb = c < RV ? (e >> 16) : 0;
-      rel[i] = (e & 0xFFFF) - o0;
-      msk[i] = nb > 0 ? ((1 << nb) - 1) : 0;
-      kof[i] = 8388608.0f + (nb > 0 ? static_cast<float>(1 << (nb - 1)) : 0.0f);
-    }
-  }
-  float acc[GP][4];
-#pragma unroll
-  for (int g = 0; g < GP; ++g)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) acc[g][i] = 0.0f;
-  for (int ti = 0; ti < n_tiles_split; ++ti) {
-    const int buf = ti & 1;
-    cp_async_wait_all();
     __syncthreads();
-    if (ti + 1 < n_tiles_split) stage_tile(vwords, valpha, tile0 + ti + 1, buf ^ 1);
-    const uint32_t* w = wt + buf * wt_elems;
-    const int tend = min(TILE, t_end - (tile0 + ti) * TILE);
-    for (int tt = tq; tt < tend; tt += 4) {
-      const uint32_t x = __funnelshift_r(w[ws_ * stride + tt], w[(ws_ + 1) * stride + tt], sh0);
-      const float* p = sc + (ti * TILE + tt) * GP;
-      float cf[4];
+
+    // ---- softmax over the tile, thread = token
+    {
+      const int tt = tid;
+      float sv_[MAX_GROUP], mx[MAX_GROUP];
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        cf[i] = __uint_as_float(((x >> rel[i]) & static_cast<uint32_t>(msk[i])) | 0x4B000000u) - kof[i];
+      for (int gq = 0; gq < MAX_GROUP; ++gq) {
+        sv_[gq] = gq < G ? stile[gq * TILE + tt] : -INFINITY;
+        mx[gq] = sv_[gq];
+      }
+      block_reduce<MAX_GROUP, true>(mx, red);
+      const bool valid = tbase + tt < t_end;
+      const float avt = valid ? av[buf * TILE + tt] : 0.0f;
+      float ps[MAX_GROUP], pp[MAX_GROUP], mnew[MAX_GROUP];
 #pragma unroll
-      for (int g4 = 0; g4 < GP; g4 += 4) {
-        const float4 pv = *reinterpret_cast<const float4*>(p + g4);
-        const float pg[4] = {pv.x, pv.y, pv.z, pv.w};
+      for (int gq = 0; gq < MAX_GROUP; ++gq) {
+        mnew[gq] = fmaxf(run[8 + gq], mx[gq]);
+        const float p = (gq < G && valid) ? exp2f(sv_[gq] - mnew[gq]) : 0.0f;
+        ps[gq] = p;
+        pp[gq] = p * avt;
+      }
+      // P' as (hi, lo) fp16 into the fragment-ordered tile: group, query, slot
+      {
+        const int g16 = tt >> 4, j = tt & 15;
+        const int slot = 4 * (j & 3) + ((j >> 3) & 1) + ((j >> 2) & 1) * 2;
 #pragma unroll
-        for (int gg = 0; gg < 4; ++gg)
+        for (int gq = 0; gq < MAX_GROUP; ++gq) {
+          float hi, lo;
+          split_hi_lo(pp[gq], hi, lo);
+          pfrag[(g16 * MAX_GROUP + gq) * 16 + slot] = pack_half2(hi, lo);
+        }
+      }
+      float sums[2 * MAX_GROUP];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) acc[g4 + gg][i] = fmaf(pg[gg], cf[i], acc[g4 + gg][i]);
+      for (int gq = 0; gq < MAX_GROUP; ++gq) {
+        sums[gq] = ps[gq];
+        sums[MAX_GROUP + gq] = pp[gq];
+      }
+      block_reduce<2 * MAX_GROUP, false>(sums, red);
+      if (tid < MAX_GROUP) {
+        const int gq = tid;
+        const float mo = run[8 + gq];
+        const float cr = mo == -INFINITY ? 0.0f : exp2f(mo - mnew[gq]);
+        run[gq] = cr;
+        run[8 + gq] = mnew[gq];
+        run[16 + gq] = run[16 + gq] * cr + sums[gq];
+        run[24 + gq] = run[24 + gq] * cr + sums[MAX_GROUP + gq];
+      }
+    }
+    __syncthreads();
+
+    // ---- phase V: warp's n-tiles over the 8 groups of the tile
+    {
+      const float cr = run[g];
+#pragma unroll
+      for (int jj = 0; jj < NTW; ++jj)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) acc[jj][r] *= cr;
+      for (int g16 = 0; g16 < kGroups; ++g16) {
+        const uint4 pf = *reinterpret_cast<const uint4*>(pfrag + (g16 * MAX_GROUP + g) * 16 + 4 * t);
+        uint4 af;
+        af.x = __byte_perm(pf.x, pf.y, 0x5410);      // hi of tokens t, t+8
+        af.y = __byte_perm(pf.x, pf.y, 0x7632);      // lo
+        af.z = __byte_perm(pf.z, pf.w, 0x5410);      // hi of tokens t+4, t+12
+        af.w = __byte_perm(pf.z, pf.w, 0x7632);      // lo
+        int cur_wd = -1;
+        uint4 vx = make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int jj = 0; jj < NTW; ++jj) {
+          const int j = j0 + jj;
+          if (j < j1) {
+            int wd, sel, sh;
+            uint32_t msk;
+            if (j < 2 * n2w_v) {
+              wd = j >> 1;
+              sel = j & 1;
+              sh = 2 * g;
+              msk = 0x00030003u;
+            } else {
+              const int r = j - 2 * n2w_v;
+              wd = n2w_v + (r >> 2);
+              sel = (r >> 1) & 1;
+              sh = g + 8 * (r & 1);
+              msk = 0x00010001u;
+            }
+            if (wd != cur_wd) {
+              vx = *reinterpret_cast<const uint4*>(vt + wd * TILE + 16 * g16 + 4 * t);
+              cur_wd = wd;
+            }
+            const uint32_t s0 = sel ? vx.y : vx.x;      // pair t: low- or high-half lane
+            const uint32_t s1 = sel ? vx.w : vx.z;      // pair t+4
+            const uint32_t b0 = hsub_magic(((s0 >> sh) & msk) | 0x64006400u);
+            const uint32_t b1 = hsub_magic(((s1 >> sh) & msk) | 0x64006400u);
+            mma_16816(acc[jj], af, b0, b1);
+          }
+        }
       }
     }
   }
   cp_async_wait_all();
-  __syncthreads();
-  // reduce the four token quarters
+
+  // ---- partials: value sums per record entry, then m, l, S'
+  if (g < G) {
+    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * (a.n_entries + 3);
 #pragma unroll
-  for (int g = 0; g < GP; ++g)
-    *reinterpret_cast<float4*>(accs + (tq * GP + g) * D + c0) = make_float4(acc[g][0], acc[g][1], acc[g][2], acc[g][3]);
-  __syncthreads();
-  for (int g = 0; g < G; ++g) {
-    const float v = accs[(0 * GP + g) * D + tid] + accs[(1 * GP + g) * D + tid] + accs[(2 * GP + g) * D + tid] +
-                    accs[(3 * GP + g) * D + tid];
-    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * (D + 2);
-    dst[tid] = v;
-    if (tid == 0) {
-      dst[D] = mloc[g];
-      dst[D + 1] = lsum[g];
+    for (int jj = 0; jj < NTW; ++jj) {
+      const int j = j0 + jj;
+      if (j < j1) {
+        dst[8 * j + 2 * t] = acc[jj][0] + acc[jj][2];
+        dst[8 * j + 2 * t + 1] = acc[jj][1] + acc[jj][3];
+      }
+    }
+    if (warp == 0 && t == 0) {
+      dst[a.n_entries] = run[8 + g];
+      dst[a.n_entries + 1] = run[16 + g];
+      dst[a.n_entries + 2] = run[24 + g];
     }
   }
 }
 
-// Merge the splits of one (sequence, query head) by log-sum-exp, scale by f^V and apply U_V.
-// With u32 == nullptr the transform is the identity (bf16 reference path).
+// Merge the splits of one (sequence, query head) by log-sum-exp, rebuild channel sums from the
+// record entries (o_c = sum_e 2^shift_e O_e - 2^(b_c-1) S'), scale by f^V / l, apply U_V.
 __global__ void __launch_bounds__(kThreads)
-    aatc_decode_combine_kernel(const float* ws, int n_splits, int n_q, int group, const float* u32, const float* f,
-                               int layer, int n_kv, float* out) {
-  __shared__ float ohat[D];
-  __shared__ float red[8];
+    aatc_decode_combine_kernel(const DecodeArgs a) {
+  extern __shared__ __align__(16) float cs[];
+  float* oe = cs;                          // [n_entries]
+  float* ohat = cs + a.n_entries;          // [128]
+  __shared__ float red[16];
   const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  const int head = j / group;
-  const float* src = ws + (static_cast<size_t>(b) * n_q + j) * n_splits * (D + 2);
+  const int head = j / a.group;
+  const int sv = (a.layer * a.n_kv + head) * 2 + 1;
+  const int stride = a.n_entries + 3;
+  const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * stride;
   float m = -INFINITY;
-  for (int s = tid; s < n_splits; s += kThreads) m = fmaxf(m, src[s * (D + 2) + D]);
+  for (int s = tid; s < a.n_splits; s += kThreads) m = fmaxf(m, src[s * stride + a.n_entries]);
   float mv[1] = {m};
   block_reduce<1, true>(mv, red);
   m = mv[0];
-  float l = 0.0f;
-  for (int s = tid; s < n_splits; s += kThreads) l += src[s * (D + 2) + D + 1] * exp2f(src[s * (D + 2) + D] - m);
-  float lv[1] = {l};
-  block_reduce<1, false>(lv, red);
-  const float inv_l = 1.0f / lv[0];
-  float acc = 0.0f;
-  for (int s = 0; s < n_splits; ++s) acc += src[s * (D + 2) + tid] * exp2f(src[s * (D + 2) + D] - m);
-  const int sv = (layer * n_kv + head) * 2 + 1;
-  const float fv = u32 ? f[sv * D + tid] : 1.0f;
-  ohat[tid] = acc * inv_l * fv;
+  float ls[2] = {0.0f, 0.0f};
+  for (int s = tid; s < a.n_splits; s += kThreads) {
+    const float w = exp2f(src[s * stride + a.n_entries] - m);
+    ls[0] += src[s * stride + a.n_entries + 1] * w;
+    ls[1] += src[s * stride + a.n_entries + 2] * w;
+  }
+  block_reduce<2, false>(ls, red);
+  const StreamLayout lv = a.lay[sv];
+  const int n_used = lv.n2 + lv.n1;
+  for (int e = tid; e < n_used; e += kThreads) {
+    float acc = 0.0f;
+    for (int s = 0; s < a.n_splits; ++s) acc += src[s * stride + e] * exp2f(src[s * stride + a.n_entries] - m);
+    oe[e] = acc;
+  }
   __syncthreads();
-  float o;
-  if (u32) {
-    const float* uv = u32 + static_cast<size_t>(sv) * D * D + tid * D;
-    o = 0.0f;
-    for (int c = 0; c < D; ++c) o = fmaf(uv[c], ohat[c], o);
-  } else {
-    o = ohat[tid];
-  }
-  out[(static_cast<size_t>(b) * n_q + j) * D + tid] = o;
-}
-
-// Dequantization hook: thread per (sequence, token, stream) of the requested range.
-__global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, const int* ext, const float* f,
-                                    int layer, int n_kv, int batch, int t0, int n, int n_tiles, int n_words,
-                                    float* out) {
-  const long idx = static_cast<long>(blockIdx.x) * blockDim.x + threadIdx.x;
-  const long total = static_cast<long>(batch) * n * n_kv * 2;
-  if (idx >= total) return;
-  const int kind = static_cast<int>(idx % 2);
-  const int head = static_cast<int>((idx / 2) % n_kv);
-  const int i = static_cast<int>((idx / (2 * n_kv)) % n);
-  const int b = static_cast<int>(idx / (2L * n_kv * n));
-  const int t = t0 + i;
-  const size_t cs = (static_cast<size_t>(b) * n_kv + head) * 2 + kind;
-  const uint32_t* rec = words + cs * n_tiles * n_words * TILE + static_cast<size_t>(t / TILE) * n_words * TILE + t % TILE;
-  const float at = alpha[cs * n_tiles * TILE + t];
-  const int s = (layer * n_kv + head) * 2 + kind;
-  float* o = out + idx * D;
-  for (int c = 0; c < D; ++c) {
-    const int e = ext[s * D + c];
-    const int off = e & 0xFFFF, nb = e >> 16;
-    float v = 0.0f;
-    if (nb > 0) {
-      const int w = off >> 5, sh = off & 31;
-      const uint32_t lo = rec[static_cast<size_t>(w) * TILE];
-      const uint32_t hi = (sh + nb > 32) ? rec[static_cast<size_t>(w + 1) * TILE] : 0u;
-      const uint32_t u = __funnelshift_r(lo, hi, sh) & ((1u << nb) - 1u);
-      const int code = static_cast<int>(u) - (1 << (nb - 1));
-      const float delta = __fmul_rn(at, f[s * D + c]);
-      v = __fmul_rn(static_cast<float>(code), delta);
+  {
+    const int c = tid;
+    const short* ce = a.chan_ent + (static_cast<size_t>(sv) * D + c) * 8;
+    const short* ent = a.entry + static_cast<size_t>(sv) * a.n_entries;
+    float o = 0.0f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int e = ce[k];
+      if (e >= 0) o += ldexpf(oe[e], ent[e] >> 8);
     }
-    o[c] = v;
+    o -= a.enc[sv * D + c].off * ls[1];
+    ohat[c] = o * a.f[sv * D + c] / ls[0];
   }
+  __syncthreads();
+  const float* ut = a.u32t + static_cast<size_t>(sv) * D * D;
+  float o = 0.0f;
+  for (int c = 0; c < D; ++c) o = fmaf(ut[c * D + tid], ohat[c], o);
+  a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = o;
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -523,33 +637,108 @@ __global__ void __launch_bounds__(kThreads)
   for (int g = 0; g < G; ++g) {
     const float v = accs[(0 * GP + g) * D + tid] + accs[(1 * GP + g) * D + tid] + accs[(2 * GP + g) * D + tid] +
                     accs[(3 * GP + g) * D + tid];
-    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * (D + 2);
+    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * (D + 3);
     dst[tid] = v;
     if (tid == 0) {
       dst[D] = mloc[g];
       dst[D + 1] = lsum[g];
+      dst[D + 2] = 0.0f;
     }
   }
 }
 
-template <int GP>
-size_t split_smem_bytes(int split_len, int n_words) {
-  using L = SplitSmem<GP>;
-  return 4 * (static_cast<size_t>(L::kScores) + static_cast<size_t>(split_len) * GP + 2 * (n_words + 2) * 132 +
-              4 * GP * D);
+// Log-sum-exp merge of bf16-reference partials (identity output transform).
+__global__ void __launch_bounds__(kThreads)
+    aatc_plain_combine_kernel(const float* ws, int n_splits, int n_q, float* out) {
+  __shared__ float red[8];
+  const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  const int stride = D + 3;
+  const float* src = ws + (static_cast<size_t>(b) * n_q + j) * n_splits * stride;
+  float m = -INFINITY;
+  for (int s = tid; s < n_splits; s += kThreads) m = fmaxf(m, src[s * stride + D]);
+  float mv[1] = {m};
+  block_reduce<1, true>(mv, red);
+  m = mv[0];
+  float l = 0.0f;
+  for (int s = tid; s < n_splits; s += kThreads) l += src[s * stride + D + 1] * exp2f(src[s * stride + D] - m);
+  float lv[1] = {l};
+  block_reduce<1, false>(lv, red);
+  float acc = 0.0f;
+  for (int s = 0; s < n_splits; ++s) acc += src[s * stride + tid] * exp2f(src[s * stride + D] - m);
+  out[(static_cast<size_t>(b) * n_q + j) * D + tid] = acc / lv[0];
 }
 
-template <int GP>
-cudaError_t launch_split(const DecodeArgs& a, int batch, int n_kv, cudaStream_t st) {
-  const size_t smem = split_smem_bytes<GP>(a.split_len, a.n_words);
+// Dequantization hook: thread per (sequence, token, stream) of the requested range; rebuilds
+// each stored value from its record entries and returns fl32(code * fl32(alpha * f_c)).
+__global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, const StreamLayout* lays,
+                                    const short* entry, const float* f, int layer, int n_kv, int batch, int t0,
+                                    int n, int n_tiles, int n_words, int n_entries, float* out) {
+  const long idx = static_cast<long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const long total = static_cast<long>(batch) * n * n_kv * 2;
+  if (idx >= total) return;
+  const int kind = static_cast<int>(idx % 2);
+  const int head = static_cast<int>((idx / 2) % n_kv);
+  const int i = static_cast<int>((idx / (2 * n_kv)) % n);
+  const int b = static_cast<int>(idx / (2L * n_kv * n));
+  const int t = t0 + i;
+  const size_t cs = (static_cast<size_t>(b) * n_kv + head) * 2 + kind;
+  const uint32_t* tile = words + cs * n_tiles * n_words * TILE + static_cast<size_t>(t / TILE) * n_words * TILE;
+  const int tt = t % TILE;
+  int lane_lo = tt, lane_hi = tt, half = 0;
+  if (kind == 1) {
+    const int j = tt & 15, pr = j & 7;
+    lane_lo = 16 * (tt >> 4) + 4 * (pr & 3) + 2 * (pr >> 2);
+    lane_hi = lane_lo + 1;
+    half = j >> 3;
+  }
+  auto rec_word = [&](int w) -> uint32_t {
+    if (kind == 0) return tile[static_cast<size_t>(w) * TILE + tt];
+    const uint32_t lo = (tile[static_cast<size_t>(w) * TILE + lane_lo] >> (16 * half)) & 0xFFFFu;
+    const uint32_t hi = (tile[static_cast<size_t>(w) * TILE + lane_hi] >> (16 * half)) & 0xFFFFu;
+    return lo | (hi << 16);
+  };
+  const int s = (layer * n_kv + head) * 2 + kind;
+  const StreamLayout ly = lays[s];
+  const short* ent = entry + static_cast<size_t>(s) * n_entries;
+  uint32_t u[D];
+  for (int c = 0; c < D; ++c) u[c] = 0u;
+  for (int e = 0; e < ly.n2 + ly.n1; ++e) {
+    const int ce = ent[e];
+    uint32_t v;
+    if (e < ly.n2) {
+      v = (rec_word(e >> 4) >> (2 * (e & 15))) & 3u;
+    } else {
+      const int e1 = e - ly.n2;
+      v = (rec_word(ly.n2 / 16 + (e1 >> 5)) >> (e1 & 31)) & 1u;
+    }
+    u[ce & 0xFF] |= v << (ce >> 8);
+  }
+  const float at = alpha[cs * n_tiles * TILE + t];
+  float* o = out + idx * D;
+  for (int c = 0; c < D; ++c) {
+    const float fc = f[s * D + c];
+    float v = 0.0f;
+    if (fc != 0.0f) {
+      int nb = 0;
+      for (int e = 0; e < ly.n2 + ly.n1; ++e)
+        if ((ent[e] & 0xFF) == c) nb = max(nb, (ent[e] >> 8) + (e < ly.n2 ? 2 : 1));
+      const int code = static_cast<int>(u[c]) - (1 << (nb - 1));
+      v = __fmul_rn(static_cast<float>(code), __fmul_rn(at, fc));
+    }
+    o[c] = v;
+  }
+}
+
+template <int NTW>
+cudaError_t launch_split_ntw(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
   static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
   if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<NTW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  aatc_decode_split_kernel<GP><<<dim3(a.n_splits, n_kv, batch), kThreads, smem, st>>>(a);
+  aatc_decode_split_kernel<NTW><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -578,10 +767,15 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.alpha = reinterpret_cast<const float*>(static_cast<const uint32_t*>(cache) + g.words_elems);
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.ws = static_cast<float*>(ws);
+  a.out = out;
   a.u32 = plan.dev.u32;
+  a.u32t = plan.dev.u32t;
   a.f = plan.dev.f;
-  a.ext = plan.dev.ext;
-  a.nret = plan.dev.nret;
+  a.enc = plan.dev.enc;
+  a.lay = plan.dev.lay;
+  a.entry = plan.dev.entry;
+  a.chan_ent = plan.dev.chan_ent;
+  a.err = plan.dev.err;
   a.layer = layer;
   a.n_kv = plan.dims.n_kv_heads;
   a.n_q = plan.dims.n_q_heads;
@@ -589,12 +783,27 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_ctx = n_ctx;
   a.n_tiles = g.n_tiles;
   a.n_words = plan.n_words;
+  a.n_entries = plan.n_entries;
   a.n_splits = sp.n_splits;
   a.split_len = sp.split_len;
-  cudaError_t e = a.group <= 4 ? launch_split<4>(a, batch, a.n_kv, st) : launch_split<8>(a, batch, a.n_kv, st);
+  // largest key k-step count and value n-tile count over the layer's streams
+  int n_ks = 1, n_nt = 1;
+  for (int h = 0; h < a.n_kv; ++h) {
+    const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
+    const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
+    n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
+    n_nt = std::max(n_nt, 2 * (lv.n2 / 16) + 4 * ((lv.n1 + 31) / 32));
+  }
+  const SplitLayout L(n_ks, plan.n_words);
+  const size_t smem = 4 * static_cast<size_t>(L.n_words_total);
+  const int ntw = (n_nt + kWarps - 1) / kWarps;
+  cudaError_t e;
+  if (ntw <= 8) e = launch_split_ntw<8>(a, batch, smem, st);
+  else if (ntw <= 16) e = launch_split_ntw<16>(a, batch, smem, st);
+  else e = launch_split_ntw<32>(a, batch, smem, st);
   if (e != cudaSuccess) return e;
-  aatc_decode_combine_kernel<<<dim3(a.n_q, batch), kThreads, 0, st>>>(a.ws, a.n_splits, a.n_q, a.group, plan.dev.u32,
-                                                                     plan.dev.f, layer, a.n_kv, out);
+  const size_t csmem = 4 * static_cast<size_t>(plan.n_entries + D);
+  aatc_decode_combine_kernel<<<dim3(a.n_q, batch), kThreads, csmem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -606,7 +815,8 @@ cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int b
   const long blocks = (total + threads - 1) / threads;
   aatc_dequant_kernel<<<static_cast<unsigned>(blocks), threads, 0, st>>>(
       static_cast<const uint32_t*>(cache), reinterpret_cast<const float*>(static_cast<const uint32_t*>(cache) + g.words_elems),
-      plan.dev.ext, plan.dev.f, layer, plan.dims.n_kv_heads, batch, t0, n, g.n_tiles, plan.n_words, out);
+      plan.dev.lay, plan.dev.entry, plan.dev.f, layer, plan.dims.n_kv_heads, batch, t0, n, g.n_tiles, plan.n_words,
+      plan.n_entries, out);
   return cudaGetLastError();
 }
 
@@ -626,8 +836,7 @@ cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int 
   a.split_len = sp.split_len;
   cudaError_t e = a.group <= 4 ? launch_bf16_split<4>(a, batch, st) : launch_bf16_split<8>(a, batch, st);
   if (e != cudaSuccess) return e;
-  aatc_decode_combine_kernel<<<dim3(n_q, batch), kThreads, 0, st>>>(a.ws, a.n_splits, n_q, a.group, nullptr, nullptr, 0,
-                                                                     n_kv, out);
+  aatc_plain_combine_kernel<<<dim3(n_q, batch), kThreads, 0, st>>>(a.ws, a.n_splits, n_q, out);
   return cudaGetLastError();
 }
 
@@ -660,7 +869,8 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(cache) & 15u) != 0) return AATC_ERR_INVALID_ARG;
   const DecodeSplit sp = decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (decode_workspace(batch, plan->dims.n_q_heads, sp) > AATC_NOALLOC_SCRATCH_BYTES) return AATC_ERR_WORKSPACE;
+  if (decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp) > AATC_NOALLOC_SCRATCH_BYTES)
+    return AATC_ERR_WORKSPACE;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return status_from_cuda(e);

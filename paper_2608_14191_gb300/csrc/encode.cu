@@ -2,11 +2,12 @@
 //
 // One persistent CTA per (basis, slice of work): a basis is one (layer, kv-head, K|V) stream,
 // an item is 128 consecutive new tokens of one sequence.  Warp roles:
-//   warp 4  : TMA producer -- 128 x 128 bf16 token tiles into a 3-stage SW128 ring,
-//   warp 5  : MMA issuer   -- tcgen05.mma (M=128 tokens, N=128 channels, K=128) into one of
-//                             two TMEM accumulators,
-//   warps 0-3: epilogue    -- thread = token = TMEM lane: token scale alpha, quantize, pack the
-//                             offset-binary fields and store the word-planar record.
+//   warp 16   : TMA producer -- 128 x 128 bf16 token tiles into a 3-stage SW128 ring,
+//   warp 17   : MMA issuer   -- tcgen05.mma (M=128 tokens, N=128 channels, K=128) into one of
+//                               four TMEM accumulators (all 512 columns),
+//   warps 0-15: four epilogue warpgroups; group e drains accumulator e (items e, e+4, ...):
+//               thread = token = TMEM lane: token scale alpha, quantize, split the stored
+//               values into base-4 digits / single bits and write the packed record.
 // The projection uses the plan's bf16 basis; accumulation is fp32.
 #include <cudaTypedefs.h>
 #include <cuda.h>
@@ -22,29 +23,36 @@ namespace {
 
 constexpr int kStages = 3;
 constexpr int kTileBytes = TILE * D * 2;          // 32 KB of bf16
-constexpr int kThreads = 192;
+constexpr int kEpiGroups = 4;
+constexpr int kEpiThreads = 128 * kEpiGroups;
+constexpr int kProducerWarp = kEpiThreads / 32;
+constexpr int kMmaWarp = kProducerWarp + 1;
+constexpr int kThreads = kEpiThreads + 64;
 constexpr int kAccCols = 128;                     // fp32 columns per accumulator
-constexpr uint32_t kTmemCols = 256;               // two accumulators
+constexpr uint32_t kTmemCols = 512;               // four accumulators
+constexpr int kMaxEntries = 32 * 32;              // 32 words x 32 one-bit fields
+constexpr int kByteRow = 132;                     // padded per-thread row of stored values
 
 struct EncodeArgs {
   const ChanEnc* enc;     // plan tables (whole plan)
-  const int* sched;
   const float* inv_s;
-  const int* nret;
+  const StreamLayout* lay;
+  const short* entry;
   int* err;
   uint32_t* words;        // cache word region (this layer)
   float* alpha;           // cache alpha region
-  int layer, n_kv, batch, start, n_tokens, n_chunks, n_words, n_tiles, ctas_per_basis;
+  int layer, n_kv, batch, start, n_tokens, n_chunks, n_words, n_tiles, n_entries, ctas_per_basis;
 };
 
 struct EncodeSmem {
-  // 1024-aligned tiles first
   alignas(1024) unsigned char u_tile[kTileBytes];
   alignas(1024) unsigned char x_tile[kStages][kTileBytes];
   ChanEnc enc[D];
   float inv_s[D];
-  int sched[D];
-  uint64_t full[kStages], empty[kStages], tfull[2], tempty[2], ubar;
+  short entry[kMaxEntries];
+  StreamLayout lay;
+  uint32_t ubytes[kEpiThreads][kByteRow / 4];     // stored values u, one byte per channel
+  uint64_t full[kStages], empty[kStages], tfull[kEpiGroups], tempty[kEpiGroups], ubar;
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -52,6 +60,35 @@ struct EncodeSmem {
 __device__ __forceinline__ void raise_abort(EncodeSmem& sm, int* err) {
   sm.abort_flag = 1;
   atomicOr(err, 2);
+}
+
+// Writes one finished record word of a token.  Keys: plain word-planar store.  Values: the
+// two 16-bit halves go to the token's low-half and high-half lanes of its 16-token pair block.
+struct RecordWriter {
+  uint32_t* key_word;     // keys: &words[.. tile][0][lane]
+  uint16_t* val_lo;       // values: half of the low-half lane
+  uint16_t* val_hi;       // values: half of the high-half lane
+  bool value;
+  __device__ __forceinline__ void put(int wi, uint32_t w) const {
+    if (!value) {
+      key_word[static_cast<size_t>(wi) * TILE] = w;
+    } else {
+      val_lo[static_cast<size_t>(wi) * TILE * 2] = static_cast<uint16_t>(w & 0xFFFFu);
+      val_hi[static_cast<size_t>(wi) * TILE * 2] = static_cast<uint16_t>(w >> 16);
+    }
+  }
+};
+
+// Append the nb low bits of v (nb <= 8, uniform across the warp) to the record bit stream.
+__device__ __forceinline__ void append_bits(uint32_t v, int nb, uint32_t& word, int& pos, int& wi,
+                                            const RecordWriter& out) {
+  word |= v << pos;
+  if (pos + nb >= 32) {
+    out.put(wi, word);
+    ++wi;
+    word = pos + nb > 32 ? (v >> (32 - pos)) : 0u;
+  }
+  pos = (pos + nb) & 31;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -73,18 +110,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int my_items = static_cast<int>(it1 - it0);
   const CUtensorMap* tmap_x = kind == 0 ? &tmap_k : &tmap_v;
 
-  // per-channel tables of this stream
+  // per-stream tables
   for (int c = tid; c < D; c += kThreads) {
     sm.enc[c] = a.enc[stream * D + c];
     sm.inv_s[c] = a.inv_s[stream * D + c];
-    sm.sched[c] = a.sched[stream * D + c];
   }
+  for (int e = tid; e < a.n_entries; e += kThreads) sm.entry[e] = a.entry[static_cast<size_t>(stream) * a.n_entries + e];
   if (tid == 0) {
+    sm.lay = a.lay[stream];
     for (int s = 0; s < kStages; ++s) {
       ptx::mbar_init(&sm.full[s], 1);
       ptx::mbar_init(&sm.empty[s], 1);
     }
-    for (int j = 0; j < 2; ++j) {
+    for (int j = 0; j < kEpiGroups; ++j) {
       ptx::mbar_init(&sm.tfull[j], 1);
       ptx::mbar_init(&sm.tempty[j], 128);
     }
@@ -92,7 +130,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.abort_flag = 0;
     ptx::fence_mbar_init();
   }
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
     ptx::tmem_relinquish();
   }
@@ -102,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = sm.tmem_base;
   volatile int* abort_flag = &sm.abort_flag;
 
-  if (warp == 4) {
+  if (warp == kProducerWarp) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0 && my_items > 0) {
       ptx::prefetch_tmap(tmap_x);
@@ -122,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tma_load_4d(sm.x_tile[s] + kTileBytes / 2, tmap_x, &sm.full[s], 64, head, i0, b);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && my_items > 0) {
       constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128);
@@ -132,8 +170,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; ok && it < my_items; ++it) {
         const int s = it % kStages;
         const uint32_t ph = (it / kStages) & 1;
-        const int acc = it & 1;
-        const uint32_t aph = (it >> 1) & 1;
+        const int acc = it % kEpiGroups;
+        const uint32_t aph = (it / kEpiGroups) & 1;
         if (!ptx::mbar_wait_bounded(&sm.tempty[acc], aph ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
         ptx::tc_fence_after();
         if (!ptx::mbar_wait_bounded(&sm.full[s], ph, abort_flag)) { raise_abort(sm, a.err); break; }
@@ -151,74 +189,119 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue: thread = token
-    const int R = a.nret[stream];
+    const int eg = warp >> 2;                                  // epilogue group = accumulator
+    const int quad = warp & 3;                                 // TMEM lane quadrant
+    const int tl = quad * 32 + lane;                           // token lane inside the tile
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-    for (int it = 0; it < my_items; ++it) {
-      const int acc = it & 1;
-      const uint32_t aph = (it >> 1) & 1;
-      if (!ptx::mbar_wait_bounded(&sm.tfull[acc], aph, abort_flag)) { raise_abort(sm, a.err); break; }
+    const StreamLayout lay = sm.lay;
+    uint32_t* my_bytes = sm.ubytes[tid];
+    for (int it = eg; it < my_items; it += kEpiGroups) {
+      const uint32_t aph = (it / kEpiGroups) & 1;
+      if (!ptx::mbar_wait_bounded(&sm.tfull[eg], aph, abort_flag)) { raise_abort(sm, a.err); break; }
       ptx::tc_fence_after();
-      float h[D];
-      const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(warp * 32) << 16);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) ptx::tmem_ld_32cols(taddr + 32 * j, h + 32 * j);
-      ptx::tmem_ld_wait();
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&sm.tempty[acc]);
-
-      const long item = it0 + it;
-      const int b = static_cast<int>(item / a.n_chunks);
-      const int i = static_cast<int>(item % a.n_chunks) * TILE + tid;     // input token index
-      if (i >= a.n_tokens) continue;
-      const int pos = a.start + i;
-      const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
-      uint32_t* wout = a.words + sidx * stream_words + static_cast<size_t>(pos / TILE) * a.n_words * TILE + (pos % TILE);
+      const uint32_t taddr = tmem + eg * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
 
       // alpha = max_c |h_c| / s_c over retained channels (inv_s = 0 for dropped ones)
       float amax = 0.0f;
 #pragma unroll
-      for (int c = 0; c < D; c += 4) {
-        const float4 is = *reinterpret_cast<const float4*>(&sm.inv_s[c]);
-        amax = fmaxf(amax, fabsf(h[c]) * is.x);
-        amax = fmaxf(amax, fabsf(h[c + 1]) * is.y);
-        amax = fmaxf(amax, fabsf(h[c + 2]) * is.z);
-        amax = fmaxf(amax, fabsf(h[c + 3]) * is.w);
+      for (int j = 0; j < 4; ++j) {
+        float h[32];
+        ptx::tmem_ld_32cols(taddr + 32 * j, h);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; i += 4) {
+          const float4 is = *reinterpret_cast<const float4*>(&sm.inv_s[32 * j + i]);
+          amax = fmaxf(amax, fabsf(h[i]) * is.x);
+          amax = fmaxf(amax, fabsf(h[i + 1]) * is.y);
+          amax = fmaxf(amax, fabsf(h[i + 2]) * is.z);
+          amax = fmaxf(amax, fabsf(h[i + 3]) * is.w);
+        }
       }
-      if (!isfinite(amax)) atomicOr(a.err, 1);
-      a.alpha[sidx * a.n_tiles * TILE + pos] = amax;
       const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
 
-      // quantize + pack, channels in storage order
-      uint32_t word = 0;
-      int wi = 0;
+      // quantize: u = clamp(floor(h / Delta + 1/2)) + 2^(b-1), one byte per channel
+      uint32_t U[32];
 #pragma unroll
-      for (int c = 0; c < D; ++c) {
-        if (c < R) {
-        const ChanEnc e = sm.enc[c];
-        const int sc = sm.sched[c];
-        float x = fmaf(h[c], e.inv_f * ia, 0.5f);                 // h / Delta + 1/2
-        x = fminf(fmaxf(x, e.lo), e.hi);                           // clamp (bounds are integers)
-        const float y = __fadd_rd(x, e.magic);                     // floor, offset binary in the mantissa
-        const uint32_t u = __float_as_uint(y) - 0x4B400000u;
-        const int sh = sched_shift(sc);
-        word |= u << sh;
-        if (sched_flush(sc)) {
-          wout[static_cast<size_t>(wi) * TILE] = word;
-          ++wi;
-          word = u >> (32 - sh);
-        }
+      for (int i = 0; i < 32; ++i) U[i] = 0u;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float h[32];
+        ptx::tmem_ld_32cols(taddr + 32 * j, h);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int c = 32 * j + i;
+          const ChanEnc e = sm.enc[c];
+          float x = fmaf(h[i], e.inv_f * ia, 0.5f);                // h / Delta + 1/2
+          x = fminf(x, e.hi);                                       // |h| / Delta <= 2^(b-1): only the top clamps
+          const float y = __fadd_rd(x, e.magic);                    // floor, offset binary in the mantissa
+          const uint32_t u = __float_as_uint(y) - 0x4B400000u;
+          U[c >> 2] |= u << (8 * (c & 3));
         }
       }
-      for (; wi < a.n_words; ++wi) {
-        wout[static_cast<size_t>(wi) * TILE] = word;
-        word = 0;
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&sm.tempty[eg]);
+
+      const long item = it0 + it;
+      const int b = static_cast<int>(item / a.n_chunks);
+      const int i = static_cast<int>(item % a.n_chunks) * TILE + tl;     // input token index
+      if (i >= a.n_tokens) continue;
+      const int pos_t = a.start + i;
+      const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
+      if (!isfinite(amax)) atomicOr(a.err, 1);
+      a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
+      uint32_t* tile_words = a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE;
+      RecordWriter out;
+      out.value = kind == 1;
+      const int tt = pos_t % TILE;
+      out.key_word = tile_words + tt;
+      {
+        const int j = tt & 15, grp = tt >> 4, pr = j & 7;
+        const int base = 16 * grp + 4 * (pr & 3) + 2 * (pr >> 2);
+        out.val_lo = reinterpret_cast<uint16_t*>(tile_words + base) + (j >> 3);
+        out.val_hi = reinterpret_cast<uint16_t*>(tile_words + base + 1) + (j >> 3);
       }
+
+      // D2: base-4 digit k of channels 0..l2[k]-1, four channels at a time
+      uint32_t word = 0;
+      int pos = 0, wi = 0;
+#pragma unroll 1
+      for (int k = 0; k < 4; ++k) {
+        const int L = lay.l2[k];
+        if (L == 0) continue;
+#pragma unroll
+        for (int g4 = 0; g4 < 32; ++g4) {
+          if (4 * g4 < L) {
+            const int n = min(4, L - 4 * g4);
+            const uint32_t x = (U[g4] >> (2 * k)) & 0x03030303u;
+            uint32_t y = ((x * 0x00041041u) >> 18) & 0xFFu;           // gather the four 2-bit digits
+            y &= (1u << (2 * n)) - 1u;
+            append_bits(y, 2 * n, word, pos, wi, out);
+          }
+        }
+      }
+      // D1: single bits listed in the entry table after the n2 digits
+      if (lay.n1 > 0) {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) my_bytes[q] = U[q];
+        const unsigned char* ub = reinterpret_cast<const unsigned char*>(my_bytes);
+        for (int e = 0; e < lay.n1; ++e) {
+          const int ce = sm.entry[lay.n2 + e];
+          const uint32_t bit = (static_cast<uint32_t>(ub[ce & 0xFF]) >> (ce >> 8)) & 1u;
+          append_bits(bit, 1, word, pos, wi, out);
+        }
+      }
+      if (pos > 0) {
+        out.put(wi, word);
+        ++wi;
+      }
+      for (; wi < a.n_words; ++wi) out.put(wi, 0u);
     }
   }
 
   ptx::tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
@@ -279,10 +362,11 @@ cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
   EncodeArgs a;
   a.enc = plan.dev.enc;
-  a.sched = plan.dev.sched;
   a.inv_s = plan.dev.inv_s;
-  a.nret = plan.dev.nret;
+  a.lay = plan.dev.lay;
+  a.entry = plan.dev.entry;
   a.err = plan.dev.err;
+  a.n_entries = plan.n_entries;
   a.words = static_cast<uint32_t*>(cache);
   a.alpha = reinterpret_cast<float*>(static_cast<uint32_t*>(cache) + g.words_elems);
   a.layer = layer;

@@ -317,6 +317,27 @@ def test_pack_round_trip_random():
         assert O.unpack_records(O.pack_records(codes, bits, nw), bits).tolist() == codes.tolist()
 
 
+def test_value_interleave_round_trip():
+    """Values are stored pair-interleaved in half-words; keys plainly.  Writing records into a
+    cache image and reading them back returns them unchanged for every token position."""
+    rng = np.random.default_rng(15)
+    bits = np.sort(rng.integers(1, 9, O.D))[::-1]
+    nw = O.record_words([bits])
+    n = 300
+    codes = [rng.integers(-(2 ** (bits - 1)), 2 ** (bits - 1), (n, O.D)) for _ in range(4)]
+    recs = [O.pack_records(c, bits, nw) for c in codes]
+    alphas = [rng.random(n).astype(np.float32) for _ in range(4)]
+    img = O.cache_image([[recs[0], recs[1]]], [[recs[2], recs[3]]], [[alphas[0], alphas[1]]],
+                        [[alphas[2], alphas[3]]], 1, 2, 384, nw)
+    for h in range(2):
+        for kind, idx in ((0, h), (1, 2 + h)):
+            rec, al = O.cache_records(img, 1, 2, 384, nw, 0, h, kind, 0, n)
+            assert np.array_equal(rec, recs[idx]) and np.array_equal(al, alphas[idx])
+            assert np.array_equal(O.unpack_records(rec, bits), codes[idx])
+    lanes = sorted({O.value_lane_of(t)[:2] for t in range(16)})
+    assert lanes == [(0, 1), (2, 3), (4, 5), (6, 7), (8, 9), (10, 11), (12, 13), (14, 15)]
+
+
 def test_record_size_matches_paper_compression():
     g = _gold("compression_ratios.json")
     cfg = W.CONFIGS["tiny"]
