@@ -106,8 +106,18 @@ struct DecodeSplit {
 };
 
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
-// Split partials: per (sequence, query head, split) n_entries value sums, then m, l, S'.
-size_t decode_workspace(int batch, int n_q, int n_entries, const DecodeSplit& sp);
+// Decode workspace: split partials per (sequence, query head, split) -- n_entries value sums,
+// then m, l, S', padded to a multiple of 4 floats -- followed by the per-call score A fragments
+// per (sequence, kv-head) (up to 2 W k-steps x 32 lanes x 16 B) and their offset corrections.
+struct DecodeWs {
+  int pstride;            // floats per partial
+  int ks_stride;          // uint4 per (sequence, kv-head) fragment block
+  size_t qfrag_off, qcorr_off, bytes;
+};
+DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
+size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
+// bf16 reference decode partials: 128 sums, then m, l, padding
+size_t bf16_decode_workspace(int batch, int n_q, const DecodeSplit& sp);
 
 // Handle check and CUDA-status mapping shared by every C entry point (defined in capi.cpp).
 Plan* plan_from_handle(aatc_plan_t p);

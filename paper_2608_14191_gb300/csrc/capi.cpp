@@ -41,12 +41,15 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 namespace aatc {
 
+constexpr long kMaxSplits = 96;   // the combine stages every split's partial in shared memory
+
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
   const int tiles = (n_ctx + TILE - 1) / TILE;
   const long units = static_cast<long>(batch) * n_kv;
-  const long target = 2L * std::max(1, num_sms);                 // ~2 CTAs per SM
+  const long target = 4L * std::max(1, num_sms);                 // ~4 CTAs per SM
   long per = (static_cast<long>(tiles) * units + target - 1) / target;
-  per = std::max(1L, std::min(per, 16L));                           // <= 2048 tokens per split
+  per = std::max(per, (static_cast<long>(tiles) + kMaxSplits - 1) / kMaxSplits);   // bounded combine
+  per = std::max(1L, per);
   DecodeSplit sp;
   sp.n_splits = static_cast<int>((tiles + per - 1) / per);
   sp.split_len = static_cast<int>(per) * TILE;
@@ -57,8 +60,22 @@ Plan* plan_from_handle(aatc_plan_t p) { return as_plan(p); }
 
 aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
 
-size_t decode_workspace(int batch, int n_q, int n_entries, const DecodeSplit& sp) {
-  return static_cast<size_t>(batch) * n_q * sp.n_splits * (n_entries + 3) * sizeof(float);
+DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
+  DecodeWs w;
+  w.pstride = (n_entries + 3 + 3) & ~3;
+  w.ks_stride = 2 * n_words * 32;
+  w.qfrag_off = align_up(static_cast<size_t>(batch) * n_q * sp.n_splits * w.pstride * sizeof(float), 256);
+  w.qcorr_off = align_up(w.qfrag_off + static_cast<size_t>(batch) * n_kv * w.ks_stride * 16, 256);
+  w.bytes = w.qcorr_off + static_cast<size_t>(batch) * n_kv * MAX_GROUP * sizeof(float);
+  return w;
+}
+
+size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
+  return decode_ws_layout(batch, n_q, n_kv, n_entries, n_words, sp).bytes;
+}
+
+size_t bf16_decode_workspace(int batch, int n_q, const DecodeSplit& sp) {
+  return static_cast<size_t>(batch) * n_q * sp.n_splits * (D + 3) * sizeof(float);
 }
 
 // D2 / D1 record layout of one stream from its (non-increasing) widths; see StreamLayout.
@@ -304,7 +321,8 @@ aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t 
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
   const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp);
+  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries,
+                                  plan->n_words, sp);
   return AATC_OK;
 }
 
@@ -319,7 +337,8 @@ aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q,
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if (!aligned16(cache) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
   const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp))
+  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries,
+                                               plan->n_words, sp))
     return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
                                          workspace, sp, static_cast<cudaStream_t>(stream)));
@@ -357,7 +376,7 @@ aatc_status_t aatc_bf16_decode_workspace_bytes(int32_t batch, int32_t n_kv, int3
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     sms = 1;
-  *bytes = aatc::decode_workspace(batch, n_q, aatc::D, aatc::decode_split(batch, n_kv, n_ctx, sms));
+  *bytes = aatc::bf16_decode_workspace(batch, n_q, aatc::decode_split(batch, n_kv, n_ctx, sms));
   return AATC_OK;
 }
 
@@ -376,7 +395,7 @@ aatc_status_t aatc_bf16_decode_attention(const void* K, const void* V, const voi
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return cuda_status(e);
   const auto sp = aatc::decode_split(batch, n_kv, n_ctx, sms);
-  if (workspace_bytes < aatc::decode_workspace(batch, n_q, aatc::D, sp)) return AATC_ERR_WORKSPACE;
+  if (workspace_bytes < aatc::bf16_decode_workspace(batch, n_q, sp)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_bf16_decode(K, V, q, batch, n_ctx, max_tokens, n_kv, n_q, out,
                                               workspace, sp, static_cast<cudaStream_t>(stream)));
 }

@@ -82,7 +82,9 @@ struct DecodeArgs {
   const short* entry;      // plan: [S][n_entries]
   const short* chan_ent;   // plan: [S][128][8]
   int* err;
-  int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len;
+  uint4* qfrag;            // workspace: score A fragments [batch][n_kv][ks_stride]
+  float* qcorr;            // workspace: offset corrections [batch][n_kv][8]
+  int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len, ks_stride, pstride;
 };
 
 __device__ __forceinline__ uint32_t hsub_magic(uint32_t x) {
@@ -106,6 +108,13 @@ __device__ __forceinline__ void mma_16816(float (&c)[4], const uint4& a, uint32_
       : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
 }
 
+// 2^x with the hardware approximation (relative error ~2^-22; -inf -> 0)
+__device__ __forceinline__ float fast_exp2(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
 // fp32 -> (hi, lo) fp16 pair with hi + lo = v to ~2^-22 relative
 __device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
   hi = __half2float(__float2half_rn(v));
@@ -117,16 +126,14 @@ constexpr int kWarps = kThreads / 32;
 
 // shared-memory carve-up of the split kernel (32-bit words)
 struct SplitLayout {
-  int qc, cg, afrag, stile, pfrag, corr, red, kw, vw, ak, av, n_words_total;
+  int cg, red, run, afrag, pfrag, kw, vw, ak, av, n_words_total;
   __host__ __device__ SplitLayout(int n_ks, int W) {
     int o = 0;
-    qc = o;    o += MAX_GROUP * D;             // folded query per channel
     cg = o;    o += MAX_GROUP;                 // offset corrections
-    red = o;   o += 4 * MAX_GROUP * 2;         // reductions
-    corr = o;  o += 4 * MAX_GROUP;             // corr, m, l, S' of the running softmax
+    red = o;   o += 3 * kWarps * MAX_GROUP;    // per-warp max / sum p / sum P'
+    run = o;   o += 3 * MAX_GROUP;             // running m, l, S'
     o = (o + 3) & ~3;
     afrag = o; o += n_ks * 32 * 4;             // uint4 per (k-step, lane)
-    stile = o; o += MAX_GROUP * TILE;          // scores of the current tile
     pfrag = o; o += kGroups * MAX_GROUP * 16;  // half2 (hi, lo) of P' per (group, query, slot)
     kw = o;    o += 2 * W * TILE;              // two stages of key words
     vw = o;    o += 2 * W * TILE;              // two stages of value words
@@ -136,7 +143,95 @@ struct SplitLayout {
   }
 };
 
-template <int NTW>
+// Per call, per (sequence, kv-head): folded query q'_{g,c} = (U_K^T q_g)_c f_c log2(e)/sqrt(128),
+// the offset corrections C_g = sum_c q'_{g,c} 2^(b_c-1), and the score A fragments: for each
+// k-step and lane, slot k -> record entry (c, shift) -> q'_c 2^shift as fp16 hi (rows g) / lo
+// (rows g+8).  512 threads: four quarters of the input dimension per channel.
+constexpr int kQThreads = 512;
+
+__global__ void __launch_bounds__(kQThreads)
+    aatc_decode_query_kernel(const DecodeArgs a) {
+  __shared__ float qf[MAX_GROUP][D];
+  __shared__ float part[4][MAX_GROUP][D];
+  __shared__ float qc[MAX_GROUP][D];
+  __shared__ float credw[kQThreads / 32][MAX_GROUP];
+  const int head = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  const int G = a.group;
+  const int sk = (a.layer * a.n_kv + head) * 2;
+  for (int i = tid; i < MAX_GROUP * D; i += kQThreads) {
+    const int gq = i / D, d = i % D;
+    qf[gq][d] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + d]) : 0.0f;
+  }
+  __syncthreads();
+  {
+    const int c = tid & (D - 1), qd = tid >> 7;
+    const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(32 * qd) * D + c;
+    float u[32];
+#pragma unroll
+    for (int d = 0; d < 32; ++d) u[d] = uk[d * D];
+    float acc[MAX_GROUP];
+#pragma unroll
+    for (int gq = 0; gq < MAX_GROUP; ++gq) {
+      acc[gq] = 0.0f;
+#pragma unroll
+      for (int d = 0; d < 32; ++d) acc[gq] = fmaf(u[d], qf[gq][32 * qd + d], acc[gq]);
+      part[qd][gq][c] = acc[gq];
+    }
+  }
+  __syncthreads();
+  if (tid < D) {
+    const int c = tid;
+    const float fk = a.f[sk * D + c] * (kLog2e * 0.08838834764831845f);   // 1/sqrt(128)
+    const float off = a.enc[sk * D + c].off;
+    float cr[MAX_GROUP];
+#pragma unroll
+    for (int gq = 0; gq < MAX_GROUP; ++gq) {
+      const float v = (part[0][gq][c] + part[1][gq][c] + part[2][gq][c] + part[3][gq][c]) * fk;
+      qc[gq][c] = v;
+      cr[gq] = v * off;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cr[gq] += __shfl_xor_sync(0xffffffffu, cr[gq], o);
+    }
+    if ((tid & 31) == 0)
+#pragma unroll
+      for (int gq = 0; gq < MAX_GROUP; ++gq) credw[tid >> 5][gq] = cr[gq];
+  }
+  __syncthreads();
+  if (tid < MAX_GROUP)
+    a.qcorr[(static_cast<size_t>(b) * a.n_kv + head) * MAX_GROUP + tid] =
+        credw[0][tid] + credw[1][tid] + credw[2][tid] + credw[3][tid];
+  const StreamLayout lk = a.lay[sk];
+  const int n2w = lk.n2 / 16, n_ks = n2w + 2 * ((lk.n1 + 31) / 32);
+  const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
+  uint4* dst = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
+  for (int i = tid; i < n_ks * 32; i += kQThreads) {
+    const int ks = i >> 5, ln = i & 31, gq = ln >> 2, tq = ln & 3;
+    int fld[4];                                   // fields for k = 2t, 2t+1, 2t+8, 2t+9
+    int ebase;
+    if (ks < n2w) {
+      ebase = 16 * ks;
+      fld[0] = tq; fld[1] = tq + 8; fld[2] = tq + 4; fld[3] = tq + 12;
+    } else {
+      const int r = ks - n2w, h8 = 8 * (r & 1);
+      ebase = lk.n2 + 32 * (r >> 1);
+      fld[0] = tq + h8; fld[1] = tq + 16 + h8; fld[2] = tq + 4 + h8; fld[3] = tq + 20 + h8;
+    }
+    float hi[4], lo[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = ebase + fld[j];
+      const int ce = (e < lk.n2 + lk.n1) ? ent[e] : -1;
+      const float coef = (ce >= 0 && gq < G) ? ldexpf(qc[gq][ce & 0xFF], ce >> 8) : 0.0f;
+      split_hi_lo(coef, hi[j], lo[j]);
+    }
+    dst[i] = make_uint4(pack_half2(hi[0], hi[1]), pack_half2(lo[0], lo[1]), pack_half2(hi[2], hi[3]),
+                        pack_half2(lo[2], lo[3]));
+  }
+}
+
+// Value n-tiles of one record word: a D2 word gives two (fields 0-7 from the low-half lane,
+// fields 8-15 from the high-half lane, shift 2g), a D1 word four (low/high lane x shift g, g+8).
+template <int WPW, int GP>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
   extern __shared__ __align__(16) uint32_t smw[];
@@ -149,15 +244,12 @@ __global__ void __launch_bounds__(kThreads)
   const int W = a.n_words;
   const int n2w_k = lk.n2 / 16, n1w_k = (lk.n1 + 31) / 32;
   const int n_ks = n2w_k + 2 * n1w_k;
-  const int n2w_v = lv.n2 / 16, n1w_v = (lv.n1 + 31) / 32;
-  const int n_nt = 2 * n2w_v + 4 * n1w_v;
+  const int n2w_v = lv.n2 / 16, nw_v = n2w_v + (lv.n1 + 31) / 32;
   const SplitLayout L(n_ks, W);
-  float* qc = reinterpret_cast<float*>(smw + L.qc);
   float* cg = reinterpret_cast<float*>(smw + L.cg);
-  float* red = reinterpret_cast<float*>(smw + L.red);
-  float* run = reinterpret_cast<float*>(smw + L.corr);         // [0..7] corr, [8..15] m, [16..23] l, [24..31] S'
+  float* red = reinterpret_cast<float*>(smw + L.red);          // [3][kWarps][8]
+  float* run = reinterpret_cast<float*>(smw + L.run);          // [3][8]: m, l, S'
   uint4* afrag = reinterpret_cast<uint4*>(smw + L.afrag);
-  float* stile = reinterpret_cast<float*>(smw + L.stile);
   uint32_t* pfrag = smw + L.pfrag;
   uint32_t* kw = smw + L.kw;
   uint32_t* vw = smw + L.vw;
@@ -189,78 +281,33 @@ __global__ void __launch_bounds__(kThreads)
   };
   stage(tile0, 0);
 
-  // ---- prologue: folded query q'_{g,c} = (U_K^T q_g)_c f_c log2(e) / sqrt(128)
+  // ---- prologue: score A fragments and offset corrections of this (sequence, kv-head), built
+  // once per call by aatc_decode_query_kernel
   {
-    float* qf = stile;                                      // scratch: fp32 query [8][128]
-    for (int i = tid; i < MAX_GROUP * D; i += kThreads) {
-      const int gq = i / D, d = i % D;
-      qf[i] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + d]) : 0.0f;
-    }
-    __syncthreads();
-    const int c = tid;
-    float accq[MAX_GROUP];
-#pragma unroll
-    for (int gq = 0; gq < MAX_GROUP; ++gq) accq[gq] = 0.0f;
-    const float* uk = a.u32 + static_cast<size_t>(sk) * D * D;
-    for (int d = 0; d < D; ++d) {
-      const float u = uk[d * D + c];
-#pragma unroll
-      for (int gq = 0; gq < MAX_GROUP; ++gq) accq[gq] = fmaf(u, qf[gq * D + d], accq[gq]);
-    }
-    const float fk = a.f[sk * D + c] * (kLog2e * 0.08838834764831845f);   // 1/sqrt(128)
-    const float off = a.enc[sk * D + c].off;
-    float corr8[MAX_GROUP];
-#pragma unroll
-    for (int gq = 0; gq < MAX_GROUP; ++gq) {
-      const float v = accq[gq] * fk;
-      qc[gq * D + c] = v;
-      corr8[gq] = v * off;
-    }
-    block_reduce<MAX_GROUP, false>(corr8, red);
-    if (tid < MAX_GROUP) cg[tid] = corr8[tid];
+    const uint4* qsrc = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
+    for (int i = tid; i < n_ks * 32; i += kThreads) cp_async16(afrag + i, qsrc + i);
+    cp_async_commit();
     if (tid < MAX_GROUP) {
-      run[tid] = 0.0f;                 // corr
-      run[8 + tid] = -INFINITY;        // m
-      run[16 + tid] = 0.0f;            // l
-      run[24 + tid] = 0.0f;            // S'
+      cg[tid] = a.qcorr[(static_cast<size_t>(b) * a.n_kv + head) * MAX_GROUP + tid];
+      run[tid] = -INFINITY;            // m
+      run[8 + tid] = 0.0f;             // l
+      run[16 + tid] = 0.0f;            // S'
     }
-  }
-  __syncthreads();
-  // score A fragments: slot k of k-step ks -> record entry -> coefficient q'_c 2^shift
-  {
-    const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
-    for (int i = tid; i < n_ks * 32; i += kThreads) {
-      const int ks = i >> 5, ln = i & 31, gq = ln >> 2, tq = ln & 3;
-      int fld[4];                                   // fields for k = 2t, 2t+1, 2t+8, 2t+9
-      int ebase;
-      if (ks < n2w_k) {
-        ebase = 16 * ks;
-        fld[0] = tq; fld[1] = tq + 8; fld[2] = tq + 4; fld[3] = tq + 12;
-      } else {
-        const int r = ks - n2w_k, h8 = 8 * (r & 1);
-        ebase = lk.n2 + 32 * (r >> 1);
-        fld[0] = tq + h8; fld[1] = tq + 16 + h8; fld[2] = tq + 4 + h8; fld[3] = tq + 20 + h8;
-      }
-      float hi[4], lo[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int e = ebase + fld[j];
-        const int ce = (e < lk.n2 + lk.n1) ? ent[e] : -1;
-        const float coef = (ce >= 0 && gq < G) ? ldexpf(qc[gq * D + (ce & 0xFF)], ce >> 8) : 0.0f;
-        split_hi_lo(coef, hi[j], lo[j]);
-      }
-      afrag[i] = make_uint4(pack_half2(hi[0], hi[1]), pack_half2(lo[0], lo[1]), pack_half2(hi[2], hi[3]),
-                            pack_half2(lo[2], lo[3]));
-    }
+    for (int i = tid; i < kGroups * MAX_GROUP * 16; i += kThreads) pfrag[i] = 0u;   // rows g >= G stay 0
+    cp_async_wait_all();
+    __syncthreads();
   }
 
-  // value n-tiles of this warp and their accumulators (rows g: P' hi part, g+8: lo part)
-  const int j0 = warp * n_nt / kWarps, j1 = (warp + 1) * n_nt / kWarps;
-  float acc[NTW][4];
+  // value words of this warp (contiguous) and their n-tile accumulators
+  const int vw0 = warp * nw_v / kWarps, vw1 = (warp + 1) * nw_v / kWarps;
+  float acc[WPW][4][4];
 #pragma unroll
-  for (int jj = 0; jj < NTW; ++jj)
+  for (int i = 0; i < WPW; ++i)
 #pragma unroll
-    for (int r = 0; r < 4; ++r) acc[jj][r] = 0.0f;
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) acc[i][q][r] = 0.0f;
+  const float c0 = cg[g];
 
   for (int ti = 0; ti < n_tiles_split; ++ti) {
     const int buf = ti & 1;
@@ -271,212 +318,237 @@ __global__ void __launch_bounds__(kThreads)
     const uint32_t* vt = vw + buf * W * TILE;
     const int tbase = (tile0 + ti) * TILE;
 
-    // ---- phase S: warp handles groups 2 warp, 2 warp + 1 (4 score n-tiles of 8 tokens)
-    {
-      float sc[4][4];
-      int tok[4];
+    // ---- scores: this warp's groups 2 warp, 2 warp + 1 as four n-tiles of 8 tokens
+    float sc[4][4];
+    int tok[4];
+#pragma unroll
+    for (int n = 0; n < 4; ++n) {
+      tok[n] = 16 * (2 * warp + (n >> 1)) + (g & 1 ? 8 : 0) + (g >> 1) + 4 * (n & 1);   // column g's token
+#pragma unroll
+      for (int r = 0; r < 4; ++r) sc[n][r] = 0.0f;
+    }
+    for (int wd = 0; wd < n2w_k; ++wd) {
+      const uint4 af = afrag[wd * 32 + lane];
 #pragma unroll
       for (int n = 0; n < 4; ++n) {
-        const int g16 = 2 * warp + (n >> 1);
-        const int half8 = n & 1;                               // n-tile A (0) or B (1)
-        tok[n] = 16 * g16 + (g & 1 ? 8 : 0) + (g >> 1) + 4 * half8;   // token of column n = g
-#pragma unroll
-        for (int r = 0; r < 4; ++r) sc[n][r] = 0.0f;
+        const uint32_t x = kt[wd * TILE + tok[n]];
+        mma_16816(sc[n], af, hsub_magic(((x >> (2 * t)) & 0x00030003u) | 0x64006400u),
+                  hsub_magic(((x >> (2 * t + 8)) & 0x00030003u) | 0x64006400u));
       }
-      for (int wd = 0; wd < n2w_k; ++wd) {
-        const uint4 af = afrag[wd * 32 + lane];
+    }
+    for (int w1 = 0; w1 < n1w_k; ++w1) {
+      const int wd = n2w_k + w1;
+      const uint4 af0 = afrag[(n2w_k + 2 * w1) * 32 + lane];
+      const uint4 af1 = afrag[(n2w_k + 2 * w1 + 1) * 32 + lane];
 #pragma unroll
-        for (int n = 0; n < 4; ++n) {
-          const uint32_t x = kt[wd * TILE + tok[n]];
-          const uint32_t b0 = hsub_magic(((x >> (2 * t)) & 0x00030003u) | 0x64006400u);
-          const uint32_t b1 = hsub_magic(((x >> (2 * t + 8)) & 0x00030003u) | 0x64006400u);
-          mma_16816(sc[n], af, b0, b1);
+      for (int n = 0; n < 4; ++n) {
+        const uint32_t x = kt[wd * TILE + tok[n]];
+        mma_16816(sc[n], af0, hsub_magic(((x >> t) & 0x00010001u) | 0x64006400u),
+                  hsub_magic(((x >> (t + 4)) & 0x00010001u) | 0x64006400u));
+        mma_16816(sc[n], af1, hsub_magic(((x >> (t + 8)) & 0x00010001u) | 0x64006400u),
+                  hsub_magic(((x >> (t + 12)) & 0x00010001u) | 0x64006400u));
+      }
+    }
+    // lane holds query g, columns 2t (token ta) and 2t+1 (token ta + 8) of each n-tile
+    float s8[4][2];
+    float mloc = -INFINITY;
+#pragma unroll
+    for (int n = 0; n < 4; ++n) {
+      const int ta = 16 * (2 * warp + (n >> 1)) + t + 4 * (n & 1);
+      const float sa = ak[buf * TILE + ta] * (sc[n][0] + sc[n][2] - c0);
+      const float sb = ak[buf * TILE + ta + 8] * (sc[n][1] + sc[n][3] - c0);
+      s8[n][0] = (g < G && tbase + ta < t_end) ? sa : -INFINITY;
+      s8[n][1] = (g < G && tbase + ta + 8 < t_end) ? sb : -INFINITY;
+      mloc = fmaxf(mloc, fmaxf(s8[n][0], s8[n][1]));
+    }
+    mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 1));
+    mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 2));
+    if (t == 0) red[warp * 8 + g] = mloc;
+    __syncthreads();
+    const float m_old = run[g];
+    float m_new = m_old;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) m_new = fmaxf(m_new, red[w * 8 + g]);
+    const float corr = m_old == -INFINITY ? 0.0f : fast_exp2(m_old - m_new);
+    // probabilities, P' = p alpha^V, partial sums, and the P' fragments for the value product
+    float lsum = 0.0f, ssum = 0.0f;
+#pragma unroll
+    for (int gg = 0; gg < 2; ++gg) {
+      float pv[4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          const int n = 2 * gg + h;
+          const int tk = 16 * (2 * warp + gg) + t + 4 * h + 8 * cc;
+          const float p = s8[n][cc] == -INFINITY ? 0.0f : fast_exp2(s8[n][cc] - m_new);
+          const float pp = p * av[buf * TILE + tk];
+          lsum += p;
+          ssum += pp;
+          pv[2 * h + cc] = pp;                 // slot 4t + {0: token t, 1: t+8, 2: t+4, 3: t+12}
         }
-      }
-      for (int w1 = 0; w1 < n1w_k; ++w1) {
-        const int wd = n2w_k + w1;
-        const uint4 af0 = afrag[(n2w_k + 2 * w1) * 32 + lane];
-        const uint4 af1 = afrag[(n2w_k + 2 * w1 + 1) * 32 + lane];
-#pragma unroll
-        for (int n = 0; n < 4; ++n) {
-          const uint32_t x = kt[wd * TILE + tok[n]];
-          mma_16816(sc[n], af0, hsub_magic(((x >> t) & 0x00010001u) | 0x64006400u),
-                    hsub_magic(((x >> (t + 4)) & 0x00010001u) | 0x64006400u));
-          mma_16816(sc[n], af1, hsub_magic(((x >> (t + 8)) & 0x00010001u) | 0x64006400u),
-                    hsub_magic(((x >> (t + 12)) & 0x00010001u) | 0x64006400u));
-        }
-      }
-      // lane holds query g, columns 2t, 2t+1 of each n-tile
       if (g < G) {
-        const float c0 = cg[g];
-#pragma unroll
-        for (int n = 0; n < 4; ++n) {
-          const int g16 = 2 * warp + (n >> 1);
-          const int half8 = n & 1;
-          const int ta = 16 * g16 + t + 4 * half8;             // column 2t
-          const int tb = ta + 8;                                // column 2t+1
-          const float sa = ak[buf * TILE + ta] * (sc[n][0] + sc[n][2] - c0);
-          const float sb = ak[buf * TILE + tb] * (sc[n][1] + sc[n][3] - c0);
-          stile[g * TILE + ta] = tbase + ta < t_end ? sa : -INFINITY;
-          stile[g * TILE + tb] = tbase + tb < t_end ? sb : -INFINITY;
-        }
+        uint4 pk;
+        float hi, lo;
+        split_hi_lo(pv[0], hi, lo); pk.x = pack_half2(hi, lo);
+        split_hi_lo(pv[1], hi, lo); pk.y = pack_half2(hi, lo);
+        split_hi_lo(pv[2], hi, lo); pk.z = pack_half2(hi, lo);
+        split_hi_lo(pv[3], hi, lo); pk.w = pack_half2(hi, lo);
+        *reinterpret_cast<uint4*>(pfrag + ((2 * warp + gg) * MAX_GROUP + g) * 16 + 4 * t) = pk;
       }
     }
-    __syncthreads();
-
-    // ---- softmax over the tile, thread = token
-    {
-      const int tt = tid;
-      float sv_[MAX_GROUP], mx[MAX_GROUP];
-#pragma unroll
-      for (int gq = 0; gq < MAX_GROUP; ++gq) {
-        sv_[gq] = gq < G ? stile[gq * TILE + tt] : -INFINITY;
-        mx[gq] = sv_[gq];
-      }
-      block_reduce<MAX_GROUP, true>(mx, red);
-      const bool valid = tbase + tt < t_end;
-      const float avt = valid ? av[buf * TILE + tt] : 0.0f;
-      float ps[MAX_GROUP], pp[MAX_GROUP], mnew[MAX_GROUP];
-#pragma unroll
-      for (int gq = 0; gq < MAX_GROUP; ++gq) {
-        mnew[gq] = fmaxf(run[8 + gq], mx[gq]);
-        const float p = (gq < G && valid) ? exp2f(sv_[gq] - mnew[gq]) : 0.0f;
-        ps[gq] = p;
-        pp[gq] = p * avt;
-      }
-      // P' as (hi, lo) fp16 into the fragment-ordered tile: group, query, slot
-      {
-        const int g16 = tt >> 4, j = tt & 15;
-        const int slot = 4 * (j & 3) + ((j >> 3) & 1) + ((j >> 2) & 1) * 2;
-#pragma unroll
-        for (int gq = 0; gq < MAX_GROUP; ++gq) {
-          float hi, lo;
-          split_hi_lo(pp[gq], hi, lo);
-          pfrag[(g16 * MAX_GROUP + gq) * 16 + slot] = pack_half2(hi, lo);
-        }
-      }
-      float sums[2 * MAX_GROUP];
-#pragma unroll
-      for (int gq = 0; gq < MAX_GROUP; ++gq) {
-        sums[gq] = ps[gq];
-        sums[MAX_GROUP + gq] = pp[gq];
-      }
-      block_reduce<2 * MAX_GROUP, false>(sums, red);
-      if (tid < MAX_GROUP) {
-        const int gq = tid;
-        const float mo = run[8 + gq];
-        const float cr = mo == -INFINITY ? 0.0f : exp2f(mo - mnew[gq]);
-        run[gq] = cr;
-        run[8 + gq] = mnew[gq];
-        run[16 + gq] = run[16 + gq] * cr + sums[gq];
-        run[24 + gq] = run[24 + gq] * cr + sums[MAX_GROUP + gq];
-      }
+    lsum += __shfl_xor_sync(0xffffffffu, lsum, 1);
+    lsum += __shfl_xor_sync(0xffffffffu, lsum, 2);
+    ssum += __shfl_xor_sync(0xffffffffu, ssum, 1);
+    ssum += __shfl_xor_sync(0xffffffffu, ssum, 2);
+    if (t == 0) {
+      red[(kWarps + warp) * 8 + g] = lsum;
+      red[(2 * kWarps + warp) * 8 + g] = ssum;
     }
     __syncthreads();
+    if (warp == 0 && t == 0) {
+      float l = 0.0f, sp = 0.0f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        l += red[(kWarps + w) * 8 + g];
+        sp += red[(2 * kWarps + w) * 8 + g];
+      }
+      run[g] = m_new;
+      run[8 + g] = run[8 + g] * corr + l;
+      run[16 + g] = run[16 + g] * corr + sp;
+    }
 
-    // ---- phase V: warp's n-tiles over the 8 groups of the tile
-    {
-      const float cr = run[g];
+    // ---- values: this warp's record words over the 8 groups of the tile
 #pragma unroll
-      for (int jj = 0; jj < NTW; ++jj)
+    for (int i = 0; i < WPW; ++i)
 #pragma unroll
-        for (int r = 0; r < 4; ++r) acc[jj][r] *= cr;
-      for (int g16 = 0; g16 < kGroups; ++g16) {
-        const uint4 pf = *reinterpret_cast<const uint4*>(pfrag + (g16 * MAX_GROUP + g) * 16 + 4 * t);
-        uint4 af;
-        af.x = __byte_perm(pf.x, pf.y, 0x5410);      // hi of tokens t, t+8
-        af.y = __byte_perm(pf.x, pf.y, 0x7632);      // lo
-        af.z = __byte_perm(pf.z, pf.w, 0x5410);      // hi of tokens t+4, t+12
-        af.w = __byte_perm(pf.z, pf.w, 0x7632);      // lo
-        int cur_wd = -1;
-        uint4 vx = make_uint4(0, 0, 0, 0);
+      for (int q = 0; q < 4; ++q)
 #pragma unroll
-        for (int jj = 0; jj < NTW; ++jj) {
-          const int j = j0 + jj;
-          if (j < j1) {
-            int wd, sel, sh;
-            uint32_t msk;
-            if (j < 2 * n2w_v) {
-              wd = j >> 1;
-              sel = j & 1;
-              sh = 2 * g;
-              msk = 0x00030003u;
-            } else {
-              const int r = j - 2 * n2w_v;
-              wd = n2w_v + (r >> 2);
-              sel = (r >> 1) & 1;
-              sh = g + 8 * (r & 1);
-              msk = 0x00010001u;
-            }
-            if (wd != cur_wd) {
-              vx = *reinterpret_cast<const uint4*>(vt + wd * TILE + 16 * g16 + 4 * t);
-              cur_wd = wd;
-            }
-            const uint32_t s0 = sel ? vx.y : vx.x;      // pair t: low- or high-half lane
-            const uint32_t s1 = sel ? vx.w : vx.z;      // pair t+4
-            const uint32_t b0 = hsub_magic(((s0 >> sh) & msk) | 0x64006400u);
-            const uint32_t b1 = hsub_magic(((s1 >> sh) & msk) | 0x64006400u);
-            mma_16816(acc[jj], af, b0, b1);
+        for (int r = 0; r < 4; ++r) acc[i][q][r] *= corr;
+#pragma unroll 2
+    for (int g16 = 0; g16 < kGroups; ++g16) {
+      const uint4 pf = *reinterpret_cast<const uint4*>(pfrag + (g16 * MAX_GROUP + g) * 16 + 4 * t);
+      uint4 af;
+      af.x = __byte_perm(pf.x, pf.y, 0x5410);      // hi of tokens t, t+8
+      af.y = __byte_perm(pf.x, pf.y, 0x7632);      // lo
+      af.z = __byte_perm(pf.z, pf.w, 0x5410);      // hi of tokens t+4, t+12
+      af.w = __byte_perm(pf.z, pf.w, 0x7632);      // lo
+#pragma unroll
+      for (int i = 0; i < WPW; ++i) {
+        const int wd = vw0 + i;
+        if (wd < vw1) {
+          const uint4 vx = *reinterpret_cast<const uint4*>(vt + wd * TILE + 16 * g16 + 4 * t);
+          if (wd < n2w_v) {
+            mma_16816(acc[i][0], af, hsub_magic(((vx.x >> (2 * g)) & 0x00030003u) | 0x64006400u),
+                      hsub_magic(((vx.z >> (2 * g)) & 0x00030003u) | 0x64006400u));
+            mma_16816(acc[i][1], af, hsub_magic(((vx.y >> (2 * g)) & 0x00030003u) | 0x64006400u),
+                      hsub_magic(((vx.w >> (2 * g)) & 0x00030003u) | 0x64006400u));
+          } else {
+            mma_16816(acc[i][0], af, hsub_magic(((vx.x >> g) & 0x00010001u) | 0x64006400u),
+                      hsub_magic(((vx.z >> g) & 0x00010001u) | 0x64006400u));
+            mma_16816(acc[i][1], af, hsub_magic(((vx.x >> (g + 8)) & 0x00010001u) | 0x64006400u),
+                      hsub_magic(((vx.z >> (g + 8)) & 0x00010001u) | 0x64006400u));
+            mma_16816(acc[i][2], af, hsub_magic(((vx.y >> g) & 0x00010001u) | 0x64006400u),
+                      hsub_magic(((vx.w >> g) & 0x00010001u) | 0x64006400u));
+            mma_16816(acc[i][3], af, hsub_magic(((vx.y >> (g + 8)) & 0x00010001u) | 0x64006400u),
+                      hsub_magic(((vx.w >> (g + 8)) & 0x00010001u) | 0x64006400u));
           }
         }
       }
     }
   }
   cp_async_wait_all();
+  __syncthreads();
 
   // ---- partials: value sums per record entry, then m, l, S'
   if (g < G) {
-    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * (a.n_entries + 3);
+    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * a.pstride;
 #pragma unroll
-    for (int jj = 0; jj < NTW; ++jj) {
-      const int j = j0 + jj;
-      if (j < j1) {
-        dst[8 * j + 2 * t] = acc[jj][0] + acc[jj][2];
-        dst[8 * j + 2 * t + 1] = acc[jj][1] + acc[jj][3];
+    for (int i = 0; i < WPW; ++i) {
+      const int wd = vw0 + i;
+      if (wd < vw1) {
+        const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
+        const int nq = wd < n2w_v ? 2 : 4;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (q < nq) {
+            dst[ebase + 8 * q + 2 * t] = acc[i][q][0] + acc[i][q][2];
+            dst[ebase + 8 * q + 2 * t + 1] = acc[i][q][1] + acc[i][q][3];
+          }
       }
     }
     if (warp == 0 && t == 0) {
-      dst[a.n_entries] = run[8 + g];
-      dst[a.n_entries + 1] = run[16 + g];
-      dst[a.n_entries + 2] = run[24 + g];
+      dst[a.n_entries] = run[g];
+      dst[a.n_entries + 1] = run[8 + g];
+      dst[a.n_entries + 2] = run[16 + g];
     }
   }
 }
 
 // Merge the splits of one (sequence, query head) by log-sum-exp, rebuild channel sums from the
 // record entries (o_c = sum_e 2^shift_e O_e - 2^(b_c-1) S'), scale by f^V / l, apply U_V.
-__global__ void __launch_bounds__(kThreads)
+// The partials of all splits are staged in shared memory with 16-byte loads first.
+constexpr int kCThreads = 256;
+
+__global__ void __launch_bounds__(kCThreads)
     aatc_decode_combine_kernel(const DecodeArgs a) {
   extern __shared__ __align__(16) float cs[];
-  float* oe = cs;                          // [n_entries]
-  float* ohat = cs + a.n_entries;          // [128]
-  __shared__ float red[16];
+  const int stride = a.pstride;                      // multiple of 4
+  float* part = cs;                                  // [n_splits][stride]
+  float* wsp = part + a.n_splits * stride;           // [n_splits] split weights
+  float* oe = wsp + ((a.n_splits + 3) & ~3);         // [n_entries]
+  float* ohat = oe + a.n_entries;                    // [128]
+  float* ut_s = ohat + D;                            // [128][128] U_V^T of this kv-head
+  __shared__ float red[2][kCThreads / 32];
+  __shared__ float lsum[2];
   const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
   const int head = j / a.group;
   const int sv = (a.layer * a.n_kv + head) * 2 + 1;
-  const int stride = a.n_entries + 3;
-  const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * stride;
+  const float4* src = reinterpret_cast<const float4*>(a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * stride);
+  const int n4 = a.n_splits * stride / 4;
+  float4* p4 = reinterpret_cast<float4*>(part);
+  for (int i = tid; i < n4; i += kCThreads) cp_async16(p4 + i, src + i);
+  const float4* us = reinterpret_cast<const float4*>(a.u32t + static_cast<size_t>(sv) * D * D);
+  for (int i = tid; i < D * D / 4; i += kCThreads) cp_async16(reinterpret_cast<float4*>(ut_s) + i, us + i);
+  cp_async_commit();
+  cp_async_wait_all();
+  __syncthreads();
+  // split weights 2^(m_s - M): every thread scans the split maxima (few dozen)
   float m = -INFINITY;
-  for (int s = tid; s < a.n_splits; s += kThreads) m = fmaxf(m, src[s * stride + a.n_entries]);
-  float mv[1] = {m};
-  block_reduce<1, true>(mv, red);
-  m = mv[0];
-  float ls[2] = {0.0f, 0.0f};
-  for (int s = tid; s < a.n_splits; s += kThreads) {
-    const float w = exp2f(src[s * stride + a.n_entries] - m);
-    ls[0] += src[s * stride + a.n_entries + 1] * w;
-    ls[1] += src[s * stride + a.n_entries + 2] * w;
+  for (int s = 0; s < a.n_splits; ++s) m = fmaxf(m, part[s * stride + a.n_entries]);
+  if (tid < a.n_splits) wsp[tid] = exp2f(part[tid * stride + a.n_entries] - m);
+  for (int s = tid + kCThreads; s < a.n_splits; s += kCThreads) wsp[s] = exp2f(part[s * stride + a.n_entries] - m);
+  __syncthreads();
+  if (tid < 64) {
+    float l = 0.0f, sp = 0.0f;
+    for (int s = tid; s < a.n_splits; s += 64) {
+      l += part[s * stride + a.n_entries + 1] * wsp[s];
+      sp += part[s * stride + a.n_entries + 2] * wsp[s];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      l += __shfl_xor_sync(0xffffffffu, l, o);
+      sp += __shfl_xor_sync(0xffffffffu, sp, o);
+    }
+    if ((tid & 31) == 0) {
+      red[0][tid >> 5] = l;
+      red[1][tid >> 5] = sp;
+    }
   }
-  block_reduce<2, false>(ls, red);
   const StreamLayout lv = a.lay[sv];
   const int n_used = lv.n2 + lv.n1;
-  for (int e = tid; e < n_used; e += kThreads) {
+  for (int e = tid; e < n_used; e += kCThreads) {
     float acc = 0.0f;
-    for (int s = 0; s < a.n_splits; ++s) acc += src[s * stride + e] * exp2f(src[s * stride + a.n_entries] - m);
+    for (int s = 0; s < a.n_splits; ++s) acc = fmaf(part[s * stride + e], wsp[s], acc);
     oe[e] = acc;
   }
   __syncthreads();
-  {
+  if (tid == 0) {
+    lsum[0] = red[0][0] + red[0][1];
+    lsum[1] = red[1][0] + red[1][1];
+  }
+  __syncthreads();
+  if (tid < D) {
     const int c = tid;
     const short* ce = a.chan_ent + (static_cast<size_t>(sv) * D + c) * 8;
     const short* ent = a.entry + static_cast<size_t>(sv) * a.n_entries;
@@ -486,14 +558,20 @@ __global__ void __launch_bounds__(kThreads)
       const int e = ce[k];
       if (e >= 0) o += ldexpf(oe[e], ent[e] >> 8);
     }
-    o -= a.enc[sv * D + c].off * ls[1];
-    ohat[c] = o * a.f[sv * D + c] / ls[0];
+    o -= a.enc[sv * D + c].off * lsum[1];
+    ohat[c] = o * a.f[sv * D + c] / lsum[0];
   }
   __syncthreads();
-  const float* ut = a.u32t + static_cast<size_t>(sv) * D * D;
-  float o = 0.0f;
-  for (int c = 0; c < D; ++c) o = fmaf(ut[c * D + tid], ohat[c], o);
-  a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = o;
+  {
+    // out[d] = sum_c U_V[d][c] ohat[c]; two threads per output dimension
+    const int d = tid & (D - 1), half = tid >> 7;
+    float o = 0.0f;
+#pragma unroll 16
+    for (int c = half * 64; c < half * 64 + 64; ++c) o = fmaf(ut_s[c * D + d], ohat[c], o);
+    if (half) oe[d] = o;
+    __syncthreads();
+    if (!half) a.out[(static_cast<size_t>(b) * a.n_q + j) * D + d] = o + oe[d];
+  }
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -729,17 +807,24 @@ __global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, c
   }
 }
 
-template <int NTW>
-cudaError_t launch_split_ntw(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
+template <int WPW, int GP>
+cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
   static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
   if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<NTW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<WPW, GP>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  aatc_decode_split_kernel<NTW><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
+  aatc_decode_split_kernel<WPW, GP><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
   return cudaGetLastError();
+}
+
+template <int GP>
+cudaError_t launch_split_g(const DecodeArgs& a, int batch, int wpw, size_t smem, cudaStream_t st) {
+  if (wpw <= 3) return launch_split_t<3, GP>(a, batch, smem, st);
+  if (wpw <= 4) return launch_split_t<4, GP>(a, batch, smem, st);
+  return launch_split_t<8, GP>(a, batch, smem, st);
 }
 
 template <int GP>
@@ -786,24 +871,38 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_entries = plan.n_entries;
   a.n_splits = sp.n_splits;
   a.split_len = sp.split_len;
-  // largest key k-step count and value n-tile count over the layer's streams
-  int n_ks = 1, n_nt = 1;
+  // largest key k-step count and value word count over the layer's streams
+  int n_ks = 1, nw_v = 1;
   for (int h = 0; h < a.n_kv; ++h) {
     const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
     const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
     n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
-    n_nt = std::max(n_nt, 2 * (lv.n2 / 16) + 4 * ((lv.n1 + 31) / 32));
+    nw_v = std::max(nw_v, lv.n2 / 16 + (lv.n1 + 31) / 32);
   }
+  const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
+  a.pstride = wsl.pstride;
+  a.ks_stride = wsl.ks_stride;
+  a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
+  a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
+  aatc_decode_query_kernel<<<dim3(a.n_kv, batch), kQThreads, 0, st>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
   const SplitLayout L(n_ks, plan.n_words);
   const size_t smem = 4 * static_cast<size_t>(L.n_words_total);
-  const int ntw = (n_nt + kWarps - 1) / kWarps;
-  cudaError_t e;
-  if (ntw <= 8) e = launch_split_ntw<8>(a, batch, smem, st);
-  else if (ntw <= 16) e = launch_split_ntw<16>(a, batch, smem, st);
-  else e = launch_split_ntw<32>(a, batch, smem, st);
+  const int wpw = (nw_v + kWarps - 1) / kWarps;
+  if (wpw > 8) return cudaErrorNotSupported;
+  e = a.group <= 4 ? launch_split_g<4>(a, batch, wpw, smem, st) : launch_split_g<8>(a, batch, wpw, smem, st);
   if (e != cudaSuccess) return e;
-  const size_t csmem = 4 * static_cast<size_t>(plan.n_entries + D);
-  aatc_decode_combine_kernel<<<dim3(a.n_q, batch), kThreads, csmem, st>>>(a);
+  const size_t csmem =
+      4 * (static_cast<size_t>(a.n_splits) * a.pstride + ((a.n_splits + 3) & ~3) + plan.n_entries + D + D * D);
+  static size_t csmem_set = 0;
+  if (csmem > 48 * 1024 && csmem > csmem_set) {
+    e = cudaFuncSetAttribute(aatc_decode_combine_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(csmem));
+    if (e != cudaSuccess) return e;
+    csmem_set = csmem;
+  }
+  aatc_decode_combine_kernel<<<dim3(a.n_q, batch), kCThreads, csmem, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -869,7 +968,8 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(cache) & 15u) != 0) return AATC_ERR_INVALID_ARG;
   const DecodeSplit sp = decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (decode_workspace(batch, plan->dims.n_q_heads, plan->n_entries, sp) > AATC_NOALLOC_SCRATCH_BYTES)
+  if (decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries, plan->n_words, sp) >
+      AATC_NOALLOC_SCRATCH_BYTES)
     return AATC_ERR_WORKSPACE;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
