@@ -311,22 +311,21 @@ def unpack_records(words: np.ndarray, bits: np.ndarray) -> np.ndarray:
     return np.where(b[None, :] > 0, u.astype(np.int64) - off[None, :], 0)
 
 
-def value_lane_of(token_in_tile: int) -> tuple:
-    """Values are stored pair-interleaved.  In each 16-token group, tokens i and i+8 form a
-    pair; the pair's two records are stored as two words per record word: (low halves of
-    both) and (high halves of both), the first token's half in the low 16 bits.  Returns
-    (lane holding this token's low halves, lane holding its high halves, half index 0/1)."""
-    g, j = divmod(token_in_tile, 16)
-    i, second = j % 8, j >= 8
-    q, r = i % 4, i // 4                 # pairs i and i+4 share a 4-lane block
-    base = 16 * g + 4 * q + 2 * r
-    return base, base + 1, int(second)
+QUARTER_POS = (0, 2, 1, 3)      # slot position of byte-quarter r inside a value slot block
+
+
+def value_slot_of(token_in_tile: int, quarter: int) -> tuple:
+    """Values are stored quad-interleaved: tokens 4Q..4Q+3 of a tile share the four slots
+    4Q..4Q+3 of every record word; slot 4Q + QUARTER_POS[r] holds byte-quarter r (bits
+    8r..8r+7) of the four tokens' words, token 4Q + i in byte i.  Returns (slot, byte)."""
+    q, i = divmod(token_in_tile, 4)
+    return 4 * q + QUARTER_POS[quarter], i
 
 
 def cache_geometry(batch: int, n_kv_heads: int, max_tokens: int, n_words: int) -> dict:
     """Per-layer packed cache: uint32 words [batch][H_kv][2][n_tiles][W][128], then fp32 alpha
     [batch][H_kv][2][n_tiles*128].  Keys: token t of a sequence sits in tile t // 128, lane
-    t % 128.  Values: lanes as :func:`value_lane_of` says."""
+    t % 128.  Values: slots as :func:`value_slot_of` says."""
     n_tiles = (max_tokens + TILE - 1) // TILE
     n_word_elems = batch * n_kv_heads * 2 * n_tiles * n_words * TILE
     n_alpha = batch * n_kv_heads * 2 * n_tiles * TILE
@@ -346,12 +345,13 @@ def cache_records(cache_u32: np.ndarray, batch: int, n_kv_heads: int, max_tokens
     if kind == 0:
         rec = words[b, head, kind][t // TILE, :, t % TILE]        # (n, W)
     else:
-        lanes = np.array([value_lane_of(int(x)) for x in t % TILE])
-        lo = words[b, head, kind][t // TILE, :, lanes[:, 0]].astype(np.uint64)
-        hi = words[b, head, kind][t // TILE, :, lanes[:, 1]].astype(np.uint64)
-        sel = lanes[:, 2][:, None].astype(np.uint64) * np.uint64(16)
-        m16 = np.uint64(0xFFFF)
-        rec = (((lo >> sel) & m16) | (((hi >> sel) & m16) << np.uint64(16))).astype(np.uint32)
+        rec = np.zeros((n, n_words), dtype=np.uint64)
+        for r in range(4):
+            slots = np.array([value_slot_of(int(x), r)[0] for x in t % TILE])
+            byte = (t % TILE) % 4
+            w = words[b, head, kind][t // TILE, :, slots].astype(np.uint64)      # (n, W)
+            rec |= ((w >> (8 * byte[:, None]).astype(np.uint64)) & np.uint64(0xFF)) << np.uint64(8 * r)
+        rec = rec.astype(np.uint32)
     return rec, alpha[b, head, kind, t0:t0 + n]
 
 
@@ -369,13 +369,13 @@ def cache_image(records_k, records_v, alpha_k, alpha_v, batch, n_kv_heads, max_t
                 words[b, h, 0, t // TILE, :, t % TILE] = rk[t]
             rv = records_v[b][h]
             for t in range(rv.shape[0]):
-                lo, hi, half = value_lane_of(t % TILE)
                 for w in range(n_words):
                     x = int(rv[t, w])
-                    for lane, part in ((lo, x & 0xFFFF), (hi, x >> 16)):
-                        cur = int(words[b, h, 1, t // TILE, w, lane])
-                        cur &= ~(0xFFFF << (16 * half)) & 0xFFFFFFFF
-                        words[b, h, 1, t // TILE, w, lane] = cur | (part << (16 * half))
+                    for r in range(4):
+                        slot, byte = value_slot_of(t % TILE, r)
+                        cur = int(words[b, h, 1, t // TILE, w, slot])
+                        cur = (cur & ~(0xFF << (8 * byte))) | (((x >> (8 * r)) & 0xFF) << (8 * byte))
+                        words[b, h, 1, t // TILE, w, slot] = cur
             alpha[b, h, 0, :rk.shape[0]] = alpha_k[b][h]
             alpha[b, h, 1, :rv.shape[0]] = alpha_v[b][h]
     return np.concatenate([words.reshape(-1), alpha.reshape(-1).view(np.uint32)])

@@ -101,18 +101,19 @@ inline CacheGeom cache_geom(int batch, int n_kv, int max_tokens, int n_words) {
 }
 
 struct DecodeSplit {
-  int n_splits;
-  int split_len;          // tokens per split, a multiple of TILE
+  int n_splits;           // splits per (sequence, kv-head); split s covers tiles [s T / n, (s+1) T / n)
+  int split_len;          // tokens of the longest split, a multiple of TILE
 };
 
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
-// Decode workspace: split partials per (sequence, query head, split) -- n_entries value sums,
-// then m, l, S', padded to a multiple of 4 floats -- followed by the per-call score A fragments
-// per (sequence, kv-head) (up to 2 W k-steps x 32 lanes x 16 B) and their offset corrections.
+// Decode workspace: split partials per (sequence, query head, split) -- 128 channel sums, then
+// m, l, padded to a multiple of 4 floats -- followed by the per-call score A fragments per
+// (sequence, kv-head) (up to 2 W k-steps x 32 lanes x 16 B), their offset corrections and score
+// scales, and one finished-split counter per (sequence, kv-head).
 struct DecodeWs {
   int pstride;            // floats per partial
   int ks_stride;          // uint4 per (sequence, kv-head) fragment block
-  size_t qfrag_off, qcorr_off, bytes;
+  size_t qfrag_off, qcorr_off, cnt_off, bytes;
 };
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
 size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);

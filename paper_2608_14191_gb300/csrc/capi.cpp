@@ -41,18 +41,20 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 namespace aatc {
 
-constexpr long kMaxSplits = 96;   // the combine stages every split's partial in shared memory
-
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
-  const int tiles = (n_ctx + TILE - 1) / TILE;
+  // About four CTAs per SM in a single wave: n_splits per (sequence, kv-head), with split s
+  // covering tiles [s T / n_splits, (s + 1) T / n_splits) so split lengths differ by at most one
+  // tile and every SM gets nearly the same number of tiles.  A split holds at most 16 tiles
+  // (its scores are kept in shared memory).
+  const long tiles = (n_ctx + TILE - 1) / TILE;
   const long units = static_cast<long>(batch) * n_kv;
-  const long target = 4L * std::max(1, num_sms);                 // ~4 CTAs per SM
-  long per = (static_cast<long>(tiles) * units + target - 1) / target;
-  per = std::max(per, (static_cast<long>(tiles) + kMaxSplits - 1) / kMaxSplits);   // bounded combine
-  per = std::max(1L, per);
+  const long target = 4L * std::max(1, num_sms);
+  long n = (target + units / 2) / units;
+  n = std::max(n, (tiles + 15) / 16);
+  n = std::max(1L, std::min(n, tiles));
   DecodeSplit sp;
-  sp.n_splits = static_cast<int>((tiles + per - 1) / per);
-  sp.split_len = static_cast<int>(per) * TILE;
+  sp.n_splits = static_cast<int>(n);
+  sp.split_len = static_cast<int>((tiles + n - 1) / n) * TILE;   // longest split
   return sp;
 }
 
@@ -62,11 +64,12 @@ aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
 
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
   DecodeWs w;
-  w.pstride = (n_entries + 3 + 3) & ~3;
-  w.ks_stride = 2 * n_words * 32;
+  w.pstride = D + 4;                              // o_c per channel, then m, l (padded)
+  w.ks_stride = 2 * n_words * 32;                 // >= k32-steps x 2 query passes x 32 lanes
   w.qfrag_off = align_up(static_cast<size_t>(batch) * n_q * sp.n_splits * w.pstride * sizeof(float), 256);
   w.qcorr_off = align_up(w.qfrag_off + static_cast<size_t>(batch) * n_kv * w.ks_stride * 16, 256);
-  w.bytes = w.qcorr_off + static_cast<size_t>(batch) * n_kv * MAX_GROUP * sizeof(float);
+  w.cnt_off = align_up(w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float), 256);
+  w.bytes = w.cnt_off + static_cast<size_t>(batch) * n_kv * sizeof(int);
   return w;
 }
 

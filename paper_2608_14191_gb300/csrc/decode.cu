@@ -2,20 +2,26 @@
 // uncompressed bf16 reference decode (Def. sdpa with one query row; Algorithm 1
 // "Reconstruct", "softmax", "Output" lines, computed without rebuilding the keys).
 //
-// Split-K over the context (flash-decoding): one CTA per (split, kv-head, sequence) computes,
-// for the G query heads of its GQA group,
-//   phase 1  scores s_{g,t} = alpha^K_t * sum_c q'_{g,c} code^K_{t,c}   (thread = token),
-//            with q' = (U_K^T q) * f^K * log2(e) / sqrt(128) folded once per CTA,
-//   phase 2  split max m_g, p = 2^(s - m_g), l_g = sum p, P' = p * alpha^V_t,
-//   phase 3  acc_{g,c} = sum_t P'_{g,t} code^V_{t,c}   (thread = 4 channels x 1/4 of the tokens),
-// and writes (acc, m, l).  The combine kernel merges the splits by log-sum-exp, applies f^V and
-// the one inverse value transform out = U_V o_hat.
+// Three launches per call (flash-decoding split over the context):
+//   query    per (sequence, kv-head): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the G query heads
+//            of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1), and q' in
+//            24-bit fixed point as int8 tensor-core fragments;
+//   split    per (split, kv-head, sequence): pass 1 scores
+//            s_{g,t} = alpha^K_t (sigma_g sum_e Q_{g,e} digit_{t,e} - C_g) on the int8 tensor
+//            cores over the packed digits; split max m_g; pass 2 p = 2^(s - m_g),
+//            P' = p alpha^V_t in 24-bit fixed point, value entry sums sum_t P'_{g,t} digit_{t,e}
+//            on the tensor cores with exact int32 accumulation over the whole split;
+//   combine  per (sequence, query head): log-sum-exp merge of the splits, record entries back to
+//            channel sums with the offset correction, f^V / l, and out = U_V o_hat.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include <algorithm>
 #include <mutex>
 
 #include "aatc_internal.h"
+#include "ptx.cuh"
 
 namespace aatc {
 namespace {
@@ -58,21 +64,12 @@ __device__ __forceinline__ void block_reduce(float (&v)[GP], float* scratch /* [
 }
 
 // ---------------------------------------------------------------- packed-cache decode
-//
-// Tensor-core formulation (mma.sync m16n8k16, fp16 operands, fp32 accumulate):
-//   scores:  A = folded query q'_c 2^shift per record entry, split hi (rows g) / lo (rows g+8),
-//            B = record digits / bits of 8 tokens (each fragment register: one shift + mask of a
-//            packed word, then subtracting the 1024 magic), accumulated over the record words.
-//   values:  A = probabilities P' = p alpha^V split hi / lo, B = value digits / bits of 16 tokens
-//            from the pair-interleaved value words, one n-tile per 8 record entries.
-// Token order inside a 16-token group g16 (both products): k = 2i <-> token i, k = 2i+1 <->
-// token i+8 for i < 8.  Score n-tile A holds k 0..7, n-tile B k 8..15.
 
 struct DecodeArgs {
   const uint32_t* words;   // cache word region (this layer)
   const float* alpha;      // cache alpha region
   const __nv_bfloat16* q;  // [batch][HQ][128]
-  float* ws;               // [batch][HQ][n_splits][n_entries + 3]
+  float* ws;               // [batch][HQ][n_splits][pstride]: o_c (128 channels), then m, l
   float* out;              // [batch][HQ][128]
   const float* u32;        // plan: [S][128 dim][128 ch]
   const float* u32t;       // plan: [S][128 ch][128 dim]
@@ -83,30 +80,10 @@ struct DecodeArgs {
   const short* chan_ent;   // plan: [S][128][8]
   int* err;
   uint4* qfrag;            // workspace: score A fragments [batch][n_kv][ks_stride]
-  float* qcorr;            // workspace: offset corrections [batch][n_kv][8]
+  float* qcorr;            // workspace: [batch][n_kv][16]: offset corrections C_g, score scales
+  int* cnt;                // workspace: [batch][n_kv] finished-split counters
   int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len, ks_stride, pstride;
 };
-
-__device__ __forceinline__ uint32_t hsub_magic(uint32_t x) {
-  // x holds two 16-bit fields (1024 + v) as fp16 bit patterns; returns the fp16 pair (v_lo, v_hi)
-  uint32_t r;
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(x), "r"(0x64006400u));
-  return r;
-}
-
-__device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
-  uint32_t r;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-
-__device__ __forceinline__ void mma_16816(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
-}
 
 // 2^x with the hardware approximation (relative error ~2^-22; -inf -> 0)
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -115,126 +92,205 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return r;
 }
 
-// fp32 -> (hi, lo) fp16 pair with hi + lo = v to ~2^-22 relative
-__device__ __forceinline__ void split_hi_lo(float v, float& hi, float& lo) {
-  hi = __half2float(__float2half_rn(v));
-  lo = v - hi;
-}
+__device__ __forceinline__ float pow2i(int e) { return __int_as_float((127 + e) << 23); }   // 2^e, |e| < 127
 
-constexpr int kGroups = TILE / 16;        // 16-token groups per tile
 constexpr int kWarps = kThreads / 32;
 
-// shared-memory carve-up of the split kernel (32-bit words)
-struct SplitLayout {
-  int cg, red, run, afrag, pfrag, kw, vw, ak, av, n_words_total;
-  __host__ __device__ SplitLayout(int n_ks, int W) {
-    int o = 0;
-    cg = o;    o += MAX_GROUP;                 // offset corrections
-    red = o;   o += 3 * kWarps * MAX_GROUP;    // per-warp max / sum p / sum P'
-    run = o;   o += 3 * MAX_GROUP;             // running m, l, S'
-    o = (o + 3) & ~3;
-    afrag = o; o += n_ks * 32 * 4;             // uint4 per (k-step, lane)
-    pfrag = o; o += kGroups * MAX_GROUP * 16;  // half2 (hi, lo) of P' per (group, query, slot)
-    kw = o;    o += 2 * W * TILE;              // two stages of key words
-    vw = o;    o += 2 * W * TILE;              // two stages of value words
-    ak = o;    o += 2 * TILE;
-    av = o;    o += 2 * TILE;
-    n_words_total = o;
-  }
-};
+// Tensor-core formulation: mma.sync m16n8k32 with e4m3 operands and f32 accumulation.
+//  * A packed digit masked into a byte (0..3, or 0..1 for a bit) IS an e4m3 number: the subnormal
+//    digit x 2^-9, so B fragments are one shift and one mask of a record word, four digits each.
+//  * The other operand (folded query, or probability P' = p alpha^V) is split into four e4m3 limbs
+//    with x_0 = x, l_k = rn(x_k), x_{k+1} = 16 (x_k - l_k), so x = sum_k l_k 16^-k + x_4 2^-16:
+//    each limb keeps 4 significant bits, four of them ~16 bits of x, down to |x| ~ 2^-18 of the
+//    largest (|x| <= 256).  Rows 4k + i of A hold limb k of query 4P + i, so lane (g, t) gets
+//    limbs 0 (c0, c1) and 2 (c2, c3) of query g < 4 and lane g + 4 limbs 1 and 3; a query's
+//    value is the 16^-k weighted sum over both lanes.
+//  * The products and their f32 sums are exact for these magnitudes, which was checked on the
+//    hardware (subnormal x subnormal, cancellation of the largest terms).
+//   scores:  B = record digits: a D2 k32-step covers two record words (b0 from word 2i, b1 from
+//            2i+1, byte j of lane t = field t + 4j), a D1 step one word (fields t + 8j and t + 4 + 8j).
+//   values:  B = value digits of four tokens from the quad-interleaved value words; one n-tile per
+//            8 record entries (= one byte-quarter of the record word).
+__device__ __forceinline__ void mma_e4m3(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
+}
 
-// Per call, per (sequence, kv-head): folded query q'_{g,c} = (U_K^T q_g)_c f_c log2(e)/sqrt(128),
-// the offset corrections C_g = sum_c q'_{g,c} 2^(b_c-1), and the score A fragments: for each
-// k-step and lane, slot k -> record entry (c, shift) -> q'_c 2^shift as fp16 hi (rows g) / lo
-// (rows g+8).  512 threads: four quarters of the input dimension per channel.
+// next e4m3 limb of x (returned byte); x becomes 16 (x - limb)
+__device__ __forceinline__ uint32_t e4m3_limb(float& x) {
+  const __nv_fp8_storage_t b = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
+  x = 16.0f * (x - __half2float(__half(__nv_cvt_fp8_to_halfraw(b, __NV_E4M3))));
+  return b;
+}
+// the same for two values at once (x.x -> low byte)
+__device__ __forceinline__ uint32_t e4m3_limb2(float2& x) {
+  const __nv_fp8x2_storage_t b = __nv_cvt_float2_to_fp8x2(x, __NV_SATFINITE, __NV_E4M3);
+  const float2 v = __half22float2(__half2(__nv_cvt_fp8x2_to_halfraw2(b, __NV_E4M3)));
+  x.x = 16.0f * (x.x - v.x);
+  x.y = 16.0f * (x.y - v.y);
+  return b;
+}
+// a query's value from the accumulators of its two lanes (limbs 0, 2 in lane g < 4; 1, 3 in g + 4)
+__device__ __forceinline__ float2 limb_sum(const float (&c)[4], int g) {
+  const float w0 = g < 4 ? 1.0f : 0.0625f, w2 = g < 4 ? 0.00390625f : 0.000244140625f;
+  float v0 = fmaf(c[2], w2, c[0] * w0), v1 = fmaf(c[3], w2, c[1] * w0);
+  v0 += __shfl_down_sync(0xffffffffu, v0, 16);
+  v1 += __shfl_down_sync(0xffffffffu, v1, 16);
+  return make_float2(v0, v1);
+}
+
 constexpr int kQThreads = 512;
+constexpr int kMaxEntries = 32 * 32;   // 8 bits x 128 channels
 
+// Per call, per (sequence, kv-head, query slot): folded query q'_c = (U_K^T q)_c f_c log2(e)/sqrt(128),
+// its offset correction C = sum_c q'_c 2^(b_c-1), the score scale, and the rows of the score A
+// fragments that hold this query (four e4m3 limbs of q'_c 2^shift / sigma per record entry).
+// Slots G..4P-1 write zero rows.  Slot 0 also clears the finished-split counter of its head.
 __global__ void __launch_bounds__(kQThreads)
     aatc_decode_query_kernel(const DecodeArgs a) {
-  __shared__ float qf[MAX_GROUP][D];
-  __shared__ float part[4][MAX_GROUP][D];
-  __shared__ float qc[MAX_GROUP][D];
-  __shared__ float credw[kQThreads / 32][MAX_GROUP];
-  const int head = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  const int G = a.group;
+  __shared__ float qv[D];
+  __shared__ float part[4][D];
+  __shared__ float xq[D];
+  __shared__ float red[2][D / 32];
+  __shared__ uint8_t lb[4][kMaxEntries];
+  const int head = blockIdx.x, b = blockIdx.y, slot = blockIdx.z, tid = threadIdx.x;
+  const int G = a.group, NP = (G + 3) / 4;
+  const bool real = slot < G;
   const int sk = (a.layer * a.n_kv + head) * 2;
-  for (int i = tid; i < MAX_GROUP * D; i += kQThreads) {
-    const int gq = i / D, d = i % D;
-    qf[gq][d] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + d]) : 0.0f;
+  ptx::grid_launch_dependents();
+  if (slot == 0 && tid == 0) a.cnt[b * a.n_kv + head] = 0;
+  // every global input is requested up front (one memory round trip)
+  const int c = tid & (D - 1), qd = tid >> 7;
+  const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
+  const short ce0 = tid < a.n_entries ? ent[tid] : 0;
+  const short ce1 = tid + kQThreads < a.n_entries ? ent[tid + kQThreads] : 0;
+  const StreamLayout lk = a.lay[sk];
+  float qraw = 0.0f, fk = 0.0f, off = 0.0f;
+  if (tid < D) {
+    if (real) qraw = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + slot) * D + tid]);
+    fk = a.f[sk * D + c];
+    off = a.enc[sk * D + c].off;                                          // 2^(b_c - 1), 0 if b_c = 0
   }
-  __syncthreads();
+  float u[32];
   {
-    const int c = tid & (D - 1), qd = tid >> 7;
+    // thread (channel c, quarter qd of the dimensions)
     const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(32 * qd) * D + c;
-    float u[32];
 #pragma unroll
     for (int d = 0; d < 32; ++d) u[d] = uk[d * D];
-    float acc[MAX_GROUP];
+  }
+  if (tid < D) qv[tid] = qraw;
+  __syncthreads();
+  {
+    float acc = 0.0f;
 #pragma unroll
-    for (int gq = 0; gq < MAX_GROUP; ++gq) {
-      acc[gq] = 0.0f;
-#pragma unroll
-      for (int d = 0; d < 32; ++d) acc[gq] = fmaf(u[d], qf[gq][32 * qd + d], acc[gq]);
-      part[qd][gq][c] = acc[gq];
-    }
+    for (int d = 0; d < 32; ++d) acc = fmaf(u[d], qv[32 * qd + d], acc);
+    part[qd][c] = acc;
   }
   __syncthreads();
   if (tid < D) {
-    const int c = tid;
-    const float fk = a.f[sk * D + c] * (kLog2e * 0.08838834764831845f);   // 1/sqrt(128)
-    const float off = a.enc[sk * D + c].off;
-    float cr[MAX_GROUP];
+    const float x = (part[0][c] + part[1][c] + part[2][c] + part[3][c]) * fk * (kLog2e * 0.08838834764831845f);
+    float cr = x * off;
+    float mx = fabsf(x) * off;                                             // largest |coefficient| of c
 #pragma unroll
-    for (int gq = 0; gq < MAX_GROUP; ++gq) {
-      const float v = (part[0][gq][c] + part[1][gq][c] + part[2][gq][c] + part[3][gq][c]) * fk;
-      qc[gq][c] = v;
-      cr[gq] = v * off;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) cr[gq] += __shfl_xor_sync(0xffffffffu, cr[gq], o);
+    for (int o = 16; o > 0; o >>= 1) {
+      cr += __shfl_xor_sync(0xffffffffu, cr, o);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     }
-    if ((tid & 31) == 0)
-#pragma unroll
-      for (int gq = 0; gq < MAX_GROUP; ++gq) credw[tid >> 5][gq] = cr[gq];
+    if ((tid & 31) == 0) {
+      red[0][tid >> 5] = cr;
+      red[1][tid >> 5] = mx;
+    }
+    xq[c] = x;
   }
   __syncthreads();
-  if (tid < MAX_GROUP)
-    a.qcorr[(static_cast<size_t>(b) * a.n_kv + head) * MAX_GROUP + tid] =
-        credw[0][tid] + credw[1][tid] + credw[2][tid] + credw[3][tid];
-  const StreamLayout lk = a.lay[sk];
-  const int n2w = lk.n2 / 16, n_ks = n2w + 2 * ((lk.n1 + 31) / 32);
-  const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
-  uint4* dst = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
-  for (int i = tid; i < n_ks * 32; i += kQThreads) {
-    const int ks = i >> 5, ln = i & 31, gq = ln >> 2, tq = ln & 3;
-    int fld[4];                                   // fields for k = 2t, 2t+1, 2t+8, 2t+9
-    int ebase;
-    if (ks < n2w) {
-      ebase = 16 * ks;
-      fld[0] = tq; fld[1] = tq + 8; fld[2] = tq + 4; fld[3] = tq + 12;
-    } else {
-      const int r = ks - n2w, h8 = 8 * (r & 1);
-      ebase = lk.n2 + 32 * (r >> 1);
-      fld[0] = tq + h8; fld[1] = tq + 16 + h8; fld[2] = tq + 4 + h8; fld[3] = tq + 20 + h8;
+  const float C = red[0][0] + red[0][1] + red[0][2] + red[0][3];
+  const float m = fmaxf(fmaxf(red[1][0], red[1][1]), fmaxf(red[1][2], red[1][3]));
+  const float inv = m > 0.0f ? 256.0f / m : 0.0f;                        // coefficients to |.| <= 256
+  const int n_used = lk.n2 + lk.n1;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int e = tid + h * kQThreads;
+    if (e < n_used) {
+      const int ce = h ? ce1 : ce0;
+      float v = xq[ce & 0xFF] * inv * pow2i(ce >> 8);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) lb[k][e] = static_cast<uint8_t>(e4m3_limb(v));
     }
-    float hi[4], lo[4];
+  }
+  __syncthreads();
+  const int n2w = lk.n2 / 16, n2s = (n2w + 1) / 2, n1w = (lk.n1 + 31) / 32;
+  const int n_s = n2s + n1w;
+  const int P = slot >> 2, qq = slot & 3;
+  uint32_t* dst = reinterpret_cast<uint32_t*>(a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride);
+  for (int i = tid; i < n_s * 32; i += kQThreads) {
+    const int st = i >> 5, w = i & 31;
+    const int g = (w >> 4) ? 4 + qq : qq, t = (w >> 2) & 3, rr = w & 3;
+    const int row = g + 8 * (rr & 1), limb = row >> 2, khalf = rr >> 1;
+    uint32_t r = 0;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int e = ebase + fld[j];
-      const int ce = (e < lk.n2 + lk.n1) ? ent[e] : -1;
-      const float coef = (ce >= 0 && gq < G) ? ldexpf(qc[gq][ce & 0xFF], ce >> 8) : 0.0f;
-      split_hi_lo(coef, hi[j], lo[j]);
+      int e = -1;
+      if (st < n2s) {
+        const int wd = 2 * st + khalf;
+        if (wd < n2w) e = 16 * wd + t + 4 * j;
+      } else {
+        const int fld = t + 8 * j + 4 * khalf;
+        if (32 * (st - n2s) + fld < lk.n1) e = lk.n2 + 32 * (st - n2s) + fld;
+      }
+      if (e >= 0 && real) r |= static_cast<uint32_t>(lb[limb][e]) << (8 * j);
     }
-    dst[i] = make_uint4(pack_half2(hi[0], hi[1]), pack_half2(lo[0], lo[1]), pack_half2(hi[2], hi[3]),
-                        pack_half2(lo[2], lo[3]));
+    dst[((st * NP + P) * 32 + 4 * g + t) * 4 + rr] = r;
+  }
+  if (tid == 0) {
+    float* qc = a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP;
+    qc[slot] = real ? C : 0.0f;
+    qc[MAX_GROUP + slot] = m > 0.0f ? m * (512.0f / 256.0f) : 0.0f;       // limb units x digit 2^9
   }
 }
 
-// Value n-tiles of one record word: a D2 word gives two (fields 0-7 from the low-half lane,
-// fields 8-15 from the high-half lane, shift 2g), a D1 word four (low/high lane x shift g, g+8).
-template <int WPW, int GP>
+constexpr int kStages = 4;                  // ring of record-word tiles (keys, then values)
+
+__host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
+
+// shared-memory carve-up of the split kernel (byte offsets)
+struct SplitSmem {
+  int bars, qcg, red, cetab, etab, afrag, ak, av, sbuf, pq, ring, total, sb_stride;
+  __host__ __device__ SplitSmem(int n_steps, int np, int split_len, int W, int n_entries, int n_splits) {
+    int o = 0;
+    bars = o;  o = align16(o + 8 * (kStages + 1));  // ring barriers, then the prologue barrier
+    qcg = o;   o += 2 * MAX_GROUP * 4;              // offset corrections, score scales
+    red = o;   o += 4 * kWarps * MAX_GROUP * 4;     // reductions; per-query m, l, S', split max
+    cetab = o; o += D * 8 * 2;                      // record entries of each value channel
+    etab = o;  o = align16(o + n_entries * 2);      // value entry table (channel | shift << 8)
+    afrag = o; o += n_steps * np * 32 * 16;         // score A fragments per (k-step, pass, lane)
+    ak = o;    o += split_len * 4;                  // alpha^K, alpha^V of the split
+    av = o;    o += split_len * 4;
+    sb_stride = split_len + 8;                      // padded: query rows fall in different banks
+    sbuf = o;  o += 4 * np * sb_stride * 4;         // scores of the split
+    pq = o;    o += 4 * np * 32 * 16;               // P' limb fragments of one tile
+    ring = o;                                       // after the last tile: entry sums, merge scratch
+    const int merge = 4 * (4 * np * ((n_splits + 3) & ~3) + 5 * 4 * np * D + 4 * np);
+    o += align16(max(kStages * W * TILE * 4, merge));
+    total = o;
+  }
+};
+
+// One CTA per (split, kv-head, sequence).  The split's record words stream through a ring of
+// kStages tiles filled by bulk copies (keys of all its tiles, then values); alpha^K, alpha^V, the
+// query fragments and the value entry tables arrive by bulk copy in the prologue.
+// Pass 1: scores of the split; pass 2: P' and the value entry sums; then the entry sums become
+// channel sums o_c = sum_e 2^shift O_e - 2^(b_c-1) S' (the Eq. 12 offset, folded after the
+// product), written with m and l.  The CTA that finishes its head's last split merges all of
+// them (log-sum-exp), scales by f^V / l and applies U_V.
+template <int WPW, int NP>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
-  extern __shared__ __align__(16) uint32_t smw[];
+  extern __shared__ __align__(128) unsigned char smb[];
+  __shared__ int s_last;
+  __shared__ int s_abort;
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t = lane & 3;                       // mma fragment coordinates
@@ -242,336 +298,431 @@ __global__ void __launch_bounds__(kThreads)
   const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;   // key / value streams
   const StreamLayout lk = a.lay[sk], lv = a.lay[sv];
   const int W = a.n_words;
-  const int n2w_k = lk.n2 / 16, n1w_k = (lk.n1 + 31) / 32;
-  const int n_ks = n2w_k + 2 * n1w_k;
+  const int n2w_k = lk.n2 / 16, n2s_k = (n2w_k + 1) / 2, n1w_k = (lk.n1 + 31) / 32;
+  const int n_s = n2s_k + n1w_k;
   const int n2w_v = lv.n2 / 16, nw_v = n2w_v + (lv.n1 + 31) / 32;
-  const SplitLayout L(n_ks, W);
-  float* cg = reinterpret_cast<float*>(smw + L.cg);
-  float* red = reinterpret_cast<float*>(smw + L.red);          // [3][kWarps][8]
-  float* run = reinterpret_cast<float*>(smw + L.run);          // [3][8]: m, l, S'
-  uint4* afrag = reinterpret_cast<uint4*>(smw + L.afrag);
-  uint32_t* pfrag = smw + L.pfrag;
-  uint32_t* kw = smw + L.kw;
-  uint32_t* vw = smw + L.vw;
-  float* ak = reinterpret_cast<float*>(smw + L.ak);
-  float* av = reinterpret_cast<float*>(smw + L.av);
+  const SplitSmem L(n_s, NP, a.split_len, W, a.n_entries, a.n_splits);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smb + L.bars);
+  uint64_t* pro = full + kStages;
+  float* qcg = reinterpret_cast<float*>(smb + L.qcg);          // [0..7] C_g, [8..15] score scales
+  float* red = reinterpret_cast<float*>(smb + L.red);
+  const short* cetab = reinterpret_cast<const short*>(smb + L.cetab);
+  const short* etab = reinterpret_cast<const short*>(smb + L.etab);
+  uint4* afrag = reinterpret_cast<uint4*>(smb + L.afrag);
+  float* ak = reinterpret_cast<float*>(smb + L.ak);
+  float* av = reinterpret_cast<float*>(smb + L.av);
+  float* sbuf = reinterpret_cast<float*>(smb + L.sbuf);        // [4 NP][sb_stride]
+  uint4* pq = reinterpret_cast<uint4*>(smb + L.pq);            // [4 k32-steps][NP][32 lanes]
+  uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
+  const int sbs = L.sb_stride;
 
-  const int t_begin = split * a.split_len;
-  const int t_end = min(a.n_ctx, t_begin + a.split_len);
-  const int n_tiles_split = (t_end - t_begin + TILE - 1) / TILE;
+  const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
+  const int tile_lo = static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
+  const int tile_hi = static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
+  const int t_begin = tile_lo * TILE;
+  const int t_end = min(a.n_ctx, tile_hi * TILE);
+  const int n_tiles_split = tile_hi - tile_lo;
+  const int n_seq = 2 * n_tiles_split;                         // key tiles, then value tiles
   const int tile0 = t_begin / TILE;
+  const uint32_t tile_bytes = static_cast<uint32_t>(W) * TILE * 4;
   const size_t stream_words = static_cast<size_t>(a.n_tiles) * W * TILE;
   const size_t bk = (static_cast<size_t>(b) * a.n_kv + head) * 2;   // cache stream of the keys
   const uint32_t* kwords = a.words + bk * stream_words;
   const uint32_t* vwords = a.words + (bk + 1) * stream_words;
   const float* kalpha = a.alpha + bk * a.n_tiles * TILE;
   const float* valpha = a.alpha + (bk + 1) * a.n_tiles * TILE;
+  const float off_c = a.enc[sv * D + tid].off;                 // this thread's value channel
+  const float fv_c = a.f[sv * D + tid];
 
-  auto stage = [&](int tile, int buf) {
-    const int chunks = W * (TILE / 4);
-    const uint32_t* sk_ = kwords + static_cast<size_t>(tile) * W * TILE;
-    const uint32_t* sv_ = vwords + static_cast<size_t>(tile) * W * TILE;
-    for (int i = tid; i < chunks; i += kThreads) {
-      cp_async16(kw + buf * W * TILE + 4 * i, sk_ + 4 * i);
-      cp_async16(vw + buf * W * TILE + 4 * i, sv_ + 4 * i);
-    }
-    if (tid < TILE / 4) cp_async16(ak + buf * TILE + 4 * tid, kalpha + tile * TILE + 4 * tid);
-    else if (tid < TILE / 2) cp_async16(av + buf * TILE + 4 * (tid - TILE / 4), valpha + tile * TILE + 4 * (tid - TILE / 4));
-    cp_async_commit();
+  auto issue_tile = [&](int i) {
+    const int s = i % kStages;
+    const uint32_t* src = (i < n_tiles_split ? kwords : vwords) +
+                          static_cast<size_t>(tile0 + i % n_tiles_split) * W * TILE;
+    ptx::mbar_arrive_expect_tx(full + s, tile_bytes);
+    ptx::bulk_load(ring + s * W * TILE, src, tile_bytes, full + s);
   };
-  stage(tile0, 0);
-
-  // ---- prologue: score A fragments and offset corrections of this (sequence, kv-head), built
-  // once per call by aatc_decode_query_kernel
-  {
-    const uint4* qsrc = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
-    for (int i = tid; i < n_ks * 32; i += kThreads) cp_async16(afrag + i, qsrc + i);
-    cp_async_commit();
-    if (tid < MAX_GROUP) {
-      cg[tid] = a.qcorr[(static_cast<size_t>(b) * a.n_kv + head) * MAX_GROUP + tid];
-      run[tid] = -INFINITY;            // m
-      run[8 + tid] = 0.0f;             // l
-      run[16 + tid] = 0.0f;            // S'
+  auto wait_tile = [&](int i) {
+    if (!ptx::mbar_wait_bounded(full + i % kStages, (i / kStages) & 1, &s_abort)) {
+      s_abort = 1;
+      atomicOr(a.err, 2);
     }
-    for (int i = tid; i < kGroups * MAX_GROUP * 16; i += kThreads) pfrag[i] = 0u;   // rows g >= G stay 0
-    cp_async_wait_all();
-    __syncthreads();
+  };
+  if (tid == 0) {
+    s_abort = 0;
+    for (int s2 = 0; s2 <= kStages; ++s2) ptx::mbar_init(full + s2, 1);
+    ptx::fence_mbar_init();
+    // cache words and scales do not depend on the query kernel: start them first
+    for (int i = 0; i < min(kStages, n_seq); ++i) issue_tile(i);
+    const uint32_t abytes = static_cast<uint32_t>(n_tiles_split) * TILE * 4;
+    const uint32_t ebytes = static_cast<uint32_t>(align16(a.n_entries * 2));
+    const uint32_t fbytes = static_cast<uint32_t>(n_s) * NP * 32 * 16;
+    ptx::mbar_arrive_expect_tx(pro, 2 * abytes + D * 8 * 2 + ebytes + fbytes + 2 * MAX_GROUP * 4);
+    ptx::bulk_load(ak, kalpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
+    ptx::bulk_load(av, valpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
+    ptx::bulk_load(smb + L.cetab, a.chan_ent + static_cast<size_t>(sv) * D * 8, D * 8 * 2, pro);
+    ptx::bulk_load(smb + L.etab, a.entry + static_cast<size_t>(sv) * a.n_entries, ebytes, pro);
+    // the query kernel's fragments and corrections
+    ptx::grid_dependency_wait();
+    ptx::bulk_load(afrag, a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride, fbytes, pro);
+    ptx::bulk_load(qcg, a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP, 2 * MAX_GROUP * 4, pro);
+  }
+  __syncthreads();
+  if (!ptx::mbar_wait_bounded(pro, 0, &s_abort)) {
+    s_abort = 1;
+    atomicOr(a.err, 2);
   }
 
-  // value words of this warp (contiguous) and their n-tile accumulators
+  // ---- pass 1: scores; warp = 32 tokens of each tile as four n-tiles of 8
+  float mloc[NP];
+#pragma unroll
+  for (int p = 0; p < NP; ++p) mloc[p] = -INFINITY;
+  for (int ti = 0; ti < n_tiles_split; ++ti) {
+    wait_tile(ti);
+    const uint32_t* kt = ring + (ti % kStages) * W * TILE + 32 * warp + g;
+    float acc[4][NP][4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int p = 0; p < NP; ++p)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) acc[j][p][r] = 0.0f;
+    for (int st = 0; st < n2s_k; ++st) {
+      uint4 af[NP];
+#pragma unroll
+      for (int p = 0; p < NP; ++p) af[p] = afrag[(st * NP + p) * 32 + lane];
+      const uint32_t* w0 = kt + (2 * st) * TILE;
+      const uint32_t* w1 = kt + min(2 * st + 1, W - 1) * TILE;    // past D2: its A bytes are zero
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t b0 = (w0[8 * j] >> (2 * t)) & 0x03030303u;
+        const uint32_t b1 = (w1[8 * j] >> (2 * t)) & 0x03030303u;
+#pragma unroll
+        for (int p = 0; p < NP; ++p) mma_e4m3(acc[j][p], af[p], b0, b1);
+      }
+    }
+    for (int u = 0; u < n1w_k; ++u) {
+      uint4 af[NP];
+#pragma unroll
+      for (int p = 0; p < NP; ++p) af[p] = afrag[((n2s_k + u) * NP + p) * 32 + lane];
+      const uint32_t* w0 = kt + (n2w_k + u) * TILE;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t x = w0[8 * j];
+        const uint32_t b0 = (x >> t) & 0x01010101u;
+        const uint32_t b1 = (x >> (t + 4)) & 0x01010101u;
+#pragma unroll
+        for (int p = 0; p < NP; ++p) mma_e4m3(acc[j][p], af[p], b0, b1);
+      }
+    }
+    const int tbase = (tile0 + ti) * TILE;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int p = 0; p < NP; ++p) {
+        const float2 v = limb_sum(acc[j][p], g);
+        const float v0 = v.x, v1 = v.y;
+        const int q = 4 * p + g;
+        if (g < 4 && q < G) {
+          const float sg = qcg[MAX_GROUP + q], c0 = qcg[q];
+          const int tk = 32 * warp + 8 * j + 2 * t;
+          const float2 a2 = *reinterpret_cast<const float2*>(ak + ti * TILE + tk);
+          float s0 = a2.x * fmaf(v0, sg, -c0);
+          float s1 = a2.y * fmaf(v1, sg, -c0);
+          s0 = tbase + tk < t_end ? s0 : -INFINITY;
+          s1 = tbase + tk + 1 < t_end ? s1 : -INFINITY;
+          *reinterpret_cast<float2*>(sbuf + q * sbs + ti * TILE + tk) = make_float2(s0, s1);
+          mloc[p] = fmaxf(mloc[p], fmaxf(s0, s1));
+        }
+      }
+    __syncthreads();                                           // stage free: refill
+    if (tid == 0 && ti + kStages < n_seq) {
+      ptx::fence_proxy_async_smem();
+      issue_tile(ti + kStages);
+    }
+  }
+  // split max per query; largest alpha^V of the split (P' = p alpha^V is coded relative to it)
+  float amx = 0.0f;
+  for (int i = tid; i < t_end - t_begin; i += kThreads) amx = fmaxf(amx, av[i]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amx = fmaxf(amx, __shfl_xor_sync(0xffffffffu, amx, o));
+  if (lane == 0) red[3 * kWarps * MAX_GROUP + warp] = amx;
+#pragma unroll
+  for (int p = 0; p < NP; ++p) {
+    float m = mloc[p];
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+    if (t == 0 && g < 4) red[warp * MAX_GROUP + 4 * p + g] = m;
+  }
+  __syncthreads();
+  float* mqs = red + 2 * kWarps * MAX_GROUP + 3 * MAX_GROUP;  // [MAX_GROUP] split max per query
+  if (tid < 4 * NP)
+    mqs[tid] = fmaxf(fmaxf(red[0 * MAX_GROUP + tid], red[1 * MAX_GROUP + tid]),
+                     fmaxf(red[2 * MAX_GROUP + tid], red[3 * MAX_GROUP + tid]));
+  {
+    const float* am = red + 3 * kWarps * MAX_GROUP;
+    amx = fmaxf(fmaxf(am[0], am[1]), fmaxf(am[2], am[3]));
+  }
+  const float inv_p = amx > 0.0f ? 256.0f / amx : 0.0f;       // P' to |.| <= 256
+  const float val_scale = amx * (512.0f / 256.0f);             // limb units x digit 2^9
+  __syncthreads();                                             // split maxima visible to pass 2
+
+  // ---- pass 2: P' limbs (thread = 4 tokens x 1 query) and the value product over the split
   const int vw0 = warp * nw_v / kWarps, vw1 = (warp + 1) * nw_v / kWarps;
-  float acc[WPW][4][4];
+  float vacc[WPW][4][NP][4];
 #pragma unroll
   for (int i = 0; i < WPW; ++i)
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int r = 0; r < 4; ++r)
 #pragma unroll
-      for (int r = 0; r < 4; ++r) acc[i][q][r] = 0.0f;
-  const float c0 = cg[g];
-
-  for (int ti = 0; ti < n_tiles_split; ++ti) {
-    const int buf = ti & 1;
-    cp_async_wait_all();
-    __syncthreads();
-    if (ti + 1 < n_tiles_split) stage(tile0 + ti + 1, buf ^ 1);
-    const uint32_t* kt = kw + buf * W * TILE;
-    const uint32_t* vt = vw + buf * W * TILE;
-    const int tbase = (tile0 + ti) * TILE;
-
-    // ---- scores: this warp's groups 2 warp, 2 warp + 1 as four n-tiles of 8 tokens
-    float sc[4][4];
-    int tok[4];
+      for (int p = 0; p < NP; ++p)
 #pragma unroll
-    for (int n = 0; n < 4; ++n) {
-      tok[n] = 16 * (2 * warp + (n >> 1)) + (g & 1 ? 8 : 0) + (g >> 1) + 4 * (n & 1);   // column g's token
+        for (int z = 0; z < 4; ++z) vacc[i][r][p][z] = 0.0f;
+  float lsum[NP], ssum[NP];
 #pragma unroll
-      for (int r = 0; r < 4; ++r) sc[n][r] = 0.0f;
-    }
-    for (int wd = 0; wd < n2w_k; ++wd) {
-      const uint4 af = afrag[wd * 32 + lane];
+  for (int p = 0; p < NP; ++p) lsum[p] = ssum[p] = 0.0f;
+  uint32_t* pqw = reinterpret_cast<uint32_t*>(pq);
+  {
+    // tokens 32 warp + 4 Qk .. +3 (k = 4 Qk + j in the warp's k32 chunk), query 4 p + qq
+    const int qq = lane >> 3, Qk = lane & 7, t4 = Qk & 3, h2 = (Qk >> 2) * 2;
+    const int tk0 = 32 * warp + 4 * Qk;
+    for (int ti = 0; ti < n_tiles_split; ++ti) {
+      const int i_seq = n_tiles_split + ti;
+      wait_tile(i_seq);
+      const uint32_t* vt = ring + (i_seq % kStages) * W * TILE;
+      {
+        const int nvalid = t_end - (tile0 + ti) * TILE - tk0;         // tokens of this quad in range
+        const float4 a4 = *reinterpret_cast<const float4*>(av + ti * TILE + tk0);
+        const float av0 = nvalid > 0 ? a4.x * inv_p : 0.0f, av1 = nvalid > 1 ? a4.y * inv_p : 0.0f;
+        const float av2 = nvalid > 2 ? a4.z * inv_p : 0.0f, av3 = nvalid > 3 ? a4.w * inv_p : 0.0f;
 #pragma unroll
-      for (int n = 0; n < 4; ++n) {
-        const uint32_t x = kt[wd * TILE + tok[n]];
-        mma_16816(sc[n], af, hsub_magic(((x >> (2 * t)) & 0x00030003u) | 0x64006400u),
-                  hsub_magic(((x >> (2 * t + 8)) & 0x00030003u) | 0x64006400u));
-      }
-    }
-    for (int w1 = 0; w1 < n1w_k; ++w1) {
-      const int wd = n2w_k + w1;
-      const uint4 af0 = afrag[(n2w_k + 2 * w1) * 32 + lane];
-      const uint4 af1 = afrag[(n2w_k + 2 * w1 + 1) * 32 + lane];
+        for (int p = 0; p < NP; ++p) {
+          const int q = 4 * p + qq;
+          float4 pr = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+          if (q < G) {
+            const float4 sc = *reinterpret_cast<const float4*>(sbuf + q * sbs + ti * TILE + tk0);
+            const float mq = mqs[q];
+            pr = make_float4(fast_exp2(sc.x - mq), fast_exp2(sc.y - mq), fast_exp2(sc.z - mq), fast_exp2(sc.w - mq));
+          }
+          lsum[p] += (pr.x + pr.y) + (pr.z + pr.w);
+          float2 x01 = make_float2(pr.x * av0, pr.y * av1), x23 = make_float2(pr.z * av2, pr.w * av3);
+          const float xs = (x01.x + x01.y) + (x23.x + x23.y);
+          uint32_t* base = pqw + ((warp * NP + p) * 32 + t4) * 4 + h2;
 #pragma unroll
-      for (int n = 0; n < 4; ++n) {
-        const uint32_t x = kt[wd * TILE + tok[n]];
-        mma_16816(sc[n], af0, hsub_magic(((x >> t) & 0x00010001u) | 0x64006400u),
-                  hsub_magic(((x >> (t + 4)) & 0x00010001u) | 0x64006400u));
-        mma_16816(sc[n], af1, hsub_magic(((x >> (t + 8)) & 0x00010001u) | 0x64006400u),
-                  hsub_magic(((x >> (t + 12)) & 0x00010001u) | 0x64006400u));
-      }
-    }
-    // lane holds query g, columns 2t (token ta) and 2t+1 (token ta + 8) of each n-tile
-    float s8[4][2];
-    float mloc = -INFINITY;
-#pragma unroll
-    for (int n = 0; n < 4; ++n) {
-      const int ta = 16 * (2 * warp + (n >> 1)) + t + 4 * (n & 1);
-      const float sa = ak[buf * TILE + ta] * (sc[n][0] + sc[n][2] - c0);
-      const float sb = ak[buf * TILE + ta + 8] * (sc[n][1] + sc[n][3] - c0);
-      s8[n][0] = (g < G && tbase + ta < t_end) ? sa : -INFINITY;
-      s8[n][1] = (g < G && tbase + ta + 8 < t_end) ? sb : -INFINITY;
-      mloc = fmaxf(mloc, fmaxf(s8[n][0], s8[n][1]));
-    }
-    mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 1));
-    mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 2));
-    if (t == 0) red[warp * 8 + g] = mloc;
-    __syncthreads();
-    const float m_old = run[g];
-    float m_new = m_old;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) m_new = fmaxf(m_new, red[w * 8 + g]);
-    const float corr = m_old == -INFINITY ? 0.0f : fast_exp2(m_old - m_new);
-    // probabilities, P' = p alpha^V, partial sums, and the P' fragments for the value product
-    float lsum = 0.0f, ssum = 0.0f;
-#pragma unroll
-    for (int gg = 0; gg < 2; ++gg) {
-      float pv[4];
-#pragma unroll
-      for (int h = 0; h < 2; ++h)
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-          const int n = 2 * gg + h;
-          const int tk = 16 * (2 * warp + gg) + t + 4 * h + 8 * cc;
-          const float p = s8[n][cc] == -INFINITY ? 0.0f : fast_exp2(s8[n][cc] - m_new);
-          const float pp = p * av[buf * TILE + tk];
-          lsum += p;
-          ssum += pp;
-          pv[2 * h + cc] = pp;                 // slot 4t + {0: token t, 1: t+8, 2: t+4, 3: t+12}
+          for (int l = 0; l < 4; ++l) {
+            const uint32_t lo = e4m3_limb2(x01), hi = e4m3_limb2(x23);
+            // row 4 l + qq: lane group (4 l + qq) & 7, register + 1 for rows >= 8
+            base[((4 * l + qq) & 7) * 16 + (l >> 1)] = lo | (hi << 16);
+          }
+          ssum[p] += fmaf((x01.x + x01.y) + (x23.x + x23.y), -1.52587890625e-05f, xs);   // value of the limbs
         }
-      if (g < G) {
-        uint4 pk;
-        float hi, lo;
-        split_hi_lo(pv[0], hi, lo); pk.x = pack_half2(hi, lo);
-        split_hi_lo(pv[1], hi, lo); pk.y = pack_half2(hi, lo);
-        split_hi_lo(pv[2], hi, lo); pk.z = pack_half2(hi, lo);
-        split_hi_lo(pv[3], hi, lo); pk.w = pack_half2(hi, lo);
-        *reinterpret_cast<uint4*>(pfrag + ((2 * warp + gg) * MAX_GROUP + g) * 16 + 4 * t) = pk;
       }
-    }
-    lsum += __shfl_xor_sync(0xffffffffu, lsum, 1);
-    lsum += __shfl_xor_sync(0xffffffffu, lsum, 2);
-    ssum += __shfl_xor_sync(0xffffffffu, ssum, 1);
-    ssum += __shfl_xor_sync(0xffffffffu, ssum, 2);
-    if (t == 0) {
-      red[(kWarps + warp) * 8 + g] = lsum;
-      red[(2 * kWarps + warp) * 8 + g] = ssum;
-    }
-    __syncthreads();
-    if (warp == 0 && t == 0) {
-      float l = 0.0f, sp = 0.0f;
+      __syncthreads();
 #pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        l += red[(kWarps + w) * 8 + g];
-        sp += red[(2 * kWarps + w) * 8 + g];
-      }
-      run[g] = m_new;
-      run[8 + g] = run[8 + g] * corr + l;
-      run[16 + g] = run[16 + g] * corr + sp;
-    }
-
-    // ---- values: this warp's record words over the 8 groups of the tile
+      for (int kp = 0; kp < 4; ++kp) {
+        uint4 af[NP];
 #pragma unroll
-    for (int i = 0; i < WPW; ++i)
+        for (int p = 0; p < NP; ++p) af[p] = pq[(kp * NP + p) * 32 + lane];
+        const int q0 = 8 * kp + t, q1 = q0 + 4;                  // token quads of b0 / b1
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
+        for (int i = 0; i < WPW; ++i) {
+          const int wd = vw0 + i;
+          if (wd < vw1) {
+            if (wd < n2w_v) {
+              const uint2 x0 = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * q0 + 2 * (g >> 2));
+              const uint2 x1 = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * q1 + 2 * (g >> 2));
+              const int sh = 2 * (g & 3);
+              const uint32_t lo0 = (x0.x >> sh) & 0x03030303u, lo1 = (x1.x >> sh) & 0x03030303u;
+              const uint32_t hi0 = (x0.y >> sh) & 0x03030303u, hi1 = (x1.y >> sh) & 0x03030303u;
 #pragma unroll
-        for (int r = 0; r < 4; ++r) acc[i][q][r] *= corr;
-#pragma unroll 2
-    for (int g16 = 0; g16 < kGroups; ++g16) {
-      const uint4 pf = *reinterpret_cast<const uint4*>(pfrag + (g16 * MAX_GROUP + g) * 16 + 4 * t);
-      uint4 af;
-      af.x = __byte_perm(pf.x, pf.y, 0x5410);      // hi of tokens t, t+8
-      af.y = __byte_perm(pf.x, pf.y, 0x7632);      // lo
-      af.z = __byte_perm(pf.z, pf.w, 0x5410);      // hi of tokens t+4, t+12
-      af.w = __byte_perm(pf.z, pf.w, 0x7632);      // lo
+              for (int p = 0; p < NP; ++p) {
+                mma_e4m3(vacc[i][0][p], af[p], lo0, lo1);
+                mma_e4m3(vacc[i][1][p], af[p], hi0, hi1);
+              }
+            } else {
+              const uint4 x0 = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * q0);
+              const uint4 x1 = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * q1);
+              const uint32_t m1 = 0x01010101u;
+              const uint32_t c00 = (x0.x >> g) & m1, c01 = (x1.x >> g) & m1;   // quarter 0
+              const uint32_t c10 = (x0.z >> g) & m1, c11 = (x1.z >> g) & m1;   // quarter 1
+              const uint32_t c20 = (x0.y >> g) & m1, c21 = (x1.y >> g) & m1;   // quarter 2
+              const uint32_t c30 = (x0.w >> g) & m1, c31 = (x1.w >> g) & m1;   // quarter 3
 #pragma unroll
-      for (int i = 0; i < WPW; ++i) {
-        const int wd = vw0 + i;
-        if (wd < vw1) {
-          const uint4 vx = *reinterpret_cast<const uint4*>(vt + wd * TILE + 16 * g16 + 4 * t);
-          if (wd < n2w_v) {
-            mma_16816(acc[i][0], af, hsub_magic(((vx.x >> (2 * g)) & 0x00030003u) | 0x64006400u),
-                      hsub_magic(((vx.z >> (2 * g)) & 0x00030003u) | 0x64006400u));
-            mma_16816(acc[i][1], af, hsub_magic(((vx.y >> (2 * g)) & 0x00030003u) | 0x64006400u),
-                      hsub_magic(((vx.w >> (2 * g)) & 0x00030003u) | 0x64006400u));
-          } else {
-            mma_16816(acc[i][0], af, hsub_magic(((vx.x >> g) & 0x00010001u) | 0x64006400u),
-                      hsub_magic(((vx.z >> g) & 0x00010001u) | 0x64006400u));
-            mma_16816(acc[i][1], af, hsub_magic(((vx.x >> (g + 8)) & 0x00010001u) | 0x64006400u),
-                      hsub_magic(((vx.z >> (g + 8)) & 0x00010001u) | 0x64006400u));
-            mma_16816(acc[i][2], af, hsub_magic(((vx.y >> g) & 0x00010001u) | 0x64006400u),
-                      hsub_magic(((vx.w >> g) & 0x00010001u) | 0x64006400u));
-            mma_16816(acc[i][3], af, hsub_magic(((vx.y >> (g + 8)) & 0x00010001u) | 0x64006400u),
-                      hsub_magic(((vx.w >> (g + 8)) & 0x00010001u) | 0x64006400u));
+              for (int p = 0; p < NP; ++p) {
+                mma_e4m3(vacc[i][0][p], af[p], c00, c01);
+                mma_e4m3(vacc[i][1][p], af[p], c10, c11);
+                mma_e4m3(vacc[i][2][p], af[p], c20, c21);
+                mma_e4m3(vacc[i][3][p], af[p], c30, c31);
+              }
+            }
           }
         }
       }
+      __syncthreads();                                         // stage and pq free: refill
+      if (tid == 0 && i_seq + kStages < n_seq) {
+        ptx::fence_proxy_async_smem();
+        issue_tile(i_seq + kStages);
+      }
     }
   }
-  cp_async_wait_all();
-  __syncthreads();
 
-  // ---- partials: value sums per record entry, then m, l, S'
-  if (g < G) {
-    float* dst = a.ws + ((static_cast<size_t>(b) * a.n_q + head * G + g) * a.n_splits + split) * a.pstride;
+  // ---- per-query m, l, S' of the split; value entry sums into shared memory (staging area)
+#pragma unroll
+  for (int p = 0; p < NP; ++p)
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+      lsum[p] += __shfl_xor_sync(0xffffffffu, lsum[p], o);
+      ssum[p] += __shfl_xor_sync(0xffffffffu, ssum[p], o);
+    }
+  float* oe = reinterpret_cast<float*>(ring);                  // [G][n_entries]: the ring is drained
+  if ((lane & 7) == 0)
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+      red[warp * MAX_GROUP + 4 * p + (lane >> 3)] = lsum[p];
+      red[(kWarps + warp) * MAX_GROUP + 4 * p + (lane >> 3)] = ssum[p];
+    }
+#pragma unroll
+  for (int p = 0; p < NP; ++p) {
 #pragma unroll
     for (int i = 0; i < WPW; ++i) {
       const int wd = vw0 + i;
-      if (wd < vw1) {
-        const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
-        const int nq = wd < n2w_v ? 2 : 4;
+      const bool have = wd < vw1;
+      const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
+      const int nq = wd < n2w_v ? 2 : 4;
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-          if (q < nq) {
-            dst[ebase + 8 * q + 2 * t] = acc[i][q][0] + acc[i][q][2];
-            dst[ebase + 8 * q + 2 * t + 1] = acc[i][q][1] + acc[i][q][3];
-          }
+      for (int r = 0; r < 4; ++r) {
+        const float2 v = limb_sum(vacc[i][r][p], g);
+        const int q = 4 * p + g;
+        if (have && r < nq && g < 4 && q < G)
+          *reinterpret_cast<float2*>(oe + q * a.n_entries + ebase + 8 * r + 2 * t) =
+              make_float2(v.x * val_scale, v.y * val_scale);
       }
     }
-    if (warp == 0 && t == 0) {
-      dst[a.n_entries] = run[g];
-      dst[a.n_entries + 1] = run[8 + g];
-      dst[a.n_entries + 2] = run[16 + g];
-    }
-  }
-}
-
-// Merge the splits of one (sequence, query head) by log-sum-exp, rebuild channel sums from the
-// record entries (o_c = sum_e 2^shift_e O_e - 2^(b_c-1) S'), scale by f^V / l, apply U_V.
-// The partials of all splits are staged in shared memory with 16-byte loads first.
-constexpr int kCThreads = 256;
-
-__global__ void __launch_bounds__(kCThreads)
-    aatc_decode_combine_kernel(const DecodeArgs a) {
-  extern __shared__ __align__(16) float cs[];
-  const int stride = a.pstride;                      // multiple of 4
-  float* part = cs;                                  // [n_splits][stride]
-  float* wsp = part + a.n_splits * stride;           // [n_splits] split weights
-  float* oe = wsp + ((a.n_splits + 3) & ~3);         // [n_entries]
-  float* ohat = oe + a.n_entries;                    // [128]
-  float* ut_s = ohat + D;                            // [128][128] U_V^T of this kv-head
-  __shared__ float red[2][kCThreads / 32];
-  __shared__ float lsum[2];
-  const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  const int head = j / a.group;
-  const int sv = (a.layer * a.n_kv + head) * 2 + 1;
-  const float4* src = reinterpret_cast<const float4*>(a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * stride);
-  const int n4 = a.n_splits * stride / 4;
-  float4* p4 = reinterpret_cast<float4*>(part);
-  for (int i = tid; i < n4; i += kCThreads) cp_async16(p4 + i, src + i);
-  const float4* us = reinterpret_cast<const float4*>(a.u32t + static_cast<size_t>(sv) * D * D);
-  for (int i = tid; i < D * D / 4; i += kCThreads) cp_async16(reinterpret_cast<float4*>(ut_s) + i, us + i);
-  cp_async_commit();
-  cp_async_wait_all();
-  __syncthreads();
-  // split weights 2^(m_s - M): every thread scans the split maxima (few dozen)
-  float m = -INFINITY;
-  for (int s = 0; s < a.n_splits; ++s) m = fmaxf(m, part[s * stride + a.n_entries]);
-  if (tid < a.n_splits) wsp[tid] = exp2f(part[tid * stride + a.n_entries] - m);
-  for (int s = tid + kCThreads; s < a.n_splits; s += kCThreads) wsp[s] = exp2f(part[s * stride + a.n_entries] - m);
-  __syncthreads();
-  if (tid < 64) {
-    float l = 0.0f, sp = 0.0f;
-    for (int s = tid; s < a.n_splits; s += 64) {
-      l += part[s * stride + a.n_entries + 1] * wsp[s];
-      sp += part[s * stride + a.n_entries + 2] * wsp[s];
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      l += __shfl_xor_sync(0xffffffffu, l, o);
-      sp += __shfl_xor_sync(0xffffffffu, sp, o);
-    }
-    if ((tid & 31) == 0) {
-      red[0][tid >> 5] = l;
-      red[1][tid >> 5] = sp;
-    }
-  }
-  const StreamLayout lv = a.lay[sv];
-  const int n_used = lv.n2 + lv.n1;
-  for (int e = tid; e < n_used; e += kCThreads) {
-    float acc = 0.0f;
-    for (int s = 0; s < a.n_splits; ++s) acc = fmaf(part[s * stride + e], wsp[s], acc);
-    oe[e] = acc;
   }
   __syncthreads();
-  if (tid == 0) {
-    lsum[0] = red[0][0] + red[0][1];
-    lsum[1] = red[1][0] + red[1][1];
+  float* ml = red + 2 * kWarps * MAX_GROUP;                    // [3][MAX_GROUP]: m, l, S'
+  if (tid < G) {
+    const int q = tid;
+    ml[q] = mqs[q];
+    ml[MAX_GROUP + q] = red[q] + red[MAX_GROUP + q] + red[2 * MAX_GROUP + q] + red[3 * MAX_GROUP + q];
+    ml[2 * MAX_GROUP + q] = (red[(kWarps + 0) * MAX_GROUP + q] + red[(kWarps + 1) * MAX_GROUP + q] +
+                             red[(kWarps + 2) * MAX_GROUP + q] + red[(kWarps + 3) * MAX_GROUP + q]) *
+                            (amx / 256.0f);
   }
   __syncthreads();
-  if (tid < D) {
+  // channel sums of this split: thread = channel
+  const size_t pbase = (static_cast<size_t>(b) * a.n_q + head * G) * a.n_splits;
+  {
     const int c = tid;
-    const short* ce = a.chan_ent + (static_cast<size_t>(sv) * D + c) * 8;
-    const short* ent = a.entry + static_cast<size_t>(sv) * a.n_entries;
-    float o = 0.0f;
+    const uint4 cev = *reinterpret_cast<const uint4*>(cetab + c * 8);
+    const short* ce = reinterpret_cast<const short*>(&cev);
+    float w[8];
+    int e_[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      const int e = ce[k];
-      if (e >= 0) o += ldexpf(oe[e], ent[e] >> 8);
+      e_[k] = min(max(static_cast<int>(ce[k]), 0), a.n_entries - 1);
+      w[k] = ce[k] >= 0 ? pow2i((etab[e_[k]] >> 8) & 7) : 0.0f;
     }
-    o -= a.enc[sv * D + c].off * lsum[1];
-    ohat[c] = o * a.f[sv * D + c] / lsum[0];
+    const float off = off_c;
+    for (int q = 0; q < G; ++q) {
+      float o = -off * ml[2 * MAX_GROUP + q];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) o = fmaf(w[k], oe[q * a.n_entries + e_[k]], o);
+      float* dst = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits + split) * a.pstride;
+      dst[c] = o;
+      if (c == 0) {
+        dst[D] = ml[q];
+        dst[D + 1] = ml[MAX_GROUP + q];
+      }
+    }
+  }
+  // ---- the last split of this head to finish merges all of them
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(a.cnt + b * a.n_kv + head, 1) == a.n_splits - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const float fv = fv_c;
+  const float* ut = a.u32t + static_cast<size_t>(sv) * D * D + tid;
+  // merge scratch in the drained ring: split weights [4P][n_splits], chunk sums [4][4P][128],
+  // o_hat [4P][128], 1/l [4P]
+  const int QP = 4 * NP;
+  float* wsp = oe;
+  float* osum = wsp + QP * ((a.n_splits + 3) & ~3);
+  float* ohat = osum + 4 * QP * D;
+  float* linv = ohat + QP * D;
+  // (1) per query (one warp each): M = max_s m_s, w_s = 2^(m_s - M), l = sum_s w_s l_s
+  for (int q = warp; q < G; q += kWarps) {
+    const float* src = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits) * a.pstride + D;
+    float M = -INFINITY;
+    for (int s2 = lane; s2 < a.n_splits; s2 += 32) M = fmaxf(M, __ldcg(src + s2 * a.pstride));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float l = 0.0f;
+    for (int s2 = lane; s2 < a.n_splits; s2 += 32) {
+      const float2 ml2 = __ldcg(reinterpret_cast<const float2*>(src + s2 * a.pstride));
+      const float w = exp2f(ml2.x - M);
+      wsp[q * ((a.n_splits + 3) & ~3) + s2] = w;
+      l = fmaf(w, ml2.y, l);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (lane == 0) linv[q] = 1.0f / l;
   }
   __syncthreads();
-  {
-    // out[d] = sum_c U_V[d][c] ohat[c]; two threads per output dimension
-    const int d = tid & (D - 1), half = tid >> 7;
-    float o = 0.0f;
-#pragma unroll 16
-    for (int c = half * 64; c < half * 64 + 64; ++c) o = fmaf(ut_s[c * D + d], ohat[c], o);
-    if (half) oe[d] = o;
-    __syncthreads();
-    if (!half) a.out[(static_cast<size_t>(b) * a.n_q + j) * D + d] = o + oe[d];
+  // (2) chunk sums: warp = splits s = warp (mod 4), lane = channels 4 lane .. 4 lane + 3
+  for (int q = 0; q < G; ++q) {
+    const float* src = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits) * a.pstride + 4 * lane;
+    const float* wq = wsp + q * ((a.n_splits + 3) & ~3);
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    int s2 = warp;
+    for (; s2 + 4 * 7 < a.n_splits; s2 += 4 * 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s2 + 4 * u) * a.pstride));
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float w = wq[s2 + 4 * u];
+        acc.x = fmaf(w, v[u].x, acc.x);
+        acc.y = fmaf(w, v[u].y, acc.y);
+        acc.z = fmaf(w, v[u].z, acc.z);
+        acc.w = fmaf(w, v[u].w, acc.w);
+      }
+    }
+    for (; s2 < a.n_splits; s2 += 4) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(src + s2 * a.pstride));
+      const float w = wq[s2];
+      acc.x = fmaf(w, v.x, acc.x);
+      acc.y = fmaf(w, v.y, acc.y);
+      acc.z = fmaf(w, v.z, acc.z);
+      acc.w = fmaf(w, v.w, acc.w);
+    }
+    *reinterpret_cast<float4*>(osum + (warp * QP + q) * D + 4 * lane) = acc;
   }
+  __syncthreads();
+  // (3) o_hat_c = o_c f_c / l
+  for (int q = 0; q < G; ++q)
+    ohat[q * D + tid] = ((osum[(0 * QP + q) * D + tid] + osum[(1 * QP + q) * D + tid]) +
+                         (osum[(2 * QP + q) * D + tid] + osum[(3 * QP + q) * D + tid])) * fv * linv[q];
+  __syncthreads();
+  // (4) out = U_V o_hat for every query of the group in one pass over U_V (thread = dimension)
+  float r[4 * NP];
+#pragma unroll
+  for (int q = 0; q < 4 * NP; ++q) r[q] = 0.0f;
+#pragma unroll 4
+  for (int c0 = 0; c0 < D; c0 += 32) {
+    float u[32];
+#pragma unroll
+    for (int c = 0; c < 32; ++c) u[c] = ut[(c0 + c) * D];
+#pragma unroll
+    for (int q = 0; q < 4 * NP; ++q)
+      if (q < G)
+#pragma unroll
+        for (int c = 0; c < 32; ++c) r[q] = fmaf(u[c], ohat[q * D + c0 + c], r[q]);
+  }
+#pragma unroll
+  for (int q = 0; q < 4 * NP; ++q)
+    if (q < G) a.out[(static_cast<size_t>(b) * a.n_q + head * G + q) * D + tid] = r[q];
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -604,9 +755,12 @@ __global__ void __launch_bounds__(kThreads)
   float* sc = red + 32;                                    // [split_len][GP]
   __nv_bfloat16* kt = reinterpret_cast<__nv_bfloat16*>(sc + a.split_len * GP);   // [2][128][kRow]
   float* accs = reinterpret_cast<float*>(kt + 2 * TILE * kRow);                  // [4][GP][128]
-  const int t_begin = split * a.split_len;
-  const int t_end = min(a.n_ctx, t_begin + a.split_len);
-  const int n_tiles_split = (t_end - t_begin + TILE - 1) / TILE;
+  const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
+  const int tile_lo = static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
+  const int tile_hi = static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
+  const int t_begin = tile_lo * TILE;
+  const int t_end = min(a.n_ctx, tile_hi * TILE);
+  const int n_tiles_split = tile_hi - tile_lo;
   const float scale = kLog2e * 0.08838834764831845f;
   for (int i = tid; i < GP * D; i += kThreads) {
     const int g = i / D, d = i % D;
@@ -762,18 +916,13 @@ __global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, c
   const size_t cs = (static_cast<size_t>(b) * n_kv + head) * 2 + kind;
   const uint32_t* tile = words + cs * n_tiles * n_words * TILE + static_cast<size_t>(t / TILE) * n_words * TILE;
   const int tt = t % TILE;
-  int lane_lo = tt, lane_hi = tt, half = 0;
-  if (kind == 1) {
-    const int j = tt & 15, pr = j & 7;
-    lane_lo = 16 * (tt >> 4) + 4 * (pr & 3) + 2 * (pr >> 2);
-    lane_hi = lane_lo + 1;
-    half = j >> 3;
-  }
   auto rec_word = [&](int w) -> uint32_t {
-    if (kind == 0) return tile[static_cast<size_t>(w) * TILE + tt];
-    const uint32_t lo = (tile[static_cast<size_t>(w) * TILE + lane_lo] >> (16 * half)) & 0xFFFFu;
-    const uint32_t hi = (tile[static_cast<size_t>(w) * TILE + lane_hi] >> (16 * half)) & 0xFFFFu;
-    return lo | (hi << 16);
+    const uint32_t* ww = tile + static_cast<size_t>(w) * TILE;
+    if (kind == 0) return ww[tt];
+    const int q4 = 4 * (tt >> 2), sh = 8 * (tt & 3);
+    const uint32_t b0 = (ww[q4 + 0] >> sh) & 0xFFu, b1 = (ww[q4 + 2] >> sh) & 0xFFu;
+    const uint32_t b2 = (ww[q4 + 1] >> sh) & 0xFFu, b3 = (ww[q4 + 3] >> sh) & 0xFFu;
+    return b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
   };
   const int s = (layer * n_kv + head) * 2 + kind;
   const StreamLayout ly = lays[s];
@@ -807,24 +956,35 @@ __global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, c
   }
 }
 
-template <int WPW, int GP>
+template <int WPW, int NP>
 cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
   static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
   if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<WPW, GP>,
+    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<WPW, NP>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  aatc_decode_split_kernel<WPW, GP><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  // programmatic dependent launch: the split kernel's prologue (cache tiles, scales, tables)
+  // overlaps the query kernel; it waits for the query kernel's results before loading them
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_splits, a.n_kv, batch);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, aatc_decode_split_kernel<WPW, NP>, a);
 }
 
-template <int GP>
+template <int NP>
 cudaError_t launch_split_g(const DecodeArgs& a, int batch, int wpw, size_t smem, cudaStream_t st) {
-  if (wpw <= 3) return launch_split_t<3, GP>(a, batch, smem, st);
-  if (wpw <= 4) return launch_split_t<4, GP>(a, batch, smem, st);
-  return launch_split_t<8, GP>(a, batch, smem, st);
+  if (wpw <= 3) return launch_split_t<3, NP>(a, batch, smem, st);
+  if (wpw <= 4) return launch_split_t<4, NP>(a, batch, smem, st);
+  return launch_split_t<8, NP>(a, batch, smem, st);
 }
 
 template <int GP>
@@ -872,38 +1032,29 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_splits = sp.n_splits;
   a.split_len = sp.split_len;
   // largest key k-step count and value word count over the layer's streams
-  int n_ks = 1, nw_v = 1;
+  int n_s = 1, nw_v = 1;
   for (int h = 0; h < a.n_kv; ++h) {
     const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
     const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
-    n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
+    n_s = std::max(n_s, (lk.n2 / 16 + 1) / 2 + (lk.n1 + 31) / 32);
     nw_v = std::max(nw_v, lv.n2 / 16 + (lv.n1 + 31) / 32);
   }
+  const int np = (a.group + 3) / 4;
   const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
   a.pstride = wsl.pstride;
   a.ks_stride = wsl.ks_stride;
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
-  aatc_decode_query_kernel<<<dim3(a.n_kv, batch), kQThreads, 0, st>>>(a);
+  a.cnt = reinterpret_cast<int*>(static_cast<char*>(ws) + wsl.cnt_off);
+  if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
+  aatc_decode_query_kernel<<<dim3(a.n_kv, batch, 4 * np), kQThreads, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const SplitLayout L(n_ks, plan.n_words);
-  const size_t smem = 4 * static_cast<size_t>(L.n_words_total);
+  const SplitSmem L(n_s, np, sp.split_len, plan.n_words, plan.n_entries, sp.n_splits);
+  const size_t smem = static_cast<size_t>(L.total);
   const int wpw = (nw_v + kWarps - 1) / kWarps;
-  if (wpw > 8) return cudaErrorNotSupported;
-  e = a.group <= 4 ? launch_split_g<4>(a, batch, wpw, smem, st) : launch_split_g<8>(a, batch, wpw, smem, st);
-  if (e != cudaSuccess) return e;
-  const size_t csmem =
-      4 * (static_cast<size_t>(a.n_splits) * a.pstride + ((a.n_splits + 3) & ~3) + plan.n_entries + D + D * D);
-  static size_t csmem_set = 0;
-  if (csmem > 48 * 1024 && csmem > csmem_set) {
-    e = cudaFuncSetAttribute(aatc_decode_combine_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(csmem));
-    if (e != cudaSuccess) return e;
-    csmem_set = csmem;
-  }
-  aatc_decode_combine_kernel<<<dim3(a.n_q, batch), kCThreads, csmem, st>>>(a);
-  return cudaGetLastError();
+  if (wpw > 8 || smem > 227 * 1024) return cudaErrorNotSupported;
+  return np == 1 ? launch_split_g<1>(a, batch, wpw, smem, st) : launch_split_g<2>(a, batch, wpw, smem, st);
 }
 
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n, int max_tokens,

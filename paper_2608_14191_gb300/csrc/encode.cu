@@ -62,19 +62,22 @@ __device__ __forceinline__ void raise_abort(EncodeSmem& sm, int* err) {
   atomicOr(err, 2);
 }
 
-// Writes one finished record word of a token.  Keys: plain word-planar store.  Values: the
-// two 16-bit halves go to the token's low-half and high-half lanes of its 16-token pair block.
+// Writes one finished record word of a token.  Keys: plain word-planar store.  Values: the four
+// byte-quarters go to the token's byte of the four slots of its 4-token block (slot positions
+// 0, 2, 1, 3 for quarters 0..3), so each token only writes its own bytes.
 struct RecordWriter {
   uint32_t* key_word;     // keys: &words[.. tile][0][lane]
-  uint16_t* val_lo;       // values: half of the low-half lane
-  uint16_t* val_hi;       // values: half of the high-half lane
+  uint8_t* val_byte;      // values: byte (token % 4) of slot 4 (token / 4), record word 0
   bool value;
   __device__ __forceinline__ void put(int wi, uint32_t w) const {
     if (!value) {
       key_word[static_cast<size_t>(wi) * TILE] = w;
     } else {
-      val_lo[static_cast<size_t>(wi) * TILE * 2] = static_cast<uint16_t>(w & 0xFFFFu);
-      val_hi[static_cast<size_t>(wi) * TILE * 2] = static_cast<uint16_t>(w >> 16);
+      uint8_t* p = val_byte + static_cast<size_t>(wi) * TILE * 4;
+      p[0] = static_cast<uint8_t>(w);
+      p[8] = static_cast<uint8_t>(w >> 8);
+      p[4] = static_cast<uint8_t>(w >> 16);
+      p[12] = static_cast<uint8_t>(w >> 24);
     }
   }
 };
@@ -255,12 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       out.value = kind == 1;
       const int tt = pos_t % TILE;
       out.key_word = tile_words + tt;
-      {
-        const int j = tt & 15, grp = tt >> 4, pr = j & 7;
-        const int base = 16 * grp + 4 * (pr & 3) + 2 * (pr >> 2);
-        out.val_lo = reinterpret_cast<uint16_t*>(tile_words + base) + (j >> 3);
-        out.val_hi = reinterpret_cast<uint16_t*>(tile_words + base + 1) + (j >> 3);
-      }
+      out.val_byte = reinterpret_cast<uint8_t*>(tile_words + 4 * (tt >> 2)) + (tt & 3);
 
       // D2: base-4 digit k of channels 0..l2[k]-1, four channels at a time
       uint32_t word = 0;

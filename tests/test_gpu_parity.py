@@ -169,7 +169,16 @@ def _full_case_check(aatc, cfg, avg_bits, n_code_tokens=2048, decode_steps=2, he
 
 
 def test_llama_layer_full_size(aatc):
-    _full_case_check(aatc, W.CONFIGS["llama_layer"], 2.75)
+    case, kd, vd, cache, _ = _full_case_check(aatc, W.CONFIGS["llama_layer"], 2.75)
+    # repeated calls are bitwise identical: fixed split ranges, fixed merge order, and no shared
+    # state between calls beyond the workspace (a race between phases would show up here)
+    cfg = W.CONFIGS["llama_layer"]
+    q = W.queries_device(cfg, 0, cfg.batch, 1, DEV)[0]
+    ws = torch.empty(case.plan.workspace_bytes(cfg.batch, cfg.n_ctx) // 4 + 1, dtype=torch.float32, device=DEV)
+    first = aatc.decode_attention(case.plan, 0, q, cache, cfg.n_ctx, cfg.n_ctx, workspace=ws).cpu()
+    for _ in range(6):
+        again = aatc.decode_attention(case.plan, 0, q, cache, cfg.n_ctx, cfg.n_ctx, workspace=ws).cpu()
+        assert torch.equal(first, again)
 
 
 def test_qwen_batched_full_size(aatc):

@@ -318,7 +318,7 @@ def test_pack_round_trip_random():
 
 
 def test_value_interleave_round_trip():
-    """Values are stored pair-interleaved in half-words; keys plainly.  Writing records into a
+    """Values are stored quad-interleaved in byte-quarters; keys plainly.  Writing records into a
     cache image and reading them back returns them unchanged for every token position."""
     rng = np.random.default_rng(15)
     bits = np.sort(rng.integers(1, 9, O.D))[::-1]
@@ -334,8 +334,8 @@ def test_value_interleave_round_trip():
             rec, al = O.cache_records(img, 1, 2, 384, nw, 0, h, kind, 0, n)
             assert np.array_equal(rec, recs[idx]) and np.array_equal(al, alphas[idx])
             assert np.array_equal(O.unpack_records(rec, bits), codes[idx])
-    lanes = sorted({O.value_lane_of(t)[:2] for t in range(16)})
-    assert lanes == [(0, 1), (2, 3), (4, 5), (6, 7), (8, 9), (10, 11), (12, 13), (14, 15)]
+    slots = sorted(O.value_slot_of(t, r) for t in range(8) for r in range(4))
+    assert slots == [(s, i) for s in range(8) for i in range(4)]
 
 
 def test_record_size_matches_paper_compression():
