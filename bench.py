@@ -300,14 +300,14 @@ def run_ours(args):
                    "frac_of_measured_hbm_on_input": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9 / peak, 4)},
         "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": _traffic_per_launch(),
-                     "kernel": "aatc_decode_query_kernel + aatc_decode_split_kernel (one decode call)",
+                     "kernel": "aatc_decode_query_kernel + aatc_decode_split_kernel + aatc_decode_merge_kernel (one decode call)",
                      "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"},
         "e2e": {"value": round(ws_ * steps_dec * dbytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "ms_per_step": round(e2e_ms, 4),
                 "what": "per step: H2D of K, V and queries from pinned host memory, encode, 256 decode calls "
                         "through the public API, D2H of all outputs"},
-        "gpu_launches": args.steps * (1 + 2 * steps_dec),
+        "gpu_launches": args.steps * (1 + 3 * steps_dec),
         "clocks": clocks,
     }
     if not args.no_cpu_baseline:

@@ -109,11 +109,11 @@ DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
 // Decode workspace: split partials per (sequence, query head, split) -- 128 channel sums, then
 // m, l, padded to a multiple of 4 floats -- followed by the per-call score A fragments per
 // (sequence, kv-head) (up to 2 W k-steps x 32 lanes x 16 B), their offset corrections and score
-// scales, and one finished-split counter per (sequence, kv-head).
+// scales.
 struct DecodeWs {
   int pstride;            // floats per partial
   int ks_stride;          // uint4 per (sequence, kv-head) fragment block
-  size_t qfrag_off, qcorr_off, cnt_off, bytes;
+  size_t qfrag_off, qcorr_off, bytes;
 };
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
 size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);

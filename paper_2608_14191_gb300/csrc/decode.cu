@@ -2,17 +2,17 @@
 // uncompressed bf16 reference decode (Def. sdpa with one query row; Algorithm 1
 // "Reconstruct", "softmax", "Output" lines, computed without rebuilding the keys).
 //
-// Three launches per call (flash-decoding split over the context):
-//   query    per (sequence, kv-head): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the G query heads
-//            of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1), and q' in
-//            24-bit fixed point as int8 tensor-core fragments;
+// Three launches per call (flash-decoding split over the context), each a programmatic
+// dependent of the one before it:
+//   query    per (sequence, kv-head, query slot): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the
+//            G query heads of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1),
+//            and q' as e4m3 tensor-core fragments (four limbs);
 //   split    per (split, kv-head, sequence): pass 1 scores
-//            s_{g,t} = alpha^K_t (sigma_g sum_e Q_{g,e} digit_{t,e} - C_g) on the int8 tensor
-//            cores over the packed digits; split max m_g; pass 2 p = 2^(s - m_g),
-//            P' = p alpha^V_t in 24-bit fixed point, value entry sums sum_t P'_{g,t} digit_{t,e}
-//            on the tensor cores with exact int32 accumulation over the whole split;
-//   combine  per (sequence, query head): log-sum-exp merge of the splits, record entries back to
-//            channel sums with the offset correction, f^V / l, and out = U_V o_hat.
+//            s_{g,t} = alpha^K_t (sum_e q'_{g,e} digit_{t,e} - C_g) on the fp8 tensor cores over
+//            the packed digits; split max m_g; pass 2 p = 2^(s - m_g), P' = p alpha^V_t, value
+//            entry sums sum_t P'_{g,t} digit_{t,e} on the tensor cores; entry sums folded into
+//            channel sums with the offset correction; (o, m, l) per split;
+//   merge    per (sequence, query head): log-sum-exp merge of the splits, f^V / l, out = U_V o_hat.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -81,7 +81,6 @@ struct DecodeArgs {
   int* err;
   uint4* qfrag;            // workspace: score A fragments [batch][n_kv][ks_stride]
   float* qcorr;            // workspace: [batch][n_kv][16]: offset corrections C_g, score scales
-  int* cnt;                // workspace: [batch][n_kv] finished-split counters
   int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len, ks_stride, pstride;
 };
 
@@ -148,7 +147,7 @@ constexpr int kMaxEntries = 32 * 32;   // 8 bits x 128 channels
 // Per call, per (sequence, kv-head, query slot): folded query q'_c = (U_K^T q)_c f_c log2(e)/sqrt(128),
 // its offset correction C = sum_c q'_c 2^(b_c-1), the score scale, and the rows of the score A
 // fragments that hold this query (four e4m3 limbs of q'_c 2^shift / sigma per record entry).
-// Slots G..4P-1 write zero rows.  Slot 0 also clears the finished-split counter of its head.
+// Slots G..4P-1 write zero rows.
 __global__ void __launch_bounds__(kQThreads)
     aatc_decode_query_kernel(const DecodeArgs a) {
   __shared__ float qv[D];
@@ -161,7 +160,6 @@ __global__ void __launch_bounds__(kQThreads)
   const bool real = slot < G;
   const int sk = (a.layer * a.n_kv + head) * 2;
   ptx::grid_launch_dependents();
-  if (slot == 0 && tid == 0) a.cnt[b * a.n_kv + head] = 0;
   // every global input is requested up front (one memory round trip)
   const int c = tid & (D - 1), qd = tid >> 7;
   const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
@@ -170,7 +168,6 @@ __global__ void __launch_bounds__(kQThreads)
   const StreamLayout lk = a.lay[sk];
   float qraw = 0.0f, fk = 0.0f, off = 0.0f;
   if (tid < D) {
-    if (real) qraw = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + slot) * D + tid]);
     fk = a.f[sk * D + c];
     off = a.enc[sk * D + c].off;                                          // 2^(b_c - 1), 0 if b_c = 0
   }
@@ -181,6 +178,10 @@ __global__ void __launch_bounds__(kQThreads)
 #pragma unroll
     for (int d = 0; d < 32; ++d) u[d] = uk[d * D];
   }
+  // plan constants above; the query (and the workspace this call reuses) only once the preceding
+  // grid in the stream is complete -- this kernel may be launched as its programmatic dependent
+  ptx::grid_dependency_wait();
+  if (tid < D && real) qraw = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + slot) * D + tid]);
   if (tid < D) qv[tid] = qraw;
   __syncthreads();
   {
@@ -258,7 +259,7 @@ __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 // shared-memory carve-up of the split kernel (byte offsets)
 struct SplitSmem {
   int bars, qcg, red, cetab, etab, afrag, ak, av, sbuf, pq, ring, total, sb_stride;
-  __host__ __device__ SplitSmem(int n_steps, int np, int split_len, int W, int n_entries, int n_splits) {
+  __host__ __device__ SplitSmem(int n_steps, int np, int split_len, int W, int n_entries) {
     int o = 0;
     bars = o;  o = align16(o + 8 * (kStages + 1));  // ring barriers, then the prologue barrier
     qcg = o;   o += 2 * MAX_GROUP * 4;              // offset corrections, score scales
@@ -271,9 +272,7 @@ struct SplitSmem {
     sb_stride = split_len + 8;                      // padded: query rows fall in different banks
     sbuf = o;  o += 4 * np * sb_stride * 4;         // scores of the split
     pq = o;    o += 4 * np * 32 * 16;               // P' limb fragments of one tile
-    ring = o;                                       // after the last tile: entry sums, merge scratch
-    const int merge = 4 * (4 * np * ((n_splits + 3) & ~3) + 5 * 4 * np * D + 4 * np);
-    o += align16(max(kStages * W * TILE * 4, merge));
+    ring = o;  o += kStages * W * TILE * 4;         // after the last tile: value entry sums
     total = o;
   }
 };
@@ -289,7 +288,6 @@ template <int WPW, int NP>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smb[];
-  __shared__ int s_last;
   __shared__ int s_abort;
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -301,7 +299,7 @@ __global__ void __launch_bounds__(kThreads)
   const int n2w_k = lk.n2 / 16, n2s_k = (n2w_k + 1) / 2, n1w_k = (lk.n1 + 31) / 32;
   const int n_s = n2s_k + n1w_k;
   const int n2w_v = lv.n2 / 16, nw_v = n2w_v + (lv.n1 + 31) / 32;
-  const SplitSmem L(n_s, NP, a.split_len, W, a.n_entries, a.n_splits);
+  const SplitSmem L(n_s, NP, a.split_len, W, a.n_entries);
   uint64_t* full = reinterpret_cast<uint64_t*>(smb + L.bars);
   uint64_t* pro = full + kStages;
   float* qcg = reinterpret_cast<float*>(smb + L.qcg);          // [0..7] C_g, [8..15] score scales
@@ -332,7 +330,7 @@ __global__ void __launch_bounds__(kThreads)
   const float* kalpha = a.alpha + bk * a.n_tiles * TILE;
   const float* valpha = a.alpha + (bk + 1) * a.n_tiles * TILE;
   const float off_c = a.enc[sv * D + tid].off;                 // this thread's value channel
-  const float fv_c = a.f[sv * D + tid];
+  ptx::grid_launch_dependents();                               // the merge kernel may get ready
 
   auto issue_tile = [&](int i) {
     const int s = i % kStages;
@@ -635,94 +633,115 @@ __global__ void __launch_bounds__(kThreads)
       }
     }
   }
-  // ---- the last split of this head to finish merges all of them
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) s_last = atomicAdd(a.cnt + b * a.n_kv + head, 1) == a.n_splits - 1;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  const float fv = fv_c;
-  const float* ut = a.u32t + static_cast<size_t>(sv) * D * D + tid;
-  // merge scratch in the drained ring: split weights [4P][n_splits], chunk sums [4][4P][128],
-  // o_hat [4P][128], 1/l [4P]
-  const int QP = 4 * NP;
-  float* wsp = oe;
-  float* osum = wsp + QP * ((a.n_splits + 3) & ~3);
-  float* ohat = osum + 4 * QP * D;
-  float* linv = ohat + QP * D;
-  // (1) per query (one warp each): M = max_s m_s, w_s = 2^(m_s - M), l = sum_s w_s l_s
-  for (int q = warp; q < G; q += kWarps) {
-    const float* src = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits) * a.pstride + D;
-    float M = -INFINITY;
-    for (int s2 = lane; s2 < a.n_splits; s2 += 32) M = fmaxf(M, __ldcg(src + s2 * a.pstride));
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float l = 0.0f;
-    for (int s2 = lane; s2 < a.n_splits; s2 += 32) {
-      const float2 ml2 = __ldcg(reinterpret_cast<const float2*>(src + s2 * a.pstride));
-      const float w = exp2f(ml2.x - M);
-      wsp[q * ((a.n_splits + 3) & ~3) + s2] = w;
-      l = fmaf(w, ml2.y, l);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (lane == 0) linv[q] = 1.0f / l;
+}
+
+// Merge of the splits of one (sequence, query head): M = max_s m_s, w_s = 2^(m_s - M),
+// o_c = sum_s w_s o_{s,c}, l = sum_s w_s l_s, o_hat_c = o_c f^V_c / l, out = U_V o_hat.
+// Launched as a programmatic dependent of the split kernel: U_V^T (a plan constant) is staged
+// while the splits finish; the partials are read only after the grid dependency resolves.
+constexpr int kMThreads = 256;
+constexpr int kMWarps = kMThreads / 32;
+
+__global__ void __launch_bounds__(kMThreads)
+    aatc_decode_merge_kernel(const DecodeArgs a) {
+  extern __shared__ __align__(16) float ms[];
+  float* ut_s = ms;                                  // [128 c][128 d]
+  float* wsp = ut_s + D * D;                         // [n_splits] split weights
+  float* osum = wsp + ((a.n_splits + 3) & ~3);       // [kMWarps][128]
+  float* ohat = osum + kMWarps * D;                  // [128]
+  __shared__ float red[2][kMWarps];
+  __shared__ uint64_t bar;
+  __shared__ int s_abort;
+  const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int head = j / a.group;
+  const int sv = (a.layer * a.n_kv + head) * 2 + 1;
+  if (tid == 0) {
+    s_abort = 0;
+    ptx::mbar_init(&bar, 1);
+    ptx::fence_mbar_init();
+    ptx::mbar_arrive_expect_tx(&bar, D * D * 4);
+    ptx::bulk_load(ut_s, a.u32t + static_cast<size_t>(sv) * D * D, D * D * 4, &bar);
   }
+  const float fv = tid < D ? a.f[sv * D + tid] : 0.0f;
+  ptx::grid_dependency_wait();                       // the split kernel's partials
+  const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * a.pstride;
+  // split maxima and weights
+  float M = -INFINITY;
+  for (int s = tid; s < a.n_splits; s += kMThreads) M = fmaxf(M, __ldcg(src + s * a.pstride + D));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  if (lane == 0) red[0][warp] = M;
   __syncthreads();
-  // (2) chunk sums: warp = splits s = warp (mod 4), lane = channels 4 lane .. 4 lane + 3
-  for (int q = 0; q < G; ++q) {
-    const float* src = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits) * a.pstride + 4 * lane;
-    const float* wq = wsp + q * ((a.n_splits + 3) & ~3);
+  M = red[0][0];
+#pragma unroll
+  for (int w = 1; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
+  float l = 0.0f;
+  for (int s = tid; s < a.n_splits; s += kMThreads) {
+    const float2 ml = __ldcg(reinterpret_cast<const float2*>(src + s * a.pstride + D));
+    const float w = exp2f(ml.x - M);
+    wsp[s] = w;
+    l = fmaf(w, ml.y, l);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  if (lane == 0) red[1][warp] = l;
+  __syncthreads();
+  // weighted channel sums: warp = splits s = warp (mod 8), lane = channels 4 lane .. 4 lane + 3
+  {
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-    int s2 = warp;
-    for (; s2 + 4 * 7 < a.n_splits; s2 += 4 * 8) {
+    int s = warp;
+    for (; s + kMWarps * 7 < a.n_splits; s += kMWarps * 8) {
       float4 v[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s2 + 4 * u) * a.pstride));
+      for (int u = 0; u < 8; ++u)
+        v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s + kMWarps * u) * a.pstride + 4 * lane));
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        const float w = wq[s2 + 4 * u];
+        const float w = wsp[s + kMWarps * u];
         acc.x = fmaf(w, v[u].x, acc.x);
         acc.y = fmaf(w, v[u].y, acc.y);
         acc.z = fmaf(w, v[u].z, acc.z);
         acc.w = fmaf(w, v[u].w, acc.w);
       }
     }
-    for (; s2 < a.n_splits; s2 += 4) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(src + s2 * a.pstride));
-      const float w = wq[s2];
-      acc.x = fmaf(w, v.x, acc.x);
-      acc.y = fmaf(w, v.y, acc.y);
-      acc.z = fmaf(w, v.z, acc.z);
-      acc.w = fmaf(w, v.w, acc.w);
-    }
-    *reinterpret_cast<float4*>(osum + (warp * QP + q) * D + 4 * lane) = acc;
+    float4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (s + kMWarps * u < a.n_splits)
+        v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s + kMWarps * u) * a.pstride + 4 * lane));
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (s + kMWarps * u < a.n_splits) {
+        const float w = wsp[s + kMWarps * u];
+        acc.x = fmaf(w, v[u].x, acc.x);
+        acc.y = fmaf(w, v[u].y, acc.y);
+        acc.z = fmaf(w, v[u].z, acc.z);
+        acc.w = fmaf(w, v[u].w, acc.w);
+      }
+    *reinterpret_cast<float4*>(osum + warp * D + 4 * lane) = acc;
   }
   __syncthreads();
-  // (3) o_hat_c = o_c f_c / l
-  for (int q = 0; q < G; ++q)
-    ohat[q * D + tid] = ((osum[(0 * QP + q) * D + tid] + osum[(1 * QP + q) * D + tid]) +
-                         (osum[(2 * QP + q) * D + tid] + osum[(3 * QP + q) * D + tid])) * fv * linv[q];
-  __syncthreads();
-  // (4) out = U_V o_hat for every query of the group in one pass over U_V (thread = dimension)
-  float r[4 * NP];
+  if (tid < D) {
+    float o = 0.0f;
 #pragma unroll
-  for (int q = 0; q < 4 * NP; ++q) r[q] = 0.0f;
-#pragma unroll 4
-  for (int c0 = 0; c0 < D; c0 += 32) {
-    float u[32];
+    for (int w = 0; w < kMWarps; ++w) o += osum[w * D + tid];
+    float lt = 0.0f;
 #pragma unroll
-    for (int c = 0; c < 32; ++c) u[c] = ut[(c0 + c) * D];
-#pragma unroll
-    for (int q = 0; q < 4 * NP; ++q)
-      if (q < G)
-#pragma unroll
-        for (int c = 0; c < 32; ++c) r[q] = fmaf(u[c], ohat[q * D + c0 + c], r[q]);
+    for (int w = 0; w < kMWarps; ++w) lt += red[1][w];
+    ohat[tid] = o * fv / lt;
   }
-#pragma unroll
-  for (int q = 0; q < 4 * NP; ++q)
-    if (q < G) a.out[(static_cast<size_t>(b) * a.n_q + head * G + q) * D + tid] = r[q];
+  if (!ptx::mbar_wait_bounded(&bar, 0, &s_abort)) atomicOr(a.err, 2);
+  __syncthreads();
+  // out[d] = sum_c U_V[d][c] o_hat[c]: two threads per dimension, halves of c
+  {
+    const int d = tid & (D - 1), half = tid >> 7;
+    float r = 0.0f;
+#pragma unroll 16
+    for (int c = half * 64; c < half * 64 + 64; ++c) r = fmaf(ut_s[c * D + d], ohat[c], r);
+    osum[half * D + d] = r;
+  }
+  __syncthreads();
+  if (tid < D) a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = osum[tid] + osum[D + tid];
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -956,6 +975,24 @@ __global__ void aatc_dequant_kernel(const uint32_t* words, const float* alpha, c
   }
 }
 
+// Launch with programmatic stream serialization: the kernel may start before the preceding
+// grid in the stream completes; it synchronizes with griddepcontrol.wait before touching
+// anything that grid produces.
+template <typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 template <int WPW, int NP>
 cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
   static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
@@ -965,19 +1002,7 @@ cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStre
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  // programmatic dependent launch: the split kernel's prologue (cache tiles, scales, tables)
-  // overlaps the query kernel; it waits for the query kernel's results before loading them
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.n_splits, a.n_kv, batch);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, aatc_decode_split_kernel<WPW, NP>, a);
+  return launch_pdl(aatc_decode_split_kernel<WPW, NP>, dim3(a.n_splits, a.n_kv, batch), dim3(kThreads), smem, st, a);
 }
 
 template <int NP>
@@ -1045,16 +1070,25 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.ks_stride = wsl.ks_stride;
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
-  a.cnt = reinterpret_cast<int*>(static_cast<char*>(ws) + wsl.cnt_off);
   if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
-  aatc_decode_query_kernel<<<dim3(a.n_kv, batch, 4 * np), kQThreads, 0, st>>>(a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, 4 * np), dim3(kQThreads), 0, st, a);
   if (e != cudaSuccess) return e;
-  const SplitSmem L(n_s, np, sp.split_len, plan.n_words, plan.n_entries, sp.n_splits);
+  const SplitSmem L(n_s, np, sp.split_len, plan.n_words, plan.n_entries);
   const size_t smem = static_cast<size_t>(L.total);
   const int wpw = (nw_v + kWarps - 1) / kWarps;
   if (wpw > 8 || smem > 227 * 1024) return cudaErrorNotSupported;
-  return np == 1 ? launch_split_g<1>(a, batch, wpw, smem, st) : launch_split_g<2>(a, batch, wpw, smem, st);
+  e = np == 1 ? launch_split_g<1>(a, batch, wpw, smem, st) : launch_split_g<2>(a, batch, wpw, smem, st);
+  if (e != cudaSuccess) return e;
+  const size_t msmem = 4 * (static_cast<size_t>(D) * D + ((sp.n_splits + 3) & ~3) + kMWarps * D + D);
+  if (msmem > 227 * 1024) return cudaErrorNotSupported;
+  static size_t msmem_set = 0;
+  if (msmem > msmem_set) {
+    e = cudaFuncSetAttribute(aatc_decode_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(msmem));
+    if (e != cudaSuccess) return e;
+    msmem_set = msmem;
+  }
+  return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msmem, st, a);
 }
 
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n, int max_tokens,
