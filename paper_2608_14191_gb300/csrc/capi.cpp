@@ -65,7 +65,7 @@ aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
   DecodeWs w;
   w.pstride = D + 4;                              // o_c per channel, then m, l (padded)
-  w.ks_stride = 2 * n_words * 32;                 // >= k32-steps x 2 query passes x 32 lanes
+  w.ks_stride = 2 * n_words * 32;                 // >= score k16-steps (<= 2 W) x 32 lanes
   w.qfrag_off = align_up(static_cast<size_t>(batch) * n_q * sp.n_splits * w.pstride * sizeof(float), 256);
   w.qcorr_off = align_up(w.qfrag_off + static_cast<size_t>(batch) * n_kv * w.ks_stride * 16, 256);
   w.bytes = w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float);

@@ -95,68 +95,60 @@ __device__ __forceinline__ float pow2i(int e) { return __int_as_float((127 + e) 
 
 constexpr int kWarps = kThreads / 32;
 
-// Tensor-core formulation: mma.sync m16n8k32 with e4m3 operands and f32 accumulation.
-//  * A packed digit masked into a byte (0..3, or 0..1 for a bit) IS an e4m3 number: the subnormal
-//    digit x 2^-9, so B fragments are one shift and one mask of a record word, four digits each.
-//  * The other operand (folded query, or probability P' = p alpha^V) is split into four e4m3 limbs
-//    with x_0 = x, l_k = rn(x_k), x_{k+1} = 16 (x_k - l_k), so x = sum_k l_k 16^-k + x_4 2^-16:
-//    each limb keeps 4 significant bits, four of them ~16 bits of x, down to |x| ~ 2^-18 of the
-//    largest (|x| <= 256).  Rows 4k + i of A hold limb k of query 4P + i, so lane (g, t) gets
-//    limbs 0 (c0, c1) and 2 (c2, c3) of query g < 4 and lane g + 4 limbs 1 and 3; a query's
-//    value is the 16^-k weighted sum over both lanes.
-//  * The products and their f32 sums are exact for these magnitudes, which was checked on the
-//    hardware (subnormal x subnormal, cancellation of the largest terms).
-//   scores:  B = record digits: a D2 k32-step covers two record words (b0 from word 2i, b1 from
-//            2i+1, byte j of lane t = field t + 4j), a D1 step one word (fields t + 8j and t + 4 + 8j).
-//   values:  B = value digits of four tokens from the quad-interleaved value words; one n-tile per
-//            8 record entries (= one byte-quarter of the record word).
-__device__ __forceinline__ void mma_e4m3(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
+// Tensor-core formulation: mma.sync m16n8k16 with f16 operands and f32 accumulation.
+//  * A packed 2-bit digit (or bit) masked into the low bits of a 16-bit half IS an f16 number:
+//    the subnormal digit * 2^-24.  So an operand register (two digits) is one shift and one AND
+//    of a record word, with no conversion.  (The e4m3 form of the same idea needs fewer masks,
+//    but mma.sync with fp8 operands costs about a dozen instructions per MMA on this GPU, the
+//    f16 form one.)
+//  * The other operand (folded query, or probability P' = p alpha^V) is an f16 hi/lo pair,
+//    hi = f16(x), lo = f16(x - hi), ~22 bits: row g of A holds hi and row g + 8 lo of query g,
+//    so lane (g, t) accumulates hi (c0, c1) and lo (c2, c3) of query g separately and a query's
+//    value is c0 + c2.  Products and their f32 sums were checked on the hardware to be exact for
+//    subnormal digits; the accumulator keeps ~22 bits relative to its own magnitude.
+//   scores:  B = record digits of 8 tokens.  One D2 word is one k16-step: b0 = word >> 2t
+//            (fields t, t + 8), b1 = word >> 2t + 8 (fields t + 4, t + 12); one D1 word is two
+//            k16-steps s: b0 = word >> t + 8s (fields t + 8s, t + 8s + 16), b1 = word >> t + 4 + 8s.
+//   values:  B = value digits of one record entry for tokens (0, 2) and (1, 3) of a token quad,
+//            from the quad-interleaved value words; A = P' of the same tokens in that order.
+__device__ __forceinline__ void mma_f16(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
   asm volatile(
-      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
       "{%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
 }
 
-// next e4m3 limb of x (returned byte); x becomes 16 (x - limb)
-__device__ __forceinline__ uint32_t e4m3_limb(float& x) {
-  const __nv_fp8_storage_t b = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
-  x = 16.0f * (x - __half2float(__half(__nv_cvt_fp8_to_halfraw(b, __NV_E4M3))));
-  return b;
+// f16 hi/lo split of two values, packed as (hi(x), hi(y)) and (lo(x), lo(y)); returns hi + lo.
+__device__ __forceinline__ float2 f16_split2(float x, float y, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(x, y);
+  const float2 hf = __half22float2(h);
+  const __half2 l = __floats2half2_rn(x - hf.x, y - hf.y);
+  const float2 lf = __half22float2(l);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+  return make_float2(hf.x + lf.x, hf.y + lf.y);
 }
-// the same for two values at once (x.x -> low byte)
-__device__ __forceinline__ uint32_t e4m3_limb2(float2& x) {
-  const __nv_fp8x2_storage_t b = __nv_cvt_float2_to_fp8x2(x, __NV_SATFINITE, __NV_E4M3);
-  const float2 v = __half22float2(__half2(__nv_cvt_fp8x2_to_halfraw2(b, __NV_E4M3)));
-  x.x = 16.0f * (x.x - v.x);
-  x.y = 16.0f * (x.y - v.y);
-  return b;
-}
-// a query's value from the accumulators of its two lanes (limbs 0, 2 in lane g < 4; 1, 3 in g + 4)
-__device__ __forceinline__ float2 limb_sum(const float (&c)[4], int g) {
-  const float w0 = g < 4 ? 1.0f : 0.0625f, w2 = g < 4 ? 0.00390625f : 0.000244140625f;
-  float v0 = fmaf(c[2], w2, c[0] * w0), v1 = fmaf(c[3], w2, c[1] * w0);
-  v0 += __shfl_down_sync(0xffffffffu, v0, 16);
-  v1 += __shfl_down_sync(0xffffffffu, v1, 16);
-  return make_float2(v0, v1);
-}
+
+constexpr float kOpMax = 16384.0f;            // |A operand| scaled to <= 2^14 (f16 max 65504)
+constexpr float kDigitScale = 16777216.0f;    // a digit's f16 value is digit * 2^-24
 
 constexpr int kQThreads = 512;
 constexpr int kMaxEntries = 32 * 32;   // 8 bits x 128 channels
 
-// Per call, per (sequence, kv-head, query slot): folded query q'_c = (U_K^T q)_c f_c log2(e)/sqrt(128),
-// its offset correction C = sum_c q'_c 2^(b_c-1), the score scale, and the rows of the score A
-// fragments that hold this query (four e4m3 limbs of q'_c 2^shift / sigma per record entry).
-// Slots G..4P-1 write zero rows.
+// Per call, per (sequence, kv-head, query slot g < 8): folded query q'_c = (U_K^T q)_c f_c
+// log2(e)/sqrt(128), its offset correction C = sum_c q'_c 2^(b_c-1), the score scale, and rows g
+// (hi) and g + 8 (lo) of the score A fragments: q'_c 2^shift per record entry, scaled so the
+// largest is 2^14.  Slots g >= G write zero rows.
 __global__ void __launch_bounds__(kQThreads)
     aatc_decode_query_kernel(const DecodeArgs a) {
   __shared__ float qv[D];
   __shared__ float part[4][D];
   __shared__ float xq[D];
   __shared__ float red[2][D / 32];
-  __shared__ uint8_t lb[4][kMaxEntries];
+  __shared__ float xe[kMaxEntries];
   const int head = blockIdx.x, b = blockIdx.y, slot = blockIdx.z, tid = threadIdx.x;
-  const int G = a.group, NP = (G + 3) / 4;
+  const int G = a.group;
   const bool real = slot < G;
   const int sk = (a.layer * a.n_kv + head) * 2;
   ptx::grid_launch_dependents();
@@ -209,46 +201,48 @@ __global__ void __launch_bounds__(kQThreads)
   __syncthreads();
   const float C = red[0][0] + red[0][1] + red[0][2] + red[0][3];
   const float m = fmaxf(fmaxf(red[1][0], red[1][1]), fmaxf(red[1][2], red[1][3]));
-  const float inv = m > 0.0f ? 256.0f / m : 0.0f;                        // coefficients to |.| <= 256
+  const float inv = m > 0.0f ? kOpMax / m : 0.0f;                       // coefficients to |.| <= 2^14
   const int n_used = lk.n2 + lk.n1;
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int e = tid + h * kQThreads;
     if (e < n_used) {
       const int ce = h ? ce1 : ce0;
-      float v = xq[ce & 0xFF] * inv * pow2i(ce >> 8);
-#pragma unroll
-      for (int k = 0; k < 4; ++k) lb[k][e] = static_cast<uint8_t>(e4m3_limb(v));
+      xe[e] = real ? xq[ce & 0xFF] * inv * pow2i(ce >> 8) : 0.0f;
     }
   }
   __syncthreads();
-  const int n2w = lk.n2 / 16, n2s = (n2w + 1) / 2, n1w = (lk.n1 + 31) / 32;
-  const int n_s = n2s + n1w;
-  const int P = slot >> 2, qq = slot & 3;
-  uint32_t* dst = reinterpret_cast<uint32_t*>(a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride);
-  for (int i = tid; i < n_s * 32; i += kQThreads) {
-    const int st = i >> 5, w = i & 31;
-    const int g = (w >> 4) ? 4 + qq : qq, t = (w >> 2) & 3, rr = w & 3;
-    const int row = g + 8 * (rr & 1), limb = row >> 2, khalf = rr >> 1;
-    uint32_t r = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      int e = -1;
-      if (st < n2s) {
-        const int wd = 2 * st + khalf;
-        if (wd < n2w) e = 16 * wd + t + 4 * j;
-      } else {
-        const int fld = t + 8 * j + 4 * khalf;
-        if (32 * (st - n2s) + fld < lk.n1) e = lk.n2 + 32 * (st - n2s) + fld;
-      }
-      if (e >= 0 && real) r |= static_cast<uint32_t>(lb[limb][e]) << (8 * j);
+  // fragment of lane (slot, t) for k-step ks: registers (row slot, k 2t | 2t+1), (row slot + 8,
+  // same k), (row slot, k 2t+8 | 2t+9), (row slot + 8, ...)
+  const int n2w = lk.n2 / 16, n1w = (lk.n1 + 31) / 32;
+  const int n_ks = n2w + 2 * n1w;
+  uint4* dst = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
+  for (int i = tid; i < n_ks * 4; i += kQThreads) {
+    const int ks = i >> 2, t = i & 3;
+    int f[4];                                          // record fields of k = 2t, 2t+1, 2t+8, 2t+9
+    int base, lim;
+    if (ks < n2w) {
+      f[0] = t; f[1] = t + 8; f[2] = t + 4; f[3] = t + 12;
+      base = 16 * ks;
+      lim = 16;
+    } else {
+      const int u = (ks - n2w) >> 1, sh = 8 * ((ks - n2w) & 1);
+      f[0] = t + sh; f[1] = t + sh + 16; f[2] = t + 4 + sh; f[3] = t + 4 + sh + 16;
+      base = lk.n2 + 32 * u;
+      lim = min(32, lk.n1 - 32 * u);
     }
-    dst[((st * NP + P) * 32 + 4 * g + t) * 4 + rr] = r;
+    float v[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = f[k] < lim ? xe[base + f[k]] : 0.0f;
+    uint32_t h01, l01, h89, l89;
+    f16_split2(v[0], v[1], h01, l01);
+    f16_split2(v[2], v[3], h89, l89);
+    dst[ks * 32 + 4 * slot + t] = make_uint4(h01, l01, h89, l89);
   }
   if (tid == 0) {
     float* qc = a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP;
     qc[slot] = real ? C : 0.0f;
-    qc[MAX_GROUP + slot] = m > 0.0f ? m * (512.0f / 256.0f) : 0.0f;       // limb units x digit 2^9
+    qc[MAX_GROUP + slot] = m > 0.0f ? m * (kDigitScale / kOpMax) : 0.0f;  // raw sum -> sum q' code
   }
 }
 
@@ -259,19 +253,19 @@ __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 // shared-memory carve-up of the split kernel (byte offsets)
 struct SplitSmem {
   int bars, qcg, red, cetab, etab, afrag, ak, av, sbuf, pq, ring, total, sb_stride;
-  __host__ __device__ SplitSmem(int n_steps, int np, int split_len, int W, int n_entries) {
+  __host__ __device__ SplitSmem(int n_ks, int np, int split_len, int W, int n_entries) {
     int o = 0;
     bars = o;  o = align16(o + 8 * (kStages + 1));  // ring barriers, then the prologue barrier
     qcg = o;   o += 2 * MAX_GROUP * 4;              // offset corrections, score scales
     red = o;   o += 4 * kWarps * MAX_GROUP * 4;     // reductions; per-query m, l, S', split max
     cetab = o; o += D * 8 * 2;                      // record entries of each value channel
     etab = o;  o = align16(o + n_entries * 2);      // value entry table (channel | shift << 8)
-    afrag = o; o += n_steps * np * 32 * 16;         // score A fragments per (k-step, pass, lane)
+    afrag = o; o += n_ks * 32 * 16;                 // score A fragments per (k-step, lane)
     ak = o;    o += split_len * 4;                  // alpha^K, alpha^V of the split
     av = o;    o += split_len * 4;
     sb_stride = split_len + 8;                      // padded: query rows fall in different banks
     sbuf = o;  o += 4 * np * sb_stride * 4;         // scores of the split
-    pq = o;    o += 4 * np * 32 * 16;               // P' limb fragments of one tile
+    pq = o;    o += (TILE / 16) * 32 * 16;          // P' A fragments of one tile (8 k16-steps)
     ring = o;  o += kStages * W * TILE * 4;         // after the last tile: value entry sums
     total = o;
   }
@@ -282,8 +276,7 @@ struct SplitSmem {
 // query fragments and the value entry tables arrive by bulk copy in the prologue.
 // Pass 1: scores of the split; pass 2: P' and the value entry sums; then the entry sums become
 // channel sums o_c = sum_e 2^shift O_e - 2^(b_c-1) S' (the Eq. 12 offset, folded after the
-// product), written with m and l.  The CTA that finishes its head's last split merges all of
-// them (log-sum-exp), scales by f^V / l and applies U_V.
+// product), written with the split's m and l for the merge kernel.
 template <int WPW, int NP>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
@@ -296,21 +289,21 @@ __global__ void __launch_bounds__(kThreads)
   const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;   // key / value streams
   const StreamLayout lk = a.lay[sk], lv = a.lay[sv];
   const int W = a.n_words;
-  const int n2w_k = lk.n2 / 16, n2s_k = (n2w_k + 1) / 2, n1w_k = (lk.n1 + 31) / 32;
-  const int n_s = n2s_k + n1w_k;
+  const int n2w_k = lk.n2 / 16, n1w_k = (lk.n1 + 31) / 32;
+  const int n_ks = n2w_k + 2 * n1w_k;                          // score k16-steps
   const int n2w_v = lv.n2 / 16, nw_v = n2w_v + (lv.n1 + 31) / 32;
-  const SplitSmem L(n_s, NP, a.split_len, W, a.n_entries);
+  const SplitSmem L(n_ks, NP, a.split_len, W, a.n_entries);
   uint64_t* full = reinterpret_cast<uint64_t*>(smb + L.bars);
   uint64_t* pro = full + kStages;
   float* qcg = reinterpret_cast<float*>(smb + L.qcg);          // [0..7] C_g, [8..15] score scales
   float* red = reinterpret_cast<float*>(smb + L.red);
   const short* cetab = reinterpret_cast<const short*>(smb + L.cetab);
   const short* etab = reinterpret_cast<const short*>(smb + L.etab);
-  uint4* afrag = reinterpret_cast<uint4*>(smb + L.afrag);
+  const uint4* afrag = reinterpret_cast<const uint4*>(smb + L.afrag);
   float* ak = reinterpret_cast<float*>(smb + L.ak);
   float* av = reinterpret_cast<float*>(smb + L.av);
   float* sbuf = reinterpret_cast<float*>(smb + L.sbuf);        // [4 NP][sb_stride]
-  uint4* pq = reinterpret_cast<uint4*>(smb + L.pq);            // [4 k32-steps][NP][32 lanes]
+  uint4* pq = reinterpret_cast<uint4*>(smb + L.pq);            // [8 k16-steps][32 lanes]
   uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
   const int sbs = L.sb_stride;
 
@@ -321,7 +314,7 @@ __global__ void __launch_bounds__(kThreads)
   const int t_end = min(a.n_ctx, tile_hi * TILE);
   const int n_tiles_split = tile_hi - tile_lo;
   const int n_seq = 2 * n_tiles_split;                         // key tiles, then value tiles
-  const int tile0 = t_begin / TILE;
+  const int tile0 = tile_lo;
   const uint32_t tile_bytes = static_cast<uint32_t>(W) * TILE * 4;
   const size_t stream_words = static_cast<size_t>(a.n_tiles) * W * TILE;
   const size_t bk = (static_cast<size_t>(b) * a.n_kv + head) * 2;   // cache stream of the keys
@@ -340,7 +333,7 @@ __global__ void __launch_bounds__(kThreads)
     ptx::bulk_load(ring + s * W * TILE, src, tile_bytes, full + s);
   };
   auto wait_tile = [&](int i) {
-    if (!ptx::mbar_wait_bounded(full + i % kStages, (i / kStages) & 1, &s_abort)) {
+    if (!ptx::mbar_wait_sleep(full + i % kStages, (i / kStages) & 1, &s_abort, 32)) {
       s_abort = 1;
       atomicOr(a.err, 2);
     }
@@ -350,88 +343,76 @@ __global__ void __launch_bounds__(kThreads)
     for (int s2 = 0; s2 <= kStages; ++s2) ptx::mbar_init(full + s2, 1);
     ptx::fence_mbar_init();
     // cache words and scales do not depend on the query kernel: start them first
-    for (int i = 0; i < min(kStages, n_seq); ++i) issue_tile(i);
     const uint32_t abytes = static_cast<uint32_t>(n_tiles_split) * TILE * 4;
     const uint32_t ebytes = static_cast<uint32_t>(align16(a.n_entries * 2));
-    const uint32_t fbytes = static_cast<uint32_t>(n_s) * NP * 32 * 16;
+    const uint32_t fbytes = static_cast<uint32_t>(n_ks) * 32 * 16;
     ptx::mbar_arrive_expect_tx(pro, 2 * abytes + D * 8 * 2 + ebytes + fbytes + 2 * MAX_GROUP * 4);
     ptx::bulk_load(ak, kalpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
+    for (int i = 0; i < min(kStages, n_seq); ++i) issue_tile(i);
     ptx::bulk_load(av, valpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
     ptx::bulk_load(smb + L.cetab, a.chan_ent + static_cast<size_t>(sv) * D * 8, D * 8 * 2, pro);
     ptx::bulk_load(smb + L.etab, a.entry + static_cast<size_t>(sv) * a.n_entries, ebytes, pro);
     // the query kernel's fragments and corrections
     ptx::grid_dependency_wait();
-    ptx::bulk_load(afrag, a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride, fbytes, pro);
+    ptx::bulk_load(smb + L.afrag, a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride, fbytes, pro);
     ptx::bulk_load(qcg, a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP, 2 * MAX_GROUP * 4, pro);
   }
+  // P' rows of absent queries (g >= G) stay zero for the whole split
+  for (int i = tid; i < (TILE / 16) * 32; i += kThreads)
+    if (((i & 31) >> 2) >= G) pq[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncthreads();
-  if (!ptx::mbar_wait_bounded(pro, 0, &s_abort)) {
+  if (!ptx::mbar_wait_sleep(pro, 0, &s_abort, 200)) {
     s_abort = 1;
     atomicOr(a.err, 2);
   }
 
   // ---- pass 1: scores; warp = 32 tokens of each tile as four n-tiles of 8
-  float mloc[NP];
-#pragma unroll
-  for (int p = 0; p < NP; ++p) mloc[p] = -INFINITY;
+  float mloc = -INFINITY;                                      // lanes g < G: query g
+  const float sg = g < G ? qcg[MAX_GROUP + g] : 0.0f, cg = g < G ? qcg[g] : 0.0f;
   for (int ti = 0; ti < n_tiles_split; ++ti) {
     wait_tile(ti);
     const uint32_t* kt = ring + (ti % kStages) * W * TILE + 32 * warp + g;
-    float acc[4][NP][4];
+    float acc[4][4];
 #pragma unroll
     for (int j = 0; j < 4; ++j)
 #pragma unroll
-      for (int p = 0; p < NP; ++p)
-#pragma unroll
-        for (int r = 0; r < 4; ++r) acc[j][p][r] = 0.0f;
-    for (int st = 0; st < n2s_k; ++st) {
-      uint4 af[NP];
-#pragma unroll
-      for (int p = 0; p < NP; ++p) af[p] = afrag[(st * NP + p) * 32 + lane];
-      const uint32_t* w0 = kt + (2 * st) * TILE;
-      const uint32_t* w1 = kt + min(2 * st + 1, W - 1) * TILE;    // past D2: its A bytes are zero
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t b0 = (w0[8 * j] >> (2 * t)) & 0x03030303u;
-        const uint32_t b1 = (w1[8 * j] >> (2 * t)) & 0x03030303u;
-#pragma unroll
-        for (int p = 0; p < NP; ++p) mma_e4m3(acc[j][p], af[p], b0, b1);
-      }
-    }
-    for (int u = 0; u < n1w_k; ++u) {
-      uint4 af[NP];
-#pragma unroll
-      for (int p = 0; p < NP; ++p) af[p] = afrag[((n2s_k + u) * NP + p) * 32 + lane];
-      const uint32_t* w0 = kt + (n2w_k + u) * TILE;
+      for (int r = 0; r < 4; ++r) acc[j][r] = 0.0f;
+    for (int ks = 0; ks < n2w_k; ++ks) {
+      const uint4 af = afrag[ks * 32 + lane];
+      const uint32_t* w0 = kt + ks * TILE;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t x = w0[8 * j];
-        const uint32_t b0 = (x >> t) & 0x01010101u;
-        const uint32_t b1 = (x >> (t + 4)) & 0x01010101u;
-#pragma unroll
-        for (int p = 0; p < NP; ++p) mma_e4m3(acc[j][p], af[p], b0, b1);
+        mma_f16(acc[j], af, (x >> (2 * t)) & 0x00030003u, (x >> (2 * t + 8)) & 0x00030003u);
       }
     }
-    const int tbase = (tile0 + ti) * TILE;
+    for (int u = 0; u < n1w_k; ++u) {
+      const uint32_t* w0 = kt + (n2w_k + u) * TILE;
+      uint32_t x[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
+      for (int j = 0; j < 4; ++j) x[j] = w0[8 * j];
 #pragma unroll
-      for (int p = 0; p < NP; ++p) {
-        const float2 v = limb_sum(acc[j][p], g);
-        const float v0 = v.x, v1 = v.y;
-        const int q = 4 * p + g;
-        if (g < 4 && q < G) {
-          const float sg = qcg[MAX_GROUP + q], c0 = qcg[q];
-          const int tk = 32 * warp + 8 * j + 2 * t;
-          const float2 a2 = *reinterpret_cast<const float2*>(ak + ti * TILE + tk);
-          float s0 = a2.x * fmaf(v0, sg, -c0);
-          float s1 = a2.y * fmaf(v1, sg, -c0);
-          s0 = tbase + tk < t_end ? s0 : -INFINITY;
-          s1 = tbase + tk + 1 < t_end ? s1 : -INFINITY;
-          *reinterpret_cast<float2*>(sbuf + q * sbs + ti * TILE + tk) = make_float2(s0, s1);
-          mloc[p] = fmaxf(mloc[p], fmaxf(s0, s1));
-        }
+      for (int hs = 0; hs < 2; ++hs) {
+        const uint4 af = afrag[(n2w_k + 2 * u + hs) * 32 + lane];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          mma_f16(acc[j], af, (x[j] >> (t + 8 * hs)) & 0x00010001u, (x[j] >> (t + 4 + 8 * hs)) & 0x00010001u);
       }
+    }
+    if (g < G) {
+      const int tbase = (tile0 + ti) * TILE;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int tk = 32 * warp + 8 * j + 2 * t;
+        const float2 a2 = *reinterpret_cast<const float2*>(ak + ti * TILE + tk);
+        float s0 = a2.x * fmaf(acc[j][0] + acc[j][2], sg, -cg);
+        float s1 = a2.y * fmaf(acc[j][1] + acc[j][3], sg, -cg);
+        s0 = tbase + tk < t_end ? s0 : -INFINITY;
+        s1 = tbase + tk + 1 < t_end ? s1 : -INFINITY;
+        *reinterpret_cast<float2*>(sbuf + g * sbs + ti * TILE + tk) = make_float2(s0, s1);
+        mloc = fmaxf(mloc, fmaxf(s0, s1));
+      }
+    }
     __syncthreads();                                           // stage free: refill
     if (tid == 0 && ti + kStages < n_seq) {
       ptx::fence_proxy_async_smem();
@@ -444,45 +425,38 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) amx = fmaxf(amx, __shfl_xor_sync(0xffffffffu, amx, o));
   if (lane == 0) red[3 * kWarps * MAX_GROUP + warp] = amx;
-#pragma unroll
-  for (int p = 0; p < NP; ++p) {
-    float m = mloc[p];
-    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
-    if (t == 0 && g < 4) red[warp * MAX_GROUP + 4 * p + g] = m;
-  }
+  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 1));
+  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 2));
+  if (t == 0) red[warp * MAX_GROUP + g] = mloc;
   __syncthreads();
   float* mqs = red + 2 * kWarps * MAX_GROUP + 3 * MAX_GROUP;  // [MAX_GROUP] split max per query
-  if (tid < 4 * NP)
+  if (tid < MAX_GROUP)
     mqs[tid] = fmaxf(fmaxf(red[0 * MAX_GROUP + tid], red[1 * MAX_GROUP + tid]),
                      fmaxf(red[2 * MAX_GROUP + tid], red[3 * MAX_GROUP + tid]));
   {
     const float* am = red + 3 * kWarps * MAX_GROUP;
     amx = fmaxf(fmaxf(am[0], am[1]), fmaxf(am[2], am[3]));
   }
-  const float inv_p = amx > 0.0f ? 256.0f / amx : 0.0f;       // P' to |.| <= 256
-  const float val_scale = amx * (512.0f / 256.0f);             // limb units x digit 2^9
+  const float inv_p = amx > 0.0f ? kOpMax / amx : 0.0f;       // P' to |.| <= 2^14
+  const float val_scale = amx * (kDigitScale / kOpMax);        // raw sum -> sum P' code
   __syncthreads();                                             // split maxima visible to pass 2
 
-  // ---- pass 2: P' limbs (thread = 4 tokens x 1 query) and the value product over the split
+  // ---- pass 2: P' (thread = 4 tokens x 1 query) and the value product over the split
   const int vw0 = warp * nw_v / kWarps, vw1 = (warp + 1) * nw_v / kWarps;
-  float vacc[WPW][4][NP][4];
+  float vacc[WPW][4][4];
 #pragma unroll
   for (int i = 0; i < WPW; ++i)
 #pragma unroll
     for (int r = 0; r < 4; ++r)
 #pragma unroll
-      for (int p = 0; p < NP; ++p)
-#pragma unroll
-        for (int z = 0; z < 4; ++z) vacc[i][r][p][z] = 0.0f;
+      for (int z = 0; z < 4; ++z) vacc[i][r][z] = 0.0f;
   float lsum[NP], ssum[NP];
 #pragma unroll
   for (int p = 0; p < NP; ++p) lsum[p] = ssum[p] = 0.0f;
-  uint32_t* pqw = reinterpret_cast<uint32_t*>(pq);
   {
-    // tokens 32 warp + 4 Qk .. +3 (k = 4 Qk + j in the warp's k32 chunk), query 4 p + qq
-    const int qq = lane >> 3, Qk = lane & 7, t4 = Qk & 3, h2 = (Qk >> 2) * 2;
-    const int tk0 = 32 * warp + 4 * Qk;
+    // tokens 4 Q .. 4 Q + 3 with Q = 8 warp + Qk (k16-step Q / 4, fragment lane column t = Q % 4)
+    const int qq = lane >> 3, Qk = lane & 7, Q = 8 * warp + Qk;
+    const int tk0 = 4 * Q;
     for (int ti = 0; ti < n_tiles_split; ++ti) {
       const int i_seq = n_tiles_split + ti;
       wait_tile(i_seq);
@@ -495,62 +469,42 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
         for (int p = 0; p < NP; ++p) {
           const int q = 4 * p + qq;
-          float4 pr = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
           if (q < G) {
             const float4 sc = *reinterpret_cast<const float4*>(sbuf + q * sbs + ti * TILE + tk0);
             const float mq = mqs[q];
-            pr = make_float4(fast_exp2(sc.x - mq), fast_exp2(sc.y - mq), fast_exp2(sc.z - mq), fast_exp2(sc.w - mq));
+            const float p0 = fast_exp2(sc.x - mq), p1 = fast_exp2(sc.y - mq);
+            const float p2 = fast_exp2(sc.z - mq), p3 = fast_exp2(sc.w - mq);
+            lsum[p] += (p0 + p1) + (p2 + p3);
+            uint32_t h02, l02, h13, l13;
+            const float2 r02 = f16_split2(p0 * av0, p2 * av2, h02, l02);   // tokens 0, 2 (k 2t, 2t+1)
+            const float2 r13 = f16_split2(p1 * av1, p3 * av3, h13, l13);   // tokens 1, 3 (k 2t+8, 2t+9)
+            ssum[p] += (r02.x + r02.y) + (r13.x + r13.y);                  // what the MMA sees
+            pq[(Q >> 2) * 32 + 4 * q + (Q & 3)] = make_uint4(h02, l02, h13, l13);
           }
-          lsum[p] += (pr.x + pr.y) + (pr.z + pr.w);
-          float2 x01 = make_float2(pr.x * av0, pr.y * av1), x23 = make_float2(pr.z * av2, pr.w * av3);
-          const float xs = (x01.x + x01.y) + (x23.x + x23.y);
-          uint32_t* base = pqw + ((warp * NP + p) * 32 + t4) * 4 + h2;
-#pragma unroll
-          for (int l = 0; l < 4; ++l) {
-            const uint32_t lo = e4m3_limb2(x01), hi = e4m3_limb2(x23);
-            // row 4 l + qq: lane group (4 l + qq) & 7, register + 1 for rows >= 8
-            base[((4 * l + qq) & 7) * 16 + (l >> 1)] = lo | (hi << 16);
-          }
-          ssum[p] += fmaf((x01.x + x01.y) + (x23.x + x23.y), -1.52587890625e-05f, xs);   // value of the limbs
         }
       }
       __syncthreads();
-#pragma unroll
-      for (int kp = 0; kp < 4; ++kp) {
-        uint4 af[NP];
-#pragma unroll
-        for (int p = 0; p < NP; ++p) af[p] = pq[(kp * NP + p) * 32 + lane];
-        const int q0 = 8 * kp + t, q1 = q0 + 4;                  // token quads of b0 / b1
+#pragma unroll 2
+      for (int ks = 0; ks < TILE / 16; ++ks) {
+        const uint4 af = pq[ks * 32 + lane];
+        const int Qv = 4 * ks + t;                                // token quad of this lane's B column
 #pragma unroll
         for (int i = 0; i < WPW; ++i) {
           const int wd = vw0 + i;
           if (wd < vw1) {
             if (wd < n2w_v) {
-              const uint2 x0 = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * q0 + 2 * (g >> 2));
-              const uint2 x1 = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * q1 + 2 * (g >> 2));
+              // quarters g>>2 (n-tile 0) and 2 + (g>>2) (n-tile 1) sit in adjacent slots
+              const uint2 x = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * Qv + 2 * (g >> 2));
               const int sh = 2 * (g & 3);
-              const uint32_t lo0 = (x0.x >> sh) & 0x03030303u, lo1 = (x1.x >> sh) & 0x03030303u;
-              const uint32_t hi0 = (x0.y >> sh) & 0x03030303u, hi1 = (x1.y >> sh) & 0x03030303u;
-#pragma unroll
-              for (int p = 0; p < NP; ++p) {
-                mma_e4m3(vacc[i][0][p], af[p], lo0, lo1);
-                mma_e4m3(vacc[i][1][p], af[p], hi0, hi1);
-              }
+              mma_f16(vacc[i][0], af, (x.x >> sh) & 0x00030003u, (x.x >> (sh + 8)) & 0x00030003u);
+              mma_f16(vacc[i][1], af, (x.y >> sh) & 0x00030003u, (x.y >> (sh + 8)) & 0x00030003u);
             } else {
-              const uint4 x0 = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * q0);
-              const uint4 x1 = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * q1);
-              const uint32_t m1 = 0x01010101u;
-              const uint32_t c00 = (x0.x >> g) & m1, c01 = (x1.x >> g) & m1;   // quarter 0
-              const uint32_t c10 = (x0.z >> g) & m1, c11 = (x1.z >> g) & m1;   // quarter 1
-              const uint32_t c20 = (x0.y >> g) & m1, c21 = (x1.y >> g) & m1;   // quarter 2
-              const uint32_t c30 = (x0.w >> g) & m1, c31 = (x1.w >> g) & m1;   // quarter 3
-#pragma unroll
-              for (int p = 0; p < NP; ++p) {
-                mma_e4m3(vacc[i][0][p], af[p], c00, c01);
-                mma_e4m3(vacc[i][1][p], af[p], c10, c11);
-                mma_e4m3(vacc[i][2][p], af[p], c20, c21);
-                mma_e4m3(vacc[i][3][p], af[p], c30, c31);
-              }
+              const uint4 x = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * Qv);
+              // quarter r sits in slot (0, 2, 1, 3)[r]
+              mma_f16(vacc[i][0], af, (x.x >> g) & 0x00010001u, (x.x >> (g + 8)) & 0x00010001u);
+              mma_f16(vacc[i][1], af, (x.z >> g) & 0x00010001u, (x.z >> (g + 8)) & 0x00010001u);
+              mma_f16(vacc[i][2], af, (x.y >> g) & 0x00010001u, (x.y >> (g + 8)) & 0x00010001u);
+              mma_f16(vacc[i][3], af, (x.w >> g) & 0x00010001u, (x.w >> (g + 8)) & 0x00010001u);
             }
           }
         }
@@ -563,7 +517,7 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
 
-  // ---- per-query m, l, S' of the split; value entry sums into shared memory (staging area)
+  // ---- per-query m, l, S' of the split; value entry sums into shared memory (drained ring)
 #pragma unroll
   for (int p = 0; p < NP; ++p)
 #pragma unroll
@@ -578,21 +532,18 @@ __global__ void __launch_bounds__(kThreads)
       red[warp * MAX_GROUP + 4 * p + (lane >> 3)] = lsum[p];
       red[(kWarps + warp) * MAX_GROUP + 4 * p + (lane >> 3)] = ssum[p];
     }
-#pragma unroll
-  for (int p = 0; p < NP; ++p) {
+  if (g < G) {
 #pragma unroll
     for (int i = 0; i < WPW; ++i) {
       const int wd = vw0 + i;
-      const bool have = wd < vw1;
-      const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
-      const int nq = wd < n2w_v ? 2 : 4;
+      if (wd < vw1) {
+        const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
+        const int nq = wd < n2w_v ? 2 : 4;
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const float2 v = limb_sum(vacc[i][r][p], g);
-        const int q = 4 * p + g;
-        if (have && r < nq && g < 4 && q < G)
-          *reinterpret_cast<float2*>(oe + q * a.n_entries + ebase + 8 * r + 2 * t) =
-              make_float2(v.x * val_scale, v.y * val_scale);
+        for (int r = 0; r < 4; ++r)
+          if (r < nq)
+            *reinterpret_cast<float2*>(oe + g * a.n_entries + ebase + 8 * r + 2 * t) =
+                make_float2((vacc[i][r][0] + vacc[i][r][2]) * val_scale, (vacc[i][r][1] + vacc[i][r][3]) * val_scale);
       }
     }
   }
@@ -604,7 +555,7 @@ __global__ void __launch_bounds__(kThreads)
     ml[MAX_GROUP + q] = red[q] + red[MAX_GROUP + q] + red[2 * MAX_GROUP + q] + red[3 * MAX_GROUP + q];
     ml[2 * MAX_GROUP + q] = (red[(kWarps + 0) * MAX_GROUP + q] + red[(kWarps + 1) * MAX_GROUP + q] +
                              red[(kWarps + 2) * MAX_GROUP + q] + red[(kWarps + 3) * MAX_GROUP + q]) *
-                            (amx / 256.0f);
+                            (amx / kOpMax);
   }
   __syncthreads();
   // channel sums of this split: thread = channel
@@ -730,7 +681,7 @@ __global__ void __launch_bounds__(kMThreads)
     for (int w = 0; w < kMWarps; ++w) lt += red[1][w];
     ohat[tid] = o * fv / lt;
   }
-  if (!ptx::mbar_wait_bounded(&bar, 0, &s_abort)) atomicOr(a.err, 2);
+  if (!ptx::mbar_wait_sleep(&bar, 0, &s_abort, 100)) atomicOr(a.err, 2);
   __syncthreads();
   // out[d] = sum_c U_V[d][c] o_hat[c]: two threads per dimension, halves of c
   {
@@ -1057,11 +1008,11 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_splits = sp.n_splits;
   a.split_len = sp.split_len;
   // largest key k-step count and value word count over the layer's streams
-  int n_s = 1, nw_v = 1;
+  int n_ks = 1, nw_v = 1;
   for (int h = 0; h < a.n_kv; ++h) {
     const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
     const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
-    n_s = std::max(n_s, (lk.n2 / 16 + 1) / 2 + (lk.n1 + 31) / 32);
+    n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
     nw_v = std::max(nw_v, lv.n2 / 16 + (lv.n1 + 31) / 32);
   }
   const int np = (a.group + 3) / 4;
@@ -1071,9 +1022,9 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
   if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
-  cudaError_t e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, 4 * np), dim3(kQThreads), 0, st, a);
+  cudaError_t e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, MAX_GROUP), dim3(kQThreads), 0, st, a);
   if (e != cudaSuccess) return e;
-  const SplitSmem L(n_s, np, sp.split_len, plan.n_words, plan.n_entries);
+  const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
   const size_t smem = static_cast<size_t>(L.total);
   const int wpw = (nw_v + kWarps - 1) / kWarps;
   if (wpw > 8 || smem > 227 * 1024) return cudaErrorNotSupported;
