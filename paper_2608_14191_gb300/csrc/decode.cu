@@ -82,6 +82,7 @@ struct DecodeArgs {
   uint4* qfrag;            // workspace: score A fragments [batch][n_kv][ks_stride]
   float* qcorr;            // workspace: [batch][n_kv][16]: offset corrections C_g, score scales
   int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len, ks_stride, pstride;
+  int num_sms, cta_per_sm;  // split-kernel work permutation (cta_per_sm = 0: identity)
 };
 
 // 2^x with the hardware approximation (relative error ~2^-22; -inf -> 0)
@@ -277,12 +278,18 @@ struct SplitSmem {
 // Pass 1: scores of the split; pass 2: P' and the value entry sums; then the entry sums become
 // channel sums o_c = sum_e 2^shift O_e - 2^(b_c-1) S' (the Eq. 12 offset, folded after the
 // product), written with the split's m and l for the merge kernel.
-template <int WPW, int NP>
+template <int JPW, int NP>
 __global__ void __launch_bounds__(kThreads)
     aatc_decode_split_kernel(const DecodeArgs a) {
   extern __shared__ __align__(128) unsigned char smb[];
   __shared__ int s_abort;
-  const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
+  // Work item of this CTA.  CTAs i, i + S, i + 2S, ... (S SMs) tend to share an SM, and split
+  // lengths follow a floor pattern with period S in that order, so without a permutation an SM
+  // would get k splits of the same length; item = (i mod S) k + i / S gives every SM k
+  // consecutive items instead (a near-equal share of tiles).
+  int item = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
+  if (a.cta_per_sm > 0) item = (item % a.num_sms) * a.cta_per_sm + item / a.num_sms;
+  const int split = item % a.n_splits, head = (item / a.n_splits) % a.n_kv, b = item / (a.n_splits * a.n_kv);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t = lane & 3;                       // mma fragment coordinates
   const int G = a.group;
@@ -442,14 +449,32 @@ __global__ void __launch_bounds__(kThreads)
   __syncthreads();                                             // split maxima visible to pass 2
 
   // ---- pass 2: P' (thread = 4 tokens x 1 query) and the value product over the split
-  const int vw0 = warp * nw_v / kWarps, vw1 = (warp + 1) * nw_v / kWarps;
-  float vacc[WPW][4][4];
+  // Value n-tile jobs: a D2 word is two n-tiles (byte-quarters 0,1 and 2,3), a D1 word four
+  // (one per quarter).  Warp w takes jobs [w J / 4, (w+1) J / 4); per job this lane keeps the
+  // offset of its slot in the tile (k16-step 0), its field shift and its mask.
+  const int n_jobs = 2 * n2w_v + 4 * (nw_v - n2w_v);
+  const int j0 = warp * n_jobs / kWarps, nj = (warp + 1) * n_jobs / kWarps - j0;
+  int joff[JPW], jsh[JPW];
+  uint32_t jmask[JPW];
 #pragma unroll
-  for (int i = 0; i < WPW; ++i)
+  for (int j = 0; j < JPW; ++j) {
+    const int jj = j0 + j;
+    if (jj < 2 * n2w_v) {
+      joff[j] = (jj >> 1) * TILE + 4 * t + 2 * (g >> 2) + (jj & 1);
+      jsh[j] = 2 * (g & 3);
+      jmask[j] = 0x00030003u;
+    } else {
+      const int u = jj - 2 * n2w_v, r = u & 3;
+      joff[j] = (n2w_v + (u >> 2)) * TILE + 4 * t + ((r & 1) << 1) + (r >> 1);   // slot (0, 2, 1, 3)[r]
+      jsh[j] = g;
+      jmask[j] = 0x00010001u;
+    }
+  }
+  float vacc[JPW][4];
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
+  for (int j = 0; j < JPW; ++j)
 #pragma unroll
-      for (int z = 0; z < 4; ++z) vacc[i][r][z] = 0.0f;
+    for (int z = 0; z < 4; ++z) vacc[j][z] = 0.0f;
   float lsum[NP], ssum[NP];
 #pragma unroll
   for (int p = 0; p < NP; ++p) lsum[p] = ssum[p] = 0.0f;
@@ -484,30 +509,15 @@ __global__ void __launch_bounds__(kThreads)
         }
       }
       __syncthreads();
-#pragma unroll 2
-      for (int ks = 0; ks < TILE / 16; ++ks) {
-        const uint4 af = pq[ks * 32 + lane];
-        const int Qv = 4 * ks + t;                                // token quad of this lane's B column
 #pragma unroll
-        for (int i = 0; i < WPW; ++i) {
-          const int wd = vw0 + i;
-          if (wd < vw1) {
-            if (wd < n2w_v) {
-              // quarters g>>2 (n-tile 0) and 2 + (g>>2) (n-tile 1) sit in adjacent slots
-              const uint2 x = *reinterpret_cast<const uint2*>(vt + wd * TILE + 4 * Qv + 2 * (g >> 2));
-              const int sh = 2 * (g & 3);
-              mma_f16(vacc[i][0], af, (x.x >> sh) & 0x00030003u, (x.x >> (sh + 8)) & 0x00030003u);
-              mma_f16(vacc[i][1], af, (x.y >> sh) & 0x00030003u, (x.y >> (sh + 8)) & 0x00030003u);
-            } else {
-              const uint4 x = *reinterpret_cast<const uint4*>(vt + wd * TILE + 4 * Qv);
-              // quarter r sits in slot (0, 2, 1, 3)[r]
-              mma_f16(vacc[i][0], af, (x.x >> g) & 0x00010001u, (x.x >> (g + 8)) & 0x00010001u);
-              mma_f16(vacc[i][1], af, (x.z >> g) & 0x00010001u, (x.z >> (g + 8)) & 0x00010001u);
-              mma_f16(vacc[i][2], af, (x.y >> g) & 0x00010001u, (x.y >> (g + 8)) & 0x00010001u);
-              mma_f16(vacc[i][3], af, (x.w >> g) & 0x00010001u, (x.w >> (g + 8)) & 0x00010001u);
-            }
+      for (int ks = 0; ks < TILE / 16; ++ks) {
+        const uint4 af = pq[ks * 32 + lane];                   // B column token quad 4 ks + t
+#pragma unroll
+        for (int j = 0; j < JPW; ++j)
+          if (j < nj) {
+            const uint32_t x = vt[joff[j] + 16 * ks];
+            mma_f16(vacc[j], af, (x >> jsh[j]) & jmask[j], (x >> (jsh[j] + 8)) & jmask[j]);
           }
-        }
       }
       __syncthreads();                                         // stage and pq free: refill
       if (tid == 0 && i_seq + kStages < n_seq) {
@@ -534,18 +544,13 @@ __global__ void __launch_bounds__(kThreads)
     }
   if (g < G) {
 #pragma unroll
-    for (int i = 0; i < WPW; ++i) {
-      const int wd = vw0 + i;
-      if (wd < vw1) {
-        const int ebase = wd < n2w_v ? 16 * wd : lv.n2 + 32 * (wd - n2w_v);
-        const int nq = wd < n2w_v ? 2 : 4;
-#pragma unroll
-        for (int r = 0; r < 4; ++r)
-          if (r < nq)
-            *reinterpret_cast<float2*>(oe + g * a.n_entries + ebase + 8 * r + 2 * t) =
-                make_float2((vacc[i][r][0] + vacc[i][r][2]) * val_scale, (vacc[i][r][1] + vacc[i][r][3]) * val_scale);
+    for (int j = 0; j < JPW; ++j)
+      if (j < nj) {
+        const int jj = j0 + j;
+        const int ebase = jj < 2 * n2w_v ? 8 * jj : lv.n2 + 8 * (jj - 2 * n2w_v);   // 8 entries per n-tile
+        *reinterpret_cast<float2*>(oe + g * a.n_entries + ebase + 2 * t) =
+            make_float2((vacc[j][0] + vacc[j][2]) * val_scale, (vacc[j][1] + vacc[j][3]) * val_scale);
       }
-    }
   }
   __syncthreads();
   float* ml = red + 2 * kWarps * MAX_GROUP;                    // [3][MAX_GROUP]: m, l, S'
@@ -944,23 +949,23 @@ cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t sm
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
-template <int WPW, int NP>
+template <int JPW, int NP>
 cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
   static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
   if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<WPW, NP>,
+    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<JPW, NP>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     smem_set = smem;
   }
-  return launch_pdl(aatc_decode_split_kernel<WPW, NP>, dim3(a.n_splits, a.n_kv, batch), dim3(kThreads), smem, st, a);
+  return launch_pdl(aatc_decode_split_kernel<JPW, NP>, dim3(a.n_splits, a.n_kv, batch), dim3(kThreads), smem, st, a);
 }
 
 template <int NP>
-cudaError_t launch_split_g(const DecodeArgs& a, int batch, int wpw, size_t smem, cudaStream_t st) {
-  if (wpw <= 3) return launch_split_t<3, NP>(a, batch, smem, st);
-  if (wpw <= 4) return launch_split_t<4, NP>(a, batch, smem, st);
-  return launch_split_t<8, NP>(a, batch, smem, st);
+cudaError_t launch_split_g(const DecodeArgs& a, int batch, int jpw, size_t smem, cudaStream_t st) {
+  if (jpw <= 8) return launch_split_t<8, NP>(a, batch, smem, st);
+  if (jpw <= 12) return launch_split_t<12, NP>(a, batch, smem, st);
+  return launch_split_t<16, NP>(a, batch, smem, st);
 }
 
 template <int GP>
@@ -1007,13 +1012,18 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_entries = plan.n_entries;
   a.n_splits = sp.n_splits;
   a.split_len = sp.split_len;
+  {
+    const long n_cta = static_cast<long>(sp.n_splits) * a.n_kv * batch;
+    a.num_sms = plan.num_sms;
+    a.cta_per_sm = plan.num_sms > 0 && n_cta % plan.num_sms == 0 ? static_cast<int>(n_cta / plan.num_sms) : 0;
+  }
   // largest key k-step count and value word count over the layer's streams
-  int n_ks = 1, nw_v = 1;
+  int n_ks = 1, n_jobs_v = 1;
   for (int h = 0; h < a.n_kv; ++h) {
     const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
     const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
     n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
-    nw_v = std::max(nw_v, lv.n2 / 16 + (lv.n1 + 31) / 32);
+    n_jobs_v = std::max(n_jobs_v, 2 * (lv.n2 / 16) + 4 * ((lv.n1 + 31) / 32));
   }
   const int np = (a.group + 3) / 4;
   const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
@@ -1026,9 +1036,9 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   if (e != cudaSuccess) return e;
   const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
   const size_t smem = static_cast<size_t>(L.total);
-  const int wpw = (nw_v + kWarps - 1) / kWarps;
-  if (wpw > 8 || smem > 227 * 1024) return cudaErrorNotSupported;
-  e = np == 1 ? launch_split_g<1>(a, batch, wpw, smem, st) : launch_split_g<2>(a, batch, wpw, smem, st);
+  const int jpw = (n_jobs_v + kWarps - 1) / kWarps;            // value n-tiles per warp
+  if (jpw > 16 || smem > 227 * 1024) return cudaErrorNotSupported;
+  e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
   if (e != cudaSuccess) return e;
   const size_t msmem = 4 * (static_cast<size_t>(D) * D + ((sp.n_splits + 3) & ~3) + kMWarps * D + D);
   if (msmem > 227 * 1024) return cudaErrorNotSupported;
