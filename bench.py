@@ -140,6 +140,23 @@ def decode_bytes(plan, cfg, batch, n_ctx):
 
 # ------------------------------------------------------------------------------------ our arm
 
+def planner_timing(aatc):
+    """Host planner rows: the global cross-layer allocation on Llama-3.1-8B-shaped statistics
+    (32 layers x 8 kv-heads x K|V x 128 channels; seeded log-normal spectra), median of 5 runs."""
+    rng = np.random.default_rng(1004)
+    L, H = 32, 8
+    s2 = -np.sort(-rng.lognormal(0.0, 1.5, (L, H, 2, 128)), axis=-1)
+    w = np.ones_like(s2)
+    dm = aatc.dims(L, H, 32)
+    ts = []
+    for _ in range(5):
+        t0 = time.perf_counter()
+        aatc.allocate_global(dm, s2, w, 2.75, 2.75, n_protect=3)
+        ts.append(time.perf_counter() - t0)
+    return {"global_allocation_ms": round(1e3 * float(np.median(ts)), 3),
+            "shape": "32 layers x 8 kv-heads x K|V x 128 channels, 2.75 bits, first 3 layers protected"}
+
+
 def run_ours(args):
     import torch
     import paper_2608_14191_gb300 as aatc
@@ -309,6 +326,7 @@ def run_ours(args):
                         "through the public API, D2H of all outputs"},
         "gpu_launches": args.steps * (1 + 3 * steps_dec),
         "clocks": clocks,
+        "planner": planner_timing(aatc),
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds)

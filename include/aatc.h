@@ -98,6 +98,29 @@ aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k, cons
                              double* sigma2_out, double* weights_out, int32_t n_threads);
 
 /*
+ * Global cross-layer bit allocation (Sec. 5 "waterfilling problem for the keys / values" summed
+ * over layers; Algorithm 1 "Allocate bits globally via reverse waterfilling over all (l, c)";
+ * the experimental-setup paragraph on AATC for the normalisation and the protected layers).
+ * Replaces the per-stream budgets of aatc_calibrate with one pool per kind (keys, values):
+ *   - layers l < n_protect get a per-stream allocation with avg_bits_v * 128 bits for values and
+ *     avg_bits_k * 128 + 128 (one bit per channel more, capped at b_max * 128) for keys;
+ *   - the rest of the kind's total budget (avg_bits * 128 * n_layers * n_kv_heads) is allocated
+ *     over all channels of all other layers and kv-heads at once, by exact integer reverse
+ *     water-filling on g = (sigma2 / P95_l(sigma2)) * (w / P95_l(w)), where P95_l is the 95th
+ *     percentile (linear interpolation) over layer l's channels of every kv-head;
+ *   - b in {0..b_max}; marginal-gain greedy, ties to the lower (layer, kv-head, channel) index.
+ *   sigma2, weights : host fp64 [L][H_kv][2][128] in storage order, as aatc_calibrate writes them
+ *   bits_out        : host uint8 [L][H_kv][2][128]; per stream non-increasing (the order of g
+ *                     within a stream is unchanged by the per-layer normalisation), so it can be
+ *                     passed to aatc_plan_create with aatc_calibrate's basis and scales.
+ * Errors: AATC_ERR_INVALID_ARG (null, negative or non-finite inputs), AATC_ERR_BUDGET (avg bits
+ * not a multiple of 1/128, or the protected layers need more than the total budget, or the rest
+ * exceeds b_max on every pooled channel).  Host only; no device work.
+ */
+aatc_status_t aatc_allocate_global(const aatc_dims_t* dims, const double* sigma2, const double* weights,
+                                   double avg_bits_k, double avg_bits_v, int32_t n_protect, uint8_t* bits_out);
+
+/*
  * Build an immutable device plan from basis / bits / scales in the layouts aatc_calibrate
  * writes (Algorithm 1 outputs).  Derives per stream: R = #{b_c >= 1}, bit offsets, the
  * record length W = ceil(max_s sum_c b_c / 32) words (plan-wide), f_c = s_c 2^(1-b_c), the

@@ -140,6 +140,47 @@ def continuous_allocation(g: np.ndarray, budget: float, b_max: float = np.inf):
     return np.clip(0.5 * (np.log2(g) - theta_log), 0.0, b_max), 2.0 ** theta_log
 
 
+def global_allocation(sigma2: np.ndarray, weights: np.ndarray, avg_bits_k: float, avg_bits_v: float,
+                      n_protect: int = 3, b_max: int = 8) -> np.ndarray:
+    """Global cross-layer allocation (Eq. waterfilling-keys and its value twin, both summed over
+    layers; Algorithm 1 'Allocate bits globally via reverse waterfilling over all (l, c)'; the
+    AATC experimental-setup paragraph for the protected layers and the normalisation).
+
+    sigma2, weights: [L][H][2][d] (kind 0 keys, 1 values), channels in storage order.
+    Per kind: layers l < n_protect are allocated per stream with the average budget (values) or
+    one bit per channel more (keys, capped at b_max d); the rest of the kind's total budget
+    avg_bits * d * L * H is water-filled over every channel of the other layers at once, with
+    sigma^2 and w each divided by the layer's own 95th percentile over its channels (all kv-heads).
+    Reading: b_max stays the plan's 8 (the paper allows 16).
+    """
+    sigma2 = np.asarray(sigma2, np.float64)
+    weights = np.asarray(weights, np.float64)
+    L, H, _, d = sigma2.shape
+    bits = np.zeros(sigma2.shape, dtype=np.int64)
+    np_ = min(n_protect, L)
+    for kind, avg in ((0, avg_bits_k), (1, avg_bits_v)):
+        per_stream = int(round(avg * d))
+        prot = min(per_stream + (d if kind == 0 else 0), b_max * d)
+        for l in range(np_):
+            for h in range(H):
+                bits[l, h, kind] = greedy_allocation(weights[l, h, kind] * sigma2[l, h, kind], prot, b_max)
+        rest = per_stream * L * H - prot * np_ * H
+        if rest < 0 or rest > b_max * d * (L - np_) * H:
+            raise ValueError("the protected layers and the pool do not fit the total budget")
+        if np_ == L:
+            continue
+        g = []
+        for l in range(np_, L):
+            ps = percentile_linear(sigma2[l, :, kind].ravel(), 95.0)
+            pw = percentile_linear(weights[l, :, kind].ravel(), 95.0)
+            ps = ps if ps > 0 else 1.0
+            pw = pw if pw > 0 else 1.0
+            g.append((sigma2[l, :, kind] / ps) * (weights[l, :, kind] / pw))
+        pooled = greedy_allocation(np.concatenate([x.ravel() for x in g]), rest, b_max)
+        bits[np_:, :, kind] = pooled.reshape(L - np_, H, d)
+    return bits
+
+
 def percentile_linear(values: np.ndarray, p: float) -> float:
     """Percentile with linear interpolation at rank (p/100)(N-1) of the sorted sample."""
     a = np.sort(np.asarray(values, np.float64))

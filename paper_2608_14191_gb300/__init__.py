@@ -46,6 +46,7 @@ SIGNATURES = {
     "aatc_last_cuda_error": (_I32, []),
     "aatc_version": (_I32, []),
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
+    "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
     "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
     "aatc_plan_destroy": (_I32, [_P]),
     "aatc_plan_info": (_I32, [_P, ctypes.POINTER(_I32), _P]),
@@ -130,6 +131,23 @@ def calibrate(dm: Dims, calib_k: np.ndarray, calib_v: np.ndarray, calib_q: np.nd
     _check(st, "aatc_calibrate")
     assert S == basis.shape[0] * H * 2
     return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
+
+
+def allocate_global(dm: Dims, sigma2: np.ndarray, weights: np.ndarray, avg_bits_k: float,
+                    avg_bits_v: float | None = None, n_protect: int = 3) -> np.ndarray:
+    """aatc_allocate_global: one water-filling pool per kind over all layers (first n_protect
+    layers per stream).  sigma2, weights: fp64 [L][H_kv][2][128] as calibrate returns them.
+    Returns bits uint8 [L][H_kv][2][128]."""
+    s2 = np.ascontiguousarray(sigma2, dtype=np.float64)
+    w = np.ascontiguousarray(weights, dtype=np.float64)
+    shape = (dm.n_layers, dm.n_kv_heads, 2, HEAD_DIM)
+    if s2.shape != shape or w.shape != shape:
+        raise ValueError("sigma2 / weights must be [L][H_kv][2][128]")
+    bits = np.empty(shape, np.uint8)
+    _check(load().aatc_allocate_global(ctypes.byref(dm), _ptr(s2), _ptr(w), float(avg_bits_k),
+                                       float(avg_bits_k if avg_bits_v is None else avg_bits_v), int(n_protect),
+                                       _ptr(bits)), "aatc_allocate_global")
+    return bits
 
 
 class Plan:

@@ -8,6 +8,7 @@
 #include <cstdint>
 #include <cstring>
 #include <numeric>
+#include <queue>
 #include <thread>
 #include <vector>
 
@@ -194,6 +195,31 @@ void plan_one_stream(const StreamJob& job) {
   }
 }
 
+// Linear-interpolation percentile (rank p (N-1), the NumPy default) of a copy of `vals`.
+double percentile_linear(std::vector<double> vals, double p) {
+  std::sort(vals.begin(), vals.end());
+  const double r = p * (static_cast<double>(vals.size()) - 1.0);
+  const size_t lo = static_cast<size_t>(std::floor(r));
+  const size_t hi = std::min(lo + 1, vals.size() - 1);
+  return vals[lo] + (r - static_cast<double>(lo)) * (vals[hi] - vals[lo]);
+}
+
+// Exact integer reverse water-filling over a pool of channels: the budget goes, one bit at a
+// time, to the largest marginal gain g_c 4^-b_c (b_c < b_max); ties to the lower pool index.
+void greedy_pool(const std::vector<double>& g, int budget, int b_max, std::vector<int>& bits) {
+  bits.assign(g.size(), 0);
+  using Item = std::pair<double, long>;                       // (gain, -index): max-heap order
+  std::priority_queue<Item> heap;
+  for (size_t i = 0; i < g.size(); ++i)
+    if (b_max > 0) heap.emplace(g[i], -static_cast<long>(i));
+  for (int it = 0; it < budget && !heap.empty(); ++it) {
+    const Item top = heap.top();
+    heap.pop();
+    const size_t i = static_cast<size_t>(-top.second);
+    if (++bits[i] < b_max) heap.emplace(std::ldexp(g[i], -2 * bits[i]), top.second);
+  }
+}
+
 bool budget_from_avg(double avg, int b_max, int* budget) {
   const double b = avg * kD;
   const double r = std::nearbyint(b);
@@ -258,5 +284,62 @@ extern "C" aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* ca
   for (int t = 1; t < nt; ++t) pool.emplace_back(worker);
   worker();
   for (auto& th : pool) th.join();
+  return AATC_OK;
+}
+
+extern "C" aatc_status_t aatc_allocate_global(const aatc_dims_t* dims, const double* sigma2,
+                                              const double* weights, double avg_bits_k, double avg_bits_v,
+                                              int32_t n_protect, uint8_t* bits_out) {
+  using namespace aatc;
+  if (!valid_dims(dims) || !sigma2 || !weights || !bits_out || n_protect < 0) return AATC_ERR_INVALID_ARG;
+  const int L = dims->n_layers, H = dims->n_kv_heads, b_max = dims->b_max;
+  const int np = std::min(n_protect, L);
+  for (size_t i = 0; i < static_cast<size_t>(L) * H * 2 * kD; ++i)
+    if (!std::isfinite(sigma2[i]) || !std::isfinite(weights[i]) || sigma2[i] < 0.0 || weights[i] < 0.0)
+      return AATC_ERR_INVALID_ARG;
+  for (int kind = 0; kind < 2; ++kind) {
+    const double avg = kind == 0 ? avg_bits_k : avg_bits_v;
+    int per_stream = 0;
+    if (!budget_from_avg(avg, b_max, &per_stream)) return AATC_ERR_BUDGET;
+    // protected layers: per-stream allocation, the average budget for values and one bit per
+    // channel more for keys (capped at b_max)
+    const int prot = std::min(per_stream + (kind == 0 ? kD : 0), b_max * kD);
+    const long total = static_cast<long>(per_stream) * L * H;
+    const long rest = total - static_cast<long>(prot) * np * H;
+    const long pool_cap = static_cast<long>(b_max) * kD * (L - np) * H;
+    if (rest < 0 || rest > pool_cap) return AATC_ERR_BUDGET;
+    auto at = [&](int l, int h, int c) { return ((static_cast<size_t>(l) * H + h) * 2 + kind) * kD + c; };
+    std::vector<int> bits;
+    for (int l = 0; l < np; ++l)
+      for (int h = 0; h < H; ++h) {
+        std::vector<double> g(kD);
+        for (int c = 0; c < kD; ++c) g[c] = weights[at(l, h, c)] * sigma2[at(l, h, c)];
+        greedy_pool(g, prot, b_max, bits);
+        for (int c = 0; c < kD; ++c) bits_out[at(l, h, c)] = static_cast<uint8_t>(bits[c]);
+      }
+    if (np == L) continue;
+    // the pool: g = (sigma^2 / P95_l(sigma^2)) (w / P95_l(w)), percentiles over the layer's
+    // channels of every kv-head
+    std::vector<double> g;
+    g.reserve(static_cast<size_t>(L - np) * H * kD);
+    for (int l = np; l < L; ++l) {
+      std::vector<double> sv, wv;
+      for (int h = 0; h < H; ++h)
+        for (int c = 0; c < kD; ++c) {
+          sv.push_back(sigma2[at(l, h, c)]);
+          wv.push_back(weights[at(l, h, c)]);
+        }
+      double ps = percentile_linear(sv, 0.95), pw = percentile_linear(wv, 0.95);
+      if (!(ps > 0.0)) ps = 1.0;
+      if (!(pw > 0.0)) pw = 1.0;
+      for (int h = 0; h < H; ++h)
+        for (int c = 0; c < kD; ++c) g.push_back((sigma2[at(l, h, c)] / ps) * (weights[at(l, h, c)] / pw));
+    }
+    greedy_pool(g, static_cast<int>(rest), b_max, bits);
+    size_t i = 0;
+    for (int l = np; l < L; ++l)
+      for (int h = 0; h < H; ++h)
+        for (int c = 0; c < kD; ++c) bits_out[at(l, h, c)] = static_cast<uint8_t>(bits[i++]);
+  }
   return AATC_OK;
 }

@@ -231,3 +231,40 @@ def test_llama_stack_full_size(aatc):
         js = sorted(ref)
         Hn.check_decode(outs[l].cpu().numpy()[0, js], np.stack([ref[j] for j in js]))
     assert case.plan.device_error() == 0
+
+
+def test_global_allocation_plan(aatc):
+    """A 5-layer stack planned with the global cross-layer allocation (protected first 3 layers,
+    one pool for the rest): streams get unequal bit totals, every record is padded to the
+    plan-wide W, and encode + decode still match the oracle on a protected and a pooled layer."""
+    cfg = W.Config(6, "global5", 5, 2, 8, 1, 2048, (2.75,), 1, "5-layer stack, global allocation")
+    L, T = cfg.n_layers, cfg.n_ctx
+    cal = [W.layer_calibration(cfg, l, anisotropic_queries=True, n=1024) for l in range(L)]
+    dm = aatc.dims(L, cfg.n_kv_heads, cfg.n_q_heads)
+    p = aatc.calibrate(dm, np.stack([c[0] for c in cal]), np.stack([c[1] for c in cal]),
+                       np.stack([c[2] for c in cal]), 2.75)
+    bits = aatc.allocate_global(dm, p["sigma2"], p["weights"], 2.75, 2.75, n_protect=3)
+    per_stream = bits.astype(np.int64).sum(axis=-1)
+    assert per_stream[:, :, 1].sum() == 352 * L * cfg.n_kv_heads
+    assert len(np.unique(per_stream[3:])) > 1                      # the pool spreads bits unevenly
+    case = Hn.Case.__new__(Hn.Case)
+    case.aatc, case.cfg, case.avg_bits, case.layers, case.dm = aatc, cfg, 2.75, list(range(L)), dm
+    case.basis, case.bits, case.scales = p["basis"], bits, p["scales"]
+    case.plan = aatc.Plan(dm, p["basis"], bits, p["scales"])
+    case.basis_bf16 = Hn.bf16_round(p["basis"])
+    for layer in (1, 4):
+        kd, vd = W.kv_device(cfg, layer, 1, T, DEV)
+        cache = case.plan.new_cache(1, T, DEV)
+        aatc.encode(case.plan, layer, kd, vd, cache, 0, T)
+        host = _host_u32(cache)
+        for h in range(cfg.n_kv_heads):
+            for kind, x in ((0, kd), (1, vd)):
+                rec, alpha = Hn.read_stream(case, host, 1, T, 0, h, kind, T - 512, 512)
+                st = Hn.check_codes(case, layer, h, kind, x[0, T - 512:, h].float().cpu().numpy(), rec, alpha)
+                assert st["mismatch"] <= max(1, Hn.MAX_NEAR_FRACTION * st["codes"])
+        q = W.queries_device(cfg, layer, 1, 1, DEV)[0]
+        out = aatc.decode_attention(case.plan, layer, q, cache, T, T).cpu().numpy()
+        ref = Hn.oracle_decode_from_cache(case, host, 1, T, layer, 0, q.float().cpu().numpy()[0], T)
+        js = sorted(ref)
+        Hn.check_decode(out[0, js], np.stack([ref[j] for j in js]))
+    assert case.plan.device_error() == 0
