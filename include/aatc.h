@@ -187,6 +187,29 @@ aatc_status_t aatc_decode_attention(aatc_plan_t plan, int32_t layer, const void*
                                     size_t workspace_bytes, void* stream);
 
 /*
+ * Decode attention over a packed range plus uncompressed tokens in one softmax: the paper's
+ * inference policy keeps the first tokens (attention sink) and a recent window in full
+ * precision and compresses the rest (Sec. 6 setup: 4 sink tokens, a 128-token window moved in
+ * steps of 16).  Per query head j, the scores of the packed tokens [t_first, t_end) of each
+ * sequence are computed as in aatc_decode_attention, the scores of the n_full uncompressed
+ * tokens as q . k / sqrt(128), and a = softmax over both sets; out = U_V sum_packed a_t h_hat^V_t
+ * + sum_full a_t v_t.  The order of the uncompressed tokens is irrelevant.
+ *   q       : device bf16 [batch][n_q_heads][128]
+ *   cache   : packed cache as written by aatc_encode; only [t_first, t_end) is read
+ *   k_full, v_full : device bf16 [batch][full_cap][n_kv_heads][128]; the first n_full tokens of
+ *             each sequence are attended (n_full may be 0; k_full/v_full may then be NULL)
+ *   out     : device fp32 [batch][n_q_heads][128]
+ *   workspace : as for aatc_decode_attention with n_ctx = t_end (not read when t_first == t_end)
+ * Errors: AATC_ERR_INVALID_ARG (t_first > t_end, both sets empty, full_cap < n_full, unaligned
+ * pointers, ...), AATC_ERR_CAPACITY (t_end > max_tokens or n_full > 8192), AATC_ERR_WORKSPACE,
+ * AATC_ERR_UNSUPPORTED (group > 8), AATC_ERR_CUDA.
+ */
+aatc_status_t aatc_decode_attention_sw(aatc_plan_t plan, int32_t layer, const void* q, const void* cache,
+                                       int32_t batch, int32_t t_first, int32_t t_end, int32_t max_tokens,
+                                       const void* k_full, const void* v_full, int32_t n_full, int32_t full_cap,
+                                       float* out, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Test hook: dequantized coefficients h_hat_c = fl32(code_c * fl32(alpha_t * f_c)) (zero for
  * dropped channels) of tokens [t0, t0 + n) of every sequence.
  *   coeffs_out : device fp32 [batch][n][n_kv_heads][2][128]

@@ -388,7 +388,7 @@ def cache_records(cache_u32: np.ndarray, batch: int, n_kv_heads: int, max_tokens
     else:
         rec = np.zeros((n, n_words), dtype=np.uint64)
         for r in range(4):
-            slots = np.array([value_slot_of(int(x), r)[0] for x in t % TILE])
+            slots = np.array([value_slot_of(int(x), r)[0] for x in t % TILE], dtype=np.int64)
             byte = (t % TILE) % 4
             w = words[b, head, kind][t // TILE, :, slots].astype(np.uint64)      # (n, W)
             rec |= ((w >> (8 * byte[:, None]).astype(np.uint64)) & np.uint64(0xFF)) << np.uint64(8 * r)
@@ -457,6 +457,41 @@ def decode_attention(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_
         a = softmax(np.asarray(hk[h], np.float64) @ qt / math.sqrt(D))
         out[j] = np.asarray(basis_v[h], np.float64) @ (a @ np.asarray(hv[h], np.float64))
     return out
+
+
+def decode_attention_mixed(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_k: np.ndarray,
+                           basis_v: np.ndarray, group: int, k_full: np.ndarray, v_full: np.ndarray) -> np.ndarray:
+    """Decode over coded tokens and uncompressed tokens in one softmax (the paper's inference
+    policy keeps an attention sink and a recent window in full precision, Sec. 6 setup).
+
+    hk, hv: (H_kv, n_coded, 128) dequantized coefficients; k_full, v_full: (H_kv, n_full, 128) in
+    the original basis.  Scores: (U_K^T q) . h_hat / sqrt(128) for coded tokens, q . k / sqrt(128)
+    for the others; a = softmax over both; out = U_V (sum_coded a h_hat^V) + sum_full a v.
+    """
+    out = np.zeros((q_heads.shape[0], D))
+    for j in range(q_heads.shape[0]):
+        h = j // group
+        q = np.asarray(q_heads[j], np.float64)
+        qt = np.asarray(basis_k[h], np.float64).T @ q
+        s_c = np.asarray(hk[h], np.float64) @ qt / math.sqrt(D)
+        s_f = np.asarray(k_full[h], np.float64) @ q / math.sqrt(D)
+        a = softmax(np.concatenate([s_c, s_f]))
+        n_c = s_c.shape[0]
+        out[j] = (np.asarray(basis_v[h], np.float64) @ (a[:n_c] @ np.asarray(hv[h], np.float64))
+                  + a[n_c:] @ np.asarray(v_full[h], np.float64))
+    return out
+
+
+def sink_window_counts(n_tokens: int, sink: int = 4, window: int = 128, step: int = 16):
+    """Token accounting of the full-precision sink and recent window (Sec. 6 setup: first 4 tokens
+    kept, a 128-token window moved in steps of 16).  Reading: the window fills up to
+    window + step tokens; adding the token that makes it window + step flushes its oldest `step`
+    tokens to the coded cache.  Returns (n_sink, n_coded, n_window) after n_tokens tokens; the
+    coded tokens are positions [n_sink, n_sink + n_coded)."""
+    n_sink = min(n_tokens, sink)
+    rest = n_tokens - n_sink
+    n_coded = step * max(0, (rest - window) // step)
+    return n_sink, n_coded, rest - n_coded
 
 
 # ----------------------------------------------------------------------------

@@ -47,6 +47,8 @@ SIGNATURES = {
     "aatc_version": (_I32, []),
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
     "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
+    "aatc_decode_attention_sw": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _SZ,
+                                        _P]),
     "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
     "aatc_plan_destroy": (_I32, [_P]),
     "aatc_plan_info": (_I32, [_P, ctypes.POINTER(_I32), _P]),
@@ -227,6 +229,27 @@ def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: i
     _check(load().aatc_decode_attention(plan.handle, layer, _ptr(q), _ptr(cache), batch, n_ctx, max_tokens,
                                         _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                         _stream(stream)), "aatc_decode_attention")
+    return out
+
+
+def decode_attention_sw(plan: Plan, layer: int, q, cache, t_first: int, t_end: int, max_tokens: int,
+                        k_full=None, v_full=None, n_full: int = 0, out=None, workspace=None, stream=None):
+    """aatc_decode_attention_sw: packed tokens [t_first, t_end) plus the first n_full tokens of
+    k_full / v_full (bf16 [batch][cap][H_kv][128]) in one softmax -> fp32 [batch][H_q][128]."""
+    import torch
+    batch = q.shape[0]
+    if out is None:
+        out = torch.empty((batch, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    cap = 0 if k_full is None else int(k_full.shape[1])
+    if t_end > t_first and workspace is None:
+        workspace = torch.empty(max(1, plan.workspace_bytes(batch, t_end) // 4), dtype=torch.float32,
+                                device=q.device)
+    ws_ptr = None if workspace is None else _ptr(workspace)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().aatc_decode_attention_sw(plan.handle, layer, _ptr(q), _ptr(cache), batch, t_first, t_end,
+                                           max_tokens, None if k_full is None else _ptr(k_full),
+                                           None if v_full is None else _ptr(v_full), int(n_full), cap, _ptr(out),
+                                           ws_ptr, ws_bytes, _stream(stream)), "aatc_decode_attention_sw")
     return out
 
 

@@ -128,9 +128,20 @@ aatc_status_t status_from_cuda(cudaError_t e);
 cudaError_t encode_tensor_maps_u(Plan& plan);
 cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch,
                           int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st);
+// Optional parts of a decode call: the packed range starts at token t_first (default 0), and
+// n_full uncompressed tokens (bf16 [batch][full_cap][n_kv][128], e.g. a full-precision sink and
+// recent window) join the same softmax.
+struct DecodeExtra {
+  int t_first = 0;
+  const void* k_full = nullptr;
+  const void* v_full = nullptr;
+  int n_full = 0;
+  int full_cap = 0;
+};
+constexpr int MAX_FULL_TOKENS = 8192;   // shared-memory scores of the uncompressed tokens
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch,
                           int n_ctx, int max_tokens, float* out, void* ws, const DecodeSplit& sp,
-                          cudaStream_t st);
+                          cudaStream_t st, const DecodeExtra& extra);
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n,
                            int max_tokens, float* out, cudaStream_t st);
 cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx,

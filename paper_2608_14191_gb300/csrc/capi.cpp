@@ -343,7 +343,39 @@ aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q,
                                                plan->n_words, sp))
     return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
-                                         workspace, sp, static_cast<cudaStream_t>(stream)));
+                                         workspace, sp, static_cast<cudaStream_t>(stream), aatc::DecodeExtra{}));
+}
+
+aatc_status_t aatc_decode_attention_sw(aatc_plan_t p, int32_t layer, const void* q, const void* cache,
+                                       int32_t batch, int32_t t_first, int32_t t_end, int32_t max_tokens,
+                                       const void* k_full, const void* v_full, int32_t n_full, int32_t full_cap,
+                                       float* out, void* workspace, size_t workspace_bytes, void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !q || !cache || !out || layer < 0 || layer >= plan->dims.n_layers || batch < 1 ||
+      max_tokens < 1 || t_first < 0 || t_end < t_first || n_full < 0 || (n_full > 0 && (!k_full || !v_full)) ||
+      full_cap < n_full || (t_end == t_first && n_full == 0))
+    return AATC_ERR_INVALID_ARG;
+  if (t_end > max_tokens || n_full > aatc::MAX_FULL_TOKENS) return AATC_ERR_CAPACITY;
+  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if (!aligned16(cache) || (n_full > 0 && (!aligned16(k_full) || !aligned16(v_full)))) return AATC_ERR_INVALID_ARG;
+  // the packed part covers tiles [t_first / 128, ceil(t_end / 128)): never more splits than a
+  // plain decode of t_end tokens, so aatc_decode_workspace_bytes(batch, t_end) suffices
+  const int range = t_end - (t_first / aatc::TILE) * aatc::TILE;
+  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, std::max(range, 1), plan->num_sms);
+  if (t_end > t_first) {
+    if (!workspace || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
+    if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads,
+                                                 plan->n_entries, plan->n_words, sp))
+      return AATC_ERR_WORKSPACE;
+  }
+  aatc::DecodeExtra ex;
+  ex.t_first = t_first;
+  ex.k_full = k_full;
+  ex.v_full = v_full;
+  ex.n_full = n_full;
+  ex.full_cap = full_cap;
+  return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, t_end, max_tokens, out, workspace, sp,
+                                         static_cast<cudaStream_t>(stream), ex));
 }
 
 aatc_status_t aatc_dequantize(aatc_plan_t p, int32_t layer, const void* cache, int32_t batch,

@@ -83,6 +83,10 @@ struct DecodeArgs {
   float* qcorr;            // workspace: [batch][n_kv][16]: offset corrections C_g, score scales
   int layer, n_kv, n_q, group, n_ctx, n_tiles, n_words, n_entries, n_splits, split_len, ks_stride, pstride;
   int num_sms, cta_per_sm;  // split-kernel work permutation (cta_per_sm = 0: identity)
+  int t_first;              // first packed token attended (tokens [t_first, n_ctx) of the cache)
+  const __nv_bfloat16* k_full;  // uncompressed tokens attended as well: [batch][full_cap][n_kv][128]
+  const __nv_bfloat16* v_full;
+  int n_full, full_cap;
 };
 
 // 2^x with the hardware approximation (relative error ~2^-22; -inf -> 0)
@@ -152,7 +156,6 @@ __global__ void __launch_bounds__(kQThreads)
   const int G = a.group;
   const bool real = slot < G;
   const int sk = (a.layer * a.n_kv + head) * 2;
-  ptx::grid_launch_dependents();
   // every global input is requested up front (one memory round trip)
   const int c = tid & (D - 1), qd = tid >> 7;
   const short* ent = a.entry + static_cast<size_t>(sk) * a.n_entries;
@@ -174,6 +177,8 @@ __global__ void __launch_bounds__(kQThreads)
   // plan constants above; the query (and the workspace this call reuses) only once the preceding
   // grid in the stream is complete -- this kernel may be launched as its programmatic dependent
   ptx::grid_dependency_wait();
+  // only now may the split kernel start: it reads the cache, which the preceding grid may write
+  ptx::grid_launch_dependents();
   if (tid < D && real) qraw = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + slot) * D + tid]);
   if (tid < D) qv[tid] = qraw;
   __syncthreads();
@@ -314,10 +319,13 @@ __global__ void __launch_bounds__(kThreads)
   uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
   const int sbs = L.sb_stride;
 
-  const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
-  const int tile_lo = static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
-  const int tile_hi = static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
-  const int t_begin = tile_lo * TILE;
+  // tiles [tile_first, ceil(n_ctx / 128)) hold the attended packed tokens [t_first, n_ctx)
+  const int tile_first = a.t_first / TILE;
+  const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE - tile_first;
+  const int tile_lo = tile_first + static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
+  const int tile_hi = tile_first + static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
+  const int t_begin = tile_lo * TILE;                          // first token of the first tile
+  const int t_lo = max(t_begin, a.t_first);                    // first attended token
   const int t_end = min(a.n_ctx, tile_hi * TILE);
   const int n_tiles_split = tile_hi - tile_lo;
   const int n_seq = 2 * n_tiles_split;                         // key tiles, then value tiles
@@ -414,8 +422,8 @@ __global__ void __launch_bounds__(kThreads)
         const float2 a2 = *reinterpret_cast<const float2*>(ak + ti * TILE + tk);
         float s0 = a2.x * fmaf(acc[j][0] + acc[j][2], sg, -cg);
         float s1 = a2.y * fmaf(acc[j][1] + acc[j][3], sg, -cg);
-        s0 = tbase + tk < t_end ? s0 : -INFINITY;
-        s1 = tbase + tk + 1 < t_end ? s1 : -INFINITY;
+        s0 = tbase + tk < t_end && tbase + tk >= t_lo ? s0 : -INFINITY;
+        s1 = tbase + tk + 1 < t_end && tbase + tk + 1 >= t_lo ? s1 : -INFINITY;
         *reinterpret_cast<float2*>(sbuf + g * sbs + ti * TILE + tk) = make_float2(s0, s1);
         mloc = fmaxf(mloc, fmaxf(s0, s1));
       }
@@ -428,7 +436,7 @@ __global__ void __launch_bounds__(kThreads)
   }
   // split max per query; largest alpha^V of the split (P' = p alpha^V is coded relative to it)
   float amx = 0.0f;
-  for (int i = tid; i < t_end - t_begin; i += kThreads) amx = fmaxf(amx, av[i]);
+  for (int i = t_lo - t_begin + tid; i < t_end - t_begin; i += kThreads) amx = fmaxf(amx, av[i]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) amx = fmaxf(amx, __shfl_xor_sync(0xffffffffu, amx, o));
   if (lane == 0) red[3 * kWarps * MAX_GROUP + warp] = amx;
@@ -487,10 +495,12 @@ __global__ void __launch_bounds__(kThreads)
       wait_tile(i_seq);
       const uint32_t* vt = ring + (i_seq % kStages) * W * TILE;
       {
-        const int nvalid = t_end - (tile0 + ti) * TILE - tk0;         // tokens of this quad in range
+        const int tq = (tile0 + ti) * TILE + tk0;                // first token of this quad
         const float4 a4 = *reinterpret_cast<const float4*>(av + ti * TILE + tk0);
-        const float av0 = nvalid > 0 ? a4.x * inv_p : 0.0f, av1 = nvalid > 1 ? a4.y * inv_p : 0.0f;
-        const float av2 = nvalid > 2 ? a4.z * inv_p : 0.0f, av3 = nvalid > 3 ? a4.w * inv_p : 0.0f;
+        const float av0 = tq >= t_lo && tq < t_end ? a4.x * inv_p : 0.0f;
+        const float av1 = tq + 1 >= t_lo && tq + 1 < t_end ? a4.y * inv_p : 0.0f;
+        const float av2 = tq + 2 >= t_lo && tq + 2 < t_end ? a4.z * inv_p : 0.0f;
+        const float av3 = tq + 3 >= t_lo && tq + 3 < t_end ? a4.w * inv_p : 0.0f;
 #pragma unroll
         for (int p = 0; p < NP; ++p) {
           const int q = 4 * p + qq;
@@ -592,7 +602,10 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // Merge of the splits of one (sequence, query head): M = max_s m_s, w_s = 2^(m_s - M),
-// o_c = sum_s w_s o_{s,c}, l = sum_s w_s l_s, o_hat_c = o_c f^V_c / l, out = U_V o_hat.
+// o_c = sum_s w_s o_{s,c}, l = sum_s w_s l_s, o_hat_c = o_c f^V_c, out = U_V o_hat / l.
+// Uncompressed tokens (the full-precision sink and recent window of Sec. 6) join the same
+// softmax here: their scores q.k/sqrt(128), weights 2^(s - m_f) and sum_t p_t v_t are taken in
+// the original basis and merged with the packed part by log-sum-exp.
 // Launched as a programmatic dependent of the split kernel: U_V^T (a plan constant) is staged
 // while the splits finish; the partials are read only after the grid dependency resolves.
 constexpr int kMThreads = 256;
@@ -605,6 +618,7 @@ __global__ void __launch_bounds__(kMThreads)
   float* wsp = ut_s + D * D;                         // [n_splits] split weights
   float* osum = wsp + ((a.n_splits + 3) & ~3);       // [kMWarps][128]
   float* ohat = osum + kMWarps * D;                  // [128]
+  float* sf = ohat + D;                              // [n_full] scores, then weights, of full tokens
   __shared__ float red[2][kMWarps];
   __shared__ uint64_t bar;
   __shared__ int s_abort;
@@ -619,31 +633,84 @@ __global__ void __launch_bounds__(kMThreads)
     ptx::bulk_load(ut_s, a.u32t + static_cast<size_t>(sv) * D * D, D * D * 4, &bar);
   }
   const float fv = tid < D ? a.f[sv * D + tid] : 0.0f;
-  ptx::grid_dependency_wait();                       // the split kernel's partials
-  const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * a.pstride;
-  // split maxima and weights
-  float M = -INFINITY;
-  for (int s = tid; s < a.n_splits; s += kMThreads) M = fmaxf(M, __ldcg(src + s * a.pstride + D));
+  // ---- uncompressed tokens (inputs of this call, not produced by the split kernel)
+  float m_f = -INFINITY, l_f = 0.0f;
+  float of = 0.0f;                                   // thread d < 128: sum_t p_t v_t[d]
+  if (a.n_full > 0) {
+    // q and the full tokens were complete before the query kernel let the split kernel start;
+    // with no packed range this kernel follows the caller's grid directly
+    if (a.n_splits == 0) ptx::grid_dependency_wait();
+    const float scale = kLog2e * 0.08838834764831845f;
+    const uint2 qq = *reinterpret_cast<const uint2*>(a.q + (static_cast<size_t>(b) * a.n_q + j) * D + 4 * lane);
+    const float2 q01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qq.x));
+    const float2 q23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qq.y));
+    float mloc = -INFINITY;
+    for (int t = warp; t < a.n_full; t += kMWarps) {
+      const size_t row = ((static_cast<size_t>(b) * a.full_cap + t) * a.n_kv + head) * D;
+      const uint2 kk = *reinterpret_cast<const uint2*>(a.k_full + row + 4 * lane);
+      const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kk.x));
+      const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kk.y));
+      float d = fmaf(q01.x, k01.x, fmaf(q01.y, k01.y, fmaf(q23.x, k23.x, q23.y * k23.y)));
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-  if (lane == 0) red[0][warp] = M;
-  __syncthreads();
-  M = red[0][0];
+      for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+      if (lane == 0) sf[t] = d * scale;
+      mloc = fmaxf(mloc, d * scale);
+    }
+    if (lane == 0) red[0][warp] = mloc;
+    __syncthreads();
+    m_f = red[0][0];
 #pragma unroll
-  for (int w = 1; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
-  float l = 0.0f;
-  for (int s = tid; s < a.n_splits; s += kMThreads) {
-    const float2 ml = __ldcg(reinterpret_cast<const float2*>(src + s * a.pstride + D));
-    const float w = exp2f(ml.x - M);
-    wsp[s] = w;
-    l = fmaf(w, ml.y, l);
+    for (int w = 1; w < kMWarps; ++w) m_f = fmaxf(m_f, red[0][w]);
+    float lp = 0.0f;
+    for (int t = tid; t < a.n_full; t += kMThreads) {
+      const float pw = exp2f(sf[t] - m_f);
+      sf[t] = pw;
+      lp += pw;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lp += __shfl_xor_sync(0xffffffffu, lp, o);
+    if (lane == 0) red[1][warp] = lp;
+    __syncthreads();
+    l_f = 0.0f;
+#pragma unroll
+    for (int w = 0; w < kMWarps; ++w) l_f += red[1][w];
+    {
+      // two threads per dimension, alternate tokens
+      const int d = tid & (D - 1), half = tid >> 7;
+      float acc = 0.0f;
+      for (int t = half; t < a.n_full; t += 2)
+        acc = fmaf(sf[t], __bfloat162float(a.v_full[((static_cast<size_t>(b) * a.full_cap + t) * a.n_kv + head) * D + d]), acc);
+      osum[half * D + d] = acc;
+    }
+    __syncthreads();
+    if (tid < D) of = osum[tid] + osum[D + tid];
+    __syncthreads();
   }
+  // ---- packed splits
+  float M = -INFINITY, L = 0.0f;
+  if (a.n_splits > 0) {
+    ptx::grid_dependency_wait();                     // the split kernel's partials
+    const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * a.pstride;
+    for (int s = tid; s < a.n_splits; s += kMThreads) M = fmaxf(M, __ldcg(src + s * a.pstride + D));
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-  if (lane == 0) red[1][warp] = l;
-  __syncthreads();
-  // weighted channel sums: warp = splits s = warp (mod 8), lane = channels 4 lane .. 4 lane + 3
-  {
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    if (lane == 0) red[0][warp] = M;
+    __syncthreads();
+    M = red[0][0];
+#pragma unroll
+    for (int w = 1; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
+    float l = 0.0f;
+    for (int s = tid; s < a.n_splits; s += kMThreads) {
+      const float2 ml = __ldcg(reinterpret_cast<const float2*>(src + s * a.pstride + D));
+      const float w = exp2f(ml.x - M);
+      wsp[s] = w;
+      l = fmaf(w, ml.y, l);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+    if (lane == 0) red[1][warp] = l;
+    __syncthreads();
+    // weighted channel sums: warp = splits s = warp (mod 8), lane = channels 4 lane .. 4 lane + 3
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     int s = warp;
     for (; s + kMWarps * 7 < a.n_splits; s += kMWarps * 8) {
@@ -675,16 +742,22 @@ __global__ void __launch_bounds__(kMThreads)
         acc.w = fmaf(w, v[u].w, acc.w);
       }
     *reinterpret_cast<float4*>(osum + warp * D + 4 * lane) = acc;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < kMWarps; ++w) L += red[1][w];
   }
-  __syncthreads();
+  // ---- log-sum-exp merge of the two parts: out = (U_V (f o) a_p + o_f a_f) / (L a_p + l_f a_f)
+  const float Mt = fmaxf(M, m_f);
+  const float ap = a.n_splits > 0 ? exp2f(M - Mt) : 0.0f;
+  const float af = a.n_full > 0 ? exp2f(m_f - Mt) : 0.0f;
+  const float inv_den = 1.0f / fmaf(L, ap, l_f * af);
   if (tid < D) {
     float o = 0.0f;
+    if (a.n_splits > 0) {
 #pragma unroll
-    for (int w = 0; w < kMWarps; ++w) o += osum[w * D + tid];
-    float lt = 0.0f;
-#pragma unroll
-    for (int w = 0; w < kMWarps; ++w) lt += red[1][w];
-    ohat[tid] = o * fv / lt;
+      for (int w = 0; w < kMWarps; ++w) o += osum[w * D + tid];
+    }
+    ohat[tid] = o * fv * ap;
   }
   if (!ptx::mbar_wait_sleep(&bar, 0, &s_abort, 100)) atomicOr(a.err, 2);
   __syncthreads();
@@ -697,7 +770,8 @@ __global__ void __launch_bounds__(kMThreads)
     osum[half * D + d] = r;
   }
   __syncthreads();
-  if (tid < D) a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = osum[tid] + osum[D + tid];
+  if (tid < D)
+    a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = (osum[tid] + osum[D + tid] + of * af) * inv_den;
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -986,7 +1060,8 @@ cudaError_t launch_bf16_split(const Bf16Args& a, int batch, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch, int n_ctx,
-                          int max_tokens, float* out, void* ws, const DecodeSplit& sp, cudaStream_t st) {
+                          int max_tokens, float* out, void* ws, const DecodeSplit& sp, cudaStream_t st,
+                          const DecodeExtra& extra) {
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
   DecodeArgs a;
   a.words = static_cast<const uint32_t*>(cache);
@@ -1010,8 +1085,13 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_tiles = g.n_tiles;
   a.n_words = plan.n_words;
   a.n_entries = plan.n_entries;
-  a.n_splits = sp.n_splits;
+  a.n_splits = extra.t_first < n_ctx ? sp.n_splits : 0;     // no packed range: merge kernel only
   a.split_len = sp.split_len;
+  a.t_first = extra.t_first;
+  a.k_full = static_cast<const __nv_bfloat16*>(extra.k_full);
+  a.v_full = static_cast<const __nv_bfloat16*>(extra.v_full);
+  a.n_full = extra.n_full;
+  a.full_cap = extra.full_cap;
   {
     const long n_cta = static_cast<long>(sp.n_splits) * a.n_kv * batch;
     a.num_sms = plan.num_sms;
@@ -1032,15 +1112,19 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
   if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
-  cudaError_t e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, MAX_GROUP), dim3(kQThreads), 0, st, a);
-  if (e != cudaSuccess) return e;
-  const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
-  const size_t smem = static_cast<size_t>(L.total);
-  const int jpw = (n_jobs_v + kWarps - 1) / kWarps;            // value n-tiles per warp
-  if (jpw > 16 || smem > 227 * 1024) return cudaErrorNotSupported;
-  e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
-  if (e != cudaSuccess) return e;
-  const size_t msmem = 4 * (static_cast<size_t>(D) * D + ((sp.n_splits + 3) & ~3) + kMWarps * D + D);
+  cudaError_t e = cudaSuccess;
+  if (a.n_splits > 0) {
+    e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, MAX_GROUP), dim3(kQThreads), 0, st, a);
+    if (e != cudaSuccess) return e;
+    const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
+    const size_t smem = static_cast<size_t>(L.total);
+    const int jpw = (n_jobs_v + kWarps - 1) / kWarps;          // value n-tiles per warp
+    if (jpw > 16 || smem > 227 * 1024) return cudaErrorNotSupported;
+    e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
+    if (e != cudaSuccess) return e;
+  }
+  const size_t msmem = 4 * (static_cast<size_t>(D) * D + ((a.n_splits + 3) & ~3) + kMWarps * D + D +
+                            static_cast<size_t>((a.n_full + 3) & ~3));
   if (msmem > 227 * 1024) return cudaErrorNotSupported;
   static size_t msmem_set = 0;
   if (msmem > msmem_set) {
@@ -1134,5 +1218,5 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
     scratch = g_noalloc_address[dev];
   }
   return status_from_cuda(launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out, scratch, sp,
-                                        static_cast<cudaStream_t>(stream)));
+                                        static_cast<cudaStream_t>(stream), DecodeExtra{}));
 }
