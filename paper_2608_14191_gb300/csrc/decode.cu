@@ -240,6 +240,14 @@ __global__ void __launch_bounds__(kQThreads)
     float v[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) v[k] = f[k] < lim ? xe[base + f[k]] : 0.0f;
+    // the split kernel masks digits in place: lane t's D2 digits arrive times 4^t, its D1 bits
+    // times 2^t (k 2t, 2t+1) and 2^(t+4) (k 2t+8, 2t+9); the query columns carry the inverse
+    const float s01 = ks < n2w ? pow2i(-2 * t) : pow2i(-t);
+    const float s89 = ks < n2w ? pow2i(-2 * t) : pow2i(-t - 4);
+    v[0] *= s01;
+    v[1] *= s01;
+    v[2] *= s89;
+    v[3] *= s89;
     uint32_t h01, l01, h89, l89;
     f16_split2(v[0], v[1], h01, l01);
     f16_split2(v[2], v[3], h89, l89);
@@ -382,6 +390,7 @@ __global__ void __launch_bounds__(kThreads)
   }
 
   // ---- pass 1: scores; warp = 32 tokens of each tile as four n-tiles of 8
+  const uint32_t m2 = 0x00030003u << (2 * t), m1a = 0x00010001u << t, m1b = 0x00010001u << (t + 4);
   float mloc = -INFINITY;                                      // lanes g < G: query g
   const float sg = g < G ? qcg[MAX_GROUP + g] : 0.0f, cg = g < G ? qcg[g] : 0.0f;
   for (int ti = 0; ti < n_tiles_split; ++ti) {
@@ -398,7 +407,7 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t x = w0[8 * j];
-        mma_f16(acc[j], af, (x >> (2 * t)) & 0x00030003u, (x >> (2 * t + 8)) & 0x00030003u);
+        mma_f16(acc[j], af, x & m2, (x >> 8) & m2);                // fields in place: digit * 4^t
       }
     }
     for (int u = 0; u < n1w_k; ++u) {
@@ -410,8 +419,10 @@ __global__ void __launch_bounds__(kThreads)
       for (int hs = 0; hs < 2; ++hs) {
         const uint4 af = afrag[(n2w_k + 2 * u + hs) * 32 + lane];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          mma_f16(acc[j], af, (x[j] >> (t + 8 * hs)) & 0x00010001u, (x[j] >> (t + 4 + 8 * hs)) & 0x00010001u);
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t y = hs ? x[j] >> 8 : x[j];
+          mma_f16(acc[j], af, y & m1a, y & m1b);                     // bits in place: * 2^t, 2^(t+4)
+        }
       }
     }
     if (g < G) {
@@ -462,20 +473,20 @@ __global__ void __launch_bounds__(kThreads)
   // offset of its slot in the tile (k16-step 0), its field shift and its mask.
   const int n_jobs = 2 * n2w_v + 4 * (nw_v - n2w_v);
   const int j0 = warp * n_jobs / kWarps, nj = (warp + 1) * n_jobs / kWarps - j0;
-  int joff[JPW], jsh[JPW];
+  int joff[JPW];
   uint32_t jmask[JPW];
 #pragma unroll
   for (int j = 0; j < JPW; ++j) {
     const int jj = j0 + j;
+    // fields masked in place: column g gets digit * 4^(g&3) (D2) or bit * 2^g (D1), divided out
+    // of the entry sums in the epilogue
     if (jj < 2 * n2w_v) {
       joff[j] = (jj >> 1) * TILE + 4 * t + 2 * (g >> 2) + (jj & 1);
-      jsh[j] = 2 * (g & 3);
-      jmask[j] = 0x00030003u;
+      jmask[j] = 0x00030003u << (2 * (g & 3));
     } else {
       const int u = jj - 2 * n2w_v, r = u & 3;
       joff[j] = (n2w_v + (u >> 2)) * TILE + 4 * t + ((r & 1) << 1) + (r >> 1);   // slot (0, 2, 1, 3)[r]
-      jsh[j] = g;
-      jmask[j] = 0x00010001u;
+      jmask[j] = 0x00010001u << g;
     }
   }
   float vacc[JPW][4];
@@ -526,7 +537,7 @@ __global__ void __launch_bounds__(kThreads)
         for (int j = 0; j < JPW; ++j)
           if (j < nj) {
             const uint32_t x = vt[joff[j] + 16 * ks];
-            mma_f16(vacc[j], af, (x >> jsh[j]) & jmask[j], (x >> (jsh[j] + 8)) & jmask[j]);
+            mma_f16(vacc[j], af, x & jmask[j], (x >> 8) & jmask[j]);
           }
       }
       __syncthreads();                                         // stage and pq free: refill
@@ -557,9 +568,13 @@ __global__ void __launch_bounds__(kThreads)
     for (int j = 0; j < JPW; ++j)
       if (j < nj) {
         const int jj = j0 + j;
-        const int ebase = jj < 2 * n2w_v ? 8 * jj : lv.n2 + 8 * (jj - 2 * n2w_v);   // 8 entries per n-tile
+        const bool d2 = jj < 2 * n2w_v;
+        const int ebase = d2 ? 8 * jj : lv.n2 + 8 * (jj - 2 * n2w_v);   // 8 entries per n-tile
+        // column n = 2t + c carried digit * 4^(n&3) (D2) or bit * 2^n (D1)
+        const float c0 = val_scale * (d2 ? pow2i(-2 * ((2 * t) & 3)) : pow2i(-2 * t));
+        const float c1 = val_scale * (d2 ? pow2i(-2 * ((2 * t + 1) & 3)) : pow2i(-2 * t - 1));
         *reinterpret_cast<float2*>(oe + g * a.n_entries + ebase + 2 * t) =
-            make_float2((vacc[j][0] + vacc[j][2]) * val_scale, (vacc[j][1] + vacc[j][3]) * val_scale);
+            make_float2((vacc[j][0] + vacc[j][2]) * c0, (vacc[j][1] + vacc[j][3]) * c1);
       }
   }
   __syncthreads();
