@@ -42,13 +42,13 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 namespace aatc {
 
 DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
-  // About four CTAs per SM in a single wave: n_splits per (sequence, kv-head), with split s
+  // About five CTAs per SM in a single wave: n_splits per (sequence, kv-head), with split s
   // covering tiles [s T / n_splits, (s + 1) T / n_splits) so split lengths differ by at most one
   // tile and every SM gets nearly the same number of tiles.  A split holds at most 16 tiles
   // (its scores are kept in shared memory).
   const long tiles = (n_ctx + TILE - 1) / TILE;
   const long units = static_cast<long>(batch) * n_kv;
-  const long target = 4L * std::max(1, num_sms);
+  const long target = 5L * std::max(1, num_sms);
   long n = (target + units / 2) / units;
   n = std::max(n, (tiles + 15) / 16);
   n = std::max(1L, std::min(n, tiles));

@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(kQThreads)
   }
 }
 
-constexpr int kStages = 4;                  // ring of record-word tiles (keys, then values)
+constexpr int kStages = 3;                  // ring of record-word tiles (keys, then values)
 
 __host__ __device__ constexpr int align16(int x) { return (x + 15) & ~15; }
 
