@@ -44,7 +44,9 @@ struct StreamLayout {
   int n1;                 // D1 entries
   int words;              // record words this stream uses
   int nret;               // retained channels R
-  int l2[4];              // D2 digit-layer lengths
+  int l2[4];              // D2 digit-layer lengths (digits kept in D2)
+  int l2all[4];           // channels with b >= 2k + 2 (digit k exists; those past l2[k] moved to D1)
+  int lodd[4];            // channels with b >= 2k + 1 (width 2k + 1 channels: [l2all[k], lodd[k]))
 };
 
 struct PlanDevice {

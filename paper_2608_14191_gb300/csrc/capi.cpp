@@ -92,6 +92,10 @@ void build_layout(const uint8_t* bits, StreamLayout* lay, std::vector<short>& en
         ++n;
       }
     lay->l2[k] = n;
+    lay->l2all[k] = n;
+    int m = 0;
+    for (int c = 0; c < D; ++c) m += bits[c] >= 2 * k + 1;
+    lay->lodd[k] = m;
   }
   for (int c = 0; c < D; ++c)
     if (bits[c] & 1) d1.push_back(ent(c, bits[c] - 1));

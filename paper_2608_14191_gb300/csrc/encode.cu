@@ -30,7 +30,6 @@ constexpr int kMmaWarp = kProducerWarp + 1;
 constexpr int kThreads = kEpiThreads + 64;
 constexpr int kAccCols = 128;                     // fp32 columns per accumulator
 constexpr uint32_t kTmemCols = 512;               // four accumulators
-constexpr int kMaxEntries = 32 * 32;              // 32 words x 32 one-bit fields
 constexpr int kByteRow = 132;                     // padded per-thread row of stored values
 
 struct EncodeArgs {
@@ -49,7 +48,6 @@ struct EncodeSmem {
   alignas(1024) unsigned char x_tile[kStages][kTileBytes];
   ChanEnc enc[D];
   float inv_s[D];
-  short entry[kMaxEntries];
   StreamLayout lay;
   uint32_t ubytes[kEpiThreads][kByteRow / 4];     // stored values u, one byte per channel
   uint64_t full[kStages], empty[kStages], tfull[kEpiGroups], tempty[kEpiGroups], ubar;
@@ -118,7 +116,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.enc[c] = a.enc[stream * D + c];
     sm.inv_s[c] = a.inv_s[stream * D + c];
   }
-  for (int e = tid; e < a.n_entries; e += kThreads) sm.entry[e] = a.entry[static_cast<size_t>(stream) * a.n_entries + e];
   if (tid == 0) {
     sm.lay = a.lay[stream];
     for (int s = 0; s < kStages; ++s) {
@@ -222,25 +219,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
 
-      // quantize: u = clamp(floor(h / Delta + 1/2)) + 2^(b-1), one byte per channel
-      uint32_t U[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) U[i] = 0u;
+      // quantize: u = clamp(floor(h / Delta + 1/2)) + 2^(b-1), one byte per channel.  The
+      // round-down add of 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         float h[32];
         ptx::tmem_ld_32cols(taddr + 32 * j, h);
         ptx::tmem_ld_wait();
+        uint32_t y[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const int c = 32 * j + i;
-          const ChanEnc e = sm.enc[c];
+          const ChanEnc e = sm.enc[32 * j + i];
           float x = fmaf(h[i], e.inv_f * ia, 0.5f);                // h / Delta + 1/2
           x = fminf(x, e.hi);                                       // |h| / Delta <= 2^(b-1): only the top clamps
-          const float y = __fadd_rd(x, e.magic);                    // floor, offset binary in the mantissa
-          const uint32_t u = __float_as_uint(y) - 0x4B400000u;
-          U[c >> 2] |= u << (8 * (c & 3));
+          y[i] = __float_as_uint(__fadd_rd(x, e.magic));            // floor, offset binary in the mantissa
         }
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          my_bytes[8 * j + q] = __byte_perm(__byte_perm(y[4 * q], y[4 * q + 1], 0x0040),
+                                            __byte_perm(y[4 * q + 2], y[4 * q + 3], 0x0040), 0x5410);
       }
       ptx::tc_fence_before();
       ptx::mbar_arrive(&sm.tempty[eg]);
@@ -260,35 +257,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       out.key_word = tile_words + tt;
       out.val_byte = reinterpret_cast<uint8_t*>(tile_words + 4 * (tt >> 2)) + (tt & 3);
 
-      // D2: base-4 digit k of channels 0..l2[k]-1, four channels at a time
+      // Record bit stream, four channels per step from this thread's byte row: field w bits at
+      // bit sh of channels [c0, c1) (w = 2: base-4 digit, w = 1: single bit), gathered by one
+      // multiply and appended LSB first.
       uint32_t word = 0;
       int pos = 0, wi = 0;
+      auto emit_run = [&](int c0, int c1, int sh, int w) {
+        for (int g4 = c0 >> 2; 4 * g4 < c1; ++g4) {
+          const int skip = max(c0 - 4 * g4, 0), n = min(c1 - 4 * g4, 4) - skip;
+          const uint32_t x = my_bytes[g4] >> sh;
+          uint32_t y = w == 2 ? (((x & 0x03030303u) * 0x00041041u) >> 18) & 0xFFu
+                              : (((x & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
+          y = (y >> (w * skip)) & ((1u << (w * n)) - 1u);
+          append_bits(y, w * n, word, pos, wi, out);
+        }
+      };
 #pragma unroll 1
-      for (int k = 0; k < 4; ++k) {
-        const int L = lay.l2[k];
-        if (L == 0) continue;
-#pragma unroll
-        for (int g4 = 0; g4 < 32; ++g4) {
-          if (4 * g4 < L) {
-            const int n = min(4, L - 4 * g4);
-            const uint32_t x = (U[g4] >> (2 * k)) & 0x03030303u;
-            uint32_t y = ((x * 0x00041041u) >> 18) & 0xFFu;           // gather the four 2-bit digits
-            y &= (1u << (2 * n)) - 1u;
-            append_bits(y, 2 * n, word, pos, wi, out);
-          }
-        }
-      }
-      // D1: single bits listed in the entry table after the n2 digits
-      if (lay.n1 > 0) {
-#pragma unroll
-        for (int q = 0; q < 32; ++q) my_bytes[q] = U[q];
-        const unsigned char* ub = reinterpret_cast<const unsigned char*>(my_bytes);
-        for (int e = 0; e < lay.n1; ++e) {
-          const int ce = sm.entry[lay.n2 + e];
-          const uint32_t bit = (static_cast<uint32_t>(ub[ce & 0xFF]) >> (ce >> 8)) & 1u;
-          append_bits(bit, 1, word, pos, wi, out);
-        }
-      }
+      for (int k = 0; k < 4; ++k) emit_run(0, lay.l2[k], 2 * k, 2);                 // D2 digits
+#pragma unroll 1
+      for (int k = 3; k >= 0; --k) emit_run(lay.l2all[k], lay.lodd[k], 2 * k, 1);  // D1: top bits of odd widths
+#pragma unroll 1
+      for (int k = 0; k < 4; ++k) emit_run(lay.l2[k], lay.l2all[k], 2 * k, 2);     // D1: digits moved out of D2
       if (pos > 0) {
         out.put(wi, word);
         ++wi;
