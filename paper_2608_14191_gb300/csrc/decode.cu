@@ -218,11 +218,15 @@ __global__ void __launch_bounds__(kQThreads)
     }
   }
   __syncthreads();
-  // fragment of lane (slot, t) for k-step ks: registers (row slot, k 2t | 2t+1), (row slot + 8,
-  // same k), (row slot, k 2t+8 | 2t+9), (row slot + 8, ...)
+  // B fragments of the score MMA (tokens are the M rows, query columns the N = 8): head group
+  // p = slot / 4 holds column g = slot % 4 (hi) and g + 4 (lo); lane (g, t) of k-step ks gets
+  // (k 2t | 2t+1, k 2t+8 | 2t+9) of its column at fragment [ks][p][lane].
   const int n2w = lk.n2 / 16, n1w = (lk.n1 + 31) / 32;
   const int n_ks = n2w + 2 * n1w;
-  uint4* dst = a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride;
+  const int np = (G + 3) / 4;
+  if (slot >= 4 * np) return;                          // beyond the last head group
+  const int p = slot >> 2, gs = slot & 3;
+  uint2* dst = reinterpret_cast<uint2*>(a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride);
   for (int i = tid; i < n_ks * 4; i += kQThreads) {
     const int ks = i >> 2, t = i & 3;
     int f[4];                                          // record fields of k = 2t, 2t+1, 2t+8, 2t+9
@@ -241,7 +245,7 @@ __global__ void __launch_bounds__(kQThreads)
 #pragma unroll
     for (int k = 0; k < 4; ++k) v[k] = f[k] < lim ? xe[base + f[k]] : 0.0f;
     // the split kernel masks digits in place: lane t's D2 digits arrive times 4^t, its D1 bits
-    // times 2^t (k 2t, 2t+1) and 2^(t+4) (k 2t+8, 2t+9); the query columns carry the inverse
+    // times 2^t (k 2t, 2t+1) and 2^(t+4) (k 2t+8, 2t+9); the query rows carry the inverse
     const float s01 = ks < n2w ? pow2i(-2 * t) : pow2i(-t);
     const float s89 = ks < n2w ? pow2i(-2 * t) : pow2i(-t - 4);
     v[0] *= s01;
@@ -251,7 +255,8 @@ __global__ void __launch_bounds__(kQThreads)
     uint32_t h01, l01, h89, l89;
     f16_split2(v[0], v[1], h01, l01);
     f16_split2(v[2], v[3], h89, l89);
-    dst[ks * 32 + 4 * slot + t] = make_uint4(h01, l01, h89, l89);
+    dst[(ks * np + p) * 32 + 4 * gs + t] = make_uint2(h01, h89);
+    dst[(ks * np + p) * 32 + 4 * (gs + 4) + t] = make_uint2(l01, l89);
   }
   if (tid == 0) {
     float* qc = a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP;
@@ -319,11 +324,11 @@ __global__ void __launch_bounds__(kThreads)
   float* red = reinterpret_cast<float*>(smb + L.red);
   const short* cetab = reinterpret_cast<const short*>(smb + L.cetab);
   const short* etab = reinterpret_cast<const short*>(smb + L.etab);
-  const uint4* afrag = reinterpret_cast<const uint4*>(smb + L.afrag);
+  const uint2* afrag = reinterpret_cast<const uint2*>(smb + L.afrag);  // [k-step][head group][lane]
   float* ak = reinterpret_cast<float*>(smb + L.ak);
   float* av = reinterpret_cast<float*>(smb + L.av);
   float* sbuf = reinterpret_cast<float*>(smb + L.sbuf);        // [4 NP][sb_stride]
-  uint4* pq = reinterpret_cast<uint4*>(smb + L.pq);            // [8 k16-steps][32 lanes]
+  uint2* pq = reinterpret_cast<uint2*>(smb + L.pq);            // [8 k16-steps][head group][32 lanes]
   uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
   const int sbs = L.sb_stride;
 
@@ -368,7 +373,7 @@ __global__ void __launch_bounds__(kThreads)
     // cache words and scales do not depend on the query kernel: start them first
     const uint32_t abytes = static_cast<uint32_t>(n_tiles_split) * TILE * 4;
     const uint32_t ebytes = static_cast<uint32_t>(align16(a.n_entries * 2));
-    const uint32_t fbytes = static_cast<uint32_t>(n_ks) * 32 * 16;
+    const uint32_t fbytes = static_cast<uint32_t>(n_ks) * NP * 32 * 8;
     ptx::mbar_arrive_expect_tx(pro, 2 * abytes + D * 8 * 2 + ebytes + fbytes + 2 * MAX_GROUP * 4);
     ptx::bulk_load(ak, kalpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
     for (int i = 0; i < min(kStages, n_seq); ++i) issue_tile(i);
@@ -380,63 +385,92 @@ __global__ void __launch_bounds__(kThreads)
     ptx::bulk_load(smb + L.afrag, a.qfrag + (static_cast<size_t>(b) * a.n_kv + head) * a.ks_stride, fbytes, pro);
     ptx::bulk_load(qcg, a.qcorr + (static_cast<size_t>(b) * a.n_kv + head) * 2 * MAX_GROUP, 2 * MAX_GROUP * 4, pro);
   }
-  // P' rows of absent queries (g >= G) stay zero for the whole split
-  for (int i = tid; i < (TILE / 16) * 32; i += kThreads)
-    if (((i & 31) >> 2) >= G) pq[i] = make_uint4(0u, 0u, 0u, 0u);
+  // P' columns of absent queries (q >= G) stay zero for the whole split
+  for (int i = tid; i < (TILE / 16) * NP * 32; i += kThreads) {
+    const int gcol = (i & 31) >> 2, q = 4 * ((i >> 5) % NP) + (gcol & 3);
+    if (q >= G) pq[i] = make_uint2(0u, 0u);
+  }
   __syncthreads();
   if (!ptx::mbar_wait_sleep(pro, 0, &s_abort, 200)) {
     s_abort = 1;
     atomicOr(a.err, 2);
   }
 
-  // ---- pass 1: scores; warp = 32 tokens of each tile as four n-tiles of 8
+  // ---- pass 1: scores.  Warp = 32 tokens of each tile; lane (g, t) reads the record words of
+  // tokens 4g .. 4g + 3 (one 128-bit load per k-step): M-tile 0 has rows g, g + 8 = tokens 4g,
+  // 4g + 1, M-tile 1 tokens 4g + 2, 4g + 3; head group p gives the N = 8 query columns.
   const uint32_t m2 = 0x00030003u << (2 * t), m1a = 0x00010001u << t, m1b = 0x00010001u << (t + 4);
-  float mloc = -INFINITY;                                      // lanes g < G: query g
-  const float sg = g < G ? qcg[MAX_GROUP + g] : 0.0f, cg = g < G ? qcg[g] : 0.0f;
+  // after the hi/lo exchange lane (g, t) owns heads 4p + 2(t & 1) + {0, 1} of tokens
+  // 4g + 2 (t >> 1) + {0, 1}
+  const int h_own = 2 * (t & 1), tk_own = 4 * g + 2 * (t >> 1);
+  float mloc[NP][2];
+  float sg[NP][2], cg[NP][2];
+#pragma unroll
+  for (int p = 0; p < NP; ++p)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int q = 4 * p + h_own + i;
+      mloc[p][i] = -INFINITY;
+      sg[p][i] = q < G ? qcg[MAX_GROUP + q] : 0.0f;
+      cg[p][i] = q < G ? qcg[q] : 0.0f;
+    }
   for (int ti = 0; ti < n_tiles_split; ++ti) {
     wait_tile(ti);
-    const uint32_t* kt = ring + (ti % kStages) * W * TILE + 32 * warp + g;
-    float acc[4][4];
+    const uint4* kt = reinterpret_cast<const uint4*>(ring + (ti % kStages) * W * TILE + 32 * warp + 4 * g);
+    float acc[2][NP][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
+    for (int mh = 0; mh < 2; ++mh)
 #pragma unroll
-      for (int r = 0; r < 4; ++r) acc[j][r] = 0.0f;
+      for (int p = 0; p < NP; ++p)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) acc[mh][p][r] = 0.0f;
     for (int ks = 0; ks < n2w_k; ++ks) {
-      const uint4 af = afrag[ks * 32 + lane];
-      const uint32_t* w0 = kt + ks * TILE;
+      const uint4 x = kt[ks * (TILE / 4)];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t x = w0[8 * j];
-        mma_f16(acc[j], af, x & m2, (x >> 8) & m2);                // fields in place: digit * 4^t
+      for (int p = 0; p < NP; ++p) {
+        const uint2 bf = afrag[(ks * NP + p) * 32 + lane];
+        mma_f16(acc[0][p], make_uint4(x.x & m2, x.y & m2, (x.x >> 8) & m2, (x.y >> 8) & m2), bf.x, bf.y);
+        mma_f16(acc[1][p], make_uint4(x.z & m2, x.w & m2, (x.z >> 8) & m2, (x.w >> 8) & m2), bf.x, bf.y);
       }
     }
     for (int u = 0; u < n1w_k; ++u) {
-      const uint32_t* w0 = kt + (n2w_k + u) * TILE;
-      uint32_t x[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) x[j] = w0[8 * j];
+      const uint4 x = kt[(n2w_k + u) * (TILE / 4)];
 #pragma unroll
       for (int hs = 0; hs < 2; ++hs) {
-        const uint4 af = afrag[(n2w_k + 2 * u + hs) * 32 + lane];
+        const uint32_t y0 = hs ? x.x >> 8 : x.x, y1 = hs ? x.y >> 8 : x.y;
+        const uint32_t y2 = hs ? x.z >> 8 : x.z, y3 = hs ? x.w >> 8 : x.w;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t y = hs ? x[j] >> 8 : x[j];
-          mma_f16(acc[j], af, y & m1a, y & m1b);                     // bits in place: * 2^t, 2^(t+4)
+        for (int p = 0; p < NP; ++p) {
+          const uint2 bf = afrag[((n2w_k + 2 * u + hs) * NP + p) * 32 + lane];
+          mma_f16(acc[0][p], make_uint4(y0 & m1a, y1 & m1a, y0 & m1b, y1 & m1b), bf.x, bf.y);   // bits in place
+          mma_f16(acc[1][p], make_uint4(y2 & m1a, y3 & m1a, y2 & m1b, y3 & m1b), bf.x, bf.y);
         }
       }
     }
-    if (g < G) {
-      const int tbase = (tile0 + ti) * TILE;
+    // columns 2t, 2t + 1 hold hi (t < 2) or lo (t >= 2) of heads 4p + 2(t & 1) + {0, 1}: lanes t
+    // and t ^ 2 exchange so each owns the hi + lo sums of two tokens
+    const int tk = ti * TILE + 32 * warp + tk_own;             // token of the split
+    const float2 a2 = *reinterpret_cast<const float2*>(ak + tk);
+    const int tb = t_begin + tk;
+    const bool ok0 = tb >= t_lo && tb < t_end, ok1 = tb + 1 >= t_lo && tb + 1 < t_end;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int tk = 32 * warp + 8 * j + 2 * t;
-        const float2 a2 = *reinterpret_cast<const float2*>(ak + ti * TILE + tk);
-        float s0 = a2.x * fmaf(acc[j][0] + acc[j][2], sg, -cg);
-        float s1 = a2.y * fmaf(acc[j][1] + acc[j][3], sg, -cg);
-        s0 = tbase + tk < t_end && tbase + tk >= t_lo ? s0 : -INFINITY;
-        s1 = tbase + tk + 1 < t_end && tbase + tk + 1 >= t_lo ? s1 : -INFINITY;
-        *reinterpret_cast<float2*>(sbuf + g * sbs + ti * TILE + tk) = make_float2(s0, s1);
-        mloc = fmaxf(mloc, fmaxf(s0, s1));
+    for (int p = 0; p < NP; ++p) {
+      float r[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float mine = t < 2 ? acc[0][p][i] : acc[1][p][i];
+        const float give = t < 2 ? acc[1][p][i] : acc[0][p][i];
+        r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int q = 4 * p + h_own + i;
+        if (q < G) {
+          const float s0 = ok0 ? a2.x * fmaf(r[i], sg[p][i], -cg[p][i]) : -INFINITY;       // c0 / c1: token A
+          const float s1 = ok1 ? a2.y * fmaf(r[2 + i], sg[p][i], -cg[p][i]) : -INFINITY;   // c2 / c3: token B
+          *reinterpret_cast<float2*>(sbuf + q * sbs + tk) = make_float2(s0, s1);
+          mloc[p][i] = fmaxf(mloc[p][i], fmaxf(s0, s1));
+        }
       }
     }
     __syncthreads();                                           // stage free: refill
@@ -451,9 +485,17 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) amx = fmaxf(amx, __shfl_xor_sync(0xffffffffu, amx, o));
   if (lane == 0) red[3 * kWarps * MAX_GROUP + warp] = amx;
-  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 1));
-  mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, 2));
-  if (t == 0) red[warp * MAX_GROUP + g] = mloc;
+#pragma unroll
+  for (int p = 0; p < NP; ++p)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      float v = mloc[p][i];
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+      v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+      if (lane < 2) red[warp * MAX_GROUP + 4 * p + 2 * lane + i] = v;      // lane t = lane < 2
+    }
   __syncthreads();
   float* mqs = red + 2 * kWarps * MAX_GROUP + 3 * MAX_GROUP;  // [MAX_GROUP] split max per query
   if (tid < MAX_GROUP)
@@ -467,38 +509,44 @@ __global__ void __launch_bounds__(kThreads)
   const float val_scale = amx * (kDigitScale / kOpMax);        // raw sum -> sum P' code
   __syncthreads();                                             // split maxima visible to pass 2
 
-  // ---- pass 2: P' (thread = 4 tokens x 1 query) and the value product over the split
-  // Value n-tile jobs: a D2 word is two n-tiles (byte-quarters 0,1 and 2,3), a D1 word four
-  // (one per quarter).  Warp w takes jobs [w J / 4, (w+1) J / 4); per job this lane keeps the
-  // offset of its slot in the tile (k16-step 0), its field shift and its mask.
-  const int n_jobs = 2 * n2w_v + 4 * (nw_v - n2w_v);
+  // ---- pass 2: P' (thread = 4 tokens x 1 query) and the value product over the split.
+  // Value M-tiles ("jobs", 16 record entries each): a D2 word is one (fields g, g + 8 of lane row
+  // g: slots 2(g / 4), 2(g / 4) + 1 of a token quad), a D1 word two (quarters 0, 1 or 2, 3:
+  // slots hb, hb + 2).  Lane (g, t) of k-step ks reads token quad 4 ks + t; per job it keeps the
+  // offsets of its two slots in the tile and its field mask.  Warp w takes jobs
+  // [w J / 4, (w+1) J / 4).
+  const int n_jobs = n2w_v + 2 * (nw_v - n2w_v);
   const int j0 = warp * n_jobs / kWarps, nj = (warp + 1) * n_jobs / kWarps - j0;
-  int joff[JPW];
+  int joff[JPW], jsec[JPW];
   uint32_t jmask[JPW];
 #pragma unroll
   for (int j = 0; j < JPW; ++j) {
     const int jj = j0 + j;
-    // fields masked in place: column g gets digit * 4^(g&3) (D2) or bit * 2^g (D1), divided out
+    // fields masked in place: a row gets digit * 4^(g & 3) (D2) or bit * 2^g (D1), divided out
     // of the entry sums in the epilogue
-    if (jj < 2 * n2w_v) {
-      joff[j] = (jj >> 1) * TILE + 4 * t + 2 * (g >> 2) + (jj & 1);
+    if (jj < n2w_v) {
+      joff[j] = jj * TILE + 2 * (g >> 2);
+      jsec[j] = 1;
       jmask[j] = 0x00030003u << (2 * (g & 3));
     } else {
-      const int u = jj - 2 * n2w_v, r = u & 3;
-      joff[j] = (n2w_v + (u >> 2)) * TILE + 4 * t + ((r & 1) << 1) + (r >> 1);   // slot (0, 2, 1, 3)[r]
+      const int u = jj - n2w_v;
+      joff[j] = (n2w_v + (u >> 1)) * TILE + (u & 1);
+      jsec[j] = 2;
       jmask[j] = 0x00010001u << g;
     }
   }
-  float vacc[JPW][4];
+  float vacc[JPW][NP][4];
 #pragma unroll
   for (int j = 0; j < JPW; ++j)
 #pragma unroll
-    for (int z = 0; z < 4; ++z) vacc[j][z] = 0.0f;
+    for (int p = 0; p < NP; ++p)
+#pragma unroll
+      for (int z = 0; z < 4; ++z) vacc[j][p][z] = 0.0f;
   float lsum[NP], ssum[NP];
 #pragma unroll
   for (int p = 0; p < NP; ++p) lsum[p] = ssum[p] = 0.0f;
   {
-    // tokens 4 Q .. 4 Q + 3 with Q = 8 warp + Qk (k16-step Q / 4, fragment lane column t = Q % 4)
+    // tokens 4 Q .. 4 Q + 3 with Q = 8 warp + Qk (k-step Q / 4, fragment lane column t = Q % 4)
     const int qq = lane >> 3, Qk = lane & 7, Q = 8 * warp + Qk;
     const int tk0 = 4 * Q;
     for (int ti = 0; ti < n_tiles_split; ++ti) {
@@ -525,19 +573,27 @@ __global__ void __launch_bounds__(kThreads)
             const float2 r02 = f16_split2(p0 * av0, p2 * av2, h02, l02);   // tokens 0, 2 (k 2t, 2t+1)
             const float2 r13 = f16_split2(p1 * av1, p3 * av3, h13, l13);   // tokens 1, 3 (k 2t+8, 2t+9)
             ssum[p] += (r02.x + r02.y) + (r13.x + r13.y);                  // what the MMA sees
-            pq[(Q >> 2) * 32 + 4 * q + (Q & 3)] = make_uint4(h02, l02, h13, l13);
+            uint2* dst = pq + ((Q >> 2) * NP + p) * 32 + (Q & 3);
+            dst[4 * qq] = make_uint2(h02, h13);                            // column qq: hi
+            dst[4 * (qq + 4)] = make_uint2(l02, l13);                      // column qq + 4: lo
           }
         }
       }
       __syncthreads();
 #pragma unroll
       for (int ks = 0; ks < TILE / 16; ++ks) {
-        const uint4 af = pq[ks * 32 + lane];                   // B column token quad 4 ks + t
+        uint2 bf[NP];
+#pragma unroll
+        for (int p = 0; p < NP; ++p) bf[p] = pq[(ks * NP + p) * 32 + lane];   // column g, quad 4 ks + t
 #pragma unroll
         for (int j = 0; j < JPW; ++j)
           if (j < nj) {
-            const uint32_t x = vt[joff[j] + 16 * ks];
-            mma_f16(vacc[j], af, x & jmask[j], (x >> 8) & jmask[j]);
+            const uint32_t* src = vt + joff[j] + 4 * (4 * ks + t);
+            const uint32_t xa = src[0], xb = src[jsec[j]];
+            const uint32_t mk = jmask[j];
+            const uint4 af = make_uint4(xa & mk, xb & mk, (xa >> 8) & mk, (xb >> 8) & mk);
+#pragma unroll
+            for (int p = 0; p < NP; ++p) mma_f16(vacc[j][p], af, bf[p].x, bf[p].y);
           }
       }
       __syncthreads();                                         // stage and pq free: refill
@@ -563,19 +619,39 @@ __global__ void __launch_bounds__(kThreads)
       red[warp * MAX_GROUP + 4 * p + (lane >> 3)] = lsum[p];
       red[(kWarps + warp) * MAX_GROUP + 4 * p + (lane >> 3)] = ssum[p];
     }
-  if (g < G) {
+  {
+    // columns 2t, 2t + 1: hi (t < 2) / lo (t >= 2) of heads 4p + 2(t & 1) + {0, 1}; after the
+    // exchange lanes t < 2 own entry row g, lanes t >= 2 entry row g + 8
 #pragma unroll
-    for (int j = 0; j < JPW; ++j)
-      if (j < nj) {
-        const int jj = j0 + j;
-        const bool d2 = jj < 2 * n2w_v;
-        const int ebase = d2 ? 8 * jj : lv.n2 + 8 * (jj - 2 * n2w_v);   // 8 entries per n-tile
-        // column n = 2t + c carried digit * 4^(n&3) (D2) or bit * 2^n (D1)
-        const float c0 = val_scale * (d2 ? pow2i(-2 * ((2 * t) & 3)) : pow2i(-2 * t));
-        const float c1 = val_scale * (d2 ? pow2i(-2 * ((2 * t + 1) & 3)) : pow2i(-2 * t - 1));
-        *reinterpret_cast<float2*>(oe + g * a.n_entries + ebase + 2 * t) =
-            make_float2((vacc[j][0] + vacc[j][2]) * c0, (vacc[j][1] + vacc[j][3]) * c1);
+    for (int j = 0; j < JPW; ++j) {
+      const int jj = j0 + j;
+      int e = 0;
+      float sc = 0.0f;
+      if (jj < n2w_v) {
+        e = 16 * jj + g + 8 * (t >> 1);
+        sc = val_scale * pow2i(-2 * (g & 3));
+      } else {
+        const int u = jj - n2w_v;
+        e = lv.n2 + 32 * (u >> 1) + 16 * (u & 1) + g + 8 * (t >> 1);
+        sc = val_scale * pow2i(-g);
       }
+#pragma unroll
+      for (int p = 0; p < NP; ++p) {
+        float r[2];
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const float mine = t < 2 ? vacc[j][p][i] : vacc[j][p][2 + i];
+          const float give = t < 2 ? vacc[j][p][2 + i] : vacc[j][p][i];
+          r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
+        }
+        if (j < nj && e < lv.n2 + lv.n1)
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            const int q = 4 * p + h_own + i;
+            if (q < G) oe[q * a.n_entries + e] = r[i] * sc;
+          }
+      }
+    }
   }
   __syncthreads();
   float* ml = red + 2 * kWarps * MAX_GROUP;                    // [3][MAX_GROUP]: m, l, S'
@@ -1052,9 +1128,9 @@ cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStre
 
 template <int NP>
 cudaError_t launch_split_g(const DecodeArgs& a, int batch, int jpw, size_t smem, cudaStream_t st) {
+  if (jpw <= 4) return launch_split_t<4, NP>(a, batch, smem, st);
   if (jpw <= 8) return launch_split_t<8, NP>(a, batch, smem, st);
-  if (jpw <= 12) return launch_split_t<12, NP>(a, batch, smem, st);
-  return launch_split_t<16, NP>(a, batch, smem, st);
+  return launch_split_t<12, NP>(a, batch, smem, st);
 }
 
 template <int GP>
@@ -1118,7 +1194,7 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     const StreamLayout& lk = plan.layout[(layer * a.n_kv + h) * 2];
     const StreamLayout& lv = plan.layout[(layer * a.n_kv + h) * 2 + 1];
     n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
-    n_jobs_v = std::max(n_jobs_v, 2 * (lv.n2 / 16) + 4 * ((lv.n1 + 31) / 32));
+    n_jobs_v = std::max(n_jobs_v, lv.n2 / 16 + 2 * ((lv.n1 + 31) / 32));
   }
   const int np = (a.group + 3) / 4;
   const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
@@ -1133,8 +1209,8 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     if (e != cudaSuccess) return e;
     const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
     const size_t smem = static_cast<size_t>(L.total);
-    const int jpw = (n_jobs_v + kWarps - 1) / kWarps;          // value n-tiles per warp
-    if (jpw > 16 || smem > 227 * 1024) return cudaErrorNotSupported;
+    const int jpw = (n_jobs_v + kWarps - 1) / kWarps;          // value M-tiles per warp
+    if (jpw > 12 || smem > 227 * 1024) return cudaErrorNotSupported;
     e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
     if (e != cudaSuccess) return e;
   }
