@@ -699,15 +699,14 @@ __global__ void __launch_bounds__(kThreads)
 // the original basis and merged with the packed part by log-sum-exp.
 // Launched as a programmatic dependent of the split kernel: U_V^T (a plan constant) is staged
 // while the splits finish; the partials are read only after the grid dependency resolves.
-constexpr int kMThreads = 256;
+constexpr int kMThreads = 512;
 constexpr int kMWarps = kMThreads / 32;
 
 __global__ void __launch_bounds__(kMThreads)
     aatc_decode_merge_kernel(const DecodeArgs a) {
   extern __shared__ __align__(16) float ms[];
   float* ut_s = ms;                                  // [128 c][128 d]
-  float* wsp = ut_s + D * D;                         // [n_splits] split weights
-  float* osum = wsp + ((a.n_splits + 3) & ~3);       // [kMWarps][128]
+  float* osum = ut_s + D * D;                        // [kMWarps][128]
   float* ohat = osum + kMWarps * D;                  // [128]
   float* sf = ohat + D;                              // [n_full] scores, then weights, of full tokens
   __shared__ float red[2][kMWarps];
@@ -766,76 +765,69 @@ __global__ void __launch_bounds__(kMThreads)
 #pragma unroll
     for (int w = 0; w < kMWarps; ++w) l_f += red[1][w];
     {
-      // two threads per dimension, alternate tokens
-      const int d = tid & (D - 1), half = tid >> 7;
+      // four threads per dimension, tokens t = quarter (mod 4)
+      const int d = tid & (D - 1), qtr = tid >> 7;
       float acc = 0.0f;
-      for (int t = half; t < a.n_full; t += 2)
+      for (int t = qtr; t < a.n_full; t += 4)
         acc = fmaf(sf[t], __bfloat162float(a.v_full[((static_cast<size_t>(b) * a.full_cap + t) * a.n_kv + head) * D + d]), acc);
-      osum[half * D + d] = acc;
+      osum[qtr * D + d] = acc;
     }
     __syncthreads();
-    if (tid < D) of = osum[tid] + osum[D + tid];
+    if (tid < D) of = (osum[tid] + osum[D + tid]) + (osum[2 * D + tid] + osum[3 * D + tid]);
     __syncthreads();
   }
-  // ---- packed splits
+  // ---- packed splits: warp w merges splits w, w + 16, ... online (running max, rescaled sums),
+  // eight splits' loads in flight per round; then the 16 warp partials are merged per channel.
   float M = -INFINITY, L = 0.0f;
   if (a.n_splits > 0) {
     ptx::grid_dependency_wait();                     // the split kernel's partials
     const float* src = a.ws + (static_cast<size_t>(b) * a.n_q + j) * a.n_splits * a.pstride;
-    for (int s = tid; s < a.n_splits; s += kMThreads) M = fmaxf(M, __ldcg(src + s * a.pstride + D));
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    if (lane == 0) red[0][warp] = M;
-    __syncthreads();
-    M = red[0][0];
-#pragma unroll
-    for (int w = 1; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
-    float l = 0.0f;
-    for (int s = tid; s < a.n_splits; s += kMThreads) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(src + s * a.pstride + D));
-      const float w = exp2f(ml.x - M);
-      wsp[s] = w;
-      l = fmaf(w, ml.y, l);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (lane == 0) red[1][warp] = l;
-    __syncthreads();
-    // weighted channel sums: warp = splits s = warp (mod 8), lane = channels 4 lane .. 4 lane + 3
+    float mw = -INFINITY, lw = 0.0f;
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-    int s = warp;
-    for (; s + kMWarps * 7 < a.n_splits; s += kMWarps * 8) {
+    for (int s0 = warp; s0 < a.n_splits; s0 += kMWarps * 8) {
+      float2 ml[8];
       float4 v[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s + kMWarps * u) * a.pstride + 4 * lane));
-#pragma unroll
       for (int u = 0; u < 8; ++u) {
-        const float w = wsp[s + kMWarps * u];
-        acc.x = fmaf(w, v[u].x, acc.x);
-        acc.y = fmaf(w, v[u].y, acc.y);
-        acc.z = fmaf(w, v[u].z, acc.z);
-        acc.w = fmaf(w, v[u].w, acc.w);
+        const int s = s0 + kMWarps * u;
+        if (s < a.n_splits) {
+          ml[u] = __ldcg(reinterpret_cast<const float2*>(src + static_cast<size_t>(s) * a.pstride + D));
+          v[u] = __ldcg(reinterpret_cast<const float4*>(src + static_cast<size_t>(s) * a.pstride + 4 * lane));
+        } else {
+          ml[u] = make_float2(-INFINITY, 0.0f);
+          v[u] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        }
+      }
+      float mc = mw;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mc = fmaxf(mc, ml[u].x);
+      if (mc > -INFINITY) {                          // else nothing attended so far: sums stay 0
+        const float r = exp2f(mw - mc);              // mw = -inf -> 0
+        lw *= r;
+        acc.x *= r; acc.y *= r; acc.z *= r; acc.w *= r;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float w = exp2f(ml[u].x - mc);
+          lw = fmaf(w, ml[u].y, lw);
+          acc.x = fmaf(w, v[u].x, acc.x);
+          acc.y = fmaf(w, v[u].y, acc.y);
+          acc.z = fmaf(w, v[u].z, acc.z);
+          acc.w = fmaf(w, v[u].w, acc.w);
+        }
+        mw = mc;
       }
     }
-    float4 v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (s + kMWarps * u < a.n_splits)
-        v[u] = __ldcg(reinterpret_cast<const float4*>(src + (s + kMWarps * u) * a.pstride + 4 * lane));
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (s + kMWarps * u < a.n_splits) {
-        const float w = wsp[s + kMWarps * u];
-        acc.x = fmaf(w, v[u].x, acc.x);
-        acc.y = fmaf(w, v[u].y, acc.y);
-        acc.z = fmaf(w, v[u].z, acc.z);
-        acc.w = fmaf(w, v[u].w, acc.w);
-      }
     *reinterpret_cast<float4*>(osum + warp * D + 4 * lane) = acc;
+    if (lane == 0) {
+      red[0][warp] = mw;
+      red[1][warp] = lw;
+    }
     __syncthreads();
 #pragma unroll
-    for (int w = 0; w < kMWarps; ++w) L += red[1][w];
+    for (int w = 0; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
+    if (M > -INFINITY)
+#pragma unroll
+      for (int w = 0; w < kMWarps; ++w) L = fmaf(exp2f(red[0][w] - M), red[1][w], L);
   }
   // ---- log-sum-exp merge of the two parts: out = (U_V (f o) a_p + o_f a_f) / (L a_p + l_f a_f)
   const float Mt = fmaxf(M, m_f);
@@ -844,25 +836,26 @@ __global__ void __launch_bounds__(kMThreads)
   const float inv_den = 1.0f / fmaf(L, ap, l_f * af);
   if (tid < D) {
     float o = 0.0f;
-    if (a.n_splits > 0) {
+    if (a.n_splits > 0 && M > -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < kMWarps; ++w) o += osum[w * D + tid];
+      for (int w = 0; w < kMWarps; ++w) o = fmaf(exp2f(red[0][w] - M), osum[w * D + tid], o);
     }
     ohat[tid] = o * fv * ap;
   }
   if (!ptx::mbar_wait_sleep(&bar, 0, &s_abort, 100)) atomicOr(a.err, 2);
   __syncthreads();
-  // out[d] = sum_c U_V[d][c] o_hat[c]: two threads per dimension, halves of c
+  // out[d] = sum_c U_V[d][c] o_hat[c]: four threads per dimension, quarters of c
   {
-    const int d = tid & (D - 1), half = tid >> 7;
+    const int d = tid & (D - 1), qtr = tid >> 7;
     float r = 0.0f;
 #pragma unroll 16
-    for (int c = half * 64; c < half * 64 + 64; ++c) r = fmaf(ut_s[c * D + d], ohat[c], r);
-    osum[half * D + d] = r;
+    for (int c = qtr * 32; c < qtr * 32 + 32; ++c) r = fmaf(ut_s[c * D + d], ohat[c], r);
+    osum[qtr * D + d] = r;
   }
   __syncthreads();
   if (tid < D)
-    a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] = (osum[tid] + osum[D + tid] + of * af) * inv_den;
+    a.out[(static_cast<size_t>(b) * a.n_q + j) * D + tid] =
+        ((osum[tid] + osum[D + tid]) + (osum[2 * D + tid] + osum[3 * D + tid]) + of * af) * inv_den;
 }
 
 // ---------------------------------------------------------------- bf16 reference decode
@@ -1214,8 +1207,7 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
     if (e != cudaSuccess) return e;
   }
-  const size_t msmem = 4 * (static_cast<size_t>(D) * D + ((a.n_splits + 3) & ~3) + kMWarps * D + D +
-                            static_cast<size_t>((a.n_full + 3) & ~3));
+  const size_t msmem = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
   if (msmem > 227 * 1024) return cudaErrorNotSupported;
   static size_t msmem_set = 0;
   if (msmem > msmem_set) {
