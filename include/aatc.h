@@ -121,6 +121,44 @@ aatc_status_t aatc_allocate_global(const aatc_dims_t* dims, const double* sigma2
                                    double avg_bits_k, double avg_bits_v, int32_t n_protect, uint8_t* bits_out);
 
 /*
+ * Transform from the model weights (Sec. 5 Step 1 "Whitening-Based Feature Decorrelation", Eq.
+ * AB-factorization; Appendix Proposition).  For one head's projection W (d_model x 128) and
+ * calibration activations X (n x d_model) it returns the paper's factorization W = A B of the
+ * whitened SVD W~ = L^T W = U S P^T (Sigma_X = X^T X / n = L L^T): A = L^-T U sqrt(S),
+ * B = sqrt(S) P^T.  Computed without forming L: W~^T W~ = W^T Sigma_X W = K^T K / n for K = X W,
+ * so P and S^2 are the eigenvectors / eigenvalues of K^T K / n (fp64 Jacobi, descending, each
+ * column's largest-|entry| positive, U flipped alike) and A = W P S^-1/2 (U = W~ P S^-1).
+ *   x        : host fp32 [n][d_model] calibration activations
+ *   w        : host fp32 [d_model][128] one head's key or value projection
+ *   a_out    : host fp32 [d_model][128] or NULL      b_out : host fp32 [128][128] or NULL
+ *   s_out    : host fp64 [128] singular values (descending) or NULL
+ *   p_out    : host fp32 [128 input dim][128 channel] right singular vectors or NULL
+ *   ahat_out : host fp32 [d_model][128] = A sqrt(S) = W P or NULL (the hidden-state encode
+ *              matrix: per-column positive rescaling leaves allocation and codes unchanged)
+ * Errors: AATC_ERR_INVALID_ARG (null x or w, n < 1, d_model < 1, non-finite input, or a zero
+ * singular value: W~ must have full column rank).  Host only.
+ */
+aatc_status_t aatc_whitening_transform(int32_t d_model, int32_t n, const float* x, const float* w,
+                                       float* a_out, float* b_out, double* s_out, float* p_out,
+                                       float* ahat_out);
+
+/*
+ * Encode operand for caching the coefficients straight from the hidden state (Sec. 5 Step 1:
+ * H = X A is cached instead of K = X W).  With the plan's orthonormal basis U_s (= P of
+ * aatc_whitening_transform for that head, in storage order) the coefficients of k = x W_s are
+ * x (W_s U_s); this writes (W_s U_s)^T rounded to bf16 (round to nearest even), the K-major B
+ * operand of aatc_encode_hidden.
+ *   w_k, w_v : host fp32 [L][d_model][n_kv_heads * 128] key / value projections (head h owns
+ *              columns 128 h .. 128 h + 127)
+ *   basis    : host fp32 [L][n_kv][2][128][128] as aatc_calibrate writes it
+ *   out      : host bf16 bits [L][n_kv][2][128 channel][d_model]
+ * Errors: AATC_ERR_INVALID_ARG (invalid dims, d_model not a positive multiple of 64, null,
+ * non-finite result).  Host only.
+ */
+aatc_status_t aatc_hidden_operand(const aatc_dims_t* dims, int32_t d_model, const float* w_k,
+                                  const float* w_v, const float* basis, uint16_t* out);
+
+/*
  * Build an immutable device plan from basis / bits / scales in the layouts aatc_calibrate
  * writes (Algorithm 1 outputs).  Derives per stream: R = #{b_c >= 1}, bit offsets, the
  * record length W = ceil(max_s sum_c b_c / 32) words (plan-wide), f_c = s_c 2^(1-b_c), the
@@ -163,6 +201,22 @@ aatc_status_t aatc_cache_bytes(aatc_plan_t plan, int32_t batch, int32_t max_toke
 aatc_status_t aatc_encode(aatc_plan_t plan, int32_t layer, const void* K, const void* V,
                           int32_t batch, int32_t start, int32_t n_tokens, void* cache,
                           int32_t max_tokens, void* stream);
+
+/*
+ * Encode straight from the hidden state (Sec. 5 Step 1: the cache holds H = X A; Algorithm 1
+ * "Project" + "Append qtz(h)").  For every kv-head of the layer, key and value coefficients
+ * h = x A_hat_s (A_hat_s = W_s U_s from aatc_hidden_operand, so h = k U_s for k = x W_s) are
+ * computed on the tensor cores (bf16 x bf16, fp32 accumulate over d_model) and quantized and
+ * packed exactly as aatc_encode does, into positions [start, start + n_tokens) of `cache`.
+ *   x       : device bf16 [batch][n_tokens][d_model], 16-byte aligned
+ *   d_model : multiple of 64, 64 .. 65536
+ *   a_hat   : device bf16 [L][n_kv][2][128][d_model] (aatc_hidden_operand's layout), 16-byte aligned
+ * Asynchronous on `stream`.  Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer,
+ * sizes or d_model), AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_CUDA.
+ */
+aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x, int32_t d_model, const void* a_hat,
+                                 int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
+                                 void* stream);
 
 /* Device workspace bytes aatc_decode_attention needs for (batch, n_ctx). */
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t plan, int32_t batch, int32_t n_ctx,

@@ -67,6 +67,38 @@ def eigenbasis(c: np.ndarray):
     return lam[order], canonical_sign(vec[:, order])
 
 
+def whitening_transform(x_calib: np.ndarray, w: np.ndarray):
+    """Whitening-based feature decorrelation from the model weights (Sec. 5 Step 1, Eq.
+    AB-factorization), in the paper's order:
+      Sigma_X = X^T X / T;  Sigma_X = L L^T (Cholesky);  W~ = L^T W;  W~ = U S P^T (reduced SVD);
+      A = L^-T U sqrt(S);  B = sqrt(S) P^T,  so that W = A B and H = X A is cached.
+    x_calib: (T, d_model) calibration activations; w: (d_model, d) one head's projection.
+    Singular vectors are sign-canonical in P (largest |entry| positive), U flipped alike, so A B
+    is unchanged.  Returns dict(A (d_model, d), B (d, d), S (d,), P (d, d), U, L)."""
+    x = np.asarray(x_calib, dtype=np.float64)
+    w = np.asarray(w, dtype=np.float64)
+    sigma_x = x.T @ x / x.shape[0]
+    l_chol = np.linalg.cholesky(sigma_x)
+    w_tilde = l_chol.T @ w
+    u, s, pt = np.linalg.svd(w_tilde, full_matrices=False)
+    p_mat = pt.T
+    cols = np.arange(p_mat.shape[1])
+    flip = np.where(p_mat[np.argmax(np.abs(p_mat), axis=0), cols] < 0, -1.0, 1.0)   # as canonical_sign
+    p_mat = p_mat * flip[None, :]
+    u = u * flip[None, :]
+    a = np.linalg.solve(l_chol.T, u) * np.sqrt(s)[None, :]
+    b = np.sqrt(s)[:, None] * p_mat.T
+    return {"A": a, "B": b, "S": s, "P": p_mat, "U": u, "L": l_chol}
+
+
+def hidden_encode_operand(a: np.ndarray, s: np.ndarray) -> np.ndarray:
+    """A sqrt(S) = W P: the encode matrix of the cached coefficients with each column rescaled
+    by sqrt(S_c).  Per-column positive scaling leaves the allocation and the codes unchanged
+    (Eq. AB-factorization with the quantizer of Sec. 5: s_c and h_c scale alike), so caching
+    x A sqrt(S) instead of x A gives the same codes as the PCA coefficients of k = x W."""
+    return np.asarray(a, dtype=np.float64) * np.sqrt(np.asarray(s, dtype=np.float64))[None, :]
+
+
 def channel_variance(encode_basis: np.ndarray, x: np.ndarray) -> np.ndarray:
     """sigma_c^2 = mean over calibration of h_c^2 with h = x A (Alg. 1 calibration, 'record latent
     variance'; uncentered because the source is zero-mean, Sec. 3.1)."""

@@ -47,6 +47,9 @@ SIGNATURES = {
     "aatc_version": (_I32, []),
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
     "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
+    "aatc_whitening_transform": (_I32, [_I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
+    "aatc_hidden_operand": (_I32, [ctypes.POINTER(Dims), _I32, _P, _P, _P, _P]),
+    "aatc_encode_hidden": (_I32, [_P, _I32, _P, _I32, _P, _I32, _I32, _I32, _P, _I32, _P]),
     "aatc_decode_attention_sw": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _SZ,
                                         _P]),
     "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
@@ -152,6 +155,41 @@ def allocate_global(dm: Dims, sigma2: np.ndarray, weights: np.ndarray, avg_bits_
     return bits
 
 
+def whitening_transform(x: np.ndarray, w: np.ndarray) -> dict:
+    """aatc_whitening_transform (Sec. 5 Step 1): x fp32 [n][d_model] calibration activations,
+    w fp32 [d_model][128] one head's projection.  Returns dict(A, B, S, P, A_hat) with
+    W = A B, A_hat = A sqrt(S) = W P."""
+    xx = np.ascontiguousarray(x, dtype=np.float32)
+    ww = np.ascontiguousarray(w, dtype=np.float32)
+    n, dm = xx.shape
+    if ww.shape != (dm, HEAD_DIM):
+        raise ValueError("w must be [d_model][128]")
+    a = np.empty((dm, HEAD_DIM), np.float32)
+    b = np.empty((HEAD_DIM, HEAD_DIM), np.float32)
+    sv = np.empty(HEAD_DIM, np.float64)
+    pm = np.empty((HEAD_DIM, HEAD_DIM), np.float32)
+    ah = np.empty((dm, HEAD_DIM), np.float32)
+    _check(load().aatc_whitening_transform(dm, n, _ptr(xx), _ptr(ww), _ptr(a), _ptr(b), _ptr(sv), _ptr(pm),
+                                           _ptr(ah)), "aatc_whitening_transform")
+    return {"A": a, "B": b, "S": sv, "P": pm, "A_hat": ah}
+
+
+def hidden_operand(dm: Dims, w_k: np.ndarray, w_v: np.ndarray, basis: np.ndarray) -> np.ndarray:
+    """aatc_hidden_operand: w_k, w_v fp32 [L][d_model][H_kv*128], basis as calibrate returns it.
+    Returns uint16 bf16 bits [L][H_kv][2][128][d_model] (copy it to the device as bfloat16)."""
+    wk = np.ascontiguousarray(w_k, dtype=np.float32)
+    wv = np.ascontiguousarray(w_v, dtype=np.float32)
+    bs = np.ascontiguousarray(basis, dtype=np.float32)
+    L, H = dm.n_layers, dm.n_kv_heads
+    if wk.ndim != 3 or wk.shape[0] != L or wk.shape[2] != H * HEAD_DIM or wv.shape != wk.shape:
+        raise ValueError("w_k / w_v must be [L][d_model][H_kv*128]")
+    d_model = wk.shape[1]
+    out = np.empty((L, H, 2, HEAD_DIM, d_model), np.uint16)
+    _check(load().aatc_hidden_operand(ctypes.byref(dm), d_model, _ptr(wk), _ptr(wv), _ptr(bs), _ptr(out)),
+           "aatc_hidden_operand")
+    return out
+
+
 class Plan:
     """Device plan (aatc_plan_t).  Create from the planner outputs; destroyed on close()."""
 
@@ -214,6 +252,15 @@ def encode(plan: Plan, layer: int, K, V, cache, start: int, max_tokens: int, str
     batch, n_tokens = K.shape[0], K.shape[1]
     _check(load().aatc_encode(plan.handle, layer, _ptr(K), _ptr(V), batch, start, n_tokens, _ptr(cache),
                               max_tokens, _stream(stream)), "aatc_encode")
+
+
+def encode_hidden(plan: Plan, layer: int, x, a_hat, cache, start: int, max_tokens: int, stream=None):
+    """aatc_encode_hidden: x bf16 [batch][n_tokens][d_model] hidden states (device), a_hat bf16
+    [L][H_kv][2][128][d_model] from hidden_operand (device); writes positions [start, start +
+    n_tokens) of the packed cache with the codes of x W U (keys and values of every kv-head)."""
+    batch, n_tokens, d_model = x.shape
+    _check(load().aatc_encode_hidden(plan.handle, layer, _ptr(x), d_model, _ptr(a_hat), batch, start, n_tokens,
+                                     _ptr(cache), max_tokens, _stream(stream)), "aatc_encode_hidden")
 
 
 def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: int, out=None, workspace=None,

@@ -130,6 +130,9 @@ aatc_status_t status_from_cuda(cudaError_t e);
 cudaError_t encode_tensor_maps_u(Plan& plan);
 cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch,
                           int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st);
+// x: bf16 [batch][n_tokens][d_model] hidden states; a_hat: bf16 [L][H][2][128][d_model].
+cudaError_t launch_encode_hidden(const Plan& plan, int layer, const void* x, int d_model, const void* a_hat,
+                                 int batch, int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st);
 // Optional parts of a decode call: the packed range starts at token t_first (default 0), and
 // n_full uncompressed tokens (bf16 [batch][full_cap][n_kv][128], e.g. a full-precision sink and
 // recent window) join the same softmax.

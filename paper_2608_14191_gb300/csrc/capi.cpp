@@ -323,6 +323,20 @@ aatc_status_t aatc_encode(aatc_plan_t p, int32_t layer, const void* K, const voi
                                          max_tokens, static_cast<cudaStream_t>(stream)));
 }
 
+aatc_status_t aatc_encode_hidden(aatc_plan_t p, int32_t layer, const void* x, int32_t d_model, const void* a_hat,
+                                 int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
+                                 void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !x || !a_hat || !cache || layer < 0 || layer >= plan->dims.n_layers || batch < 1 || start < 0 ||
+      n_tokens < 0 || max_tokens < 1 || d_model < 64 || d_model % 64 != 0 || d_model > 65536)
+    return AATC_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(start) + n_tokens > max_tokens) return AATC_ERR_CAPACITY;
+  if (!aligned16(x) || !aligned16(a_hat) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
+  if (n_tokens == 0) return AATC_OK;
+  return cuda_status(aatc::launch_encode_hidden(*plan, layer, x, d_model, a_hat, batch, start, n_tokens, cache,
+                                                max_tokens, static_cast<cudaStream_t>(stream)));
+}
+
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;

@@ -55,7 +55,8 @@ struct EncodeSmem {
   int abort_flag;
 };
 
-__device__ __forceinline__ void raise_abort(EncodeSmem& sm, int* err) {
+template <typename Smem>
+__device__ __forceinline__ void raise_abort(Smem& sm, int* err) {
   sm.abort_flag = 1;
   atomicOr(err, 2);
 }
@@ -90,6 +91,92 @@ __device__ __forceinline__ void append_bits(uint32_t v, int nb, uint32_t& word, 
     word = pos + nb > 32 ? (v >> (32 - pos)) : 0u;
   }
   pos = (pos + nb) & 31;
+}
+
+// Token scale and stored values of one token (thread = token = TMEM lane): alpha = max over
+// retained channels of |h_c| / s_c (inv_s = 0 for dropped ones), then u_c = clamp(floor(h_c /
+// Delta_c + 1/2)) + 2^(b_c - 1) with Delta_c = alpha f_c, one byte per channel into `row`.  The
+// 128 coefficients are read from TMEM columns taddr .. taddr + 127 (twice: amax, then quantize).
+__device__ __forceinline__ float quantize_token(uint32_t taddr, const ChanEnc* enc, const float* inv_s,
+                                                uint32_t* row) {
+  float amax = 0.0f;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float h[32];
+    ptx::tmem_ld_32cols(taddr + 32 * j, h);
+    ptx::tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 32; i += 4) {
+      const float4 is = *reinterpret_cast<const float4*>(&inv_s[32 * j + i]);
+      amax = fmaxf(amax, fabsf(h[i]) * is.x);
+      amax = fmaxf(amax, fabsf(h[i + 1]) * is.y);
+      amax = fmaxf(amax, fabsf(h[i + 2]) * is.z);
+      amax = fmaxf(amax, fabsf(h[i + 3]) * is.w);
+    }
+  }
+  const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+  // The round-down add of 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float h[32];
+    ptx::tmem_ld_32cols(taddr + 32 * j, h);
+    ptx::tmem_ld_wait();
+    uint32_t y[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const ChanEnc e = enc[32 * j + i];
+      float x = fmaf(h[i], e.inv_f * ia, 0.5f);                // h / Delta + 1/2
+      x = fminf(x, e.hi);                                       // |h| / Delta <= 2^(b-1): only the top clamps
+      y[i] = __float_as_uint(__fadd_rd(x, e.magic));            // floor, offset binary in the mantissa
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      row[8 * j + q] = __byte_perm(__byte_perm(y[4 * q], y[4 * q + 1], 0x0040),
+                                   __byte_perm(y[4 * q + 2], y[4 * q + 3], 0x0040), 0x5410);
+  }
+  return amax;
+}
+
+// Packed record of one token from its byte row: the bit stream of Sec. 5's stored values in the
+// D2 / D1 layout, four channels per step (field w bits at bit sh of channels [c0, c1), w = 2: a
+// base-4 digit, w = 1: a single bit; one multiply gathers four of them), appended LSB first.
+__device__ __forceinline__ void pack_token(const StreamLayout& lay, const uint32_t* row, const RecordWriter& out,
+                                           int n_words) {
+  uint32_t word = 0;
+  int pos = 0, wi = 0;
+  auto emit_run = [&](int c0, int c1, int sh, int w) {
+    for (int g4 = c0 >> 2; 4 * g4 < c1; ++g4) {
+      const int skip = max(c0 - 4 * g4, 0), n = min(c1 - 4 * g4, 4) - skip;
+      const uint32_t x = row[g4] >> sh;
+      uint32_t y = w == 2 ? (((x & 0x03030303u) * 0x00041041u) >> 18) & 0xFFu
+                          : (((x & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
+      y = (y >> (w * skip)) & ((1u << (w * n)) - 1u);
+      append_bits(y, w * n, word, pos, wi, out);
+    }
+  };
+#pragma unroll 1
+  for (int k = 0; k < 4; ++k) emit_run(0, lay.l2[k], 2 * k, 2);                 // D2 digits
+#pragma unroll 1
+  for (int k = 3; k >= 0; --k) emit_run(lay.l2all[k], lay.lodd[k], 2 * k, 1);  // D1: top bits of odd widths
+#pragma unroll 1
+  for (int k = 0; k < 4; ++k) emit_run(lay.l2[k], lay.l2all[k], 2 * k, 2);     // D1: digits moved out of D2
+  if (pos > 0) {
+    out.put(wi, word);
+    ++wi;
+  }
+  for (; wi < n_words; ++wi) out.put(wi, 0u);
+}
+
+// Writer for token position pos_t of cache stream sidx.
+__device__ __forceinline__ RecordWriter record_writer(uint32_t* words, size_t sidx, size_t stream_words,
+                                                      int n_words, int pos_t, bool value) {
+  uint32_t* tile_words = words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * n_words * TILE;
+  RecordWriter out;
+  out.value = value;
+  const int tt = pos_t % TILE;
+  out.key_word = tile_words + tt;
+  out.val_byte = reinterpret_cast<uint8_t*>(tile_words + 4 * (tt >> 2)) + (tt & 3);
+  return out;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -201,44 +288,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_after();
       const uint32_t taddr = tmem + eg * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
 
-      // alpha = max_c |h_c| / s_c over retained channels (inv_s = 0 for dropped ones)
-      float amax = 0.0f;
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float h[32];
-        ptx::tmem_ld_32cols(taddr + 32 * j, h);
-        ptx::tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 32; i += 4) {
-          const float4 is = *reinterpret_cast<const float4*>(&sm.inv_s[32 * j + i]);
-          amax = fmaxf(amax, fabsf(h[i]) * is.x);
-          amax = fmaxf(amax, fabsf(h[i + 1]) * is.y);
-          amax = fmaxf(amax, fabsf(h[i + 2]) * is.z);
-          amax = fmaxf(amax, fabsf(h[i + 3]) * is.w);
-        }
-      }
-      const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
-
-      // quantize: u = clamp(floor(h / Delta + 1/2)) + 2^(b-1), one byte per channel.  The
-      // round-down add of 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float h[32];
-        ptx::tmem_ld_32cols(taddr + 32 * j, h);
-        ptx::tmem_ld_wait();
-        uint32_t y[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const ChanEnc e = sm.enc[32 * j + i];
-          float x = fmaf(h[i], e.inv_f * ia, 0.5f);                // h / Delta + 1/2
-          x = fminf(x, e.hi);                                       // |h| / Delta <= 2^(b-1): only the top clamps
-          y[i] = __float_as_uint(__fadd_rd(x, e.magic));            // floor, offset binary in the mantissa
-        }
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          my_bytes[8 * j + q] = __byte_perm(__byte_perm(y[4 * q], y[4 * q + 1], 0x0040),
-                                            __byte_perm(y[4 * q + 2], y[4 * q + 3], 0x0040), 0x5410);
-      }
+      const float amax = quantize_token(taddr, sm.enc, sm.inv_s, my_bytes);
       ptx::tc_fence_before();
       ptx::mbar_arrive(&sm.tempty[eg]);
 
@@ -250,39 +300,166 @@ __global__ void __launch_bounds__(kThreads, 1)
       const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
       if (!isfinite(amax)) atomicOr(a.err, 1);
       a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
-      uint32_t* tile_words = a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE;
-      RecordWriter out;
-      out.value = kind == 1;
-      const int tt = pos_t % TILE;
-      out.key_word = tile_words + tt;
-      out.val_byte = reinterpret_cast<uint8_t*>(tile_words + 4 * (tt >> 2)) + (tt & 3);
+      pack_token(lay, my_bytes, record_writer(a.words, sidx, stream_words, a.n_words, pos_t, kind == 1), a.n_words);
+    }
+  }
 
-      // Record bit stream, four channels per step from this thread's byte row: field w bits at
-      // bit sh of channels [c0, c1) (w = 2: base-4 digit, w = 1: single bit), gathered by one
-      // multiply and appended LSB first.
-      uint32_t word = 0;
-      int pos = 0, wi = 0;
-      auto emit_run = [&](int c0, int c1, int sh, int w) {
-        for (int g4 = c0 >> 2; 4 * g4 < c1; ++g4) {
-          const int skip = max(c0 - 4 * g4, 0), n = min(c1 - 4 * g4, 4) - skip;
-          const uint32_t x = my_bytes[g4] >> sh;
-          uint32_t y = w == 2 ? (((x & 0x03030303u) * 0x00041041u) >> 18) & 0xFFu
-                              : (((x & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
-          y = (y >> (w * skip)) & ((1u << (w * n)) - 1u);
-          append_bits(y, w * n, word, pos, wi, out);
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ encode from hidden states
+// Sec. 5 Step 1 caches H = X A, the coefficients computed from the layer input x rather than
+// from k = x W.  With A_hat = W U (the plan basis, = A sqrt(S) up to channel order) the MMA
+// gives h = x A_hat = k U directly, K = d_model.  One persistent CTA per (kv-head, slice of
+// 128-token tiles); warp roles as aatc_encode_kernel:
+//   warp 16   : TMA producer -- per 64-wide d_model block: the 128 x 64 x tile and the 256 x 64
+//               A_hat tile of the head's key and value channels (two 128-row boxes, one operand),
+//   warp 17   : MMA issuer   -- tcgen05.mma M=128 tokens, N=256 (key | value channels), K=16,
+//               into one of two 256-column TMEM accumulators,
+//   warps 0-15: four epilogue groups (stream = group & 1, accumulator = group >> 1), thread =
+//               token: the quantize / pack epilogue of aatc_encode_kernel.
+// CTA i takes kv-head i mod H and tiles i / H, i / H + J, ... (J CTAs per head), so the H CTAs
+// working on one token tile at a time read its x block from L2 after the first.
+constexpr int kHStages = 3;
+constexpr int kHK = 64;                            // d_model elements per stage (one 128-byte row)
+constexpr int kHXBytes = TILE * kHK * 2;           // 16 KB
+constexpr int kHABytes = 2 * D * kHK * 2;          // 32 KB
+
+struct EncodeHiddenArgs {
+  const ChanEnc* enc;
+  const float* inv_s;
+  const StreamLayout* lay;
+  int* err;
+  uint32_t* words;
+  float* alpha;
+  int layer, n_kv, batch, start, n_tokens, n_chunks, n_words, n_tiles, d_model;
+};
+
+struct EncodeHiddenSmem {
+  alignas(1024) unsigned char x_tile[kHStages][kHXBytes];
+  alignas(1024) unsigned char a_tile[kHStages][kHABytes];
+  ChanEnc enc[2][D];
+  float inv_s[2][D];
+  StreamLayout lay[2];
+  uint32_t ubytes[kEpiThreads][kByteRow / 4];
+  uint64_t full[kHStages], empty[kHStages], tfull[2], tempty[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    aatc_encode_hidden_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_a,
+                              const EncodeHiddenArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  EncodeHiddenSmem& sm =
+      *reinterpret_cast<EncodeHiddenSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int head = blockIdx.x % a.n_kv, j = blockIdx.x / a.n_kv, J = gridDim.x / a.n_kv;
+  const long n_items = static_cast<long>(a.batch) * a.n_chunks;
+  const int my_items = n_items > j ? static_cast<int>((n_items - 1 - j) / J + 1) : 0;
+  const int nk = a.d_model / kHK;
+  const int sk = (a.layer * a.n_kv + head) * 2;                // key stream; values sk + 1
+
+  for (int i = tid; i < 2 * D; i += kThreads) {
+    sm.enc[i >> 7][i & (D - 1)] = a.enc[sk * D + i];
+    sm.inv_s[i >> 7][i & (D - 1)] = a.inv_s[sk * D + i];
+  }
+  if (tid == 0) {
+    sm.lay[0] = a.lay[sk];
+    sm.lay[1] = a.lay[sk + 1];
+    for (int s = 0; s < kHStages; ++s) {
+      ptx::mbar_init(&sm.full[s], 1);
+      ptx::mbar_init(&sm.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      ptx::mbar_init(&sm.tfull[b], 1);
+      ptx::mbar_init(&sm.tempty[b], 256);
+    }
+    sm.abort_flag = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (warp == kProducerWarp) {
+    if (lane == 0 && my_items > 0) {
+      ptx::prefetch_tmap(&tmap_x);
+      ptx::prefetch_tmap(&tmap_a);
+      bool ok = true;
+      for (int it = 0; ok && it < my_items; ++it) {
+        const long tile = j + static_cast<long>(it) * J;
+        const int b = static_cast<int>(tile / a.n_chunks);
+        const int t0 = static_cast<int>(tile % a.n_chunks) * TILE;
+        for (int ks = 0; ks < nk; ++ks) {
+          const int u = it * nk + ks, s = u % kHStages;
+          const uint32_t ph = (u / kHStages) & 1;
+          if (!ptx::mbar_wait_bounded(&sm.empty[s], ph ^ 1, abort_flag)) { raise_abort(sm, a.err); ok = false; break; }
+          ptx::mbar_arrive_expect_tx(&sm.full[s], kHXBytes + kHABytes);
+          ptx::tma_load_3d(sm.x_tile[s], &tmap_x, &sm.full[s], ks * kHK, t0, b);
+          ptx::tma_load_2d(sm.a_tile[s], &tmap_a, &sm.full[s], ks * kHK, sk * D);
+          ptx::tma_load_2d(sm.a_tile[s] + kHABytes / 2, &tmap_a, &sm.full[s], ks * kHK, (sk + 1) * D);
         }
-      };
-#pragma unroll 1
-      for (int k = 0; k < 4; ++k) emit_run(0, lay.l2[k], 2 * k, 2);                 // D2 digits
-#pragma unroll 1
-      for (int k = 3; k >= 0; --k) emit_run(lay.l2all[k], lay.lodd[k], 2 * k, 1);  // D1: top bits of odd widths
-#pragma unroll 1
-      for (int k = 0; k < 4; ++k) emit_run(lay.l2[k], lay.l2all[k], 2 * k, 2);     // D1: digits moved out of D2
-      if (pos > 0) {
-        out.put(wi, word);
-        ++wi;
       }
-      for (; wi < a.n_words; ++wi) out.put(wi, 0u);
+    }
+  } else if (warp == kMmaWarp) {
+    if (lane == 0 && my_items > 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 2 * D);
+      bool ok = true;
+      for (int it = 0; ok && it < my_items; ++it) {
+        const int bf = it & 1;
+        if (!ptx::mbar_wait_bounded(&sm.tempty[bf], ((it >> 1) & 1) ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
+        ptx::tc_fence_after();
+        for (int ks = 0; ks < nk; ++ks) {
+          const int u = it * nk + ks, s = u % kHStages;
+          const uint32_t ph = (u / kHStages) & 1;
+          if (!ptx::mbar_wait_bounded(&sm.full[s], ph, abort_flag)) { raise_abort(sm, a.err); ok = false; break; }
+          ptx::tc_fence_after();
+          const uint32_t x_base = ptx::smem_u32(sm.x_tile[s]), a_base = ptx::smem_u32(sm.a_tile[s]);
+#pragma unroll
+          for (int kk = 0; kk < kHK / 16; ++kk)
+            ptx::umma_bf16(tmem + 2 * D * bf, ptx::sdesc_kmajor_sw128(x_base + kk * 32),
+                           ptx::sdesc_kmajor_sw128(a_base + kk * 32), idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+          ptx::umma_commit(&sm.empty[s]);
+        }
+        if (ok) ptx::umma_commit(&sm.tfull[bf]);
+      }
+    }
+  } else {
+    const int eg = warp >> 2, sidx = eg & 1, bf = eg >> 1;
+    const int quad = warp & 3;
+    const int tl = quad * 32 + lane;
+    const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
+    const StreamLayout lay = sm.lay[sidx];
+    uint32_t* my_bytes = sm.ubytes[tid];
+    for (int it = bf; it < my_items; it += 2) {
+      if (!ptx::mbar_wait_bounded(&sm.tfull[bf], (it >> 1) & 1, abort_flag)) { raise_abort(sm, a.err); break; }
+      ptx::tc_fence_after();
+      const uint32_t taddr = tmem + 2 * D * bf + D * sidx + (static_cast<uint32_t>(quad * 32) << 16);
+      const float amax = quantize_token(taddr, sm.enc[sidx], sm.inv_s[sidx], my_bytes);
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&sm.tempty[bf]);
+
+      const long tile = j + static_cast<long>(it) * J;
+      const int b = static_cast<int>(tile / a.n_chunks);
+      const int i = static_cast<int>(tile % a.n_chunks) * TILE + tl;     // input token index
+      if (i >= a.n_tokens) continue;
+      const int pos_t = a.start + i;
+      const size_t cs = (static_cast<size_t>(b) * a.n_kv + head) * 2 + sidx;
+      if (!isfinite(amax)) atomicOr(a.err, 1);
+      a.alpha[cs * a.n_tiles * TILE + pos_t] = amax;
+      pack_token(lay, my_bytes, record_writer(a.words, cs, stream_words, a.n_words, pos_t, sidx == 1), a.n_words);
     }
   }
 
@@ -379,6 +556,68 @@ cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void
   }
   const auto* mu = reinterpret_cast<const CUtensorMap*>(plan.tmap_u);
   aatc_encode_kernel<<<n_basis * k, kThreads, smem, st>>>(mk, mv, *mu, a);
+  return cudaGetLastError();
+}
+
+
+cudaError_t launch_encode_hidden(const Plan& plan, int layer, const void* x, int d_model, const void* a_hat,
+                                 int batch, int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  CUtensorMap mx, ma;
+  {
+    // x: bf16 [batch][n_tokens][d_model]; box 64 x 128 tokens x 1 (rows past n_tokens read 0)
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(d_model), static_cast<cuuint64_t>(n_tokens),
+                                static_cast<cuuint64_t>(batch)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(d_model) * 2,
+                                   static_cast<cuuint64_t>(n_tokens) * d_model * 2};
+    const cuuint32_t box[3] = {kHK, TILE, 1};
+    const cuuint32_t es[3] = {1, 1, 1};
+    if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(x), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  {
+    // A_hat: bf16 [L * H * 2 * 128 rows][d_model]; box 64 x 128 rows
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(d_model), static_cast<cuuint64_t>(plan.n_streams) * D};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(d_model) * 2};
+    const cuuint32_t box[2] = {kHK, TILE};
+    const cuuint32_t es[2] = {1, 1};
+    if (enc(&ma, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a_hat), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
+  EncodeHiddenArgs a;
+  a.enc = plan.dev.enc;
+  a.inv_s = plan.dev.inv_s;
+  a.lay = plan.dev.lay;
+  a.err = plan.dev.err;
+  a.words = static_cast<uint32_t*>(cache);
+  a.alpha = reinterpret_cast<float*>(static_cast<uint32_t*>(cache) + g.words_elems);
+  a.layer = layer;
+  a.n_kv = plan.dims.n_kv_heads;
+  a.batch = batch;
+  a.start = start;
+  a.n_tokens = n_tokens;
+  a.n_chunks = (n_tokens + TILE - 1) / TILE;
+  a.n_words = plan.n_words;
+  a.n_tiles = g.n_tiles;
+  a.d_model = d_model;
+  const long n_items = static_cast<long>(batch) * a.n_chunks;
+  long per_head = std::max(1, plan.num_sms / a.n_kv);
+  per_head = std::min(per_head, n_items);
+  const size_t smem = sizeof(EncodeHiddenSmem) + 1024;
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(aatc_encode_hidden_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  aatc_encode_hidden_kernel<<<static_cast<unsigned>(per_head * a.n_kv), kThreads, smem, st>>>(mx, ma, a);
   return cudaGetLastError();
 }
 

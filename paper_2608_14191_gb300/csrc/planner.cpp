@@ -343,3 +343,119 @@ extern "C" aatc_status_t aatc_allocate_global(const aatc_dims_t* dims, const dou
   }
   return AATC_OK;
 }
+
+// ------------------------------------------------------------------ transform from model weights
+
+namespace aatc {
+namespace {
+
+// Round an fp32 value to bf16 bits, round to nearest even (finite inputs).
+uint16_t bf16_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  const uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7FFFu + lsb;
+  return static_cast<uint16_t>(u >> 16);
+}
+
+}  // namespace
+}  // namespace aatc
+
+extern "C" aatc_status_t aatc_whitening_transform(int32_t d_model, int32_t n, const float* x, const float* w,
+                                                  float* a_out, float* b_out, double* s_out, float* p_out,
+                                                  float* ahat_out) {
+  using namespace aatc;
+  if (d_model < 1 || n < 1 || !x || !w) return AATC_ERR_INVALID_ARG;
+  const size_t dm = static_cast<size_t>(d_model);
+  for (size_t i = 0; i < dm * kD; ++i)
+    if (!std::isfinite(w[i])) return AATC_ERR_INVALID_ARG;
+  // C = K^T K / n with K = X W (= W^T Sigma_X W = W~^T W~ for W~ = L^T W, any L L^T = Sigma_X)
+  std::vector<double> c(kD * kD, 0.0), k(kD), wd(dm * kD);
+  for (size_t i = 0; i < dm * kD; ++i) wd[i] = w[i];
+  for (int t = 0; t < n; ++t) {
+    const float* xt = x + static_cast<size_t>(t) * dm;
+    std::fill(k.begin(), k.end(), 0.0);
+    for (size_t i = 0; i < dm; ++i) {
+      const double xi = xt[i];
+      if (!std::isfinite(xi)) return AATC_ERR_INVALID_ARG;
+      if (xi == 0.0) continue;
+      const double* wi = wd.data() + i * kD;
+      for (int j = 0; j < kD; ++j) k[j] += xi * wi[j];
+    }
+    for (int i = 0; i < kD; ++i) {
+      double* ci = c.data() + i * kD;
+      const double ki = k[i];
+      for (int j = i; j < kD; ++j) ci[j] += ki * k[j];
+    }
+  }
+  for (int i = 0; i < kD; ++i)
+    for (int j = i; j < kD; ++j) {
+      c[i * kD + j] /= n;
+      c[j * kD + i] = c[i * kD + j];
+    }
+  // C = P diag(S^2) P^T: eigenvalues descending (stable), sign-canonical columns
+  std::vector<double> v;
+  jacobi_eigen(c, v);
+  std::vector<int> ord(kD);
+  std::iota(ord.begin(), ord.end(), 0);
+  std::stable_sort(ord.begin(), ord.end(), [&](int i, int j) { return c[i * kD + i] > c[j * kD + j]; });
+  std::vector<double> s(kD), p(kD * kD);                      // p[d][k]
+  for (int kk = 0; kk < kD; ++kk) {
+    const int src = ord[kk];
+    const double lam = c[src * kD + src];
+    if (!(lam > 0.0)) return AATC_ERR_INVALID_ARG;             // W~ must have full column rank
+    s[kk] = std::sqrt(lam);
+    int imax = 0;
+    double amax = -1.0;
+    for (int d = 0; d < kD; ++d) {
+      const double a = std::fabs(v[d * kD + src]);
+      if (a > amax) { amax = a; imax = d; }
+    }
+    const double sgn = v[imax * kD + src] < 0 ? -1.0 : 1.0;
+    for (int d = 0; d < kD; ++d) p[d * kD + kk] = sgn * v[d * kD + src];
+  }
+  // A_hat = W P;  A = A_hat S^-1/2;  B = S^1/2 P^T
+  for (size_t i = 0; i < dm; ++i) {
+    const double* wi = wd.data() + i * kD;
+    for (int kk = 0; kk < kD; ++kk) {
+      double acc = 0.0;
+      for (int d = 0; d < kD; ++d) acc += wi[d] * p[d * kD + kk];
+      if (ahat_out) ahat_out[i * kD + kk] = static_cast<float>(acc);
+      if (a_out) a_out[i * kD + kk] = static_cast<float>(acc / std::sqrt(s[kk]));
+    }
+  }
+  for (int kk = 0; kk < kD; ++kk) {
+    if (s_out) s_out[kk] = s[kk];
+    for (int d = 0; d < kD; ++d) {
+      if (b_out) b_out[kk * kD + d] = static_cast<float>(std::sqrt(s[kk]) * p[d * kD + kk]);
+      if (p_out) p_out[d * kD + kk] = static_cast<float>(p[d * kD + kk]);
+    }
+  }
+  return AATC_OK;
+}
+
+extern "C" aatc_status_t aatc_hidden_operand(const aatc_dims_t* dims, int32_t d_model, const float* w_k,
+                                             const float* w_v, const float* basis, uint16_t* out) {
+  using namespace aatc;
+  if (!valid_dims(dims) || d_model < 64 || d_model % 64 != 0 || !w_k || !w_v || !basis || !out)
+    return AATC_ERR_INVALID_ARG;
+  const int L = dims->n_layers, H = dims->n_kv_heads;
+  const size_t dm = static_cast<size_t>(d_model), ld = static_cast<size_t>(H) * kD;
+  for (int l = 0; l < L; ++l)
+    for (int h = 0; h < H; ++h)
+      for (int kind = 0; kind < 2; ++kind) {
+        const float* wl = (kind == 0 ? w_k : w_v) + static_cast<size_t>(l) * dm * ld + static_cast<size_t>(h) * kD;
+        const float* u = basis + ((static_cast<size_t>(l) * H + h) * 2 + kind) * kD * kD;   // [dim][channel]
+        uint16_t* o = out + ((static_cast<size_t>(l) * H + h) * 2 + kind) * kD * dm;        // [channel][d_model]
+        for (size_t i = 0; i < dm; ++i) {
+          const float* wi = wl + i * ld;
+          for (int c2 = 0; c2 < kD; ++c2) {
+            double acc = 0.0;
+            for (int d = 0; d < kD; ++d) acc += static_cast<double>(wi[d]) * u[d * kD + c2];
+            if (!std::isfinite(acc)) return AATC_ERR_INVALID_ARG;
+            o[static_cast<size_t>(c2) * dm + i] = bf16_bits(static_cast<float>(acc));
+          }
+        }
+      }
+  return AATC_OK;
+}

@@ -7,6 +7,8 @@ exactly one level and must be fewer than 1e-5 of all codes; dequantized coeffici
 bit-exact; attention outputs within max-abs 1e-2 and relative L2 1e-3 of the oracle's fp64
 attention over the GPU's own packed cache.
 """
+from __future__ import annotations
+
 import numpy as np
 import torch
 
@@ -58,10 +60,13 @@ def read_stream(case: Case, cache_host_u32: np.ndarray, batch: int, max_tokens: 
     return rec, alpha
 
 
-def check_codes(case: Case, layer: int, head: int, kind: int, x: np.ndarray, rec: np.ndarray, alpha_gpu: np.ndarray):
-    """x: (n,128) bf16-exact inputs of one stream; rec/alpha_gpu: the GPU's records. Returns stats."""
+def check_codes(case: Case, layer: int, head: int, kind: int, x: np.ndarray, rec: np.ndarray, alpha_gpu: np.ndarray,
+                encode_matrix: np.ndarray | None = None):
+    """x: (n, d_in) bf16-exact inputs of one stream; rec/alpha_gpu: the GPU's records.  The
+    coefficients are h = x E with E = the plan's bf16 basis (d_in = 128), or `encode_matrix`
+    (d_in x 128, e.g. the bf16 hidden-state operand).  Returns stats."""
     _, bits, scales = case.stream(layer, head, kind)
-    ub = case.basis_bf16[layer, head, kind].astype(np.float64)
+    ub = (case.basis_bf16[layer, head, kind] if encode_matrix is None else encode_matrix).astype(np.float64)
     codes, alpha, t = O.encode_stream(x.astype(np.float64), ub, bits.astype(np.int64), scales.astype(np.float64))
     got = O.unpack_records(rec, bits.astype(np.int64))
     keep = bits > 0

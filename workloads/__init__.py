@@ -30,7 +30,8 @@ N_CALIB = 4096           # calibration vectors per stream and queries per q-head
 N_OUTLIERS = 4
 OUTLIER_GAIN = 8.0
 KIND_K, KIND_V = 0, 1
-_PURPOSE = {"basis": 0, "calib": 1, "data": 2, "query": 3, "calib_query": 4, "query_model": 5}
+_PURPOSE = {"basis": 0, "calib": 1, "data": 2, "query": 3, "calib_query": 4, "query_model": 5,
+            "hidden_model": 6, "hidden_calib": 7, "hidden_data": 8, "weight": 9}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -213,3 +214,59 @@ def queries_device(cfg: Config, layer: int, batch: int, steps: int, device, peak
 def queries_host(cfg: Config, layer: int, batch: int, steps: int, peaky: float = 1.0) -> np.ndarray:
     rng = _rng(cfg.seed, layer, 0, 0, "query")
     return to_bf16(rng.standard_normal((steps, batch, cfg.n_q_heads, D)) * peaky)
+
+
+# ----------------------------------------------------------------------------
+# Hidden states and projection weights (the transform from model weights, Sec. 5 Step 1)
+# ----------------------------------------------------------------------------
+# Stand-in for a layer's input activations X (T x d_model) and its key / value projection
+# W (d_model x n_kv*128), which the paper takes from the model checkpoints:
+#   * x = (z * sqrt(lam)) @ M / sqrt(d_model) with z ~ N(0, I), lam_i = i**-1.0 over d_model
+#     coordinates, M a Gaussian d_model x d_model matrix (anisotropic, correlated activations),
+#     plus 4 outlier coordinates x 20 (the heavy channels of transformer hidden states);
+#   * W ~ N(0, 1/d_model), one matrix per (layer, kind), columns head-major (head h owns
+#     columns 128h .. 128h + 127).
+N_HIDDEN_OUTLIERS = 4
+HIDDEN_OUTLIER_GAIN = 20.0
+
+
+def hidden_model(seed: int, layer: int, d_model: int):
+    """(mix (d_model x d_model), outlier indices) of the hidden-state model of one layer."""
+    rng = _rng(seed, layer, 0, 0, "hidden_model")
+    lam = np.arange(1, d_model + 1, dtype=np.float64) ** -1.0
+    mix = (np.sqrt(lam)[:, None] * rng.standard_normal((d_model, d_model))) / np.sqrt(d_model)
+    idx = np.sort(rng.choice(d_model, N_HIDDEN_OUTLIERS, replace=False))
+    return mix, idx
+
+
+def hidden_states(seed: int, layer: int, d_model: int, n: int, purpose: str = "hidden_calib") -> np.ndarray:
+    """(n, d_model) float32 bf16-exact hidden states of one layer (host)."""
+    mix, idx = hidden_model(seed, layer, d_model)
+    z = _rng(seed, layer, 0, 0, purpose).standard_normal((n, d_model)).astype(np.float32)
+    x = z @ mix.astype(np.float32)
+    x[:, idx] *= HIDDEN_OUTLIER_GAIN
+    return to_bf16(x)
+
+
+def hidden_states_device(seed: int, layer: int, d_model: int, batch: int, n_tokens: int, device):
+    """bf16 [batch][n_tokens][d_model] hidden states drawn on the device (same model, torch
+    generator seeded from the (layer, "hidden_data") key)."""
+    import torch
+    mix, idx = hidden_model(seed, layer, d_model)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(torch_seed(seed, layer, 0, 0, "hidden_data"))
+    m = torch.from_numpy(mix.astype(np.float32)).to(device)
+    x = torch.empty((batch * n_tokens, d_model), dtype=torch.bfloat16, device=device)
+    for r0 in range(0, batch * n_tokens, 8192):
+        r1 = min(batch * n_tokens, r0 + 8192)
+        z = torch.randn((r1 - r0, d_model), generator=gen, device=device, dtype=torch.float32)
+        y = z @ m
+        y[:, torch.from_numpy(idx).to(device)] *= HIDDEN_OUTLIER_GAIN
+        x[r0:r1] = y.to(torch.bfloat16)
+    return x.view(batch, n_tokens, d_model)
+
+
+def projection_weight(seed: int, layer: int, kind: int, d_model: int, n_kv: int) -> np.ndarray:
+    """(d_model, n_kv * 128) float32 bf16-exact key (kind 0) or value (kind 1) projection."""
+    rng = _rng(seed, layer, 0, kind, "weight")
+    return to_bf16(rng.standard_normal((d_model, n_kv * D)) / np.sqrt(d_model))
