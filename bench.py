@@ -38,6 +38,7 @@ METRIC = "compressed-KV decode attn GB/s & % of HBM peak; encode Mtok/s (1 GB300
 N_COPIES = 16
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
 DECODE_SRC = os.path.join(ROOT, "paper_2608_14191_gb300", "csrc", "decode.cu")
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 
 
 def _peaks():
@@ -177,6 +178,50 @@ def sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_d
             "policy": "sink 4 + recent window 128 (step 16) in bf16, the rest coded"}
 
 
+def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32768, iters=10):
+    """Encode straight from the layer input (Sec. 5 Step 1: the cache holds the coefficients of
+    x A): Llama-3.1-8B-shaped layer input, d_model 4096, 8 kv-heads x K|V, 32768 tokens.  The
+    plan is calibrated on K = X W of 4096 seeded hidden states and seeded projections; the
+    kernel is a tensor-core GEMM (2 x 32768 x 4096 x 2048 flop) with the quantize / pack
+    epilogue.  x is 268 MB (> L2), so back-to-back calls re-read it from HBM."""
+    import torch
+    seed = 1002
+    x_cal = W.hidden_states(seed, 0, d_model, 4096)
+    w_k = W.projection_weight(seed, 0, 0, d_model, n_kv)
+    w_v = W.projection_weight(seed, 0, 1, d_model, n_kv)
+    ck = (x_cal @ w_k).reshape(4096, n_kv, 128).transpose(1, 0, 2)[None]
+    cv = (x_cal @ w_v).reshape(4096, n_kv, 128).transpose(1, 0, 2)[None]
+    cfg = W.CONFIGS["llama_layer"]
+    cq = np.stack([W.calibration_queries(cfg, 0, j) for j in range(n_q)])[None]
+    dm = aatc.dims(1, n_kv, n_q)
+    p = aatc.calibrate(dm, np.ascontiguousarray(ck), np.ascontiguousarray(cv), cq, 2.75)
+    plan = aatc.Plan(dm, p["basis"], p["bits"], p["scales"])
+    ah = aatc.hidden_operand(dm, w_k[None], w_v[None], p["basis"])
+    a_hat = torch.from_numpy(ah.view(np.int16)).view(torch.bfloat16).to(device).contiguous()
+    x = W.hidden_states_device(seed, 0, d_model, 1, n_tokens, device)
+    cache = plan.new_cache(1, n_tokens, device)
+    for _ in range(3):
+        aatc.encode_hidden(plan, 0, x, a_hat, cache, 0, n_tokens)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        aatc.encode_hidden(plan, 0, x, a_hat, cache, 0, n_tokens)
+    e1.record()
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    us = e0.elapsed_time(e1) * 1e3 / iters
+    flop = 2.0 * n_tokens * d_model * n_kv * 2 * 128
+    peaks = json.load(open(PEAKS_FILE)) if os.path.exists(PEAKS_FILE) else {}
+    bf16 = float(peaks.get("bf16_tflops", 1900.0))
+    tf = flop / (us * 1e-6) / 1e12
+    plan.close()
+    return {"us_per_call": round(us, 2), "mtok_s": round(n_tokens / us, 2), "tflops": round(tf, 1),
+            "frac_of_measured_bf16": round(tf / bf16, 4),
+            "workload": f"Llama-3.1-8B-shaped layer input: d_model {d_model}, {n_kv} kv-heads x K|V, "
+                        f"{n_tokens} tokens, 2.75 bits"}
+
+
 def planner_timing(aatc):
     """Host planner rows: the global cross-layer allocation on Llama-3.1-8B-shaped statistics
     (32 layers x 8 kv-heads x K|V x 128 channels; seeded log-normal spectra), median of 5 runs."""
@@ -311,6 +356,7 @@ def run_ours(args):
     assert plan.device_error() == 0
 
     sw = sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_dec)
+    hid = hidden_encode_timing(aatc, dev)
 
     # max over ranks
     vals = torch.tensor([total_ms, float(np.mean(dec_ms)), float(np.mean(enc_ms)), e2e_ms], device=dev)
@@ -367,6 +413,7 @@ def run_ours(args):
         "clocks": clocks,
         "planner": planner_timing(aatc),
         "sink_window": sw,
+        "encode_hidden": hid,
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds)

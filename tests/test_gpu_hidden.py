@@ -98,3 +98,28 @@ def test_encode_hidden_argument_errors(aatc):
         aatc.encode_hidden(case.plan, 0, x, case.a_hat, cache, 60, 64)                        # capacity
     with pytest.raises(aatc.AatcError):
         aatc.encode_hidden(case.plan, 1, x, case.a_hat, cache, 0, 64)                         # layer
+
+
+def test_encode_hidden_llama_shape_sampled(aatc):
+    """Bench configuration: Llama-3.1-8B-shaped layer input (d_model 4096, 8 kv-heads), 32768
+    tokens in the launch the bench times; codes and scales compared on sampled heads and tokens."""
+    d_model, n_kv, n_tok = 4096, 8, 32768
+    case = HiddenCase(aatc, d_model, n_kv=n_kv, n_q=32)
+    x = W.hidden_states_device(SEED, 0, d_model, 1, n_tok, DEV)
+    cache = case.plan.new_cache(1, n_tok, DEV)
+    aatc.encode_hidden(case.plan, 0, x, case.a_hat, cache, 0, n_tok)
+    torch.cuda.synchronize()
+    assert case.plan.device_error() == 0
+    u32 = cache.cpu().numpy().view(np.uint32)
+    rng = np.random.default_rng(7)
+    toks = np.sort(rng.choice(n_tok, 256, replace=False))
+    xs = x[0, torch.from_numpy(toks).to(DEV)].float().cpu().numpy()
+    total = mis = 0
+    for h in (0, 5):
+        for kind in (0, 1):
+            rec_all, alpha_all = O.cache_records(u32, 1, n_kv, n_tok, case.plan.n_words, 0, h, kind, 0, n_tok)
+            s = Hn.check_codes(case, 0, h, kind, xs, rec_all[toks], alpha_all[toks],
+                               encode_matrix=case.a_hat_host[0, h, kind].T)
+            total += s["codes"]
+            mis += s["mismatch"]
+    assert mis <= Hn.MAX_NEAR_FRACTION * total + 1, (mis, total)
