@@ -18,7 +18,9 @@ form (Eq. bit-allocation, Sec. 3.1), brute force over integer allocations at d=4
 (Eq. waterfilling-keys), a Monte Carlo check of Theorem 1, the whitening-SVD /
 PCA equivalence (Appendix, Proposition), the quantizer error bound
 (Def. uniform-quant), library SDPA for decode, hand-computed small cases and
-the compression ratio the paper prints (Sec. 6.1).
+the compression ratio the paper prints (Sec. 6.1); the transform from the model
+weights (:func:`whitening_transform`, tests/test_whitening.py) is pinned by
+W = A B, A^T Sigma_X A = S and both statements of the appendix Proposition.
 
 parity unpinned: the packed record bit layout (:func:`record_entries`,
 :func:`pack_records`, :func:`cache_records`) is defined by this build, not by the
