@@ -178,7 +178,7 @@ def sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_d
             "policy": "sink 4 + recent window 128 (step 16) in bf16, the rest coded"}
 
 
-def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32768, iters=10):
+def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32768, iters=10, warmup=3):
     """Encode straight from the layer input (Sec. 5 Step 1: the cache holds the coefficients of
     x A): Llama-3.1-8B-shaped layer input, d_model 4096, 8 kv-heads x K|V, 32768 tokens.  The
     plan is calibrated on K = X W of 4096 seeded hidden states and seeded projections; the
@@ -200,9 +200,13 @@ def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32
     a_hat = torch.from_numpy(ah.view(np.int16)).view(torch.bfloat16).to(device).contiguous()
     x = W.hidden_states_device(seed, 0, d_model, 1, n_tokens, device)
     cache = plan.new_cache(1, n_tokens, device)
-    for _ in range(3):
+    for _ in range(warmup):
         aatc.encode_hidden(plan, 0, x, a_hat, cache, 0, n_tokens)
     torch.cuda.synchronize()
+    if iters == 0:
+        assert plan.device_error() == 0
+        plan.close()
+        return {}
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(iters):
@@ -568,11 +572,20 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-once", action="store_true", help="one encode + two decodes, for ncu")
+    ap.add_argument("--profile-hidden", action="store_true", help="one encode from hidden states, for ncu")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.profile_once:
         run_profile_once(args)
+    elif args.profile_hidden:
+        import torch
+        import paper_2608_14191_gb300 as aatc
+        from paper_2608_14191_gb300 import build as bld
+        bld.build()
+        aatc.load()
+        hidden_encode_timing(aatc, torch.device("cuda", 0), iters=0, warmup=1)
+        print(json.dumps({"profile_hidden": "llama layer input, d_model 4096, 32768 tokens"}))
     elif args.impl == "reference":
         run_reference(args)
     else:
