@@ -218,6 +218,27 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x,
                                  int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
                                  void* stream);
 
+/*
+ * Prefill attention over the packed cache (Def. sdpa for each row of a chunk of new query tokens,
+ * causal; Algorithm 1's reconstruct / attend lines in the transformed space: scores
+ * alpha_t (U_K^T q) . (f o code_t) / sqrt(128), output U_V (f o sum_t p_t alpha^V_t code^V_t)).
+ * The chunk's own keys and values must already be in the cache (aatc_encode / aatc_encode_hidden).
+ *   q         : device bf16 [batch][n_q][n_q_heads][128], the queries of positions
+ *               q_start .. q_start + n_q - 1; each attends to cached tokens 0 .. its position
+ *   cache     : the packed cache holding tokens [0, n_ctx), q_start + n_q <= n_ctx <= max_tokens
+ *   out       : device fp32 [batch][n_q][n_q_heads][128]
+ *   workspace : device, >= aatc_prefill_workspace_bytes(batch, n_ctx) (the signed codes of the
+ *               context as f16, [batch][n_kv][K|V][ceil(n_ctx/128)*128][128]); contents ignored
+ * Query head j reads kv-head j / (n_q_heads / n_kv_heads).  Asynchronous on `stream`.
+ * Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer or sizes, q_start + n_q >
+ * n_ctx), AATC_ERR_CAPACITY (n_ctx > max_tokens), AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (W > 32),
+ * AATC_ERR_CUDA.
+ */
+aatc_status_t aatc_prefill_workspace_bytes(aatc_plan_t plan, int32_t batch, int32_t n_ctx, size_t* bytes);
+aatc_status_t aatc_prefill_attention(aatc_plan_t plan, int32_t layer, const void* q, int32_t q_start, int32_t n_q,
+                                     const void* cache, int32_t batch, int32_t n_ctx, int32_t max_tokens, float* out,
+                                     void* workspace, size_t workspace_bytes, void* stream);
+
 /* Device workspace bytes aatc_decode_attention needs for (batch, n_ctx). */
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t plan, int32_t batch, int32_t n_ctx,
                                           size_t* bytes);

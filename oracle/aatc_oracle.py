@@ -493,6 +493,19 @@ def decode_attention(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_
     return out
 
 
+def prefill_attention(q_tokens: np.ndarray, positions: np.ndarray, hk: np.ndarray, hv: np.ndarray,
+                      basis_k: np.ndarray, basis_v: np.ndarray, group: int) -> np.ndarray:
+    """Causal attention of a chunk of new tokens over the coded cache of one sequence (Def. sdpa
+    applied to every query row of the chunk; the cached coefficients stand in for K, V as in
+    Alg. 1's reconstruct / attend lines).  q_tokens: (n_q, H_q, 128) queries at absolute
+    positions `positions` (n_q,); hk, hv: (H_kv, n_ctx, 128) dequantized coefficients; query
+    token at position p attends to cached tokens 0 .. p.  Returns (n_q, H_q, 128)."""
+    out = np.zeros((q_tokens.shape[0], q_tokens.shape[1], D))
+    for i, pos in enumerate(np.asarray(positions, np.int64)):
+        out[i] = decode_attention(q_tokens[i], hk[:, :pos + 1], hv[:, :pos + 1], basis_k, basis_v, group)
+    return out
+
+
 def decode_attention_mixed(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_k: np.ndarray,
                            basis_v: np.ndarray, group: int, k_full: np.ndarray, v_full: np.ndarray) -> np.ndarray:
     """Decode over coded tokens and uncompressed tokens in one softmax (the paper's inference

@@ -50,6 +50,8 @@ SIGNATURES = {
     "aatc_whitening_transform": (_I32, [_I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "aatc_hidden_operand": (_I32, [ctypes.POINTER(Dims), _I32, _P, _P, _P, _P]),
     "aatc_encode_hidden": (_I32, [_P, _I32, _P, _I32, _P, _I32, _I32, _I32, _P, _I32, _P]),
+    "aatc_prefill_workspace_bytes": (_I32, [_P, _I32, _I32, ctypes.POINTER(_SZ)]),
+    "aatc_prefill_attention": (_I32, [_P, _I32, _P, _I32, _I32, _P, _I32, _I32, _I32, _P, _P, _SZ, _P]),
     "aatc_decode_attention_sw": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _SZ,
                                         _P]),
     "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
@@ -261,6 +263,26 @@ def encode_hidden(plan: Plan, layer: int, x, a_hat, cache, start: int, max_token
     batch, n_tokens, d_model = x.shape
     _check(load().aatc_encode_hidden(plan.handle, layer, _ptr(x), d_model, _ptr(a_hat), batch, start, n_tokens,
                                      _ptr(cache), max_tokens, _stream(stream)), "aatc_encode_hidden")
+
+
+def prefill_attention(plan: Plan, layer: int, q, q_start: int, cache, n_ctx: int, max_tokens: int, out=None,
+                      workspace=None, stream=None):
+    """aatc_prefill_attention: q bf16 [batch][n_q][H_q][128] at positions q_start .. q_start + n_q - 1,
+    causal over the packed cache tokens [0, n_ctx) -> fp32 [batch][n_q][H_q][128]."""
+    import torch
+    batch, n_q = q.shape[0], q.shape[1]
+    if out is None:
+        out = torch.empty((batch, n_q, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    nb = _SZ()
+    _check(load().aatc_prefill_workspace_bytes(plan.handle, batch, n_ctx, ctypes.byref(nb)),
+           "aatc_prefill_workspace_bytes")
+    if workspace is None:
+        workspace = torch.empty(max(4, (nb.value + 3) // 4), dtype=torch.float32, device=q.device)
+    _check(load().aatc_prefill_attention(plan.handle, layer, _ptr(q), q_start, n_q, _ptr(cache), batch, n_ctx,
+                                         max_tokens, _ptr(out), _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(), _stream(stream)),
+           "aatc_prefill_attention")
+    return out
 
 
 def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: int, out=None, workspace=None,

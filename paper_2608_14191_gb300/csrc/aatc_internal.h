@@ -147,6 +147,10 @@ constexpr int MAX_FULL_TOKENS = 8192;   // shared-memory scores of the uncompres
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch,
                           int n_ctx, int max_tokens, float* out, void* ws, const DecodeSplit& sp,
                           cudaStream_t st, const DecodeExtra& extra);
+// Prefill attention: codes workspace bytes, and the two launches (codes, attention).
+size_t prefill_workspace(int batch, int n_kv, int n_ctx);
+cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_start, int n_q, const void* cache,
+                           int batch, int n_ctx, int max_tokens, float* out, void* ws, cudaStream_t st);
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n,
                            int max_tokens, float* out, cudaStream_t st);
 cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx,

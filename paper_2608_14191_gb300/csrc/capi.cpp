@@ -337,6 +337,29 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t p, int32_t layer, const void* x, in
                                                 max_tokens, static_cast<cudaStream_t>(stream)));
 }
 
+aatc_status_t aatc_prefill_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
+  *bytes = aatc::prefill_workspace(batch, plan->dims.n_kv_heads, n_ctx);
+  return AATC_OK;
+}
+
+aatc_status_t aatc_prefill_attention(aatc_plan_t p, int32_t layer, const void* q, int32_t q_start, int32_t n_q,
+                                     const void* cache, int32_t batch, int32_t n_ctx, int32_t max_tokens, float* out,
+                                     void* workspace, size_t workspace_bytes, void* stream) {
+  aatc::Plan* plan = as_plan(p);
+  if (!plan || !q || !cache || !out || !workspace || layer < 0 || layer >= plan->dims.n_layers || batch < 1 ||
+      q_start < 0 || n_q < 1 || n_ctx < 1 || max_tokens < 1)
+    return AATC_ERR_INVALID_ARG;
+  if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
+  if (static_cast<int64_t>(q_start) + n_q > n_ctx) return AATC_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(cache) || !aligned16(out) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
+  if (plan->n_words > 32) return AATC_ERR_UNSUPPORTED;
+  if (workspace_bytes < aatc::prefill_workspace(batch, plan->dims.n_kv_heads, n_ctx)) return AATC_ERR_WORKSPACE;
+  return cuda_status(aatc::launch_prefill(*plan, layer, q, q_start, n_q, cache, batch, n_ctx, max_tokens, out,
+                                          workspace, static_cast<cudaStream_t>(stream)));
+}
+
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;

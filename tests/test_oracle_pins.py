@@ -360,3 +360,27 @@ def test_dequantize_f32_is_two_roundings():
     f1 = np.float32(0.7) * np.float32(2.0 ** -1)
     assert got[0, 0] == np.float32(np.float32(3) * np.float32(alpha[0] * f0))
     assert got[0, 1] == np.float32(np.float32(-2) * np.float32(alpha[0] * f1))
+
+
+# --- prefill attention over the coded cache (Def. sdpa with a causal chunk of queries) ----------
+
+def test_prefill_attention_equals_causal_sdpa_on_reconstructed_kv():
+    """Every query row of the chunk is Def. sdpa over the reconstructed keys / values up to its own
+    position: library scaled_dot_product_attention with a causal mask on K = h_K U_K^T, V = h_V U_V^T."""
+    import torch
+    rng = np.random.default_rng(11)
+    hkv, g, n_ctx, n_q = 2, 3, 40, 12
+    q0 = n_ctx - n_q
+    bk = np.stack([np.linalg.qr(rng.standard_normal((O.D, O.D)))[0] for _ in range(hkv)])
+    bv = np.stack([np.linalg.qr(rng.standard_normal((O.D, O.D)))[0] for _ in range(hkv)])
+    hk, hv = rng.standard_normal((hkv, n_ctx, O.D)), rng.standard_normal((hkv, n_ctx, O.D))
+    q = rng.standard_normal((n_q, hkv * g, O.D))
+    out = O.prefill_attention(q, np.arange(q0, n_ctx), hk, hv, bk, bv, g)
+    k = torch.from_numpy(np.einsum("hnc,hdc->hnd", hk, bk))
+    v = torch.from_numpy(np.einsum("hnc,hdc->hnd", hv, bv))
+    for j in range(hkv * g):
+        h = j // g
+        mask = torch.from_numpy(np.arange(n_ctx)[None, :] <= np.arange(q0, n_ctx)[:, None])
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[:, j])[None], k[h][None], v[h][None], attn_mask=mask[None]).numpy()[0]
+        np.testing.assert_allclose(out[:, j], ref, rtol=1e-9, atol=1e-12)
