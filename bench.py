@@ -226,6 +226,57 @@ def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32
                         f"{n_tokens} tokens, 2.75 bits"}
 
 
+def prefill_timing(aatc, device, iters=2):
+    """Prefill attention over the packed cache on the Qwen-2.5-7B-shaped layer: 16 sequences x
+    8192 tokens, 28 query heads over 4 kv-heads, causal (the chunk is the whole context, encoded
+    first).  Flop = 2 (QK) + 2 (PV) x 128 x 28 heads x 16 x 8192 x 8193 / 2 causal pairs.  For
+    context, the same attention on the uncompressed bf16 K/V by torch's scaled_dot_product_attention
+    (a library kernel, not this path)."""
+    import torch
+    cfg = W.CONFIGS["qwen"]
+    B, T = cfg.batch, cfg.n_ctx
+    plan, _ = build_case(aatc, cfg, 2.75, device)
+    kd, vd = W.kv_device(cfg, 0, B, T, device)
+    cache = plan.new_cache(B, T, device)
+    aatc.encode(plan, 0, kd, vd, cache, 0, T)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(W.torch_seed(cfg.seed, 0, 0, 0, "query"))
+    q = torch.randn((B, T, cfg.n_q_heads, 128), generator=gen, device=device).to(torch.bfloat16)
+    out = torch.empty((B, T, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
+    aatc.prefill_attention(plan, 0, q, 0, cache, T, T, out=out)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(iters):
+        aatc.prefill_attention(plan, 0, q, 0, cache, T, T, out=out)
+    e1.record()
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    ms = e0.elapsed_time(e1) / iters
+    flop = 4.0 * 128 * cfg.n_q_heads * B * T * (T + 1) / 2
+    # uncompressed bf16 reference (library SDPA), same shapes, causal, GQA by repeating kv-heads
+    g = cfg.n_q_heads // cfg.n_kv_heads
+    qt = q.transpose(1, 2)
+    kt = kd.transpose(1, 2).repeat_interleave(g, dim=1)
+    vt = vd.transpose(1, 2).repeat_interleave(g, dim=1)
+    torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(iters):
+        torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+    e1.record()
+    torch.cuda.synchronize()
+    ms_ref = e0.elapsed_time(e1) / iters
+    peaks = json.load(open(PEAKS_FILE)) if os.path.exists(PEAKS_FILE) else {}
+    bf16 = float(peaks.get("bf16_tflops", 1900.0))
+    tf = flop / (ms * 1e-3) / 1e12
+    plan.close()
+    return {"ms_per_call": round(ms, 3), "tflops": round(tf, 1), "frac_of_measured_bf16": round(tf / bf16, 4),
+            "bf16_sdpa_ms_uncompressed": round(ms_ref, 3),
+            "workload": f"Qwen-2.5-7B-shaped layer: {B} x {T} tokens, {cfg.n_q_heads}/{cfg.n_kv_heads} heads, "
+                        f"causal prefill over the packed cache (2.75 bits)"}
+
+
 def planner_timing(aatc):
     """Host planner rows: the global cross-layer allocation on Llama-3.1-8B-shaped statistics
     (32 layers x 8 kv-heads x K|V x 128 channels; seeded log-normal spectra), median of 5 runs."""
@@ -361,6 +412,7 @@ def run_ours(args):
 
     sw = sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_dec)
     hid = hidden_encode_timing(aatc, dev)
+    pre = prefill_timing(aatc, dev)
 
     # max over ranks
     vals = torch.tensor([total_ms, float(np.mean(dec_ms)), float(np.mean(enc_ms)), e2e_ms], device=dev)
@@ -418,6 +470,7 @@ def run_ours(args):
         "planner": planner_timing(aatc),
         "sink_window": sw,
         "encode_hidden": hid,
+        "prefill": pre,
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds)
