@@ -226,7 +226,7 @@ def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32
                         f"{n_tokens} tokens, 2.75 bits"}
 
 
-def prefill_timing(aatc, device, iters=2):
+def prefill_timing(aatc, device, iters=2, batch=None, reference=True):
     """Prefill attention over the packed cache on the Qwen-2.5-7B-shaped layer: 16 sequences x
     8192 tokens, 28 query heads over 4 kv-heads, causal (the chunk is the whole context, encoded
     first).  Flop = 2 (QK) + 2 (PV) x 128 x 28 heads x 16 x 8192 x 8193 / 2 causal pairs.  For
@@ -234,7 +234,7 @@ def prefill_timing(aatc, device, iters=2):
     (a library kernel, not this path)."""
     import torch
     cfg = W.CONFIGS["qwen"]
-    B, T = cfg.batch, cfg.n_ctx
+    B, T = cfg.batch if batch is None else batch, cfg.n_ctx
     plan, _ = build_case(aatc, cfg, 2.75, device)
     kd, vd = W.kv_device(cfg, 0, B, T, device)
     cache = plan.new_cache(B, T, device)
@@ -245,6 +245,10 @@ def prefill_timing(aatc, device, iters=2):
     out = torch.empty((B, T, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
     aatc.prefill_attention(plan, 0, q, 0, cache, T, T, out=out)
     torch.cuda.synchronize()
+    if iters == 0:
+        assert plan.device_error() == 0
+        plan.close()
+        return {}
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(iters):
@@ -626,6 +630,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-once", action="store_true", help="one encode + two decodes, for ncu")
     ap.add_argument("--profile-hidden", action="store_true", help="one encode from hidden states, for ncu")
+    ap.add_argument("--profile-prefill", action="store_true", help="one Qwen-shaped prefill at batch 2, for ncu")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -639,6 +644,14 @@ def main():
         aatc.load()
         hidden_encode_timing(aatc, torch.device("cuda", 0), iters=0, warmup=1)
         print(json.dumps({"profile_hidden": "llama layer input, d_model 4096, 32768 tokens"}))
+    elif args.profile_prefill:
+        import torch
+        import paper_2608_14191_gb300 as aatc
+        from paper_2608_14191_gb300 import build as bld
+        bld.build()
+        aatc.load()
+        prefill_timing(aatc, torch.device("cuda", 0), iters=0, batch=2)
+        print(json.dumps({"profile_prefill": "qwen layer, batch 2 x 8192, causal"}))
     elif args.impl == "reference":
         run_reference(args)
     else:
