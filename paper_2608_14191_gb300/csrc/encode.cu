@@ -99,33 +99,28 @@ __device__ __forceinline__ void append_bits(uint32_t v, int nb, uint32_t& word, 
 // 128 coefficients are read from TMEM columns taddr .. taddr + 127 (twice: amax, then quantize).
 __device__ __forceinline__ float quantize_token(uint32_t taddr, const ChanEnc* enc, const float* inv_s,
                                                 uint32_t* row) {
+  // Eight 32-column TMEM loads (four per pass), each issued before the previous chunk is
+  // processed so its latency overlaps that work; registers alternate between ra and rb.
+  uint32_t ra[32], rb[32];
   float amax = 0.0f;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    float h[32];
-    ptx::tmem_ld_32cols(taddr + 32 * j, h);
-    ptx::tmem_ld_wait();
+  auto amax_chunk = [&](const uint32_t (&r)[32], int j) {
 #pragma unroll
     for (int i = 0; i < 32; i += 4) {
       const float4 is = *reinterpret_cast<const float4*>(&inv_s[32 * j + i]);
-      amax = fmaxf(amax, fabsf(h[i]) * is.x);
-      amax = fmaxf(amax, fabsf(h[i + 1]) * is.y);
-      amax = fmaxf(amax, fabsf(h[i + 2]) * is.z);
-      amax = fmaxf(amax, fabsf(h[i + 3]) * is.w);
+      amax = fmaxf(amax, fabsf(__uint_as_float(r[i])) * is.x);
+      amax = fmaxf(amax, fabsf(__uint_as_float(r[i + 1])) * is.y);
+      amax = fmaxf(amax, fabsf(__uint_as_float(r[i + 2])) * is.z);
+      amax = fmaxf(amax, fabsf(__uint_as_float(r[i + 3])) * is.w);
     }
-  }
-  const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+  };
+  float ia = 0.0f;
   // The round-down add of 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    float h[32];
-    ptx::tmem_ld_32cols(taddr + 32 * j, h);
-    ptx::tmem_ld_wait();
+  auto quant_chunk = [&](const uint32_t (&r)[32], int j) {
     uint32_t y[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       const ChanEnc e = enc[32 * j + i];
-      float x = fmaf(h[i], e.inv_f * ia, 0.5f);                // h / Delta + 1/2
+      float x = fmaf(__uint_as_float(r[i]), e.inv_f * ia, 0.5f);   // h / Delta + 1/2
       x = fminf(x, e.hi);                                       // |h| / Delta <= 2^(b-1): only the top clamps
       y[i] = __float_as_uint(__fadd_rd(x, e.magic));            // floor, offset binary in the mantissa
     }
@@ -133,7 +128,40 @@ __device__ __forceinline__ float quantize_token(uint32_t taddr, const ChanEnc* e
     for (int q = 0; q < 8; ++q)
       row[8 * j + q] = __byte_perm(__byte_perm(y[4 * q], y[4 * q + 1], 0x0040),
                                    __byte_perm(y[4 * q + 2], y[4 * q + 3], 0x0040), 0x5410);
-  }
+  };
+  ptx::tmem_ld_32raw(taddr, ra);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  amax_chunk(ra, 0);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  amax_chunk(rb, 1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  amax_chunk(ra, 2);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr, ra);
+  amax_chunk(rb, 3);
+  ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  quant_chunk(ra, 0);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  quant_chunk(rb, 1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  quant_chunk(ra, 2);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  quant_chunk(rb, 3);
   return amax;
 }
 
