@@ -56,6 +56,21 @@ def _dist():
     return ws, rank
 
 
+def max_over_ranks(values, ws, device=None):
+    """Each timing's maximum over the ranks (the slowest replica defines the job's time); a
+    collective only when ws > 1 (any torch.distributed backend)."""
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if ws > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(x) for x in t.cpu()]
+
+
+def whole_job_rate(units_per_rank, ws, ms):
+    """Weak scaling: every rank processes units_per_rank in the same (max-over-ranks) time."""
+    return ws * units_per_rank / (ms * 1e-3)
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled every 200 ms during the timed region."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -414,24 +429,22 @@ def run_ours(args):
     d2h = out.numel() * 4
     assert plan.device_error() == 0
 
+    # max over ranks, then only rank 0 goes on (the context legs below are single-GPU figures)
+    total_ms, dec_mean, enc_mean, e2e_ms = max_over_ranks(
+        [total_ms, float(np.mean(dec_ms)), float(np.mean(enc_ms)), e2e_ms], ws_, device=dev)
+    if ws_ > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return
+
     sw = sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_dec)
     hid = hidden_encode_timing(aatc, dev)
     pre = prefill_timing(aatc, dev)
 
-    # max over ranks
-    vals = torch.tensor([total_ms, float(np.mean(dec_ms)), float(np.mean(enc_ms)), e2e_ms], device=dev)
-    if ws_ > 1:
-        torch.distributed.all_reduce(vals, op=torch.distributed.ReduceOp.MAX)
-    total_ms, dec_mean, enc_mean, e2e_ms = [float(x) for x in vals.cpu()]
-    if rank != 0:
-        if ws_ > 1:
-            torch.distributed.destroy_process_group()
-        return
-
     peak, peak_kind = _peaks()
     dbytes = decode_bytes(plan, cfg, B, T)
     per_decode_ms = dec_mean / steps_dec
-    gbs = ws_ * dbytes / (per_decode_ms * 1e-3) / 1e9           # whole job
+    gbs = whole_job_rate(dbytes, ws_, per_decode_ms) / 1e9      # whole job
     achieved = dbytes / (per_decode_ms * 1e-3) / 1e9              # per launch (one GPU)
     enc_tokens = B * T
     enc_in_bytes = B * T * cfg.n_kv_heads * 2 * 128 * 2
