@@ -127,6 +127,10 @@ Plan* plan_from_handle(aatc_plan_t p);
 aatc_status_t status_from_cuda(cudaError_t e);
 
 // Kernel launchers (defined in the .cu files); return the CUDA error of the launch.
+// 2D tiled tensor map with 128-byte swizzle (16-bit elements): `map` is a 128-byte, 64-aligned
+// CUtensorMap; rows of `inner` elements, `row_bytes` apart; box box_inner x box_rows.
+cudaError_t make_tensor_map_2d(void* map, bool f16, const void* base, uint64_t inner, uint64_t rows,
+                               uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows);
 cudaError_t encode_tensor_maps_u(Plan& plan);
 cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void* V, int batch,
                           int start, int n_tokens, void* cache, int max_tokens, cudaStream_t st);

@@ -529,6 +529,21 @@ cudaError_t make_kv_map(CUtensorMap* map, const void* base, int batch, int n_tok
 
 }  // namespace
 
+cudaError_t make_tensor_map_2d(void* map, bool f16, const void* base, uint64_t inner, uint64_t rows,
+                               uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
+  const cuuint32_t box[2] = {box_inner, box_rows};
+  const cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(reinterpret_cast<CUtensorMap*>(map),
+                   f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                   const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 cudaError_t encode_tensor_maps_u(Plan& plan) {
   auto enc = tensor_map_encoder();
   if (!enc) return cudaErrorNotSupported;

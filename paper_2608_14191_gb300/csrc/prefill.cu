@@ -4,26 +4,25 @@
 //
 // Two launches per call:
 //   codes    per (128-token tile, kv-head x K|V, sequence): the packed records -> the signed codes
-//            code_c = u_c - 2^(b_c - 1) as f16 (exact: |code| <= 128), [b][h][K|V][n_ctx_pad][128];
-//   attn     per (64 query rows, kv-head, sequence), rows = (query token, head of the GQA group):
-//            q' = (U_K^T q) f^K log2(e) / sqrt(128) as f16 hi/lo (CUDA cores, fp32), then per
-//            64-token tile S = alpha^K (q'_hi + q'_lo) . code^K (mma.sync m16n8k16), causal mask,
-//            online softmax, P' = 2^(S - m) alpha^V (f16) and O += P' code^V, finally
-//            out = U_V (f^V O / l) (CUDA cores, fp32).
+//            code_c = u_c - 2^(b_c - 1) as f16 (exact: |code| <= 128) in a workspace of rows of 128
+//            f16, [b][h][K|V][n_ctx_pad][128]: key rows are tokens, value tiles are stored
+//            transposed ([tile][channel][token]) so both are K-major tensor-core operands;
+//   attn     per (128 query rows, kv-head, sequence), rows = (query token, head of the GQA group),
+//            everything on the tensor cores (tcgen05): q' = (U_K^T q) f^K log2(e) / sqrt(128),
+//            per 128-token tile S = alpha^K (q'_hi + q'_lo) . code^K, causal mask, lazily
+//            rescaled softmax, P' = 2^(S - m) alpha^V (f16) and O += P' code^V, finally
+//            out = U_V (f^V O / l).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include <algorithm>
 
 #include "aatc_internal.h"
+#include "ptx.cuh"
 
 namespace aatc {
 namespace {
 
-constexpr int kPThreads = 128;      // 4 warps x 16 query rows
-constexpr int kPRows = 64;
-constexpr int kPKV = 64;            // cached tokens per tile
-constexpr int kPStride = D + 8;     // f16 row stride of the code tiles (272 B: ldmatrix rows in distinct banks)
 constexpr float kPLog2e = 1.4426950408889634f;
 constexpr float kPOpMax = 16384.0f; // q' rows scaled so the largest |value| is 2^14
 
@@ -41,6 +40,7 @@ struct PrefillArgs {
   const short* entry;        // plan: [S][n_entries]
   const short* chan_ent;     // plan: [S][128][8]
   int layer, n_kv, n_q_heads, group, q_start, n_q, n_ctx, n_ctx_pad, n_tiles, n_words, n_entries;
+  int* err;
 };
 
 __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillArgs a) {
@@ -51,8 +51,14 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
   const int tok = tile * TILE + t;
   __half* dst = a.codes + (cs * a.n_ctx_pad + tok) * D;
   if (tok >= a.n_ctx) {                        // padding rows of the last tile: zero codes
-    if (tok < a.n_ctx_pad)
-      for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(dst + c) = make_uint4(0u, 0u, 0u, 0u);
+    if (tok < a.n_ctx_pad) {
+      if (kind == 1) {
+        __half* d2 = a.codes + cs * a.n_ctx_pad * D + static_cast<size_t>(tile) * TILE * D + t;
+        for (int c = 0; c < D; ++c) d2[c * TILE] = __float2half_rn(0.0f);
+      } else {
+        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(dst + c) = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
     return;
   }
   const int s = (a.layer * a.n_kv + head) * 2 + kind;
@@ -73,6 +79,9 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
   }
   const short* ce = a.chan_ent + static_cast<size_t>(s) * D * 8;
   const short* ent = a.entry + static_cast<size_t>(s) * a.n_entries;
+  // values for the tensor-core kernel: per 128-token tile [channel][token]
+  __half* dst_t = a.codes + cs * a.n_ctx_pad * D + static_cast<size_t>(tile) * TILE * D + t;
+  const bool transposed = kind == 1;
   for (int c = 0; c < D; c += 2) {
     float v2[2];
 #pragma unroll
@@ -93,32 +102,15 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
       }
       v2[i] = static_cast<float>(u) - a.enc[s * D + cc].off;   // dropped channels: u = off = 0
     }
-    *reinterpret_cast<__half2*>(dst + c) = __floats2half2_rn(v2[0], v2[1]);
+    if (transposed) {
+      dst_t[c * TILE] = __float2half_rn(v2[0]);
+      dst_t[(c + 1) * TILE] = __float2half_rn(v2[1]);
+    } else {
+      *reinterpret_cast<__half2*>(dst + c) = __floats2half2_rn(v2[0], v2[1]);
+    }
   }
 }
 
-__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))));
-}
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
-               "l"(src)
-               : "memory");
-}
 __device__ __forceinline__ float ex2(float x) {
   float r;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
@@ -129,266 +121,430 @@ __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-struct PrefillSmem {
-  __half kc[2][kPKV][kPStride];
-  __half vc[2][kPKV][kPStride];
-  float ak[2][kPKV], av[2][kPKV];
-  float qs[kPRows][D];          // q (fp32), then q', then o_hat
-};
+// ---------------------------------------------------------------- tensor-core (tcgen05) attention
+// Per CTA 128 query rows (= TMEM lanes) of one (kv-head, sequence); 8 warps, warp w owns TMEM
+// lanes 32 (w & 3) .. + 31 and the column half w >> 2 of every 128-column TMEM block.
+//   prologue  q' = (q U_K) f^K log2(e) / sqrt(128) on the tensor cores: q (bf16, exact) against
+//             U_K split into three bf16 parts (about 2^-25 relative), rows scaled to 2^14 and
+//             split into f16 hi / lo operands
+//   per 128-token tile (TMA, 128-byte swizzle, key and value tiles double-buffered):
+//             S = q'_hi . code_K + q'_lo . code_K   tcgen05.mma M = N = 128, K = 128; S of tile
+//             t + 1 is issued before the softmax of tile t (two S buffers in TMEM)
+//             softmax from TMEM with the scores held in registers between the maximum and the
+//             exponent: s = S rs alpha^K (causal mask), lazy maximum (O rescaled only when a
+//             row's maximum grows by more than 2^8, so P' = 2^(s - m) alpha^V stays inside f16)
+//             P' stored to TMEM as f16 pairs: the A operand of O += P' . code_V^T
+//   epilogue  out = (f^V O / l) U_V^T on the tensor cores, both operands split hi / lo in bf16.
+constexpr int kTRows = 128;
+constexpr int kTThreads = 256;
+constexpr int kTAtom = 128 * 128;                  // one 128-row K-atom (64 16-bit values per row)
+constexpr int kTOp = 2 * kTAtom;                   // one 128 x 128 16-bit operand (two K-atoms)
+constexpr float kLazyLog2 = 8.0f;
+constexpr uint32_t kIdescTT = ptx::idesc_f16_f32(128, 128);
+constexpr uint32_t kIdescBB = ptx::idesc_bf16_f32(128, 128);
+constexpr uint32_t kColS = 0;                      // two score buffers (0, 128); projection results
+constexpr uint32_t kColO = 256;                    // O accumulator
+constexpr uint32_t kColP = 384;                    // P' (64 columns of f16 pairs)
 
-__global__ void __launch_bounds__(kPThreads) aatc_prefill_attn_kernel(const PrefillArgs a) {
-  extern __shared__ __align__(16) unsigned char psm[];
-  PrefillSmem& sm = *reinterpret_cast<PrefillSmem*>(psm);
+struct PrefillTcSmem {
+  alignas(1024) unsigned char qh[kTOp];            // q' hi: K-atoms = channels 0-63 | 64-127, rows = query rows
+  alignas(1024) unsigned char ql[kTOp];            // q' lo
+  alignas(1024) unsigned char kt[2][kTOp];         // key codes: K-atoms = channels, rows = tokens
+  alignas(1024) unsigned char vt[2][kTOp];         // value codes: K-atoms = tokens 0-63 | 64-127, rows = channels
+  float ak[2][TILE], av[2][TILE];
+  float xch[2][kTRows];                            // per-row partials of the two column halves
+  uint64_t bar_k[2], bar_v[2], bar_s[2], bar_o, bar_p;
+  uint32_t tmem;
+  int abort_flag;
+};
+// kt and vt together hold the four projection operands (prologue, epilogue)
+static_assert(offsetof(PrefillTcSmem, vt) == offsetof(PrefillTcSmem, kt) + 2 * kTOp, "operand slots contiguous");
+
+// byte offset of element (row, k) of a 128-row K-major operand with the 128-byte swizzle
+__device__ __forceinline__ int sw128_off(int row, int k) {
+  return (k >> 6) * kTAtom + (row >> 3) * 1024 + (row & 7) * 128 + ((((k & 63) >> 3) ^ (row & 7)) << 4) + (k & 7) * 2;
+}
+
+__device__ __forceinline__ uint32_t pack_bf2(__nv_bfloat16 lo, __nv_bfloat16 hi) {
+  return static_cast<uint32_t>(__bfloat16_as_ushort(lo)) | (static_cast<uint32_t>(__bfloat16_as_ushort(hi)) << 16);
+}
+
+// 8 fp32 values -> `parts` bf16 parts (u = p0 + p1 + p2 up to the last part's rounding), each
+// stored as one 16-byte granule at dst[i * kTOp]
+__device__ __forceinline__ void store_split_bf16(unsigned char* dst, const float (&u)[8], int parts) {
+  uint32_t w[3][4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    float x0 = u[2 * j], x1 = u[2 * j + 1];
+#pragma unroll
+    for (int p = 0; p < 3; ++p) {
+      const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+      w[p][j] = pack_bf2(h0, h1);
+      x0 -= __bfloat162float(h0);
+      x1 -= __bfloat162float(h1);
+    }
+  }
+#pragma unroll
+  for (int p = 0; p < 3; ++p)
+    if (p < parts) *reinterpret_cast<uint4*>(dst + p * kTOp) = make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
+}
+
+__global__ void __launch_bounds__(kTThreads, 1)
+    aatc_prefill_tc_kernel(const __grid_constant__ CUtensorMap tm, const PrefillArgs a) {
+  extern __shared__ unsigned char smraw[];
+  PrefillTcSmem& sm =
+      *reinterpret_cast<PrefillTcSmem*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   const int rb = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = a.group, n_rows = a.n_q * G;
   const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;
   const size_t csk = (static_cast<size_t>(b) * a.n_kv + head) * 2, csv = csk + 1;
-  // rows of this CTA: R = 64 rb + r -> query token R / G, head head * G + R % G
-  auto row_pos = [&](int r) { return a.q_start + (rb * kPRows + r) / G; };
-  const int r_last = min(n_rows - 1, rb * kPRows + kPRows - 1) - rb * kPRows;
-  const int kv_end = min(a.n_ctx, row_pos(r_last) + 1);       // tokens [0, kv_end) can be attended
-  const int n_kv_tiles = (kv_end + kPKV - 1) / kPKV;
-
-  auto load_tile = [&](int jt, int buf) {
-    const __half* kg = a.codes + (csk * a.n_ctx_pad + static_cast<size_t>(jt) * kPKV) * D;
-    const __half* vg = a.codes + (csv * a.n_ctx_pad + static_cast<size_t>(jt) * kPKV) * D;
-    for (int i = tid; i < kPKV * (D / 8); i += kPThreads) {
-      const int r = i >> 4, c8 = (i & 15) * 8;
-      cp_async16(&sm.kc[buf][r][c8], kg + r * D + c8);
-      cp_async16(&sm.vc[buf][r][c8], vg + r * D + c8);
+  const int R0 = rb * kTRows;
+  const int r_last = min(n_rows - 1, R0 + kTRows - 1) - R0;
+  const int kv_end = min(a.n_ctx, a.q_start + (R0 + r_last) / G + 1);
+  const int n_kv_tiles = (kv_end + TILE - 1) / TILE;
+  const int r = 32 * (warp & 3) + lane, half = warp >> 2, hc = 64 * half;
+  const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
+  const int R = R0 + r;
+  unsigned char* const pj = sm.kt[0];              // projection operand i at pj + i * kTOp
+  volatile int* abort_flag = &sm.abort_flag;
+  auto wait = [&](uint64_t* bar, uint32_t parity) {
+    if (!ptx::mbar_wait_bounded(bar, parity, abort_flag)) {
+      sm.abort_flag = 1;
+      atomicOr(a.err, 2);
     }
-    if (tid < kPKV) {
-      const int tok = jt * kPKV + tid;
-      sm.ak[buf][tid] = a.alpha[csk * a.n_tiles * TILE + tok];
-      sm.av[buf][tid] = a.alpha[csv * a.n_tiles * TILE + tok];
-    }
-    asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  if (n_kv_tiles > 0) load_tile(0, 0);
 
-  // ---- q' rows: q (bf16 -> fp32) into shared memory, then (U_K^T q) f^K log2(e) / sqrt(128)
-  for (int i = tid; i < kPRows * D; i += kPThreads) {
-    const int r = i >> 7, d = i & (D - 1);
-    const int R = rb * kPRows + r;
-    float v = 0.0f;
-    if (R < n_rows) {
-      const int qi = R / G, qh = head * G + R % G;
-      v = __bfloat162float(a.q[((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh) * D + d]);
-    }
-    sm.qs[r][d] = v;
+  if (tid == 0) {
+    ptx::mbar_init(&sm.bar_k[0], 1);
+    ptx::mbar_init(&sm.bar_k[1], 1);
+    ptx::mbar_init(&sm.bar_v[0], 1);
+    ptx::mbar_init(&sm.bar_v[1], 1);
+    ptx::mbar_init(&sm.bar_s[0], 1);
+    ptx::mbar_init(&sm.bar_s[1], 1);
+    ptx::mbar_init(&sm.bar_o, 1);
+    ptx::mbar_init(&sm.bar_p, 1);
+    sm.abort_flag = 0;
+    ptx::fence_mbar_init();
+    ptx::prefetch_tmap(&tm);
   }
+  if (warp == 0) {
+    ptx::tmem_alloc(&sm.tmem, 512);
+    ptx::tmem_relinquish();
+  }
+  // ---- projection operands: q rows (bf16) in slot 0, U_K^T (rows = channel, K = dim) in three
+  // bf16 parts in slots 1-3
+  for (int g = tid; g < kTRows * 16; g += kTThreads) {
+    const int row = g >> 4, k8 = (g & 15) * 8, RR = R0 + row;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (RR < n_rows) {
+      const int qi = RR / G, qh = head * G + RR % G;
+      v = *reinterpret_cast<const uint4*>(a.q + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh) * D + k8);
+    }
+    *reinterpret_cast<uint4*>(pj + sw128_off(row, k8)) = v;
+  }
+  {
+    const float* ukt = a.u32t + static_cast<size_t>(sk) * D * D;
+    for (int g = tid; g < D * 16; g += kTThreads) {
+      const int c = g >> 4, k8 = (g & 15) * 8;
+      const float4 u0 = *reinterpret_cast<const float4*>(ukt + c * D + k8);
+      const float4 u1 = *reinterpret_cast<const float4*>(ukt + c * D + k8 + 4);
+      const float u[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+      store_split_bf16(pj + kTOp + sw128_off(c, k8), u, 3);
+    }
+  }
+  ptx::fence_proxy_async_smem();
+  ptx::tc_fence_before();
   __syncthreads();
-  float rs[2];                                  // score scale of rows g, g + 8 of this warp
-  {
-    // warp = 16 rows, lane = channels 4 lane .. 4 lane + 3
-    float acc[16][4];
+  ptx::tc_fence_after();
+  const uint32_t tmem = sm.tmem;
+  const uint32_t pj_a = ptx::smem_u32(pj);
+  if (tid == 0) {
+#pragma unroll 1
+    for (int part = 0; part < 3; ++part)
 #pragma unroll
-    for (int r = 0; r < 16; ++r)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
-    const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + 4 * lane;
-    for (int d = 0; d < D; ++d) {
-      const float4 u4 = *reinterpret_cast<const float4*>(uk + d * D);
-#pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        const float qv = sm.qs[16 * warp + r][d];
-        acc[r][0] = fmaf(qv, u4.x, acc[r][0]);
-        acc[r][1] = fmaf(qv, u4.y, acc[r][1]);
-        acc[r][2] = fmaf(qv, u4.z, acc[r][2]);
-        acc[r][3] = fmaf(qv, u4.w, acc[r][3]);
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+        ptx::umma_bf16(tmem + kColS, ptx::sdesc_kmajor_sw128(pj_a + off),
+                       ptx::sdesc_kmajor_sw128(pj_a + (1 + part) * kTOp + off), kIdescBB, (part | kk) ? 1u : 0u);
       }
-    }
-    const float4 f4 = *reinterpret_cast<const float4*>(a.f + sk * D + 4 * lane);
-    const float sc = kPLog2e * 0.08838834764831845f;
-    float mx[16];
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      acc[r][0] *= f4.x * sc;
-      acc[r][1] *= f4.y * sc;
-      acc[r][2] *= f4.z * sc;
-      acc[r][3] *= f4.w * sc;
-      float m = fmaxf(fmaxf(fabsf(acc[r][0]), fabsf(acc[r][1])), fmaxf(fabsf(acc[r][2]), fabsf(acc[r][3])));
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-      mx[r] = m;
-    }
-    __syncwarp();
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      const float inv = mx[r] > 0.0f ? kPOpMax / mx[r] : 0.0f;
-      *reinterpret_cast<float4*>(&sm.qs[16 * warp + r][4 * lane]) =
-          make_float4(acc[r][0] * inv, acc[r][1] * inv, acc[r][2] * inv, acc[r][3] * inv);
-    }
-    rs[0] = rs[1] = 0.0f;
-    // mx[] is indexed by g (lane-dependent): pick without local memory
-#pragma unroll
-    for (int r = 0; r < 8; ++r)
-      if (r == g) {
-        rs[0] = mx[r] / kPOpMax;
-        rs[1] = mx[r + 8] / kPOpMax;
-      }
+    ptx::umma_commit(&sm.bar_p);
   }
-  __syncwarp();
-  // A fragments of q' (rows g, g + 8 of this warp), hi and lo
-  uint32_t qh[8][4], ql[8][4];
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks) {
-    const float* r0 = sm.qs[16 * warp + g];
-    const float* r1 = sm.qs[16 * warp + g + 8];
-    const int k0 = 16 * ks + 2 * t, k1 = k0 + 8;
-    const float v[8] = {r0[k0], r0[k0 + 1], r1[k0], r1[k0 + 1], r0[k1], r0[k1 + 1], r1[k1], r1[k1 + 1]};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const __half2 h = __floats2half2_rn(v[2 * j], v[2 * j + 1]);
-      const float2 hf = __half22float2(h);
-      qh[ks][j] = *reinterpret_cast<const uint32_t*>(&h);
-      ql[ks][j] = pack_h2(v[2 * j] - hf.x, v[2 * j + 1] - hf.y);
-    }
-  }
-  const int pos0 = row_pos(16 * warp + g), pos1 = row_pos(16 * warp + g + 8);
+  wait(&sm.bar_p, 0);
+  ptx::tc_fence_after();
 
-  // ---- online softmax over the cached tokens
-  float o[16][4];
-#pragma unroll
-  for (int n = 0; n < 16; ++n)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) o[n][j] = 0.0f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
-  for (int jt = 0; jt < n_kv_tiles; ++jt) {
-    const int buf = jt & 1;
-    if (jt + 1 < n_kv_tiles) {
-      load_tile(jt + 1, buf ^ 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();
-    float s[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) s[n][j] = 0.0f;
-#pragma unroll
-    for (int np = 0; np < 4; ++np)
-#pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        // matrices: tokens 16np + (0..7 | 8..15) x channels 16ks + (0..7 | 8..15)
-        const int mi = lane >> 3;
-        uint32_t bb[4];
-        ldsm_x4(bb, &sm.kc[buf][16 * np + (mi >> 1) * 8 + (lane & 7)][16 * ks + (mi & 1) * 8]);
-        mma16816(s[2 * np], qh[ks], bb[0], bb[1]);
-        mma16816(s[2 * np], ql[ks], bb[0], bb[1]);
-        mma16816(s[2 * np + 1], qh[ks], bb[2], bb[3]);
-        mma16816(s[2 * np + 1], ql[ks], bb[2], bb[3]);
-      }
-    // scores: rows g (c0, c1) and g + 8 (c2, c3), tokens 64 jt + 8n + 2t + {0, 1}
-    float mt0 = m0, mt1 = m1;
-#pragma unroll
-    for (int n = 0; n < 8; ++n)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int tl = 8 * n + 2 * t + (j & 1), tok = jt * kPKV + tl;
-        const bool row1 = j >= 2;
-        const bool ok = tok <= (row1 ? pos1 : pos0) && tok < a.n_ctx;
-        const float v = ok ? s[n][j] * (row1 ? rs[1] : rs[0]) * sm.ak[buf][tl] : -INFINITY;
-        s[n][j] = v;
-        if (row1) mt1 = fmaxf(mt1, v); else mt0 = fmaxf(mt0, v);
-      }
-#pragma unroll
-    for (int off = 1; off < 4; off <<= 1) {
-      mt0 = fmaxf(mt0, __shfl_xor_sync(0xffffffffu, mt0, off));
-      mt1 = fmaxf(mt1, __shfl_xor_sync(0xffffffffu, mt1, off));
-    }
-    const float c0 = mt0 == -INFINITY ? 1.0f : ex2(m0 - mt0), c1 = mt1 == -INFINITY ? 1.0f : ex2(m1 - mt1);
-    m0 = mt0;
-    m1 = mt1;
-    l0 *= c0;
-    l1 *= c1;
-#pragma unroll
-    for (int n = 0; n < 16; ++n) {
-      o[n][0] *= c0;
-      o[n][1] *= c0;
-      o[n][2] *= c1;
-      o[n][3] *= c1;
-    }
-    uint32_t pa[4][4];                          // P' A fragments, k16-step = 16 tokens
-#pragma unroll
-    for (int n = 0; n < 8; ++n) {
-      float p[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int tl = 8 * n + 2 * t + (j & 1);
-        const float mm = j >= 2 ? m1 : m0;
-        const float e = s[n][j] == -INFINITY ? 0.0f : ex2(s[n][j] - mm);
-        if (j >= 2) l1 += e; else l0 += e;
-        p[j] = e * sm.av[buf][tl];
-        if (s[n][j] == -INFINITY) p[j] = 0.0f;
-      }
-      pa[n >> 1][(n & 1) * 2 + 0] = pack_h2(p[0], p[1]);     // row g, tokens 2t, 2t+1 (+8 for odd n)
-      pa[n >> 1][(n & 1) * 2 + 1] = pack_h2(p[2], p[3]);     // row g + 8
-    }
-#pragma unroll
-    for (int ks2 = 0; ks2 < 4; ++ks2) {
-      // A: a0 = (row g, k 2t..), a1 = (row g+8, k 2t..), a2 = (row g, k 2t+8..), a3 = (row g+8, k 2t+8..)
-      const uint32_t af[4] = {pa[ks2][0], pa[ks2][1], pa[ks2][2], pa[ks2][3]};
-#pragma unroll
-      for (int cp = 0; cp < 8; ++cp) {
-        // matrices: tokens 16ks2 + (0..7 | 8..15) x channels 16cp + (0..7 | 8..15), transposed
-        const int mi = lane >> 3;
-        uint32_t bb[4];
-        ldsm_x4_t(bb, &sm.vc[buf][16 * ks2 + (mi & 1) * 8 + (lane & 7)][16 * cp + (mi >> 1) * 8]);
-        mma16816(o[2 * cp], af, bb[0], bb[1]);
-        mma16816(o[2 * cp + 1], af, bb[2], bb[3]);
-      }
-    }
-    __syncthreads();                            // buffer `buf` is refilled by the next iteration
-  }
-  // ---- o_hat = f^V O / l, then out = U_V o_hat
-#pragma unroll
-  for (int off = 1; off < 4; off <<= 1) {
-    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-  }
-  const float il0 = l0 > 0.0f ? 1.0f / l0 : 0.0f, il1 = l1 > 0.0f ? 1.0f / l1 : 0.0f;
-  __syncwarp();
-#pragma unroll
-  for (int n = 0; n < 16; ++n) {
-    const int c = 8 * n + 2 * t;
-    const float f0 = a.f[sv * D + c], f1 = a.f[sv * D + c + 1];
-    sm.qs[16 * warp + g][c] = o[n][0] * il0 * f0;
-    sm.qs[16 * warp + g][c + 1] = o[n][1] * il0 * f1;
-    sm.qs[16 * warp + g + 8][c] = o[n][2] * il1 * f0;
-    sm.qs[16 * warp + g + 8][c + 1] = o[n][3] * il1 * f1;
-  }
-  __syncwarp();
+  // ---- q' rows scaled to 2^14, f16 hi / lo into the score operands
+  float rsr;
   {
-    float acc[16][4];
+    uint32_t q0[32], q1[32];
+    ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc, q0);
+    ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc + 32, q1);
+    ptx::tmem_ld_wait();
+    ptx::tmem_regs_ready(q0);
+    ptx::tmem_regs_ready(q1);
+    const float sc = kPLog2e * 0.08838834764831845f;
+    const float* fk = a.f + sk * D + hc;
+    float x[64];
+    float m = 0.0f;
 #pragma unroll
-    for (int r = 0; r < 16; ++r)
+    for (int i = 0; i < 32; ++i) {
+      x[i] = __uint_as_float(q0[i]) * fk[i] * sc;
+      x[32 + i] = __uint_as_float(q1[i]) * fk[32 + i] * sc;
+      m = fmaxf(m, fmaxf(fabsf(x[i]), fabsf(x[32 + i])));
+    }
+    sm.xch[half][r] = m;
+    __syncthreads();
+    m = fmaxf(sm.xch[0][r], sm.xch[1][r]);
+    const float inv = m > 0.0f ? kPOpMax / m : 0.0f;
+    rsr = m > 0.0f ? m / kPOpMax : 1.0f;             // > 0, so the mask's -inf survives the scaling
 #pragma unroll
-      for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
-    const float* ut = a.u32t + static_cast<size_t>(sv) * D * D + 4 * lane;   // [ch][dim]
-    for (int c = 0; c < D; ++c) {
-      const float4 u4 = *reinterpret_cast<const float4*>(ut + c * D);
+    for (int g8 = 0; g8 < 8; ++g8) {
+      uint32_t hv[4], lv[4];
 #pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        const float ov = sm.qs[16 * warp + r][c];
-        acc[r][0] = fmaf(ov, u4.x, acc[r][0]);
-        acc[r][1] = fmaf(ov, u4.y, acc[r][1]);
-        acc[r][2] = fmaf(ov, u4.z, acc[r][2]);
-        acc[r][3] = fmaf(ov, u4.w, acc[r][3]);
+      for (int j = 0; j < 4; ++j) {
+        const float y0 = x[8 * g8 + 2 * j] * inv, y1 = x[8 * g8 + 2 * j + 1] * inv;
+        const __half2 h = __floats2half2_rn(y0, y1);
+        const float2 hf = __half22float2(h);
+        hv[j] = *reinterpret_cast<const uint32_t*>(&h);
+        lv[j] = pack_h2(y0 - hf.x, y1 - hf.y);
       }
+      const int off = sw128_off(r, hc + 8 * g8);
+      *reinterpret_cast<uint4*>(sm.qh + off) = make_uint4(hv[0], hv[1], hv[2], hv[3]);
+      *reinterpret_cast<uint4*>(sm.ql + off) = make_uint4(lv[0], lv[1], lv[2], lv[3]);
+    }
+  }
+  ptx::fence_proxy_async_smem();
+  ptx::tc_fence_before();
+  __syncthreads();                                        // q' complete; slots and S buffers free
+  ptx::tc_fence_after();
+
+  // ---- tiles
+  const int pos = R < n_rows ? a.q_start + R / G : -1;     // padding rows attend to nothing
+  const int last = min(pos, a.n_ctx - 1);                 // last token this row attends to
+  float m_used = -INFINITY, l = 0.0f;
+  const uint32_t qh_a = ptx::smem_u32(sm.qh), ql_a = ptx::smem_u32(sm.ql);
+  auto load_k = [&](int t) {                                // tid 0
+    const int buf = t & 1;
+    const int krow = static_cast<int>(csk * a.n_ctx_pad) + t * TILE;
+    ptx::mbar_arrive_expect_tx(&sm.bar_k[buf], kTOp);
+    ptx::tma_load_2d(sm.kt[buf], &tm, &sm.bar_k[buf], 0, krow);
+    ptx::tma_load_2d(sm.kt[buf] + kTAtom, &tm, &sm.bar_k[buf], 64, krow);
+  };
+  auto load_v = [&](int t) {                                // tid 0
+    const int buf = t & 1;
+    const int vrow = static_cast<int>(csv * a.n_ctx_pad) + t * TILE;
+    ptx::mbar_arrive_expect_tx(&sm.bar_v[buf], kTOp);
+    ptx::tma_load_2d(sm.vt[buf], &tm, &sm.bar_v[buf], 0, vrow);
+    ptx::tma_load_2d(sm.vt[buf] + kTAtom, &tm, &sm.bar_v[buf], 64, vrow);
+  };
+  auto load_alpha = [&](int t) {                            // threads 0-127: alpha^K, 128-255: alpha^V
+    const int tl = tid & (TILE - 1), tok = t * TILE + tl;
+    const size_t cs = tid < TILE ? csk : csv;
+    const float v = tok < a.n_ctx ? a.alpha[cs * a.n_tiles * TILE + tok] : 0.0f;
+    (tid < TILE ? sm.ak : sm.av)[t & 1][tl] = v;
+  };
+  auto issue_s = [&](int t) {                               // tid 0, after its key tile landed
+    const int buf = t & 1;
+    const uint32_t kt_a = ptx::smem_u32(sm.kt[buf]), d = tmem + kColS + 128 * buf;
+    ptx::tc_fence_after();
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+      const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+      ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(qh_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
+                     kk > 0 ? 1u : 0u);
     }
 #pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      const int R = rb * kPRows + 16 * warp + r;
-      if (R < n_rows) {
-        const int qi = R / G, qh2 = head * G + R % G;
-        *reinterpret_cast<float4*>(a.out + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh2) * D + 4 * lane) =
-            make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]);
+    for (int kk = 0; kk < 8; ++kk) {
+      const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+      ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(ql_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT, 1u);
+    }
+    ptx::umma_commit(&sm.bar_s[buf]);
+  };
+  if (n_kv_tiles > 0) {
+    if (tid == 0) {
+      load_k(0);
+      if (n_kv_tiles > 1) load_k(1);
+      load_v(0);
+    }
+    load_alpha(0);
+    if (tid == 0) {
+      wait(&sm.bar_k[0], 0);
+      issue_s(0);
+    }
+  }
+  __syncthreads();                                          // alpha of tile 0 visible
+  for (int t = 0; t < n_kv_tiles; ++t) {
+    const int buf = t & 1;
+    if (t + 1 < n_kv_tiles) {
+      load_alpha(t + 1);
+      if (tid == 0) {
+        wait(&sm.bar_k[buf ^ 1], ((t + 1) >> 1) & 1);
+        issue_s(t + 1);
       }
     }
+    wait(&sm.bar_s[buf], (t >> 1) & 1);
+    ptx::tc_fence_after();
+    if (tid == 0 && t + 2 < n_kv_tiles) load_k(t + 2);      // S(t) has read kt[buf]
+    // pass 1: x = S alpha^K over this thread's 64 tokens (masked), partial row maximum
+    const float* akt = sm.ak[buf] + hc;
+    const float* avt = sm.av[buf] + hc;
+    const int lim = last - t * TILE - hc;                   // tokens i <= lim are attended
+    float x[64];
+    {
+      uint32_t s0[32], s1[32];
+      ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc, s0);
+      ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc + 32, s1);
+      ptx::tmem_ld_wait();
+      ptx::tmem_regs_ready(s0);
+      ptx::tmem_regs_ready(s1);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        x[i] = __uint_as_float(s0[i]) * akt[i];
+        x[32 + i] = __uint_as_float(s1[i]) * akt[32 + i];
+      }
+    }
+    if (!__all_sync(0xffffffffu, lim >= 63)) {
+#pragma unroll
+      for (int i = 0; i < 64; ++i) x[i] = i <= lim ? x[i] : -INFINITY;
+    }
+    float mt = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 64; ++i) mt = fmaxf(mt, x[i]);
+    sm.xch[half][r] = mt;
+    __syncthreads();                                        // (A) partial maxima exchanged
+    mt = fmaxf(sm.xch[0][r], sm.xch[1][r]) * rsr;
+    const bool need = mt > m_used + kLazyLog2;
+    if (t > 0) wait(&sm.bar_o, (t - 1) & 1);                // value MMA of tile t - 1 done: O, P', vt[buf ^ 1] free
+    ptx::tc_fence_after();
+    if (tid == 0 && t + 1 < n_kv_tiles) load_v(t + 1);
+    if (__any_sync(0xffffffffu, need && t > 0)) {           // rescale this half of O
+      const float c = need ? (m_used == -INFINITY ? 0.0f : ex2(m_used - mt)) : 1.0f;
+#pragma unroll 1
+      for (int ch = 0; ch < 2; ++ch) {
+        uint32_t o[32];
+        ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32 * ch, o);
+        ptx::tmem_ld_wait();
+        ptx::tmem_regs_ready(o);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * c);
+        ptx::tmem_st32(tmem + lane_base + kColO + hc + 32 * ch, o);
+      }
+      ptx::tmem_wait_st();
+    }
+    if (need) {
+      l = m_used == -INFINITY ? 0.0f : l * ex2(m_used - mt);
+      m_used = mt;
+    }
+    // pass 2: P' = 2^(x rs - m) alpha^V, f16 pairs into TMEM
+    {
+      const float msub = m_used == -INFINITY ? 0.0f : m_used;
+      uint32_t pw[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float e0 = ex2(fmaf(x[2 * i], rsr, -msub)), e1 = ex2(fmaf(x[2 * i + 1], rsr, -msub));
+        l += e0 + e1;
+        pw[i] = pack_h2(e0 * avt[2 * i], e1 * avt[2 * i + 1]);
+      }
+      ptx::tmem_st32(tmem + lane_base + kColP + 32 * half, pw);
+      ptx::tmem_wait_st();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();                                        // (B) P' complete; alpha of t + 1 visible
+    if (tid == 0) {
+      wait(&sm.bar_v[buf], (t >> 1) & 1);
+      ptx::tc_fence_after();
+      const uint32_t vt_a = ptx::smem_u32(sm.vt[buf]);
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+        ptx::umma_f16_ta(tmem + kColO, tmem + kColP + 8 * kk, ptx::sdesc_kmajor_sw128(vt_a + off), kIdescTT,
+                         (t > 0 || kk > 0) ? 1u : 0u);
+      }
+      ptx::umma_commit(&sm.bar_o);
+    }
+  }
+  if (n_kv_tiles > 0) wait(&sm.bar_o, (n_kv_tiles - 1) & 1);
+  ptx::tc_fence_after();
+
+  // ---- o_hat = f^V O / l, hi / lo bf16 in slots 0 / 1; U_V (rows = dim, K = channel) hi / lo in
+  // slots 2 / 3; out = o_hat U_V^T = hi.hi + hi.lo + lo.hi
+  sm.xch[half][r] = l;
+  __syncthreads();
+  const float lt = sm.xch[0][r] + sm.xch[1][r];
+  {
+    const float il = lt > 0.0f ? 1.0f / lt : 0.0f;
+    uint32_t o0[32], o1[32];
+    ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc, o0);
+    ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32, o1);
+    ptx::tmem_ld_wait();
+    ptx::tmem_regs_ready(o0);
+    ptx::tmem_regs_ready(o1);
+    const float* fv = a.f + sv * D + hc;
+#pragma unroll
+    for (int g8 = 0; g8 < 8; ++g8) {
+      float u[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int i = 8 * g8 + j;
+        const float ov = __uint_as_float(i < 32 ? o0[i & 31] : o1[i & 31]);
+        u[j] = lt > 0.0f ? ov * il * fv[i] : 0.0f;
+      }
+      store_split_bf16(pj + sw128_off(r, hc + 8 * g8), u, 2);
+    }
+  }
+  {
+    const float* uv = a.u32 + static_cast<size_t>(sv) * D * D;
+    for (int g = tid; g < D * 16; g += kTThreads) {
+      const int d = g >> 4, k8 = (g & 15) * 8;
+      const float4 u0 = *reinterpret_cast<const float4*>(uv + d * D + k8);
+      const float4 u1 = *reinterpret_cast<const float4*>(uv + d * D + k8 + 4);
+      const float u[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+      store_split_bf16(pj + 2 * kTOp + sw128_off(d, k8), u, 2);
+    }
+  }
+  ptx::fence_proxy_async_smem();
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  if (tid == 0) {
+#pragma unroll 1
+    for (int pr = 0; pr < 3; ++pr) {
+      const uint32_t as = pr == 2 ? 1u : 0u, bs = pr == 1 ? 3u : 2u;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+        ptx::umma_bf16(tmem + kColS, ptx::sdesc_kmajor_sw128(pj_a + as * kTOp + off),
+                       ptx::sdesc_kmajor_sw128(pj_a + bs * kTOp + off), kIdescBB, (pr | kk) ? 1u : 0u);
+      }
+    }
+    ptx::umma_commit(&sm.bar_p);
+  }
+  wait(&sm.bar_p, 1);
+  ptx::tc_fence_after();
+  {
+    uint32_t o0[32], o1[32];
+    ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc, o0);
+    ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc + 32, o1);
+    ptx::tmem_ld_wait();
+    ptx::tmem_regs_ready(o0);
+    ptx::tmem_regs_ready(o1);
+    if (R < n_rows) {
+      const int qi = R / G, qh2 = head * G + R % G;
+      float4* dst = reinterpret_cast<float4*>(a.out + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh2) * D + hc);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        dst[i] = make_float4(__uint_as_float(o0[4 * i]), __uint_as_float(o0[4 * i + 1]), __uint_as_float(o0[4 * i + 2]),
+                             __uint_as_float(o0[4 * i + 3]));
+        dst[8 + i] = make_float4(__uint_as_float(o1[4 * i]), __uint_as_float(o1[4 * i + 1]),
+                                 __uint_as_float(o1[4 * i + 2]), __uint_as_float(o1[4 * i + 3]));
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 512);
   }
 }
 
@@ -426,20 +582,27 @@ cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_sta
   a.n_tiles = g.n_tiles;
   a.n_words = plan.n_words;
   a.n_entries = plan.n_entries;
+  a.err = plan.dev.err;
   if (plan.n_words > 32) return cudaErrorNotSupported;
   aatc_prefill_codes_kernel<<<dim3(a.n_ctx_pad / TILE, a.n_kv * 2, batch), TILE, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  // one 2D map over the whole codes workspace: rows of 128 f16 (a key token, or a value channel
+  // of a 128-token tile), box 64 x 128
+  alignas(64) unsigned char tmap[128];
+  e = make_tensor_map_2d(tmap, true, ws, D, static_cast<uint64_t>(batch) * a.n_kv * 2 * a.n_ctx_pad, D * 2, 64, TILE);
+  if (e != cudaSuccess) return e;
   static bool attr_done = false;
-  const size_t smem = sizeof(PrefillSmem);
+  const size_t smem = sizeof(PrefillTcSmem) + 1024;
   if (!attr_done) {
-    e = cudaFuncSetAttribute(aatc_prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(aatc_prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
   const int n_rows = n_q * a.group;
-  aatc_prefill_attn_kernel<<<dim3((n_rows + kPRows - 1) / kPRows, a.n_kv, batch), kPThreads, smem, st>>>(a);
+  aatc_prefill_tc_kernel<<<dim3((n_rows + kTRows - 1) / kTRows, a.n_kv, batch), kTThreads, smem, st>>>(
+      *reinterpret_cast<const CUtensorMap*>(tmap), a);
   return cudaGetLastError();
 }
 
