@@ -122,21 +122,25 @@ __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
 }
 
 // ---------------------------------------------------------------- tensor-core (tcgen05) attention
-// Per CTA 128 query rows (= TMEM lanes) of one (kv-head, sequence); 8 warps, warp w owns TMEM
-// lanes 32 (w & 3) .. + 31 and the column half w >> 2 of every 128-column TMEM block.
+// Per CTA 128 query rows (= TMEM lanes) of one (kv-head, sequence).  Warps 0-7 do the softmax:
+// warp w owns TMEM lanes 32 (w & 3) .. + 31 and the column half w >> 2 of every 128-column TMEM
+// block.  Warp 8 is the control warp: one thread issues every TMA copy and tensor-core MMA and
+// talks to the softmax warps through mbarriers only.
 //   prologue  q' = (q U_K) f^K log2(e) / sqrt(128) on the tensor cores: q (bf16, exact) against
 //             U_K split into three bf16 parts (about 2^-25 relative), rows scaled to 2^14 and
 //             split into f16 hi / lo operands
 //   per 128-token tile (TMA, 128-byte swizzle, key and value tiles double-buffered):
-//             S = q'_hi . code_K + q'_lo . code_K   tcgen05.mma M = N = 128, K = 128; S of tile
-//             t + 1 is issued before the softmax of tile t (two S buffers in TMEM)
+//             S = q'_hi . code_K + q'_lo . code_K   tcgen05.mma M = N = 128, K = 128, two S
+//             buffers in TMEM: S of tile t + 1 is computed during the softmax of tile t
 //             softmax from TMEM with the scores held in registers between the maximum and the
 //             exponent: s = S rs alpha^K (causal mask), lazy maximum (O rescaled only when a
 //             row's maximum grows by more than 2^8, so P' = 2^(s - m) alpha^V stays inside f16)
 //             P' stored to TMEM as f16 pairs: the A operand of O += P' . code_V^T
 //   epilogue  out = (f^V O / l) U_V^T on the tensor cores, both operands split hi / lo in bf16.
 constexpr int kTRows = 128;
-constexpr int kTThreads = 256;
+constexpr int kTSoftmax = 256;                     // softmax threads (warps 0-7)
+constexpr int kTThreads = kTSoftmax + 32;          // + the control warp
+constexpr int kTCtl = kTSoftmax;                   // the thread that issues copies and MMAs
 constexpr int kTAtom = 128 * 128;                  // one 128-row K-atom (64 16-bit values per row)
 constexpr int kTOp = 2 * kTAtom;                   // one 128 x 128 16-bit operand (two K-atoms)
 constexpr float kLazyLog2 = 8.0f;
@@ -151,9 +155,9 @@ struct PrefillTcSmem {
   alignas(1024) unsigned char ql[kTOp];            // q' lo
   alignas(1024) unsigned char kt[2][kTOp];         // key codes: K-atoms = channels, rows = tokens
   alignas(1024) unsigned char vt[2][kTOp];         // value codes: K-atoms = tokens 0-63 | 64-127, rows = channels
-  float ak[2][TILE], av[2][TILE];
-  float xch[2][kTRows];                            // per-row partials of the two column halves
-  uint64_t bar_k[2], bar_v[2], bar_s[2], bar_o, bar_p;
+  float al[3][2][TILE];                            // alpha^K, alpha^V of three tiles
+  float xch[2][2][kTRows];                         // per-row partials of the two column halves (two slots)
+  uint64_t bar_k[2], bar_v[2], bar_s[2], sfree[2], vfree[2], bar_o, pready, bar_p;
   uint32_t tmem;
   int abort_flag;
 };
@@ -189,6 +193,9 @@ __device__ __forceinline__ void store_split_bf16(unsigned char* dst, const float
     if (p < parts) *reinterpret_cast<uint4*>(dst + p * kTOp) = make_uint4(w[p][0], w[p][1], w[p][2], w[p][3]);
 }
 
+// barrier among the softmax warps only
+__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kTSoftmax) : "memory"); }
+
 __global__ void __launch_bounds__(kTThreads, 1)
     aatc_prefill_tc_kernel(const __grid_constant__ CUtensorMap tm, const PrefillArgs a) {
   extern __shared__ unsigned char smraw[];
@@ -196,6 +203,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
       *reinterpret_cast<PrefillTcSmem*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
   const int rb = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool softmax = tid < kTSoftmax;
   const int G = a.group, n_rows = a.n_q * G;
   const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;
   const size_t csk = (static_cast<size_t>(b) * a.n_kv + head) * 2, csv = csk + 1;
@@ -203,7 +211,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   const int r_last = min(n_rows - 1, R0 + kTRows - 1) - R0;
   const int kv_end = min(a.n_ctx, a.q_start + (R0 + r_last) / G + 1);
   const int n_kv_tiles = (kv_end + TILE - 1) / TILE;
-  const int r = 32 * (warp & 3) + lane, half = warp >> 2, hc = 64 * half;
+  const int r = 32 * (warp & 3) + lane, half = (warp >> 2) & 1, hc = 64 * half;
   const uint32_t lane_base = static_cast<uint32_t>(32 * (warp & 3)) << 16;
   const int R = R0 + r;
   unsigned char* const pj = sm.kt[0];              // projection operand i at pj + i * kTOp
@@ -215,14 +223,16 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
   };
 
-  if (tid == 0) {
-    ptx::mbar_init(&sm.bar_k[0], 1);
-    ptx::mbar_init(&sm.bar_k[1], 1);
-    ptx::mbar_init(&sm.bar_v[0], 1);
-    ptx::mbar_init(&sm.bar_v[1], 1);
-    ptx::mbar_init(&sm.bar_s[0], 1);
-    ptx::mbar_init(&sm.bar_s[1], 1);
+  if (tid == kTCtl) {
+    for (int i = 0; i < 2; ++i) {
+      ptx::mbar_init(&sm.bar_k[i], 1);
+      ptx::mbar_init(&sm.bar_v[i], 1);
+      ptx::mbar_init(&sm.bar_s[i], 1);
+      ptx::mbar_init(&sm.sfree[i], kTSoftmax / 32);
+      ptx::mbar_init(&sm.vfree[i], 1);
+    }
     ptx::mbar_init(&sm.bar_o, 1);
+    ptx::mbar_init(&sm.pready, kTSoftmax / 32);
     ptx::mbar_init(&sm.bar_p, 1);
     sm.abort_flag = 0;
     ptx::fence_mbar_init();
@@ -234,18 +244,19 @@ __global__ void __launch_bounds__(kTThreads, 1)
   }
   // ---- projection operands: q rows (bf16) in slot 0, U_K^T (rows = channel, K = dim) in three
   // bf16 parts in slots 1-3
-  for (int g = tid; g < kTRows * 16; g += kTThreads) {
-    const int row = g >> 4, k8 = (g & 15) * 8, RR = R0 + row;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (RR < n_rows) {
-      const int qi = RR / G, qh = head * G + RR % G;
-      v = *reinterpret_cast<const uint4*>(a.q + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh) * D + k8);
+  if (softmax) {
+    for (int g = tid; g < kTRows * 16; g += kTSoftmax) {
+      const int row = g >> 4, k8 = (g & 15) * 8, RR = R0 + row;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (RR < n_rows) {
+        const int qi = RR / G, qh = head * G + RR % G;
+        v = *reinterpret_cast<const uint4*>(a.q + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh) * D +
+                                            k8);
+      }
+      *reinterpret_cast<uint4*>(pj + sw128_off(row, k8)) = v;
     }
-    *reinterpret_cast<uint4*>(pj + sw128_off(row, k8)) = v;
-  }
-  {
     const float* ukt = a.u32t + static_cast<size_t>(sk) * D * D;
-    for (int g = tid; g < D * 16; g += kTThreads) {
+    for (int g = tid; g < D * 16; g += kTSoftmax) {
       const int c = g >> 4, k8 = (g & 15) * 8;
       const float4 u0 = *reinterpret_cast<const float4*>(ukt + c * D + k8);
       const float4 u1 = *reinterpret_cast<const float4*>(ukt + c * D + k8 + 4);
@@ -259,7 +270,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
   ptx::tc_fence_after();
   const uint32_t tmem = sm.tmem;
   const uint32_t pj_a = ptx::smem_u32(pj);
-  if (tid == 0) {
+  if (tid == kTCtl) {
 #pragma unroll 1
     for (int part = 0; part < 3; ++part)
 #pragma unroll
@@ -270,12 +281,11 @@ __global__ void __launch_bounds__(kTThreads, 1)
       }
     ptx::umma_commit(&sm.bar_p);
   }
-  wait(&sm.bar_p, 0);
-  ptx::tc_fence_after();
-
   // ---- q' rows scaled to 2^14, f16 hi / lo into the score operands
-  float rsr;
-  {
+  float rsr = 1.0f;
+  if (softmax) {
+    wait(&sm.bar_p, 0);
+    ptx::tc_fence_after();
     uint32_t q0[32], q1[32];
     ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc, q0);
     ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc + 32, q1);
@@ -292,9 +302,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
       x[32 + i] = __uint_as_float(q1[i]) * fk[32 + i] * sc;
       m = fmaxf(m, fmaxf(fabsf(x[i]), fabsf(x[32 + i])));
     }
-    sm.xch[half][r] = m;
-    __syncthreads();
-    m = fmaxf(sm.xch[0][r], sm.xch[1][r]);
+    sm.xch[0][half][r] = m;
+    softmax_sync();
+    m = fmaxf(sm.xch[0][0][r], sm.xch[0][1][r]);
     const float inv = m > 0.0f ? kPOpMax / m : 0.0f;
     rsr = m > 0.0f ? m / kPOpMax : 1.0f;             // > 0, so the mask's -inf survives the scaling
 #pragma unroll
@@ -313,188 +323,207 @@ __global__ void __launch_bounds__(kTThreads, 1)
       *reinterpret_cast<uint4*>(sm.ql + off) = make_uint4(lv[0], lv[1], lv[2], lv[3]);
     }
   }
-  ptx::fence_proxy_async_smem();
-  ptx::tc_fence_before();
-  __syncthreads();                                        // q' complete; slots and S buffers free
-  ptx::tc_fence_after();
-
-  // ---- tiles
-  const int pos = R < n_rows ? a.q_start + R / G : -1;     // padding rows attend to nothing
-  const int last = min(pos, a.n_ctx - 1);                 // last token this row attends to
-  float m_used = -INFINITY, l = 0.0f;
-  const uint32_t qh_a = ptx::smem_u32(sm.qh), ql_a = ptx::smem_u32(sm.ql);
-  auto load_k = [&](int t) {                                // tid 0
-    const int buf = t & 1;
-    const int krow = static_cast<int>(csk * a.n_ctx_pad) + t * TILE;
-    ptx::mbar_arrive_expect_tx(&sm.bar_k[buf], kTOp);
-    ptx::tma_load_2d(sm.kt[buf], &tm, &sm.bar_k[buf], 0, krow);
-    ptx::tma_load_2d(sm.kt[buf] + kTAtom, &tm, &sm.bar_k[buf], 64, krow);
-  };
-  auto load_v = [&](int t) {                                // tid 0
-    const int buf = t & 1;
-    const int vrow = static_cast<int>(csv * a.n_ctx_pad) + t * TILE;
-    ptx::mbar_arrive_expect_tx(&sm.bar_v[buf], kTOp);
-    ptx::tma_load_2d(sm.vt[buf], &tm, &sm.bar_v[buf], 0, vrow);
-    ptx::tma_load_2d(sm.vt[buf] + kTAtom, &tm, &sm.bar_v[buf], 64, vrow);
-  };
-  auto load_alpha = [&](int t) {                            // threads 0-127: alpha^K, 128-255: alpha^V
+  // alpha^K / alpha^V of one tile: thread tid < 256 owns entry tid (K for tid < 128)
+  auto alpha_of = [&](int t) -> float {
     const int tl = tid & (TILE - 1), tok = t * TILE + tl;
     const size_t cs = tid < TILE ? csk : csv;
-    const float v = tok < a.n_ctx ? a.alpha[cs * a.n_tiles * TILE + tok] : 0.0f;
-    (tid < TILE ? sm.ak : sm.av)[t & 1][tl] = v;
+    return tok < a.n_ctx ? a.alpha[cs * a.n_tiles * TILE + tok] : 0.0f;
   };
-  auto issue_s = [&](int t) {                               // tid 0, after its key tile landed
-    const int buf = t & 1;
-    const uint32_t kt_a = ptx::smem_u32(sm.kt[buf]), d = tmem + kColS + 128 * buf;
-    ptx::tc_fence_after();
-#pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-      const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-      ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(qh_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
-                     kk > 0 ? 1u : 0u);
-    }
-#pragma unroll
-    for (int kk = 0; kk < 8; ++kk) {
-      const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-      ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(ql_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT, 1u);
-    }
-    ptx::umma_commit(&sm.bar_s[buf]);
-  };
-  if (n_kv_tiles > 0) {
-    if (tid == 0) {
-      load_k(0);
-      if (n_kv_tiles > 1) load_k(1);
-      load_v(0);
-    }
-    load_alpha(0);
-    if (tid == 0) {
-      wait(&sm.bar_k[0], 0);
-      issue_s(0);
-    }
+  float a_next = 0.0f;
+  if (softmax && n_kv_tiles > 0) {
+    sm.al[0][tid >> 7][tid & (TILE - 1)] = alpha_of(0);
+    if (n_kv_tiles > 1) a_next = alpha_of(1);
   }
-  __syncthreads();                                          // alpha of tile 0 visible
-  for (int t = 0; t < n_kv_tiles; ++t) {
-    const int buf = t & 1;
-    if (t + 1 < n_kv_tiles) {
-      load_alpha(t + 1);
-      if (tid == 0) {
-        wait(&sm.bar_k[buf ^ 1], ((t + 1) >> 1) & 1);
-        issue_s(t + 1);
-      }
-    }
-    wait(&sm.bar_s[buf], (t >> 1) & 1);
-    ptx::tc_fence_after();
-    if (tid == 0 && t + 2 < n_kv_tiles) load_k(t + 2);      // S(t) has read kt[buf]
-    // pass 1: x = S alpha^K over this thread's 64 tokens (masked), partial row maximum
-    const float* akt = sm.ak[buf] + hc;
-    const float* avt = sm.av[buf] + hc;
-    const int lim = last - t * TILE - hc;                   // tokens i <= lim are attended
-    float x[64];
-    {
-      uint32_t s0[32], s1[32];
-      ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc, s0);
-      ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc + 32, s1);
-      ptx::tmem_ld_wait();
-      ptx::tmem_regs_ready(s0);
-      ptx::tmem_regs_ready(s1);
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        x[i] = __uint_as_float(s0[i]) * akt[i];
-        x[32 + i] = __uint_as_float(s1[i]) * akt[32 + i];
-      }
-    }
-    if (!__all_sync(0xffffffffu, lim >= 63)) {
-#pragma unroll
-      for (int i = 0; i < 64; ++i) x[i] = i <= lim ? x[i] : -INFINITY;
-    }
-    float mt = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 64; ++i) mt = fmaxf(mt, x[i]);
-    sm.xch[half][r] = mt;
-    __syncthreads();                                        // (A) partial maxima exchanged
-    mt = fmaxf(sm.xch[0][r], sm.xch[1][r]) * rsr;
-    const bool need = mt > m_used + kLazyLog2;
-    if (t > 0) wait(&sm.bar_o, (t - 1) & 1);                // value MMA of tile t - 1 done: O, P', vt[buf ^ 1] free
-    ptx::tc_fence_after();
-    if (tid == 0 && t + 1 < n_kv_tiles) load_v(t + 1);
-    if (__any_sync(0xffffffffu, need && t > 0)) {           // rescale this half of O
-      const float c = need ? (m_used == -INFINITY ? 0.0f : ex2(m_used - mt)) : 1.0f;
-#pragma unroll 1
-      for (int ch = 0; ch < 2; ++ch) {
-        uint32_t o[32];
-        ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32 * ch, o);
-        ptx::tmem_ld_wait();
-        ptx::tmem_regs_ready(o);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * c);
-        ptx::tmem_st32(tmem + lane_base + kColO + hc + 32 * ch, o);
-      }
-      ptx::tmem_wait_st();
-    }
-    if (need) {
-      l = m_used == -INFINITY ? 0.0f : l * ex2(m_used - mt);
-      m_used = mt;
-    }
-    // pass 2: P' = 2^(x rs - m) alpha^V, f16 pairs into TMEM
-    {
-      const float msub = m_used == -INFINITY ? 0.0f : m_used;
-      uint32_t pw[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float e0 = ex2(fmaf(x[2 * i], rsr, -msub)), e1 = ex2(fmaf(x[2 * i + 1], rsr, -msub));
-        l += e0 + e1;
-        pw[i] = pack_h2(e0 * avt[2 * i], e1 * avt[2 * i + 1]);
-      }
-      ptx::tmem_st32(tmem + lane_base + kColP + 32 * half, pw);
-      ptx::tmem_wait_st();
-    }
-    ptx::tc_fence_before();
-    __syncthreads();                                        // (B) P' complete; alpha of t + 1 visible
-    if (tid == 0) {
-      wait(&sm.bar_v[buf], (t >> 1) & 1);
-      ptx::tc_fence_after();
-      const uint32_t vt_a = ptx::smem_u32(sm.vt[buf]);
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-        ptx::umma_f16_ta(tmem + kColO, tmem + kColP + 8 * kk, ptx::sdesc_kmajor_sw128(vt_a + off), kIdescTT,
-                         (t > 0 || kk > 0) ? 1u : 0u);
-      }
-      ptx::umma_commit(&sm.bar_o);
-    }
-  }
-  if (n_kv_tiles > 0) wait(&sm.bar_o, (n_kv_tiles - 1) & 1);
+  ptx::fence_proxy_async_smem();
+  ptx::tc_fence_before();
+  __syncthreads();                                        // q' and alpha of tile 0 complete; slots, S free
   ptx::tc_fence_after();
 
-  // ---- o_hat = f^V O / l, hi / lo bf16 in slots 0 / 1; U_V (rows = dim, K = channel) hi / lo in
-  // slots 2 / 3; out = o_hat U_V^T = hi.hi + hi.lo + lo.hi
-  sm.xch[half][r] = l;
-  __syncthreads();
-  const float lt = sm.xch[0][r] + sm.xch[1][r];
-  {
-    const float il = lt > 0.0f ? 1.0f / lt : 0.0f;
-    uint32_t o0[32], o1[32];
-    ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc, o0);
-    ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32, o1);
-    ptx::tmem_ld_wait();
-    ptx::tmem_regs_ready(o0);
-    ptx::tmem_regs_ready(o1);
-    const float* fv = a.f + sv * D + hc;
+  if (!softmax) {
+    // ---- control thread: TMA copies and MMAs.  Every wait below is on a phase that cannot be
+    // overtaken: the next arrival on that barrier needs an action this thread takes later.
+    if (lane == 0 && n_kv_tiles > 0) {
+      const uint32_t qh_a = ptx::smem_u32(sm.qh), ql_a = ptx::smem_u32(sm.ql);
+      auto load_k = [&](int t) {
+        const int buf = t & 1;
+        const int krow = static_cast<int>(csk * a.n_ctx_pad) + t * TILE;
+        ptx::mbar_arrive_expect_tx(&sm.bar_k[buf], kTOp);
+        ptx::tma_load_2d(sm.kt[buf], &tm, &sm.bar_k[buf], 0, krow);
+        ptx::tma_load_2d(sm.kt[buf] + kTAtom, &tm, &sm.bar_k[buf], 64, krow);
+      };
+      auto load_v = [&](int t) {
+        const int buf = t & 1;
+        const int vrow = static_cast<int>(csv * a.n_ctx_pad) + t * TILE;
+        ptx::mbar_arrive_expect_tx(&sm.bar_v[buf], kTOp);
+        ptx::tma_load_2d(sm.vt[buf], &tm, &sm.bar_v[buf], 0, vrow);
+        ptx::tma_load_2d(sm.vt[buf] + kTAtom, &tm, &sm.bar_v[buf], 64, vrow);
+      };
+      auto issue_s = [&](int t) {
+        const int buf = t & 1;
+        const uint32_t kt_a = ptx::smem_u32(sm.kt[buf]), d = tmem + kColS + 128 * buf;
+        ptx::tc_fence_after();
 #pragma unroll
-    for (int g8 = 0; g8 < 8; ++g8) {
-      float u[8];
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+          ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(qh_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
+                         kk > 0 ? 1u : 0u);
+        }
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int i = 8 * g8 + j;
-        const float ov = __uint_as_float(i < 32 ? o0[i & 31] : o1[i & 31]);
-        u[j] = lt > 0.0f ? ov * il * fv[i] : 0.0f;
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+          ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(ql_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT, 1u);
+        }
+        ptx::umma_commit(&sm.bar_s[buf]);
+      };
+      load_k(0);
+      load_v(0);
+      if (n_kv_tiles > 1) {
+        load_k(1);
+        load_v(1);
       }
-      store_split_bf16(pj + sw128_off(r, hc + 8 * g8), u, 2);
+      wait(&sm.bar_k[0], 0);
+      issue_s(0);
+      for (int t = 0; t < n_kv_tiles; ++t) {
+        const int buf = t & 1;
+        if (t + 2 < n_kv_tiles) {                       // S(t) has read kt[buf]
+          wait(&sm.bar_s[buf], (t >> 1) & 1);
+          load_k(t + 2);
+        }
+        if (t + 1 < n_kv_tiles) {
+          if (t >= 1) wait(&sm.sfree[buf ^ 1], ((t - 1) >> 1) & 1);   // S(t - 1) read out
+          wait(&sm.bar_k[buf ^ 1], ((t + 1) >> 1) & 1);
+          issue_s(t + 1);
+          if (t >= 1) {                                 // PV(t - 1) has read vt[buf ^ 1]
+            wait(&sm.vfree[buf ^ 1], ((t - 1) >> 1) & 1);
+            load_v(t + 1);
+          }
+        }
+        wait(&sm.pready, t & 1);
+        wait(&sm.bar_v[buf], (t >> 1) & 1);
+        ptx::tc_fence_after();
+        const uint32_t vt_a = ptx::smem_u32(sm.vt[buf]);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
+          ptx::umma_f16_ta(tmem + kColO, tmem + kColP + 8 * kk, ptx::sdesc_kmajor_sw128(vt_a + off), kIdescTT,
+                           (t > 0 || kk > 0) ? 1u : 0u);
+        }
+        ptx::umma_commit(&sm.bar_o);
+        ptx::umma_commit(&sm.vfree[buf]);
+      }
     }
-  }
-  {
+    __syncwarp();                                         // the control warp reconverges
+  } else {
+    // ---- softmax warps
+    const int pos = R < n_rows ? a.q_start + R / G : -1;   // padding rows attend to nothing
+    const int last = min(pos, a.n_ctx - 1);               // last token this row attends to
+    float m_used = -INFINITY, l = 0.0f;
+    for (int t = 0; t < n_kv_tiles; ++t) {
+      const int buf = t & 1;
+      // alpha one tile ahead: store tile t + 1 (fetched last iteration), fetch tile t + 2
+      if (t + 1 < n_kv_tiles) sm.al[(t + 1) % 3][tid >> 7][tid & (TILE - 1)] = a_next;
+      if (t + 2 < n_kv_tiles) a_next = alpha_of(t + 2);
+      const float* akt = sm.al[t % 3][0] + hc;
+      const float* avt = sm.al[t % 3][1] + hc;
+      wait(&sm.bar_s[buf], (t >> 1) & 1);
+      ptx::tc_fence_after();
+      // pass 1: x = S alpha^K over this thread's 64 tokens (masked), partial row maximum
+      const int lim = last - t * TILE - hc;                 // tokens i <= lim are attended
+      float x[64];
+      {
+        uint32_t s0[32], s1[32];
+        ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc, s0);
+        ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc + 32, s1);
+        ptx::tmem_ld_wait();
+        ptx::tmem_regs_ready(s0);
+        ptx::tmem_regs_ready(s1);
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&sm.sfree[buf]);    // this warp's part of S(t) read out
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          x[i] = __uint_as_float(s0[i]) * akt[i];
+          x[32 + i] = __uint_as_float(s1[i]) * akt[32 + i];
+        }
+      }
+      const bool full = __all_sync(0xffffffffu, lim >= 63);
+      if (!full) {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] = i <= lim ? x[i] : -INFINITY;
+      }
+      float mt = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 64; ++i) mt = fmaxf(mt, x[i]);
+      sm.xch[buf][half][r] = mt;
+      softmax_sync();                                       // partial maxima exchanged
+      mt = fmaxf(sm.xch[buf][0][r], sm.xch[buf][1][r]) * rsr;
+      const bool need = mt > m_used + kLazyLog2;
+      if (t > 0) wait(&sm.bar_o, (t - 1) & 1);              // PV(t - 1) done: O and P' free
+      ptx::tc_fence_after();
+      if (__any_sync(0xffffffffu, need && t > 0)) {         // rescale this half of O
+        const float c = need ? (m_used == -INFINITY ? 0.0f : ex2(m_used - mt)) : 1.0f;
+#pragma unroll 1
+        for (int ch = 0; ch < 2; ++ch) {
+          uint32_t o[32];
+          ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32 * ch, o);
+          ptx::tmem_ld_wait();
+          ptx::tmem_regs_ready(o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * c);
+          ptx::tmem_st32(tmem + lane_base + kColO + hc + 32 * ch, o);
+        }
+      }
+      if (need) {
+        l = m_used == -INFINITY ? 0.0f : l * ex2(m_used - mt);
+        m_used = mt;
+      }
+      // pass 2: P' = 2^(x rs - m) alpha^V, f16 pairs into TMEM (masked tokens: 0, whatever alpha^V)
+      {
+        const float msub = m_used == -INFINITY ? 0.0f : m_used;
+        uint32_t pw[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float e0 = ex2(fmaf(x[2 * i], rsr, -msub)), e1 = ex2(fmaf(x[2 * i + 1], rsr, -msub));
+          l += e0 + e1;
+          pw[i] = pack_h2(e0 * avt[2 * i], e1 * avt[2 * i + 1]);
+        }
+        ptx::tmem_st32(tmem + lane_base + kColP + 32 * half, pw);
+      }
+      ptx::tmem_wait_st();
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&sm.pready);
+    }
+    if (n_kv_tiles > 0) wait(&sm.bar_o, (n_kv_tiles - 1) & 1);
+    ptx::tc_fence_after();
+    // ---- o_hat = f^V O / l, hi / lo bf16 in slots 0 / 1; U_V (rows = dim, K = channel) hi / lo
+    // in slots 2 / 3
+    sm.xch[0][half][r] = l;                               // slot 0 of the exchange is idle here
+    softmax_sync();
+    const float lt = sm.xch[0][0][r] + sm.xch[0][1][r];
+    {
+      const float il = lt > 0.0f ? 1.0f / lt : 0.0f;
+      uint32_t o0[32], o1[32];
+      ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc, o0);
+      ptx::tmem_ld_32raw(tmem + lane_base + kColO + hc + 32, o1);
+      ptx::tmem_ld_wait();
+      ptx::tmem_regs_ready(o0);
+      ptx::tmem_regs_ready(o1);
+      const float* fv = a.f + sv * D + hc;
+#pragma unroll
+      for (int g8 = 0; g8 < 8; ++g8) {
+        float u[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int i = 8 * g8 + j;
+          const float ov = __uint_as_float(i < 32 ? o0[i & 31] : o1[i & 31]);
+          u[j] = lt > 0.0f ? ov * il * fv[i] : 0.0f;
+        }
+        store_split_bf16(pj + sw128_off(r, hc + 8 * g8), u, 2);
+      }
+    }
     const float* uv = a.u32 + static_cast<size_t>(sv) * D * D;
-    for (int g = tid; g < D * 16; g += kTThreads) {
+    for (int g = tid; g < D * 16; g += kTSoftmax) {
       const int d = g >> 4, k8 = (g & 15) * 8;
       const float4 u0 = *reinterpret_cast<const float4*>(uv + d * D + k8);
       const float4 u1 = *reinterpret_cast<const float4*>(uv + d * D + k8 + 4);
@@ -506,7 +535,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
-  if (tid == 0) {
+  // ---- out = o_hat U_V^T = hi.hi + hi.lo + lo.hi
+  if (tid == kTCtl) {
 #pragma unroll 1
     for (int pr = 0; pr < 3; ++pr) {
       const uint32_t as = pr == 2 ? 1u : 0u, bs = pr == 1 ? 3u : 2u;
@@ -519,9 +549,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
     }
     ptx::umma_commit(&sm.bar_p);
   }
-  wait(&sm.bar_p, 1);
-  ptx::tc_fence_after();
-  {
+  if (softmax) {
+    wait(&sm.bar_p, 1);
+    ptx::tc_fence_after();
     uint32_t o0[32], o1[32];
     ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc, o0);
     ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc + 32, o1);
@@ -530,7 +560,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
     ptx::tmem_regs_ready(o1);
     if (R < n_rows) {
       const int qi = R / G, qh2 = head * G + R % G;
-      float4* dst = reinterpret_cast<float4*>(a.out + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh2) * D + hc);
+      float4* dst =
+          reinterpret_cast<float4*>(a.out + ((static_cast<size_t>(b) * a.n_q + qi) * a.n_q_heads + qh2) * D + hc);
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         dst[i] = make_float4(__uint_as_float(o0[4 * i]), __uint_as_float(o0[4 * i + 1]), __uint_as_float(o0[4 * i + 2]),
