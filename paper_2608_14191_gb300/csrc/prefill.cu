@@ -148,7 +148,7 @@ constexpr uint32_t kIdescTT = ptx::idesc_f16_f32(128, 128);
 constexpr uint32_t kIdescBB = ptx::idesc_bf16_f32(128, 128);
 constexpr uint32_t kColS = 0;                      // two score buffers (0, 128); projection results
 constexpr uint32_t kColO = 256;                    // O accumulator
-constexpr uint32_t kColP = 384;                    // P' (64 columns of f16 pairs)
+constexpr uint32_t kColP = 384;                    // two P' buffers (384, 448): 64 columns of f16 pairs
 
 struct PrefillTcSmem {
   alignas(1024) unsigned char qh[kTOp];            // q' hi: K-atoms = channels 0-63 | 64-127, rows = query rows
@@ -157,7 +157,7 @@ struct PrefillTcSmem {
   alignas(1024) unsigned char vt[2][kTOp];         // value codes: K-atoms = tokens 0-63 | 64-127, rows = channels
   float al[3][2][TILE];                            // alpha^K, alpha^V of three tiles
   float xch[2][2][kTRows];                         // per-row partials of the two column halves (two slots)
-  uint64_t bar_k[2], bar_v[2], bar_s[2], sfree[2], vfree[2], bar_o, pready, bar_p;
+  uint64_t bar_k[2], bar_v[2], bar_s[2], sfree[2], ofree[2], pready, bar_p;
   uint32_t tmem;
   int abort_flag;
 };
@@ -201,7 +201,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
   extern __shared__ unsigned char smraw[];
   PrefillTcSmem& sm =
       *reinterpret_cast<PrefillTcSmem*>((reinterpret_cast<uintptr_t>(smraw) + 1023) & ~uintptr_t(1023));
-  const int rb = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
+  // row blocks in reverse: the longest causal ranges start first, the shortest fill the tail
+  const int rb = gridDim.x - 1 - blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool softmax = tid < kTSoftmax;
   const int G = a.group, n_rows = a.n_q * G;
@@ -229,9 +230,8 @@ __global__ void __launch_bounds__(kTThreads, 1)
       ptx::mbar_init(&sm.bar_v[i], 1);
       ptx::mbar_init(&sm.bar_s[i], 1);
       ptx::mbar_init(&sm.sfree[i], kTSoftmax / 32);
-      ptx::mbar_init(&sm.vfree[i], 1);
+      ptx::mbar_init(&sm.ofree[i], 1);          // PV of tiles i, i + 2, ... done
     }
-    ptx::mbar_init(&sm.bar_o, 1);
     ptx::mbar_init(&sm.pready, kTSoftmax / 32);
     ptx::mbar_init(&sm.bar_p, 1);
     sm.abort_flag = 0;
@@ -394,7 +394,7 @@ __global__ void __launch_bounds__(kTThreads, 1)
           wait(&sm.bar_k[buf ^ 1], ((t + 1) >> 1) & 1);
           issue_s(t + 1);
           if (t >= 1) {                                 // PV(t - 1) has read vt[buf ^ 1]
-            wait(&sm.vfree[buf ^ 1], ((t - 1) >> 1) & 1);
+            wait(&sm.ofree[buf ^ 1], ((t - 1) >> 1) & 1);
             load_v(t + 1);
           }
         }
@@ -405,11 +405,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-          ptx::umma_f16_ta(tmem + kColO, tmem + kColP + 8 * kk, ptx::sdesc_kmajor_sw128(vt_a + off), kIdescTT,
-                           (t > 0 || kk > 0) ? 1u : 0u);
+          ptx::umma_f16_ta(tmem + kColO, tmem + kColP + 64 * buf + 8 * kk, ptx::sdesc_kmajor_sw128(vt_a + off),
+                           kIdescTT, (t > 0 || kk > 0) ? 1u : 0u);
         }
-        ptx::umma_commit(&sm.bar_o);
-        ptx::umma_commit(&sm.vfree[buf]);
+        ptx::umma_commit(&sm.ofree[buf]);
       }
     }
     __syncwarp();                                         // the control warp reconverges
@@ -458,9 +457,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
       softmax_sync();                                       // partial maxima exchanged
       mt = fmaxf(sm.xch[buf][0][r], sm.xch[buf][1][r]) * rsr;
       const bool need = mt > m_used + kLazyLog2;
-      if (t > 0) wait(&sm.bar_o, (t - 1) & 1);              // PV(t - 1) done: O and P' free
-      ptx::tc_fence_after();
-      if (__any_sync(0xffffffffu, need && t > 0)) {         // rescale this half of O
+      if (__any_sync(0xffffffffu, need && t > 0)) {         // rescale this half of O once PV(t - 1) is done
+        wait(&sm.ofree[buf ^ 1], ((t - 1) >> 1) & 1);
+        ptx::tc_fence_after();
         const float c = need ? (m_used == -INFINITY ? 0.0f : ex2(m_used - mt)) : 1.0f;
 #pragma unroll 1
         for (int ch = 0; ch < 2; ++ch) {
@@ -477,7 +476,11 @@ __global__ void __launch_bounds__(kTThreads, 1)
         l = m_used == -INFINITY ? 0.0f : l * ex2(m_used - mt);
         m_used = mt;
       }
-      // pass 2: P' = 2^(x rs - m) alpha^V, f16 pairs into TMEM (masked tokens: 0, whatever alpha^V)
+      // pass 2: P' = 2^(x rs - m) alpha^V, f16 pairs into P' buffer `buf` once PV(t - 2) has read it
+      if (t >= 2) {
+        wait(&sm.ofree[buf], ((t - 2) >> 1) & 1);
+        ptx::tc_fence_after();
+      }
       {
         const float msub = m_used == -INFINITY ? 0.0f : m_used;
         uint32_t pw[32];
@@ -487,18 +490,19 @@ __global__ void __launch_bounds__(kTThreads, 1)
           l += e0 + e1;
           pw[i] = pack_h2(e0 * avt[2 * i], e1 * avt[2 * i + 1]);
         }
-        ptx::tmem_st32(tmem + lane_base + kColP + 32 * half, pw);
+        ptx::tmem_st32(tmem + lane_base + kColP + 64 * buf + 32 * half, pw);
       }
       ptx::tmem_wait_st();
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(&sm.pready);
     }
-    if (n_kv_tiles > 0) wait(&sm.bar_o, (n_kv_tiles - 1) & 1);
+    if (n_kv_tiles > 0) wait(&sm.ofree[(n_kv_tiles - 1) & 1], ((n_kv_tiles - 1) >> 1) & 1);
     ptx::tc_fence_after();
     // ---- o_hat = f^V O / l, hi / lo bf16 in slots 0 / 1; U_V (rows = dim, K = channel) hi / lo
     // in slots 2 / 3
-    sm.xch[0][half][r] = l;                               // slot 0 of the exchange is idle here
+    softmax_sync();                                       // every warp is past its last maximum exchange
+    sm.xch[0][half][r] = l;
     softmax_sync();
     const float lt = sm.xch[0][0][r] + sm.xch[0][1][r];
     {
