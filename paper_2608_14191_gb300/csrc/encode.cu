@@ -81,17 +81,6 @@ struct RecordWriter {
   }
 };
 
-// Append the nb low bits of v (nb <= 8, uniform across the warp) to the record bit stream.
-__device__ __forceinline__ void append_bits(uint32_t v, int nb, uint32_t& word, int& pos, int& wi,
-                                            const RecordWriter& out) {
-  word |= v << pos;
-  if (pos + nb >= 32) {
-    out.put(wi, word);
-    ++wi;
-    word = pos + nb > 32 ? (v >> (32 - pos)) : 0u;
-  }
-  pos = (pos + nb) & 31;
-}
 
 // Token scale and stored values of one token (thread = token = TMEM lane): alpha = max over
 // retained channels of |h_c| / s_c (inv_s = 0 for dropped ones), then u_c = clamp(floor(h_c /
@@ -165,28 +154,66 @@ __device__ __forceinline__ float quantize_token(uint32_t taddr, const ChanEnc* e
   return amax;
 }
 
+// 16 base-4 digits (bits sh, sh + 1 of the bytes of channels 4q .. 4q + 15) as one 32-bit chunk,
+// channel order LSB first.  Per row word, mask and multiply drop its four digits into the top
+// byte: digit i sits at bit 8i + sh, the multiplier terms 2^(24 - sh - 6j) move it to 24 + 2i
+// (j = i); every cross term lands below bit 24 at its own position or above bit 31, so no carry
+// reaches the top byte.
+__device__ __forceinline__ uint32_t gather_d2(const uint32_t* row, int q, int sh) {
+  const uint32_t m = 0x03030303u << sh, mul = 0x01041040u >> sh;
+  uint32_t p[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p[i] = (row[min(q + i, 31)] & m) * mul;
+  return __byte_perm(__byte_perm(p[0], p[1], 0x0073), __byte_perm(p[2], p[3], 0x0073), 0x5410);
+}
+// 32 single bits (bit sh of channels 4q .. 4q + 31) as one chunk.  Two row words are merged
+// first (the second one's bits 4 higher), then multiplier terms 2^(24 - s - 7j) move bit i of the
+// first word to 24 + i and of the second to 28 + i: eight channels per top byte.
+__device__ __forceinline__ uint32_t gather_d1(const uint32_t* row, int q, int sh) {
+  const int pre = sh >= 4 ? 4 : 0, s = sh - pre;        // the multiplier needs s <= 3
+  const uint32_t m = 0x01010101u << s, mul = 0x01020408u >> s;
+  uint32_t p[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t x0 = row[min(q + 2 * i, 31)] >> pre, x1 = row[min(q + 2 * i + 1, 31)] >> pre;
+    p[i] = ((x0 & m) | ((x1 << 4) & (m << 4))) * mul;
+  }
+  return __byte_perm(__byte_perm(p[0], p[1], 0x0073), __byte_perm(p[2], p[3], 0x0073), 0x5410);
+}
+
 // Packed record of one token from its byte row: the bit stream of Sec. 5's stored values in the
-// D2 / D1 layout, four channels per step (field w bits at bit sh of channels [c0, c1), w = 2: a
-// base-4 digit, w = 1: a single bit; one multiply gathers four of them), appended LSB first.
+// D2 / D1 layout (field w bits at bit sh of channels [c0, c1), w = 2: a base-4 digit, w = 1: a
+// single bit), appended LSB first in 32-bit chunks.
 __device__ __forceinline__ void pack_token(const StreamLayout& lay, const uint32_t* row, const RecordWriter& out,
                                            int n_words) {
   uint32_t word = 0;
-  int pos = 0, wi = 0;
+  int pos = 0, wi = 0;                                  // uniform across the warp: same layout
+  auto append = [&](uint32_t v, int nb) {               // v: nb (1 .. 32) valid bits, zero above
+    word |= v << pos;
+    if (pos + nb >= 32) {
+      out.put(wi, word);
+      ++wi;
+      word = __funnelshift_rc(v, 0u, 32 - pos);         // the bits that did not fit (none at pos 0)
+    }
+    pos = (pos + nb) & 31;
+  };
   auto emit_run = [&](int c0, int c1, int sh, int w) {
-    for (int g4 = c0 >> 2; 4 * g4 < c1; ++g4) {
-      const int skip = max(c0 - 4 * g4, 0), n = min(c1 - 4 * g4, 4) - skip;
-      const uint32_t x = row[g4] >> sh;
-      uint32_t y = w == 2 ? (((x & 0x03030303u) * 0x00041041u) >> 18) & 0xFFu
-                          : (((x & 0x01010101u) * 0x00204081u) >> 21) & 0xFu;
-      y = (y >> (w * skip)) & ((1u << (w * n)) - 1u);
-      append_bits(y, w * n, word, pos, wi, out);
+    int drop = w * (c0 & 3);                            // chunks start on row words
+    for (int cb = c0 & ~3; cb < c1; cb += 32 / w) {
+      uint32_t v = w == 2 ? gather_d2(row, cb >> 2, sh) : gather_d1(row, cb >> 2, sh);
+      int nb = min(w * (c1 - cb), 32);
+      if (nb < 32) v &= (1u << nb) - 1u;
+      v >>= drop;
+      nb -= drop;
+      drop = 0;
+      append(v, nb);
     }
   };
-#pragma unroll 1
+#pragma unroll
   for (int k = 0; k < 4; ++k) emit_run(0, lay.l2[k], 2 * k, 2);                 // D2 digits
-#pragma unroll 1
+#pragma unroll
   for (int k = 3; k >= 0; --k) emit_run(lay.l2all[k], lay.lodd[k], 2 * k, 1);  // D1: top bits of odd widths
-#pragma unroll 1
+#pragma unroll
   for (int k = 0; k < 4; ++k) emit_run(lay.l2[k], lay.l2all[k], 2 * k, 2);     // D1: digits moved out of D2
   if (pos > 0) {
     out.put(wi, word);
@@ -308,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;                                 // TMEM lane quadrant
     const int tl = quad * 32 + lane;                           // token lane inside the tile
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-    const StreamLayout lay = sm.lay;
+    const StreamLayout& lay = sm.lay;
     uint32_t* my_bytes = sm.ubytes[tid];
     for (int it = eg; it < my_items; it += kEpiGroups) {
       const uint32_t aph = (it / kEpiGroups) & 1;
@@ -469,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     const int tl = quad * 32 + lane;
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-    const StreamLayout lay = sm.lay[sidx];
+    const StreamLayout& lay = sm.lay[sidx];
     uint32_t* my_bytes = sm.ubytes[tid];
     for (int it = bf; it < my_items; it += 2) {
       if (!ptx::mbar_wait_bounded(&sm.tfull[bf], (it >> 1) & 1, abort_flag)) { raise_abort(sm, a.err); break; }
