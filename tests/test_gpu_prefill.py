@@ -62,3 +62,49 @@ def test_prefill_argument_errors(aatc):
         aatc.prefill_attention(case.plan, 0, q, 60, cache, 64, 64)        # q_start + n_q > n_ctx
     with pytest.raises(aatc.AatcError):
         aatc.prefill_attention(case.plan, 0, q, 0, cache, 80, 64)         # n_ctx > max_tokens
+
+
+def _run_prefill(aatc, case, batch, n_ctx, n_q, q_scale, seed):
+    cfg = case.cfg
+    max_tokens = n_ctx
+    k, v = W.kv_host(cfg, 0, batch, n_ctx)
+    cache = case.plan.new_cache(batch, max_tokens, DEV)
+    aatc.encode(case.plan, 0, torch.from_numpy(k).to(DEV).to(torch.bfloat16), torch.from_numpy(v).to(DEV).to(torch.bfloat16),
+                cache, 0, n_ctx)
+    qh = W.to_bf16(q_scale * np.random.default_rng(seed).standard_normal((batch, n_q, cfg.n_q_heads, 128)))
+    q0 = n_ctx - n_q
+    out = aatc.prefill_attention(case.plan, 0, torch.from_numpy(qh).to(DEV).to(torch.bfloat16), q0, cache, n_ctx,
+                                 max_tokens).cpu().numpy()
+    return qh, q0, out, cache.cpu().numpy().view(np.uint32), max_tokens
+
+
+def test_prefill_peaky_scores_rescale(aatc):
+    """Queries x 24: score ranges of hundreds (log2 units), so row maxima keep jumping by more
+    than the lazy-rescale threshold from tile to tile and the O rescale path runs often."""
+    cfg = W.CONFIGS["qwen"]
+    case = Hn.Case(aatc, cfg, 2.75)
+    batch, n_ctx, n_q = 1, 1100, 300
+    qh, q0, out, u32, max_tokens = _run_prefill(aatc, case, batch, n_ctx, n_q, 24.0, 11)
+    rows = np.sort(np.random.default_rng(12).choice(n_q, 48, replace=False))
+    hk, hv = _coeffs(case, u32, batch, max_tokens, 0, n_ctx)
+    ref = O.prefill_attention(qh[0, rows].astype(np.float64), q0 + rows, hk, hv, case.basis[0, :, 0],
+                              case.basis[0, :, 1], cfg.group)
+    Hn.check_decode(out[0, rows].reshape(-1, 128), ref.reshape(-1, 128))
+    assert case.plan.device_error() == 0
+
+
+def test_prefill_qwen_full_length_sampled(aatc):
+    """One sequence of the bench's prefill shape (8192 queries over 8192 cached tokens, 28 / 4
+    heads): rows sampled over the whole range, including the first and the last row block."""
+    cfg = W.CONFIGS["qwen"]
+    case = Hn.Case(aatc, cfg, 2.75)
+    batch, n_ctx = 1, cfg.n_ctx
+    qh, q0, out, u32, max_tokens = _run_prefill(aatc, case, batch, n_ctx, n_ctx, 1.0, 13)
+    rows = np.unique(np.concatenate([np.arange(3), n_ctx - 1 - np.arange(3),
+                                     np.random.default_rng(14).choice(n_ctx, 18, replace=False)]))
+    hk, hv = _coeffs(case, u32, batch, max_tokens, 0, n_ctx)
+    ref = O.prefill_attention(qh[0, rows].astype(np.float64), q0 + rows, hk, hv, case.basis[0, :, 0],
+                              case.basis[0, :, 1], cfg.group)
+    Hn.check_decode(out[0, rows].reshape(-1, 128), ref.reshape(-1, 128))
+    assert np.isfinite(out).all()
+    assert case.plan.device_error() == 0
