@@ -128,10 +128,12 @@ __device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
 // talks to the softmax warps through mbarriers only.
 //   prologue  q' = (q U_K) f^K log2(e) / sqrt(128) on the tensor cores: q (bf16, exact) against
 //             U_K split into three bf16 parts (about 2^-25 relative), rows scaled to 2^14 and
-//             split into f16 hi / lo operands
+//             split into f16 hi / lo operands kept in TMEM (the A operand of the score MMA, so
+//             only the key tile is read from shared memory)
 //   per 128-token tile (TMA, 128-byte swizzle, key and value tiles double-buffered):
-//             S = q'_hi . code_K + q'_lo . code_K   tcgen05.mma M = N = 128, K = 128, two S
-//             buffers in TMEM: S of tile t + 1 is computed during the softmax of tile t
+//             S = q'_hi . code_K + q'_lo . code_K   tcgen05.mma M = N = 128, K = 128; the softmax
+//             keeps its scores in registers, so S of tile t + 1 is computed into the same TMEM
+//             columns as soon as every warp has read S(t)
 //             softmax from TMEM with the scores held in registers between the maximum and the
 //             exponent: s = S rs alpha^K (causal mask), lazy maximum (O rescaled only when a
 //             row's maximum grows by more than 2^8, so P' = 2^(s - m) alpha^V stays inside f16)
@@ -146,18 +148,17 @@ constexpr int kTOp = 2 * kTAtom;                   // one 128 x 128 16-bit opera
 constexpr float kLazyLog2 = 8.0f;
 constexpr uint32_t kIdescTT = ptx::idesc_f16_f32(128, 128);
 constexpr uint32_t kIdescBB = ptx::idesc_bf16_f32(128, 128);
-constexpr uint32_t kColS = 0;                      // two score buffers (0, 128); projection results
-constexpr uint32_t kColO = 256;                    // O accumulator
-constexpr uint32_t kColP = 384;                    // two P' buffers (384, 448): 64 columns of f16 pairs
+constexpr uint32_t kColS = 0;                      // score buffer; projection results
+constexpr uint32_t kColO = 128;                    // O accumulator
+constexpr uint32_t kColP = 256;                    // two P' buffers (256, 320): 64 columns of f16 pairs
+constexpr uint32_t kColQ = 384;                    // q' hi (384) and lo (448): A operands of the score MMA
 
 struct PrefillTcSmem {
-  alignas(1024) unsigned char qh[kTOp];            // q' hi: K-atoms = channels 0-63 | 64-127, rows = query rows
-  alignas(1024) unsigned char ql[kTOp];            // q' lo
   alignas(1024) unsigned char kt[2][kTOp];         // key codes: K-atoms = channels, rows = tokens
   alignas(1024) unsigned char vt[2][kTOp];         // value codes: K-atoms = tokens 0-63 | 64-127, rows = channels
   float al[3][2][TILE];                            // alpha^K, alpha^V of three tiles
   float xch[2][2][kTRows];                         // per-row partials of the two column halves (two slots)
-  uint64_t bar_k[2], bar_v[2], bar_s[2], sfree[2], ofree[2], pready, bar_p;
+  uint64_t bar_k[2], bar_v[2], ofree[2], bar_s, sfree, pready, bar_p;
   uint32_t tmem;
   int abort_flag;
 };
@@ -228,10 +229,10 @@ __global__ void __launch_bounds__(kTThreads, 1)
     for (int i = 0; i < 2; ++i) {
       ptx::mbar_init(&sm.bar_k[i], 1);
       ptx::mbar_init(&sm.bar_v[i], 1);
-      ptx::mbar_init(&sm.bar_s[i], 1);
-      ptx::mbar_init(&sm.sfree[i], kTSoftmax / 32);
       ptx::mbar_init(&sm.ofree[i], 1);          // PV of tiles i, i + 2, ... done
     }
+    ptx::mbar_init(&sm.bar_s, 1);                    // S(t) computed
+    ptx::mbar_init(&sm.sfree, kTSoftmax / 32);       // S(t) read out by every softmax warp
     ptx::mbar_init(&sm.pready, kTSoftmax / 32);
     ptx::mbar_init(&sm.bar_p, 1);
     sm.abort_flag = 0;
@@ -307,21 +308,20 @@ __global__ void __launch_bounds__(kTThreads, 1)
     m = fmaxf(sm.xch[0][0][r], sm.xch[0][1][r]);
     const float inv = m > 0.0f ? kPOpMax / m : 0.0f;
     rsr = m > 0.0f ? m / kPOpMax : 1.0f;             // > 0, so the mask's -inf survives the scaling
+    // this thread's 64 channels as 32 f16 pairs of hi and of lo: TMEM columns kColQ + 32 half ..
+    // (hi) and kColQ + 64 + 32 half .. (lo), row = lane
+    uint32_t hw[32], lw[32];
 #pragma unroll
-    for (int g8 = 0; g8 < 8; ++g8) {
-      uint32_t hv[4], lv[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float y0 = x[8 * g8 + 2 * j] * inv, y1 = x[8 * g8 + 2 * j + 1] * inv;
-        const __half2 h = __floats2half2_rn(y0, y1);
-        const float2 hf = __half22float2(h);
-        hv[j] = *reinterpret_cast<const uint32_t*>(&h);
-        lv[j] = pack_h2(y0 - hf.x, y1 - hf.y);
-      }
-      const int off = sw128_off(r, hc + 8 * g8);
-      *reinterpret_cast<uint4*>(sm.qh + off) = make_uint4(hv[0], hv[1], hv[2], hv[3]);
-      *reinterpret_cast<uint4*>(sm.ql + off) = make_uint4(lv[0], lv[1], lv[2], lv[3]);
+    for (int j = 0; j < 32; ++j) {
+      const float y0 = x[2 * j] * inv, y1 = x[2 * j + 1] * inv;
+      const __half2 h = __floats2half2_rn(y0, y1);
+      const float2 hf = __half22float2(h);
+      hw[j] = *reinterpret_cast<const uint32_t*>(&h);
+      lw[j] = pack_h2(y0 - hf.x, y1 - hf.y);
     }
+    ptx::tmem_st32(tmem + lane_base + kColQ + 32 * half, hw);
+    ptx::tmem_st32(tmem + lane_base + kColQ + 64 + 32 * half, lw);
+    ptx::tmem_wait_st();
   }
   // alpha^K / alpha^V of one tile: thread tid < 256 owns entry tid (K for tid < 128)
   auto alpha_of = [&](int t) -> float {
@@ -343,7 +343,6 @@ __global__ void __launch_bounds__(kTThreads, 1)
     // ---- control thread: TMA copies and MMAs.  Every wait below is on a phase that cannot be
     // overtaken: the next arrival on that barrier needs an action this thread takes later.
     if (lane == 0 && n_kv_tiles > 0) {
-      const uint32_t qh_a = ptx::smem_u32(sm.qh), ql_a = ptx::smem_u32(sm.ql);
       auto load_k = [&](int t) {
         const int buf = t & 1;
         const int krow = static_cast<int>(csk * a.n_ctx_pad) + t * TILE;
@@ -358,22 +357,22 @@ __global__ void __launch_bounds__(kTThreads, 1)
         ptx::tma_load_2d(sm.vt[buf], &tm, &sm.bar_v[buf], 0, vrow);
         ptx::tma_load_2d(sm.vt[buf] + kTAtom, &tm, &sm.bar_v[buf], 64, vrow);
       };
-      auto issue_s = [&](int t) {
-        const int buf = t & 1;
-        const uint32_t kt_a = ptx::smem_u32(sm.kt[buf]), d = tmem + kColS + 128 * buf;
+      auto issue_s = [&](int t) {                       // S = q'_hi . code_K + q'_lo . code_K, A from TMEM
+        const uint32_t kt_a = ptx::smem_u32(sm.kt[t & 1]);
         ptx::tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-          ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(qh_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
-                         kk > 0 ? 1u : 0u);
+          ptx::umma_f16_ta(tmem + kColS, tmem + kColQ + 8 * kk, ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
+                           kk > 0 ? 1u : 0u);
         }
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t off = (kk >> 2) * kTAtom + (kk & 3) * 32;
-          ptx::umma_bf16(d, ptx::sdesc_kmajor_sw128(ql_a + off), ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT, 1u);
+          ptx::umma_f16_ta(tmem + kColS, tmem + kColQ + 64 + 8 * kk, ptx::sdesc_kmajor_sw128(kt_a + off), kIdescTT,
+                           1u);
         }
-        ptx::umma_commit(&sm.bar_s[buf]);
+        ptx::umma_commit(&sm.bar_s);
       };
       load_k(0);
       load_v(0);
@@ -385,12 +384,9 @@ __global__ void __launch_bounds__(kTThreads, 1)
       issue_s(0);
       for (int t = 0; t < n_kv_tiles; ++t) {
         const int buf = t & 1;
-        if (t + 2 < n_kv_tiles) {                       // S(t) has read kt[buf]
-          wait(&sm.bar_s[buf], (t >> 1) & 1);
-          load_k(t + 2);
-        }
         if (t + 1 < n_kv_tiles) {
-          if (t >= 1) wait(&sm.sfree[buf ^ 1], ((t - 1) >> 1) & 1);   // S(t - 1) read out
+          wait(&sm.sfree, t & 1);                       // S(t) read out: the S buffer and kt[buf] are free
+          if (t + 2 < n_kv_tiles) load_k(t + 2);
           wait(&sm.bar_k[buf ^ 1], ((t + 1) >> 1) & 1);
           issue_s(t + 1);
           if (t >= 1) {                                 // PV(t - 1) has read vt[buf ^ 1]
@@ -424,21 +420,21 @@ __global__ void __launch_bounds__(kTThreads, 1)
       if (t + 2 < n_kv_tiles) a_next = alpha_of(t + 2);
       const float* akt = sm.al[t % 3][0] + hc;
       const float* avt = sm.al[t % 3][1] + hc;
-      wait(&sm.bar_s[buf], (t >> 1) & 1);
+      wait(&sm.bar_s, t & 1);
       ptx::tc_fence_after();
       // pass 1: x = S alpha^K over this thread's 64 tokens (masked), partial row maximum
       const int lim = last - t * TILE - hc;                 // tokens i <= lim are attended
       float x[64];
       {
         uint32_t s0[32], s1[32];
-        ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc, s0);
-        ptx::tmem_ld_32raw(tmem + lane_base + kColS + 128 * buf + hc + 32, s1);
+        ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc, s0);
+        ptx::tmem_ld_32raw(tmem + lane_base + kColS + hc + 32, s1);
         ptx::tmem_ld_wait();
         ptx::tmem_regs_ready(s0);
         ptx::tmem_regs_ready(s1);
         ptx::tc_fence_before();
         __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(&sm.sfree[buf]);    // this warp's part of S(t) read out
+        if (lane == 0) ptx::mbar_arrive(&sm.sfree);         // this warp's part of S(t) read out
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           x[i] = __uint_as_float(s0[i]) * akt[i];
