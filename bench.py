@@ -241,6 +241,46 @@ def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32
                         f"{n_tokens} tokens, 2.75 bits"}
 
 
+def bf16_decode_timing(aatc, kd, vd, qs, n_ctx, packed_us, n_calls=64, reps=3):
+    """The uncompressed reference decode (split-K attention over the bf16 K/V with the same shapes
+    and queries), timed like the packed decode: a CUDA graph of calls alternating two K/V copies
+    (2 x 134 MB > L2).  GB/s on the bf16 bytes a call reads, and the packed decode's speed-up
+    over it (the byte ratio 512 / 96 = 5.3 bounds it at 2.75 bits)."""
+    import torch
+    pairs = [(kd, vd), (kd.clone(), vd.clone())]
+    batch, n_kv, n_q = kd.shape[0], kd.shape[2], qs.shape[2]
+    out = torch.empty((batch, n_q, 128), dtype=torch.float32, device=kd.device)
+    ws = torch.empty(max(1, aatc.bf16_workspace_bytes(batch, n_kv, n_q, n_ctx) // 4), dtype=torch.float32,
+                     device=kd.device)
+
+    def calls():
+        for i in range(n_calls):
+            k_, v_ = pairs[i & 1]
+            aatc.bf16_decode_attention(k_, v_, qs[i % qs.shape[0]], n_ctx, out=out, workspace=ws)
+
+    calls()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        calls()
+    graph.replay()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) * 1e3 / (reps * n_calls)
+    nbytes = (kd.numel() + vd.numel()) * 2
+    peak, _ = _peaks()
+    return {"us_per_call": round(us, 3), "gbs": round(nbytes / (us * 1e-6) / 1e9, 2), "bytes_per_call": nbytes,
+            "frac_of_measured_hbm": round(nbytes / (us * 1e-6) / 1e9 / peak, 4),
+            "packed_speedup": round(us / packed_us, 3),
+            "what": "uncompressed bf16 K/V reference decode, same shapes and queries, 64 calls per CUDA graph"}
+
+
 def prefill_timing(aatc, device, iters=2, batch=None, reference=True):
     """Prefill attention over the packed cache on the Qwen-2.5-7B-shaped layer: 16 sequences x
     8192 tokens, 28 query heads over 4 kv-heads, causal (the chunk is the whole context, encoded
@@ -438,6 +478,7 @@ def run_ours(args):
         return
 
     sw = sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_dec)
+    ref16 = bf16_decode_timing(aatc, kd, vd, qs, T, dec_mean / steps_dec * 1e3)
     hid = hidden_encode_timing(aatc, dev)
     pre = prefill_timing(aatc, dev)
 
@@ -486,6 +527,7 @@ def run_ours(args):
         "clocks": clocks,
         "planner": planner_timing(aatc),
         "sink_window": sw,
+        "bf16_decode": ref16,
         "encode_hidden": hid,
         "prefill": pre,
     }

@@ -107,7 +107,12 @@ struct DecodeSplit {
   int split_len;          // tokens of the longest split, a multiple of TILE
 };
 
-DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms);
+DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms, int ctas_per_sm = 5);
+// Split plan of the bf16 reference decode: the most CTAs per SM (up to 4) its shared memory
+// allows, in one wave.
+DecodeSplit bf16_decode_split(int batch, int n_kv, int n_q, int n_ctx, int num_sms);
+// Dynamic shared memory of one bf16 reference split CTA (query columns padded to gp = 4 or 8).
+size_t bf16_split_smem(int gp, int split_len);
 // Decode workspace: split partials per (sequence, query head, split) -- 128 channel sums, then
 // m, l, padded to a multiple of 4 floats -- followed by the per-call score A fragments per
 // (sequence, kv-head) (up to 2 W k-steps x 32 lanes x 16 B), their offset corrections and score

@@ -41,14 +41,14 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 namespace aatc {
 
-DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
-  // About five CTAs per SM in a single wave: n_splits per (sequence, kv-head), with split s
-  // covering tiles [s T / n_splits, (s + 1) T / n_splits) so split lengths differ by at most one
-  // tile and every SM gets nearly the same number of tiles.  A split holds at most 16 tiles
+DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms, int ctas_per_sm) {
+  // About ctas_per_sm CTAs per SM in a single wave: n_splits per (sequence, kv-head), with split
+  // s covering tiles [s T / n_splits, (s + 1) T / n_splits) so split lengths differ by at most
+  // one tile and every SM gets nearly the same number of tiles.  A split holds at most 16 tiles
   // (its scores are kept in shared memory).
   const long tiles = (n_ctx + TILE - 1) / TILE;
   const long units = static_cast<long>(batch) * n_kv;
-  const long target = 5L * std::max(1, num_sms);
+  const long target = static_cast<long>(std::max(1, ctas_per_sm)) * std::max(1, num_sms);
   long n = (target + units / 2) / units;
   n = std::max(n, (tiles + 15) / 16);
   n = std::max(1L, std::min(n, tiles));
@@ -56,6 +56,16 @@ DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms) {
   sp.n_splits = static_cast<int>(n);
   sp.split_len = static_cast<int>((tiles + n - 1) / n) * TILE;   // longest split
   return sp;
+}
+
+DecodeSplit bf16_decode_split(int batch, int n_kv, int n_q, int n_ctx, int num_sms) {
+  const int gp = n_q / n_kv <= 4 ? 4 : 8;
+  constexpr size_t kSmPerSm = 228 * 1024, kReserved = 1024;   // per SM; reserved per CTA
+  for (int c = 4; c > 1; --c) {
+    const DecodeSplit sp = decode_split(batch, n_kv, n_ctx, num_sms, c);
+    if (static_cast<size_t>(c) * (bf16_split_smem(gp, sp.split_len) + kReserved) <= kSmPerSm) return sp;
+  }
+  return decode_split(batch, n_kv, n_ctx, num_sms, 1);
 }
 
 Plan* plan_from_handle(aatc_plan_t p) { return as_plan(p); }
@@ -451,7 +461,7 @@ aatc_status_t aatc_bf16_decode_workspace_bytes(int32_t batch, int32_t n_kv, int3
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     sms = 1;
-  *bytes = aatc::bf16_decode_workspace(batch, n_q, aatc::decode_split(batch, n_kv, n_ctx, sms));
+  *bytes = aatc::bf16_decode_workspace(batch, n_q, aatc::bf16_decode_split(batch, n_kv, n_q, n_ctx, sms));
   return AATC_OK;
 }
 
@@ -469,7 +479,7 @@ aatc_status_t aatc_bf16_decode_attention(const void* K, const void* V, const voi
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return cuda_status(e);
-  const auto sp = aatc::decode_split(batch, n_kv, n_ctx, sms);
+  const auto sp = aatc::bf16_decode_split(batch, n_kv, n_q, n_ctx, sms);
   if (workspace_bytes < aatc::bf16_decode_workspace(batch, n_q, sp)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_bf16_decode(K, V, q, batch, n_ctx, max_tokens, n_kv, n_q, out,
                                               workspace, sp, static_cast<cudaStream_t>(stream)));

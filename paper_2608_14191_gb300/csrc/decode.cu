@@ -911,7 +911,13 @@ __global__ void __launch_bounds__(kThreads)
     cp_async_commit();
   };
   const int tile0 = t_begin / TILE;
-  stage(a.k, tile0, 0);
+  // key tiles, then value tiles, stream through the two buffers: the first value tile is in
+  // flight during the last key tile and the softmax in between
+  auto stage_seq = [&](int i, int buf) {
+    if (i < n_tiles_split) stage(a.k, tile0 + i, buf);
+    else stage(a.v, tile0 + i - n_tiles_split, buf);
+  };
+  stage_seq(0, 0);
   __syncthreads();
   float mloc[GP];
 #pragma unroll
@@ -920,7 +926,7 @@ __global__ void __launch_bounds__(kThreads)
     const int buf = ti & 1;
     cp_async_wait_all();
     __syncthreads();
-    if (ti + 1 < n_tiles_split) stage(a.k, tile0 + ti + 1, buf ^ 1);
+    stage_seq(ti + 1, buf ^ 1);                            // the next key tile, or value tile 0
     const __nv_bfloat16* row = kt + buf * TILE * kRow + tid * kRow;
     float s[GP];
 #pragma unroll
@@ -948,10 +954,8 @@ __global__ void __launch_bounds__(kThreads)
       mloc[g] = fmaxf(mloc[g], v);
     }
   }
-  cp_async_wait_all();
   __syncthreads();
   block_reduce<GP, true>(mloc, red);
-  stage(a.v, tile0, 0);
   float lsum[GP];
 #pragma unroll
   for (int g = 0; g < GP; ++g) lsum[g] = 0.0f;
@@ -972,10 +976,10 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
     for (int i = 0; i < 4; ++i) acc[g][i] = 0.0f;
   for (int ti = 0; ti < n_tiles_split; ++ti) {
-    const int buf = ti & 1;
+    const int buf = (n_tiles_split + ti) & 1;
     cp_async_wait_all();
     __syncthreads();
-    if (ti + 1 < n_tiles_split) stage(a.v, tile0 + ti + 1, buf ^ 1);
+    if (ti + 1 < n_tiles_split) stage_seq(n_tiles_split + ti + 1, buf ^ 1);
     const int tend = min(TILE, t_end - (tile0 + ti) * TILE);
     for (int tt = tq; tt < tend; tt += 4) {
       const uint2 r = *reinterpret_cast<const uint2*>(kt + buf * TILE * kRow + tt * kRow + dg * 4);
@@ -1128,8 +1132,7 @@ cudaError_t launch_split_g(const DecodeArgs& a, int batch, int jpw, size_t smem,
 
 template <int GP>
 cudaError_t launch_bf16_split(const Bf16Args& a, int batch, cudaStream_t st) {
-  const size_t smem = 4 * (static_cast<size_t>(D) * GP + 32 + static_cast<size_t>(a.split_len) * GP + 4 * GP * D) +
-                      2 * static_cast<size_t>(TILE) * (D + 8) * 2;
+  const size_t smem = bf16_split_smem(GP, a.split_len);
   static size_t smem_set = 0;
   if (smem > smem_set) {
     cudaError_t e = cudaFuncSetAttribute(aatc_bf16_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1230,6 +1233,13 @@ cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int b
       plan.dev.lay, plan.dev.entry, plan.dev.f, layer, plan.dims.n_kv_heads, batch, t0, n, g.n_tiles, plan.n_words,
       plan.n_entries, out);
   return cudaGetLastError();
+}
+
+size_t bf16_split_smem(int gp, int split_len) {
+  // query columns [128][gp], reduction scratch, scores [split_len][gp], per-quarter sums
+  // [4][gp][128] (fp32); two padded bf16 tiles [128][136]
+  return 4 * (static_cast<size_t>(D) * gp + 32 + static_cast<size_t>(split_len) * gp + 4 * static_cast<size_t>(gp) * D) +
+         2 * static_cast<size_t>(TILE) * (D + 8) * 2;
 }
 
 cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx, int max_tokens,
