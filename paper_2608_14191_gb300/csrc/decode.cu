@@ -722,6 +722,9 @@ __global__ void __launch_bounds__(kMThreads)
     ptx::mbar_arrive_expect_tx(&bar, D * D * 4);
     ptx::bulk_load(ut_s, a.u32t + static_cast<size_t>(sv) * D * D, D * D * 4, &bar);
   }
+  // the next call's query kernel may start its plan-constant prologue now; it reads the query
+  // and the workspace only after this grid has completed (its griddepcontrol.wait)
+  ptx::grid_launch_dependents();
   const float fv = tid < D ? a.f[sv * D + tid] : 0.0f;
   // ---- uncompressed tokens (inputs of this call, not produced by the split kernel)
   float m_f = -INFINITY, l_f = 0.0f;
