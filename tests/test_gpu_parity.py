@@ -90,6 +90,24 @@ def test_tiny_bf16_reference_decode(aatc, tiny):
             np.testing.assert_allclose(out[j], ref, atol=2e-5, rtol=1e-4)
 
 
+def test_bf16_reference_decode_qwen_group7(aatc):
+    """The uncompressed reference decode with G = 7 (query columns padded to 8, its own split
+    plan), two sequences, a ragged context, against plain attention per query head."""
+    cfg = W.CONFIGS["qwen"]
+    batch, n_ctx = 2, 3000
+    k, v = W.kv_host(cfg, 0, batch, n_ctx)
+    qs = W.queries_host(cfg, 0, batch, 1)[0]                     # (batch, H_q, 128)
+    kd = torch.from_numpy(k).to(DEV).to(torch.bfloat16)
+    vd = torch.from_numpy(v).to(DEV).to(torch.bfloat16)
+    out = aatc.bf16_decode_attention(kd, vd, torch.from_numpy(qs).to(DEV).to(torch.bfloat16), n_ctx - 17)
+    out = out.cpu().numpy()
+    g = cfg.group
+    for b in range(batch):
+        for j in range(0, cfg.n_q_heads, 3):
+            ref = O.attention(qs[b, j], k[b, :n_ctx - 17, j // g], v[b, :n_ctx - 17, j // g])
+            np.testing.assert_allclose(out[b, j], ref, atol=2e-5, rtol=1e-4)
+
+
 def test_append_in_pieces_equals_one_shot(aatc, tiny):
     """Position-addressed layout: appending 300 + 1 + 211 tokens (ragged, crossing tile
     boundaries) writes the same bytes as one encode of 512 (Alg. 1 'Append')."""
