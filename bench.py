@@ -72,7 +72,7 @@ def whole_job_rate(units_per_rank, ws, ms):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms during the timed region."""
+    """nvidia-smi clocks and throttle reasons sampled every 50 ms during the timed region."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -88,11 +88,22 @@ class ClockSampler:
             os.close(fd)
             self.out = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.out,
+                                          "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.out,
                                          stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
         return self
+
+    def wait_first_sample(self, timeout_s: float = 3.0):
+        """Block until nvidia-smi has written its first sample, so the timed region is covered."""
+        if self.proc is None or not self.path:
+            return
+        t_end = time.time() + timeout_s
+        while time.time() < t_end:
+            self.out.flush()
+            if os.path.getsize(self.path) > 0:
+                return
+            time.sleep(0.01)
 
     def __exit__(self, *exc):
         if self.proc is not None:
@@ -419,6 +430,8 @@ def run_ours(args):
     if ws_ > 1:
         torch.distributed.barrier()
     with ClockSampler(local) as clk:
+        clk.wait_first_sample()
+        step_dev(0)                                  # untimed: clocks back up after the wait
         torch.cuda.synchronize()
         t_start = torch.cuda.Event(enable_timing=True)
         t_end = torch.cuda.Event(enable_timing=True)
