@@ -108,3 +108,35 @@ def test_prefill_qwen_full_length_sampled(aatc):
     Hn.check_decode(out[0, rows].reshape(-1, 128), ref.reshape(-1, 128))
     assert np.isfinite(out).all()
     assert case.plan.device_error() == 0
+
+
+def test_prefill_second_layer_of_a_plan(aatc):
+    """A two-layer plan, prefill on layer 1: the kernels index the layer's basis, scales and
+    record layout (layer 0 holds a different, identity-basis plan)."""
+    cfg = W.Config(7, "two_layer", 2, 2, 10, 1, 700, (2.75,), 1, "two-layer plan, prefill on layer 1")
+    case = Hn.Case(aatc, cfg, 2.75, layers=[1])
+    batch, n_ctx, n_q = 1, 700, 90
+    k, v = W.kv_host(cfg, 1, batch, n_ctx)
+    cache = case.plan.new_cache(batch, n_ctx, DEV)
+    aatc.encode(case.plan, 1, torch.from_numpy(k).to(DEV).to(torch.bfloat16),
+                torch.from_numpy(v).to(DEV).to(torch.bfloat16), cache, 0, n_ctx)
+    qh = W.to_bf16(np.random.default_rng(21).standard_normal((batch, n_q, cfg.n_q_heads, 128)))
+    q0 = n_ctx - n_q
+    out = aatc.prefill_attention(case.plan, 1, torch.from_numpy(qh).to(DEV).to(torch.bfloat16), q0, cache, n_ctx,
+                                 n_ctx).cpu().numpy()
+    u32 = cache.cpu().numpy().view(np.uint32)
+    hk, hv = [], []
+    for h in range(cfg.n_kv_heads):
+        hh = []
+        for kind in (0, 1):
+            rec, alpha = Hn.read_stream(case, u32, batch, n_ctx, 0, h, kind, 0, n_ctx)
+            _, bits, scales = case.stream(1, h, kind)
+            hh.append(O.dequantize_f32(O.unpack_records(rec, bits.astype(np.int64)), alpha, scales,
+                                       bits.astype(np.int64)))
+        hk.append(hh[0])
+        hv.append(hh[1])
+    rows = np.array([0, 1, 44, n_q - 2, n_q - 1])
+    ref = O.prefill_attention(qh[0, rows].astype(np.float64), q0 + rows, np.stack(hk), np.stack(hv),
+                              case.basis[1, :, 0], case.basis[1, :, 1], cfg.group)
+    Hn.check_decode(out[0, rows].reshape(-1, 128), ref.reshape(-1, 128))
+    assert case.plan.device_error() == 0
