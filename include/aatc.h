@@ -228,7 +228,8 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x,
  *   cache     : the packed cache holding tokens [0, n_ctx), q_start + n_q <= n_ctx <= max_tokens
  *   out       : device fp32 [batch][n_q][n_q_heads][128]
  *   workspace : device, >= aatc_prefill_workspace_bytes(batch, n_ctx) (the signed codes of the
- *               context as f16, [batch][n_kv][K|V][ceil(n_ctx/128)*128][128]); contents ignored
+ *               context as f16, [batch][n_kv][K|V][ceil(n_ctx/128)*128][128], value tiles stored
+ *               transposed as [channel][token] per 128-token tile); contents ignored
  * Query head j reads kv-head j / (n_q_heads / n_kv_heads).  Asynchronous on `stream`.
  * Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer or sizes, q_start + n_q >
  * n_ctx), AATC_ERR_CAPACITY (n_ctx > max_tokens), AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (W > 32),
