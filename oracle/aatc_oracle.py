@@ -21,6 +21,12 @@ PCA equivalence (Appendix, Proposition), the quantizer error bound
 the compression ratio the paper prints (Sec. 6.1); the transform from the model
 weights (:func:`whitening_transform`, tests/test_whitening.py) is pinned by
 W = A B, A^T Sigma_X A = S and both statements of the appendix Proposition.
+Head-group bases (:func:`plan_head_group`, :func:`decode_attention_head_group`,
+tests/test_head_groups.py) are pinned by the reduction to the per-head plan and
+decode at one head per group, plain attention per query head when the group
+coefficients are exact, the split of an exactly block-diagonal second moment
+into the heads' own eigenbases, the budget identity, and the transform-coding
+gain of one group transform over separate heads for correlated heads.
 
 parity unpinned: the packed record bit layout (:func:`record_entries`,
 :func:`pack_records`, :func:`cache_records`) is defined by this build, not by the
@@ -490,6 +496,72 @@ def decode_attention(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_
         qt = np.asarray(basis_k[h], np.float64).T @ np.asarray(q_heads[j], np.float64)
         a = softmax(np.asarray(hk[h], np.float64) @ qt / math.sqrt(D))
         out[j] = np.asarray(basis_v[h], np.float64) @ (a @ np.asarray(hv[h], np.float64))
+    return out
+
+
+# ----------------------------------------------------------------------------
+# Head-group bases (Sec. 5 Step 1, remark on multi-head attention): the kv-heads of a group share
+# one transform of width 128 G_h; every query head still attends with its own 128-dim block.
+# ----------------------------------------------------------------------------
+
+def embed_query(q: np.ndarray, block: int, n_blocks: int) -> np.ndarray:
+    """A query head's vector placed at its kv-head's 128-dim block of the group's concatenated
+    space (zeros elsewhere), so q . k_block = q_embedded . k_group."""
+    q = np.asarray(q, np.float64)
+    out = np.zeros(q.shape[:-1] + (D * n_blocks,))
+    out[..., D * block:D * (block + 1)] = q
+    return out
+
+
+def plan_head_group(x_calib_heads: np.ndarray, avg_bits: float, b_max: int = 8, queries_by_head=None,
+                    group: int = 1, weights: str = "aatc"):
+    """Calibrate one head-group stream: the G_h kv-heads of the group (x_calib_heads: (G_h, N, 128),
+    the same N calibration tokens) are concatenated into 128 G_h-dim vectors, which get one PCA
+    basis, one weighted reverse water-filling over all 128 G_h channels with budget
+    avg_bits * 128 G_h (Eq. waterfilling-keys over the group's channels) and one P99 scale per
+    channel -- the steps of :func:`plan_stream` at the group's width.
+
+    queries_by_head: for keys, the calibration queries of the group's query heads in kv-head
+    order (G_h * group arrays of (T, 128)); query head i belongs to kv-head i // group, and its
+    weight contribution uses the query embedded at that kv-head's block (the score it sees is
+    q . k_block).  None for values (w = 1, W_O = I).  weights = 'var' gives w = 1 (var-only).
+    """
+    xh = np.asarray(x_calib_heads, np.float64)
+    g_h = xh.shape[0]
+    x = np.concatenate([xh[m] for m in range(g_h)], axis=1)           # (N, 128 G_h)
+    width = D * g_h
+    c = second_moment(x)
+    lam, u = eigenbasis(c)
+    if weights == "var" or queries_by_head is None:
+        w = np.ones(width) if weights == "var" else value_weights(u.T)
+    else:
+        embedded = [embed_query(q, i // group, g_h) for i, q in enumerate(queries_by_head)]
+        w = key_weights(u.T, embedded)
+    gsc = w * lam
+    order = np.argsort(-gsc, kind="stable")
+    u, lam, w, gsc = u[:, order], lam[order], w[order], gsc[order]
+    bits = greedy_allocation(gsc, int(round(avg_bits * width)), b_max)
+    scales = channel_scales(u, x)
+    return {"basis": u, "bits": bits, "scales": scales, "sigma2": lam, "weights": w, "g": gsc}
+
+
+def decode_attention_head_group(q_heads: np.ndarray, hk: np.ndarray, hv: np.ndarray, basis_k: np.ndarray,
+                                basis_v: np.ndarray, group: int) -> np.ndarray:
+    """Decode over one head-group stream of one sequence (Alg. 1 reconstruct / attend lines at the
+    group's width): q_heads (G_h * group, 128) are the group's query heads in kv-head order;
+    hk, hv (n, 128 G_h) the dequantized group coefficients; basis_k, basis_v (128 G_h, 128 G_h)
+    the group transforms (K_group_hat = h_hat U^T).  Query head i reads kv-head block m = i // group:
+    s = (U_K^T q~) . h_hat / sqrt(128) with q~ the embedded query (the head dimension stays 128),
+    a = softmax(s), out = (U_V (a h_hat^V)) restricted to block m."""
+    hk = np.asarray(hk, np.float64)
+    hv = np.asarray(hv, np.float64)
+    g_h = hk.shape[1] // D
+    out = np.zeros((q_heads.shape[0], D))
+    for i in range(q_heads.shape[0]):
+        m = i // group
+        qt = np.asarray(basis_k, np.float64).T @ embed_query(q_heads[i], m, g_h)
+        a = softmax(hk @ qt / math.sqrt(D))
+        out[i] = (np.asarray(basis_v, np.float64) @ (a @ hv))[D * m:D * (m + 1)]
     return out
 
 
