@@ -98,6 +98,30 @@ aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k, cons
                              double* sigma2_out, double* weights_out, int32_t n_threads);
 
 /*
+ * Head-group calibration (Sec. 5 Step 1, remark on multi-head attention: the heads of a group
+ * share one transform).  The g_h kv-heads of a group are concatenated into vectors of width
+ * d = 128 g_h; the planner computes one PCA basis over them (uncentered second moment, Jacobi,
+ * descending eigenvalues, canonical signs), the weights w^K_c = sum over the group's query heads j
+ * of u_c[block(j)]^T M_j u_c[block(j)] (query head j belongs to kv-head j / group and its score
+ * sees only that kv-head's 128-dim block; M_j = mean q q^T of its calibration queries), or w = 1
+ * for values / var-only, the exact integer reverse water-filling over the d channels with budget
+ * avg_bits * d, b in {0..b_max}, and one P99 scale per channel.  Channels are returned in storage
+ * order (g = w sigma^2 descending), so the widths are non-increasing.
+ *   calib      : host fp32 [g_h][n_calib][128], the group's kv-heads on the same tokens
+ *   calib_q    : host fp32 [g_h * group][n_calib_q][128] in kv-head order, or NULL (values)
+ *   basis_out  : host fp32 [d][d] (dim x channel); bits_out uint8 [d]; scales_out fp32 [d];
+ *   sigma2_out, weights_out : host fp64 [d] or NULL
+ * Errors: AATC_ERR_INVALID_ARG (g_h outside 1..8, group < 1, n_calib < 2, null outputs, b_max
+ * outside 1..8), AATC_ERR_BUDGET (avg_bits * d not an integer in [0, b_max d]).  Host only.
+ * The plan, encode and decode kernels take per-kv-head streams; head-group streams are planned
+ * here and checked against the oracle, and their device path is not built yet.
+ */
+aatc_status_t aatc_calibrate_head_group(int32_t g_h, int32_t group, const float* calib, int32_t n_calib,
+                                        const float* calib_q, int32_t n_calib_q, double avg_bits, int32_t b_max,
+                                        int32_t weights_mode, float* basis_out, uint8_t* bits_out,
+                                        float* scales_out, double* sigma2_out, double* weights_out);
+
+/*
  * Global cross-layer bit allocation (Sec. 5 "waterfilling problem for the keys / values" summed
  * over layers; Algorithm 1 "Allocate bits globally via reverse waterfilling over all (l, c)";
  * the experimental-setup paragraph on AATC for the normalisation and the protected layers).

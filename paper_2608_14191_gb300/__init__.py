@@ -46,6 +46,7 @@ SIGNATURES = {
     "aatc_last_cuda_error": (_I32, []),
     "aatc_version": (_I32, []),
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
+    "aatc_calibrate_head_group": (_I32, [_I32, _I32, _P, _I32, _P, _I32, _F64, _I32, _I32, _P, _P, _P, _P, _P]),
     "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
     "aatc_whitening_transform": (_I32, [_I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "aatc_hidden_operand": (_I32, [ctypes.POINTER(Dims), _I32, _P, _P, _P, _P]),
@@ -137,6 +138,31 @@ def calibrate(dm: Dims, calib_k: np.ndarray, calib_v: np.ndarray, calib_q: np.nd
                             _ptr(basis), _ptr(bits), _ptr(scales), _ptr(sigma2), _ptr(weights), int(n_threads))
     _check(st, "aatc_calibrate")
     assert S == basis.shape[0] * H * 2
+    return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
+
+
+def calibrate_head_group(calib: np.ndarray, calib_q: np.ndarray | None, avg_bits: float, group: int = 1,
+                         b_max: int = 8, var_only: bool = False):
+    """aatc_calibrate_head_group: one transform and one allocation over the concatenated kv-heads
+    of a group.  calib: fp32 [g_h][N][128]; calib_q: fp32 [g_h * group][Nq][128] (keys) or None.
+    Returns dict(basis [d][d], bits [d], scales [d], sigma2 [d], weights [d]), d = 128 g_h."""
+    c = np.ascontiguousarray(calib, dtype=np.float32)
+    if c.ndim != 3 or c.shape[2] != HEAD_DIM:
+        raise ValueError("calib must be [g_h][N][128]")
+    g_h = c.shape[0]
+    cq = None if calib_q is None else np.ascontiguousarray(calib_q, dtype=np.float32)
+    if cq is not None and (cq.ndim != 3 or cq.shape[0] != g_h * group or cq.shape[2] != HEAD_DIM):
+        raise ValueError("calib_q must be [g_h * group][Nq][128]")
+    d = HEAD_DIM * g_h
+    basis = np.empty((d, d), np.float32)
+    bits = np.empty(d, np.uint8)
+    scales = np.empty(d, np.float32)
+    sigma2 = np.empty(d, np.float64)
+    weights = np.empty(d, np.float64)
+    _check(load().aatc_calibrate_head_group(g_h, int(group), _ptr(c), c.shape[1], None if cq is None else _ptr(cq),
+                                            0 if cq is None else cq.shape[1], float(avg_bits), int(b_max),
+                                            1 if var_only else 0, _ptr(basis), _ptr(bits), _ptr(scales),
+                                            _ptr(sigma2), _ptr(weights)), "aatc_calibrate_head_group")
     return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
 
 

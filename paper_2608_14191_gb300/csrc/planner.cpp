@@ -20,43 +20,45 @@ namespace {
 
 constexpr int kD = 128;
 
-// C = (1/N) sum_n x_n x_n^T over fp32 rows, accumulated in fp64 (Sec. 5 Step 1: Sigma = X^T X / T).
-void second_moment(const float* x, int n, std::vector<double>& c) {
-  c.assign(kD * kD, 0.0);
-  std::vector<double> row(kD);
+// C = (1/N) sum_n x_n x_n^T over fp32 rows of width d, accumulated in fp64 (Sec. 5 Step 1:
+// Sigma = X^T X / T).
+void second_moment(const float* x, int n, std::vector<double>& c, int d = kD) {
+  c.assign(static_cast<size_t>(d) * d, 0.0);
+  std::vector<double> row(d);
   for (int t = 0; t < n; ++t) {
-    const float* xt = x + static_cast<size_t>(t) * kD;
-    for (int i = 0; i < kD; ++i) row[i] = xt[i];
-    for (int i = 0; i < kD; ++i) {
+    const float* xt = x + static_cast<size_t>(t) * d;
+    for (int i = 0; i < d; ++i) row[i] = xt[i];
+    for (int i = 0; i < d; ++i) {
       const double xi = row[i];
-      double* ci = c.data() + i * kD;
-      for (int j = i; j < kD; ++j) ci[j] += xi * row[j];
+      double* ci = c.data() + static_cast<size_t>(i) * d;
+      for (int j = i; j < d; ++j) ci[j] += xi * row[j];
     }
   }
   const double inv = 1.0 / n;
-  for (int i = 0; i < kD; ++i)
-    for (int j = i; j < kD; ++j) {
-      c[i * kD + j] *= inv;
-      c[j * kD + i] = c[i * kD + j];
+  for (int i = 0; i < d; ++i)
+    for (int j = i; j < d; ++j) {
+      c[static_cast<size_t>(i) * d + j] *= inv;
+      c[static_cast<size_t>(j) * d + i] = c[static_cast<size_t>(i) * d + j];
     }
 }
 
 // Cyclic Jacobi: rotate away each off-diagonal element in turn until the off-diagonal mass is
 // negligible.  a is overwritten (its diagonal converges to the eigenvalues); v accumulates the
 // rotations, so columns of v are the eigenvectors.
-void jacobi_eigen(std::vector<double>& a, std::vector<double>& v) {
+void jacobi_eigen(std::vector<double>& a, std::vector<double>& v, int n = kD) {
+  const size_t kD = static_cast<size_t>(n);   // the matrix width (128, or 128 G_h for a head group)
   v.assign(kD * kD, 0.0);
-  for (int i = 0; i < kD; ++i) v[i * kD + i] = 1.0;
+  for (size_t i = 0; i < kD; ++i) v[i * kD + i] = 1.0;
   double frob = 0.0;
   for (double e : a) frob += e * e;
   const double tiny = 1e-300;
   for (int sweep = 0; sweep < 100; ++sweep) {
     double off = 0.0;
-    for (int p = 0; p < kD; ++p)
-      for (int q = p + 1; q < kD; ++q) off += a[p * kD + q] * a[p * kD + q];
+    for (size_t p = 0; p < kD; ++p)
+      for (size_t q = p + 1; q < kD; ++q) off += a[p * kD + q] * a[p * kD + q];
     if (off <= 1e-30 * frob || off < tiny) break;
-    for (int p = 0; p < kD - 1; ++p) {
-      for (int q = p + 1; q < kD; ++q) {
+    for (size_t p = 0; p + 1 < kD; ++p) {
+      for (size_t q = p + 1; q < kD; ++q) {
         const double apq = a[p * kD + q];
         if (std::fabs(apq) < tiny) continue;
         const double app = a[p * kD + p], aqq = a[q * kD + q];
@@ -66,18 +68,18 @@ void jacobi_eigen(std::vector<double>& a, std::vector<double>& v) {
         const double t = (theta >= 0 ? 1.0 : -1.0) / (std::fabs(theta) + std::sqrt(theta * theta + 1.0));
         const double c = 1.0 / std::sqrt(t * t + 1.0);
         const double s = t * c;
-        for (int k = 0; k < kD; ++k) {          // A <- A J (columns p, q)
+        for (size_t k = 0; k < kD; ++k) {       // A <- A J (columns p, q)
           const double akp = a[k * kD + p], akq = a[k * kD + q];
           a[k * kD + p] = c * akp - s * akq;
           a[k * kD + q] = s * akp + c * akq;
         }
-        for (int k = 0; k < kD; ++k) {          // A <- J^T A (rows p, q)
+        for (size_t k = 0; k < kD; ++k) {       // A <- J^T A (rows p, q)
           const double apk = a[p * kD + k], aqk = a[q * kD + k];
           a[p * kD + k] = c * apk - s * aqk;
           a[q * kD + k] = s * apk + c * aqk;
         }
         a[p * kD + q] = a[q * kD + p] = 0.0;
-        for (int k = 0; k < kD; ++k) {          // V <- V J
+        for (size_t k = 0; k < kD; ++k) {       // V <- V J
           const double vkp = v[k * kD + p], vkq = v[k * kD + q];
           v[k * kD + p] = c * vkp - s * vkq;
           v[k * kD + q] = s * vkp + c * vkq;
@@ -284,6 +286,96 @@ extern "C" aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* ca
   for (int t = 1; t < nt; ++t) pool.emplace_back(worker);
   worker();
   for (auto& th : pool) th.join();
+  return AATC_OK;
+}
+
+// Head-group stream (Sec. 5 Step 1, remark on multi-head attention): the g_h kv-heads of a group
+// concatenated into vectors of width d = 128 g_h get one PCA basis, one weighted reverse
+// water-filling over the d channels (budget avg_bits * d) and one P99 scale per channel.  Query
+// head j of the group belongs to kv-head j / group; its score q . k_block sees only that block, so
+// its key weight is u_c[block]^T M_j u_c[block] with M_j the second moment of its calibration
+// queries (Eq. waterfilling-keys with the query embedded at its block).
+extern "C" aatc_status_t aatc_calibrate_head_group(int32_t g_h, int32_t group, const float* calib, int32_t n_calib,
+                                                   const float* calib_q, int32_t n_calib_q, double avg_bits,
+                                                   int32_t b_max, int32_t weights_mode, float* basis_out,
+                                                   uint8_t* bits_out, float* scales_out, double* sigma2_out,
+                                                   double* weights_out) {
+  using namespace aatc;
+  if (g_h < 1 || g_h > 8 || group < 1 || !calib || n_calib < 2 || !basis_out || !bits_out || !scales_out ||
+      (calib_q && n_calib_q < 1) || (weights_mode != 0 && weights_mode != 1) || b_max < 1 || b_max > 8)
+    return AATC_ERR_INVALID_ARG;
+  const int d = kD * g_h;
+  const double bd = avg_bits * d, br = std::nearbyint(bd);
+  if (!std::isfinite(bd) || std::fabs(bd - br) > 1e-9 || br < 0 || br > static_cast<double>(b_max) * d)
+    return AATC_ERR_BUDGET;
+  const int budget = static_cast<int>(br);
+  const size_t n = static_cast<size_t>(n_calib);
+  std::vector<float> x(n * d);                             // concatenated group vectors [n][d]
+  for (int m = 0; m < g_h; ++m)
+    for (size_t t = 0; t < n; ++t)
+      for (int i = 0; i < kD; ++i) x[t * d + m * kD + i] = calib[(m * n + t) * kD + i];
+  std::vector<double> c, v;
+  second_moment(x.data(), n_calib, c, d);
+  jacobi_eigen(c, v, d);
+  // eigenvalues descending (stable on the Jacobi index order), canonical signs
+  std::vector<int> ord(d);
+  std::iota(ord.begin(), ord.end(), 0);
+  std::stable_sort(ord.begin(), ord.end(),
+                   [&](int i, int j) { return c[static_cast<size_t>(i) * d + i] > c[static_cast<size_t>(j) * d + j]; });
+  std::vector<double> lam(d), u(static_cast<size_t>(d) * d);   // u[dim][k]
+  for (int k = 0; k < d; ++k) {
+    const int src = ord[k];
+    lam[k] = c[static_cast<size_t>(src) * d + src];
+    int imax = 0;
+    double amax = -1.0;
+    for (int r = 0; r < d; ++r) {
+      const double a = std::fabs(v[static_cast<size_t>(r) * d + src]);
+      if (a > amax) { amax = a; imax = r; }
+    }
+    const double sgn = v[static_cast<size_t>(imax) * d + src] < 0 ? -1.0 : 1.0;
+    for (int r = 0; r < d; ++r) u[static_cast<size_t>(r) * d + k] = sgn * v[static_cast<size_t>(r) * d + src];
+  }
+  std::vector<double> w(d, 1.0);
+  if (weights_mode == 0 && calib_q) {
+    std::fill(w.begin(), w.end(), 0.0);
+    std::vector<double> mj;
+    for (int j = 0; j < g_h * group; ++j) {
+      second_moment(calib_q + static_cast<size_t>(j) * n_calib_q * kD, n_calib_q, mj);
+      const int b0 = (j / group) * kD;                     // the query's kv-head block
+      for (int k = 0; k < d; ++k) {
+        double acc = 0.0;
+        for (int i = 0; i < kD; ++i) {
+          double row = 0.0;
+          for (int i2 = 0; i2 < kD; ++i2) row += mj[i * kD + i2] * u[static_cast<size_t>(b0 + i2) * d + k];
+          acc += u[static_cast<size_t>(b0 + i) * d + k] * row;
+        }
+        w[k] += acc;
+      }
+    }
+  }
+  std::vector<double> g(d);
+  for (int k = 0; k < d; ++k) g[k] = w[k] * lam[k];
+  std::vector<int> so(d);
+  std::iota(so.begin(), so.end(), 0);
+  std::stable_sort(so.begin(), so.end(), [&](int i, int j) { return g[i] > g[j]; });
+  std::vector<double> gs(d);
+  for (int c2 = 0; c2 < d; ++c2) gs[c2] = g[so[c2]];
+  std::vector<int> bits;
+  greedy_pool(gs, budget, b_max, bits);
+  std::vector<double> col(n);
+  for (int c2 = 0; c2 < d; ++c2) {
+    const int k = so[c2];
+    for (size_t t = 0; t < n; ++t) {
+      double h = 0.0;
+      for (int r = 0; r < d; ++r) h += static_cast<double>(x[t * d + r]) * u[static_cast<size_t>(r) * d + k];
+      col[t] = std::fabs(h);
+    }
+    scales_out[c2] = static_cast<float>(percentile99(col));
+    bits_out[c2] = static_cast<uint8_t>(bits[c2]);
+    for (int r = 0; r < d; ++r) basis_out[static_cast<size_t>(r) * d + c2] = static_cast<float>(u[static_cast<size_t>(r) * d + k]);
+    if (sigma2_out) sigma2_out[c2] = lam[k];
+    if (weights_out) weights_out[c2] = w[k];
+  }
   return AATC_OK;
 }
 

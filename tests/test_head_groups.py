@@ -136,3 +136,46 @@ def test_group_quantized_decode_error_falls_with_bits():
         errs.append(np.linalg.norm(got - exact) / (np.sqrt(np.mean(vg * vg) * D) * np.sqrt(len(q))))
     assert all(b < a for a, b in zip(errs, errs[1:])), errs
     assert errs[-1] < 0.01, errs
+
+
+def _distinct_spectra_heads(rng, g_h, n):
+    """g_h heads with different spectral decays and scales and a shared component (no
+    near-degenerate eigenvalues between heads), for comparing two eigen-solvers."""
+    heads = []
+    common = rng.standard_normal((n, D))
+    for m in range(g_h):
+        lam = (1.0 + 0.7 * m) * np.arange(1, D + 1, dtype=np.float64) ** -(1.2 + 0.17 * m)
+        basis = np.linalg.qr(rng.standard_normal((D, D)))[0]
+        own = (rng.standard_normal((n, D)) * np.sqrt(lam)) @ basis
+        heads.append(own + 0.3 * (common * np.sqrt(lam)) @ np.linalg.qr(rng.standard_normal((D, D)))[0])
+    return np.stack(heads).astype(np.float32)
+
+
+def test_library_head_group_planner_matches_oracle(aatc):
+    """aatc_calibrate_head_group against plan_head_group: bits exact, basis / scales to fp32
+    rounding, sigma^2 and weights to fp64 rounding (keys with query weights, values var-only)."""
+    rng = np.random.default_rng(7)
+    g_h, group, n, nq = 4, 4, 2048, 512
+    x = _distinct_spectra_heads(rng, g_h, n)
+    aniso = np.exp(-np.arange(D) / 40.0)
+    q = (rng.standard_normal((g_h * group, nq, D)) * aniso).astype(np.float32)
+    for qq, var in ((q, False), (None, True)):
+        lib = aatc.calibrate_head_group(x, qq, 2.75, group=group, var_only=var)
+        ref = O.plan_head_group(x.astype(np.float64), 2.75, queries_by_head=None if qq is None else list(qq.astype(np.float64)),
+                                group=group, weights="var" if var else "aatc")
+        np.testing.assert_array_equal(lib["bits"].astype(np.int64), ref["bits"])
+        np.testing.assert_allclose(lib["sigma2"], ref["sigma2"], rtol=1e-9, atol=1e-14)
+        np.testing.assert_allclose(lib["weights"], ref["weights"], rtol=1e-9, atol=1e-14)
+        np.testing.assert_allclose(lib["basis"], ref["basis"], rtol=0, atol=2e-6)
+        np.testing.assert_allclose(lib["scales"], ref["scales"], rtol=2e-6)
+
+
+def test_library_head_group_planner_rejects_bad_arguments(aatc):
+    x = np.zeros((2, 16, D), np.float32)
+    import pytest
+    with pytest.raises(aatc.AatcError):
+        aatc.calibrate_head_group(x[:, :1], None, 2.0)                # n_calib < 2
+    with pytest.raises(aatc.AatcError):
+        aatc.calibrate_head_group(x, None, 2.0 + 1.0 / 1000)         # budget not an integer
+    with pytest.raises(ValueError):
+        aatc.calibrate_head_group(x, np.zeros((3, 4, D), np.float32), 2.0, group=2)   # wrong query count
