@@ -36,6 +36,7 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
 
 // Block-wide max / sum of GP values per thread (128 threads).
 template <int GP, bool kMax>
@@ -879,64 +880,74 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4 r, float* o) {
   }
 }
 
+// bf16 tiles of 128 tokens x 128 dims in a ring of three, 256 B rows with the 16-byte chunks
+// XOR-swizzled by the row (chunk c of row r at chunk c ^ (r & 7)): the row-per-thread 128-bit
+// reads of the score pass and the row-shared 64-bit reads of the value pass are both free of
+// bank conflicts without padding.
+constexpr int kB16Stages = 3;
+constexpr int kB16Tile = TILE * D;                         // bf16 elements per tile
+
 template <int GP>
 __global__ void __launch_bounds__(kThreads)
     aatc_bf16_split_kernel(const Bf16Args a) {
   extern __shared__ __align__(16) float sm[];
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int G = a.group;
-  constexpr int kRow = D + 8;                              // padded bf16 row (272 B)
   float* qs = sm;                                          // [128][GP]
   float* red = qs + D * GP;                                // [32]
   float* sc = red + 32;                                    // [split_len][GP]
-  __nv_bfloat16* kt = reinterpret_cast<__nv_bfloat16*>(sc + a.split_len * GP);   // [2][128][kRow]
-  float* accs = reinterpret_cast<float*>(kt + 2 * TILE * kRow);                  // [4][GP][128]
+  __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(sc + a.split_len * GP);   // [3][128][128]
+  float* accs = reinterpret_cast<float*>(ring);            // [4][GP][128], over the drained ring
   const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
   const int tile_lo = static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
   const int tile_hi = static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
   const int t_begin = tile_lo * TILE;
   const int t_end = min(a.n_ctx, tile_hi * TILE);
   const int n_tiles_split = tile_hi - tile_lo;
+  const int n_seq = 2 * n_tiles_split;                     // key tiles, then value tiles
   const float scale = kLog2e * 0.08838834764831845f;
   for (int i = tid; i < GP * D; i += kThreads) {
     const int g = i / D, d = i % D;
     qs[d * GP + g] =
         g < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + g) * D + d]) * scale : 0.0f;
   }
-  auto stage = [&](const __nv_bfloat16* base, int tile, int buf) {
-    __nv_bfloat16* dst = kt + buf * TILE * kRow;
-    for (int i = tid; i < TILE * 16; i += kThreads) {
-      const int r = i >> 4, ch = i & 15;
-      int t = tile * TILE + r;
-      t = min(t, a.n_ctx - 1);                             // clamp padding rows to a valid token
-      cp_async16(dst + r * kRow + ch * 8, base + ((static_cast<size_t>(b) * a.max_tokens + t) * a.n_kv + head) * D + ch * 8);
+  const int tile0 = t_begin / TILE;
+  auto stage_seq = [&](int i) {                            // tile i of the sequence into buffer i % 3
+    const __nv_bfloat16* base = i < n_tiles_split ? a.k : a.v;
+    const int tile = tile0 + (i < n_tiles_split ? i : i - n_tiles_split);
+    __nv_bfloat16* dst = ring + (i % kB16Stages) * kB16Tile;
+    for (int e = tid; e < TILE * 16; e += kThreads) {
+      const int r = e >> 4, ch = e & 15;
+      const int t = min(tile * TILE + r, a.n_ctx - 1);     // padding rows: a valid token, masked later
+      cp_async16(dst + r * D + ((ch ^ (r & 7)) << 3),
+                 base + ((static_cast<size_t>(b) * a.max_tokens + t) * a.n_kv + head) * D + ch * 8);
     }
     cp_async_commit();
   };
-  const int tile0 = t_begin / TILE;
-  // key tiles, then value tiles, stream through the two buffers: the first value tile is in
-  // flight during the last key tile and the softmax in between
-  auto stage_seq = [&](int i, int buf) {
-    if (i < n_tiles_split) stage(a.k, tile0 + i, buf);
-    else stage(a.v, tile0 + i - n_tiles_split, buf);
+  // before tile i: it has landed (tile i + 1 may still be in flight), every thread is past tile
+  // i - 1, and tile i + 2 goes into the buffer tile i - 1 used
+  auto next_tile = [&](int i) {
+    if (i + 1 < n_seq) cp_async_wait_one(); else cp_async_wait_all();
+    __syncthreads();
+    if (i + 2 < n_seq) stage_seq(i + 2);
+    return ring + (i % kB16Stages) * kB16Tile;
   };
-  stage_seq(0, 0);
-  __syncthreads();
+  stage_seq(0);
+  if (n_seq > 1) stage_seq(1);
+  __syncthreads();                                         // query columns visible
   float mloc[GP];
 #pragma unroll
   for (int g = 0; g < GP; ++g) mloc[g] = -INFINITY;
   for (int ti = 0; ti < n_tiles_split; ++ti) {
-    const int buf = ti & 1;
-    cp_async_wait_all();
-    __syncthreads();
-    stage_seq(ti + 1, buf ^ 1);                            // the next key tile, or value tile 0
-    const __nv_bfloat16* row = kt + buf * TILE * kRow + tid * kRow;
+    const __nv_bfloat16* row = next_tile(ti) + tid * D;   // thread = token tid of the tile
     float s[GP];
 #pragma unroll
     for (int g = 0; g < GP; ++g) s[g] = 0.0f;
-    for (int d0 = 0; d0 < D; d0 += 8) {
+#pragma unroll 4
+    for (int c = 0; c < 16; ++c) {
       float kv[8];
-      bf16x8_to_f32(*reinterpret_cast<const uint4*>(row + d0), kv);
+      bf16x8_to_f32(*reinterpret_cast<const uint4*>(row + ((c ^ (tid & 7)) << 3)), kv);
+      const int d0 = 8 * c;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
@@ -973,19 +984,17 @@ __global__ void __launch_bounds__(kThreads)
   }
   block_reduce<GP, false>(lsum, red);
   const int dg = tid & 31, tq = tid >> 5;
+  const int dch = dg >> 1, dsub = 4 * (dg & 1);            // dims 4 dg .. 4 dg + 3: chunk, position
   float acc[GP][4];
 #pragma unroll
   for (int g = 0; g < GP; ++g)
 #pragma unroll
     for (int i = 0; i < 4; ++i) acc[g][i] = 0.0f;
   for (int ti = 0; ti < n_tiles_split; ++ti) {
-    const int buf = (n_tiles_split + ti) & 1;
-    cp_async_wait_all();
-    __syncthreads();
-    if (ti + 1 < n_tiles_split) stage_seq(n_tiles_split + ti + 1, buf ^ 1);
+    const __nv_bfloat16* vt = next_tile(n_tiles_split + ti);
     const int tend = min(TILE, t_end - (tile0 + ti) * TILE);
     for (int tt = tq; tt < tend; tt += 4) {
-      const uint2 r = *reinterpret_cast<const uint2*>(kt + buf * TILE * kRow + tt * kRow + dg * 4);
+      const uint2 r = *reinterpret_cast<const uint2*>(vt + tt * D + ((dch ^ (tt & 7)) << 3) + dsub);
       const float vv[4] = {__uint_as_float(r.x << 16), __uint_as_float(r.x & 0xFFFF0000u),
                            __uint_as_float(r.y << 16), __uint_as_float(r.y & 0xFFFF0000u)};
       const float* p = sc + (ti * TILE + tt) * GP;
@@ -1001,7 +1010,7 @@ __global__ void __launch_bounds__(kThreads)
     }
   }
   cp_async_wait_all();
-  __syncthreads();
+  __syncthreads();                                         // ring drained: accs may overwrite it
 #pragma unroll
   for (int g = 0; g < GP; ++g)
     *reinterpret_cast<float4*>(accs + (tq * GP + g) * D + dg * 4) = make_float4(acc[g][0], acc[g][1], acc[g][2], acc[g][3]);
@@ -1239,10 +1248,10 @@ cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int b
 }
 
 size_t bf16_split_smem(int gp, int split_len) {
-  // query columns [128][gp], reduction scratch, scores [split_len][gp], per-quarter sums
-  // [4][gp][128] (fp32); two padded bf16 tiles [128][136]
-  return 4 * (static_cast<size_t>(D) * gp + 32 + static_cast<size_t>(split_len) * gp + 4 * static_cast<size_t>(gp) * D) +
-         2 * static_cast<size_t>(TILE) * (D + 8) * 2;
+  // query columns [128][gp], reduction scratch, scores [split_len][gp] (fp32); a ring of three
+  // bf16 tiles [128][128], which the per-quarter sums [4][gp][128] reuse at the end
+  return 4 * (static_cast<size_t>(D) * gp + 32 + static_cast<size_t>(split_len) * gp) +
+         static_cast<size_t>(kB16Stages) * TILE * D * 2;
 }
 
 cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx, int max_tokens,
