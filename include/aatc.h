@@ -318,6 +318,15 @@ aatc_status_t aatc_dequantize(aatc_plan_t plan, int32_t layer, const void* cache
                               int32_t t0, int32_t n, int32_t max_tokens, float* coeffs_out,
                               void* stream);
 
+/*
+ * Test hook for failure detection without a GPU fault: launches one CTA that waits on an mbarrier
+ * nothing arrives on, with the bounded wait every kernel of this library uses, limited to
+ * limit_us microseconds.  The wait runs out, the kernel sets bit 1 (value 2) of *dev_flags (a
+ * device int32 the caller zeroes) as the library's kernels do on a timeout, and returns normally.
+ * Errors: AATC_ERR_INVALID_ARG (null flags, limit outside 1 .. 2 000 000 us), AATC_ERR_CUDA.
+ */
+aatc_status_t aatc_selftest_bounded_wait(int32_t limit_us, int32_t* dev_flags, void* stream);
+
 /* Sticky device error flags of the plan (bit 0: non-finite token scale seen by encode;
  * bit 1: a bounded wait inside a kernel timed out).  Synchronizes; clear != 0 resets them. */
 aatc_status_t aatc_get_device_error(aatc_plan_t plan, int32_t* flags, int32_t clear);

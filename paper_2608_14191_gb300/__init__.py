@@ -47,6 +47,7 @@ SIGNATURES = {
     "aatc_version": (_I32, []),
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
     "aatc_calibrate_head_group": (_I32, [_I32, _I32, _P, _I32, _P, _I32, _F64, _I32, _I32, _P, _P, _P, _P, _P]),
+    "aatc_selftest_bounded_wait": (_I32, [_I32, _P, _P]),
     "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
     "aatc_whitening_transform": (_I32, [_I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "aatc_hidden_operand": (_I32, [ctypes.POINTER(Dims), _I32, _P, _P, _P, _P]),
@@ -164,6 +165,13 @@ def calibrate_head_group(calib: np.ndarray, calib_q: np.ndarray | None, avg_bits
                                             1 if var_only else 0, _ptr(basis), _ptr(bits), _ptr(scales),
                                             _ptr(sigma2), _ptr(weights)), "aatc_calibrate_head_group")
     return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
+
+
+def selftest_bounded_wait(limit_us: int, flags, stream=None):
+    """aatc_selftest_bounded_wait: a kernel whose bounded wait runs out (nothing arrives); it sets
+    bit 1 of the device int32 `flags` (a torch tensor) and returns."""
+    _check(load().aatc_selftest_bounded_wait(int(limit_us), _ptr(flags), _stream(stream)),
+           "aatc_selftest_bounded_wait")
 
 
 def allocate_global(dm: Dims, sigma2: np.ndarray, weights: np.ndarray, avg_bits_k: float,

@@ -46,15 +46,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase with the given parity to complete, for at most ~1 s of wall time.
-// Returns false on timeout or when another role of the CTA raised `abort_flag`.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+// Wait for the phase with the given parity to complete, for at most limit_ns of wall time (~1 s
+// by default).  Returns false on timeout or when another role of the CTA raised `abort_flag`.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                                  uint64_t limit_ns = 1000000000ull) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > 1000000000ull) return false;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
   }
 }
 

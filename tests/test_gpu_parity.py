@@ -130,6 +130,30 @@ def test_nonfinite_input_sets_device_flag(aatc, tiny):
     assert case.plan.device_error() == 0
 
 
+def test_bounded_wait_times_out_with_error_status(aatc, tiny):
+    """A wait on an mbarrier that nothing arrives on gives up after its limit (here 2 ms), sets bit
+    1 of the device flags and returns; the context stays usable (a decode afterwards still
+    matches the one before)."""
+    case, k, v, cache = tiny
+    q = torch.from_numpy(W.to_bf16(np.random.default_rng(3).standard_normal((1, case.cfg.n_q_heads, 128)))).to(DEV).to(torch.bfloat16)
+    before = aatc.decode_attention(case.plan, 0, q, cache, case.cfg.n_ctx, case.cfg.n_ctx).clone()
+    flags = torch.zeros(1, dtype=torch.int32, device=DEV)
+    s = torch.cuda.current_stream()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(s)
+    aatc.selftest_bounded_wait(2000, flags, s)
+    t1.record(s)
+    torch.cuda.synchronize()
+    assert int(flags.item()) == 2
+    assert 1.9 <= t0.elapsed_time(t1) < 500.0
+    after = aatc.decode_attention(case.plan, 0, q, cache, case.cfg.n_ctx, case.cfg.n_ctx)
+    torch.cuda.synchronize()
+    assert torch.equal(before, after)
+    assert case.plan.device_error() == 0
+    with pytest.raises(aatc.AatcError):
+        aatc.selftest_bounded_wait(0, flags, s)
+
+
 def test_argument_errors_leave_outputs_untouched(aatc, tiny):
     case, k, v, cache = tiny
     q = torch.zeros((1, 4, 128), dtype=torch.bfloat16, device=DEV)
