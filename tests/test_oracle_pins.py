@@ -108,6 +108,19 @@ def test_greedy_integer_local_optimality_and_monotone():
                     assert O.allocation_objective(g, bb) >= base * (1 - 1e-12)
 
 
+def test_greedy_saturates_at_b_max():
+    """A budget of at least d b_max bits fills every channel to b_max and no further (widths in
+    {0..b_max}, Eq. waterfilling-keys); a budget of d b_max - 1 leaves exactly the channel with
+    the smallest g one bit short."""
+    g = np.exp(np.random.default_rng(4).normal(0, 3, 16))
+    for b_max in (1, 3, 8):
+        np.testing.assert_array_equal(O.greedy_allocation(g, 16 * b_max + 40, b_max), np.full(16, b_max))
+        short = O.greedy_allocation(g, 16 * b_max - 1, b_max)
+        want = np.full(16, b_max)
+        want[int(np.argmin(g))] -= 1
+        np.testing.assert_array_equal(short, want)
+
+
 # --- (4) Theorem 1: D ~= D_K + D_V under the white-noise model -------------------------------
 
 def test_theorem1_monte_carlo():
@@ -262,6 +275,21 @@ def test_percentile_definition():
     assert O.percentile_linear(np.array([2.0, 0.0]), 50) == 1.0
 
 
+def test_channel_scale_is_p99_of_magnitudes():
+    """s_c is the 99th percentile of |h_c| over the calibration tokens (Sec. 5): with the identity
+    basis and a column holding -100 .. 0 (magnitudes 0 .. 100, 101 samples) it is exactly 99; a
+    column of +-1 gives 1; a scaled column scales s_c."""
+    x = np.zeros((101, O.D))
+    x[:, 0] = -np.arange(101.0)[::-1]
+    x[:, 1] = np.where(np.arange(101) % 2 == 0, 1.0, -1.0)
+    x[:, 2] = 0.5 * np.arange(101.0)
+    s = O.channel_scales(np.eye(O.D), x)
+    assert s[0] == pytest.approx(99.0, rel=1e-15)
+    assert s[1] == 1.0
+    assert s[2] == pytest.approx(49.5, rel=1e-15)
+    assert np.all(s[3:] == 0.0)
+
+
 # --- decode = SDPA over reconstructed keys and values (Alg. 1, Def. sdpa) ----------------------
 
 def test_decode_matches_library_sdpa():
@@ -360,6 +388,42 @@ def test_dequantize_f32_is_two_roundings():
     f1 = np.float32(0.7) * np.float32(2.0 ** -1)
     assert got[0, 0] == np.float32(np.float32(3) * np.float32(alpha[0] * f0))
     assert got[0, 1] == np.float32(np.float32(-2) * np.float32(alpha[0] * f1))
+
+
+def _rn32(x):
+    """Round an exact rational to the nearest fp32 value, ties to even (normal range), with
+    integer arithmetic only."""
+    from fractions import Fraction
+    if x == 0:
+        return Fraction(0)
+    sign, x = (-1 if x < 0 else 1), abs(x)
+    e = x.numerator.bit_length() - x.denominator.bit_length()
+    e += 1 if Fraction(2) ** (e + 1) <= x else 0
+    e -= 1 if Fraction(2) ** e > x else 0
+    ulp = Fraction(2) ** (e - 23)
+    m = x / ulp
+    fl = m.numerator // m.denominator
+    rem = m - fl
+    if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and fl % 2 == 1):
+        fl += 1
+    return sign * fl * ulp
+
+
+def test_dequantize_f32_rounding_order_exact_rationals():
+    """The two roundings fl32(code * fl32(alpha f_c)) checked in exact rational arithmetic, on
+    inputs where one rounding of the exact product code * alpha * f_c gives a different fp32
+    value (so the order of the roundings is what the case decides)."""
+    from fractions import Fraction
+    cases = [(1081809706, 1088184628, 8, 38), (1080294143, 1075205050, 6, 7), (1075107180, 1078175588, 8, 44)]
+    for a_bits, s_bits, b, code in cases:
+        alpha = np.array([a_bits], np.uint32).view(np.float32)
+        scale = np.array([s_bits], np.uint32).view(np.float32)
+        f = Fraction(float(scale[0])) * Fraction(2) ** (1 - b)
+        two = _rn32(code * _rn32(Fraction(float(alpha[0])) * f))
+        one = _rn32(code * Fraction(float(alpha[0])) * f)
+        assert two != one
+        got = O.dequantize_f32(np.array([[code]]), alpha, scale, np.array([b]))
+        assert Fraction(float(got[0, 0])) == two
 
 
 # --- prefill attention over the coded cache (Def. sdpa with a causal chunk of queries) ----------
