@@ -403,6 +403,75 @@ def prefill_timing(aatc, device, iters=2, batch=None, reference=True):
                         f"causal prefill over the packed cache (2.75 bits)"}
 
 
+def sweep_timing(aatc, device, n_calls=32, reps=3, enc_iters=6):
+    """Bit-budget sweep on the Llama shape at batch 4 x 32768 tokens: per budget (1.5 / 2 / 2.75 /
+    4 bits) a plan, the encode of all K/V (536.9 MB of bf16 input, > L2) and the decode (a CUDA
+    graph of calls alternating two packed-cache copies), against the bf16 reference decode of the
+    same K/V and queries.  The speed-up is bounded by the byte ratio 512 / (sum b / 8 + 4)."""
+    import torch
+    cfg = W.CONFIGS["sweep"]
+    B, T = cfg.batch, cfg.n_ctx
+    kd, vd = W.kv_device(cfg, 0, B, T, device)
+    qs = W.queries_device(cfg, 0, B, 4, device)
+    stream = torch.cuda.current_stream()
+    peak, _ = _peaks()
+    ref = bf16_decode_timing(aatc, kd, vd, qs, T, 1.0, n_calls=n_calls, reps=reps)
+    in_bytes = (kd.numel() + vd.numel()) * 2
+
+    def timed(fn, iters):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(iters):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / iters              # us per iteration
+
+    rows = []
+    for bits in cfg.avg_bits:
+        plan, _ = build_case(aatc, cfg, bits, device)
+        caches = [plan.new_cache(B, T, device) for _ in range(2)]
+        ctr = [0]
+
+        def enc():
+            aatc.encode(plan, 0, kd, vd, caches[ctr[0] & 1], 0, T)
+            ctr[0] += 1
+
+        enc_us = timed(enc, enc_iters)
+        for c in caches:
+            aatc.encode(plan, 0, kd, vd, c, 0, T)
+        out = torch.empty((B, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
+        ws = torch.empty(max(1, plan.workspace_bytes(B, T) // 4), dtype=torch.float32, device=device)
+
+        def calls():
+            for i in range(n_calls):
+                aatc.decode_attention(plan, 0, qs[i % qs.shape[0]], caches[i & 1], T, T, out=out, workspace=ws)
+
+        calls()
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            calls()
+        dec_us = timed(graph.replay, reps) / n_calls
+        nbytes = decode_bytes(plan, cfg, B, T)
+        per_token = nbytes / (B * T * cfg.n_kv_heads)
+        rows.append({"avg_bits": bits, "bytes_per_token_kvhead": per_token,
+                     "encode_us": round(enc_us, 2), "encode_mtok_s": round(B * T / enc_us, 2),
+                     "encode_input_gbs": round(in_bytes / (enc_us * 1e-6) / 1e9, 2),
+                     "decode_us": round(dec_us, 3), "decode_gbs": round(nbytes / (dec_us * 1e-6) / 1e9, 2),
+                     "decode_frac_of_measured_hbm": round(nbytes / (dec_us * 1e-6) / 1e9 / peak, 4),
+                     "speedup_vs_bf16": round(ref["us_per_call"] / dec_us, 3),
+                     "byte_ratio_vs_bf16": round(512.0 / per_token, 3)})
+        del graph
+        plan.close()
+    return {"workload": cfg.workload, "bf16_decode_us": ref["us_per_call"], "bf16_decode_gbs": ref["gbs"],
+            "budgets": rows,
+            "timing": f"encode: {enc_iters} calls alternating two caches; decode: {n_calls}-call CUDA graph x {reps}, "
+                      "two packed-cache copies alternating; bf16: two K/V copies alternating (537 MB each)"}
+
+
 def planner_timing(aatc):
     """Host planner rows: the global cross-layer allocation on Llama-3.1-8B-shaped statistics
     (32 layers x 8 kv-heads x K|V x 128 channels; seeded log-normal spectra), median of 5 runs."""
@@ -585,6 +654,7 @@ def run_ours(args):
     stack = stack_decode_timing(aatc, dev)
     hid = hidden_encode_timing(aatc, dev)
     pre = prefill_timing(aatc, dev)
+    sweep = sweep_timing(aatc, dev)
 
     peak, peak_kind = _peaks()
     dbytes = decode_bytes(plan, cfg, B, T)
@@ -636,6 +706,7 @@ def run_ours(args):
         "decode_llama_stack": stack,
         "encode_hidden": hid,
         "prefill": pre,
+        "sweep": sweep,
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds)
