@@ -205,7 +205,7 @@ aatc_status_t aatc_plan_info(aatc_plan_t plan, int32_t* n_words, int32_t* retain
  * Bytes of one layer's packed cache for `batch` sequences of capacity max_tokens:
  *   uint32 words [batch][H_kv][2][n_tiles][W][128], then fp32 alpha [batch][H_kv][2][n_tiles*128],
  *   n_tiles = ceil(max_tokens / 128).  Token t of a sequence lives in tile t/128, lane t%128
- *   (build-defined layout: the paper leaves the storage format open).
+ *   (library-defined layout: the paper leaves the storage format open).
  */
 aatc_status_t aatc_cache_bytes(aatc_plan_t plan, int32_t batch, int32_t max_tokens, size_t* bytes);
 

@@ -29,7 +29,7 @@ into the heads' own eigenbases, the budget identity, and the transform-coding
 gain of one group transform over separate heads for correlated heads.
 
 parity unpinned: the packed record bit layout (:func:`record_entries`,
-:func:`pack_records`, :func:`cache_records`) is defined by this build, not by the
+:func:`pack_records`, :func:`cache_records`) is defined by this library, not by the
 paper, which prints no worked encoding.  It is pinned only by the round trip
 unpack(pack(c)) == c, the record-size identity (352 code bits per token and stream
 at 2.75 bits, i.e. the paper's 16/2.75 = 5.82x, in exactly 11 words) and
@@ -57,7 +57,7 @@ def second_moment(x: np.ndarray) -> np.ndarray:
 def canonical_sign(vectors: np.ndarray) -> np.ndarray:
     """Flip each column so that its largest-magnitude entry (lowest index on ties) is positive.
 
-    The paper leaves eigenvector signs open; this is the build's convention.
+    The paper leaves eigenvector signs open; this is the library's convention.
     """
     v = np.array(vectors, dtype=np.float64, copy=True)
     for j in range(v.shape[1]):
@@ -323,7 +323,7 @@ def dequantize_f32(codes: np.ndarray, alpha_f32: np.ndarray, scales_f32: np.ndar
 
 
 # ----------------------------------------------------------------------------
-# Packed layout (build-defined; the paper prints none)
+# Packed layout (library-defined; the paper prints none)
 #
 # Each stored code is u = code + 2^(b-1) (offset binary, b bits).  The record of one token
 # and stream splits u into base-4 digits and single top bits, grouped by significance:

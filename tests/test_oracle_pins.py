@@ -324,7 +324,7 @@ def test_decode_special_cases():
     np.testing.assert_allclose(out[0], u @ hv[0].mean(axis=0), atol=1e-12)
 
 
-# --- packed layout (build-defined) and the paper's compression figure -------------------------
+# --- packed layout (library-defined) and the paper's compression figure -------------------------
 
 @pytest.mark.parametrize("case", _gold("packing_examples.json")["cases"])
 def test_pack_hand_examples(case):
