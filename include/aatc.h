@@ -32,7 +32,8 @@ extern "C" {
 #endif
 
 #define AATC_HEAD_DIM 128
-#define AATC_MAX_BITS 8      /* widest channel code (bits); widths are 0..AATC_MAX_BITS */
+#define AATC_MAX_BITS 8        /* widest channel code a device plan holds; widths 0..AATC_MAX_BITS */
+#define AATC_MAX_PLAN_BITS 16  /* widest width the host planner allocates (Sec. 5 allows b in 0..16) */
 
 typedef struct aatc_plan_s* aatc_plan_t;   /* opaque; immutable after creation */
 
@@ -48,7 +49,9 @@ typedef enum {
   AATC_ERR_DEVICE_FLAG = 8    /* reserved for callers that turn device flags into status */
 } aatc_status_t;
 
-/* Model dimensions.  d must be 128; n_q_heads % n_kv_heads == 0; b_max in 1..8. */
+/* Model dimensions.  d must be 128; n_q_heads % n_kv_heads == 0; b_max in 1..AATC_MAX_PLAN_BITS for
+ * the host planner calls, in 1..AATC_MAX_BITS for aatc_plan_create (wider plans are
+ * AATC_ERR_UNSUPPORTED: the record layout and kernels take widths up to 8). */
 typedef struct {
   int32_t d;
   int32_t n_layers;
@@ -112,7 +115,8 @@ aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k, cons
  *   basis_out  : host fp32 [d][d] (dim x channel); bits_out uint8 [d]; scales_out fp32 [d];
  *   sigma2_out, weights_out : host fp64 [d] or NULL
  * Errors: AATC_ERR_INVALID_ARG (g_h outside 1..8, group < 1, n_calib < 2, null outputs, b_max
- * outside 1..8), AATC_ERR_BUDGET (avg_bits * d not an integer in [0, b_max d]).  Host only.
+ * outside 1..AATC_MAX_PLAN_BITS), AATC_ERR_BUDGET (avg_bits * d not an integer in [0, b_max d]).
+ * Host only.
  * The plan, encode and decode kernels take per-kv-head streams; head-group streams are planned
  * here and checked against the oracle, and their device path is not built yet.
  */
@@ -189,7 +193,9 @@ aatc_status_t aatc_hidden_operand(const aatc_dims_t* dims, int32_t d_model, cons
  * bf16 encode basis (round-to-nearest-even of `basis`), and uploads everything with one
  * copy on `stream`, then synchronizes it.  Host inputs are copied; the caller keeps them.
  * Errors: AATC_ERR_INVALID_ARG (null, bits > b_max, bits not non-increasing, scale <= 0 or
- * non-finite where bits > 0, non-finite basis), AATC_ERR_CUDA, AATC_ERR_NOMEM.
+ * non-finite where bits > 0, non-finite basis), AATC_ERR_UNSUPPORTED (dims->b_max above
+ * AATC_MAX_BITS: a plan the planner made with wider widths), AATC_ERR_CUDA, AATC_ERR_NOMEM.
+ * All argument checks run before any CUDA call.
  */
 aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
                                const float* scales, void* stream, aatc_plan_t* plan_out);

@@ -191,7 +191,7 @@ def global_allocation(sigma2: np.ndarray, weights: np.ndarray, avg_bits_k: float
     one bit per channel more (keys, capped at b_max d); the rest of the kind's total budget
     avg_bits * d * L * H is water-filled over every channel of the other layers at once, with
     sigma^2 and w each divided by the layer's own 95th percentile over its channels (all kv-heads).
-    Reading: b_max stays the plan's 8 (the paper allows 16).
+    b_max: 8 for what a device plan holds; the paper allows 16, which the planner also takes.
     """
     sigma2 = np.asarray(sigma2, np.float64)
     weights = np.asarray(weights, np.float64)
@@ -327,7 +327,7 @@ def dequantize_f32(codes: np.ndarray, alpha_f32: np.ndarray, scales_f32: np.ndar
 #
 # Each stored code is u = code + 2^(b-1) (offset binary, b bits).  The record of one token
 # and stream splits u into base-4 digits and single top bits, grouped by significance:
-#   D2 = for k = 0..3: digit k (bits 2k, 2k+1) of every channel with b >= 2k+2
+#   D2 = for k = 0..7: digit k (bits 2k, 2k+1) of every channel with b >= 2k+2 (b up to 16)
 #   D1 = the top bit (bit b-1) of every odd-width channel, in channel order
 # Channels are in storage order (widths non-increasing), so each D2 layer is a prefix.  If |D2| is not a multiple of 16, its last |D2| mod 16
 # entries move to the end of D1 as two single bits each.  Record words: the D2 entries at
@@ -338,8 +338,9 @@ def dequantize_f32(codes: np.ndarray, alpha_f32: np.ndarray, scales_f32: np.ndar
 def record_entries(bits: np.ndarray):
     """(D2, D1): lists of (channel, bit shift) entries of one stream's record."""
     b = [int(x) for x in bits]
+    assert max(b, default=0) <= 16
     d2 = []
-    for k in range(4):
+    for k in range(8):
         d2 += [(c, 2 * k) for c in range(len(b)) if b[c] >= 2 * k + 2]
     d1 = [(c, b[c] - 1) for c in range(len(b)) if b[c] % 2 == 1]
     r = len(d2) % 16

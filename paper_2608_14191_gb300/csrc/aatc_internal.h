@@ -80,9 +80,11 @@ struct Plan {
   bool tmap_ok = false;
 };
 
+// Shape check shared by the planner (widths up to AATC_MAX_PLAN_BITS) and plan creation, which
+// also rejects b_max > AATC_MAX_BITS as unsupported.
 inline bool valid_dims(const aatc_dims_t* d) {
   return d && d->d == D && d->n_layers >= 1 && d->n_kv_heads >= 1 && d->n_q_heads >= d->n_kv_heads &&
-         d->n_q_heads % d->n_kv_heads == 0 && d->b_max >= 1 && d->b_max <= AATC_MAX_BITS &&
+         d->n_q_heads % d->n_kv_heads == 0 && d->b_max >= 1 && d->b_max <= AATC_MAX_PLAN_BITS &&
          d->n_layers <= 4096 && d->n_q_heads <= 4096;
 }
 

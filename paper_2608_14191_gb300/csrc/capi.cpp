@@ -155,6 +155,7 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
                                const float* scales, void* stream, aatc_plan_t* plan_out) {
   using namespace aatc;
   if (!valid_dims(dims) || !basis || !bits || !scales || !plan_out) return AATC_ERR_INVALID_ARG;
+  if (dims->b_max > AATC_MAX_BITS) return AATC_ERR_UNSUPPORTED;   // records hold widths up to 8
   const int S = dims->n_layers * dims->n_kv_heads * 2;
   const size_t SD = static_cast<size_t>(S) * D;
   // validate

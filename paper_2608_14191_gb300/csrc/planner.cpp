@@ -302,7 +302,8 @@ extern "C" aatc_status_t aatc_calibrate_head_group(int32_t g_h, int32_t group, c
                                                    double* weights_out) {
   using namespace aatc;
   if (g_h < 1 || g_h > 8 || group < 1 || !calib || n_calib < 2 || !basis_out || !bits_out || !scales_out ||
-      (calib_q && n_calib_q < 1) || (weights_mode != 0 && weights_mode != 1) || b_max < 1 || b_max > 8)
+      (calib_q && n_calib_q < 1) || (weights_mode != 0 && weights_mode != 1) || b_max < 1 ||
+      b_max > AATC_MAX_PLAN_BITS)
     return AATC_ERR_INVALID_ARG;
   const int d = kD * g_h;
   const double bd = avg_bits * d, br = std::nearbyint(bd);

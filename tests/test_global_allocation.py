@@ -94,6 +94,19 @@ def test_library_global_allocation_matches_oracle(aatc, L, H, n_protect, avg):
     assert np.array_equal(got.astype(np.int64), want)
 
 
+@pytest.mark.parametrize("L,H,n_protect,avg", [(5, 2, 3, 6.0), (4, 2, 0, 9.0)])
+def test_library_global_allocation_up_to_16_bits_matches_oracle(aatc, L, H, n_protect, avg):
+    """Widths in {0..16} (the paper's range): the pool gives some channels more than 8 bits and
+    the library still matches the oracle bit for bit."""
+    rng = np.random.default_rng(200 + L * 10 + H)
+    s2, w = _random_stats(rng, L, H, 128, layer_scale=np.exp(rng.normal(0, 2, L)))
+    dm = aatc.dims(L, H, 4 * H, b_max=16)
+    got = aatc.allocate_global(dm, s2, w, avg, avg, n_protect=n_protect).astype(np.int64)
+    want = O.global_allocation(s2, w, avg, avg, n_protect=n_protect, b_max=16)
+    assert np.array_equal(got, want)
+    assert got.max() > 8 and got.max() <= 16
+
+
 def test_library_global_allocation_rejects_bad_budgets(aatc):
     rng = np.random.default_rng(3)
     s2, w = _random_stats(rng, 4, 2, 128)

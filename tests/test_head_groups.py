@@ -170,6 +170,18 @@ def test_library_head_group_planner_matches_oracle(aatc):
         np.testing.assert_allclose(lib["scales"], ref["scales"], rtol=2e-6)
 
 
+def test_library_head_group_planner_up_to_16_bits(aatc):
+    """Two kv-heads (256 channels) at 6 bits with b_max = 16: bits match the oracle exactly and the
+    leading channels take more than 8 bits."""
+    rng = np.random.default_rng(8)
+    x = _distinct_spectra_heads(rng, 2, 1024)
+    lib = aatc.calibrate_head_group(x, None, 6.0, b_max=16)
+    ref = O.plan_head_group(x.astype(np.float64), 6.0, b_max=16)
+    got = lib["bits"].astype(np.int64)
+    np.testing.assert_array_equal(got, ref["bits"])
+    assert got.sum() == 6 * 256 and 8 < got.max() <= 16
+
+
 def test_library_head_group_planner_rejects_bad_arguments(aatc):
     x = np.zeros((2, 16, D), np.float32)
     import pytest

@@ -89,6 +89,20 @@ def test_greedy_matches_brute_force_d4():
         assert O.allocation_objective(g, got) == pytest.approx(best, rel=1e-12), (g, budget)
 
 
+def test_greedy_matches_brute_force_d3_up_to_16_bits():
+    """The paper's widths b in {0..16}: exhaustive search over 17^3 allocations at d = 3."""
+    rng = np.random.default_rng(12)
+    grid = np.array(list(itertools.product(range(17), repeat=3)))
+    for trial in range(40):
+        g = np.exp(rng.normal(0, 6, 3))
+        budget = int(rng.integers(0, 49))
+        ok = grid.sum(axis=1) <= budget
+        best = np.min(np.sum(g[None, :] * 4.0 ** -grid[ok], axis=1))
+        got = O.greedy_allocation(g, budget, 16)
+        assert got.sum() == budget and got.max() <= 16
+        assert O.allocation_objective(g, got) == pytest.approx(best, rel=1e-12), (g, budget)
+
+
 def test_greedy_integer_local_optimality_and_monotone():
     """Exchange optimality of the integer allocation: moving one bit between any two channels
     never lowers the objective; with g sorted descending the widths are non-increasing."""
@@ -219,7 +233,7 @@ def test_key_weights_gqa_hand_example():
 def test_quantizer_error_bound_and_clamp():
     rng = np.random.default_rng(9)
     s = np.ones(O.D)
-    for b in (1, 2, 3, 5, 8):
+    for b in (1, 2, 3, 5, 8, 12, 16):
         bits = np.full(O.D, b)
         h = rng.uniform(-1, 1, (400, O.D))
         alpha = O.token_scale(h, s, bits)
@@ -229,9 +243,12 @@ def test_quantizer_error_bound_and_clamp():
         assert codes.min() >= -2 ** (b - 1) and codes.max() <= 2 ** (b - 1) - 1
         top = codes == 2 ** (b - 1) - 1
         err = np.abs(h - hhat)
-        # within range error <= Delta/2; at the clamped positive extreme error <= Delta
-        assert np.all(err[~top] <= delta.repeat(O.D, 1)[~top] / 2 * (1 + 1e-12))
-        assert np.all(err <= delta.repeat(O.D, 1) * (1 + 1e-12))
+        # within range error <= Delta/2; at the clamped positive extreme error <= Delta (slack: the
+        # fp64 rounding of h - h_hat, ~2^-52 |h|, with |h| up to 2^(b-1) Delta)
+        slack = 1e-15 * np.abs(h)
+        dd = delta.repeat(O.D, 1)
+        assert np.all(err[~top] <= dd[~top] / 2 * (1 + 1e-12) + slack[~top])
+        assert np.all(err <= dd * (1 + 1e-12) + slack)
         # the argmax coefficient sits exactly at +-2^(b-1) steps
         tmax = np.max(np.abs(h), axis=1) / delta[:, 0]
         np.testing.assert_allclose(tmax, 2.0 ** (b - 1), rtol=1e-12)
@@ -335,10 +352,12 @@ def test_pack_hand_examples(case):
     assert O.unpack_records(words, bits).tolist() == [case["codes"]]
 
 
-def test_pack_round_trip_random():
-    rng = np.random.default_rng(14)
+@pytest.mark.parametrize("b_hi", [9, 17])
+def test_pack_round_trip_random(b_hi):
+    """Widths up to 8 (device plans) and up to 16 (the planner's range)."""
+    rng = np.random.default_rng(14 + b_hi)
     for _ in range(20):
-        bits = np.sort(rng.integers(0, 9, O.D))[::-1]
+        bits = np.sort(rng.integers(0, b_hi, O.D))[::-1]
         half = np.where(bits > 0, 2 ** np.maximum(bits - 1, 0), 0)
         codes = np.where(bits > 0, rng.integers(-half, np.maximum(half, 1), (64, O.D)), 0)
         nw = O.record_words([bits])

@@ -58,3 +58,20 @@ def test_planner_layout_identity(aatc):
     assert np.all(np.diff(b, axis=1) <= 0)
     assert np.all(b.sum(axis=1) == 352)
     assert O.record_words(list(b)) == 11
+
+
+def test_planner_up_to_16_bits_matches_oracle(aatc):
+    """b_max = 16 (Sec. 5 allows b in 0..16): at 7 average bits the leading channels take more
+    than 8 bits; widths match the oracle exactly and the budget is met."""
+    cfg = W.CONFIGS["tiny"]
+    ck, cv, cq = W.layer_calibration(cfg, 0, n=1024)
+    lib = aatc.calibrate(aatc.dims(1, 1, 4, b_max=16), ck[None], cv[None], cq[None], 7.0)
+    for kind, x in ((0, ck[0]), (1, cv[0])):
+        qs = [cq[j].astype(np.float64) for j in range(4)] if kind == 0 else None
+        ref = O.plan_stream(x.astype(np.float64), 7.0, b_max=16, queries_by_head=qs)
+        got = lib["bits"][0, 0, kind].astype(np.int64)
+        assert np.array_equal(got, ref["bits"])
+        assert got.sum() == 7 * 128 and got.max() > 8 and got.max() <= 16
+    with pytest.raises(aatc.AatcError) as e:
+        aatc.calibrate(aatc.dims(1, 1, 4, b_max=17), ck[None], cv[None], cq[None], 7.0)
+    assert e.value.status == 1
