@@ -226,7 +226,7 @@ aatc_status_t aatc_cache_bytes(aatc_plan_t plan, int32_t batch, int32_t max_toke
  *            at positions [start, start + n_tokens) of every sequence; other positions untouched.
  * A non-finite alpha sets device error flag bit 0 (aatc_get_device_error).
  * Errors: AATC_ERR_INVALID_ARG, AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_CUDA.
- * n_tokens == 0 is a no-op.
+ * n_tokens == 0 is a no-op (K, V and cache may then be NULL: nothing is read or written).
  */
 aatc_status_t aatc_encode(aatc_plan_t plan, int32_t layer, const void* K, const void* V,
                           int32_t batch, int32_t start, int32_t n_tokens, void* cache,
@@ -243,6 +243,7 @@ aatc_status_t aatc_encode(aatc_plan_t plan, int32_t layer, const void* K, const 
  *   a_hat   : device bf16 [L][n_kv][2][128][d_model] (aatc_hidden_operand's layout), 16-byte aligned
  * Asynchronous on `stream`.  Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer,
  * sizes or d_model), AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_CUDA.
+ * n_tokens == 0 is a no-op (x, a_hat and cache may then be NULL).
  */
 aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x, int32_t d_model, const void* a_hat,
                                  int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,

@@ -324,12 +324,12 @@ aatc_status_t aatc_encode(aatc_plan_t p, int32_t layer, const void* K, const voi
                           int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
                           void* stream) {
   aatc::Plan* plan = as_plan(p);
-  if (!plan || !K || !V || !cache || layer < 0 || layer >= plan->dims.n_layers || batch < 1 ||
-      start < 0 || n_tokens < 0 || max_tokens < 1)
+  if (!plan || layer < 0 || layer >= plan->dims.n_layers || batch < 1 || start < 0 || n_tokens < 0 ||
+      max_tokens < 1)
     return AATC_ERR_INVALID_ARG;
   if (static_cast<int64_t>(start) + n_tokens > max_tokens) return AATC_ERR_CAPACITY;
-  if (!aligned16(K) || !aligned16(V) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
-  if (n_tokens == 0) return AATC_OK;
+  if (n_tokens == 0) return AATC_OK;                   // an empty append reads no pointer
+  if (!K || !V || !cache || !aligned16(K) || !aligned16(V) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
   return cuda_status(aatc::launch_encode(*plan, layer, K, V, batch, start, n_tokens, cache,
                                          max_tokens, static_cast<cudaStream_t>(stream)));
 }
@@ -338,12 +338,13 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t p, int32_t layer, const void* x, in
                                  int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
                                  void* stream) {
   aatc::Plan* plan = as_plan(p);
-  if (!plan || !x || !a_hat || !cache || layer < 0 || layer >= plan->dims.n_layers || batch < 1 || start < 0 ||
-      n_tokens < 0 || max_tokens < 1 || d_model < 64 || d_model % 64 != 0 || d_model > 65536)
+  if (!plan || layer < 0 || layer >= plan->dims.n_layers || batch < 1 || start < 0 || n_tokens < 0 ||
+      max_tokens < 1 || d_model < 64 || d_model % 64 != 0 || d_model > 65536)
     return AATC_ERR_INVALID_ARG;
   if (static_cast<int64_t>(start) + n_tokens > max_tokens) return AATC_ERR_CAPACITY;
-  if (!aligned16(x) || !aligned16(a_hat) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
-  if (n_tokens == 0) return AATC_OK;
+  if (n_tokens == 0) return AATC_OK;                   // an empty append reads no pointer
+  if (!x || !a_hat || !cache || !aligned16(x) || !aligned16(a_hat) || !aligned16(cache))
+    return AATC_ERR_INVALID_ARG;
   return cuda_status(aatc::launch_encode_hidden(*plan, layer, x, d_model, a_hat, batch, start, n_tokens, cache,
                                                 max_tokens, static_cast<cudaStream_t>(stream)));
 }

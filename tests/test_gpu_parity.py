@@ -172,7 +172,17 @@ def test_argument_errors_leave_outputs_untouched(aatc, tiny):
     with pytest.raises(aatc.AatcError) as e:
         aatc.encode(case.plan, 0, kd, kd, cache, 505, 512)
     assert e.value.status == 3
+    with pytest.raises(aatc.AatcError) as e:                   # empty context: no softmax to take
+        aatc.decode_attention(case.plan, 0, q, cache, 0, 512, out=out, workspace=torch.empty(1 << 20, device=DEV))
+    assert e.value.status == 1
     assert torch.all(out == 7.0)
+    # an empty append (the data pointer of an empty tensor is NULL) is a no-op at any position
+    before = cache.clone()
+    empty = torch.empty((1, 0, 1, 128), dtype=torch.bfloat16, device=DEV)
+    for start in (0, 300, 512):
+        aatc.encode(case.plan, 0, empty, empty, cache, start, 512)
+    torch.cuda.synchronize()
+    assert torch.equal(cache, before)
 
 
 # ----------------------------------------------------------------------------- full-size workloads
