@@ -97,7 +97,7 @@ struct CacheGeom {
 
 inline CacheGeom cache_geom(int batch, int n_kv, int max_tokens, int n_words) {
   CacheGeom g;
-  g.n_tiles = (max_tokens + TILE - 1) / TILE;
+  g.n_tiles = static_cast<int>((static_cast<int64_t>(max_tokens) + TILE - 1) / TILE);   // no int overflow
   g.words_elems = static_cast<size_t>(batch) * n_kv * 2 * g.n_tiles * n_words * TILE;
   g.alpha_elems = static_cast<size_t>(batch) * n_kv * 2 * g.n_tiles * TILE;
   g.bytes = 4 * (g.words_elems + g.alpha_elems);

@@ -46,7 +46,7 @@ DecodeSplit decode_split(int batch, int n_kv, int n_ctx, int num_sms, int ctas_p
   // s covering tiles [s T / n_splits, (s + 1) T / n_splits) so split lengths differ by at most
   // one tile and every SM gets nearly the same number of tiles.  A split holds at most 16 tiles
   // (its scores are kept in shared memory).
-  const long tiles = (n_ctx + TILE - 1) / TILE;
+  const long tiles = (static_cast<long>(n_ctx) + TILE - 1) / TILE;
   const long units = static_cast<long>(batch) * n_kv;
   const long target = static_cast<long>(std::max(1, ctas_per_sm)) * std::max(1, num_sms);
   long n = (target + units / 2) / units;
