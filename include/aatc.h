@@ -46,7 +46,8 @@ typedef enum {
   AATC_ERR_UNSUPPORTED = 5,   /* shape the kernels do not implement (e.g. GQA group > 8) */
   AATC_ERR_CUDA = 6,          /* a CUDA runtime call or kernel launch failed             */
   AATC_ERR_NOMEM = 7,         /* host or device allocation failed                        */
-  AATC_ERR_DEVICE_FLAG = 8    /* reserved for callers that turn device flags into status */
+  AATC_ERR_DEVICE_FLAG = 8,   /* reserved for callers that turn device flags into status */
+  AATC_ERR_IO = 9             /* plan file missing, unreadable, short, corrupt or another version */
 } aatc_status_t;
 
 /* Model dimensions.  d must be 128; n_q_heads % n_kv_heads == 0; b_max in 1..AATC_MAX_PLAN_BITS for
@@ -185,6 +186,26 @@ aatc_status_t aatc_whitening_transform(int32_t d_model, int32_t n, const float* 
  */
 aatc_status_t aatc_hidden_operand(const aatc_dims_t* dims, int32_t d_model, const float* w_k,
                                   const float* w_v, const float* basis, uint16_t* out);
+
+/*
+ * Plan files (calibration is offline and once per model, Algorithm 1's first half): the host
+ * arrays a plan is made of, written to and read from a versioned little-endian file with a
+ * checksum, so aatc_plan_create can rebuild the plan without recalibrating.
+ *   aatc_plan_save      : dims (planner range, b_max up to AATC_MAX_PLAN_BITS), basis fp32
+ *                         [L][H_kv][2][128][128], bits uint8 [L][H_kv][2][128] (<= b_max),
+ *                         scales fp32 [L][H_kv][2][128], all host; bit-exact copies are stored.
+ *   aatc_plan_file_dims : the dims of a file (to size the load buffers).
+ *   aatc_plan_load      : fills caller-owned host buffers of those sizes; `dims` must equal the
+ *                         file's dims.
+ * Errors: AATC_ERR_INVALID_ARG (null, invalid dims, bits > b_max on save, dims that differ from
+ * the file's on load), AATC_ERR_IO (file cannot be opened or written; wrong magic, version or
+ * sizes; trailing bytes; checksum mismatch).  Host only; no device work.
+ */
+aatc_status_t aatc_plan_save(const char* path, const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
+                             const float* scales);
+aatc_status_t aatc_plan_file_dims(const char* path, aatc_dims_t* dims_out);
+aatc_status_t aatc_plan_load(const char* path, const aatc_dims_t* dims, float* basis_out, uint8_t* bits_out,
+                             float* scales_out);
 
 /*
  * Build an immutable device plan from basis / bits / scales in the layouts aatc_calibrate

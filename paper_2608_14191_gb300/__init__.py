@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libaatc.so")
 _STATUS = {
     0: "ok", 1: "invalid argument", 2: "bit budget not representable", 3: "token range exceeds cache capacity",
     4: "workspace too small", 5: "unsupported shape", 6: "CUDA error", 7: "out of memory", 8: "device error flag set",
+    9: "plan file unreadable or corrupt",
 }
 
 
@@ -48,6 +49,9 @@ SIGNATURES = {
     "aatc_calibrate": (_I32, [ctypes.POINTER(Dims), _P, _P, _I32, _P, _I32, _F64, _F64, _I32, _P, _P, _P, _P, _P, _I32]),
     "aatc_calibrate_head_group": (_I32, [_I32, _I32, _P, _I32, _P, _I32, _F64, _I32, _I32, _P, _P, _P, _P, _P]),
     "aatc_selftest_bounded_wait": (_I32, [_I32, _P, _P]),
+    "aatc_plan_save": (_I32, [ctypes.c_char_p, _P, _P, _P, _P]),
+    "aatc_plan_file_dims": (_I32, [ctypes.c_char_p, _P]),
+    "aatc_plan_load": (_I32, [ctypes.c_char_p, _P, _P, _P, _P]),
     "aatc_allocate_global": (_I32, [ctypes.POINTER(Dims), _P, _P, _F64, _F64, _I32, _P]),
     "aatc_whitening_transform": (_I32, [_I32, _I32, _P, _P, _P, _P, _P, _P, _P]),
     "aatc_hidden_operand": (_I32, [ctypes.POINTER(Dims), _I32, _P, _P, _P, _P]),
@@ -165,6 +169,33 @@ def calibrate_head_group(calib: np.ndarray, calib_q: np.ndarray | None, avg_bits
                                             1 if var_only else 0, _ptr(basis), _ptr(bits), _ptr(scales),
                                             _ptr(sigma2), _ptr(weights)), "aatc_calibrate_head_group")
     return {"basis": basis, "bits": bits, "scales": scales, "sigma2": sigma2, "weights": weights}
+
+
+def save_plan(path: str, dm: Dims, basis: np.ndarray, bits: np.ndarray, scales: np.ndarray):
+    """aatc_plan_save: write a plan's host arrays (as calibrate returns them) to a plan file."""
+    L, H = dm.n_layers, dm.n_kv_heads
+    b = np.ascontiguousarray(basis, dtype=np.float32)
+    w = np.ascontiguousarray(bits, dtype=np.uint8)
+    sc = np.ascontiguousarray(scales, dtype=np.float32)
+    if b.size != L * H * 2 * HEAD_DIM * HEAD_DIM or w.size != L * H * 2 * HEAD_DIM or sc.size != w.size:
+        raise ValueError("basis / bits / scales do not match the dims")
+    _check(load().aatc_plan_save(os.fsencode(path), ctypes.byref(dm), _ptr(b), _ptr(w), _ptr(sc)),
+           "aatc_plan_save")
+
+
+def load_plan(path: str):
+    """aatc_plan_file_dims + aatc_plan_load: (dims, dict(basis, bits, scales)) from a plan file, in
+    the layouts calibrate returns."""
+    lib = load()
+    dm = Dims()
+    _check(lib.aatc_plan_file_dims(os.fsencode(path), ctypes.byref(dm)), "aatc_plan_file_dims")
+    shape = (dm.n_layers, dm.n_kv_heads, 2, HEAD_DIM)
+    basis = np.empty(shape + (HEAD_DIM,), np.float32)
+    bits = np.empty(shape, np.uint8)
+    scales = np.empty(shape, np.float32)
+    _check(lib.aatc_plan_load(os.fsencode(path), ctypes.byref(dm), _ptr(basis), _ptr(bits), _ptr(scales)),
+           "aatc_plan_load")
+    return dm, {"basis": basis, "bits": bits, "scales": scales}
 
 
 def selftest_bounded_wait(limit_us: int, flags, stream=None):

@@ -143,6 +143,7 @@ const char* aatc_status_string(aatc_status_t s) {
     case AATC_ERR_CUDA: return "CUDA error";
     case AATC_ERR_NOMEM: return "out of memory";
     case AATC_ERR_DEVICE_FLAG: return "device error flag set";
+    case AATC_ERR_IO: return "plan file unreadable or corrupt";
   }
   return "unknown status";
 }
