@@ -113,6 +113,43 @@ def _stream(stream=None) -> int:
     return s.cuda_stream
 
 
+def _arg_error(where: str, what: str):
+    raise AatcError(1, f"{where} ({what})")
+
+
+_DEVICE_TYPE = "cuda"     # where device arguments must live
+
+
+def _dev_tensor(t, where: str, name: str, dtype=None, ndim: int | None = None, shape=None):
+    """Checks a device argument before its pointer goes to the library, which cannot see sizes:
+    a CUDA tensor, of `dtype`, with `ndim` dimensions and the given sizes (None = any)."""
+    import torch
+    if not isinstance(t, torch.Tensor) or t.device.type != _DEVICE_TYPE:
+        _arg_error(where, f"{name} must be a {_DEVICE_TYPE} tensor")
+    if dtype is not None and t.dtype != dtype:
+        _arg_error(where, f"{name} must be {dtype}, not {t.dtype}")
+    if ndim is not None and t.dim() != ndim:
+        _arg_error(where, f"{name} must have {ndim} dimensions, not {t.dim()}")
+    if shape is not None:
+        for i, n in enumerate(shape):
+            if n is not None and t.shape[i] != n:
+                _arg_error(where, f"{name} size {i} must be {n}, not {t.shape[i]}")
+
+
+def _cache_ok(plan, cache, batch: int, max_tokens: int, where: str):
+    _dev_tensor(cache, where, "cache")
+    need = plan.cache_bytes(batch, max_tokens)
+    if cache.numel() * cache.element_size() < need:
+        _arg_error(where, f"cache holds {cache.numel() * cache.element_size()} bytes, {need} needed")
+
+
+def _out_ok(out, n: int, where: str):
+    import torch
+    _dev_tensor(out, where, "out", torch.float32)
+    if out.numel() < n:
+        _arg_error(where, f"out holds {out.numel()} values, {n} needed")
+
+
 def dims(n_layers: int, n_kv_heads: int, n_q_heads: int, b_max: int = 8) -> Dims:
     return Dims(HEAD_DIM, n_layers, n_kv_heads, n_q_heads, b_max)
 
@@ -282,9 +319,13 @@ class Plan:
         return self.dims.n_q_heads // self.dims.n_kv_heads
 
     def cache_bytes(self, batch: int, max_tokens: int) -> int:
-        n = _SZ()
-        _check(load().aatc_cache_bytes(self.handle, batch, max_tokens, ctypes.byref(n)), "aatc_cache_bytes")
-        return n.value
+        key = (int(batch), int(max_tokens))
+        memo = self.__dict__.setdefault("_cache_bytes", {})
+        if key not in memo:
+            n = _SZ()
+            _check(load().aatc_cache_bytes(self.handle, batch, max_tokens, ctypes.byref(n)), "aatc_cache_bytes")
+            memo[key] = n.value
+        return memo[key]
 
     def new_cache(self, batch: int, max_tokens: int, device="cuda"):
         import torch
@@ -316,7 +357,11 @@ class Plan:
 def encode(plan: Plan, layer: int, K, V, cache, start: int, max_tokens: int, stream=None):
     """aatc_encode: K, V bf16 [batch][n_tokens][H_kv][128] (device); writes positions
     [start, start + n_tokens) of the packed cache."""
+    import torch
+    _dev_tensor(K, "aatc_encode", "K", torch.bfloat16, 4, (None, None, plan.dims.n_kv_heads, HEAD_DIM))
+    _dev_tensor(V, "aatc_encode", "V", torch.bfloat16, 4, tuple(K.shape))
     batch, n_tokens = K.shape[0], K.shape[1]
+    _cache_ok(plan, cache, batch, max_tokens, "aatc_encode")
     _check(load().aatc_encode(plan.handle, layer, _ptr(K), _ptr(V), batch, start, n_tokens, _ptr(cache),
                               max_tokens, _stream(stream)), "aatc_encode")
 
@@ -325,7 +370,13 @@ def encode_hidden(plan: Plan, layer: int, x, a_hat, cache, start: int, max_token
     """aatc_encode_hidden: x bf16 [batch][n_tokens][d_model] hidden states (device), a_hat bf16
     [L][H_kv][2][128][d_model] from hidden_operand (device); writes positions [start, start +
     n_tokens) of the packed cache with the codes of x W U (keys and values of every kv-head)."""
+    import torch
+    _dev_tensor(x, "aatc_encode_hidden", "x", torch.bfloat16, 3)
     batch, n_tokens, d_model = x.shape
+    _dev_tensor(a_hat, "aatc_encode_hidden", "a_hat", torch.bfloat16)
+    if a_hat.numel() != plan.dims.n_layers * plan.dims.n_kv_heads * 2 * HEAD_DIM * d_model:
+        _arg_error("aatc_encode_hidden", "a_hat must be [L][H_kv][2][128][d_model] for the d_model of x")
+    _cache_ok(plan, cache, batch, max_tokens, "aatc_encode_hidden")
     _check(load().aatc_encode_hidden(plan.handle, layer, _ptr(x), d_model, _ptr(a_hat), batch, start, n_tokens,
                                      _ptr(cache), max_tokens, _stream(stream)), "aatc_encode_hidden")
 
@@ -335,9 +386,12 @@ def prefill_attention(plan: Plan, layer: int, q, q_start: int, cache, n_ctx: int
     """aatc_prefill_attention: q bf16 [batch][n_q][H_q][128] at positions q_start .. q_start + n_q - 1,
     causal over the packed cache tokens [0, n_ctx) -> fp32 [batch][n_q][H_q][128]."""
     import torch
+    _dev_tensor(q, "aatc_prefill_attention", "q", torch.bfloat16, 4, (None, None, plan.dims.n_q_heads, HEAD_DIM))
     batch, n_q = q.shape[0], q.shape[1]
+    _cache_ok(plan, cache, batch, max_tokens, "aatc_prefill_attention")
     if out is None:
         out = torch.empty((batch, n_q, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    _out_ok(out, batch * n_q * plan.dims.n_q_heads * HEAD_DIM, "aatc_prefill_attention")
     nb = _SZ()
     _check(load().aatc_prefill_workspace_bytes(plan.handle, batch, n_ctx, ctypes.byref(nb)),
            "aatc_prefill_workspace_bytes")
@@ -354,9 +408,12 @@ def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: i
                      stream=None):
     """aatc_decode_attention: q bf16 [batch][H_q][128] -> fp32 [batch][H_q][128]."""
     import torch
+    _dev_tensor(q, "aatc_decode_attention", "q", torch.bfloat16, 3, (None, plan.dims.n_q_heads, HEAD_DIM))
     batch = q.shape[0]
+    _cache_ok(plan, cache, batch, max_tokens, "aatc_decode_attention")
     if out is None:
         out = torch.empty((batch, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    _out_ok(out, batch * plan.dims.n_q_heads * HEAD_DIM, "aatc_decode_attention")
     nbytes = plan.workspace_bytes(batch, n_ctx)
     if workspace is None:
         workspace = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device=q.device)
@@ -371,9 +428,16 @@ def decode_attention_sw(plan: Plan, layer: int, q, cache, t_first: int, t_end: i
     """aatc_decode_attention_sw: packed tokens [t_first, t_end) plus the first n_full tokens of
     k_full / v_full (bf16 [batch][cap][H_kv][128]) in one softmax -> fp32 [batch][H_q][128]."""
     import torch
+    where = "aatc_decode_attention_sw"
+    _dev_tensor(q, where, "q", torch.bfloat16, 3, (None, plan.dims.n_q_heads, HEAD_DIM))
     batch = q.shape[0]
+    _cache_ok(plan, cache, batch, max_tokens, where)
+    if k_full is not None or v_full is not None:
+        _dev_tensor(k_full, where, "k_full", torch.bfloat16, 4, (batch, None, plan.dims.n_kv_heads, HEAD_DIM))
+        _dev_tensor(v_full, where, "v_full", torch.bfloat16, 4, tuple(k_full.shape))
     if out is None:
         out = torch.empty((batch, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
+    _out_ok(out, batch * plan.dims.n_q_heads * HEAD_DIM, where)
     cap = 0 if k_full is None else int(k_full.shape[1])
     if t_end > t_first and workspace is None:
         workspace = torch.empty(max(1, plan.workspace_bytes(batch, t_end) // 4), dtype=torch.float32,
@@ -390,6 +454,11 @@ def decode_attention_sw(plan: Plan, layer: int, q, cache, t_first: int, t_end: i
 def decode_attention_noalloc(plan: Plan, layer: int, q, out, cache, n_ctx: int, max_tokens: int, stream=None):
     """aatc_decode_attention_noalloc: as decode_attention, but with no workspace and no allocation
     (the caller passes `out`; the library's fixed scratch holds the split partials)."""
+    import torch
+    where = "aatc_decode_attention_noalloc"
+    _dev_tensor(q, where, "q", torch.bfloat16, 3, (None, plan.dims.n_q_heads, HEAD_DIM))
+    _cache_ok(plan, cache, q.shape[0], max_tokens, where)
+    _out_ok(out, q.shape[0] * plan.dims.n_q_heads * HEAD_DIM, where)
     _check(load().aatc_decode_attention_noalloc(plan.handle, layer, _ptr(q), _ptr(cache), q.shape[0], n_ctx,
                                                 max_tokens, _ptr(out), _stream(stream)),
            "aatc_decode_attention_noalloc")
@@ -399,6 +468,7 @@ def decode_attention_noalloc(plan: Plan, layer: int, q, out, cache, n_ctx: int, 
 def dequantize(plan: Plan, layer: int, cache, batch: int, t0: int, n: int, max_tokens: int, stream=None):
     """aatc_dequantize test hook -> fp32 [batch][n][H_kv][2][128]."""
     import torch
+    _cache_ok(plan, cache, batch, max_tokens, "aatc_dequantize")
     out = torch.empty((batch, n, plan.dims.n_kv_heads, 2, HEAD_DIM), dtype=torch.float32, device=cache.device)
     _check(load().aatc_dequantize(plan.handle, layer, _ptr(cache), batch, t0, n, max_tokens, _ptr(out),
                                   _stream(stream)), "aatc_dequantize")
@@ -415,10 +485,15 @@ def bf16_workspace_bytes(batch: int, n_kv: int, n_q: int, n_ctx: int) -> int:
 def bf16_decode_attention(K, V, q, n_ctx: int, out=None, workspace=None, stream=None):
     """Uncompressed reference decode: K, V bf16 [batch][max_tokens][H_kv][128]; q bf16 [batch][H_q][128]."""
     import torch
+    where = "aatc_bf16_decode_attention"
+    _dev_tensor(K, where, "K", torch.bfloat16, 4, (None, None, None, HEAD_DIM))
+    _dev_tensor(V, where, "V", torch.bfloat16, 4, tuple(K.shape))
     batch, max_tokens, n_kv = K.shape[0], K.shape[1], K.shape[2]
+    _dev_tensor(q, where, "q", torch.bfloat16, 3, (batch, None, HEAD_DIM))
     n_q = q.shape[1]
     if out is None:
         out = torch.empty((batch, n_q, HEAD_DIM), dtype=torch.float32, device=q.device)
+    _out_ok(out, batch * n_q * HEAD_DIM, where)
     if workspace is None:
         workspace = torch.empty(max(1, bf16_workspace_bytes(batch, n_kv, n_q, n_ctx) // 4), dtype=torch.float32,
                                 device=q.device)
