@@ -113,6 +113,13 @@ def _stream(stream=None) -> int:
     return s.cuda_stream
 
 
+try:                      # the binding's device helpers compare against torch dtypes
+    import torch as _torch
+    _F32 = _torch.float32
+except ImportError:       # host-only use (planner, plan files) works without torch
+    _F32 = None
+
+
 def _arg_error(where: str, what: str):
     raise AatcError(1, f"{where} ({what})")
 
@@ -120,32 +127,40 @@ def _arg_error(where: str, what: str):
 _DEVICE_TYPE = "cuda"     # where device arguments must live
 
 
+def _on_device(t) -> bool:
+    try:
+        return t.is_cuda if _DEVICE_TYPE == "cuda" else t.device.type == _DEVICE_TYPE
+    except AttributeError:
+        return False
+
+
 def _dev_tensor(t, where: str, name: str, dtype=None, ndim: int | None = None, shape=None):
     """Checks a device argument before its pointer goes to the library, which cannot see sizes:
     a CUDA tensor, of `dtype`, with `ndim` dimensions and the given sizes (None = any)."""
-    import torch
-    if not isinstance(t, torch.Tensor) or t.device.type != _DEVICE_TYPE:
+    if not _on_device(t):
         _arg_error(where, f"{name} must be a {_DEVICE_TYPE} tensor")
     if dtype is not None and t.dtype != dtype:
         _arg_error(where, f"{name} must be {dtype}, not {t.dtype}")
-    if ndim is not None and t.dim() != ndim:
-        _arg_error(where, f"{name} must have {ndim} dimensions, not {t.dim()}")
+    sh = t.shape
+    if ndim is not None and len(sh) != ndim:
+        _arg_error(where, f"{name} must have {ndim} dimensions, not {len(sh)}")
     if shape is not None:
         for i, n in enumerate(shape):
-            if n is not None and t.shape[i] != n:
-                _arg_error(where, f"{name} size {i} must be {n}, not {t.shape[i]}")
+            if n is not None and sh[i] != n:
+                _arg_error(where, f"{name} size {i} must be {n}, not {sh[i]}")
 
 
 def _cache_ok(plan, cache, batch: int, max_tokens: int, where: str):
-    _dev_tensor(cache, where, "cache")
+    if not _on_device(cache):
+        _arg_error(where, f"cache must be a {_DEVICE_TYPE} tensor")
     need = plan.cache_bytes(batch, max_tokens)
-    if cache.numel() * cache.element_size() < need:
-        _arg_error(where, f"cache holds {cache.numel() * cache.element_size()} bytes, {need} needed")
+    if cache.nbytes < need:
+        _arg_error(where, f"cache holds {cache.nbytes} bytes, {need} needed")
 
 
 def _out_ok(out, n: int, where: str):
-    import torch
-    _dev_tensor(out, where, "out", torch.float32)
+    if not _on_device(out) or out.dtype != _F32:
+        _arg_error(where, f"out must be a {_DEVICE_TYPE} tensor of torch.float32")
     if out.numel() < n:
         _arg_error(where, f"out holds {out.numel()} values, {n} needed")
 

@@ -84,7 +84,7 @@ def test_decode_and_prefill(fake):
     _binding_refused(e, "aatc_decode_attention", "values")
     with pytest.raises(aatc.AatcError) as e:
         aatc.decode_attention(plan, 0, q, cache, 64, 64, out=torch.zeros((2, 8, 128), dtype=torch.float64), stream=S)
-    _binding_refused(e, "aatc_decode_attention", "out must be torch.float32")
+    _binding_refused(e, "aatc_decode_attention", "out must be a cpu tensor of torch.float32")
     qp = torch.zeros((2, 3, 8, 128), dtype=bf16)
     with pytest.raises(aatc.AatcError) as e:
         aatc.prefill_attention(plan, 0, qp, 0, cache, 64, 64, stream=S)
