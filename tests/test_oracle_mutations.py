@@ -196,6 +196,11 @@ def _pack_msb_first(codes, bits, n_words):
     return words.astype(np.uint32)
 
 
+def _value_slot_identity(token_in_tile, quarter):
+    q, i = divmod(token_in_tile, 4)
+    return 4 * q + quarter, i
+
+
 def _softmax_unnormalised(s):
     s = np.asarray(s, np.float64)
     return np.exp(s - np.max(s))
@@ -418,6 +423,8 @@ MUTANTS = [
     ("record_entries", "odd top bit taken from bit 0", _record_entries_top_bit_low,
      [_pack_round_trips, _packing_examples]),
     ("pack_records", "fields MSB-first", _pack_msb_first, [_packing_examples]),
+    ("value_slot_of", "byte-quarters in slot order 0, 1, 2, 3", _value_slot_identity,
+     [P.test_value_interleave_hand_example]),
     ("softmax", "no normalisation", _softmax_unnormalised, [P.test_decode_matches_library_sdpa]),
     ("attention", "scores without 1/sqrt(d)", _attention_unscaled,
      [HG.test_group_decode_with_exact_coefficients_is_plain_attention,

@@ -385,6 +385,21 @@ def test_value_interleave_round_trip():
     assert slots == [(s, i) for s in range(8) for i in range(4)]
 
 
+def test_value_interleave_hand_example():
+    """The value layout written out by hand for one token quad: token t's record word has bytes
+    16t + r (r = 0..3); slot (0, 2, 1, 3)[r] of the quad holds byte-quarter r of the four tokens,
+    token i in byte i, so the slots read 0x30201000, 0x32221202, 0x31211101, 0x33231303.  Keys
+    are stored plainly: slot t holds token t's word."""
+    words = np.array([[sum((16 * t + r) << (8 * r) for r in range(4))] for t in range(4)], np.uint32)
+    img = O.cache_image([[words]], [[words]], [[np.zeros(4, np.float32)]], [[np.zeros(4, np.float32)]],
+                        1, 1, 128, 1)
+    plane_k = img[0:128]
+    plane_v = img[128:256]
+    assert plane_v[:4].tolist() == [0x30201000, 0x32221202, 0x31211101, 0x33231303]
+    assert plane_k[:4].tolist() == words[:, 0].tolist()
+    assert not plane_v[4:].any() and not plane_k[4:].any()
+
+
 def test_record_size_matches_paper_compression():
     g = _gold("compression_ratios.json")
     cfg = W.CONFIGS["tiny"]
