@@ -150,7 +150,7 @@ const char* aatc_status_string(aatc_status_t s) {
 
 int32_t aatc_last_cuda_error(void) { return g_last_cuda_error; }
 
-int32_t aatc_version(void) { return 100; }
+int32_t aatc_version(void) { return 200; }   // 0.2.0: plan files, AATC_ERR_IO, planner widths to 16
 
 aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
                                const float* scales, void* stream, aatc_plan_t* plan_out) {
