@@ -35,9 +35,9 @@ sys.path.insert(0, ROOT)
 import workloads as W  # noqa: E402
 
 METRIC = "compressed-KV decode attn GB/s & % of HBM peak; encode Mtok/s (1 GB300)"
+DECODE_KERNELS = "aatc_decode_query_kernel + aatc_decode_split_kernel + aatc_decode_merge_kernel"
 N_COPIES = 16
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "decode_traffic.json")
-DECODE_SRC = os.path.join(ROOT, "paper_2608_14191_gb300", "csrc", "decode.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 
 
@@ -139,15 +139,19 @@ def _source_hash(path):
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def _traffic_per_launch():
-    """DRAM bytes per decode launch from the committed ncu summary, if it was taken on this source."""
+def _traffic(key):
+    """DRAM bytes per launch of one measured kernel call from the committed ncu summaries
+    (profiles/traffic.json), or None when the source it was taken on has changed since."""
     if not os.path.exists(TRAFFIC_FILE):
         return None
     with open(TRAFFIC_FILE) as f:
-        d = json.load(f)
-    if d.get("decode_cu_sha256_16") != _source_hash(DECODE_SRC):
+        d = json.load(f).get(key)
+    if not d:
         return None
-    return d.get("bytes_per_decode_call")
+    src = os.path.join(ROOT, d["source"])
+    if not os.path.exists(src) or d.get("source_sha256_16") != _source_hash(src):
+        return None
+    return d.get("bytes_per_call")
 
 
 def build_case(aatc, cfg, avg_bits, device):
@@ -204,6 +208,46 @@ def sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_d
             "policy": "sink 4 + recent window 128 (step 16) in bf16, the rest coded"}
 
 
+def sink_window_stream_timing(aatc, plan, cfg, kd, vd, qs, device, n_steps=256):
+    """Token-by-token generation with the paper's sink / window policy on the Llama-shaped layer:
+    the cache manager holds 32768 - 2 n_steps tokens (prefilled in one append), then n_steps
+    untimed and n_steps timed steps of (append one token to every kv-head, decode attention).
+    Appends write the new token in place; every 16th token flushes 16 window tokens through
+    the encode.  Timed with CUDA events (device time of the whole loop, host dispatch included
+    where the host is slower) and the host clock."""
+    import torch
+    from paper_2608_14191_gb300.sink_window import SinkWindowCache
+    B, T = cfg.batch, cfg.n_ctx
+    swc = SinkWindowCache(plan, 0, B, T, device)
+    t0 = T - 2 * n_steps
+    swc.append(kd[:, :t0], vd[:, :t0])
+    out = torch.empty((B, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
+    ws = torch.empty(max(1, plan.workspace_bytes(B, T) // 4), dtype=torch.float32, device=device)
+    stream = torch.cuda.current_stream()
+
+    def steps(a):
+        for t in range(a, a + n_steps):
+            swc.append(kd[:, t:t + 1], vd[:, t:t + 1])
+            swc.decode(qs[t % qs.shape[0]], out=out, workspace=ws)
+
+    steps(t0)
+    torch.cuda.synchronize()
+    flushes0 = swc.state.n_coded
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    h0 = time.perf_counter()
+    e0.record(stream)
+    steps(t0 + n_steps)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    host_us = (time.perf_counter() - h0) * 1e6 / n_steps
+    us = e0.elapsed_time(e1) * 1e3 / n_steps
+    assert plan.device_error() == 0
+    return {"us_per_token": round(us, 3), "host_us_per_token": round(host_us, 3),
+            "tokens_flushed": swc.state.n_coded - flushes0, "block_relocations": swc.relocations,
+            "what": f"{n_steps} steps of (append 1 token x {cfg.n_kv_heads} kv-heads, decode) at "
+                    f"{T - n_steps} tokens, sink 4 + window 128 (step 16) kept in place"}
+
+
 def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32768, iters=10, warmup=3):
     """Encode straight from the layer input (Sec. 5 Step 1: the cache holds the coefficients of
     x A): Llama-3.1-8B-shaped layer input, d_model 4096, 8 kv-heads x K|V, 32768 tokens.  The
@@ -252,19 +296,36 @@ def hidden_encode_timing(aatc, device, d_model=4096, n_kv=8, n_q=32, n_tokens=32
                         f"{n_tokens} tokens, 2.75 bits"}
 
 
+def stack_plan(aatc, cfg, avg_bits=2.75):
+    """One plan for the whole stack with a separately calibrated basis, allocation and scales per
+    layer and kv-head (each layer from its own seeded calibration set); layers are calibrated in
+    parallel host threads (the planner call releases the GIL)."""
+    import concurrent.futures as cf
+    L, H = cfg.n_layers, cfg.n_kv_heads
+
+    def one(layer):
+        ck, cv, cq = W.layer_calibration(cfg, layer)
+        return aatc.calibrate(aatc.dims(1, H, cfg.n_q_heads), ck[None], cv[None], cq[None], avg_bits)
+
+    with cf.ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 4)) as ex:
+        ps = list(ex.map(one, range(L)))
+    basis = np.concatenate([p["basis"] for p in ps])
+    bits = np.concatenate([p["bits"] for p in ps])
+    scales = np.concatenate([p["scales"] for p in ps])
+    return aatc.Plan(aatc.dims(L, H, cfg.n_q_heads), basis, bits, scales), bits
+
+
 def stack_decode_timing(aatc, device, reps=10):
     """Decode through the Llama-3.1-8B-shaped 32-layer stack at 131072 tokens (one decode step =
     one call per layer, 101 MB of packed codes and alpha each, 3.2 GB in all, far above L2),
-    timed as one CUDA graph of the 32 calls.  The calibrated plan of layer 0 serves every layer
-    (the decode's cost depends on the bit layout, not on the basis values); every layer's cache
-    is encoded from its own synthetic K/V."""
+    timed as one CUDA graph of the 32 calls.  Every layer has its own calibrated plan (basis,
+    widths and scales per kv-head) and its cache is encoded from its own synthetic K/V."""
     import torch
     cfg = W.CONFIGS["llama_stack"]
     n_layers, n_ctx = cfg.n_layers, cfg.n_ctx
-    ck, cv, cq = W.layer_calibration(cfg, 0)
-    p1 = aatc.calibrate(aatc.dims(1, cfg.n_kv_heads, cfg.n_q_heads), ck[None], cv[None], cq[None], 2.75)
-    plan = aatc.Plan(aatc.dims(n_layers, cfg.n_kv_heads, cfg.n_q_heads), np.repeat(p1["basis"], n_layers, axis=0),
-                     np.repeat(p1["bits"], n_layers, axis=0), np.repeat(p1["scales"], n_layers, axis=0))
+    t0 = time.perf_counter()
+    plan, bits = stack_plan(aatc, cfg)
+    plan_s = time.perf_counter() - t0
     caches = []
     for layer in range(n_layers):
         kd, vd = W.kv_device(cfg, layer, 1, n_ctx, device)
@@ -297,15 +358,93 @@ def stack_decode_timing(aatc, device, reps=10):
     torch.cuda.synchronize()
     assert plan.device_error() == 0
     us = e0.elapsed_time(e1) * 1e3 / (reps * n_layers)
-    # one layer's call: packed codes (sum of widths / 8) + 4 B alpha per (token, kv-head, K|V)
-    nbytes = float(n_ctx * (np.sum(p1["bits"]) / 8.0 + 4 * cfg.n_kv_heads * 2))
-    peak, _ = _peaks()
+    # bytes of one step: packed codes (each layer's widths / 8) + 4 B alpha per (token, kv-head, K|V)
+    step_bytes = float(n_ctx * (np.sum(bits.astype(np.int64)) / 8.0 + 4 * n_layers * cfg.n_kv_heads * 2))
+    nbytes = step_bytes / n_layers
+    peak, kind = _peaks()
     gbs = nbytes / (us * 1e-6) / 1e9
     plan.close()
     return {"us_per_layer_call": round(us, 3), "gbs": round(gbs, 2), "bytes_per_call": nbytes,
-            "frac_of_measured_hbm": round(gbs / peak, 4), "step_ms": round(us * n_layers / 1e3, 3),
+            "frac_of_measured_hbm": round(gbs / peak, 4), "frac_of_nominal_8tbs": round(gbs / 8000.0, 4),
+            "step_ms": round(us * n_layers / 1e3, 3), "plan_seconds": round(plan_s, 2),
+            "roofline": {"bound": "hbm", "achieved": round(gbs, 2), "peak": peak, "unit": "GB/s",
+                         "frac": round(gbs / peak, 4), "traffic": _traffic("decode_stack"),
+                         "kernel": "one decode call (131072 tokens x 8 kv-heads)",
+                         "peak_source": f"{kind} hbm_gbs (MEASURED_PEAKS.json)"},
             "workload": "Llama-3.1-8B-shaped stack: 32 layers x 131072 tokens x 8 kv-heads, one decode step "
-                        "(32 calls in a CUDA graph); the layer-0 plan serves every layer"}
+                        "(32 calls in a CUDA graph), a separately calibrated plan per layer and kv-head"}
+
+
+def qwen_timing(aatc, device, n_calls=64, reps=3, enc_iters=6, n_copies=4):
+    """The Qwen-2.5-7B-shaped layer: prefill-encode of 16 sequences x 8192 tokens (28 query heads
+    over 4 kv-heads, 268 MB of bf16 K/V input, > L2) as one encode call, then one batched decode
+    step of all 16 sequences (G = 7, 50 MB of packed codes and alpha), timed as a CUDA graph of
+    calls rotating over four packed-cache copies (201 MB > L2)."""
+    import torch
+    cfg = W.CONFIGS["qwen"]
+    B, T = cfg.batch, cfg.n_ctx
+    plan, _ = build_case(aatc, cfg, 2.75, device)
+    kd, vd = W.kv_device(cfg, 0, B, T, device)
+    qs = W.queries_device(cfg, 0, B, 4, device)
+    caches = [plan.new_cache(B, T, device) for _ in range(n_copies)]
+    stream = torch.cuda.current_stream()
+    peak, kind = _peaks()
+    ctr = [0]
+
+    def enc():
+        aatc.encode(plan, 0, kd, vd, caches[ctr[0] % n_copies], 0, T)
+        ctr[0] += 1
+
+    for _ in range(n_copies):
+        enc()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(enc_iters):
+        enc()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    enc_us = e0.elapsed_time(e1) * 1e3 / enc_iters
+    in_bytes = (kd.numel() + vd.numel()) * 2
+    out = torch.empty((B, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
+    ws = torch.empty(max(1, plan.workspace_bytes(B, T) // 4), dtype=torch.float32, device=device)
+
+    def calls():
+        for i in range(n_calls):
+            aatc.decode_attention(plan, 0, qs[i % qs.shape[0]], caches[i % n_copies], T, T, out=out, workspace=ws)
+
+    calls()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        calls()
+    graph.replay()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    dec_us = e0.elapsed_time(e1) * 1e3 / (reps * n_calls)
+    dbytes = decode_bytes(plan, cfg, B, T)
+    dec_gbs = dbytes / (dec_us * 1e-6) / 1e9
+    enc_gbs = in_bytes / (enc_us * 1e-6) / 1e9
+    plan.close()
+    return {"workload": cfg.workload,
+            "encode": {"us_per_call": round(enc_us, 2), "mtok_s": round(B * T / enc_us, 2),
+                       "input_gbs": round(enc_gbs, 2), "frac_of_measured_hbm_on_input": round(enc_gbs / peak, 4),
+                       "frac_of_nominal_8tbs": round(enc_gbs / 8000.0, 4), "input_bytes": in_bytes},
+            "decode": {"us_per_call": round(dec_us, 3), "gbs": round(dec_gbs, 2), "bytes_per_call": dbytes,
+                       "frac_of_measured_hbm": round(dec_gbs / peak, 4),
+                       "frac_of_nominal_8tbs": round(dec_gbs / 8000.0, 4),
+                       "mtok_s": round(B * T / dec_us, 2)},
+            "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 2), "peak": peak, "unit": "GB/s",
+                         "frac": round(dec_gbs / peak, 4), "traffic": _traffic("decode_qwen"),
+                         "kernel": "one batched decode call (16 x 8192 tokens x 4 kv-heads, G = 7)",
+                         "peak_source": f"{kind} hbm_gbs (MEASURED_PEAKS.json)"},
+            "timing": f"encode: {enc_iters} calls rotating over {n_copies} caches; decode: {n_calls}-call CUDA graph "
+                      f"x {reps} over {n_copies} packed-cache copies"}
 
 
 def bf16_decode_timing(aatc, kd, vd, qs, n_ctx, packed_us, n_calls=64, reps=3):
@@ -510,7 +649,7 @@ def run_ours(args):
     cfg = W.CONFIGS[args.config]
     avg_bits = cfg.avg_bits[-1] if args.bits is None else args.bits
     B, T, steps_dec = cfg.batch, cfg.n_ctx, cfg.decode_steps
-    plan, _ = build_case(aatc, cfg, avg_bits, dev)
+    plan, params = build_case(aatc, cfg, avg_bits, dev)
     kd, vd = W.kv_device(cfg, 0, B, T, dev)
     qs = W.queries_device(cfg, 0, B, steps_dec, dev)
     caches = [plan.new_cache(B, T, dev) for _ in range(N_COPIES)]
@@ -650,7 +789,9 @@ def run_ours(args):
         return
 
     sw = sink_window_timing(aatc, plan, cfg, caches, kd, vd, qs, out, wspace, steps_dec)
+    sw["streaming"] = sink_window_stream_timing(aatc, plan, cfg, kd, vd, qs, dev)
     ref16 = bf16_decode_timing(aatc, kd, vd, qs, T, dec_mean / steps_dec * 1e3)
+    qwen = qwen_timing(aatc, dev)
     stack = stack_decode_timing(aatc, dev)
     hid = hidden_encode_timing(aatc, dev)
     pre = prefill_timing(aatc, dev)
@@ -689,9 +830,15 @@ def run_ours(args):
                    "input_gbs": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9, 2),
                    "frac_of_measured_hbm_on_input": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9 / peak, 4)},
         "roofline": {"bound": "hbm", "achieved": round(achieved, 2), "peak": peak, "unit": "GB/s",
-                     "frac": round(achieved / peak, 4), "traffic": _traffic_per_launch(),
-                     "kernel": "aatc_decode_query_kernel + aatc_decode_split_kernel + aatc_decode_merge_kernel (one decode call)",
+                     "frac": round(achieved / peak, 4), "traffic": _traffic("decode_layer"),
+                     "kernel": DECODE_KERNELS + " (one decode call)",
                      "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"},
+        "roofline_encode": {"bound": "hbm", "achieved": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9, 2),
+                            "peak": peak, "unit": "GB/s",
+                            "frac": round(enc_in_bytes / (enc_mean * 1e-3) / 1e9 / peak, 4),
+                            "traffic": _traffic("encode_layer"), "algorithmic_bytes": enc_in_bytes,
+                            "kernel": "aatc_encode_kernel (one encode of the layer: bf16 K/V input bytes)",
+                            "peak_source": f"{peak_kind} hbm_gbs (MEASURED_PEAKS.json)"},
         "e2e": {"value": round(ws_ * steps_dec * dbytes / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
                 "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "ms_per_step": round(e2e_ms, 4),
@@ -703,6 +850,7 @@ def run_ours(args):
         "planner": planner_timing(aatc),
         "sink_window": sw,
         "bf16_decode": ref16,
+        "qwen_layer": qwen,
         "decode_llama_stack": stack,
         "encode_hidden": hid,
         "prefill": pre,
@@ -711,6 +859,8 @@ def run_ours(args):
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, avg_bits, budget_s=args.cpu_seconds,
                                             all_cores_s=min(10.0, args.cpu_seconds))
+        line["cpu_baseline"]["oracle_encode_and_planner"] = oracle_encode_timing(cfg, avg_bits)
+        line["cpu_baseline"]["code_agreement"] = oracle_code_agreement(params, caches[0], kd, vd, cfg, plan.n_words)
     print(json.dumps(line), flush=True)
     if ws_ > 1:
         torch.distributed.destroy_process_group()
@@ -801,6 +951,91 @@ def _run_oracle_children(path, budget_s, n_proc):
         out["decodes"] += res["decodes"]
         out["bytes"] += res["bytes"]
     return out, err
+
+
+_ORACLE_ENCODE_CHILD = r"""
+import json, sys, time
+import numpy as np
+sys.path.insert(0, sys.argv[1])
+from oracle import aatc_oracle as O
+import workloads as W
+cfg = W.CONFIGS[sys.argv[2]]
+avg_bits = float(sys.argv[3]); n_tok = int(sys.argv[4]); budget = float(sys.argv[5])
+ck, cv, cq = W.layer_calibration(cfg, 0)
+k, v = W.kv_host(cfg, 0, 1, n_tok)
+g = cfg.group
+t0 = time.perf_counter()
+plans = []
+for h in range(cfg.n_kv_heads):
+    for kind, cal in ((0, ck), (1, cv)):
+        qsh = [cq[j].astype(np.float64) for j in range(h * g, (h + 1) * g)] if kind == 0 else None
+        plans.append(O.plan_stream(cal[h].astype(np.float64), avg_bits, queries_by_head=qsh))
+plan_s = time.perf_counter() - t0
+t0 = time.perf_counter(); reps = 0
+while True:
+    i = 0
+    for h in range(cfg.n_kv_heads):
+        for kind, x in ((0, k), (1, v)):
+            p = plans[i]; i += 1
+            ub = W.to_bf16(p["basis"]).astype(np.float64)
+            codes, alpha, _ = O.encode_stream(x[0, :, h, :].astype(np.float64), ub, p["bits"], p["scales"])
+            O.pack_records(codes, p["bits"], O.record_words([p["bits"]]))
+    reps += 1
+    if time.perf_counter() - t0 > budget:
+        break
+print(json.dumps({"plan_seconds": plan_s, "encode_seconds": time.perf_counter() - t0, "reps": reps}))
+"""
+
+
+def oracle_encode_timing(cfg, avg_bits, n_tokens=2048, budget_s=8.0):
+    """The oracle planner (16 streams of the layer from their 4096-vector calibration sets) and
+    the oracle encode (project, scale, quantize, pack) of n_tokens per stream, on one host thread."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    r = subprocess.run([sys.executable, "-c", _ORACLE_ENCODE_CHILD, ROOT, cfg.name, str(avg_bits), str(n_tokens),
+                        str(budget_s)], capture_output=True, text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        return {"error": r.stderr[-300:]}
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    toks = d["reps"] * n_tokens
+    return {"encode_mtok_s": round(toks / d["encode_seconds"] / 1e6, 6),
+            "encode_input_gbs": round(toks * cfg.n_kv_heads * 2 * 128 * 2 / d["encode_seconds"] / 1e9, 6),
+            "planner_seconds_per_layer": round(d["plan_seconds"], 3), "cores": 1,
+            "sample": f"oracle encode of {n_tokens} tokens x {cfg.n_kv_heads} kv-heads x K|V (numpy fp64, 1 thread), "
+                      f"{d['reps']} repetitions in {d['encode_seconds']:.1f} s; oracle planner of the layer's "
+                      f"{2 * cfg.n_kv_heads} streams from 4096 calibration vectors each"}
+
+
+def oracle_code_agreement(p, cache, kd, vd, cfg, n_words, n_tokens=4096):
+    """The oracle encode of the first n_tokens of every stream with the library's plan (basis,
+    widths, scales), against the codes the GPU wrote into `cache`: codes equal, codes one level
+    off at a decision threshold (|h/Delta - (k + 1/2)| <= 1e-4 relative), and any other
+    difference (must be none)."""
+    from oracle import aatc_oracle as O
+    import torch
+    torch.cuda.synchronize()
+    host = cache.cpu().numpy().view(np.uint32)
+    B, Tc = kd.shape[0], kd.shape[1]
+    n = min(n_tokens, Tc)
+    tot = mis = far = 0
+    for h in range(cfg.n_kv_heads):
+        for kind, x in ((0, kd), (1, vd)):
+            bits = p["bits"][0, h, kind].astype(np.int64)
+            ub = W.to_bf16(p["basis"][0, h, kind]).astype(np.float64)
+            xs = x[0, :n, h].float().cpu().numpy().astype(np.float64)
+            codes, _, t = O.encode_stream(xs, ub, bits, p["scales"][0, h, kind].astype(np.float64))
+            rec, _ = O.cache_records(host, B, cfg.n_kv_heads, Tc, n_words, 0, h, kind, 0, n)
+            got = O.unpack_records(rec, bits)
+            keep = bits > 0
+            diff = got[:, keep] - codes[:, keep]
+            tk = t[:, keep]
+            thr = np.floor(tk) + 0.5
+            near = np.abs(tk - thr) <= 1e-4 * np.abs(thr)
+            tot += int(keep.sum()) * n
+            mis += int(np.count_nonzero(diff))
+            far += int(np.count_nonzero((diff != 0) & ~((np.abs(diff) == 1) & near)))
+    return {"codes": tot, "near_threshold_one_level": mis - far, "other_differences": far,
+            "fraction": mis / max(tot, 1),
+            "sample": f"first {n} tokens of sequence 0, all {cfg.n_kv_heads} kv-heads x K|V, library plan"}
 
 
 def cpu_baseline(cfg, avg_bits, budget_s=15.0, n_tokens=4096, all_cores_s=0.0):

@@ -128,7 +128,7 @@ aatc_status_t aatc_calibrate_head_group(int32_t g_h, int32_t group, const float*
 
 /*
  * Global cross-layer bit allocation (Sec. 5 "waterfilling problem for the keys / values" summed
- * over layers; Algorithm 1 "Allocate bits globally via reverse waterfilling over all (l, c)";
+ * over layers; Algorithm 1, global reverse water-filling over every (layer, channel) pair;
  * the experimental-setup paragraph on AATC for the normalisation and the protected layers).
  * Replaces the per-stream budgets of aatc_calibrate with one pool per kind (keys, values):
  *   - layers l < n_protect get a per-stream allocation with avg_bits_v * 128 bits for values and
@@ -325,7 +325,10 @@ aatc_status_t aatc_decode_attention(aatc_plan_t plan, int32_t layer, const void*
  *   q       : device bf16 [batch][n_q_heads][128]
  *   cache   : packed cache as written by aatc_encode; only [t_first, t_end) is read
  *   k_full, v_full : device bf16 [batch][full_cap][n_kv_heads][128]; the first n_full tokens of
- *             each sequence are attended (n_full may be 0; k_full/v_full may then be NULL)
+ *             each sequence are attended (n_full may be 0; k_full/v_full may then be NULL).
+ *             full_cap is the row stride between sequences, so the pointers may point at any
+ *             row of a larger per-sequence buffer as long as every sequence's n_full rows lie
+ *             inside it (a sink / window block kept in place inside a ring-like buffer).
  *   out     : device fp32 [batch][n_q_heads][128]
  *   workspace : as for aatc_decode_attention with n_ctx = t_end (not read when t_first == t_end)
  * Errors: AATC_ERR_INVALID_ARG (t_first > t_end, both sets empty, full_cap < n_full, unaligned
@@ -375,6 +378,8 @@ aatc_status_t aatc_get_device_error(aatc_plan_t plan, int32_t* flags, int32_t cl
  * GPU that loads it, until the process exits.  Nothing is allocated or freed by this call.
  *   - The first call on a device looks up that device's scratch address (with the device
  *     current); make that first call before any stream capture.
+ *   - Call with the plan's device current: the array used is the current device's, so a call
+ *     made with another device current returns AATC_ERR_INVALID_ARG before any launch.
  *   - Every call on a device shares the one array, and it keeps the previous call's contents.
  *     Nothing in it has to start at zero (each partial is written before it is read), but
  *     calls that overlap on the GPU (different streams, or concurrent host threads) race on it:

@@ -183,7 +183,7 @@ def continuous_allocation(g: np.ndarray, budget: float, b_max: float = np.inf):
 def global_allocation(sigma2: np.ndarray, weights: np.ndarray, avg_bits_k: float, avg_bits_v: float,
                       n_protect: int = 3, b_max: int = 8) -> np.ndarray:
     """Global cross-layer allocation (Eq. waterfilling-keys and its value twin, both summed over
-    layers; Algorithm 1 'Allocate bits globally via reverse waterfilling over all (l, c)'; the
+    layers; Algorithm 1, global reverse water-filling over every (layer, channel) pair; the
     AATC experimental-setup paragraph for the protected layers and the normalisation).
 
     sigma2, weights: [L][H][2][d] (kind 0 keys, 1 values), channels in storage order.

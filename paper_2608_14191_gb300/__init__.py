@@ -439,9 +439,11 @@ def decode_attention(plan: Plan, layer: int, q, cache, n_ctx: int, max_tokens: i
 
 
 def decode_attention_sw(plan: Plan, layer: int, q, cache, t_first: int, t_end: int, max_tokens: int,
-                        k_full=None, v_full=None, n_full: int = 0, out=None, workspace=None, stream=None):
-    """aatc_decode_attention_sw: packed tokens [t_first, t_end) plus the first n_full tokens of
-    k_full / v_full (bf16 [batch][cap][H_kv][128]) in one softmax -> fp32 [batch][H_q][128]."""
+                        k_full=None, v_full=None, n_full: int = 0, out=None, workspace=None, stream=None,
+                        full_row0: int = 0):
+    """aatc_decode_attention_sw: packed tokens [t_first, t_end) plus the n_full tokens at rows
+    [full_row0, full_row0 + n_full) of k_full / v_full (bf16 [batch][cap][H_kv][128]; the row
+    stride between sequences stays cap) in one softmax -> fp32 [batch][H_q][128]."""
     import torch
     where = "aatc_decode_attention_sw"
     _dev_tensor(q, where, "q", torch.bfloat16, 3, (None, plan.dims.n_q_heads, HEAD_DIM))
@@ -454,14 +456,19 @@ def decode_attention_sw(plan: Plan, layer: int, q, cache, t_first: int, t_end: i
         out = torch.empty((batch, plan.dims.n_q_heads, HEAD_DIM), dtype=torch.float32, device=q.device)
     _out_ok(out, batch * plan.dims.n_q_heads * HEAD_DIM, where)
     cap = 0 if k_full is None else int(k_full.shape[1])
+    if full_row0 < 0 or (k_full is not None and (not k_full.is_contiguous() or not v_full.is_contiguous()
+                                                 or full_row0 + int(n_full) > cap)):
+        _arg_error(where, "k_full / v_full must be contiguous and hold rows [full_row0, full_row0 + n_full)")
     if t_end > t_first and workspace is None:
         workspace = torch.empty(max(1, plan.workspace_bytes(batch, t_end) // 4), dtype=torch.float32,
                                 device=q.device)
     ws_ptr = None if workspace is None else _ptr(workspace)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    row_bytes = int(full_row0) * plan.dims.n_kv_heads * HEAD_DIM * 2
     _check(load().aatc_decode_attention_sw(plan.handle, layer, _ptr(q), _ptr(cache), batch, t_first, t_end,
-                                           max_tokens, None if k_full is None else _ptr(k_full),
-                                           None if v_full is None else _ptr(v_full), int(n_full), cap, _ptr(out),
+                                           max_tokens, None if k_full is None else _ptr(k_full) + row_bytes,
+                                           None if v_full is None else _ptr(v_full) + row_bytes, int(n_full), cap,
+                                           _ptr(out),
                                            ws_ptr, ws_bytes, _stream(stream)), "aatc_decode_attention_sw")
     return out
 

@@ -133,6 +133,12 @@ size_t bf16_decode_workspace(int batch, int n_q, const DecodeSplit& sp);
 Plan* plan_from_handle(aatc_plan_t p);
 aatc_status_t status_from_cuda(cudaError_t e);
 
+// Raise `kernel`'s dynamic shared-memory limit on the current device to at least `bytes`.  The
+// attribute belongs to a (device, kernel) pair, so what has been set is recorded per device and
+// kernel under one mutex: host threads making first calls at the same time, and a process that
+// drives several GPUs, both get the opt-in on every device they launch on (defined in capi.cpp).
+cudaError_t ensure_smem_optin(const void* kernel, size_t bytes);
+
 // Kernel launchers (defined in the .cu files); return the CUDA error of the launch.
 // 2D tiled tensor map with 128-byte swizzle (16-bit elements): `map` is a 128-byte, 64-aligned
 // CUtensorMap; rows of `inner` elements, `row_bytes` apart; box box_inner x box_rows.

@@ -3,7 +3,10 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <new>
+#include <utility>
 #include <vector>
 
 #include "aatc.h"
@@ -71,6 +74,20 @@ DecodeSplit bf16_decode_split(int batch, int n_kv, int n_q, int n_ctx, int num_s
 Plan* plan_from_handle(aatc_plan_t p) { return as_plan(p); }
 
 aatc_status_t status_from_cuda(cudaError_t e) { return cuda_status(e); }
+
+cudaError_t ensure_smem_optin(const void* kernel, size_t bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, size_t> done;   // (device, kernel) -> bytes set
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  size_t& have = done[std::make_pair(dev, kernel)];
+  if (bytes <= have) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  if (e == cudaSuccess) have = bytes;
+  return e;
+}
 
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
   DecodeWs w;

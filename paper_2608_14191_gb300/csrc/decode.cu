@@ -6,16 +6,16 @@
 // dependent of the one before it:
 //   query    per (sequence, kv-head, query slot): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the
 //            G query heads of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1),
-//            and q' as e4m3 tensor-core fragments (four limbs);
+//            and q' per record entry as f16 hi/lo tensor-core fragments (mma.sync m16n8k16);
 //   split    per (split, kv-head, sequence): pass 1 scores
-//            s_{g,t} = alpha^K_t (sum_e q'_{g,e} digit_{t,e} - C_g) on the fp8 tensor cores over
-//            the packed digits; split max m_g; pass 2 p = 2^(s - m_g), P' = p alpha^V_t, value
-//            entry sums sum_t P'_{g,t} digit_{t,e} on the tensor cores; entry sums folded into
-//            channel sums with the offset correction; (o, m, l) per split;
+//            s_{g,t} = alpha^K_t (sum_e q'_{g,e} digit_{t,e} - C_g) by f16 mma.sync over the
+//            packed digits (each masked in place as a subnormal f16); split max m_g; pass 2
+//            p = 2^(s - m_g), P' = p alpha^V_t as f16 hi/lo, value entry sums
+//            sum_t P'_{g,t} digit_{t,e} by the same MMA; entry sums folded into channel sums with
+//            the offset correction; (o, m, l) per split;
 //   merge    per (sequence, query head): log-sum-exp merge of the splits, f^V / l, out = U_V o_hat.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
-#include <cuda_fp8.h>
 
 #include <algorithm>
 #include <mutex>
@@ -1125,13 +1125,8 @@ cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t sm
 
 template <int JPW, int NP>
 cudaError_t launch_split_t(const DecodeArgs& a, int batch, size_t smem, cudaStream_t st) {
-  static size_t smem_set = 0;                                  // raise the opt-in limit only when needed
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_decode_split_kernel<JPW, NP>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    smem_set = smem;
-  }
+  cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_split_kernel<JPW, NP>), smem);
+  if (e != cudaSuccess) return e;
   return launch_pdl(aatc_decode_split_kernel<JPW, NP>, dim3(a.n_splits, a.n_kv, batch), dim3(kThreads), smem, st, a);
 }
 
@@ -1145,13 +1140,8 @@ cudaError_t launch_split_g(const DecodeArgs& a, int batch, int jpw, size_t smem,
 template <int GP>
 cudaError_t launch_bf16_split(const Bf16Args& a, int batch, cudaStream_t st) {
   const size_t smem = bf16_split_smem(GP, a.split_len);
-  static size_t smem_set = 0;
-  if (smem > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_bf16_split_kernel<GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    smem_set = smem;
-  }
+  cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_bf16_split_kernel<GP>), smem);
+  if (e != cudaSuccess) return e;
   aatc_bf16_split_kernel<GP><<<dim3(a.n_splits, a.n_kv, batch), kThreads, smem, st>>>(a);
   return cudaGetLastError();
 }
@@ -1224,13 +1214,8 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   }
   const size_t msmem = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
   if (msmem > 227 * 1024) return cudaErrorNotSupported;
-  static size_t msmem_set = 0;
-  if (msmem > msmem_set) {
-    e = cudaFuncSetAttribute(aatc_decode_merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(msmem));
-    if (e != cudaSuccess) return e;
-    msmem_set = msmem;
-  }
+  e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msmem);
+  if (e != cudaSuccess) return e;
   return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msmem, st, a);
 }
 
@@ -1309,6 +1294,7 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return status_from_cuda(e);
+  if (dev != plan->device) return AATC_ERR_INVALID_ARG;       // the array used is the current device's
   if (dev < 0 || dev >= kMaxDevices) return AATC_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   {

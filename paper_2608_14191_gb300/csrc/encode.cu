@@ -617,13 +617,8 @@ cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void
   if (k > items_per_basis) k = static_cast<int>(items_per_basis);
   a.ctas_per_basis = k;
   const size_t smem = sizeof(EncodeSmem) + 1024;
-  static bool attr_done = false;
-  if (!attr_done) {
-    e = cudaFuncSetAttribute(aatc_encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_kernel), smem);
+  if (e != cudaSuccess) return e;
   const auto* mu = reinterpret_cast<const CUtensorMap*>(plan.tmap_u);
   aatc_encode_kernel<<<n_basis * k, kThreads, smem, st>>>(mk, mv, *mu, a);
   return cudaGetLastError();
@@ -680,13 +675,8 @@ cudaError_t launch_encode_hidden(const Plan& plan, int layer, const void* x, int
   long per_head = std::max(1, plan.num_sms / a.n_kv);
   per_head = std::min(per_head, n_items);
   const size_t smem = sizeof(EncodeHiddenSmem) + 1024;
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(aatc_encode_hidden_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_hidden_kernel), smem);
+  if (e != cudaSuccess) return e;
   aatc_encode_hidden_kernel<<<static_cast<unsigned>(per_head * a.n_kv), kThreads, smem, st>>>(mx, ma, a);
   return cudaGetLastError();
 }

@@ -623,14 +623,9 @@ cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_sta
   alignas(64) unsigned char tmap[128];
   e = make_tensor_map_2d(tmap, true, ws, D, static_cast<uint64_t>(batch) * a.n_kv * 2 * a.n_ctx_pad, D * 2, 64, TILE);
   if (e != cudaSuccess) return e;
-  static bool attr_done = false;
   const size_t smem = sizeof(PrefillTcSmem) + 1024;
-  if (!attr_done) {
-    e = cudaFuncSetAttribute(aatc_prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_prefill_tc_kernel), smem);
+  if (e != cudaSuccess) return e;
   const int n_rows = n_q * a.group;
   aatc_prefill_tc_kernel<<<dim3((n_rows + kTRows - 1) / kTRows, a.n_kv, batch), kTThreads, smem, st>>>(
       *reinterpret_cast<const CUtensorMap*>(tmap), a);

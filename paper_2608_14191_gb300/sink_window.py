@@ -54,43 +54,86 @@ class SinkWindowState:
 
 
 class SinkWindowCache:
-    """One layer of a batch of sequences: packed cache + bf16 sink and window on the device."""
+    """One layer of a batch of sequences: packed cache + bf16 sink and window on the device.
+
+    The sink and window live in one buffer of `sink + window + step + spare` rows per sequence
+    as a contiguous block [sink | window] starting at row `y` (window tokens oldest first).  An
+    append writes its new tokens in place after the window; a flush codes the oldest `step`
+    window tokens (from their rows) and moves the block start up by the flushed count, copying
+    only the sink rows; when the block would run past the buffer's end it is moved back to row 0
+    once (every spare / step flushes).  The decode reads the block where it is, so no token is
+    copied per append."""
 
     def __init__(self, plan, layer: int, batch: int, max_tokens: int, device, sink: int = 4,
-                 window: int = 128, step: int = 16):
+                 window: int = 128, step: int = 16, spare_flushes: int = 64):
         import torch
         self.plan, self.layer, self.batch, self.max_tokens = plan, layer, batch, max_tokens
         self.state = SinkWindowState(sink, window, step)
         h = plan.dims.n_kv_heads
-        cap = sink + window + step
+        self.cap = sink + window + step + step * max(0, spare_flushes)
         self.cache = plan.new_cache(batch, max_tokens, device)
-        self.k_full = torch.zeros((batch, cap, h, HEAD_DIM), dtype=torch.bfloat16, device=device)
+        self.k_full = torch.zeros((batch, self.cap, h, HEAD_DIM), dtype=torch.bfloat16, device=device)
         self.v_full = torch.zeros_like(self.k_full)
+        self.y = 0                      # first row of the [sink | window] block
+        self.relocations = 0
+
+    def _rows(self, a, b):
+        return self.k_full[:, a:b], self.v_full[:, a:b]
 
     def append(self, k, v):
         """k, v: device bf16 [batch][m][H_kv][128], the next m tokens of every sequence."""
         import torch
         st = self.state
+        S = st.sink
+        m = k.shape[1]
         s0, n_win0 = st.n_sink, st.n_window
-        to_sink, n_flush, pos = st.append(k.shape[1])
+        to_sink, n_flush, pos = st.append(m)
+        y = self.y
         if to_sink:
-            self.k_full[:, s0:s0 + to_sink] = k[:, :to_sink]
-            self.v_full[:, s0:s0 + to_sink] = v[:, :to_sink]
-        s = st.sink
-        ks = torch.cat([self.k_full[:, s:s + n_win0], k[:, to_sink:]], dim=1)
-        vs = torch.cat([self.v_full[:, s:s + n_win0], v[:, to_sink:]], dim=1)
+            self.k_full[:, y + s0:y + s0 + to_sink] = k[:, :to_sink]
+            self.v_full[:, y + s0:y + s0 + to_sink] = v[:, :to_sink]
+        r = m - to_sink
+        kn, vn = k[:, to_sink:], v[:, to_sink:]
         if n_flush:
+            # the oldest n_flush tokens of (old window ++ new tokens) go to the coded cache
             if pos + n_flush > self.max_tokens:
                 raise ValueError("packed cache capacity exceeded")
-            encode(self.plan, self.layer, ks[:, :n_flush].contiguous(), vs[:, :n_flush].contiguous(), self.cache,
-                   pos, self.max_tokens)
-        n_win = st.n_window
-        self.k_full[:, s:s + n_win] = ks[:, n_flush:]
-        self.v_full[:, s:s + n_win] = vs[:, n_flush:]
+            from_old = min(n_flush, n_win0)
+            ko, vo = self._rows(y + S, y + S + from_old)
+            if n_flush > from_old:
+                kf = torch.cat([ko, kn[:, :n_flush - from_old]], dim=1)
+                vf = torch.cat([vo, vn[:, :n_flush - from_old]], dim=1)
+            else:
+                kf, vf = ko.contiguous(), vo.contiguous()
+            encode(self.plan, self.layer, kf, vf, self.cache, pos, self.max_tokens)
+        if r == 0 and n_flush == 0:
+            return
+        old_keep = max(0, n_win0 - n_flush)          # old window tokens kept (the newest of them)
+        new_keep = r - max(0, n_flush - n_win0)      # new tokens kept (the tail of the append)
+        y1 = y + (n_win0 - old_keep)                 # the block start follows the kept tokens
+        if y1 + S + old_keep + new_keep > self.cap:
+            # move the block (sink and kept window tokens) back to row 0
+            kb = torch.cat([self.k_full[:, y:y + S], self.k_full[:, y1 + S:y1 + S + old_keep]], dim=1)
+            vb = torch.cat([self.v_full[:, y:y + S], self.v_full[:, y1 + S:y1 + S + old_keep]], dim=1)
+            if S + old_keep + new_keep > self.cap:
+                raise ValueError("append longer than the window buffer")
+            self.k_full[:, :S + old_keep] = kb
+            self.v_full[:, :S + old_keep] = vb
+            y1 = 0
+            self.relocations += 1
+        elif y1 != y and S:
+            ks, vs = self.k_full[:, y:y + S].clone(), self.v_full[:, y:y + S].clone()
+            self.k_full[:, y1:y1 + S] = ks
+            self.v_full[:, y1:y1 + S] = vs
+        if new_keep:
+            a = y1 + S + old_keep
+            self.k_full[:, a:a + new_keep] = kn[:, r - new_keep:]
+            self.v_full[:, a:a + new_keep] = vn[:, r - new_keep:]
+        self.y = y1
 
     def decode(self, q, out=None, workspace=None, stream=None):
         st = self.state
         n_full = st.n_sink + st.n_window
         return decode_attention_sw(self.plan, self.layer, q, self.cache, st.sink, st.sink + st.n_coded,
                                    self.max_tokens, self.k_full, self.v_full, n_full, out=out, workspace=workspace,
-                                   stream=stream)
+                                   stream=stream, full_row0=self.y)

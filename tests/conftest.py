@@ -38,3 +38,31 @@ def aatc():
     import paper_2608_14191_gb300 as m
     m.load()
     return m
+
+
+@pytest.fixture(scope="session")
+def oracle_pool():
+    """Spawned worker processes for the oracle side of the full-size parity checks (numpy only;
+    spawn, so no worker inherits this process's CUDA state)."""
+    import multiprocessing as mp
+    n = max(1, min(16, len(os.sched_getaffinity(0))))
+    pool = mp.get_context("spawn").Pool(n)
+    try:
+        yield pool
+    finally:
+        pool.close()
+        pool.join()
+
+
+def pytest_terminal_summary(terminalreporter):
+    try:
+        import harness
+    except Exception:  # pragma: no cover
+        return
+    rows = harness.NearThreshold.rows
+    if not rows:
+        return
+    terminalreporter.section("near-threshold codes (one level off, |h/Delta - (k + 1/2)| <= 1e-4 rel)")
+    for name, (mis, tot, near) in sorted(rows.items()):
+        terminalreporter.write_line(f"{name}: {mis} of {tot} codes ({mis / max(tot, 1):.2e}); "
+                                    f"{near} codes near a threshold in the oracle")

@@ -51,7 +51,8 @@ def _check_all(case, cache, x_host, batch, max_tokens, t0, n):
                                    encode_matrix=case.a_hat_host[0, h, kind].T)
                 stats["codes"] += s["codes"]
                 stats["mismatch"] += s["mismatch"]
-    assert stats["mismatch"] <= Hn.MAX_NEAR_FRACTION * stats["codes"] + 1, stats
+                Hn.NearThreshold.add("hidden-state encode (small cases)", s["mismatch"], s["codes"], s["near"])
+    Hn.NearThreshold.assert_bound("hidden-state encode (small cases)")
     return u32
 
 
@@ -102,7 +103,8 @@ def test_encode_hidden_argument_errors(aatc):
 
 def test_encode_hidden_llama_shape_sampled(aatc):
     """Bench configuration: Llama-3.1-8B-shaped layer input (d_model 4096, 8 kv-heads), 32768
-    tokens in the launch the bench times; codes and scales compared on sampled heads and tokens."""
+    tokens in the launch the bench times; codes and scales of every kv-head compared on 256
+    sampled tokens (the oracle's fp64 projection over d_model 4096 is the slow part)."""
     d_model, n_kv, n_tok = 4096, 8, 32768
     case = HiddenCase(aatc, d_model, n_kv=n_kv, n_q=32)
     x = W.hidden_states_device(SEED, 0, d_model, 1, n_tok, DEV)
@@ -115,11 +117,13 @@ def test_encode_hidden_llama_shape_sampled(aatc):
     toks = np.sort(rng.choice(n_tok, 256, replace=False))
     xs = x[0, torch.from_numpy(toks).to(DEV)].float().cpu().numpy()
     total = mis = 0
-    for h in (0, 5):
+    for h in range(n_kv):
         for kind in (0, 1):
             rec_all, alpha_all = O.cache_records(u32, 1, n_kv, n_tok, case.plan.n_words, 0, h, kind, 0, n_tok)
             s = Hn.check_codes(case, 0, h, kind, xs, rec_all[toks], alpha_all[toks],
                                encode_matrix=case.a_hat_host[0, h, kind].T)
             total += s["codes"]
             mis += s["mismatch"]
-    assert mis <= Hn.MAX_NEAR_FRACTION * total + 1, (mis, total)
+            Hn.NearThreshold.add("hidden-state encode (Llama layer input, 256 tokens x 8 kv-heads)", s["mismatch"],
+                                 s["codes"], s["near"])
+    Hn.NearThreshold.assert_bound("hidden-state encode (Llama layer input, 256 tokens x 8 kv-heads)")

@@ -103,7 +103,7 @@ def test_sink_window_cache_streaming(aatc):
 
 def test_sw_decode_llama_layer_full_size(aatc):
     """Llama-shaped layer at 32768 tokens with the paper's policy: sink 4, window 140, coded
-    [4, 32628); sampled heads against the oracle."""
+    [4, 32628); every kv-head and query head against the oracle."""
     cfg = W.CONFIGS["llama_layer"]
     case = Hn.Case(aatc, cfg, 2.75)
     T = cfg.n_ctx
@@ -120,7 +120,7 @@ def test_sw_decode_llama_layer_full_size(aatc):
     out = aatc.decode_attention_sw(case.plan, 0, q, cache, n_sink, n_sink + n_coded, T, kf, vf,
                                    len(full_idx)).cpu().numpy()
     qh = q.float().cpu().numpy()[0]
-    for h in (0, cfg.n_kv_heads - 1):
+    for h in range(cfg.n_kv_heads):
         rk, ak = Hn.read_stream(case, host, 1, T, 0, h, 0, n_sink, n_coded)
         rv, av = Hn.read_stream(case, host, 1, T, 0, h, 1, n_sink, n_coded)
         _, bk, sk = case.stream(0, h, 0)

@@ -78,3 +78,52 @@ def test_cache_manager_bookkeeping_matches_policy():
         assert to_sink == O.sink_window_counts(n)[0] - O.sink_window_counts(n - m)[0]
         pos += n_flush
     assert pos == 4 + st.n_coded
+
+
+class _FakePlan:
+    """Just enough of a Plan for the cache manager's host logic on CPU tensors."""
+
+    class dims:
+        n_kv_heads = 2
+
+    def new_cache(self, batch, max_tokens, device):
+        import torch
+        return torch.zeros(8, dtype=torch.int32)
+
+
+@pytest.mark.parametrize("spare", [64, 1])
+def test_cache_manager_keeps_sink_and_window_in_place(monkeypatch, spare):
+    """SinkWindowCache on CPU tensors with the encode call recorded: after every append the block
+    [y, y + n_sink + n_window) holds the sink tokens and then the newest window tokens in order,
+    the flushed tokens are exactly the coded positions in order, and appends of one token copy
+    no window token (only a flush moves the four sink rows, and the block is moved back to row 0
+    once every `spare` flushes)."""
+    import torch
+    import paper_2608_14191_gb300.sink_window as sw
+    coded = []
+
+    def fake_encode(plan, layer, k, v, cache, pos, max_tokens):
+        assert k.is_contiguous() and v.is_contiguous() and torch.equal(k, v - 0.5)
+        assert pos == 4 + sum(c.shape[1] for c in coded)
+        coded.append(k.clone())
+
+    monkeypatch.setattr(sw, "encode", fake_encode)
+    batch, H, n_max = 2, 2, 3000
+    tok = torch.arange(batch * n_max, dtype=torch.float32).reshape(batch, n_max, 1, 1).expand(batch, n_max, H, 128)
+    swc = sw.SinkWindowCache(_FakePlan(), 0, batch, n_max, "cpu", spare_flushes=spare)
+    swc.k_full = swc.k_full.float()
+    swc.v_full = swc.v_full.float()
+    n = 0
+    for m in [1, 2, 1, 200, 16, 15, 1, 1, 40, 333] + [1] * 300 + [17, 5, 900]:
+        swc.append(tok[:, n:n + m].contiguous(), tok[:, n:n + m].contiguous() + 0.5)
+        n += m
+        st = swc.state
+        assert (st.n_sink, st.n_coded, st.n_window) == O.sink_window_counts(n)
+        want = list(range(st.n_sink)) + list(range(st.sink + st.n_coded, n))
+        blk = swc.k_full[:, swc.y:swc.y + len(want), 0, 0]
+        assert torch.equal(blk, tok[:, want, 0, 0]), n
+        assert torch.equal(swc.v_full[:, swc.y:swc.y + len(want), 0, 0], blk + 0.5)
+    got = torch.cat(coded, dim=1)[:, :, 0, 0]
+    assert torch.equal(got, tok[:, 4:4 + swc.state.n_coded, 0, 0])
+    if spare == 64:
+        assert swc.relocations <= 1 + swc.state.n_coded // (16 * 64)

@@ -44,3 +44,18 @@ def test_calibration_and_data_are_bf16_exact_and_distinct():
     x = W.calibration_vectors(CFG, 0, 1, W.KIND_V).astype(np.float64)
     emp = np.sort(np.linalg.eigvalsh(x.T @ x / x.shape[0]))[::-1]
     assert np.abs(emp[:8] / W.power_law()[:8] - 1).max() < 0.1
+
+
+def test_bf16_rounding_matches_torch_cast():
+    """to_bf16 (round to nearest even on the float32 bit pattern) gives the same values as
+    torch's float32 -> bfloat16 cast: random magnitudes over 2^+-86, exact ties both ways,
+    signed zeros, subnormals and the largest finite bf16 values."""
+    import torch
+    rng = np.random.default_rng(0)
+    x = (rng.standard_normal(1 << 18) * np.exp(rng.uniform(-60, 60, 1 << 18))).astype(np.float32)
+    ties = (np.arange(1, 4097, dtype=np.uint32) << 16 | 0x8000).view(np.float32)
+    x = np.concatenate([x, ties, -ties, np.array([0.0, -0.0, 3.3895314e38, -3.3895314e38, 1e-40, -1e-40],
+                                                 np.float32)])
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float32).numpy()
+    assert np.array_equal(W.to_bf16(x).view(np.uint32), ref.view(np.uint32))
+    assert W.to_bf16(x.reshape(-1, 2)).shape == (x.size // 2, 2)

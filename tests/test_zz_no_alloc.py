@@ -37,6 +37,8 @@ def test_noalloc_decode_matches_workspace_decode_twice(aatc):
                                                cfg.n_ctx, out.data_ptr(), stream)
         assert st == 0, st
         torch.cuda.synchronize()
+        # the same kernels with the same split plan: bit for bit the workspace decode's outputs
+        assert torch.equal(out, ref), float((out - ref).abs().max())
         Hn.check_decode(out.cpu().numpy()[0], ref.cpu().numpy()[0].astype(np.float64))
     # a request whose split partials exceed the fixed scratch is refused before any launch
     need = ctypes.c_size_t()

@@ -120,10 +120,14 @@ def stream_model(seed: int, layer: int, head: int, kind: int) -> StreamModel:
 
 
 def to_bf16(x):
-    """Round float data to bf16 (round-to-nearest-even); returns float32 numpy values."""
-    import torch
-    t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32))
-    return t.to(torch.bfloat16).to(torch.float32).numpy()
+    """Round float data to bf16 (round-to-nearest-even on the float32 value); returns float32
+    numpy values.  Done on the float32 bit pattern: add 0x7FFF plus the lowest kept bit, then
+    clear the low 16 bits (the same values as torch's float32 -> bfloat16 cast for finite
+    inputs, which tests/test_workloads.py checks)."""
+    f = np.ascontiguousarray(x, dtype=np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32).reshape(f.shape)
 
 
 def calibration_vectors(cfg: Config, layer: int, head: int, kind: int, n: int = N_CALIB) -> np.ndarray:
