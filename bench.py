@@ -35,7 +35,8 @@ sys.path.insert(0, ROOT)
 import workloads as W  # noqa: E402
 
 METRIC = "compressed-KV decode attn GB/s & % of HBM peak; encode Mtok/s (1 GB300)"
-DECODE_KERNELS = "aatc_decode_query_kernel + aatc_decode_split_kernel + aatc_decode_merge_kernel"
+DECODE_KERNELS = "aatc_decode_fused_kernel"        # one launch per decode call (per-stream plans)
+DECODE_LAUNCHES_PER_CALL = 1
 N_COPIES = 16
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -845,7 +846,7 @@ def run_ours(args):
                 "what": "per step: H2D of K, V and queries from pinned host memory, encode, 256 decode calls "
                         "through the public API, D2H of all outputs; the next step's H2D and this step's "
                         "D2H run on a second stream, overlapping compute"},
-        "gpu_launches": args.steps * (1 + 3 * steps_dec),
+        "gpu_launches": args.steps * (1 + DECODE_LAUNCHES_PER_CALL * steps_dec),
         "clocks": clocks,
         "planner": planner_timing(aatc),
         "sink_window": sw,

@@ -122,10 +122,19 @@ size_t bf16_split_smem(int gp, int split_len);
 struct DecodeWs {
   int pstride;            // floats per partial
   int ks_stride;          // uint4 per (sequence, kv-head) fragment block
-  size_t qfrag_off, qcorr_off, bytes;
+  size_t qfrag_off, qcorr_off, sem_off, bytes;   // sem: a 64-bit completion flag per (sequence, kv-head, split)
 };
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
 size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
+// The decode has two launch plans: the fused split + merge kernel (CTAs of 8-16 warps, about
+// FUSED_CTAS_PER_SM per SM) for layers whose streams share one of the record shapes it is built
+// for, and the split + merge kernels (about 5 CTAs per SM, at most 16 tiles per split) for any
+// other layer.  `range` = the packed tokens a call covers, counted from the first tile it reads.
+constexpr int FUSED_CTAS_PER_SM = 1;
+DecodeSplit decode_split_for(int batch, int n_kv, int range, int num_sms, bool fused);
+// Workspace bytes that serve a decode of `range` tokens on any layer of the plan, whichever path
+// it takes.
+size_t decode_workspace_for(const Plan& plan, int batch, int range);
 // bf16 reference decode partials: 128 sums, then m, l, padding
 size_t bf16_decode_workspace(int batch, int n_q, const DecodeSplit& sp);
 
@@ -162,8 +171,8 @@ struct DecodeExtra {
 };
 constexpr int MAX_FULL_TOKENS = 8192;   // shared-memory scores of the uncompressed tokens
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch,
-                          int n_ctx, int max_tokens, float* out, void* ws, const DecodeSplit& sp,
-                          cudaStream_t st, const DecodeExtra& extra);
+                          int n_ctx, int max_tokens, float* out, void* ws, cudaStream_t st,
+                          const DecodeExtra& extra);
 // Prefill attention: codes workspace bytes, and the two launches (codes, attention).
 size_t prefill_workspace(int batch, int n_kv, int n_ctx);
 cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_start, int n_q, const void* cache,

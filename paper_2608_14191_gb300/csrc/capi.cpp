@@ -95,8 +95,31 @@ DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_wor
   w.ks_stride = 2 * n_words * 32;                 // >= score k16-steps (<= 2 W) x 32 lanes
   w.qfrag_off = align_up(static_cast<size_t>(batch) * n_q * sp.n_splits * w.pstride * sizeof(float), 256);
   w.qcorr_off = align_up(w.qfrag_off + static_cast<size_t>(batch) * n_kv * w.ks_stride * 16, 256);
-  w.bytes = w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float);
+  w.sem_off = align_up(w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float), 256);
+  w.bytes = w.sem_off + static_cast<size_t>(batch) * n_kv * sp.n_splits * sizeof(unsigned long long);
   return w;
+}
+
+DecodeSplit decode_split_for(int batch, int n_kv, int range, int num_sms, bool fused) {
+  if (!fused) return decode_split(batch, n_kv, std::max(range, 1), num_sms, 5);
+  // fused kernel: one wave of at most FUSED_CTAS_PER_SM CTAs per SM; split lengths are not
+  // bounded (the online softmax keeps no per-token scores)
+  const long tiles = (static_cast<long>(std::max(range, 1)) + TILE - 1) / TILE;
+  const long units = static_cast<long>(batch) * n_kv;
+  long n = static_cast<long>(FUSED_CTAS_PER_SM) * std::max(1, num_sms) / units;
+  n = std::max(1L, std::min(n, tiles));
+  DecodeSplit sp;
+  sp.n_splits = static_cast<int>(n);
+  sp.split_len = static_cast<int>((tiles + n - 1) / n) * TILE;
+  return sp;
+}
+
+size_t decode_workspace_for(const Plan& plan, int batch, int range) {
+  const int hq = plan.dims.n_q_heads, hk = plan.dims.n_kv_heads;
+  return std::max(decode_workspace(batch, hq, hk, plan.n_entries, plan.n_words,
+                                   decode_split_for(batch, hk, range, plan.num_sms, false)),
+                  decode_workspace(batch, hq, hk, plan.n_entries, plan.n_words,
+                                   decode_split_for(batch, hk, range, plan.num_sms, true)));
 }
 
 size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp) {
@@ -393,9 +416,7 @@ aatc_status_t aatc_prefill_attention(aatc_plan_t p, int32_t layer, const void* q
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
-  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  *bytes = aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries,
-                                  plan->n_words, sp);
+  *bytes = aatc::decode_workspace_for(*plan, batch, n_ctx);
   return AATC_OK;
 }
 
@@ -409,12 +430,9 @@ aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q,
   if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if (!aligned16(cache) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
-  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries,
-                                               plan->n_words, sp))
-    return AATC_ERR_WORKSPACE;
+  if (workspace_bytes < aatc::decode_workspace_for(*plan, batch, n_ctx)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
-                                         workspace, sp, static_cast<cudaStream_t>(stream), aatc::DecodeExtra{}));
+                                         workspace, static_cast<cudaStream_t>(stream), aatc::DecodeExtra{}));
 }
 
 aatc_status_t aatc_decode_attention_sw(aatc_plan_t p, int32_t layer, const void* q, const void* cache,
@@ -432,12 +450,9 @@ aatc_status_t aatc_decode_attention_sw(aatc_plan_t p, int32_t layer, const void*
   // the packed part covers tiles [t_first / 128, ceil(t_end / 128)): never more splits than a
   // plain decode of t_end tokens, so aatc_decode_workspace_bytes(batch, t_end) suffices
   const int range = t_end - (t_first / aatc::TILE) * aatc::TILE;
-  const auto sp = aatc::decode_split(batch, plan->dims.n_kv_heads, std::max(range, 1), plan->num_sms);
   if (t_end > t_first) {
     if (!workspace || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
-    if (workspace_bytes < aatc::decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads,
-                                                 plan->n_entries, plan->n_words, sp))
-      return AATC_ERR_WORKSPACE;
+    if (workspace_bytes < aatc::decode_workspace_for(*plan, batch, range)) return AATC_ERR_WORKSPACE;
   }
   aatc::DecodeExtra ex;
   ex.t_first = t_first;
@@ -445,7 +460,7 @@ aatc_status_t aatc_decode_attention_sw(aatc_plan_t p, int32_t layer, const void*
   ex.v_full = v_full;
   ex.n_full = n_full;
   ex.full_cap = full_cap;
-  return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, t_end, max_tokens, out, workspace, sp,
+  return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, t_end, max_tokens, out, workspace,
                                          static_cast<cudaStream_t>(stream), ex));
 }
 

@@ -2,8 +2,12 @@
 // uncompressed bf16 reference decode (Def. sdpa with one query row; Algorithm 1
 // "Reconstruct", "softmax", "Output" lines, computed without rebuilding the keys).
 //
-// Three launches per call (flash-decoding split over the context), each a programmatic
-// dependent of the one before it:
+// Two launch plans.  For layers whose key and value streams share one record shape (every
+// per-stream plan at 1.5, 2, 2.75 or 4 bits) one launch per call: aatc_decode_fused_kernel (see
+// there) rotates the queries, streams the split's tiles through per-warp-group rings, and the
+// CTA that finishes a (sequence, kv-head) last merges its splits.  Any other layer takes three
+// launches (flash-decoding split over the context), each a programmatic dependent of the one
+// before it:
 //   query    per (sequence, kv-head, query slot): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the
 //            G query heads of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1),
 //            and q' per record entry as f16 hi/lo tensor-core fragments (mma.sync m16n8k16);
@@ -18,6 +22,7 @@
 #include <cuda_fp16.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "aatc_internal.h"
@@ -88,6 +93,9 @@ struct DecodeArgs {
   const __nv_bfloat16* k_full;  // uncompressed tokens attended as well: [batch][full_cap][n_kv][128]
   const __nv_bfloat16* v_full;
   int n_full, full_cap;
+  unsigned long long* sem;  // fused kernel: completion flag per (sequence, kv-head, split)
+  unsigned long long epoch; // this launch's number (never 0)
+  int n_stages;             // fused kernel: tile ring depth
 };
 
 // 2^x with the hardware approximation (relative error ~2^-22; -inf -> 0)
@@ -245,8 +253,10 @@ __global__ void __launch_bounds__(kQThreads)
     float v[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) v[k] = f[k] < lim ? xe[base + f[k]] : 0.0f;
-    // the split kernel masks digits in place: lane t's D2 digits arrive times 4^t, its D1 bits
-    // times 2^t (k 2t, 2t+1) and 2^(t+4) (k 2t+8, 2t+9); the query rows carry the inverse
+    // the split kernels mask digits in place: lane t's D2 digits arrive times 4^t, its D1 bits
+    // times 2^t (k 2t, 2t+1) and 2^(t+4) (k 2t+8, 2t+9); the query rows carry the inverse.  (Only
+    // bits 0..9 of a half are mantissa: the upper byte of each half is shifted down first, since
+    // a digit in the exponent bits 10..15 would not be a multiple of the subnormal unit.)
     const float s01 = ks < n2w ? pow2i(-2 * t) : pow2i(-t);
     const float s89 = ks < n2w ? pow2i(-2 * t) : pow2i(-t - 4);
     v[0] *= s01;
@@ -689,6 +699,689 @@ __global__ void __launch_bounds__(kThreads)
         dst[D] = ml[q];
         dst[D + 1] = ml[MAX_GROUP + q];
       }
+    }
+  }
+}
+
+// ---------------------------------------------------------------- fused split + merge kernel
+// One launch per call, for plans whose key and value streams of the layer share one record shape
+// (N2W D2 words, N1W D1 words).  CTA = (split, kv-head, sequence) with WG warp groups of four
+// warps; the query rotation and the merge are folded in: every CTA rotates its group's queries
+// itself (while its first tiles are in flight), and the CTA that finds every split of its
+// (sequence, kv-head) done merges them.
+//  * Warp group wg takes tiles wg, wg + WG, ... of the split through its own ring of NS stages (a
+//    tile's keys, values and scales arrive together in one stage; the last of the group's four
+//    warps to finish a stage refills it).  Each warp owns a quarter (32 tokens) of a tile and runs
+//    its own online softmax, keys then values of the same tile, so warps never wait for each
+//    other inside the loop.
+//  * Reference maximum m per query, kept within 2^8 of the running maximum of e_t = s_t +
+//    floor(log2 alpha^V_t) (floored at s_t - 64), and raised (with the sums rescaled) only when a
+//    tile exceeds it by more than that: the value weight P' = 2^(s - m) alpha^V stays below 2^9
+//    and p = 2^(s - m) below 2^72 whatever the scales, so the split needs no pass over its alpha
+//    values first.  m is only a reference point: o = sum P' code and l = sum p share it, and the
+//    merge rescales both alike.
+//  * Completion flags: one 64-bit word per split in the workspace.  A CTA writes its partial,
+//    fences, sets its flag to the call's epoch (a per-launch number, never 0), fences, and reads
+//    all flags of its (sequence, kv-head): with both fences at least one CTA sees every flag set
+//    (two may, and then both write the same merged output).  Flags left from other calls hold
+//    other epochs, so the workspace needs no zeroing; a merging CTA clears the flags so that a
+//    replay of the same captured call (same epoch) starts clean.
+__host__ __device__ constexpr int fused_stage_bytes(int wu) { return 2 * wu * TILE * 4 + 2 * TILE * 4; }
+constexpr float kPScale = 32.0f;            // P' < 2^9 times 2^5: f16 operands below 2^14
+
+// The last CTA's merge region (float offsets into the drained rings): o_hat [gmax][128], split
+// weights and denominators [g][n_splits] each, 1 / l [8], U_V^T [128][128].
+struct FusedMerge {
+  int oh, wsp, lsp, rinv, uvt, floats;
+  __host__ __device__ FusedMerge(int gmax, int g, int n_splits) {
+    oh = 0;
+    wsp = gmax * D;
+    lsp = wsp + g * n_splits;
+    rinv = (lsp + g * n_splits + 3) & ~3;
+    uvt = (rinv + 8 + 31) & ~31;                  // U_V^T [128 c][128 d], bulk-copied (128-byte aligned)
+    floats = uvt + D * D;
+  }
+};
+
+struct FusedSmem {
+  int bars, cnt, qf, qc, pf, cetab, etab, ketab, fold, ring, total;
+  __host__ __device__ FusedSmem(int wu, int nks, int np, int wg, int n_entries, int n_stages, int n_splits) {
+    const int gmax = 4 * np, warps = 4 * wg;
+    int o = 0;
+    bars = o;  o = align16(o + 8 * wg * n_stages);
+    cnt = o;   o = align16(o + 4 * wg * n_stages);
+    qf = o;    o += nks * np * 32 * 8;                        // query B fragments [ks][p][lane]
+    qc = o;    o += 2 * MAX_GROUP * 4;                        // C_g, score scales
+    pf = o;    o += warps * 2 * np * 32 * 8;                  // P' B fragments [warp][ks][p][lane]
+    cetab = o; o += D * 8 * 2;                                // value channel -> record entries
+    etab = o;  o = align16(o + n_entries * 2);                // value entry table
+    ketab = o; o = align16(o + n_entries * 2);                // key entry table
+    fold = o;  o += ((2 + wg) * gmax * D + 2 * warps * gmax) * 4;   // q, q', partial q' [wg]; reductions
+    o = (o + 127) & ~127;
+    ring = o;
+    const int rings = wg * n_stages * fused_stage_bytes(wu);
+    // after the loop the rings hold each warp's (m, l, S', entry sums) per query, then the merge
+    const int epi = warps * (3 * MAX_GROUP + gmax * n_entries) * 4;
+    const int merge = 4 * FusedMerge(gmax, gmax, n_splits).floats;
+    int region = rings > epi ? rings : epi;
+    region = region > merge ? region : merge;
+    total = ring + region;
+  }
+};
+
+template <int N2W, int N1W, int NP, int WG>
+__global__ void __launch_bounds__(128 * WG, 1)
+    aatc_decode_fused_kernel(const DecodeArgs a) {
+  constexpr int WU = N2W + N1W;                  // record words the streams use
+  constexpr int NKS = N2W + 2 * N1W;             // score k16-steps
+  constexpr int NJ = N2W + 2 * N1W;              // value M-tiles (16 record entries each)
+  constexpr int GMAX = 4 * NP;
+  constexpr int NW = 4 * WG;                     // warps
+  constexpr int NT = 32 * NW;                    // threads
+  constexpr uint32_t kTileWords = WU * TILE;
+  constexpr uint32_t kStage = fused_stage_bytes(WU);
+  extern __shared__ __align__(128) unsigned char smb[];
+  __shared__ int s_abort, s_last, s_issued[WG];
+  __shared__ __align__(8) uint64_t s_uvbar;
+  int item = blockIdx.x;
+  if (a.cta_per_sm > 0) item = (item % a.num_sms) * a.cta_per_sm + item / a.num_sms;
+  const int split = item % a.n_splits, head = (item / a.n_splits) % a.n_kv, b = item / (a.n_splits * a.n_kv);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int wg = warp >> 2, wq = warp & 3;       // warp group, token quarter
+  const int g = lane >> 2, t = lane & 3;
+  const int G = a.group;
+  const int NS = a.n_stages;
+  const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;
+  const FusedSmem L(WU, NKS, NP, WG, a.n_entries, NS, a.n_splits);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smb + L.bars) + wg * NS;   // this group's ring barriers
+  int* cnt = reinterpret_cast<int*>(smb + L.cnt) + wg * NS;
+  const uint2* qf = reinterpret_cast<const uint2*>(smb + L.qf);
+  unsigned char* pfw = smb + L.pf + warp * (2 * NP * 32 * 8);
+  const short* cetab = reinterpret_cast<const short*>(smb + L.cetab);
+  const short* etab = reinterpret_cast<const short*>(smb + L.etab);
+  const short* ketab = reinterpret_cast<const short*>(smb + L.ketab);
+  unsigned char* ring = smb + L.ring + wg * NS * kStage;
+
+  const int tile_first = a.t_first / TILE;
+  const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE - tile_first;
+  const int tile_lo = tile_first + static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
+  const int tile_hi = tile_first + static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
+  const int t_lo = a.t_first, t_end = a.n_ctx;
+  const int n_tl = tile_hi - tile_lo;
+  const int n_j = n_tl > wg ? (n_tl - wg + WG - 1) / WG : 0;     // tiles of this warp group
+  const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
+  const size_t bk = (static_cast<size_t>(b) * a.n_kv + head) * 2;
+  const uint32_t* kwords = a.words + bk * stream_words;
+  const uint32_t* vwords = kwords + stream_words;
+  const float* kalpha = a.alpha + bk * a.n_tiles * TILE;
+  const float* valpha = kalpha + static_cast<size_t>(a.n_tiles) * TILE;
+
+  auto issue = [&](int j, int s) {             // the group's j-th tile into stage s = j mod NS
+    unsigned char* st = ring + s * kStage;
+    const int tile = tile_lo + wg + WG * j;
+    const size_t tw = static_cast<size_t>(tile) * a.n_words * TILE;
+    const size_t ta = static_cast<size_t>(tile) * TILE;
+    // the cache is read once per call: evict-first keeps the plan tables in L2
+    const uint64_t pol = ptx::l2_policy_evict_first();
+    ptx::mbar_arrive_expect_tx(full + s, kStage);
+    ptx::bulk_load_hint(st, kwords + tw, kTileWords * 4, full + s, pol);
+    ptx::bulk_load_hint(st + kTileWords * 4, vwords + tw, kTileWords * 4, full + s, pol);
+    ptx::bulk_load_hint(st + 2 * kTileWords * 4, kalpha + ta, TILE * 4, full + s, pol);
+    ptx::bulk_load_hint(st + 2 * kTileWords * 4 + TILE * 4, valpha + ta, TILE * 4, full + s, pol);
+    s_issued[wg] = j + 1;
+  };
+  const bool leader = (tid & 127) == 0;          // thread 0 of a warp group
+  if (leader) {
+    s_issued[wg] = 0;
+    for (int s = 0; s < NS; ++s) ptx::mbar_init(full + s, 1);
+    ptx::fence_mbar_init();
+  }
+  if (tid == 0) {
+    s_abort = 0;
+    s_last = 0;
+    ptx::mbar_init(&s_uvbar, 1);
+    ptx::fence_mbar_init();
+  }
+  // plan constants (never written by a kernel): the streams' entry tables, key channel constants
+  for (int i = tid; i < D * 8; i += NT)
+    reinterpret_cast<short*>(smb + L.cetab)[i] = a.chan_ent[static_cast<size_t>(sv) * D * 8 + i];
+  for (int i = tid; i < a.n_entries; i += NT) {
+    reinterpret_cast<short*>(smb + L.etab)[i] = a.entry[static_cast<size_t>(sv) * a.n_entries + i];
+    reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
+  }
+  const int c = tid & (D - 1), part = tid >> 7;                 // channel, part of the fold (WG parts)
+  const float fk = a.f[sk * D + c];
+  const float offk = a.enc[sk * D + c].off;                     // 2^(b_c - 1), 0 if b_c = 0
+  const StreamLayout lk = a.lay[sk];
+  if (tid < WG * NS) reinterpret_cast<int*>(smb + L.cnt)[tid] = 0;
+  // everything below may read what the preceding grid in the stream wrote (cache, q, workspace)
+  ptx::grid_dependency_wait();
+  if (leader && n_j > 0) issue(0, 0);          // first tile now, the rest of the ring after the fold
+
+  // ---- query rotation and fold, while the first tiles are in flight:
+  //   q'_{g,c} = (U_K^T q_g)_c f^K_c log2(e) / sqrt(128),  C_g = sum_c q'_{g,c} 2^(b_c - 1),
+  // and the score B fragments: q'_{g,c(e)} 2^shift(e) per record entry e, scaled so the largest
+  // is 2^14, as f16 hi / lo; column gs (hi) and gs + 4 (lo) of query group p for query 4p + gs
+  float* qv = reinterpret_cast<float*>(smb + L.fold);           // [GMAX][128] q
+  float* xq = qv + GMAX * D;                                    // [GMAX][128] q'
+  float* xpart = xq + GMAX * D;                                 // [WG][GMAX][128] partial U_K^T q
+  float* fred = xpart + WG * GMAX * D;                          // [2][NW][GMAX]
+  for (int i = tid; i < GMAX * D; i += NT) {
+    const int gq = i >> 7;
+    qv[i] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + (i & (D - 1))]) : 0.0f;
+  }
+  __syncthreads();
+  {
+    // part p of the thread sums dimensions [p D / WG, (p + 1) D / WG), RR rows of U_K in flight
+    constexpr int DR = D / WG, RR = DR < 64 ? DR : 64;
+    float acc[GMAX];
+#pragma unroll
+    for (int q = 0; q < GMAX; ++q) acc[q] = 0.0f;
+    const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(part * DR) * D + c;
+#pragma unroll 1
+    for (int r = 0; r < DR / RR; ++r) {
+      float u[RR];
+#pragma unroll
+      for (int k = 0; k < RR; ++k) u[k] = __ldg(uk + (RR * r + k) * D);
+#pragma unroll
+      for (int k4 = 0; k4 < RR / 4; ++k4)
+#pragma unroll
+        for (int q = 0; q < GMAX; ++q) {
+          const float4 qq = *reinterpret_cast<const float4*>(qv + q * D + part * DR + RR * r + 4 * k4);
+          acc[q] = fmaf(u[4 * k4], qq.x, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 1], qq.y, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 2], qq.z, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 3], qq.w, acc[q]);
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < GMAX; ++q) xpart[(part * GMAX + q) * D + c] = acc[q];
+  }
+  __syncthreads();
+  if (part == 0) {
+#pragma unroll
+    for (int q = 0; q < GMAX; ++q) {
+      float sum = 0.0f;
+#pragma unroll
+      for (int p2 = 0; p2 < WG; ++p2) sum += xpart[(p2 * GMAX + q) * D + c];
+      const float x = sum * fk * (kLog2e * 0.08838834764831845f);
+      xq[q * D + c] = x;
+      float cr = x * offk, mx = fabsf(x) * offk;                  // largest |coefficient| of c
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        cr += __shfl_xor_sync(0xffffffffu, cr, o);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      }
+      if (lane == 0) {
+        fred[warp * GMAX + q] = cr;
+        fred[(NW + warp) * GMAX + q] = mx;
+      }
+    }
+  }
+  __syncthreads();
+  {
+    float* qcw = reinterpret_cast<float*>(smb + L.qc);
+    float inv[GMAX];
+#pragma unroll
+    for (int q = 0; q < GMAX; ++q) {
+      float cs = 0.0f, m = 0.0f;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {                               // the four warps of part 0
+        cs += fred[w * GMAX + q];
+        m = fmaxf(m, fred[(NW + w) * GMAX + q]);
+      }
+      inv[q] = m > 0.0f ? kOpMax / m : 0.0f;
+      if (tid == q) {
+        qcw[q] = q < G ? cs : 0.0f;
+        qcw[MAX_GROUP + q] = q < G && m > 0.0f ? m * (kDigitScale / kOpMax) : 0.0f;   // raw sum -> sum q' u
+      }
+    }
+    // lane t of k-step ks holds fields (k 2t, 2t+1, 2t+8, 2t+9) = D2 (t, t+8, t+4, t+12) of word
+    // ks, or D1 bits (t, t+16, t+4, t+20) + 8 hs of word u for k-step ks = N2W + 2u + hs; the
+    // split loop masks them in place (times 4^t, or 2^t and 2^(t+4)), the fragments divide it out
+    uint2* qfw = reinterpret_cast<uint2*>(smb + L.qf);
+    for (int i = tid; i < NKS * 4 * GMAX; i += NT) {
+      const int q = i % GMAX, tt = (i / GMAX) & 3, ks = i / (4 * GMAX);
+      int f[4], base, lim;
+      float s01, s89;
+      if (ks < N2W) {
+        f[0] = tt; f[1] = tt + 8; f[2] = tt + 4; f[3] = tt + 12;
+        base = 16 * ks;
+        lim = 16;
+        s01 = s89 = pow2i(-2 * tt);
+      } else {
+        const int u = (ks - N2W) >> 1, sh = 8 * ((ks - N2W) & 1);
+        f[0] = tt + sh; f[1] = tt + sh + 16; f[2] = tt + 4 + sh; f[3] = tt + 4 + sh + 16;
+        base = lk.n2 + 32 * u;
+        lim = min(32, lk.n1 - 32 * u);
+        s01 = pow2i(-tt);
+        s89 = pow2i(-tt - 4);
+      }
+      float v[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int ce = f[k] < lim && q < G ? ketab[base + f[k]] : 0;
+        v[k] = f[k] < lim && q < G ? xq[q * D + (ce & 0xFF)] * inv[q] * pow2i(ce >> 8) * (k < 2 ? s01 : s89) : 0.0f;
+      }
+      uint32_t h01, l01, h89, l89;
+      f16_split2(v[0], v[1], h01, l01);
+      f16_split2(v[2], v[3], h89, l89);
+      const int p = q >> 2, gs = q & 3;
+      qfw[(ks * NP + p) * 32 + 4 * gs + tt] = make_uint2(h01, h89);
+      qfw[(ks * NP + p) * 32 + 4 * (gs + 4) + tt] = make_uint2(l01, l89);
+    }
+  }
+  const float* qc = reinterpret_cast<const float*>(smb + L.qc);
+  if (leader)
+    for (int j = 1; j < min(NS, n_j); ++j) issue(j, j);
+  ptx::grid_launch_dependents();
+  __syncthreads();
+
+  // masks: scores (lane t's fields of a k-step), values (lane row g's fields of an M-tile)
+  const uint32_t km2 = 0x00030003u << (2 * t);
+  const uint32_t km1a = 0x00010001u << t, km1b = 0x00010001u << (t + 4);
+  const uint32_t vm2 = 0x00030003u << (2 * (g & 3));
+  const uint32_t vm1 = 0x00010001u << g;
+  const int d2off = 2 * (g >> 2);
+  // lane (g, t) owns tokens tA = 32 wq + 4g + 2(t >> 1), tA + 1 of each tile and queries
+  // q_i = 4p + 2(t & 1) + i after the key-pass hi/lo exchange; the same queries are its value
+  // accumulator columns
+  const int tA = 32 * wq + 4 * g + 2 * (t >> 1);
+  float sg[NP][2], cg[NP][2], mrun[NP][2], lsum[NP][2], ssum[NP][2];
+#pragma unroll
+  for (int p = 0; p < NP; ++p)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int q = 4 * p + 2 * (t & 1) + i;
+      sg[p][i] = q < G ? qc[MAX_GROUP + q] : 0.0f;
+      cg[p][i] = q < G ? qc[q] : 0.0f;
+      mrun[p][i] = -INFINITY;
+      lsum[p][i] = 0.0f;
+      ssum[p][i] = 0.0f;
+    }
+  float vacc[NJ][NP][4];
+#pragma unroll
+  for (int j = 0; j < NJ; ++j)
+#pragma unroll
+    for (int p = 0; p < NP; ++p)
+#pragma unroll
+      for (int z = 0; z < 4; ++z) vacc[j][p][z] = 0.0f;
+
+  int s = 0;                                     // stage of tile j and the parity of its phase
+  uint32_t ph = 0;
+  for (int j = 0; j < n_j; ++j) {
+    if (!ptx::mbar_wait_sleep(full + s, ph, &s_abort, 20)) {
+      s_abort = 1;
+      atomicOr(a.err, 2);
+    }
+    if (s_abort) break;
+    const int ti = wg + WG * j;                  // tile of the split
+    const unsigned char* st = ring + s * kStage;
+    const uint32_t* kt = reinterpret_cast<const uint32_t*>(st);
+    const uint32_t* vt = kt + kTileWords;
+    const float* ak = reinterpret_cast<const float*>(vt + kTileWords);
+    const float* av = ak + TILE;
+    // ---- scores of the warp's 32 tokens: M-tile 0 rows (g, g + 8) = tokens 4g, 4g + 1, M-tile 1
+    // tokens 4g + 2, 4g + 3; N = 8 columns of query group p (hi 0..3, lo 4..7)
+    float kacc[2][NP][4];
+#pragma unroll
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+      for (int p = 0; p < NP; ++p)
+#pragma unroll
+        for (int z = 0; z < 4; ++z) kacc[m][p][z] = 0.0f;
+    const uint4* kp = reinterpret_cast<const uint4*>(kt + 32 * wq + 4 * g);
+#pragma unroll
+    for (int ks = 0; ks < N2W; ++ks) {
+      const uint4 x = kp[ks * (TILE / 4)];
+#pragma unroll
+      for (int p = 0; p < NP; ++p) {
+        const uint2 bf = qf[(ks * NP + p) * 32 + lane];
+        mma_f16(kacc[0][p], make_uint4(x.x & km2, x.y & km2, (x.x >> 8) & km2, (x.y >> 8) & km2), bf.x, bf.y);
+        mma_f16(kacc[1][p], make_uint4(x.z & km2, x.w & km2, (x.z >> 8) & km2, (x.w >> 8) & km2), bf.x, bf.y);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < N1W; ++u) {
+      const uint4 x = kp[(N2W + u) * (TILE / 4)];
+#pragma unroll
+      for (int hs = 0; hs < 2; ++hs) {
+        const uint4 y = hs ? make_uint4(x.x >> 8, x.y >> 8, x.z >> 8, x.w >> 8) : x;
+#pragma unroll
+        for (int p = 0; p < NP; ++p) {
+          const uint2 bf = qf[((N2W + 2 * u + hs) * NP + p) * 32 + lane];
+          mma_f16(kacc[0][p], make_uint4(y.x & km1a, y.y & km1a, y.x & km1b, y.y & km1b), bf.x, bf.y);
+          mma_f16(kacc[1][p], make_uint4(y.z & km1a, y.w & km1a, y.z & km1b, y.w & km1b), bf.x, bf.y);
+        }
+      }
+    }
+    // ---- scores, value exponents, running maximum
+    const float2 a2k = *reinterpret_cast<const float2*>(ak + tA);
+    const float2 a2v = *reinterpret_cast<const float2*>(av + tA);
+    const int tg = (tile_lo + ti) * TILE + tA;
+    const bool okA = tg >= t_lo && tg < t_end, okB = tg + 1 >= t_lo && tg + 1 < t_end;
+    // floor(log2 alpha^V) from the exponent field (>= -64; 0 and subnormals -> -64)
+    const float lgA = static_cast<float>(max(static_cast<int>((__float_as_uint(a2v.x) >> 23) & 0xFF) - 127, -64));
+    const float lgB = static_cast<float>(max(static_cast<int>((__float_as_uint(a2v.y) >> 23) & 0xFF) - 127, -64));
+    float sA[NP][2], sB[NP][2], eT[NP][2];
+    bool over = false;
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+      float r[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float mine = t < 2 ? kacc[0][p][i] : kacc[1][p][i];
+        const float give = t < 2 ? kacc[1][p][i] : kacc[0][p][i];
+        r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        sA[p][i] = okA ? a2k.x * fmaf(r[i], sg[p][i], -cg[p][i]) : -INFINITY;
+        sB[p][i] = okB ? a2k.y * fmaf(r[2 + i], sg[p][i], -cg[p][i]) : -INFINITY;
+        eT[p][i] = fmaxf(sA[p][i] + lgA, sB[p][i] + lgB);
+        over |= eT[p][i] > mrun[p][i] + 8.0f;
+      }
+    }
+    if (__any_sync(0xffffffffu, over)) {
+      // a token exceeds the reference by more than 2^8: raise it to the tile's maximum
+#pragma unroll
+      for (int p = 0; p < NP; ++p)
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          float e = eT[p][i];
+          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 2));
+          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 4));
+          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 8));
+          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 16));
+          const float mn = fmaxf(mrun[p][i], e);
+          if (mn > mrun[p][i]) {
+            const float mnew_ = mn;
+            const float f = fast_exp2(mrun[p][i] - mnew_);           // mrun = -inf -> 0
+            lsum[p][i] *= f;
+            ssum[p][i] *= f;
+#pragma unroll
+            for (int jj = 0; jj < NJ; ++jj) {
+              vacc[jj][p][i] *= f;
+              vacc[jj][p][2 + i] *= f;
+            }
+            mrun[p][i] = mnew_;
+          }
+        }
+    }
+    // ---- P' = 2^(s - m) alpha^V (times 2^5 into f16 range), as f16 hi / lo value B fragments:
+    // token quad g of the warp is value k-step g >> 2, fragment lane column t' = g & 3, and a
+    // column's registers are b0 = (token 0, token 2), b1 = (token 1, token 3).  Lanes t and t ^ 2
+    // hold tokens (0, 1) and (2, 3) of the quad: they swap lo (t < 2) against hi (t >= 2), and
+    // each writes whole registers (hi columns from t < 2, lo columns from t >= 2)
+#pragma unroll
+    for (int p = 0; p < NP; ++p)
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const float pA = okA ? fast_exp2(sA[p][i] - mrun[p][i]) : 0.0f;
+        const float pB = okB ? fast_exp2(sB[p][i] - mrun[p][i]) : 0.0f;
+        // masked tokens may hold any bits in alpha (beyond the context): select, never multiply
+        const float PA = okA ? pA * a2v.x * kPScale : 0.0f, PB = okB ? pB * a2v.y * kPScale : 0.0f;
+        lsum[p][i] += pA + pB;
+        ssum[p][i] += PA + PB;
+        const __half2 h2 = __floats2half2_rn(PA, PB);
+        const float2 hf = __half22float2(h2);
+        const __half2 l2 = __floats2half2_rn(PA - hf.x, PB - hf.y);
+        const uint32_t hw = *reinterpret_cast<const uint32_t*>(&h2), lw = *reinterpret_cast<const uint32_t*>(&l2);
+        const uint32_t mine = t < 2 ? hw : lw;
+        const uint32_t other = __shfl_xor_sync(0xffffffffu, t < 2 ? lw : hw, 2);   // partner's tokens
+        // low halves = the quad's tokens 0 / 1 (lane t < 2), high halves = tokens 2 / 3
+        const uint32_t w01 = t < 2 ? mine : other, w23 = t < 2 ? other : mine;
+        const uint2 reg = make_uint2(__byte_perm(w01, w23, 0x5410), __byte_perm(w01, w23, 0x7632));
+        const int col = 2 * (t & 1) + i + 4 * (t >> 1);
+        reinterpret_cast<uint2*>(pfw)[((g >> 2) * NP + p) * 32 + 4 * col + (g & 3)] = reg;
+      }
+    __syncwarp();
+    // ---- values: M-tile rows are record entries, K = the 16 tokens of k-step kv (quads
+    // 8 wq + 4 kv + t); lane t's K columns 2t, 2t + 1 are tokens 0, 2 of its quad (bytes 0, 2 of
+    // a slot word), 2t + 8, 2t + 9 tokens 1, 3 (bytes 1, 3, shifted down)
+#pragma unroll
+    for (int kv = 0; kv < 2; ++kv) {
+      uint2 bf[NP];
+#pragma unroll
+      for (int p = 0; p < NP; ++p) bf[p] = reinterpret_cast<const uint2*>(pfw)[(kv * NP + p) * 32 + lane];
+      const uint32_t* vq = vt + 4 * (8 * wq + 4 * kv + t);
+#pragma unroll
+      for (int jw = 0; jw < N2W; ++jw) {
+        const uint2 xx = *reinterpret_cast<const uint2*>(vq + jw * TILE + d2off);
+        const uint4 af = make_uint4(xx.x & vm2, xx.y & vm2, (xx.x >> 8) & vm2, (xx.y >> 8) & vm2);
+#pragma unroll
+        for (int p = 0; p < NP; ++p) mma_f16(vacc[jw][p], af, bf[p].x, bf[p].y);
+      }
+#pragma unroll
+      for (int u = 0; u < N1W; ++u) {
+        const uint4 s4 = *reinterpret_cast<const uint4*>(vq + (N2W + u) * TILE);
+        const uint4 afa = make_uint4(s4.x & vm1, s4.z & vm1, (s4.x >> 8) & vm1, (s4.z >> 8) & vm1);  // fields 0..15
+        const uint4 afb = make_uint4(s4.y & vm1, s4.w & vm1, (s4.y >> 8) & vm1, (s4.w >> 8) & vm1);  // 16..31
+#pragma unroll
+        for (int p = 0; p < NP; ++p) {
+          mma_f16(vacc[N2W + 2 * u][p], afa, bf[p].x, bf[p].y);
+          mma_f16(vacc[N2W + 2 * u + 1][p], afb, bf[p].x, bf[p].y);
+        }
+      }
+    }
+    __syncwarp();
+    // ---- release the stage; the last of the group's four warps refills it
+    if (lane == 0) {
+      __threadfence_block();
+      const int old = atomicAdd(cnt + s, 1);
+      if ((old & 3) == 3 && j + NS < n_j) {
+        __threadfence_block();
+        ptx::fence_proxy_async_smem();
+        issue(j + NS, s);
+      }
+    }
+    if (++s == NS) {
+      s = 0;
+      ph ^= 1;
+    }
+  }
+
+  __syncthreads();
+  if (s_abort) {
+    // a wait gave up: let every copy still in flight land (bounded) before leaving
+    if (leader)
+      for (int j = max(0, s_issued[wg] - NS); j < s_issued[wg]; ++j)
+        ptx::mbar_wait_sleep(full + j % NS, (j / NS) & 1, &s_last /* still 0 */, 20);
+    return;
+  }
+  // ---- per-warp (m, l, S') and entry sums into the drained rings
+  float* epi = reinterpret_cast<float*>(smb + L.ring);
+  const int NE = a.n_entries;
+  constexpr int kEpiStride = 3 * MAX_GROUP;                  // + GMAX * NE floats per warp
+  float* wm = epi + warp * (kEpiStride + GMAX * NE);         // [m, l, S'][MAX_GROUP], then E[GMAX][NE]
+  float* wE = wm + kEpiStride;
+#pragma unroll
+  for (int p = 0; p < NP; ++p)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+#pragma unroll
+      for (int o = 2; o < 32; o <<= 1) {
+        lsum[p][i] += __shfl_xor_sync(0xffffffffu, lsum[p][i], o);
+        ssum[p][i] += __shfl_xor_sync(0xffffffffu, ssum[p][i], o);
+      }
+      if (lane < 2) {
+        const int q = 4 * p + 2 * lane + i;
+        wm[q] = mrun[p][i];
+        wm[MAX_GROUP + q] = lsum[p][i];
+        wm[2 * MAX_GROUP + q] = ssum[p][i] * (1.0f / kPScale);
+      }
+    }
+  {
+    // after the hi / lo exchange lane (g, t) holds entry row g + 8 (t >> 1) of every M-tile for
+    // queries 4p + 2 (t & 1) + {0, 1}; raw sums times 2^24 / (row scale) / 2^5 = sum P' digit
+    const int row = g + 8 * (t >> 1);
+#pragma unroll
+    for (int jj = 0; jj < NJ; ++jj) {
+      int e;
+      float sc;
+      if (jj < N2W) {
+        e = 16 * jj + row;
+        sc = pow2i(19 - 2 * (g & 3));
+      } else {
+        const int u = (jj - N2W) >> 1, half = (jj - N2W) & 1;
+        e = 16 * N2W + 32 * u + 16 * half + row;
+        sc = pow2i(19 - g);
+      }
+#pragma unroll
+      for (int p = 0; p < NP; ++p) {
+        float r[2];
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const float mine = t < 2 ? vacc[jj][p][i] : vacc[jj][p][2 + i];
+          const float give = t < 2 ? vacc[jj][p][2 + i] : vacc[jj][p][i];
+          r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
+        }
+        if (e < NE)
+#pragma unroll
+          for (int i = 0; i < 2; ++i) wE[(4 * p + 2 * (t & 1) + i) * NE + e] = r[i] * sc;
+      }
+    }
+  }
+  __syncthreads();
+  // ---- the split's partial per query: thread = (value channel c, query parity part)
+  const size_t pbase = (static_cast<size_t>(b) * a.n_q + head * G) * a.n_splits;
+  {
+    const uint4 cev = *reinterpret_cast<const uint4*>(cetab + c * 8);
+    const short* ce = reinterpret_cast<const short*>(&cev);
+    float w8[8];
+    int e8[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      e8[k] = min(max(static_cast<int>(ce[k]), 0), NE - 1);
+      w8[k] = ce[k] >= 0 ? pow2i((etab[e8[k]] >> 8) & 15) : 0.0f;
+    }
+    const float off = a.enc[sv * D + c].off;
+    for (int q = part; q < G; q += WG) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, epi[w * (kEpiStride + GMAX * NE) + q]);
+      float o = 0.0f, l = 0.0f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float* ww = epi + w * (kEpiStride + GMAX * NE);
+        const float f = ww[q] > -INFINITY ? fast_exp2(ww[q] - M) : 0.0f;
+        float ow = -off * ww[2 * MAX_GROUP + q];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) ow = fmaf(w8[k], ww[kEpiStride + q * NE + e8[k]], ow);
+        o = fmaf(f, ow, o);
+        l = fmaf(f, ww[MAX_GROUP + q], l);
+      }
+      float* dst = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits + split) * a.pstride;
+      dst[c] = o;
+      if (c == 0) {
+        dst[D] = M;
+        dst[D + 1] = l;
+      }
+    }
+  }
+  // ---- the CTA that sees every split of this (sequence, kv-head) done merges: M = max_s m_s,
+  // w_s = 2^(m_s - M), o_hat_c = f^V_c sum_s w_s o_{s,c} / sum_s w_s l_s, out = U_V o_hat
+  __syncthreads();
+  unsigned long long* flags = a.sem + (static_cast<size_t>(b) * a.n_kv + head) * a.n_splits;
+  if (tid == 0) {
+    __threadfence();                      // cumulative over the CTA's partial writes (barrier above)
+    atomicExch(flags + split, a.epoch);
+    __threadfence();
+  }
+  __syncthreads();
+  int done = 1;
+  for (int i = tid; i < a.n_splits; i += NT)
+    done &= *reinterpret_cast<volatile unsigned long long*>(flags + i) == a.epoch;
+  s_last = __syncthreads_and(done);
+  if (!s_last) return;
+  __threadfence();
+  ptx::fence_proxy_async_smem();                     // the bulk copy below reuses the epilogue area
+  __syncthreads();
+  for (int i = tid; i < a.n_splits; i += NT) flags[i] = 0;      // a replay starts clean
+  const int NSP = a.n_splits;
+  const FusedMerge MG(GMAX, G, NSP);
+  float* uvt = epi + MG.uvt;
+  if (tid == 0) {                                    // U_V^T lands while the partials are read
+    ptx::mbar_arrive_expect_tx(&s_uvbar, D * D * 4);
+    ptx::bulk_load(uvt, a.u32t + static_cast<size_t>(sv) * D * D, D * D * 4, &s_uvbar);
+  }
+  float* oh = epi + MG.oh;                           // [GMAX][128] o_hat
+  float* wsp = epi + MG.wsp;                         // [G][NSP] split weights
+  float* lsp = epi + MG.lsp;                         // [G][NSP] split denominators
+  float* rinv = epi + MG.rinv;                       // [G] 1 / l
+  for (int i = tid; i < G * NSP; i += NT) {          // query i / NSP, split i % NSP: one round of loads
+    const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.ws + (pbase + static_cast<size_t>(i)) * a.pstride + D));
+    wsp[i] = ml.x;
+    lsp[i] = ml.y;
+  }
+  __syncthreads();
+  if (tid < G) {
+    float M = -INFINITY;
+    for (int s0 = 0; s0 < NSP; ++s0) M = fmaxf(M, wsp[tid * NSP + s0]);
+    float l = 0.0f;
+    for (int s0 = 0; s0 < NSP; ++s0) {
+      const float m = wsp[tid * NSP + s0];
+      const float w = m > -INFINITY ? fast_exp2(m - M) : 0.0f;
+      wsp[tid * NSP + s0] = w;
+      l = fmaf(w, lsp[tid * NSP + s0], l);
+    }
+    rinv[tid] = 1.0f / l;
+  }
+  __syncthreads();
+  {
+    // o_hat[q][c] = f^V_c sum_s w_s o_{s,c} / l: thread = (channel, part); its queries are
+    // part, part + WG, ...; eight splits of each in flight
+    constexpr int QPT = GMAX / WG;                     // queries per thread at most
+    const float fv = a.f[sv * D + c];
+    float o_acc[QPT];
+#pragma unroll
+    for (int qi = 0; qi < QPT; ++qi) o_acc[qi] = 0.0f;
+    for (int s0 = 0; s0 < NSP; s0 += 8) {
+      float v[QPT][8];
+#pragma unroll
+      for (int qi = 0; qi < QPT; ++qi) {
+        const int q = part + WG * qi;
+        const float* src = a.ws + (pbase + static_cast<size_t>(q) * NSP + s0) * a.pstride + c;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[qi][u] = q < G && s0 + u < NSP ? __ldcg(src + static_cast<size_t>(u) * a.pstride) : 0.0f;
+      }
+#pragma unroll
+      for (int qi = 0; qi < QPT; ++qi) {
+        const int q = part + WG * qi;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (q < G && s0 + u < NSP) o_acc[qi] = fmaf(wsp[q * NSP + s0 + u], v[qi][u], o_acc[qi]);
+      }
+    }
+#pragma unroll
+    for (int qi = 0; qi < QPT; ++qi) {
+      const int q = part + WG * qi;
+      if (q < G) oh[q * D + c] = o_acc[qi] * fv * rinv[q];
+    }
+  }
+  if (!ptx::mbar_wait_sleep(&s_uvbar, 0, &s_abort, 20)) atomicOr(a.err, 2);
+  __syncthreads();
+  {
+    // out[q][d] = sum_c U_V[d][c] o_hat[q][c] from shared memory: thread = (dimension d, part);
+    // its queries are part, part + WG, ...
+    constexpr int QPT = GMAX / WG;
+    const int d = c;
+    float acc[QPT];
+#pragma unroll
+    for (int qi = 0; qi < QPT; ++qi) acc[qi] = 0.0f;
+#pragma unroll 8
+    for (int cc = 0; cc < D; ++cc) {
+      const float u = uvt[cc * D + d];
+#pragma unroll
+      for (int qi = 0; qi < QPT; ++qi) {
+        const int q = part + WG * qi;
+        if (q < G) acc[qi] = fmaf(u, oh[q * D + cc], acc[qi]);
+      }
+    }
+#pragma unroll
+    for (int qi = 0; qi < QPT; ++qi) {
+      const int q = part + WG * qi;
+      if (q < G) a.out[(static_cast<size_t>(b) * a.n_q + head * G + q) * D + d] = acc[qi];
     }
   }
 }
@@ -1148,9 +1841,45 @@ cudaError_t launch_bf16_split(const Bf16Args& a, int batch, cudaStream_t st) {
 
 }  // namespace
 
+// Record shape shared by every key and value stream of `layer` (D2 words, D1 words), or false.
+static bool layer_shape(const Plan& plan, int layer, int* n2w, int* n1w) {
+  const int hk = plan.dims.n_kv_heads;
+  for (int s = 0; s < 2 * hk; ++s) {
+    const StreamLayout& l = plan.layout[layer * 2 * hk + s];
+    const int a = l.n2 / 16, b = (l.n1 + 31) / 32;
+    if (s == 0) {
+      *n2w = a;
+      *n1w = b;
+    } else if (a != *n2w || b != *n1w) {
+      return false;
+    }
+  }
+  return true;
+}
+
+using FusedKernel = void (*)(const DecodeArgs);
+
+// The record shapes the fused kernel is built for: (D2 words, D1 words) of the per-stream plans at
+// 1.5, 2, 2.75 and 4 bits per channel.
+// Warp groups per CTA (one CTA per SM): four for up to four query heads per kv-head (16 warps, at
+// most 128 registers), two for five to eight (twice the value accumulators).
+template <int NP>
+constexpr int fused_groups() { return NP == 1 ? 4 : 2; }
+
+template <int NP>
+static FusedKernel fused_kernel_for(int n2w, int n1w) {
+  constexpr int WG = fused_groups<NP>();
+  if (n2w == 9 && n1w == 2) return aatc_decode_fused_kernel<9, 2, NP, WG>;
+  if (n2w == 3 && n1w == 3) return aatc_decode_fused_kernel<3, 3, NP, WG>;
+  if (n2w == 5 && n1w == 3) return aatc_decode_fused_kernel<5, 3, NP, WG>;
+  if (n2w == 13 && n1w == 3) return aatc_decode_fused_kernel<13, 3, NP, WG>;
+  return nullptr;
+}
+
+static std::atomic<unsigned long long> g_decode_epoch{0};
+
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch, int n_ctx,
-                          int max_tokens, float* out, void* ws, const DecodeSplit& sp, cudaStream_t st,
-                          const DecodeExtra& extra) {
+                          int max_tokens, float* out, void* ws, cudaStream_t st, const DecodeExtra& extra) {
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
   DecodeArgs a;
   a.words = static_cast<const uint32_t*>(cache);
@@ -1174,17 +1903,49 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_tiles = g.n_tiles;
   a.n_words = plan.n_words;
   a.n_entries = plan.n_entries;
-  a.n_splits = extra.t_first < n_ctx ? sp.n_splits : 0;     // no packed range: merge kernel only
-  a.split_len = sp.split_len;
   a.t_first = extra.t_first;
   a.k_full = static_cast<const __nv_bfloat16*>(extra.k_full);
   a.v_full = static_cast<const __nv_bfloat16*>(extra.v_full);
   a.n_full = extra.n_full;
   a.full_cap = extra.full_cap;
+  const int np = (a.group + 3) / 4;
+  // the fused split + merge kernel: a packed range, no uncompressed tokens, one record shape
+  int n2w = 0, n1w = 0;
+  FusedKernel fk = nullptr;
+  if (extra.n_full == 0 && extra.t_first < n_ctx && layer_shape(plan, layer, &n2w, &n1w))
+    fk = np == 1 ? fused_kernel_for<1>(n2w, n1w) : fused_kernel_for<2>(n2w, n1w);
+  const int range = n_ctx - (extra.t_first / TILE) * TILE;
+  const DecodeSplit sp = decode_split_for(batch, a.n_kv, range, plan.num_sms, fk != nullptr);
+  a.n_splits = extra.t_first < n_ctx ? sp.n_splits : 0;     // no packed range: merge kernel only
+  a.split_len = sp.split_len;
   {
     const long n_cta = static_cast<long>(sp.n_splits) * a.n_kv * batch;
     a.num_sms = plan.num_sms;
     a.cta_per_sm = plan.num_sms > 0 && n_cta % plan.num_sms == 0 ? static_cast<int>(n_cta / plan.num_sms) : 0;
+  }
+  const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
+  a.pstride = wsl.pstride;
+  a.ks_stride = wsl.ks_stride;
+  a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
+  a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
+  a.sem = reinterpret_cast<unsigned long long*>(static_cast<char*>(ws) + wsl.sem_off);
+  if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
+  cudaError_t e = cudaSuccess;
+  if (fk) {
+    const int wu = n2w + n1w, nks = n2w + 2 * n1w;
+    a.epoch = g_decode_epoch.fetch_add(1, std::memory_order_relaxed) + 1;
+    const int wg = np == 1 ? fused_groups<1>() : fused_groups<2>();
+    // the deepest ring (up to 3 stages per warp group) that fits the shared memory of one SM
+    size_t smem = 0;
+    for (a.n_stages = 3; a.n_stages >= 2; --a.n_stages) {
+      smem = static_cast<size_t>(FusedSmem(wu, nks, np, wg, plan.n_entries, a.n_stages, a.n_splits).total);
+      if (smem <= 227 * 1024) break;
+    }
+    if (a.n_stages < 2) return cudaErrorNotSupported;
+    e = ensure_smem_optin(reinterpret_cast<const void*>(fk), smem);
+    if (e != cudaSuccess) return e;
+    const unsigned n_cta = static_cast<unsigned>(static_cast<long>(sp.n_splits) * a.n_kv * batch);
+    return launch_pdl(fk, dim3(n_cta), dim3(128 * wg), smem, st, a);
   }
   // largest key k-step count and value word count over the layer's streams
   int n_ks = 1, n_jobs_v = 1;
@@ -1194,14 +1955,6 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
     n_jobs_v = std::max(n_jobs_v, lv.n2 / 16 + 2 * ((lv.n1 + 31) / 32));
   }
-  const int np = (a.group + 3) / 4;
-  const DecodeWs wsl = decode_ws_layout(batch, a.n_q, a.n_kv, plan.n_entries, plan.n_words, sp);
-  a.pstride = wsl.pstride;
-  a.ks_stride = wsl.ks_stride;
-  a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
-  a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
-  if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
-  cudaError_t e = cudaSuccess;
   if (a.n_splits > 0) {
     e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, MAX_GROUP), dim3(kQThreads), 0, st, a);
     if (e != cudaSuccess) return e;
@@ -1287,10 +2040,7 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
   if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(cache) & 15u) != 0) return AATC_ERR_INVALID_ARG;
-  const DecodeSplit sp = decode_split(batch, plan->dims.n_kv_heads, n_ctx, plan->num_sms);
-  if (decode_workspace(batch, plan->dims.n_q_heads, plan->dims.n_kv_heads, plan->n_entries, plan->n_words, sp) >
-      AATC_NOALLOC_SCRATCH_BYTES)
-    return AATC_ERR_WORKSPACE;
+  if (decode_workspace_for(*plan, batch, n_ctx) > AATC_NOALLOC_SCRATCH_BYTES) return AATC_ERR_WORKSPACE;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return status_from_cuda(e);
@@ -1308,6 +2058,6 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
     }
     scratch = g_noalloc_address[dev];
   }
-  return status_from_cuda(launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out, scratch, sp,
+  return status_from_cuda(launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out, scratch,
                                         static_cast<cudaStream_t>(stream), DecodeExtra{}));
 }
