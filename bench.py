@@ -35,8 +35,8 @@ sys.path.insert(0, ROOT)
 import workloads as W  # noqa: E402
 
 METRIC = "compressed-KV decode attn GB/s & % of HBM peak; encode Mtok/s (1 GB300)"
-DECODE_KERNELS = "aatc_decode_fused_kernel"        # one launch per decode call (per-stream plans)
-DECODE_LAUNCHES_PER_CALL = 1
+DECODE_KERNELS = "aatc_decode_fused_kernel + aatc_decode_merge_kernel"
+DECODE_LAUNCHES_PER_CALL = 2
 N_COPIES = 16
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")

@@ -122,14 +122,14 @@ size_t bf16_split_smem(int gp, int split_len);
 struct DecodeWs {
   int pstride;            // floats per partial
   int ks_stride;          // uint4 per (sequence, kv-head) fragment block
-  size_t qfrag_off, qcorr_off, sem_off, bytes;   // sem: a 64-bit completion flag per (sequence, kv-head, split)
+  size_t qfrag_off, qcorr_off, bytes;
 };
 DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
 size_t decode_workspace(int batch, int n_q, int n_kv, int n_entries, int n_words, const DecodeSplit& sp);
-// The decode has two launch plans: the fused split + merge kernel (CTAs of 8-16 warps, about
-// FUSED_CTAS_PER_SM per SM) for layers whose streams share one of the record shapes it is built
-// for, and the split + merge kernels (about 5 CTAs per SM, at most 16 tiles per split) for any
-// other layer.  `range` = the packed tokens a call covers, counted from the first tile it reads.
+// The decode has two launch plans: the fused kernel (query rotation and split streaming in CTAs of
+// 8-16 warps, FUSED_CTAS_PER_SM per SM, one wave) then the merge kernel, for layers whose streams
+// share one of the record shapes it is built for; the query, split and merge kernels (about 5 CTAs
+// per SM, at most 16 tiles per split) for any other layer.  `range` = the packed tokens a call covers, counted from the first tile it reads.
 constexpr int FUSED_CTAS_PER_SM = 1;
 DecodeSplit decode_split_for(int batch, int n_kv, int range, int num_sms, bool fused);
 // Workspace bytes that serve a decode of `range` tokens on any layer of the plan, whichever path

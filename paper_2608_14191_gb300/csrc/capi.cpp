@@ -95,8 +95,7 @@ DecodeWs decode_ws_layout(int batch, int n_q, int n_kv, int n_entries, int n_wor
   w.ks_stride = 2 * n_words * 32;                 // >= score k16-steps (<= 2 W) x 32 lanes
   w.qfrag_off = align_up(static_cast<size_t>(batch) * n_q * sp.n_splits * w.pstride * sizeof(float), 256);
   w.qcorr_off = align_up(w.qfrag_off + static_cast<size_t>(batch) * n_kv * w.ks_stride * 16, 256);
-  w.sem_off = align_up(w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float), 256);
-  w.bytes = w.sem_off + static_cast<size_t>(batch) * n_kv * sp.n_splits * sizeof(unsigned long long);
+  w.bytes = w.qcorr_off + static_cast<size_t>(batch) * n_kv * 2 * MAX_GROUP * sizeof(float);
   return w;
 }
 

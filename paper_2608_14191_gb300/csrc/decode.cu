@@ -2,12 +2,11 @@
 // uncompressed bf16 reference decode (Def. sdpa with one query row; Algorithm 1
 // "Reconstruct", "softmax", "Output" lines, computed without rebuilding the keys).
 //
-// Two launch plans.  For layers whose key and value streams share one record shape (every
-// per-stream plan at 1.5, 2, 2.75 or 4 bits) one launch per call: aatc_decode_fused_kernel (see
-// there) rotates the queries, streams the split's tiles through per-warp-group rings, and the
-// CTA that finishes a (sequence, kv-head) last merges its splits.  Any other layer takes three
-// launches (flash-decoding split over the context), each a programmatic dependent of the one
-// before it:
+// Two launch plans, each a chain of programmatic dependents.  For layers whose key and value
+// streams share one record shape (every per-stream plan at 1.5, 2, 2.75 or 4 bits) two launches
+// per call: aatc_decode_fused_kernel (see there) rotates the queries and streams each split's
+// tiles through per-warp-group rings, then the merge kernel below.  Any other layer takes three
+// launches (flash-decoding split over the context):
 //   query    per (sequence, kv-head, query slot): q' = (U_K^T q) f^K log2(e)/sqrt(128) for the
 //            G query heads of the GQA group, the offset corrections C_g = sum_c q'_c 2^(b_c-1),
 //            and q' per record entry as f16 hi/lo tensor-core fragments (mma.sync m16n8k16);
@@ -22,7 +21,6 @@
 #include <cuda_fp16.h>
 
 #include <algorithm>
-#include <atomic>
 #include <mutex>
 
 #include "aatc_internal.h"
@@ -93,8 +91,6 @@ struct DecodeArgs {
   const __nv_bfloat16* k_full;  // uncompressed tokens attended as well: [batch][full_cap][n_kv][128]
   const __nv_bfloat16* v_full;
   int n_full, full_cap;
-  unsigned long long* sem;  // fused kernel: completion flag per (sequence, kv-head, split)
-  unsigned long long epoch; // this launch's number (never 0)
   int n_stages;             // fused kernel: tile ring depth
 };
 
@@ -704,11 +700,13 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // ---------------------------------------------------------------- fused split + merge kernel
-// One launch per call, for plans whose key and value streams of the layer share one record shape
-// (N2W D2 words, N1W D1 words).  CTA = (split, kv-head, sequence) with WG warp groups of four
-// warps; the query rotation and the merge are folded in: every CTA rotates its group's queries
-// itself (while its first tiles are in flight), and the CTA that finds every split of its
-// (sequence, kv-head) done merges them.
+// For plans whose key and value streams of the layer share one record shape (N2W D2 words, N1W D1
+// words).  CTA = (split, kv-head, sequence) with WG warp groups of four warps, one CTA per SM in
+// one wave; the query rotation is folded in (every CTA rotates its group's queries itself, while
+// its first tiles are in flight) and the split's partial (o, m, l) per query goes to the
+// workspace for the merge kernel, which follows as this grid's programmatic dependent.  (A merge
+// by the last CTA of each (sequence, kv-head), behind completion flags, measured slower: its
+// fences, flag round and serial partial reads cost more than the grid boundary.)
 //  * Warp group wg takes tiles wg, wg + WG, ... of the split through its own ring of NS stages (a
 //    tile's keys, values and scales arrive together in one stage; the last of the group's four
 //    warps to finish a stage refills it).  Each warp owns a quarter (32 tokens) of a tile and runs
@@ -720,32 +718,12 @@ __global__ void __launch_bounds__(kThreads)
 //    and p = 2^(s - m) below 2^72 whatever the scales, so the split needs no pass over its alpha
 //    values first.  m is only a reference point: o = sum P' code and l = sum p share it, and the
 //    merge rescales both alike.
-//  * Completion flags: one 64-bit word per split in the workspace.  A CTA writes its partial,
-//    fences, sets its flag to the call's epoch (a per-launch number, never 0), fences, and reads
-//    all flags of its (sequence, kv-head): with both fences at least one CTA sees every flag set
-//    (two may, and then both write the same merged output).  Flags left from other calls hold
-//    other epochs, so the workspace needs no zeroing; a merging CTA clears the flags so that a
-//    replay of the same captured call (same epoch) starts clean.
 __host__ __device__ constexpr int fused_stage_bytes(int wu) { return 2 * wu * TILE * 4 + 2 * TILE * 4; }
 constexpr float kPScale = 32.0f;            // P' < 2^9 times 2^5: f16 operands below 2^14
 
-// The last CTA's merge region (float offsets into the drained rings): o_hat [gmax][128], split
-// weights and denominators [g][n_splits] each, 1 / l [8], U_V^T [128][128].
-struct FusedMerge {
-  int oh, wsp, lsp, rinv, uvt, floats;
-  __host__ __device__ FusedMerge(int gmax, int g, int n_splits) {
-    oh = 0;
-    wsp = gmax * D;
-    lsp = wsp + g * n_splits;
-    rinv = (lsp + g * n_splits + 3) & ~3;
-    uvt = (rinv + 8 + 31) & ~31;                  // U_V^T [128 c][128 d], bulk-copied (128-byte aligned)
-    floats = uvt + D * D;
-  }
-};
-
 struct FusedSmem {
   int bars, cnt, qf, qc, pf, cetab, etab, ketab, fold, ring, total;
-  __host__ __device__ FusedSmem(int wu, int nks, int np, int wg, int n_entries, int n_stages, int n_splits) {
+  __host__ __device__ FusedSmem(int wu, int nks, int np, int wg, int n_entries, int n_stages) {
     const int gmax = 4 * np, warps = 4 * wg;
     int o = 0;
     bars = o;  o = align16(o + 8 * wg * n_stages);
@@ -760,12 +738,9 @@ struct FusedSmem {
     o = (o + 127) & ~127;
     ring = o;
     const int rings = wg * n_stages * fused_stage_bytes(wu);
-    // after the loop the rings hold each warp's (m, l, S', entry sums) per query, then the merge
+    // after the loop the rings hold each warp's (m, l, S', entry sums) per query
     const int epi = warps * (3 * MAX_GROUP + gmax * n_entries) * 4;
-    const int merge = 4 * FusedMerge(gmax, gmax, n_splits).floats;
-    int region = rings > epi ? rings : epi;
-    region = region > merge ? region : merge;
-    total = ring + region;
+    total = ring + (rings > epi ? rings : epi);
   }
 };
 
@@ -781,8 +756,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   constexpr uint32_t kTileWords = WU * TILE;
   constexpr uint32_t kStage = fused_stage_bytes(WU);
   extern __shared__ __align__(128) unsigned char smb[];
-  __shared__ int s_abort, s_last, s_issued[WG];
-  __shared__ __align__(8) uint64_t s_uvbar;
+  __shared__ int s_abort, s_never, s_issued[WG];
   int item = blockIdx.x;
   if (a.cta_per_sm > 0) item = (item % a.num_sms) * a.cta_per_sm + item / a.num_sms;
   const int split = item % a.n_splits, head = (item / a.n_splits) % a.n_kv, b = item / (a.n_splits * a.n_kv);
@@ -792,7 +766,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   const int G = a.group;
   const int NS = a.n_stages;
   const int sk = (a.layer * a.n_kv + head) * 2, sv = sk + 1;
-  const FusedSmem L(WU, NKS, NP, WG, a.n_entries, NS, a.n_splits);
+  const FusedSmem L(WU, NKS, NP, WG, a.n_entries, NS);
   uint64_t* full = reinterpret_cast<uint64_t*>(smb + L.bars) + wg * NS;   // this group's ring barriers
   int* cnt = reinterpret_cast<int*>(smb + L.cnt) + wg * NS;
   const uint2* qf = reinterpret_cast<const uint2*>(smb + L.qf);
@@ -838,9 +812,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   }
   if (tid == 0) {
     s_abort = 0;
-    s_last = 0;
-    ptx::mbar_init(&s_uvbar, 1);
-    ptx::fence_mbar_init();
+    s_never = 0;
   }
   // plan constants (never written by a kernel): the streams' entry tables, key channel constants
   for (int i = tid; i < D * 8; i += NT)
@@ -850,6 +822,12 @@ __global__ void __launch_bounds__(128 * WG, 1)
     reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
   }
   const int c = tid & (D - 1), part = tid >> 7;                 // channel, part of the fold (WG parts)
+  // U_K rows of this thread's part of the fold: plan constants, requested before the wait
+  constexpr int DR = D / WG, RR = DR < 64 ? DR : 64;
+  const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(part * DR) * D + c;
+  float u0[RR];
+#pragma unroll
+  for (int k = 0; k < RR; ++k) u0[k] = __ldg(uk + k * D);
   const float fk = a.f[sk * D + c];
   const float offk = a.enc[sk * D + c].off;                     // 2^(b_c - 1), 0 if b_c = 0
   const StreamLayout lk = a.lay[sk];
@@ -861,7 +839,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   // ---- query rotation and fold, while the first tiles are in flight:
   //   q'_{g,c} = (U_K^T q_g)_c f^K_c log2(e) / sqrt(128),  C_g = sum_c q'_{g,c} 2^(b_c - 1),
   // and the score B fragments: q'_{g,c(e)} 2^shift(e) per record entry e, scaled so the largest
-  // is 2^14, as f16 hi / lo; column gs (hi) and gs + 4 (lo) of query group p for query 4p + gs
+  // is 2^14, as f16 hi / lo; columns 2 gs (hi) and 2 gs + 1 (lo) of query group p for query 4p + gs
   float* qv = reinterpret_cast<float*>(smb + L.fold);           // [GMAX][128] q
   float* xq = qv + GMAX * D;                                    // [GMAX][128] q'
   float* xpart = xq + GMAX * D;                                 // [WG][GMAX][128] partial U_K^T q
@@ -873,16 +851,14 @@ __global__ void __launch_bounds__(128 * WG, 1)
   __syncthreads();
   {
     // part p of the thread sums dimensions [p D / WG, (p + 1) D / WG), RR rows of U_K in flight
-    constexpr int DR = D / WG, RR = DR < 64 ? DR : 64;
     float acc[GMAX];
 #pragma unroll
     for (int q = 0; q < GMAX; ++q) acc[q] = 0.0f;
-    const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(part * DR) * D + c;
 #pragma unroll 1
     for (int r = 0; r < DR / RR; ++r) {
       float u[RR];
 #pragma unroll
-      for (int k = 0; k < RR; ++k) u[k] = __ldg(uk + (RR * r + k) * D);
+      for (int k = 0; k < RR; ++k) u[k] = r == 0 ? u0[k] : __ldg(uk + (RR * r + k) * D);
 #pragma unroll
       for (int k4 = 0; k4 < RR / 4; ++k4)
 #pragma unroll
@@ -967,8 +943,8 @@ __global__ void __launch_bounds__(128 * WG, 1)
       f16_split2(v[0], v[1], h01, l01);
       f16_split2(v[2], v[3], h89, l89);
       const int p = q >> 2, gs = q & 3;
-      qfw[(ks * NP + p) * 32 + 4 * gs + tt] = make_uint2(h01, h89);
-      qfw[(ks * NP + p) * 32 + 4 * (gs + 4) + tt] = make_uint2(l01, l89);
+      qfw[(ks * NP + p) * 32 + 4 * (2 * gs) + tt] = make_uint2(h01, h89);        // column 2 gs: hi
+      qfw[(ks * NP + p) * 32 + 4 * (2 * gs + 1) + tt] = make_uint2(l01, l89);    // column 2 gs + 1: lo
     }
   }
   const float* qc = reinterpret_cast<const float*>(smb + L.qc);
@@ -983,22 +959,21 @@ __global__ void __launch_bounds__(128 * WG, 1)
   const uint32_t vm2 = 0x00030003u << (2 * (g & 3));
   const uint32_t vm1 = 0x00010001u << g;
   const int d2off = 2 * (g >> 2);
-  // lane (g, t) owns tokens tA = 32 wq + 4g + 2(t >> 1), tA + 1 of each tile and queries
-  // q_i = 4p + 2(t & 1) + i after the key-pass hi/lo exchange; the same queries are its value
-  // accumulator columns
-  const int tA = 32 * wq + 4 * g + 2 * (t >> 1);
-  float sg[NP][2], cg[NP][2], mrun[NP][2], lsum[NP][2], ssum[NP][2];
+  // With the hi and lo columns of a query side by side, lane (g, t)'s accumulators c0 + c1 and
+  // c2 + c3 are whole sums for query 4p + t: in the key pass of tokens 4g + {0, 1} (M-tile 0) and
+  // 4g + {2, 3} (M-tile 1), i.e. the lane owns query 4p + t over the token quad g of its warp; in
+  // the value pass of record-entry rows g and g + 8
+  const int tq = 32 * wq + 4 * g;                // first token of the lane's quad in a tile
+  float sg[NP], cg[NP], mrun[NP], lsum[NP], ssum[NP];
 #pragma unroll
-  for (int p = 0; p < NP; ++p)
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int q = 4 * p + 2 * (t & 1) + i;
-      sg[p][i] = q < G ? qc[MAX_GROUP + q] : 0.0f;
-      cg[p][i] = q < G ? qc[q] : 0.0f;
-      mrun[p][i] = -INFINITY;
-      lsum[p][i] = 0.0f;
-      ssum[p][i] = 0.0f;
-    }
+  for (int p = 0; p < NP; ++p) {
+    const int q = 4 * p + t;
+    sg[p] = q < G ? qc[MAX_GROUP + q] : 0.0f;
+    cg[p] = q < G ? qc[q] : 0.0f;
+    mrun[p] = -INFINITY;
+    lsum[p] = 0.0f;
+    ssum[p] = 0.0f;
+  }
   float vacc[NJ][NP][4];
 #pragma unroll
   for (int j = 0; j < NJ; ++j)
@@ -1022,7 +997,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
     const float* ak = reinterpret_cast<const float*>(vt + kTileWords);
     const float* av = ak + TILE;
     // ---- scores of the warp's 32 tokens: M-tile 0 rows (g, g + 8) = tokens 4g, 4g + 1, M-tile 1
-    // tokens 4g + 2, 4g + 3; N = 8 columns of query group p (hi 0..3, lo 4..7)
+    // tokens 4g + 2, 4g + 3; N = 8 columns of query group p (hi, lo of queries 4p .. 4p + 3)
     float kacc[2][NP][4];
 #pragma unroll
     for (int m = 0; m < 2; ++m)
@@ -1030,7 +1005,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
       for (int p = 0; p < NP; ++p)
 #pragma unroll
         for (int z = 0; z < 4; ++z) kacc[m][p][z] = 0.0f;
-    const uint4* kp = reinterpret_cast<const uint4*>(kt + 32 * wq + 4 * g);
+    const uint4* kp = reinterpret_cast<const uint4*>(kt + tq);
 #pragma unroll
     for (int ks = 0; ks < N2W; ++ks) {
       const uint4 x = kp[ks * (TILE / 4)];
@@ -1055,86 +1030,74 @@ __global__ void __launch_bounds__(128 * WG, 1)
         }
       }
     }
-    // ---- scores, value exponents, running maximum
-    const float2 a2k = *reinterpret_cast<const float2*>(ak + tA);
-    const float2 a2v = *reinterpret_cast<const float2*>(av + tA);
-    const int tg = (tile_lo + ti) * TILE + tA;
-    const bool okA = tg >= t_lo && tg < t_end, okB = tg + 1 >= t_lo && tg + 1 < t_end;
-    // floor(log2 alpha^V) from the exponent field (>= -64; 0 and subnormals -> -64)
-    const float lgA = static_cast<float>(max(static_cast<int>((__float_as_uint(a2v.x) >> 23) & 0xFF) - 127, -64));
-    const float lgB = static_cast<float>(max(static_cast<int>((__float_as_uint(a2v.y) >> 23) & 0xFF) - 127, -64));
-    float sA[NP][2], sB[NP][2], eT[NP][2];
+    // ---- scores, value exponents, reference maximum
+    const float4 a4k = *reinterpret_cast<const float4*>(ak + tq);
+    const float4 a4v = *reinterpret_cast<const float4*>(av + tq);
+    const float akv[4] = {a4k.x, a4k.y, a4k.z, a4k.w};
+    const float avv[4] = {a4v.x, a4v.y, a4v.z, a4v.w};
+    const int tg = (tile_lo + ti) * TILE + tq;
+    bool ok[4];
+    float lg[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      ok[k] = tg + k >= t_lo && tg + k < t_end;
+      // floor(log2 alpha^V) from the exponent field (>= -64; 0 and subnormals -> -64)
+      lg[k] = static_cast<float>(max(static_cast<int>((__float_as_uint(avv[k]) >> 23) & 0xFF) - 127, -64));
+    }
+    float sc4[NP][4];
     bool over = false;
 #pragma unroll
     for (int p = 0; p < NP; ++p) {
-      float r[4];
+      const float r[4] = {kacc[0][p][0] + kacc[0][p][1], kacc[0][p][2] + kacc[0][p][3],
+                          kacc[1][p][0] + kacc[1][p][1], kacc[1][p][2] + kacc[1][p][3]};
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float mine = t < 2 ? kacc[0][p][i] : kacc[1][p][i];
-        const float give = t < 2 ? kacc[1][p][i] : kacc[0][p][i];
-        r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
-      }
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        sA[p][i] = okA ? a2k.x * fmaf(r[i], sg[p][i], -cg[p][i]) : -INFINITY;
-        sB[p][i] = okB ? a2k.y * fmaf(r[2 + i], sg[p][i], -cg[p][i]) : -INFINITY;
-        eT[p][i] = fmaxf(sA[p][i] + lgA, sB[p][i] + lgB);
-        over |= eT[p][i] > mrun[p][i] + 8.0f;
+      for (int k = 0; k < 4; ++k) {
+        sc4[p][k] = ok[k] ? akv[k] * fmaf(r[k], sg[p], -cg[p]) : -INFINITY;
+        over |= sc4[p][k] + lg[k] > mrun[p] + 8.0f;
       }
     }
     if (__any_sync(0xffffffffu, over)) {
       // a token exceeds the reference by more than 2^8: raise it to the tile's maximum
 #pragma unroll
-      for (int p = 0; p < NP; ++p)
+      for (int p = 0; p < NP; ++p) {
+        float e = fmaxf(fmaxf(sc4[p][0] + lg[0], sc4[p][1] + lg[1]), fmaxf(sc4[p][2] + lg[2], sc4[p][3] + lg[3]));
+        e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 4));
+        e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 8));
+        e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 16));
+        if (e > mrun[p]) {
+          const float f = fast_exp2(mrun[p] - e);                  // mrun = -inf -> 0
+          lsum[p] *= f;
+          ssum[p] *= f;
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          float e = eT[p][i];
-          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 2));
-          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 4));
-          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 8));
-          e = fmaxf(e, __shfl_xor_sync(0xffffffffu, e, 16));
-          const float mn = fmaxf(mrun[p][i], e);
-          if (mn > mrun[p][i]) {
-            const float mnew_ = mn;
-            const float f = fast_exp2(mrun[p][i] - mnew_);           // mrun = -inf -> 0
-            lsum[p][i] *= f;
-            ssum[p][i] *= f;
+          for (int jj = 0; jj < NJ; ++jj)
 #pragma unroll
-            for (int jj = 0; jj < NJ; ++jj) {
-              vacc[jj][p][i] *= f;
-              vacc[jj][p][2 + i] *= f;
-            }
-            mrun[p][i] = mnew_;
-          }
+            for (int z = 0; z < 4; ++z) vacc[jj][p][z] *= f;
+          mrun[p] = e;
         }
-    }
-    // ---- P' = 2^(s - m) alpha^V (times 2^5 into f16 range), as f16 hi / lo value B fragments:
-    // token quad g of the warp is value k-step g >> 2, fragment lane column t' = g & 3, and a
-    // column's registers are b0 = (token 0, token 2), b1 = (token 1, token 3).  Lanes t and t ^ 2
-    // hold tokens (0, 1) and (2, 3) of the quad: they swap lo (t < 2) against hi (t >= 2), and
-    // each writes whole registers (hi columns from t < 2, lo columns from t >= 2)
-#pragma unroll
-    for (int p = 0; p < NP; ++p)
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const float pA = okA ? fast_exp2(sA[p][i] - mrun[p][i]) : 0.0f;
-        const float pB = okB ? fast_exp2(sB[p][i] - mrun[p][i]) : 0.0f;
-        // masked tokens may hold any bits in alpha (beyond the context): select, never multiply
-        const float PA = okA ? pA * a2v.x * kPScale : 0.0f, PB = okB ? pB * a2v.y * kPScale : 0.0f;
-        lsum[p][i] += pA + pB;
-        ssum[p][i] += PA + PB;
-        const __half2 h2 = __floats2half2_rn(PA, PB);
-        const float2 hf = __half22float2(h2);
-        const __half2 l2 = __floats2half2_rn(PA - hf.x, PB - hf.y);
-        const uint32_t hw = *reinterpret_cast<const uint32_t*>(&h2), lw = *reinterpret_cast<const uint32_t*>(&l2);
-        const uint32_t mine = t < 2 ? hw : lw;
-        const uint32_t other = __shfl_xor_sync(0xffffffffu, t < 2 ? lw : hw, 2);   // partner's tokens
-        // low halves = the quad's tokens 0 / 1 (lane t < 2), high halves = tokens 2 / 3
-        const uint32_t w01 = t < 2 ? mine : other, w23 = t < 2 ? other : mine;
-        const uint2 reg = make_uint2(__byte_perm(w01, w23, 0x5410), __byte_perm(w01, w23, 0x7632));
-        const int col = 2 * (t & 1) + i + 4 * (t >> 1);
-        reinterpret_cast<uint2*>(pfw)[((g >> 2) * NP + p) * 32 + 4 * col + (g & 3)] = reg;
       }
+    }
+    // ---- P' = 2^(s - m) alpha^V (times 2^5 into f16 range) as f16 hi / lo value B fragments:
+    // token quad g of the warp is value k-step g >> 2, fragment lane column t' = g & 3, with
+    // registers b0 = (token 0, token 2), b1 = (token 1, token 3) in columns 2t (hi) and 2t + 1 (lo)
+#pragma unroll
+    for (int p = 0; p < NP; ++p) {
+      float pv[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float pk = ok[k] ? fast_exp2(sc4[p][k] - mrun[p]) : 0.0f;
+        // masked tokens may hold any bits in alpha (beyond the context): select, never multiply
+        pv[k] = ok[k] ? pk * avv[k] * kPScale : 0.0f;
+        lsum[p] += pk;
+      }
+      ssum[p] += (pv[0] + pv[1]) + (pv[2] + pv[3]);
+      const __half2 h02 = __floats2half2_rn(pv[0], pv[2]), h13 = __floats2half2_rn(pv[1], pv[3]);
+      const float2 f02 = __half22float2(h02), f13 = __half22float2(h13);
+      const __half2 l02 = __floats2half2_rn(pv[0] - f02.x, pv[2] - f02.y);
+      const __half2 l13 = __floats2half2_rn(pv[1] - f13.x, pv[3] - f13.y);
+      uint2* dst = reinterpret_cast<uint2*>(pfw) + ((g >> 2) * NP + p) * 32 + (g & 3);
+      dst[4 * (2 * t)] = make_uint2(*reinterpret_cast<const uint32_t*>(&h02), *reinterpret_cast<const uint32_t*>(&h13));
+      dst[4 * (2 * t + 1)] = make_uint2(*reinterpret_cast<const uint32_t*>(&l02), *reinterpret_cast<const uint32_t*>(&l13));
+    }
     __syncwarp();
     // ---- values: M-tile rows are record entries, K = the 16 tokens of k-step kv (quads
     // 8 wq + 4 kv + t); lane t's K columns 2t, 2t + 1 are tokens 0, 2 of its quad (bytes 0, 2 of
@@ -1186,7 +1149,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
     // a wait gave up: let every copy still in flight land (bounded) before leaving
     if (leader)
       for (int j = max(0, s_issued[wg] - NS); j < s_issued[wg]; ++j)
-        ptx::mbar_wait_sleep(full + j % NS, (j / NS) & 1, &s_last /* still 0 */, 20);
+        ptx::mbar_wait_sleep(full + j % NS, (j / NS) & 1, &s_never, 20);
     return;
   }
   // ---- per-warp (m, l, S') and entry sums into the drained rings
@@ -1196,49 +1159,39 @@ __global__ void __launch_bounds__(128 * WG, 1)
   float* wm = epi + warp * (kEpiStride + GMAX * NE);         // [m, l, S'][MAX_GROUP], then E[GMAX][NE]
   float* wE = wm + kEpiStride;
 #pragma unroll
-  for (int p = 0; p < NP; ++p)
+  for (int p = 0; p < NP; ++p) {
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-#pragma unroll
-      for (int o = 2; o < 32; o <<= 1) {
-        lsum[p][i] += __shfl_xor_sync(0xffffffffu, lsum[p][i], o);
-        ssum[p][i] += __shfl_xor_sync(0xffffffffu, ssum[p][i], o);
-      }
-      if (lane < 2) {
-        const int q = 4 * p + 2 * lane + i;
-        wm[q] = mrun[p][i];
-        wm[MAX_GROUP + q] = lsum[p][i];
-        wm[2 * MAX_GROUP + q] = ssum[p][i] * (1.0f / kPScale);
-      }
+    for (int o = 4; o < 32; o <<= 1) {
+      lsum[p] += __shfl_xor_sync(0xffffffffu, lsum[p], o);
+      ssum[p] += __shfl_xor_sync(0xffffffffu, ssum[p], o);
     }
+    if (lane < 4) {
+      const int q = 4 * p + lane;
+      wm[q] = mrun[p];
+      wm[MAX_GROUP + q] = lsum[p];
+      wm[2 * MAX_GROUP + q] = ssum[p] * (1.0f / kPScale);
+    }
+  }
   {
-    // after the hi / lo exchange lane (g, t) holds entry row g + 8 (t >> 1) of every M-tile for
-    // queries 4p + 2 (t & 1) + {0, 1}; raw sums times 2^24 / (row scale) / 2^5 = sum P' digit
-    const int row = g + 8 * (t >> 1);
+    // lane (g, t) holds entry rows g (c0 + c1) and g + 8 (c2 + c3) of every M-tile for query
+    // 4p + t; raw sums times 2^24 / (row scale) / 2^5 = sum P' digit
 #pragma unroll
     for (int jj = 0; jj < NJ; ++jj) {
       int e;
       float sc;
       if (jj < N2W) {
-        e = 16 * jj + row;
+        e = 16 * jj + g;
         sc = pow2i(19 - 2 * (g & 3));
       } else {
         const int u = (jj - N2W) >> 1, half = (jj - N2W) & 1;
-        e = 16 * N2W + 32 * u + 16 * half + row;
+        e = 16 * N2W + 32 * u + 16 * half + g;
         sc = pow2i(19 - g);
       }
 #pragma unroll
       for (int p = 0; p < NP; ++p) {
-        float r[2];
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const float mine = t < 2 ? vacc[jj][p][i] : vacc[jj][p][2 + i];
-          const float give = t < 2 ? vacc[jj][p][2 + i] : vacc[jj][p][i];
-          r[i] = mine + __shfl_xor_sync(0xffffffffu, give, 2);
-        }
-        if (e < NE)
-#pragma unroll
-          for (int i = 0; i < 2; ++i) wE[(4 * p + 2 * (t & 1) + i) * NE + e] = r[i] * sc;
+        float* dst = wE + (4 * p + t) * NE;
+        if (e < NE) dst[e] = (vacc[jj][p][0] + vacc[jj][p][1]) * sc;
+        if (e + 8 < NE) dst[e + 8] = (vacc[jj][p][2] + vacc[jj][p][3]) * sc;
       }
     }
   }
@@ -1277,111 +1230,6 @@ __global__ void __launch_bounds__(128 * WG, 1)
         dst[D] = M;
         dst[D + 1] = l;
       }
-    }
-  }
-  // ---- the CTA that sees every split of this (sequence, kv-head) done merges: M = max_s m_s,
-  // w_s = 2^(m_s - M), o_hat_c = f^V_c sum_s w_s o_{s,c} / sum_s w_s l_s, out = U_V o_hat
-  __syncthreads();
-  unsigned long long* flags = a.sem + (static_cast<size_t>(b) * a.n_kv + head) * a.n_splits;
-  if (tid == 0) {
-    __threadfence();                      // cumulative over the CTA's partial writes (barrier above)
-    atomicExch(flags + split, a.epoch);
-    __threadfence();
-  }
-  __syncthreads();
-  int done = 1;
-  for (int i = tid; i < a.n_splits; i += NT)
-    done &= *reinterpret_cast<volatile unsigned long long*>(flags + i) == a.epoch;
-  s_last = __syncthreads_and(done);
-  if (!s_last) return;
-  __threadfence();
-  ptx::fence_proxy_async_smem();                     // the bulk copy below reuses the epilogue area
-  __syncthreads();
-  for (int i = tid; i < a.n_splits; i += NT) flags[i] = 0;      // a replay starts clean
-  const int NSP = a.n_splits;
-  const FusedMerge MG(GMAX, G, NSP);
-  float* uvt = epi + MG.uvt;
-  if (tid == 0) {                                    // U_V^T lands while the partials are read
-    ptx::mbar_arrive_expect_tx(&s_uvbar, D * D * 4);
-    ptx::bulk_load(uvt, a.u32t + static_cast<size_t>(sv) * D * D, D * D * 4, &s_uvbar);
-  }
-  float* oh = epi + MG.oh;                           // [GMAX][128] o_hat
-  float* wsp = epi + MG.wsp;                         // [G][NSP] split weights
-  float* lsp = epi + MG.lsp;                         // [G][NSP] split denominators
-  float* rinv = epi + MG.rinv;                       // [G] 1 / l
-  for (int i = tid; i < G * NSP; i += NT) {          // query i / NSP, split i % NSP: one round of loads
-    const float2 ml = __ldcg(reinterpret_cast<const float2*>(a.ws + (pbase + static_cast<size_t>(i)) * a.pstride + D));
-    wsp[i] = ml.x;
-    lsp[i] = ml.y;
-  }
-  __syncthreads();
-  if (tid < G) {
-    float M = -INFINITY;
-    for (int s0 = 0; s0 < NSP; ++s0) M = fmaxf(M, wsp[tid * NSP + s0]);
-    float l = 0.0f;
-    for (int s0 = 0; s0 < NSP; ++s0) {
-      const float m = wsp[tid * NSP + s0];
-      const float w = m > -INFINITY ? fast_exp2(m - M) : 0.0f;
-      wsp[tid * NSP + s0] = w;
-      l = fmaf(w, lsp[tid * NSP + s0], l);
-    }
-    rinv[tid] = 1.0f / l;
-  }
-  __syncthreads();
-  {
-    // o_hat[q][c] = f^V_c sum_s w_s o_{s,c} / l: thread = (channel, part); its queries are
-    // part, part + WG, ...; eight splits of each in flight
-    constexpr int QPT = GMAX / WG;                     // queries per thread at most
-    const float fv = a.f[sv * D + c];
-    float o_acc[QPT];
-#pragma unroll
-    for (int qi = 0; qi < QPT; ++qi) o_acc[qi] = 0.0f;
-    for (int s0 = 0; s0 < NSP; s0 += 8) {
-      float v[QPT][8];
-#pragma unroll
-      for (int qi = 0; qi < QPT; ++qi) {
-        const int q = part + WG * qi;
-        const float* src = a.ws + (pbase + static_cast<size_t>(q) * NSP + s0) * a.pstride + c;
-#pragma unroll
-        for (int u = 0; u < 8; ++u) v[qi][u] = q < G && s0 + u < NSP ? __ldcg(src + static_cast<size_t>(u) * a.pstride) : 0.0f;
-      }
-#pragma unroll
-      for (int qi = 0; qi < QPT; ++qi) {
-        const int q = part + WG * qi;
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (q < G && s0 + u < NSP) o_acc[qi] = fmaf(wsp[q * NSP + s0 + u], v[qi][u], o_acc[qi]);
-      }
-    }
-#pragma unroll
-    for (int qi = 0; qi < QPT; ++qi) {
-      const int q = part + WG * qi;
-      if (q < G) oh[q * D + c] = o_acc[qi] * fv * rinv[q];
-    }
-  }
-  if (!ptx::mbar_wait_sleep(&s_uvbar, 0, &s_abort, 20)) atomicOr(a.err, 2);
-  __syncthreads();
-  {
-    // out[q][d] = sum_c U_V[d][c] o_hat[q][c] from shared memory: thread = (dimension d, part);
-    // its queries are part, part + WG, ...
-    constexpr int QPT = GMAX / WG;
-    const int d = c;
-    float acc[QPT];
-#pragma unroll
-    for (int qi = 0; qi < QPT; ++qi) acc[qi] = 0.0f;
-#pragma unroll 8
-    for (int cc = 0; cc < D; ++cc) {
-      const float u = uvt[cc * D + d];
-#pragma unroll
-      for (int qi = 0; qi < QPT; ++qi) {
-        const int q = part + WG * qi;
-        if (q < G) acc[qi] = fmaf(u, oh[q * D + cc], acc[qi]);
-      }
-    }
-#pragma unroll
-    for (int qi = 0; qi < QPT; ++qi) {
-      const int q = part + WG * qi;
-      if (q < G) a.out[(static_cast<size_t>(b) * a.n_q + head * G + q) * D + d] = acc[qi];
     }
   }
 }
@@ -1876,8 +1724,6 @@ static FusedKernel fused_kernel_for(int n2w, int n1w) {
   return nullptr;
 }
 
-static std::atomic<unsigned long long> g_decode_epoch{0};
-
 cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch, int n_ctx,
                           int max_tokens, float* out, void* ws, cudaStream_t st, const DecodeExtra& extra) {
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
@@ -1928,24 +1774,27 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.ks_stride = wsl.ks_stride;
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
-  a.sem = reinterpret_cast<unsigned long long*>(static_cast<char*>(ws) + wsl.sem_off);
   if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
   cudaError_t e = cudaSuccess;
   if (fk) {
     const int wu = n2w + n1w, nks = n2w + 2 * n1w;
-    a.epoch = g_decode_epoch.fetch_add(1, std::memory_order_relaxed) + 1;
     const int wg = np == 1 ? fused_groups<1>() : fused_groups<2>();
     // the deepest ring (up to 3 stages per warp group) that fits the shared memory of one SM
     size_t smem = 0;
     for (a.n_stages = 3; a.n_stages >= 2; --a.n_stages) {
-      smem = static_cast<size_t>(FusedSmem(wu, nks, np, wg, plan.n_entries, a.n_stages, a.n_splits).total);
+      smem = static_cast<size_t>(FusedSmem(wu, nks, np, wg, plan.n_entries, a.n_stages).total);
       if (smem <= 227 * 1024) break;
     }
     if (a.n_stages < 2) return cudaErrorNotSupported;
     e = ensure_smem_optin(reinterpret_cast<const void*>(fk), smem);
     if (e != cudaSuccess) return e;
     const unsigned n_cta = static_cast<unsigned>(static_cast<long>(sp.n_splits) * a.n_kv * batch);
-    return launch_pdl(fk, dim3(n_cta), dim3(128 * wg), smem, st, a);
+    e = launch_pdl(fk, dim3(n_cta), dim3(128 * wg), smem, st, a);
+    if (e != cudaSuccess) return e;
+    const size_t msm = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D);
+    e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msm);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msm, st, a);
   }
   // largest key k-step count and value word count over the layer's streams
   int n_ks = 1, n_jobs_v = 1;
