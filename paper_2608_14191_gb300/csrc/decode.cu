@@ -1755,10 +1755,11 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.n_full = extra.n_full;
   a.full_cap = extra.full_cap;
   const int np = (a.group + 3) / 4;
-  // the fused split + merge kernel: a packed range, no uncompressed tokens, one record shape
+  // the fused kernel: a packed range and one record shape (uncompressed tokens, if any, join in
+  // the merge kernel)
   int n2w = 0, n1w = 0;
   FusedKernel fk = nullptr;
-  if (extra.n_full == 0 && extra.t_first < n_ctx && layer_shape(plan, layer, &n2w, &n1w))
+  if (extra.t_first < n_ctx && layer_shape(plan, layer, &n2w, &n1w))
     fk = np == 1 ? fused_kernel_for<1>(n2w, n1w) : fused_kernel_for<2>(n2w, n1w);
   const int range = n_ctx - (extra.t_first / TILE) * TILE;
   const DecodeSplit sp = decode_split_for(batch, a.n_kv, range, plan.num_sms, fk != nullptr);
@@ -1791,7 +1792,8 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     const unsigned n_cta = static_cast<unsigned>(static_cast<long>(sp.n_splits) * a.n_kv * batch);
     e = launch_pdl(fk, dim3(n_cta), dim3(128 * wg), smem, st, a);
     if (e != cudaSuccess) return e;
-    const size_t msm = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D);
+    const size_t msm = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
+    if (msm > 227 * 1024) return cudaErrorNotSupported;
     e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msm);
     if (e != cudaSuccess) return e;
     return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msm, st, a);
