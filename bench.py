@@ -1093,7 +1093,8 @@ def run_reference(args):
 
 
 def run_profile_once(args):
-    """Minimal launch sequence for ncu captures: one encode, two decodes, one bf16 decode."""
+    """Minimal launch sequence for ncu captures: one encode, two decodes, one bf16 decode (with
+    --config llama_stack: one 131072-token layer of the stack)."""
     import torch
     import paper_2608_14191_gb300 as aatc
     from paper_2608_14191_gb300 import build as bld
@@ -1101,6 +1102,9 @@ def run_profile_once(args):
     aatc.load()
     dev = torch.device("cuda", 0)
     cfg = W.CONFIGS[args.config]
+    if cfg.n_layers > 1:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, n_layers=1)
     avg_bits = cfg.avg_bits[-1] if args.bits is None else args.bits
     B, T = cfg.batch, cfg.n_ctx
     plan, _ = build_case(aatc, cfg, avg_bits, dev)
