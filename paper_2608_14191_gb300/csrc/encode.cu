@@ -1,13 +1,15 @@
 // AATC encode on sm_103a (Algorithm 1 "Project" + "Append qtz(h)"; quantizer of Sec. 5).
 //
-// One persistent CTA per (basis, slice of work): a basis is one (layer, kv-head, K|V) stream,
-// an item is 128 consecutive new tokens of one sequence.  Warp roles:
-//   warp 16   : TMA producer -- 128 x 128 bf16 token tiles into a 3-stage SW128 ring,
-//   warp 17   : MMA issuer   -- tcgen05.mma (M=128 tokens, N=128 channels, K=128) into one of
-//                               four TMEM accumulators (all 512 columns),
-//   warps 0-15: four epilogue warpgroups; group e drains accumulator e (items e, e+4, ...):
-//               thread = token = TMEM lane: token scale alpha, quantize, split the stored
-//               values into base-4 digits / single bits and write the packed record.
+// aatc_encode_kernel: one persistent CTA per (basis, slice of work): a basis is one (layer,
+// kv-head, K|V) stream, an item is 128 consecutive new tokens of one sequence.  Warp roles:
+//   warp 12   : TMA producer -- 128 x 128 bf16 token tiles into a 5-stage SW128 ring,
+//   warp 13   : MMA issuer   -- tcgen05.mma (M=128 tokens, N=128 channels, K=128) into one of
+//                               four TMEM accumulators (all 512 columns; item i -> accumulator i % 4),
+//   warps 0-11: three epilogue warpgroups; group e drains items e, e+3, ...: thread = token =
+//               TMEM lane: token scale alpha, quantize, and the packed record built from the
+//               token's stored values held in registers (128 registers a thread: four of the
+//               14 warps share a scheduler's 16 K registers).
+// aatc_encode_hidden_kernel (further down) computes the coefficients from the layer input.
 // The projection uses the plan's bf16 basis; accumulation is fp32.
 #include <cudaTypedefs.h>
 #include <cuda.h>
@@ -21,7 +23,6 @@
 namespace aatc {
 namespace {
 
-constexpr int kStages = 3;
 constexpr int kTileBytes = TILE * D * 2;          // 32 KB of bf16
 constexpr int kEpiGroups = 4;
 constexpr int kEpiThreads = 128 * kEpiGroups;
@@ -41,18 +42,6 @@ struct EncodeArgs {
   uint32_t* words;        // cache word region (this layer)
   float* alpha;           // cache alpha region
   int layer, n_kv, batch, start, n_tokens, n_chunks, n_words, n_tiles, n_entries, ctas_per_basis;
-};
-
-struct EncodeSmem {
-  alignas(1024) unsigned char u_tile[kTileBytes];
-  alignas(1024) unsigned char x_tile[kStages][kTileBytes];
-  ChanEnc enc[D];
-  float inv_s[D];
-  StreamLayout lay;
-  uint32_t ubytes[kEpiThreads][kByteRow / 4];     // stored values u, one byte per channel
-  uint64_t full[kStages], empty[kStages], tfull[kEpiGroups], tempty[kEpiGroups], ubar;
-  uint32_t tmem_base;
-  int abort_flag;
 };
 
 template <typename Smem>
@@ -234,7 +223,235 @@ __device__ __forceinline__ RecordWriter record_writer(uint32_t* words, size_t si
   return out;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// ------------------------------------------------------------------ register-resident epilogue
+constexpr int kKStages = 5;                       // input stages of aatc_encode_kernel
+constexpr int kKGroups = 3;                       // epilogue warpgroups
+constexpr int kKAcc = 4;                          // TMEM accumulators
+constexpr int kKEpiThreads = 128 * kKGroups;
+constexpr int kKProducerWarp = kKEpiThreads / 32;
+constexpr int kKMmaWarp = kKProducerWarp + 1;
+constexpr int kKThreads = kKEpiThreads + 64;
+
+struct QuantTables {      // per channel, structure of arrays (16-byte aligned)
+  const float* inv_s;     // 1 / s_c (0 for dropped channels)
+  const float* inv_f;     // 1 / f_c
+  const float* hi;        // upper clamp of h / Delta + 1/2
+  const float* magic;     // 1.5 2^23 + 2^(b_c - 1)
+};
+
+// Token scale and stored values of one token (thread = token = TMEM lane), as quantize_token
+// but two channels per fp32 instruction and the stored values kept in registers: U[w] holds the
+// bytes u_c of channels 4w .. 4w + 3.  The arithmetic (and so every code) is the same.
+__device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const QuantTables& tb, uint32_t (&U)[32]) {
+  uint32_t ra[32], rb[32];
+  float am0 = 0.0f, am1 = 0.0f;
+  auto amax_chunk = [&](const uint32_t (&r)[32], int j) {
+#pragma unroll
+    for (int i = 0; i < 32; i += 4) {
+      const float4 is = ptx::lds_f4(&tb.inv_s[32 * j + i]);
+      float a0, a1, a2, a3;
+      ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
+                                 ptx::f2_pack(is.x, is.y)), a0, a1);
+      ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])),
+                                 ptx::f2_pack(is.z, is.w)), a2, a3);
+      am0 = ptx::fmax3(am0, fabsf(a0), fabsf(a1));
+      am1 = ptx::fmax3(am1, fabsf(a2), fabsf(a3));
+    }
+  };
+  uint64_t ia2 = 0;
+  const uint64_t half2 = ptx::f2_pack(0.5f, 0.5f);
+  // x = h / Delta + 1/2 = h (ia / f_c) + 1/2, clamped above, then the round-down add of
+  // 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
+  auto quant_chunk = [&](const uint32_t (&r)[32], int j) {
+#pragma unroll
+    for (int i = 0; i < 32; i += 4) {
+      const float4 f = ptx::lds_f4(&tb.inv_f[32 * j + i]);
+      const float4 h = ptx::lds_f4(&tb.hi[32 * j + i]);
+      const float4 m = ptx::lds_f4(&tb.magic[32 * j + i]);
+      float x0, x1, x2, x3;
+      ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
+                                 ptx::f2_mul(ptx::f2_pack(f.x, f.y), ia2), half2), x0, x1);
+      ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])),
+                                 ptx::f2_mul(ptx::f2_pack(f.z, f.w), ia2), half2), x2, x3);
+      float y0, y1, y2, y3;
+      ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x0, h.x), fminf(x1, h.y)), ptx::f2_pack(m.x, m.y)), y0, y1);
+      ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x2, h.z), fminf(x3, h.w)), ptx::f2_pack(m.z, m.w)), y2, y3);
+      U[8 * j + i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0040),
+                                     __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0040), 0x5410);
+    }
+  };
+  // Eight 32-column TMEM loads (four per pass), each issued before the previous chunk is
+  // processed so its latency overlaps that work.
+  ptx::tmem_ld_32raw(taddr, ra);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  amax_chunk(ra, 0);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  amax_chunk(rb, 1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  amax_chunk(ra, 2);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr, ra);
+  amax_chunk(rb, 3);
+  const float amax = fmaxf(am0, am1);
+  const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+  ia2 = ptx::f2_pack(ia, ia);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  quant_chunk(ra, 0);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  quant_chunk(rb, 1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  quant_chunk(ra, 2);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  quant_chunk(rb, 3);
+  return amax;
+}
+
+// Base-4 digit k of the 16 channels held in w0 .. w3, channel order LSB first: the mask-and-
+// multiply of gather_d2 on registers (m = 0x03030303 << 2k, mul = 0x01041040 >> 2k).
+__device__ __forceinline__ uint32_t digits16(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3, uint32_t m,
+                                             uint32_t mul) {
+  return __byte_perm(__byte_perm((w0 & m) * mul, (w1 & m) * mul, 0x0073),
+                     __byte_perm((w2 & m) * mul, (w3 & m) * mul, 0x0073), 0x5410);
+}
+// Bit sh = pre + s (s <= 3) of the 8 channels held in w0, w1 as the top byte (gather_d1's merge
+// and multiply: m = 0x01010101 << s, mul = 0x01020408 >> s).
+__device__ __forceinline__ uint32_t bits8_top(uint32_t w0, uint32_t w1, int pre, uint32_t m, uint32_t mul) {
+  return (((w0 >> pre) & m) | (((w1 >> pre) << 4) & (m << 4))) * mul;
+}
+// That bit of the 32 channels held in U[8i] .. U[8i + 7], channel order LSB first.
+__device__ __forceinline__ uint32_t bits32(const uint32_t (&U)[32], int i, int pre, uint32_t m, uint32_t mul) {
+  return __byte_perm(__byte_perm(bits8_top(U[8 * i], U[8 * i + 1], pre, m, mul),
+                                 bits8_top(U[8 * i + 2], U[8 * i + 3], pre, m, mul), 0x0073),
+                     __byte_perm(bits8_top(U[8 * i + 4], U[8 * i + 5], pre, m, mul),
+                                 bits8_top(U[8 * i + 6], U[8 * i + 7], pre, m, mul), 0x0073),
+                     0x5410);
+}
+
+// Writes one token's record words in order.  Keys: word-planar, token lane t of a tile in column
+// t of each record word.  Values: tokens 4Q .. 4Q+3 share slots 4Q .. 4Q+3 of each record word,
+// slot 4Q + (0, 2, 1, 3)[r] holding byte-quarter r of the four tokens' words (token 4Q + i in
+// byte i).  When the lane quad is one whole token quad of this call, a byte transpose across the
+// quad (two shuffles) gives lane i the slot of quarter i, stored as one word; otherwise each token
+// writes its own four bytes.  Every lane of the warp calls it at the same record word.
+struct RecordFlush {
+  uint32_t* tile_words;   // record word 0 of the token's tile
+  int tt;                 // token lane inside the tile
+  uint32_t s1, s2;        // byte selectors of the two transpose steps (values)
+  int qpos;               // slot of byte-quarter (lane & 3) (values)
+  bool value, quad_ok, ok;
+  int wi;
+  __device__ __forceinline__ void operator()(uint32_t w) {
+    uint32_t* rw = tile_words + static_cast<size_t>(wi) * TILE;
+    if (!value) {
+      if (ok) rw[tt] = w;
+    } else {
+      const uint32_t y1 = __byte_perm(w, __shfl_xor_sync(0xffffffffu, w, 1), s1);
+      const uint32_t y2 = __byte_perm(y1, __shfl_xor_sync(0xffffffffu, y1, 2), s2);
+      if (quad_ok) {
+        rw[4 * (tt >> 2) + qpos] = y2;
+      } else if (ok) {
+        uint8_t* q = reinterpret_cast<uint8_t*>(rw + 4 * (tt >> 2)) + (tt & 3);
+        q[0] = static_cast<uint8_t>(w);
+        q[8] = static_cast<uint8_t>(w >> 8);
+        q[4] = static_cast<uint8_t>(w >> 16);
+        q[12] = static_cast<uint8_t>(w >> 24);
+      }
+    }
+    ++wi;
+  }
+};
+
+// The packed record of one token from its stored values in registers, in the layout of
+// pack_token: D2 digits layer by layer (the last n2 % 16 of them moved behind the D1 top bits),
+// the top bit of every odd-width channel, the moved digits, zeros up to n_words.  Digit layers
+// and bit positions run as loops; the channel chunks inside them are unrolled (registers are
+// indexed at compile time) and guarded by the stream's run bounds, which are the same for every
+// thread of the CTA.
+__device__ __forceinline__ void pack_token_regs(const StreamLayout& lay, const uint32_t (&U)[32], RecordFlush& flush,
+                                                int n_words) {
+  uint32_t word = 0;
+  int pos = 0;
+  auto put = [&](uint32_t v, int nb) {                   // v: nb (1 .. 32) valid bits, zero above
+    word |= v << pos;
+    if (pos + nb >= 32) {
+      flush(word);
+      word = __funnelshift_rc(v, 0u, 32 - pos);           // the bits that did not fit (none at pos 0)
+    }
+    pos = (pos + nb) & 31;
+  };
+  uint32_t moved = 0;
+  int mpos = 0;
+#pragma unroll 1
+  for (int k = 0; k < 4; ++k) {
+    const int lk = lay.l2[k], la = lay.l2all[k];          // non-increasing in k
+    if (la == 0) break;
+    const uint32_t m = 0x03030303u << (2 * k), mul = 0x01041040u >> (2 * k);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      if (16 * c >= la) break;
+      const uint32_t v = digits16(U[4 * c], U[4 * c + 1], U[4 * c + 2], U[4 * c + 3], m, mul);
+      if (16 * c + 16 <= lk) {                             // the whole chunk stays in D2
+        put(v, 32);
+        continue;
+      }
+      const int nm = max(lk - 16 * c, 0);                  // digits that stay in D2 (< 16)
+      const int nt = min(la - 16 * c, 16);                 // digits of this chunk
+      if (nm > 0) put(v & ((1u << (2 * nm)) - 1u), 2 * nm);
+      if (nt > nm) {                                       // at most 15 digits move in all
+        moved |= (__funnelshift_rc(v, 0u, 2 * nm) & ((1u << (2 * (nt - nm))) - 1u)) << mpos;
+        mpos += 2 * (nt - nm);
+      }
+    }
+  }
+#pragma unroll 1
+  for (int k = 3; k >= 0; --k) {
+    const int a = lay.l2all[k], b = lay.lodd[k];          // width 2k + 1 channels [a, b)
+    if (a >= b) continue;
+    const int pre = k >= 2 ? 4 : 0, s = 2 * k - pre;
+    const uint32_t m = 0x01010101u << s, mul = 0x01020408u >> s;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (a < 32 * i + 32 && b > 32 * i) {
+        const int lo = max(a - 32 * i, 0), n = min(b - 32 * i, 32) - lo;
+        uint32_t v = __funnelshift_rc(bits32(U, i, pre, m, mul), 0u, lo);
+        if (n < 32) v &= (1u << n) - 1u;
+        put(v, n);
+      }
+    }
+  }
+  if (mpos > 0) put(moved, mpos);
+  if (pos > 0) flush(word);
+  while (flush.wi < n_words) flush(0u);
+}
+
+struct EncodeSmem {
+  alignas(1024) unsigned char u_tile[kTileBytes];
+  alignas(1024) unsigned char x_tile[kKStages][kTileBytes];
+  alignas(16) float inv_s[D];
+  alignas(16) float inv_f[D];
+  alignas(16) float hi[D];
+  alignas(16) float magic[D];
+  StreamLayout lay;
+  uint64_t full[kKStages], empty[kKStages], tfull[kKAcc], tempty[kKAcc], ubar;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+__global__ void __launch_bounds__(kKThreads, 1)
     aatc_encode_kernel(const __grid_constant__ CUtensorMap tmap_k, const __grid_constant__ CUtensorMap tmap_v,
                        const __grid_constant__ CUtensorMap tmap_u, const EncodeArgs a) {
   extern __shared__ unsigned char smem_raw[];
@@ -254,17 +471,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const CUtensorMap* tmap_x = kind == 0 ? &tmap_k : &tmap_v;
 
   // per-stream tables
-  for (int c = tid; c < D; c += kThreads) {
-    sm.enc[c] = a.enc[stream * D + c];
+  for (int c = tid; c < D; c += kKThreads) {
+    const ChanEnc e = a.enc[stream * D + c];
     sm.inv_s[c] = a.inv_s[stream * D + c];
+    sm.inv_f[c] = e.inv_f;
+    sm.hi[c] = e.hi;
+    sm.magic[c] = e.magic;
   }
   if (tid == 0) {
     sm.lay = a.lay[stream];
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       ptx::mbar_init(&sm.full[s], 1);
       ptx::mbar_init(&sm.empty[s], 1);
     }
-    for (int j = 0; j < kEpiGroups; ++j) {
+    for (int j = 0; j < kKAcc; ++j) {
       ptx::mbar_init(&sm.tfull[j], 1);
       ptx::mbar_init(&sm.tempty[j], 128);
     }
@@ -272,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.abort_flag = 0;
     ptx::fence_mbar_init();
   }
-  if (warp == kMmaWarp) {
+  if (warp == kKMmaWarp) {
     ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
     ptx::tmem_relinquish();
   }
@@ -282,7 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = sm.tmem_base;
   volatile int* abort_flag = &sm.abort_flag;
 
-  if (warp == kProducerWarp) {
+  if (warp == kKProducerWarp) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0 && my_items > 0) {
       ptx::prefetch_tmap(tmap_x);
@@ -291,8 +511,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tma_load_2d(sm.u_tile, &tmap_u, &sm.ubar, 0, stream * D);
       ptx::tma_load_2d(sm.u_tile + kTileBytes / 2, &tmap_u, &sm.ubar, 64, stream * D);
       for (int it = 0; it < my_items; ++it) {
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
+        const int s = it % kKStages;
+        const uint32_t ph = (it / kKStages) & 1;
         if (!ptx::mbar_wait_bounded(&sm.empty[s], ph ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
         const long item = it0 + it;
         const int b = static_cast<int>(item / a.n_chunks);
@@ -302,7 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tma_load_4d(sm.x_tile[s] + kTileBytes / 2, tmap_x, &sm.full[s], 64, head, i0, b);
       }
     }
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kKMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && my_items > 0) {
       constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128);
@@ -310,10 +530,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = ptx::mbar_wait_bounded(&sm.ubar, 0, abort_flag);
       if (!ok) raise_abort(sm, a.err);
       for (int it = 0; ok && it < my_items; ++it) {
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
-        const int acc = it % kEpiGroups;
-        const uint32_t aph = (it / kEpiGroups) & 1;
+        const int s = it % kKStages;
+        const uint32_t ph = (it / kKStages) & 1;
+        const int acc = it % kKAcc;
+        const uint32_t aph = (it / kKAcc) & 1;
         if (!ptx::mbar_wait_bounded(&sm.tempty[acc], aph ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
         ptx::tc_fence_after();
         if (!ptx::mbar_wait_bounded(&sm.full[s], ph, abort_flag)) { raise_abort(sm, a.err); break; }
@@ -331,37 +551,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue: thread = token
-    const int eg = warp >> 2;                                  // epilogue group = accumulator
+    const int eg = warp >> 2;                                  // epilogue group
     const int quad = warp & 3;                                 // TMEM lane quadrant
     const int tl = quad * 32 + lane;                           // token lane inside the tile
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-    const StreamLayout& lay = sm.lay;
-    uint32_t* my_bytes = sm.ubytes[tid];
-    for (int it = eg; it < my_items; it += kEpiGroups) {
-      const uint32_t aph = (it / kEpiGroups) & 1;
-      if (!ptx::mbar_wait_bounded(&sm.tfull[eg], aph, abort_flag)) { raise_abort(sm, a.err); break; }
+    const QuantTables tb{sm.inv_s, sm.inv_f, sm.hi, sm.magic};
+    const int t4 = lane & 3;                                   // position in the lane quad
+    const uint32_t s1 = (t4 & 1) ? 0x3715u : 0x6240u, s2 = (t4 & 2) ? 0x3276u : 0x5410u;
+    const int qpos = ((t4 & 1) << 1) | (t4 >> 1);              // slot of byte-quarter t4
+#pragma unroll 1
+    for (int it = eg; it < my_items; it += kKGroups) {
+      const int acc = it % kKAcc;
+      const uint32_t aph = (it / kKAcc) & 1;
+      if (!ptx::mbar_wait_bounded(&sm.tfull[acc], aph, abort_flag)) { raise_abort(sm, a.err); break; }
       ptx::tc_fence_after();
-      const uint32_t taddr = tmem + eg * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
-
-      const float amax = quantize_token(taddr, sm.enc, sm.inv_s, my_bytes);
+      const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
+      uint32_t U[32];
+      const float amax = quantize_token_regs(taddr, tb, U);
       ptx::tc_fence_before();
-      ptx::mbar_arrive(&sm.tempty[eg]);
+      ptx::mbar_arrive(&sm.tempty[acc]);
 
       const long item = it0 + it;
       const int b = static_cast<int>(item / a.n_chunks);
       const int i = static_cast<int>(item % a.n_chunks) * TILE + tl;     // input token index
-      if (i >= a.n_tokens) continue;
+      const bool ok = i < a.n_tokens;
+      if (!__any_sync(0xffffffffu, ok)) continue;
       const int pos_t = a.start + i;
       const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
-      if (!isfinite(amax)) atomicOr(a.err, 1);
-      a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
-      pack_token(lay, my_bytes, record_writer(a.words, sidx, stream_words, a.n_words, pos_t, kind == 1), a.n_words);
+      if (ok) {
+        if (!isfinite(amax)) atomicOr(a.err, 1);
+        a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
+      }
+      // lanes 4Q' .. 4Q'+3 are one token quad of the cache when start is a multiple of 4
+      RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
+                    pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
+      pack_token_regs(sm.lay, U, f, a.n_words);
     }
   }
 
   ptx::tc_fence_before();
   __syncthreads();
-  if (warp == kMmaWarp) {
+  if (warp == kKMmaWarp) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
@@ -620,7 +850,7 @@ cudaError_t launch_encode(const Plan& plan, int layer, const void* K, const void
   e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_kernel), smem);
   if (e != cudaSuccess) return e;
   const auto* mu = reinterpret_cast<const CUtensorMap*>(plan.tmap_u);
-  aatc_encode_kernel<<<n_basis * k, kThreads, smem, st>>>(mk, mv, *mu, a);
+  aatc_encode_kernel<<<n_basis * k, kKThreads, smem, st>>>(mk, mv, *mu, a);
   return cudaGetLastError();
 }
 
