@@ -32,7 +32,7 @@ extern "C" {
 #endif
 
 #define AATC_HEAD_DIM 128
-#define AATC_MAX_BITS 8        /* widest channel code a device plan holds; widths 0..AATC_MAX_BITS */
+#define AATC_MAX_BITS 16       /* widest channel code a device plan holds; widths 0..AATC_MAX_BITS */
 #define AATC_MAX_PLAN_BITS 16  /* widest width the host planner allocates (Sec. 5 allows b in 0..16) */
 
 typedef struct aatc_plan_s* aatc_plan_t;   /* opaque; immutable after creation */
@@ -51,8 +51,8 @@ typedef enum {
 } aatc_status_t;
 
 /* Model dimensions.  d must be 128; n_q_heads % n_kv_heads == 0; b_max in 1..AATC_MAX_PLAN_BITS for
- * the host planner calls, in 1..AATC_MAX_BITS for aatc_plan_create (wider plans are
- * AATC_ERR_UNSUPPORTED: the record layout and kernels take widths up to 8). */
+ * the host planner calls and in 1..AATC_MAX_BITS for aatc_plan_create (the paper's range
+ * b in 0..16 of Sec. 6 for both). */
 typedef struct {
   int32_t d;
   int32_t n_layers;
@@ -215,7 +215,8 @@ aatc_status_t aatc_plan_load(const char* path, const aatc_dims_t* dims, float* b
  * copy on `stream`, then synchronizes it.  Host inputs are copied; the caller keeps them.
  * Errors: AATC_ERR_INVALID_ARG (null, bits > b_max, bits not non-increasing, scale <= 0 or
  * non-finite where bits > 0, non-finite basis), AATC_ERR_UNSUPPORTED (dims->b_max above
- * AATC_MAX_BITS: a plan the planner made with wider widths), AATC_ERR_CUDA, AATC_ERR_NOMEM.
+ * AATC_MAX_BITS, or a stream with more than 32 channels wider than 8 bits: the encode keeps
+ * the high bytes of the first 32 stored values only), AATC_ERR_CUDA, AATC_ERR_NOMEM.
  * All argument checks run before any CUDA call.
  */
 aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
@@ -263,8 +264,9 @@ aatc_status_t aatc_encode(aatc_plan_t plan, int32_t layer, const void* K, const 
  *   d_model : multiple of 64, 64 .. 65536
  *   a_hat   : device bf16 [L][n_kv][2][128][d_model] (aatc_hidden_operand's layout), 16-byte aligned
  * Asynchronous on `stream`.  Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer,
- * sizes or d_model), AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_CUDA.
- * n_tokens == 0 is a no-op (x, a_hat and cache may then be NULL).
+ * sizes or d_model), AATC_ERR_CAPACITY (start + n_tokens > max_tokens), AATC_ERR_UNSUPPORTED (a
+ * plan with a width above 8: this kernel's epilogue packs one byte per stored value),
+ * AATC_ERR_CUDA.  n_tokens == 0 is a no-op (x, a_hat and cache may then be NULL).
  */
 aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x, int32_t d_model, const void* a_hat,
                                  int32_t batch, int32_t start, int32_t n_tokens, void* cache, int32_t max_tokens,
@@ -284,7 +286,8 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t plan, int32_t layer, const void* x,
  *               transposed as [channel][token] per 128-token tile); contents ignored
  * Query head j reads kv-head j / (n_q_heads / n_kv_heads).  Asynchronous on `stream`.
  * Errors: AATC_ERR_INVALID_ARG (null or unaligned pointers, bad layer or sizes, q_start + n_q >
- * n_ctx), AATC_ERR_CAPACITY (n_ctx > max_tokens), AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (W > 32),
+ * n_ctx), AATC_ERR_CAPACITY (n_ctx > max_tokens), AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (W > 32,
+ * or a width above 12: the codes are tensor-core operands in f16, exact up to |code| = 2048),
  * AATC_ERR_CUDA.
  */
 aatc_status_t aatc_prefill_workspace_bytes(aatc_plan_t plan, int32_t batch, int32_t n_ctx, size_t* bytes);

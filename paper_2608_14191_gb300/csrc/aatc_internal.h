@@ -33,7 +33,7 @@ struct ChanEnc {
 
 // Record layout of one stream.  The stored value u = code + 2^(b-1) of every retained channel
 // is split into base-4 digits and single top bits:
-//   D2: for k = 0..3, digit k (bits 2k, 2k+1) of channels 0..l2[k]-1  (16 two-bit fields/word)
+//   D2: for k = 0..7, digit k (bits 2k, 2k+1) of channels 0..l2[k]-1  (16 two-bit fields/word)
 //   D1: the top bit of every odd-width channel (channel order), then the digits that did not
 //       fill the last D2 word, each as two single bits (32 one-bit fields/word)
 // Record words: n2/16 D2 words, then ceil(n1/32) D1 words, then zeros up to the plan's W.
@@ -44,10 +44,17 @@ struct StreamLayout {
   int n1;                 // D1 entries
   int words;              // record words this stream uses
   int nret;               // retained channels R
-  int l2[4];              // D2 digit-layer lengths (digits kept in D2)
-  int l2all[4];           // channels with b >= 2k + 2 (digit k exists; those past l2[k] moved to D1)
-  int lodd[4];            // channels with b >= 2k + 1 (width 2k + 1 channels: [l2all[k], lodd[k]))
+  int l2[8];              // D2 digit-layer lengths (digits kept in D2)
+  int l2all[8];           // channels with b >= 2k + 2 (digit k exists; those past l2[k] moved to D1)
+  int lodd[8];            // channels with b >= 2k + 1 (width 2k + 1 channels: [l2all[k], lodd[k]))
 };
+
+// Record entries of one channel: at most 8 digits, or 7 with one moved to D1 as two bits plus an
+// odd top bit, so 9 at 16 bits; the per-channel entry table keeps kChanEnt slots.
+constexpr int kChanEnt = 16;
+// The register-resident encode keeps the high bytes of the first 32 stored values: channels
+// wider than 8 bits must lie in that prefix (widths are non-increasing in storage order).
+constexpr int kMaxWideChannels = 32;
 
 struct PlanDevice {
   const void* ubf16_t;    // bf16 [S][128 channel][128 dim]   encode basis (MMA B operand, K-major)
@@ -68,6 +75,7 @@ struct Plan {
   int n_streams = 0;
   int n_words = 0;        // W, words per record (plan-wide)
   int n_entries = 0;      // entries per stream in `entry` (32 * W)
+  int max_bits = 0;       // widest channel of any stream
   int num_sms = 0;
   int device = 0;
   std::vector<int> retained;

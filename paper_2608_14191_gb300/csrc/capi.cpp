@@ -133,7 +133,7 @@ size_t bf16_decode_workspace(int batch, int n_q, const DecodeSplit& sp) {
 void build_layout(const uint8_t* bits, StreamLayout* lay, std::vector<short>& entries) {
   std::vector<short> d2, d1;
   auto ent = [](int c, int sh) { return static_cast<short>(c | (sh << 8)); };
-  for (int k = 0; k < 4; ++k) {
+  for (int k = 0; k < 8; ++k) {
     int n = 0;
     for (int c = 0; c < D; ++c)
       if (bits[c] >= 2 * k + 2) {
@@ -155,7 +155,7 @@ void build_layout(const uint8_t* bits, StreamLayout* lay, std::vector<short>& en
     d1.push_back(ent(c, sh + 1));
   }
   d2.resize(d2.size() - r);
-  for (int k = 3, left = r; k >= 0 && left > 0; --k) {      // the moved digits came off the last layers
+  for (int k = 7, left = r; k >= 0 && left > 0; --k) {      // the moved digits came off the last layers
     const int take = std::min(left, lay->l2[k]);
     lay->l2[k] -= take;
     left -= take;
@@ -195,7 +195,7 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
                                const float* scales, void* stream, aatc_plan_t* plan_out) {
   using namespace aatc;
   if (!valid_dims(dims) || !basis || !bits || !scales || !plan_out) return AATC_ERR_INVALID_ARG;
-  if (dims->b_max > AATC_MAX_BITS) return AATC_ERR_UNSUPPORTED;   // records hold widths up to 8
+  if (dims->b_max > AATC_MAX_BITS) return AATC_ERR_UNSUPPORTED;
   const int S = dims->n_layers * dims->n_kv_heads * 2;
   const size_t SD = static_cast<size_t>(S) * D;
   // validate
@@ -206,6 +206,7 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
       const int b = bits[s * D + c];
       if (b > dims->b_max) return AATC_ERR_INVALID_ARG;
       if (c > 0 && b > bits[s * D + c - 1]) return AATC_ERR_INVALID_ARG;   // non-increasing
+      if (b > 8 && c >= kMaxWideChannels) return AATC_ERR_UNSUPPORTED;
       if (b > 0) {
         const float sc = scales[s * D + c];
         if (!(std::isfinite(sc) && sc > 0.0f)) return AATC_ERR_INVALID_ARG;
@@ -238,7 +239,7 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   const size_t o_f = off;    off = align_up(off + SD * 4, 256);
   const size_t o_lay = off;  off = align_up(off + static_cast<size_t>(S) * sizeof(StreamLayout), 256);
   const size_t o_ent = off;  off = align_up(off + static_cast<size_t>(S) * E * sizeof(short), 256);
-  const size_t o_che = off;  off = align_up(off + SD * 8 * sizeof(short), 256);
+  const size_t o_che = off;  off = align_up(off + SD * kChanEnt * sizeof(short), 256);
   const size_t o_err = off;  off = align_up(off + 16, 256);
   const size_t total = off;
   std::vector<unsigned char> host;
@@ -282,12 +283,12 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
     lay[s] = layout[s];
     for (int e = 0; e < E; ++e)
       ent[static_cast<size_t>(s) * E + e] = e < static_cast<int>(entries[s].size()) ? entries[s][e] : short(-1);
-    short* ce = che + static_cast<size_t>(s) * D * 8;
-    for (int i = 0; i < D * 8; ++i) ce[i] = -1;
+    short* ce = che + static_cast<size_t>(s) * D * kChanEnt;
+    for (int i = 0; i < D * kChanEnt; ++i) ce[i] = -1;
     int fill[D] = {0};
     for (int e = 0; e < static_cast<int>(entries[s].size()); ++e) {
       const int c = entries[s][e] & 0xFF;
-      if (fill[c] < 8) ce[c * 8 + fill[c]++] = static_cast<short>(e);
+      if (fill[c] < kChanEnt) ce[c * kChanEnt + fill[c]++] = static_cast<short>(e);
     }
   }
 
@@ -297,6 +298,7 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   plan->n_streams = S;
   plan->n_words = W;
   plan->n_entries = E;
+  for (size_t i = 0; i < SD; ++i) plan->max_bits = std::max(plan->max_bits, static_cast<int>(bits[i]));
   plan->retained = retained;
   plan->nbits = nbits;
   plan->layout = layout;
@@ -385,6 +387,7 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t p, int32_t layer, const void* x, in
   if (n_tokens == 0) return AATC_OK;                   // an empty append reads no pointer
   if (!x || !a_hat || !cache || !aligned16(x) || !aligned16(a_hat) || !aligned16(cache))
     return AATC_ERR_INVALID_ARG;
+  if (plan->max_bits > 8) return AATC_ERR_UNSUPPORTED;   // this epilogue packs one byte per stored value
   return cuda_status(aatc::launch_encode_hidden(*plan, layer, x, d_model, a_hat, batch, start, n_tokens, cache,
                                                 max_tokens, static_cast<cudaStream_t>(stream)));
 }
@@ -407,6 +410,7 @@ aatc_status_t aatc_prefill_attention(aatc_plan_t p, int32_t layer, const void* q
   if (static_cast<int64_t>(q_start) + n_q > n_ctx) return AATC_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(cache) || !aligned16(out) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
   if (plan->n_words > 32) return AATC_ERR_UNSUPPORTED;
+  if (plan->max_bits > 12) return AATC_ERR_UNSUPPORTED;   // f16 code operands are exact up to |code| = 2048
   if (workspace_bytes < aatc::prefill_workspace(batch, plan->dims.n_kv_heads, n_ctx)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_prefill(*plan, layer, q, q_start, n_q, cache, batch, n_ctx, max_tokens, out,
                                           workspace, static_cast<cudaStream_t>(stream)));

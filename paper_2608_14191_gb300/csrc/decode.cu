@@ -81,7 +81,7 @@ struct DecodeArgs {
   const ChanEnc* enc;      // plan: [S][128] (offsets 2^(b-1))
   const StreamLayout* lay; // plan: [S]
   const short* entry;      // plan: [S][n_entries]
-  const short* chan_ent;   // plan: [S][128][8]
+  const short* chan_ent;   // plan: [S][128][kChanEnt] record entries of each channel (-1 padded)
   int* err;
   uint4* qfrag;            // workspace: score A fragments [batch][n_kv][ks_stride]
   float* qcorr;            // workspace: [batch][n_kv][16]: offset corrections C_g, score scales
@@ -144,7 +144,7 @@ constexpr float kOpMax = 16384.0f;            // |A operand| scaled to <= 2^14 (
 constexpr float kDigitScale = 16777216.0f;    // a digit's f16 value is digit * 2^-24
 
 constexpr int kQThreads = 512;
-constexpr int kMaxEntries = 32 * 32;   // 8 bits x 128 channels
+constexpr int kMaxEntries = 64 * 32;   // 16 bits x 128 channels
 
 // Per call, per (sequence, kv-head, query slot g < 8): folded query q'_c = (U_K^T q)_c f_c
 // log2(e)/sqrt(128), its offset correction C = sum_c q'_c 2^(b_c-1), the score scale, and rows g
@@ -284,7 +284,7 @@ struct SplitSmem {
     bars = o;  o = align16(o + 8 * (kStages + 1));  // ring barriers, then the prologue barrier
     qcg = o;   o += 2 * MAX_GROUP * 4;              // offset corrections, score scales
     red = o;   o += 4 * kWarps * MAX_GROUP * 4;     // reductions; per-query m, l, S', split max
-    cetab = o; o += D * 8 * 2;                      // record entries of each value channel
+    cetab = o; o += D * kChanEnt * 2;               // record entries of each value channel
     etab = o;  o = align16(o + n_entries * 2);      // value entry table (channel | shift << 8)
     afrag = o; o += n_ks * 32 * 16;                 // score A fragments per (k-step, lane)
     ak = o;    o += split_len * 4;                  // alpha^K, alpha^V of the split
@@ -381,11 +381,11 @@ __global__ void __launch_bounds__(kThreads)
     const uint32_t abytes = static_cast<uint32_t>(n_tiles_split) * TILE * 4;
     const uint32_t ebytes = static_cast<uint32_t>(align16(a.n_entries * 2));
     const uint32_t fbytes = static_cast<uint32_t>(n_ks) * NP * 32 * 8;
-    ptx::mbar_arrive_expect_tx(pro, 2 * abytes + D * 8 * 2 + ebytes + fbytes + 2 * MAX_GROUP * 4);
+    ptx::mbar_arrive_expect_tx(pro, 2 * abytes + D * kChanEnt * 2 + ebytes + fbytes + 2 * MAX_GROUP * 4);
     ptx::bulk_load(ak, kalpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
     for (int i = 0; i < min(kStages, n_seq); ++i) issue_tile(i);
     ptx::bulk_load(av, valpha + static_cast<size_t>(tile0) * TILE, abytes, pro);
-    ptx::bulk_load(smb + L.cetab, a.chan_ent + static_cast<size_t>(sv) * D * 8, D * 8 * 2, pro);
+    ptx::bulk_load(smb + L.cetab, a.chan_ent + static_cast<size_t>(sv) * D * kChanEnt, D * kChanEnt * 2, pro);
     ptx::bulk_load(smb + L.etab, a.entry + static_cast<size_t>(sv) * a.n_entries, ebytes, pro);
     // the query kernel's fragments and corrections
     ptx::grid_dependency_wait();
@@ -675,20 +675,22 @@ __global__ void __launch_bounds__(kThreads)
   const size_t pbase = (static_cast<size_t>(b) * a.n_q + head * G) * a.n_splits;
   {
     const int c = tid;
-    const uint4 cev = *reinterpret_cast<const uint4*>(cetab + c * 8);
-    const short* ce = reinterpret_cast<const short*>(&cev);
-    float w[8];
-    int e_[8];
+    // up to kChanEnt record entries of the channel (more than 8 only for widths above 8)
+    const short* ce = cetab + c * kChanEnt;
+    const int nce = ce[8] >= 0 ? kChanEnt : 8;
+    float w[kChanEnt];
+    int e_[kChanEnt];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      e_[k] = min(max(static_cast<int>(ce[k]), 0), a.n_entries - 1);
-      w[k] = ce[k] >= 0 ? pow2i((etab[e_[k]] >> 8) & 7) : 0.0f;
+    for (int k = 0; k < kChanEnt; ++k) {
+      const int ek = k < nce ? ce[k] : -1;
+      e_[k] = min(max(ek, 0), a.n_entries - 1);
+      w[k] = ek >= 0 ? pow2i((etab[e_[k]] >> 8) & 15) : 0.0f;
     }
     const float off = off_c;
     for (int q = 0; q < G; ++q) {
       float o = -off * ml[2 * MAX_GROUP + q];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) o = fmaf(w[k], oe[q * a.n_entries + e_[k]], o);
+      for (int k = 0; k < kChanEnt; ++k) o = fmaf(w[k], oe[q * a.n_entries + e_[k]], o);
       float* dst = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits + split) * a.pstride;
       dst[c] = o;
       if (c == 0) {
@@ -815,8 +817,10 @@ __global__ void __launch_bounds__(128 * WG, 1)
     s_never = 0;
   }
   // plan constants (never written by a kernel): the streams' entry tables, key channel constants
+  // (the first 8 entries of each channel: all of them for widths up to 8, the only plans this
+  // kernel is launched for)
   for (int i = tid; i < D * 8; i += NT)
-    reinterpret_cast<short*>(smb + L.cetab)[i] = a.chan_ent[static_cast<size_t>(sv) * D * 8 + i];
+    reinterpret_cast<short*>(smb + L.cetab)[i] = a.chan_ent[(static_cast<size_t>(sv) * D + (i >> 3)) * kChanEnt + (i & 7)];
   for (int i = tid; i < a.n_entries; i += NT) {
     reinterpret_cast<short*>(smb + L.etab)[i] = a.entry[static_cast<size_t>(sv) * a.n_entries + i];
     reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
@@ -1759,7 +1763,7 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   // the merge kernel)
   int n2w = 0, n1w = 0;
   FusedKernel fk = nullptr;
-  if (extra.t_first < n_ctx && layer_shape(plan, layer, &n2w, &n1w))
+  if (extra.t_first < n_ctx && plan.max_bits <= 8 && layer_shape(plan, layer, &n2w, &n1w))
     fk = np == 1 ? fused_kernel_for<1>(n2w, n1w) : fused_kernel_for<2>(n2w, n1w);
   const int range = n_ctx - (extra.t_first / TILE) * TILE;
   const DecodeSplit sp = decode_split_for(batch, a.n_kv, range, plan.num_sms, fk != nullptr);

@@ -16,6 +16,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "aatc_internal.h"
 #include "ptx.cuh"
@@ -241,8 +242,11 @@ struct QuantTables {      // per channel, structure of arrays (16-byte aligned)
 
 // Token scale and stored values of one token (thread = token = TMEM lane), as quantize_token
 // but two channels per fp32 instruction and the stored values kept in registers: U[w] holds the
-// bytes u_c of channels 4w .. 4w + 3.  The arithmetic (and so every code) is the same.
-__device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const QuantTables& tb, uint32_t (&U)[32]) {
+// low bytes of u_c for channels 4w .. 4w + 3, UH[w] the high bytes (u_c >= 256 only for widths
+// above 8, which lie in the first 32 channels).  The arithmetic (and so every code) is the same.
+template <bool kWide>
+__device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const QuantTables& tb, uint32_t (&U)[32],
+                                                     uint32_t (&UH)[8]) {
   uint32_t ra[32], rb[32];
   float am0 = 0.0f, am1 = 0.0f;
   auto amax_chunk = [&](const uint32_t (&r)[32], int j) {
@@ -261,7 +265,7 @@ __device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const Quant
   uint64_t ia2 = 0;
   const uint64_t half2 = ptx::f2_pack(0.5f, 0.5f);
   // x = h / Delta + 1/2 = h (ia / f_c) + 1/2, clamped above, then the round-down add of
-  // 1.5 2^23 + 2^(b-1) leaves u (< 256) in the low byte of the float.
+  // 1.5 2^23 + 2^(b-1) leaves u (< 2^16) in the low two bytes of the float.
   auto quant_chunk = [&](const uint32_t (&r)[32], int j) {
 #pragma unroll
     for (int i = 0; i < 32; i += 4) {
@@ -278,6 +282,9 @@ __device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const Quant
       ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x2, h.z), fminf(x3, h.w)), ptx::f2_pack(m.z, m.w)), y2, y3);
       U[8 * j + i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0040),
                                      __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0040), 0x5410);
+      if (kWide && j == 0)
+        UH[i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0051),
+                                __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0051), 0x5410);
     }
   };
   // Eight 32-column TMEM loads (four per pass), each issued before the previous chunk is
@@ -333,7 +340,8 @@ __device__ __forceinline__ uint32_t bits8_top(uint32_t w0, uint32_t w1, int pre,
   return (((w0 >> pre) & m) | (((w1 >> pre) << 4) & (m << 4))) * mul;
 }
 // That bit of the 32 channels held in U[8i] .. U[8i + 7], channel order LSB first.
-__device__ __forceinline__ uint32_t bits32(const uint32_t (&U)[32], int i, int pre, uint32_t m, uint32_t mul) {
+template <int N>
+__device__ __forceinline__ uint32_t bits32(const uint32_t (&U)[N], int i, int pre, uint32_t m, uint32_t mul) {
   return __byte_perm(__byte_perm(bits8_top(U[8 * i], U[8 * i + 1], pre, m, mul),
                                  bits8_top(U[8 * i + 2], U[8 * i + 3], pre, m, mul), 0x0073),
                      __byte_perm(bits8_top(U[8 * i + 4], U[8 * i + 5], pre, m, mul),
@@ -380,9 +388,11 @@ struct RecordFlush {
 // the top bit of every odd-width channel, the moved digits, zeros up to n_words.  Digit layers
 // and bit positions run as loops; the channel chunks inside them are unrolled (registers are
 // indexed at compile time) and guarded by the stream's run bounds, which are the same for every
-// thread of the CTA.
-__device__ __forceinline__ void pack_token_regs(const StreamLayout& lay, const uint32_t (&U)[32], RecordFlush& flush,
-                                                int n_words) {
+// thread of the CTA.  Digit layers 4..7 and the top bits of widths 9..15 come from the high
+// bytes UH (channels 0..31).
+template <bool kWide>
+__device__ __forceinline__ void pack_token_regs(const StreamLayout& lay, const uint32_t (&U)[32],
+                                                const uint32_t (&UH)[8], RecordFlush& flush, int n_words) {
   uint32_t word = 0;
   int pos = 0;
   auto put = [&](uint32_t v, int nb) {                   // v: nb (1 .. 32) valid bits, zero above
@@ -395,42 +405,60 @@ __device__ __forceinline__ void pack_token_regs(const StreamLayout& lay, const u
   };
   uint32_t moved = 0;
   int mpos = 0;
+  // chunk c (channels 16c .. 16c + 15) of a digit layer whose run is [0, la), the first lk kept
+  auto digit_chunk = [&](uint32_t v, int c, int lk, int la) {
+    if (16 * c + 16 <= lk) {                               // the whole chunk stays in D2
+      put(v, 32);
+      return;
+    }
+    const int nm = max(lk - 16 * c, 0);                    // digits that stay in D2 (< 16)
+    const int nt = min(la - 16 * c, 16);                   // digits of this chunk
+    if (nm > 0) put(v & ((1u << (2 * nm)) - 1u), 2 * nm);
+    if (nt > nm) {                                         // at most 15 digits move in all
+      moved |= (__funnelshift_rc(v, 0u, 2 * nm) & ((1u << (2 * (nt - nm))) - 1u)) << mpos;
+      mpos += 2 * (nt - nm);
+    }
+  };
 #pragma unroll 1
-  for (int k = 0; k < 4; ++k) {
+  for (int k = 0; k < (kWide ? 8 : 4); ++k) {
     const int lk = lay.l2[k], la = lay.l2all[k];          // non-increasing in k
     if (la == 0) break;
-    const uint32_t m = 0x03030303u << (2 * k), mul = 0x01041040u >> (2 * k);
+    const uint32_t m = 0x03030303u << (2 * (k & 3)), mul = 0x01041040u >> (2 * (k & 3));
+    if (!kWide || k < 4) {
 #pragma unroll
-    for (int c = 0; c < 8; ++c) {
-      if (16 * c >= la) break;
-      const uint32_t v = digits16(U[4 * c], U[4 * c + 1], U[4 * c + 2], U[4 * c + 3], m, mul);
-      if (16 * c + 16 <= lk) {                             // the whole chunk stays in D2
-        put(v, 32);
-        continue;
+      for (int c = 0; c < 8; ++c) {
+        if (16 * c >= la) break;
+        digit_chunk(digits16(U[4 * c], U[4 * c + 1], U[4 * c + 2], U[4 * c + 3], m, mul), c, lk, la);
       }
-      const int nm = max(lk - 16 * c, 0);                  // digits that stay in D2 (< 16)
-      const int nt = min(la - 16 * c, 16);                 // digits of this chunk
-      if (nm > 0) put(v & ((1u << (2 * nm)) - 1u), 2 * nm);
-      if (nt > nm) {                                       // at most 15 digits move in all
-        moved |= (__funnelshift_rc(v, 0u, 2 * nm) & ((1u << (2 * (nt - nm))) - 1u)) << mpos;
-        mpos += 2 * (nt - nm);
+    } else {                                               // la <= 32: widths above 8
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        if (16 * c >= la) break;
+        digit_chunk(digits16(UH[4 * c], UH[4 * c + 1], UH[4 * c + 2], UH[4 * c + 3], m, mul), c, lk, la);
       }
     }
   }
 #pragma unroll 1
-  for (int k = 3; k >= 0; --k) {
+  for (int k = kWide ? 7 : 3; k >= 0; --k) {
     const int a = lay.l2all[k], b = lay.lodd[k];          // width 2k + 1 channels [a, b)
     if (a >= b) continue;
-    const int pre = k >= 2 ? 4 : 0, s = 2 * k - pre;
+    const int pre = (k & 3) >= 2 ? 4 : 0, s = 2 * (k & 3) - pre;
     const uint32_t m = 0x01010101u << s, mul = 0x01020408u >> s;
+    if (!kWide || k < 4) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (a < 32 * i + 32 && b > 32 * i) {
-        const int lo = max(a - 32 * i, 0), n = min(b - 32 * i, 32) - lo;
-        uint32_t v = __funnelshift_rc(bits32(U, i, pre, m, mul), 0u, lo);
-        if (n < 32) v &= (1u << n) - 1u;
-        put(v, n);
+      for (int i = 0; i < 4; ++i) {
+        if (a < 32 * i + 32 && b > 32 * i) {
+          const int lo = max(a - 32 * i, 0), n = min(b - 32 * i, 32) - lo;
+          uint32_t v = __funnelshift_rc(bits32(U, i, pre, m, mul), 0u, lo);
+          if (n < 32) v &= (1u << n) - 1u;
+          put(v, n);
+        }
       }
+    } else {                                               // widths 9 .. 15: b <= 32
+      const int n = b - a;
+      uint32_t v = __funnelshift_rc(bits32(UH, 0, pre, m, mul), 0u, a);
+      if (n < 32) v &= (1u << n) - 1u;
+      put(v, n);
     }
   }
   if (mpos > 0) put(moved, mpos);
@@ -559,34 +587,42 @@ __global__ void __launch_bounds__(kKThreads, 1)
     const int t4 = lane & 3;                                   // position in the lane quad
     const uint32_t s1 = (t4 & 1) ? 0x3715u : 0x6240u, s2 = (t4 & 2) ? 0x3276u : 0x5410u;
     const int qpos = ((t4 & 1) << 1) | (t4 >> 1);              // slot of byte-quarter t4
+    // one instantiation for streams with a channel wider than 8 bits (high bytes kept), one without
+    auto drain = [&](auto wide_tag) {
+      constexpr bool kWide = decltype(wide_tag)::value;
 #pragma unroll 1
-    for (int it = eg; it < my_items; it += kKGroups) {
-      const int acc = it % kKAcc;
-      const uint32_t aph = (it / kKAcc) & 1;
-      if (!ptx::mbar_wait_bounded(&sm.tfull[acc], aph, abort_flag)) { raise_abort(sm, a.err); break; }
-      ptx::tc_fence_after();
-      const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
-      uint32_t U[32];
-      const float amax = quantize_token_regs(taddr, tb, U);
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&sm.tempty[acc]);
+      for (int it = eg; it < my_items; it += kKGroups) {
+        const int acc = it % kKAcc;
+        const uint32_t aph = (it / kKAcc) & 1;
+        if (!ptx::mbar_wait_bounded(&sm.tfull[acc], aph, abort_flag)) { raise_abort(sm, a.err); break; }
+        ptx::tc_fence_after();
+        const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(quad * 32) << 16);
+        uint32_t U[32], UH[8];
+        const float amax = quantize_token_regs<kWide>(taddr, tb, U, UH);
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&sm.tempty[acc]);
 
-      const long item = it0 + it;
-      const int b = static_cast<int>(item / a.n_chunks);
-      const int i = static_cast<int>(item % a.n_chunks) * TILE + tl;     // input token index
-      const bool ok = i < a.n_tokens;
-      if (!__any_sync(0xffffffffu, ok)) continue;
-      const int pos_t = a.start + i;
-      const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
-      if (ok) {
-        if (!isfinite(amax)) atomicOr(a.err, 1);
-        a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
+        const long item = it0 + it;
+        const int b = static_cast<int>(item / a.n_chunks);
+        const int i = static_cast<int>(item % a.n_chunks) * TILE + tl;     // input token index
+        const bool ok = i < a.n_tokens;
+        if (!__any_sync(0xffffffffu, ok)) continue;
+        const int pos_t = a.start + i;
+        const size_t sidx = (static_cast<size_t>(b) * a.n_kv + head) * 2 + kind;
+        if (ok) {
+          if (!isfinite(amax)) atomicOr(a.err, 1);
+          a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
+        }
+        // lanes 4Q' .. 4Q'+3 are one token quad of the cache when start is a multiple of 4
+        RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
+                      pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
+        pack_token_regs<kWide>(sm.lay, U, UH, f, a.n_words);
       }
-      // lanes 4Q' .. 4Q'+3 are one token quad of the cache when start is a multiple of 4
-      RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
-                    pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
-      pack_token_regs(sm.lay, U, f, a.n_words);
-    }
+    };
+    if (sm.lay.lodd[4] > 0)
+      drain(std::true_type{});
+    else
+      drain(std::false_type{});
   }
 
   ptx::tc_fence_before();

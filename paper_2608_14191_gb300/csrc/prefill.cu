@@ -38,7 +38,7 @@ struct PrefillArgs {
   const ChanEnc* enc;        // plan: [S][128] (offsets 2^(b-1))
   const StreamLayout* lay;   // plan: [S]
   const short* entry;        // plan: [S][n_entries]
-  const short* chan_ent;     // plan: [S][128][8]
+  const short* chan_ent;     // plan: [S][128][kChanEnt]
   int layer, n_kv, n_q_heads, group, q_start, n_q, n_ctx, n_ctx_pad, n_tiles, n_words, n_entries;
   int* err;
 };
@@ -77,7 +77,7 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
     }
     rec[w][t] = x;                             // each thread reads back only its own column
   }
-  const short* ce = a.chan_ent + static_cast<size_t>(s) * D * 8;
+  const short* ce = a.chan_ent + static_cast<size_t>(s) * D * kChanEnt;
   const short* ent = a.entry + static_cast<size_t>(s) * a.n_entries;
   // values for the tensor-core kernel: per 128-token tile [channel][token]
   __half* dst_t = a.codes + cs * a.n_ctx_pad * D + static_cast<size_t>(tile) * TILE * D + t;
@@ -88,8 +88,8 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
     for (int i = 0; i < 2; ++i) {
       const int cc = c + i;
       uint32_t u = 0;
-      for (int k = 0; k < 8; ++k) {
-        const int e = ce[cc * 8 + k];
+      for (int k = 0; k < kChanEnt; ++k) {
+        const int e = ce[cc * kChanEnt + k];
         if (e < 0) break;
         uint32_t v;
         if (e < ly.n2) {
@@ -98,7 +98,7 @@ __global__ void __launch_bounds__(TILE) aatc_prefill_codes_kernel(const PrefillA
           const int e1 = e - ly.n2;
           v = (rec[ly.n2 / 16 + (e1 >> 5)][t] >> (e1 & 31)) & 1u;
         }
-        u |= v << ((ent[e] >> 8) & 7);
+        u |= v << ((ent[e] >> 8) & 15);
       }
       v2[i] = static_cast<float>(u) - a.enc[s * D + cc].off;   // dropped channels: u = off = 0
     }

@@ -72,8 +72,13 @@ def test_plan_create_validates_before_any_cuda_call(aatc):
     nan_basis[0, 3, 3] = np.nan
     assert lib.aatc_plan_create(ctypes.byref(dm), nan_basis.ctypes.data, ok_bits.ctypes.data, scales.ctypes.data,
                                 None, ctypes.byref(h)) == 1
-    wide = aatc.dims(1, 1, 4, b_max=16)                                # planner-only widths
-    assert lib.aatc_plan_create(ctypes.byref(wide), basis.ctypes.data, ok_bits.ctypes.data, scales.ctypes.data,
+    over = aatc.dims(1, 1, 4, b_max=17)                                # above the paper's 16
+    assert lib.aatc_plan_create(ctypes.byref(over), basis.ctypes.data, ok_bits.ctypes.data, scales.ctypes.data,
+                                None, ctypes.byref(h)) == 1
+    wide = aatc.dims(1, 1, 4, b_max=16)
+    many_wide = np.full((2, 128), 2, np.uint8)
+    many_wide[1, :33] = 9                                              # 33 channels above 8 bits
+    assert lib.aatc_plan_create(ctypes.byref(wide), basis.ctypes.data, many_wide.ctypes.data, scales.ctypes.data,
                                 None, ctypes.byref(h)) == 5
     assert lib.aatc_plan_destroy(None) == 0
     # a plan handle without the live magic is rejected (use after destroy / garbage handle)
