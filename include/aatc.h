@@ -118,8 +118,7 @@ aatc_status_t aatc_calibrate(const aatc_dims_t* dims, const float* calib_k, cons
  * Errors: AATC_ERR_INVALID_ARG (g_h outside 1..8, group < 1, n_calib < 2, null outputs, b_max
  * outside 1..AATC_MAX_PLAN_BITS), AATC_ERR_BUDGET (avg_bits * d not an integer in [0, b_max d]).
  * Host only.
- * The plan, encode and decode kernels take per-kv-head streams; head-group streams are planned
- * here and checked against the oracle, and their device path is not built yet.
+ * aatc_group_plan_create builds the device plan from these outputs.
  */
 aatc_status_t aatc_calibrate_head_group(int32_t g_h, int32_t group, const float* calib, int32_t n_calib,
                                         const float* calib_q, int32_t n_calib_q, double avg_bits, int32_t b_max,
@@ -221,6 +220,34 @@ aatc_status_t aatc_plan_load(const char* path, const aatc_dims_t* dims, float* b
  */
 aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
                                const float* scales, void* stream, aatc_plan_t* plan_out);
+
+/*
+ * Build a device plan whose streams are head groups (Sec. 5 Step 1, remark on multi-head
+ * attention: the g_h kv-heads of a group share one transform; the paper's Llama setting has two
+ * groups of four).  Inputs in the layouts aatc_calibrate_head_group writes, one group stream per
+ * (layer, group, K|V), n = 128 g_h:
+ *   basis  : host fp32 [L][H_kv / g_h][2][n][n] (dim x channel, channels in storage order)
+ *   bits   : host uint8 [L][H_kv / g_h][2][n] non-increasing, each <= dims->b_max
+ *   scales : host fp32 [L][H_kv / g_h][2][n]
+ * A group stream is kept as g_h slice streams in the plan's and the cache's per-kv-head slots:
+ * slot (layer, g g_h + s, kind) holds the group's storage channels s, s + g_h, s + 2 g_h, ...
+ * (so every slice keeps non-increasing widths), and one alpha per token (the maximum over all n
+ * channels, Sec. 5) is written to every slice's slot.  The cache size is the per-kv-head one for
+ * the record length W of the widest slice.  aatc_encode and aatc_decode_attention (and
+ * aatc_decode_workspace_bytes, aatc_cache_bytes, aatc_dequantize of the slices) take such a
+ * plan: the encode projects the concatenated kv-heads of a group, h = [k_g g_h, ..., k_(g+1) g_h - 1] U,
+ * and query head j (kv-head j / group of its group) is embedded at its kv-head's 128-dim block:
+ * score (U_K^T q~) . h_hat / sqrt(128), output the block's rows of U_V (sum_t p_t h_hat^V_t).
+ * Other entry points (prefill, the sink / window decode, the no-allocation decode, the
+ * hidden-state encode) answer AATC_ERR_UNSUPPORTED for a group plan.
+ * Errors: AATC_ERR_INVALID_ARG (null, invalid dims, g_h outside 2..8 or not dividing H_kv, bits
+ * above b_max or increasing, scale <= 0 or non-finite where bits > 0, non-finite basis),
+ * AATC_ERR_UNSUPPORTED (b_max > 8, g_h other than 2 or 4 -- the encode holds all 128 g_h channels
+ * of a token tile in the 512 TMEM columns -- or more than 16 query heads per group stream),
+ * AATC_ERR_CUDA, AATC_ERR_NOMEM.  All argument checks run before any CUDA call.
+ */
+aatc_status_t aatc_group_plan_create(const aatc_dims_t* dims, int32_t g_h, const float* basis, const uint8_t* bits,
+                                     const float* scales, void* stream, aatc_plan_t* plan_out);
 
 /* Free the plan and its device tables (synchronizes the device).  NULL is a no-op. */
 aatc_status_t aatc_plan_destroy(aatc_plan_t plan);

@@ -61,6 +61,7 @@ SIGNATURES = {
     "aatc_decode_attention_sw": (_I32, [_P, _I32, _P, _P, _I32, _I32, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _SZ,
                                         _P]),
     "aatc_plan_create": (_I32, [ctypes.POINTER(Dims), _P, _P, _P, _P, ctypes.POINTER(_P)]),
+    "aatc_group_plan_create": (_I32, [_P, _I32, _P, _P, _P, _P, _P]),
     "aatc_plan_destroy": (_I32, [_P]),
     "aatc_plan_info": (_I32, [_P, ctypes.POINTER(_I32), _P]),
     "aatc_cache_bytes": (_I32, [_P, _I32, _I32, ctypes.POINTER(_SZ)]),
@@ -333,6 +334,8 @@ class Plan:
     def group(self) -> int:
         return self.dims.n_q_heads // self.dims.n_kv_heads
 
+    group_heads = 1
+
     def cache_bytes(self, batch: int, max_tokens: int) -> int:
         key = (int(batch), int(max_tokens))
         memo = self.__dict__.setdefault("_cache_bytes", {})
@@ -367,6 +370,35 @@ class Plan:
             self.close()
         except Exception:
             pass
+
+
+class GroupPlan(Plan):
+    """Head-group device plan (aatc_group_plan_create): one transform per group of g_h kv-heads.
+    basis fp32 [L][H_kv / g_h][2][n][n], bits uint8 [L][H_kv / g_h][2][n], scales fp32 of the
+    same shape, n = 128 g_h (aatc_calibrate_head_group's outputs per group stream)."""
+
+    def __init__(self, dm: Dims, g_h: int, basis: np.ndarray, bits: np.ndarray, scales: np.ndarray, stream=None):
+        lib = load()
+        self.dims = dm
+        self.group_heads = int(g_h)
+        n = HEAD_DIM * self.group_heads
+        ng = dm.n_kv_heads // max(1, self.group_heads)
+        self._basis = np.ascontiguousarray(basis, dtype=np.float32)
+        self._bits = np.ascontiguousarray(bits, dtype=np.uint8)
+        self._scales = np.ascontiguousarray(scales, dtype=np.float32)
+        if (self._basis.shape != (dm.n_layers, ng, 2, n, n) or self._bits.shape != (dm.n_layers, ng, 2, n)
+                or self._scales.shape != (dm.n_layers, ng, 2, n)):
+            raise ValueError("group plan arrays must be [L][H_kv/g_h][2][n][n], [L][H_kv/g_h][2][n] (n = 128 g_h)")
+        h = ctypes.c_void_p()
+        st = lib.aatc_group_plan_create(ctypes.byref(dm), self.group_heads, _ptr(self._basis), _ptr(self._bits),
+                                        _ptr(self._scales), _stream(stream), ctypes.byref(h))
+        _check(st, "aatc_group_plan_create")
+        self.handle = h.value
+        w = _I32()
+        ret = np.empty((dm.n_layers, dm.n_kv_heads, 2), np.int32)
+        _check(lib.aatc_plan_info(self.handle, ctypes.byref(w), _ptr(ret)), "aatc_plan_info")
+        self.n_words = w.value
+        self.retained = ret
 
 
 def encode(plan: Plan, layer: int, K, V, cache, start: int, max_tokens: int, stream=None):

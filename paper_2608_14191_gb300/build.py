@@ -15,7 +15,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libaatc.so")
-SOURCES = ["planner.cpp", "planfile.cpp", "capi.cpp", "encode.cu", "decode.cu", "prefill.cu", "selftest.cu"]
+SOURCES = ["planner.cpp", "planfile.cpp", "capi.cpp", "encode.cu", "decode.cu", "prefill.cu", "group.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

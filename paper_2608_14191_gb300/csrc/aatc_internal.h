@@ -69,6 +69,20 @@ struct PlanDevice {
   int* err;               // [4] sticky device flags
 };
 
+// Head-group plans (one transform over the n = 128 g_h channels of g_h kv-heads, Sec. 5 Step 1):
+// a group stream is kept as g_h slice streams in the per-kv-head slots (layer, g g_h + s, K|V) of
+// the plan tables and of the cache; slice s holds the group's storage-order channels s, s + g_h,
+// s + 2 g_h, ... (widths stay non-increasing in every slice) and all slices of a token share one
+// alpha, written to every slice's slot.  Group tables, channels in slice-major order
+// (j' = 128 s + c for storage channel j = c g_h + s):
+struct GroupDevice {
+  const void* ubf;        // bf16 [L][n_groups][2][n channel][n dim]   encode operand (K-major)
+  const float* uk;        // fp32 [L][n_groups][n dim][n channel]      key rotation U_K
+  const float* uvt;       // fp32 [L][n_groups][n channel][n dim]      value transform U_V, transposed
+};
+constexpr int MAX_GROUP_HEADS = 8;      // kv-heads per head group
+constexpr int MAX_GROUP_QUERIES = 16;   // query heads per head-group stream (the decode's M tile)
+
 struct Plan {
   uint32_t magic = PLAN_MAGIC;
   aatc_dims_t dims{};
@@ -86,6 +100,9 @@ struct Plan {
   size_t block_bytes = 0;
   alignas(64) unsigned char tmap_u[128];   // CUtensorMap over ubf16_t (2D: 128 dims x S*128 rows)
   bool tmap_ok = false;
+  int group_heads = 1;    // g_h: 1 for per-kv-head plans
+  GroupDevice gdev{};
+  alignas(64) unsigned char tmap_g[128];   // group plans: CUtensorMap over gdev.ubf (n dims x rows)
 };
 
 // Shape check shared by the planner (widths up to AATC_MAX_PLAN_BITS) and plan creation, which
@@ -183,10 +200,21 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
                           const DecodeExtra& extra);
 // Prefill attention: codes workspace bytes, and the two launches (codes, attention).
 size_t prefill_workspace(int batch, int n_kv, int n_ctx);
+// The codes launch alone: the signed codes of every slot of `layer` for tokens [0, n_ctx) as f16
+// in the prefill workspace layout ([b][slot][K|V][n_ctx_pad][128], value tiles transposed).
+cudaError_t launch_codes(const Plan& plan, int layer, const void* cache, int batch, int n_ctx, int max_tokens,
+                         void* ws, cudaStream_t st);
 cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_start, int n_q, const void* cache,
                            int batch, int n_ctx, int max_tokens, float* out, void* ws, cudaStream_t st);
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n,
                            int max_tokens, float* out, cudaStream_t st);
+// Head-group plans (group.cu): encode of every group stream of a layer; decode workspace and
+// launches (codes of the slices, folded queries, split attention, merge).
+cudaError_t launch_group_encode(const Plan& plan, int layer, const void* K, const void* V, int batch, int start,
+                                int n_tokens, void* cache, int max_tokens, cudaStream_t st);
+size_t group_decode_workspace(const Plan& plan, int batch, int n_ctx);
+cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, const void* cache, int batch, int n_ctx,
+                                int max_tokens, float* out, void* ws, cudaStream_t st);
 cudaError_t launch_bf16_decode(const void* K, const void* V, const void* q, int batch, int n_ctx,
                                int max_tokens, int n_kv, int n_q, float* out, void* ws,
                                const DecodeSplit& sp, cudaStream_t st);

@@ -191,10 +191,15 @@ int32_t aatc_last_cuda_error(void) { return g_last_cuda_error; }
 
 int32_t aatc_version(void) { return 200; }   // 0.2.0: plan files, AATC_ERR_IO, planner widths to 16
 
-aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
-                               const float* scales, void* stream, aatc_plan_t* plan_out) {
+namespace {
+
+// Device plan from per-slot widths and scales ([L][H_kv][2][128]).  Per-kv-head plans pass the
+// per-slot bases (g_h = 1); head-group plans pass g_h > 1, no per-slot basis, and the group bases
+// gbasis [L][H_kv / g_h][2][n][n] (dim x storage channel, n = 128 g_h) whose slices the slots hold.
+aatc_status_t create_plan(const aatc_dims_t* dims, const float* basis, const uint8_t* bits, const float* scales,
+                          int g_h, const float* gbasis, void* stream, aatc_plan_t* plan_out) {
   using namespace aatc;
-  if (!valid_dims(dims) || !basis || !bits || !scales || !plan_out) return AATC_ERR_INVALID_ARG;
+  if (!valid_dims(dims) || (!basis && !gbasis) || !bits || !scales || !plan_out) return AATC_ERR_INVALID_ARG;
   if (dims->b_max > AATC_MAX_BITS) return AATC_ERR_UNSUPPORTED;
   const int S = dims->n_layers * dims->n_kv_heads * 2;
   const size_t SD = static_cast<size_t>(S) * D;
@@ -217,8 +222,15 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
     retained[s] = r;
     nbits[s] = nb;
   }
-  for (size_t i = 0; i < SD * D; ++i)
-    if (!std::isfinite(basis[i])) return AATC_ERR_INVALID_ARG;
+  const int n_g = D * g_h, NG = dims->n_kv_heads / g_h;
+  const size_t GB = static_cast<size_t>(dims->n_layers) * NG * 2 * n_g * n_g;   // group basis elements
+  if (basis) {
+    for (size_t i = 0; i < SD * D; ++i)
+      if (!std::isfinite(basis[i])) return AATC_ERR_INVALID_ARG;
+  } else {
+    for (size_t i = 0; i < GB; ++i)
+      if (!std::isfinite(gbasis[i])) return AATC_ERR_INVALID_ARG;
+  }
   std::vector<StreamLayout> layout(S);
   std::vector<std::vector<short>> entries(S);
   int W = 1;
@@ -231,9 +243,14 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
 
   // host staging of every table, in one block
   size_t off = 0;
-  const size_t o_ubf = off;  off = align_up(off + SD * D * 2, 256);
-  const size_t o_u32 = off;  off = align_up(off + SD * D * 4, 256);
-  const size_t o_u32t = off; off = align_up(off + SD * D * 4, 256);
+  const size_t SDD = basis ? SD * D : 0;                            // per-slot basis tables
+  const size_t GBk = basis ? 0 : GB;                                // group tables
+  const size_t o_ubf = off;  off = align_up(off + SDD * 2, 256);
+  const size_t o_u32 = off;  off = align_up(off + SDD * 4, 256);
+  const size_t o_u32t = off; off = align_up(off + SDD * 4, 256);
+  const size_t o_gubf = off; off = align_up(off + GBk * 2, 256);
+  const size_t o_guk = off;  off = align_up(off + GBk / 2 * 4, 256);
+  const size_t o_guvt = off; off = align_up(off + GBk / 2 * 4, 256);
   const size_t o_enc = off;  off = align_up(off + SD * sizeof(ChanEnc), 256);
   const size_t o_invs = off; off = align_up(off + SD * 4, 256);
   const size_t o_f = off;    off = align_up(off + SD * 4, 256);
@@ -257,14 +274,39 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   auto* lay = reinterpret_cast<StreamLayout*>(host.data() + o_lay);
   auto* ent = reinterpret_cast<short*>(host.data() + o_ent);
   auto* che = reinterpret_cast<short*>(host.data() + o_che);
+  if (!basis) {
+    // group tables, channels in slice-major order: j' = 128 s + c holds storage channel c g_h + s
+    auto* gubf = reinterpret_cast<uint16_t*>(host.data() + o_gubf);
+    auto* guk = reinterpret_cast<float*>(host.data() + o_guk);
+    auto* guvt = reinterpret_cast<float*>(host.data() + o_guvt);
+    const size_t nn = static_cast<size_t>(n_g) * n_g;
+    for (int l = 0; l < dims->n_layers; ++l)
+      for (int g = 0; g < NG; ++g)
+        for (int kind = 0; kind < 2; ++kind) {
+          const size_t sg = (static_cast<size_t>(l) * NG + g) * 2 + kind;
+          const float* ub = gbasis + sg * nn;                       // [dim][storage channel]
+          for (int jp = 0; jp < n_g; ++jp) {
+            const int j = (jp % D) * g_h + jp / D;
+            for (int d = 0; d < n_g; ++d) {
+              const float v = ub[static_cast<size_t>(d) * n_g + j];
+              gubf[sg * nn + static_cast<size_t>(jp) * n_g + d] = f32_to_bf16_rne(v);
+              const size_t lg = (static_cast<size_t>(l) * NG + g) * nn;
+              if (kind == 0) guk[lg + static_cast<size_t>(d) * n_g + jp] = v;
+              else guvt[lg + static_cast<size_t>(jp) * n_g + d] = v;
+            }
+          }
+        }
+  }
   for (int s = 0; s < S; ++s) {
-    const float* bs = basis + static_cast<size_t>(s) * D * D;     // [dim][channel]
-    for (int d = 0; d < D; ++d)
-      for (int c = 0; c < D; ++c) {
-        ubf[(static_cast<size_t>(s) * D + c) * D + d] = f32_to_bf16_rne(bs[d * D + c]);
-        u32[(static_cast<size_t>(s) * D + d) * D + c] = bs[d * D + c];
-        u32t[(static_cast<size_t>(s) * D + c) * D + d] = bs[d * D + c];
-      }
+    if (basis) {
+      const float* bs = basis + static_cast<size_t>(s) * D * D;   // [dim][channel]
+      for (int d = 0; d < D; ++d)
+        for (int c = 0; c < D; ++c) {
+          ubf[(static_cast<size_t>(s) * D + c) * D + d] = f32_to_bf16_rne(bs[d * D + c]);
+          u32[(static_cast<size_t>(s) * D + d) * D + c] = bs[d * D + c];
+          u32t[(static_cast<size_t>(s) * D + c) * D + d] = bs[d * D + c];
+        }
+    }
     for (int c = 0; c < D; ++c) {
       const size_t i = static_cast<size_t>(s) * D + c;
       const int b = bits[i];
@@ -324,7 +366,20 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   plan->dev.entry = reinterpret_cast<const short*>(base + o_ent);
   plan->dev.chan_ent = reinterpret_cast<const short*>(base + o_che);
   plan->dev.err = reinterpret_cast<int*>(base + o_err);
-  if (e == cudaSuccess) e = encode_tensor_maps_u(*plan);
+  plan->group_heads = g_h;
+  if (basis) {
+    if (e == cudaSuccess) e = encode_tensor_maps_u(*plan);
+  } else {
+    plan->dev.ubf16_t = nullptr;
+    plan->dev.u32 = plan->dev.u32t = nullptr;
+    plan->gdev.ubf = base + o_gubf;
+    plan->gdev.uk = reinterpret_cast<const float*>(base + o_guk);
+    plan->gdev.uvt = reinterpret_cast<const float*>(base + o_guvt);
+    // rows of n_g dims, one per (layer, group, kind, slice-major channel); box 64 dims x 256 rows
+    if (e == cudaSuccess)
+      e = make_tensor_map_2d(plan->tmap_g, false, plan->gdev.ubf, static_cast<uint64_t>(n_g), GB / n_g,
+                             static_cast<uint64_t>(n_g) * 2, 64, 256);
+  }
   if (e != cudaSuccess) {
     cudaFree(plan->block);
     delete plan;
@@ -332,6 +387,45 @@ aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, cons
   }
   *plan_out = reinterpret_cast<aatc_plan_t>(plan);
   return AATC_OK;
+}
+
+}  // namespace
+
+aatc_status_t aatc_plan_create(const aatc_dims_t* dims, const float* basis, const uint8_t* bits,
+                               const float* scales, void* stream, aatc_plan_t* plan_out) {
+  if (!basis) return AATC_ERR_INVALID_ARG;
+  return create_plan(dims, basis, bits, scales, 1, nullptr, stream, plan_out);
+}
+
+aatc_status_t aatc_group_plan_create(const aatc_dims_t* dims, int32_t g_h, const float* basis, const uint8_t* bits,
+                                     const float* scales, void* stream, aatc_plan_t* plan_out) {
+  using namespace aatc;
+  if (!valid_dims(dims) || !basis || !bits || !scales || !plan_out || g_h < 2 || g_h > MAX_GROUP_HEADS ||
+      dims->n_kv_heads % g_h != 0)
+    return AATC_ERR_INVALID_ARG;
+  if (dims->b_max > 8 || (g_h != 2 && g_h != 4) || (dims->n_q_heads / dims->n_kv_heads) * g_h > MAX_GROUP_QUERIES)
+    return AATC_ERR_UNSUPPORTED;                    // TMEM holds the 128 g_h channels of a token tile: g_h <= 4
+  const int n = D * g_h, NG = dims->n_kv_heads / g_h, L = dims->n_layers;
+  // the slots' slices: slot (l, g g_h + s, kind) channel c = storage channel c g_h + s
+  const size_t S = static_cast<size_t>(L) * dims->n_kv_heads * 2;
+  std::vector<uint8_t> sb(S * D);
+  std::vector<float> ss(S * D);
+  for (int l = 0; l < L; ++l)
+    for (int g = 0; g < NG; ++g)
+      for (int kind = 0; kind < 2; ++kind) {
+        const size_t sg = (static_cast<size_t>(l) * NG + g) * 2 + kind;
+        const uint8_t* gb = bits + sg * n;
+        const float* gs = scales + sg * n;
+        for (int j = 0; j < n; ++j) {
+          if (gb[j] > dims->b_max || (j > 0 && gb[j] > gb[j - 1])) return AATC_ERR_INVALID_ARG;
+          if (gb[j] > 0 && !(std::isfinite(gs[j]) && gs[j] > 0.0f)) return AATC_ERR_INVALID_ARG;
+          const int sl = j % g_h, c = j / g_h;
+          const size_t slot = (static_cast<size_t>(l) * dims->n_kv_heads + g * g_h + sl) * 2 + kind;
+          sb[slot * D + c] = gb[j];
+          ss[slot * D + c] = gs[j];
+        }
+      }
+  return create_plan(dims, nullptr, sb.data(), ss.data(), g_h, basis, stream, plan_out);
 }
 
 aatc_status_t aatc_plan_destroy(aatc_plan_t p) {
@@ -372,6 +466,9 @@ aatc_status_t aatc_encode(aatc_plan_t p, int32_t layer, const void* K, const voi
   if (static_cast<int64_t>(start) + n_tokens > max_tokens) return AATC_ERR_CAPACITY;
   if (n_tokens == 0) return AATC_OK;                   // an empty append reads no pointer
   if (!K || !V || !cache || !aligned16(K) || !aligned16(V) || !aligned16(cache)) return AATC_ERR_INVALID_ARG;
+  if (plan->group_heads > 1)
+    return cuda_status(aatc::launch_group_encode(*plan, layer, K, V, batch, start, n_tokens, cache, max_tokens,
+                                                 static_cast<cudaStream_t>(stream)));
   return cuda_status(aatc::launch_encode(*plan, layer, K, V, batch, start, n_tokens, cache,
                                          max_tokens, static_cast<cudaStream_t>(stream)));
 }
@@ -387,7 +484,7 @@ aatc_status_t aatc_encode_hidden(aatc_plan_t p, int32_t layer, const void* x, in
   if (n_tokens == 0) return AATC_OK;                   // an empty append reads no pointer
   if (!x || !a_hat || !cache || !aligned16(x) || !aligned16(a_hat) || !aligned16(cache))
     return AATC_ERR_INVALID_ARG;
-  if (plan->max_bits > 8) return AATC_ERR_UNSUPPORTED;   // this epilogue packs one byte per stored value
+  if (plan->max_bits > 8 || plan->group_heads > 1) return AATC_ERR_UNSUPPORTED;   // one byte per stored value; per-kv-head slots
   return cuda_status(aatc::launch_encode_hidden(*plan, layer, x, d_model, a_hat, batch, start, n_tokens, cache,
                                                 max_tokens, static_cast<cudaStream_t>(stream)));
 }
@@ -411,6 +508,7 @@ aatc_status_t aatc_prefill_attention(aatc_plan_t p, int32_t layer, const void* q
   if (!aligned16(q) || !aligned16(cache) || !aligned16(out) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
   if (plan->n_words > 32) return AATC_ERR_UNSUPPORTED;
   if (plan->max_bits > 12) return AATC_ERR_UNSUPPORTED;   // f16 code operands are exact up to |code| = 2048
+  if (plan->group_heads > 1) return AATC_ERR_UNSUPPORTED;
   if (workspace_bytes < aatc::prefill_workspace(batch, plan->dims.n_kv_heads, n_ctx)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_prefill(*plan, layer, q, q_start, n_q, cache, batch, n_ctx, max_tokens, out,
                                           workspace, static_cast<cudaStream_t>(stream)));
@@ -419,7 +517,8 @@ aatc_status_t aatc_prefill_attention(aatc_plan_t p, int32_t layer, const void* q
 aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t p, int32_t batch, int32_t n_ctx, size_t* bytes) {
   aatc::Plan* plan = as_plan(p);
   if (!plan || !bytes || batch < 1 || n_ctx < 1) return AATC_ERR_INVALID_ARG;
-  *bytes = aatc::decode_workspace_for(*plan, batch, n_ctx);
+  *bytes = plan->group_heads > 1 ? aatc::group_decode_workspace(*plan, batch, n_ctx)
+                                 : aatc::decode_workspace_for(*plan, batch, n_ctx);
   return AATC_OK;
 }
 
@@ -433,6 +532,12 @@ aatc_status_t aatc_decode_attention(aatc_plan_t p, int32_t layer, const void* q,
   if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
   if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
   if (!aligned16(cache) || !aligned16(workspace)) return AATC_ERR_INVALID_ARG;
+  if (plan->group_heads > 1) {
+    if (!aligned16(q) || !aligned16(out)) return AATC_ERR_INVALID_ARG;
+    if (workspace_bytes < aatc::group_decode_workspace(*plan, batch, n_ctx)) return AATC_ERR_WORKSPACE;
+    return cuda_status(aatc::launch_group_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out, workspace,
+                                                 static_cast<cudaStream_t>(stream)));
+  }
   if (workspace_bytes < aatc::decode_workspace_for(*plan, batch, n_ctx)) return AATC_ERR_WORKSPACE;
   return cuda_status(aatc::launch_decode(*plan, layer, q, cache, batch, n_ctx, max_tokens, out,
                                          workspace, static_cast<cudaStream_t>(stream), aatc::DecodeExtra{}));
@@ -448,7 +553,8 @@ aatc_status_t aatc_decode_attention_sw(aatc_plan_t p, int32_t layer, const void*
       full_cap < n_full || (t_end == t_first && n_full == 0))
     return AATC_ERR_INVALID_ARG;
   if (t_end > max_tokens || n_full > aatc::MAX_FULL_TOKENS) return AATC_ERR_CAPACITY;
-  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > aatc::MAX_GROUP || plan->group_heads > 1)
+    return AATC_ERR_UNSUPPORTED;
   if (!aligned16(cache) || (n_full > 0 && (!aligned16(k_full) || !aligned16(v_full)))) return AATC_ERR_INVALID_ARG;
   // the packed part covers tiles [t_first / 128, ceil(t_end / 128)): never more splits than a
   // plain decode of t_end tokens, so aatc_decode_workspace_bytes(batch, t_end) suffices

@@ -1893,7 +1893,7 @@ extern "C" aatc_status_t aatc_decode_attention_noalloc(aatc_plan_t p, int32_t la
       max_tokens < 1)
     return AATC_ERR_INVALID_ARG;
   if (n_ctx > max_tokens) return AATC_ERR_CAPACITY;
-  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP) return AATC_ERR_UNSUPPORTED;
+  if (plan->dims.n_q_heads / plan->dims.n_kv_heads > MAX_GROUP || plan->group_heads > 1) return AATC_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(cache) & 15u) != 0) return AATC_ERR_INVALID_ARG;
   if (decode_workspace_for(*plan, batch, n_ctx) > AATC_NOALLOC_SCRATCH_BYTES) return AATC_ERR_WORKSPACE;
   int dev = 0;

@@ -240,91 +240,141 @@ struct QuantTables {      // per channel, structure of arrays (16-byte aligned)
   const float* magic;     // 1.5 2^23 + 2^(b_c - 1)
 };
 
+// alpha pass over 32 channels (TMEM columns 32 j ..): running maxima of |h_c| / s_c, two per
+// instruction (inv_s = 0 for dropped channels).
+__device__ __forceinline__ void amax_chunk_regs(const uint32_t (&r)[32], int j, const float* inv_s, float& am0,
+                                                float& am1) {
+#pragma unroll
+  for (int i = 0; i < 32; i += 4) {
+    const float4 is = ptx::lds_f4(&inv_s[32 * j + i]);
+    float a0, a1, a2, a3;
+    ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), ptx::f2_pack(is.x, is.y)),
+                   a0, a1);
+    ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])), ptx::f2_pack(is.z, is.w)),
+                   a2, a3);
+    am0 = ptx::fmax3(am0, fabsf(a0), fabsf(a1));
+    am1 = ptx::fmax3(am1, fabsf(a2), fabsf(a3));
+  }
+}
+// quantize pass over 32 channels: x = h / Delta + 1/2 = h (ia / f_c) + 1/2, clamped above, then
+// the round-down add of 1.5 2^23 + 2^(b-1) leaves u (< 2^16) in the low two bytes of the float;
+// U gets the low bytes of channels 32 j .., UH (kWide, j = 0 only) the high bytes.
+template <bool kWide>
+__device__ __forceinline__ void quant_chunk_regs(const uint32_t (&r)[32], int j, const QuantTables& tb, uint64_t ia2,
+                                                 uint32_t (&U)[32], uint32_t (&UH)[8]) {
+  const uint64_t half2 = ptx::f2_pack(0.5f, 0.5f);
+#pragma unroll
+  for (int i = 0; i < 32; i += 4) {
+    const float4 f = ptx::lds_f4(&tb.inv_f[32 * j + i]);
+    const float4 h = ptx::lds_f4(&tb.hi[32 * j + i]);
+    const float4 m = ptx::lds_f4(&tb.magic[32 * j + i]);
+    float x0, x1, x2, x3;
+    ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
+                               ptx::f2_mul(ptx::f2_pack(f.x, f.y), ia2), half2), x0, x1);
+    ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])),
+                               ptx::f2_mul(ptx::f2_pack(f.z, f.w), ia2), half2), x2, x3);
+    float y0, y1, y2, y3;
+    ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x0, h.x), fminf(x1, h.y)), ptx::f2_pack(m.x, m.y)), y0, y1);
+    ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x2, h.z), fminf(x3, h.w)), ptx::f2_pack(m.z, m.w)), y2, y3);
+    U[8 * j + i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0040),
+                                   __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0040), 0x5410);
+    if (kWide && j == 0)
+      UH[i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0051),
+                              __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0051), 0x5410);
+  }
+}
+
 // Token scale and stored values of one token (thread = token = TMEM lane), as quantize_token
 // but two channels per fp32 instruction and the stored values kept in registers: U[w] holds the
 // low bytes of u_c for channels 4w .. 4w + 3, UH[w] the high bytes (u_c >= 256 only for widths
 // above 8, which lie in the first 32 channels).  The arithmetic (and so every code) is the same.
+// Eight 32-column TMEM loads (four per pass), each issued before the previous chunk is processed
+// so its latency overlaps that work.
 template <bool kWide>
 __device__ __forceinline__ float quantize_token_regs(uint32_t taddr, const QuantTables& tb, uint32_t (&U)[32],
                                                      uint32_t (&UH)[8]) {
   uint32_t ra[32], rb[32];
   float am0 = 0.0f, am1 = 0.0f;
-  auto amax_chunk = [&](const uint32_t (&r)[32], int j) {
-#pragma unroll
-    for (int i = 0; i < 32; i += 4) {
-      const float4 is = ptx::lds_f4(&tb.inv_s[32 * j + i]);
-      float a0, a1, a2, a3;
-      ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
-                                 ptx::f2_pack(is.x, is.y)), a0, a1);
-      ptx::f2_unpack(ptx::f2_mul(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])),
-                                 ptx::f2_pack(is.z, is.w)), a2, a3);
-      am0 = ptx::fmax3(am0, fabsf(a0), fabsf(a1));
-      am1 = ptx::fmax3(am1, fabsf(a2), fabsf(a3));
-    }
-  };
-  uint64_t ia2 = 0;
-  const uint64_t half2 = ptx::f2_pack(0.5f, 0.5f);
-  // x = h / Delta + 1/2 = h (ia / f_c) + 1/2, clamped above, then the round-down add of
-  // 1.5 2^23 + 2^(b-1) leaves u (< 2^16) in the low two bytes of the float.
-  auto quant_chunk = [&](const uint32_t (&r)[32], int j) {
-#pragma unroll
-    for (int i = 0; i < 32; i += 4) {
-      const float4 f = ptx::lds_f4(&tb.inv_f[32 * j + i]);
-      const float4 h = ptx::lds_f4(&tb.hi[32 * j + i]);
-      const float4 m = ptx::lds_f4(&tb.magic[32 * j + i]);
-      float x0, x1, x2, x3;
-      ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i]), __uint_as_float(r[i + 1])),
-                                 ptx::f2_mul(ptx::f2_pack(f.x, f.y), ia2), half2), x0, x1);
-      ptx::f2_unpack(ptx::f2_fma(ptx::f2_pack(__uint_as_float(r[i + 2]), __uint_as_float(r[i + 3])),
-                                 ptx::f2_mul(ptx::f2_pack(f.z, f.w), ia2), half2), x2, x3);
-      float y0, y1, y2, y3;
-      ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x0, h.x), fminf(x1, h.y)), ptx::f2_pack(m.x, m.y)), y0, y1);
-      ptx::f2_unpack(ptx::f2_add_rd(ptx::f2_pack(fminf(x2, h.z), fminf(x3, h.w)), ptx::f2_pack(m.z, m.w)), y2, y3);
-      U[8 * j + i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0040),
-                                     __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0040), 0x5410);
-      if (kWide && j == 0)
-        UH[i / 4] = __byte_perm(__byte_perm(__float_as_uint(y0), __float_as_uint(y1), 0x0051),
-                                __byte_perm(__float_as_uint(y2), __float_as_uint(y3), 0x0051), 0x5410);
-    }
-  };
-  // Eight 32-column TMEM loads (four per pass), each issued before the previous chunk is
-  // processed so its latency overlaps that work.
   ptx::tmem_ld_32raw(taddr, ra);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(ra);
   ptx::tmem_ld_32raw(taddr + 32, rb);
-  amax_chunk(ra, 0);
+  amax_chunk_regs(ra, 0, tb.inv_s, am0, am1);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(rb);
   ptx::tmem_ld_32raw(taddr + 64, ra);
-  amax_chunk(rb, 1);
+  amax_chunk_regs(rb, 1, tb.inv_s, am0, am1);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(ra);
   ptx::tmem_ld_32raw(taddr + 96, rb);
-  amax_chunk(ra, 2);
+  amax_chunk_regs(ra, 2, tb.inv_s, am0, am1);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(rb);
   ptx::tmem_ld_32raw(taddr, ra);
-  amax_chunk(rb, 3);
+  amax_chunk_regs(rb, 3, tb.inv_s, am0, am1);
   const float amax = fmaxf(am0, am1);
   const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
-  ia2 = ptx::f2_pack(ia, ia);
+  const uint64_t ia2 = ptx::f2_pack(ia, ia);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(ra);
   ptx::tmem_ld_32raw(taddr + 32, rb);
-  quant_chunk(ra, 0);
+  quant_chunk_regs<kWide>(ra, 0, tb, ia2, U, UH);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(rb);
   ptx::tmem_ld_32raw(taddr + 64, ra);
-  quant_chunk(rb, 1);
+  quant_chunk_regs<kWide>(rb, 1, tb, ia2, U, UH);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(ra);
   ptx::tmem_ld_32raw(taddr + 96, rb);
-  quant_chunk(ra, 2);
+  quant_chunk_regs<kWide>(ra, 2, tb, ia2, U, UH);
   ptx::tmem_ld_wait();
   ptx::tmem_regs_ready(rb);
-  quant_chunk(rb, 3);
+  quant_chunk_regs<kWide>(rb, 3, tb, ia2, U, UH);
   return amax;
+}
+
+// The two passes separately, for head-group streams whose alpha spans several slices: the
+// slice's maximum of |h_c| / s_c, then its stored values for a given 1 / alpha.
+__device__ __forceinline__ float token_amax_regs(uint32_t taddr, const float* inv_s) {
+  uint32_t ra[32], rb[32];
+  float am0 = 0.0f, am1 = 0.0f;
+  ptx::tmem_ld_32raw(taddr, ra);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  amax_chunk_regs(ra, 0, inv_s, am0, am1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  amax_chunk_regs(rb, 1, inv_s, am0, am1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  amax_chunk_regs(ra, 2, inv_s, am0, am1);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  amax_chunk_regs(rb, 3, inv_s, am0, am1);
+  return fmaxf(am0, am1);
+}
+__device__ __forceinline__ void token_quant_regs(uint32_t taddr, const QuantTables& tb, float ia, uint32_t (&U)[32]) {
+  uint32_t ra[32], rb[32], uh[8];
+  const uint64_t ia2 = ptx::f2_pack(ia, ia);
+  ptx::tmem_ld_32raw(taddr, ra);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 32, rb);
+  quant_chunk_regs<false>(ra, 0, tb, ia2, U, uh);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  ptx::tmem_ld_32raw(taddr + 64, ra);
+  quant_chunk_regs<false>(rb, 1, tb, ia2, U, uh);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(ra);
+  ptx::tmem_ld_32raw(taddr + 96, rb);
+  quant_chunk_regs<false>(ra, 2, tb, ia2, U, uh);
+  ptx::tmem_ld_wait();
+  ptx::tmem_regs_ready(rb);
+  quant_chunk_regs<false>(rb, 3, tb, ia2, U, uh);
 }
 
 // Base-4 digit k of the 16 channels held in w0 .. w3, channel order LSB first: the mask-and-
@@ -630,6 +680,217 @@ __global__ void __launch_bounds__(kKThreads, 1)
   if (warp == kKMmaWarp) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ head-group streams
+// A head-group stream (Sec. 5 Step 1: the g_h kv-heads of a group share one transform) projects
+// the concatenated kv-heads of a group, n = 128 g_h input dims, onto n channels, held as g_h
+// slice streams (slice s = storage channels s, s + g_h, ...; slice-major operand rows).  One
+// persistent CTA per (group, kind, slice of 128-token items); all n channels of an item sit in
+// TMEM at once (n <= 512 columns), so alpha, the maximum over all of them, is known before any
+// slice is quantized.  Warp roles:
+//   warp 8    : TMA producer -- per 64-dim block of the input: the 128 x 64 x tile of the group's
+//               kv-heads and the n x 64 operand tile, into a 2-stage SW128 ring,
+//   warp 9    : MMA issuer   -- tcgen05.mma M=128 tokens, N=256, K=16, n / 256 per k-step, into
+//               the n-column accumulator,
+//   warps 0-7 : two epilogue warpgroups, thread = token; warpgroup e owns slices e g_h / 2 ..:
+//               their maxima meet through shared memory (an mbarrier round), then each slice is
+//               quantized, the accumulator released, and the slice records packed
+//               (register-resident, as aatc_encode_kernel, widths up to 8).
+constexpr int kGStages = 2;
+constexpr int kGXBytes = TILE * 64 * 2;            // 16 KB: 128 tokens x 64 dims
+constexpr int kGEpiThreads = 256;
+constexpr int kGProducerWarp = kGEpiThreads / 32;
+constexpr int kGMmaWarp = kGProducerWarp + 1;
+constexpr int kGThreads = kGEpiThreads + 64;
+
+struct GroupEncodeArgs {
+  const ChanEnc* enc;
+  const float* inv_s;
+  const StreamLayout* lay;
+  int* err;
+  uint32_t* words;
+  float* alpha;
+  int layer, n_kv, gh, n_groups, batch, start, n_tokens, n_chunks, n_words, n_tiles, ctas_per_basis;
+};
+
+template <int GH>
+struct GroupEncodeSmem {
+  static constexpr int N = D * GH;
+  alignas(1024) unsigned char x_tile[kGStages][kGXBytes];
+  alignas(1024) unsigned char u_tile[kGStages][N * 64 * 2];
+  alignas(16) float inv_s[GH][D];
+  alignas(16) float inv_f[GH][D];
+  alignas(16) float hi[GH][D];
+  alignas(16) float magic[GH][D];
+  StreamLayout lay[GH];
+  float xch[2][TILE];                              // per-warpgroup maxima of each token
+  uint64_t full[kGStages], empty[kGStages], tfull, tempty, xbar;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+template <int GH>
+__global__ void __launch_bounds__(kGThreads, 1)
+    aatc_encode_group_kernel(const __grid_constant__ CUtensorMap tmap_k, const __grid_constant__ CUtensorMap tmap_v,
+                             const __grid_constant__ CUtensorMap tmap_g, const GroupEncodeArgs a) {
+  constexpr int N = D * GH, NKB = N / 64, NH = N / 256, SPW = GH / 2;
+  constexpr uint32_t kUBytes = N * 64 * 2;
+  constexpr uint32_t kCols = N <= 256 ? 256 : 512;
+  extern __shared__ unsigned char smem_raw[];
+  auto& sm = *reinterpret_cast<GroupEncodeSmem<GH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int basis = blockIdx.x / a.ctas_per_basis;           // (group, kind) of the layer
+  const int sub = blockIdx.x % a.ctas_per_basis;
+  const int grp = basis >> 1, kind = basis & 1;
+  const long n_items = static_cast<long>(a.batch) * a.n_chunks;
+  const long it0 = n_items * sub / a.ctas_per_basis;
+  const int my_items = static_cast<int>(n_items * (sub + 1) / a.ctas_per_basis - it0);
+  const CUtensorMap* tmap_x = kind == 0 ? &tmap_k : &tmap_v;
+  const int row0 = ((a.layer * a.n_groups + grp) * 2 + kind) * N;   // operand rows of this stream
+
+  for (int i = tid; i < GH * D; i += kGThreads) {
+    const int sl = i / D, c = i % D;
+    const int slot = (a.layer * a.n_kv + grp * GH + sl) * 2 + kind;
+    const ChanEnc e = a.enc[slot * D + c];
+    sm.inv_s[sl][c] = a.inv_s[slot * D + c];
+    sm.inv_f[sl][c] = e.inv_f;
+    sm.hi[sl][c] = e.hi;
+    sm.magic[sl][c] = e.magic;
+  }
+  if (tid < GH) sm.lay[tid] = a.lay[(a.layer * a.n_kv + grp * GH + tid) * 2 + kind];
+  if (tid == 0) {
+    for (int st = 0; st < kGStages; ++st) {
+      ptx::mbar_init(&sm.full[st], 1);
+      ptx::mbar_init(&sm.empty[st], 1);
+    }
+    ptx::mbar_init(&sm.tfull, 1);
+    ptx::mbar_init(&sm.tempty, kGEpiThreads);
+    ptx::mbar_init(&sm.xbar, kGEpiThreads);
+    sm.abort_flag = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == kGMmaWarp) {
+    ptx::tmem_alloc(&sm.tmem_base, kCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  volatile int* abort_flag = &sm.abort_flag;
+
+  if (warp == kGProducerWarp) {
+    if (lane == 0 && my_items > 0) {
+      ptx::prefetch_tmap(tmap_x);
+      ptx::prefetch_tmap(&tmap_g);
+      bool ok = true;
+      for (int it = 0; ok && it < my_items; ++it) {
+        const long item = it0 + it;
+        const int b = static_cast<int>(item / a.n_chunks);
+        const int t0 = static_cast<int>(item % a.n_chunks) * TILE;
+        for (int kb = 0; kb < NKB; ++kb) {
+          const int u = it * NKB + kb, st = u % kGStages;
+          if (!ptx::mbar_wait_bounded(&sm.empty[st], ((u / kGStages) & 1) ^ 1, abort_flag)) {
+            raise_abort(sm, a.err);
+            ok = false;
+            break;
+          }
+          ptx::mbar_arrive_expect_tx(&sm.full[st], kGXBytes + kUBytes);
+          // the group's kv-heads are adjacent: dims grp N + 64 kb .. of the [n_kv 128]-wide rows
+          ptx::tma_load_3d(sm.x_tile[st], tmap_x, &sm.full[st], grp * N + kb * 64, t0, b);
+#pragma unroll
+          for (int h = 0; h < NH; ++h)
+            ptx::tma_load_2d(sm.u_tile[st] + h * (256 * 128), &tmap_g, &sm.full[st], kb * 64, row0 + h * 256);
+        }
+      }
+    }
+  } else if (warp == kGMmaWarp) {
+    if (lane == 0 && my_items > 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 256);
+      bool ok = true;
+      for (int it = 0; ok && it < my_items; ++it) {
+        if (!ptx::mbar_wait_bounded(&sm.tempty, (it & 1) ^ 1, abort_flag)) { raise_abort(sm, a.err); break; }
+        ptx::tc_fence_after();
+        for (int kb = 0; kb < NKB; ++kb) {
+          const int u = it * NKB + kb, st = u % kGStages;
+          if (!ptx::mbar_wait_bounded(&sm.full[st], (u / kGStages) & 1, abort_flag)) {
+            raise_abort(sm, a.err);
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          const uint32_t x_base = ptx::smem_u32(sm.x_tile[st]), u_base = ptx::smem_u32(sm.u_tile[st]);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+            for (int h = 0; h < NH; ++h)
+              ptx::umma_bf16(tmem + h * 256, ptx::sdesc_kmajor_sw128(x_base + kk * 32),
+                             ptx::sdesc_kmajor_sw128(u_base + h * (256 * 128) + kk * 32), idesc,
+                             (kb > 0 || kk > 0) ? 1u : 0u);
+          ptx::umma_commit(&sm.empty[st]);
+        }
+        if (ok) ptx::umma_commit(&sm.tfull);
+      }
+    }
+  } else {
+    const int eg = warp >> 2, quad = warp & 3, tl = quad * 32 + lane;
+    const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
+    const int t4 = lane & 3;
+    const uint32_t s1 = (t4 & 1) ? 0x3715u : 0x6240u, s2 = (t4 & 2) ? 0x3276u : 0x5410u;
+    const int qpos = ((t4 & 1) << 1) | (t4 >> 1);
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    uint32_t uh[8];
+#pragma unroll 1
+    for (int it = 0; it < my_items; ++it) {
+      if (!ptx::mbar_wait_bounded(&sm.tfull, it & 1, abort_flag)) { raise_abort(sm, a.err); break; }
+      ptx::tc_fence_after();
+      float pm = 0.0f;
+#pragma unroll
+      for (int k = 0; k < SPW; ++k) {
+        const int sl = eg * SPW + k;
+        pm = fmaxf(pm, token_amax_regs(lane_base + sl * D, sm.inv_s[sl]));
+      }
+      sm.xch[eg][tl] = pm;
+      ptx::mbar_arrive(&sm.xbar);                              // (a bounded wait, unlike a named barrier)
+      if (!ptx::mbar_wait_bounded(&sm.xbar, it & 1, abort_flag)) { raise_abort(sm, a.err); break; }
+      const float amax = fmaxf(sm.xch[0][tl], sm.xch[1][tl]);
+      const float ia = amax > 0.0f ? 1.0f / amax : 0.0f;
+      uint32_t U[SPW][32];
+#pragma unroll
+      for (int k = 0; k < SPW; ++k) {
+        const int sl = eg * SPW + k;
+        token_quant_regs(lane_base + sl * D, QuantTables{sm.inv_s[sl], sm.inv_f[sl], sm.hi[sl], sm.magic[sl]}, ia,
+                         U[k]);
+      }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&sm.tempty);
+
+      const long item = it0 + it;
+      const int b = static_cast<int>(item / a.n_chunks);
+      const int i = static_cast<int>(item % a.n_chunks) * TILE + tl;
+      const bool ok = i < a.n_tokens;
+      if (!__any_sync(0xffffffffu, ok)) continue;
+      const int pos_t = a.start + i;
+      if (ok && !isfinite(amax)) atomicOr(a.err, 1);
+#pragma unroll
+      for (int k = 0; k < SPW; ++k) {
+        const int sl = eg * SPW + k;
+        const size_t sidx = (static_cast<size_t>(b) * a.n_kv + grp * GH + sl) * 2 + kind;
+        if (ok) a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
+        RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
+                      pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
+        pack_token_regs<false>(sm.lay[sl], U[k], uh, f, a.n_words);
+      }
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == kGMmaWarp) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kCols);
   }
 }
 
@@ -944,6 +1205,64 @@ cudaError_t launch_encode_hidden(const Plan& plan, int layer, const void* x, int
   cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_hidden_kernel), smem);
   if (e != cudaSuccess) return e;
   aatc_encode_hidden_kernel<<<static_cast<unsigned>(per_head * a.n_kv), kThreads, smem, st>>>(mx, ma, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_encode(const Plan& plan, int layer, const void* K, const void* V, int batch, int start,
+                                int n_tokens, void* cache, int max_tokens, cudaStream_t st) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return cudaErrorNotSupported;
+  const int gh = plan.group_heads, n_kv = plan.dims.n_kv_heads;
+  if (gh != 2 && gh != 4) return cudaErrorNotSupported;
+  CUtensorMap mk, mv;
+  // K or V as bf16 [batch][n_tokens][n_kv * 128]: box 64 dims x 128 tokens x 1 sequence
+  for (int kind = 0; kind < 2; ++kind) {
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(n_kv) * D, static_cast<cuuint64_t>(n_tokens),
+                                static_cast<cuuint64_t>(batch)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(n_kv) * D * 2,
+                                   static_cast<cuuint64_t>(n_tokens) * n_kv * D * 2};
+    const cuuint32_t box[3] = {64, TILE, 1};
+    const cuuint32_t es[3] = {1, 1, 1};
+    if (enc(kind == 0 ? &mk : &mv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(kind == 0 ? K : V), dims,
+            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  const CacheGeom g = cache_geom(batch, n_kv, max_tokens, plan.n_words);
+  GroupEncodeArgs a;
+  a.enc = plan.dev.enc;
+  a.inv_s = plan.dev.inv_s;
+  a.lay = plan.dev.lay;
+  a.err = plan.dev.err;
+  a.words = static_cast<uint32_t*>(cache);
+  a.alpha = reinterpret_cast<float*>(static_cast<uint32_t*>(cache) + g.words_elems);
+  a.layer = layer;
+  a.n_kv = n_kv;
+  a.gh = gh;
+  a.n_groups = n_kv / gh;
+  a.batch = batch;
+  a.start = start;
+  a.n_tokens = n_tokens;
+  a.n_chunks = (n_tokens + TILE - 1) / TILE;
+  a.n_words = plan.n_words;
+  a.n_tiles = g.n_tiles;
+  const int n_basis = 2 * a.n_groups;
+  const long items = static_cast<long>(batch) * a.n_chunks;
+  long k = std::max(1, plan.num_sms / n_basis);
+  a.ctas_per_basis = static_cast<int>(std::min(k, items));
+  const auto* mg = reinterpret_cast<const CUtensorMap*>(plan.tmap_g);
+  const unsigned grid = static_cast<unsigned>(n_basis * a.ctas_per_basis);
+  if (gh == 2) {
+    const size_t smem = sizeof(GroupEncodeSmem<2>) + 1024;
+    cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_group_kernel<2>), smem);
+    if (e != cudaSuccess) return e;
+    aatc_encode_group_kernel<2><<<grid, kGThreads, smem, st>>>(mk, mv, *mg, a);
+  } else {
+    const size_t smem = sizeof(GroupEncodeSmem<4>) + 1024;
+    cudaError_t e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_encode_group_kernel<4>), smem);
+    if (e != cudaSuccess) return e;
+    aatc_encode_group_kernel<4><<<grid, kGThreads, smem, st>>>(mk, mv, *mg, a);
+  }
   return cudaGetLastError();
 }
 

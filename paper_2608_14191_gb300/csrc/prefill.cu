@@ -586,6 +586,31 @@ size_t prefill_workspace(int batch, int n_kv, int n_ctx) {
   return static_cast<size_t>(batch) * n_kv * 2 * pad * D * sizeof(__half);
 }
 
+cudaError_t launch_codes(const Plan& plan, int layer, const void* cache, int batch, int n_ctx, int max_tokens,
+                         void* ws, cudaStream_t st) {
+  const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
+  PrefillArgs a{};
+  a.words = static_cast<const uint32_t*>(cache);
+  a.alpha = reinterpret_cast<const float*>(static_cast<const uint32_t*>(cache) + g.words_elems);
+  a.codes = static_cast<__half*>(ws);
+  a.f = plan.dev.f;
+  a.enc = plan.dev.enc;
+  a.lay = plan.dev.lay;
+  a.entry = plan.dev.entry;
+  a.chan_ent = plan.dev.chan_ent;
+  a.layer = layer;
+  a.n_kv = plan.dims.n_kv_heads;
+  a.n_ctx = n_ctx;
+  a.n_ctx_pad = (n_ctx + TILE - 1) / TILE * TILE;
+  a.n_tiles = g.n_tiles;
+  a.n_words = plan.n_words;
+  a.n_entries = plan.n_entries;
+  a.err = plan.dev.err;
+  if (plan.n_words > 32) return cudaErrorNotSupported;
+  aatc_prefill_codes_kernel<<<dim3(a.n_ctx_pad / TILE, a.n_kv * 2, batch), TILE, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_prefill(const Plan& plan, int layer, const void* q, int q_start, int n_q, const void* cache,
                            int batch, int n_ctx, int max_tokens, float* out, void* ws, cudaStream_t st) {
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
