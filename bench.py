@@ -448,6 +448,105 @@ def qwen_timing(aatc, device, n_calls=64, reps=3, enc_iters=6, n_copies=4):
                       f"x {reps} over {n_copies} packed-cache copies"}
 
 
+def group_plan_for(aatc, cfg, g_h, avg_bits=2.75):
+    """Head-group plan of layer 0 of `cfg` from the host group planner (one call per (group,
+    kind) stream, run on host threads at once); returns (plan, seconds)."""
+    import concurrent.futures as cf
+    H, G = cfg.n_kv_heads, cfg.group
+    ng, n = H // g_h, 128 * g_h
+    ck, cv, cq = W.layer_calibration(cfg, 0)
+    jobs = []
+    for g in range(ng):
+        hk = slice(g * g_h, (g + 1) * g_h)
+        jobs.append((g, 0, ck[hk], cq[g * g_h * G:(g + 1) * g_h * G]))
+        jobs.append((g, 1, cv[hk], None))
+    basis = np.zeros((1, ng, 2, n, n), np.float32)
+    bits = np.zeros((1, ng, 2, n), np.uint8)
+    scales = np.ones((1, ng, 2, n), np.float32)
+    t0 = time.time()
+    with cf.ThreadPoolExecutor(max_workers=len(jobs)) as ex:
+        res = list(ex.map(lambda j: aatc.calibrate_head_group(j[2], j[3], avg_bits, group=G), jobs))
+    for (g, kind, _, _), p in zip(jobs, res):
+        basis[0, g, kind], bits[0, g, kind], scales[0, g, kind] = p["basis"], p["bits"], p["scales"]
+    plan = aatc.GroupPlan(aatc.dims(1, H, cfg.n_q_heads), g_h, basis, bits, scales)
+    return plan, time.time() - t0
+
+
+def group_timing(aatc, device, g_h=4, n_calls=64, reps=3, enc_iters=6, n_copies=16):
+    """Head-group bases on the Llama-shaped layer (Sec. 5 Step 1 with the paper's Llama grouping:
+    two groups of four kv-heads, 512 channels per group stream): encode of 32768 tokens and the
+    decode of all 32 query heads, timed like the headline (decode calls as one CUDA graph over
+    packed-cache copies larger than L2)."""
+    import torch
+    cfg = W.CONFIGS["llama_layer"]
+    B, T = 1, cfg.n_ctx
+    plan, plan_s = group_plan_for(aatc, cfg, g_h)
+    kd, vd = W.kv_device(cfg, 0, B, T, device)
+    qs = W.queries_device(cfg, 0, B, 8, device)
+    caches = [plan.new_cache(B, T, device) for _ in range(n_copies)]
+    stream = torch.cuda.current_stream()
+    peak, kind = _peaks()
+    ctr = [0]
+
+    def enc():
+        aatc.encode(plan, 0, kd, vd, caches[ctr[0] % n_copies], 0, T)
+        ctr[0] += 1
+
+    for _ in range(n_copies):
+        enc()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(enc_iters):
+        enc()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    enc_us = e0.elapsed_time(e1) * 1e3 / enc_iters
+    in_bytes = (kd.numel() + vd.numel()) * 2
+    out = torch.empty((B, cfg.n_q_heads, 128), dtype=torch.float32, device=device)
+    ws = torch.empty(max(1, plan.workspace_bytes(B, T) // 4), dtype=torch.float32, device=device)
+
+    def calls():
+        for i in range(n_calls):
+            aatc.decode_attention(plan, 0, qs[i % qs.shape[0]], caches[i % n_copies], T, T, out=out, workspace=ws)
+
+    calls()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        calls()
+    graph.replay()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    dec_us = e0.elapsed_time(e1) * 1e3 / (reps * n_calls)
+    # algorithmic bytes: the packed codes (sum of widths) and one fp32 alpha per group stream
+    ng = cfg.n_kv_heads // g_h
+    dbytes = float(B * T * (plan._bits.astype(np.int64).sum() / 8.0 + 4 * ng * 2))
+    dec_gbs = dbytes / (dec_us * 1e-6) / 1e9
+    enc_gbs = in_bytes / (enc_us * 1e-6) / 1e9
+    res = {"workload": f"Llama-3.1-8B-shaped layer with head-group bases: 2 groups x {g_h} kv-heads "
+                       f"({128 * g_h} channels per group stream), {T} tokens, 32 query heads, 2.75 bits",
+           "encode": {"us_per_call": round(enc_us, 2), "input_gbs": round(enc_gbs, 2),
+                      "frac_of_measured_hbm_on_input": round(enc_gbs / peak, 4)},
+           "decode": {"us_per_call": round(dec_us, 3), "gbs": round(dec_gbs, 2), "bytes_per_call": dbytes,
+                      "frac_of_measured_hbm": round(dec_gbs / peak, 4),
+                      "workspace_bytes": plan.workspace_bytes(B, T)},
+           "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 2), "peak": peak, "unit": "GB/s",
+                        "frac": round(dec_gbs / peak, 4), "traffic": None,
+                        "kernel": "one group decode call (codes + query + attention + merge kernels)",
+                        "peak_source": f"{kind} hbm_gbs (MEASURED_PEAKS.json)"},
+           "planner_seconds": round(plan_s, 2),
+           "timing": f"encode: {enc_iters} calls rotating over {n_copies} caches; decode: {n_calls}-call CUDA graph "
+                     f"x {reps} over {n_copies} packed-cache copies"}
+    plan.close()
+    return res
+
+
 def bf16_decode_timing(aatc, kd, vd, qs, n_ctx, packed_us, n_calls=64, reps=3):
     """The uncompressed reference decode (split-K attention over the bf16 K/V with the same shapes
     and queries), timed like the packed decode: a CUDA graph of calls alternating two K/V copies
@@ -793,6 +892,7 @@ def run_ours(args):
     sw["streaming"] = sink_window_stream_timing(aatc, plan, cfg, kd, vd, qs, dev)
     ref16 = bf16_decode_timing(aatc, kd, vd, qs, T, dec_mean / steps_dec * 1e3)
     qwen = qwen_timing(aatc, dev)
+    groups = group_timing(aatc, dev)
     stack = stack_decode_timing(aatc, dev)
     hid = hidden_encode_timing(aatc, dev)
     pre = prefill_timing(aatc, dev)
@@ -852,6 +952,7 @@ def run_ours(args):
         "sink_window": sw,
         "bf16_decode": ref16,
         "qwen_layer": qwen,
+        "head_groups": groups,
         "decode_llama_stack": stack,
         "encode_hidden": hid,
         "prefill": pre,

@@ -8,7 +8,8 @@
 //   score_t = (U_K^T q~) . h_hat_t / sqrt(128) = alpha_t sum_c q'_c f_c code_tc,
 //   out     = rows of block m of U_V applied to sum_t p_t h_hat^V_t.
 // Four launches per call:
-//   codes  the prefill codes kernel: every slice's signed codes as f16 (exact for widths <= 8)
+//   codes  every slice's signed codes as f16 (exact for widths <= 8), rebuilt in closed form from
+//          the record layout's run bounds
 //   query  per (query head, group, sequence): q'' = (U_K^T q~) f log2(e) / sqrt(128) over the n
 //          slice-major channels (thread = channel)
 //   attn   per (split, group, sequence), 8 warps: per 128-token tile the key codes of every slice
@@ -84,6 +85,110 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t&
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
+// Signed codes of every slot's records as f16 (exact for widths <= 8), in the prefill codes
+// layout ([b][slot][K|V][n_ctx_pad][128]; value tiles transposed to [channel][token]).  Thread =
+// token of one 128-token tile of one slot and kind.  Each stored value is rebuilt in closed form
+// from the stream's run bounds (no entry tables): digit k of channel c (c < l2all[k]) is D2 entry
+// sum_{k' < k} l2[k'] + c when c < l2[k], else the moved pair at D1 bit n_odd + 2 (moved before
+// it); the top bit of a width 2k + 1 channel is D1 bit (odd channels of wider widths) + (c -
+// l2all[k]).  Widths are non-increasing in storage order, which makes every run a prefix.
+__global__ void __launch_bounds__(TILE) aatc_group_codes_kernel(const uint32_t* words, const StreamLayout* lays,
+                                                                __half* codes, int layer, int n_kv, int n_ctx,
+                                                                int n_ctx_pad, int n_tiles, int n_words) {
+  __shared__ uint32_t rec[32][TILE];
+  const int tile = blockIdx.x, hk = blockIdx.y, b = blockIdx.z, t = threadIdx.x;
+  const int head = hk >> 1, kind = hk & 1;
+  const size_t cs = (static_cast<size_t>(b) * n_kv + head) * 2 + kind;
+  const int tok = tile * TILE + t;
+  __half* krow = codes + (cs * n_ctx_pad + tok) * D;
+  __half* vcol = codes + cs * n_ctx_pad * D + static_cast<size_t>(tile) * TILE * D + t;
+  const __half zero = __float2half_rn(0.0f);
+  if (tok >= n_ctx) {                              // padding tokens of the last tile: zero codes
+    if (tok < n_ctx_pad) {
+      if (kind == 1) {
+        for (int c = 0; c < D; ++c) vcol[c * TILE] = zero;
+      } else {
+        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(krow + c) = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    return;
+  }
+  const StreamLayout ly = lays[(layer * n_kv + head) * 2 + kind];
+  const int nw = ly.n2 / 16 + (ly.n1 + 31) / 32;
+  const uint32_t* tw = words + (cs * n_tiles + tile) * static_cast<size_t>(n_words) * TILE;
+  for (int w = 0; w < nw; ++w) {
+    const uint32_t* ww = tw + static_cast<size_t>(w) * TILE;
+    uint32_t x;
+    if (kind == 0) {
+      x = ww[t];
+    } else {                                       // quad-interleaved: quarter r in slot 4Q + (0, 2, 1, 3)[r]
+      const int q4 = 4 * (t >> 2), sh = 8 * (t & 3);
+      x = ((ww[q4] >> sh) & 0xFFu) | (((ww[q4 + 2] >> sh) & 0xFFu) << 8) | (((ww[q4 + 1] >> sh) & 0xFFu) << 16) |
+          (((ww[q4 + 3] >> sh) & 0xFFu) << 24);
+    }
+    rec[w][t] = x;                                 // each thread reads back only its own column
+  }
+  int e0[8], mo[8], od[8];
+  int n_odd = 0;
+  {
+    int e = 0, m = 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      e0[k] = e;
+      mo[k] = m;
+      e += ly.l2[k];
+      m += ly.l2all[k] - ly.l2[k];
+    }
+#pragma unroll
+    for (int k = 7; k >= 0; --k) {
+      od[k] = n_odd;
+      n_odd += ly.lodd[k] - ly.l2all[k];
+    }
+  }
+  const int d1w = ly.n2 / 16;
+  auto d1bit = [&](int p) -> uint32_t { return (rec[d1w + (p >> 5)][t] >> (p & 31)) & 1u; };
+  for (int c0 = 0; c0 < D; c0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int c = c0 + i;
+      uint32_t u = 0;
+      int nb = 0;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (c >= ly.lodd[k]) break;                // lodd is non-increasing in k
+        if (c < ly.l2all[k]) {
+          uint32_t dg;
+          if (c < ly.l2[k]) {
+            const int e = e0[k] + c;
+            dg = (rec[e >> 4][t] >> (2 * (e & 15))) & 3u;
+          } else {
+            const int p = n_odd + 2 * (mo[k] + c - ly.l2[k]);
+            dg = d1bit(p) | (d1bit(p + 1) << 1);
+          }
+          u |= dg << (2 * k);
+          nb = 2 * k + 2;
+        } else {
+          u |= d1bit(od[k] + c - ly.l2all[k]) << (2 * k);
+          nb = 2 * k + 1;
+        }
+      }
+      v[i] = nb > 0 ? static_cast<float>(static_cast<int>(u) - (1 << (nb - 1))) : 0.0f;
+    }
+    if (kind == 1) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) vcol[(c0 + i) * TILE] = __float2half_rn(v[i]);
+    } else {
+      uint4 q;
+      q.x = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[0], v[1]));
+      q.y = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[2], v[3]));
+      q.z = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[4], v[5]));
+      q.w = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[6], v[7]));
+      *reinterpret_cast<uint4*>(krow + c0) = q;
+    }
+  }
+}
+
 // q'' of one query head over the group's n channels (thread = slice-major channel j' = 128 s + c).
 __global__ void aatc_group_query_kernel(const GroupDecodeArgs a) {
   __shared__ float qv[D];
@@ -92,12 +197,18 @@ __global__ void aatc_group_query_kernel(const GroupDecodeArgs a) {
   if (j < D) qv[j] = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q_heads + hq) * D + j]);
   __syncthreads();
   const float* u = a.uk + (static_cast<size_t>(a.layer) * a.n_groups + g) * a.n * a.n + static_cast<size_t>(m) * D * a.n;
-  float acc = 0.0f;
-  for (int d = 0; d < D; ++d) acc = fmaf(u[static_cast<size_t>(d) * a.n + j], qv[d], acc);
+  float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+  for (int d = 0; d < D; d += 16) {                // 16 loads in flight per thread
+    float x[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) x[k] = u[static_cast<size_t>(d + k) * a.n + j];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) acc[k & 3] = fmaf(x[k], qv[d + k], acc[k & 3]);
+  }
   const int s = j / D, c = j % D;
   const int slot = (a.layer * a.n_kv + g * a.gh + s) * 2;
   a.qf[((static_cast<size_t>(b) * a.n_groups + g) * a.nq + i) * a.n + j] =
-      acc * a.f[slot * D + c] * (kGLog2e * 0.08838834764831845f);
+      ((acc[0] + acc[1]) + (acc[2] + acc[3])) * a.f[slot * D + c] * (kGLog2e * 0.08838834764831845f);
 }
 
 template <int GH>
@@ -355,42 +466,74 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_attn_kernel(const Gr
   }
 }
 
-// Per (query head, group, sequence): combine the splits, o_hat_j = f^V_j O_j / l, and
-// out = U_V[block rows] o_hat (thread = output dim; the first loop thread = channel).
-__global__ void __launch_bounds__(256) aatc_group_merge_kernel(const GroupDecodeArgs a) {
-  extern __shared__ float ohat[];                 // [n]
-  __shared__ float wsp[1];
+// Per (query head, group, sequence), 512 threads: combine the splits (weights 2^(m_s - M)),
+// o_hat_j = f^V_j O_j / l (thread = channel), then out = U_V[block rows] o_hat with four threads
+// per output dim, each over a quarter of the channels.
+constexpr int kGMThreads = 512;
+__global__ void __launch_bounds__(kGMThreads) aatc_group_merge_kernel(const GroupDecodeArgs a) {
+  extern __shared__ float msm[];                  // ohat [n], w [n_splits], part [4][128]
+  float* ohat = msm;
+  float* wsp = msm + a.n;
+  float* psum = wsp + ((a.n_splits + 3) & ~3);
+  __shared__ float red[kGMThreads / 32];
+  __shared__ float s_l;
   const int i = blockIdx.x, g = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int N = a.n, m = i / a.group;
   const size_t pstride = static_cast<size_t>(N) + 4;
   const float* pb = a.part + (((static_cast<size_t>(b) * a.n_groups + g) * a.nq + i) * a.n_splits) * pstride;
+  // M = max_s m_s (block reduction), then w_s and l = sum_s w_s l_s
+  float mloc = -INFINITY;
+  for (int s2 = tid; s2 < a.n_splits; s2 += kGMThreads) mloc = fmaxf(mloc, pb[s2 * pstride + N]);
+  for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+  if ((tid & 31) == 0) red[tid >> 5] = mloc;
+  __syncthreads();
   float M = -INFINITY;
-  for (int s = 0; s < a.n_splits; ++s) M = fmaxf(M, pb[s * pstride + N]);
-  float l = 0.0f;
-  for (int s = 0; s < a.n_splits; ++s) {
-    const float ms = pb[s * pstride + N];
-    if (ms != -INFINITY) l += exp2f(ms - M) * pb[s * pstride + N + 1];
+  for (int w = 0; w < kGMThreads / 32; ++w) M = fmaxf(M, red[w]);
+  __syncthreads();
+  float lloc = 0.0f;
+  for (int s2 = tid; s2 < a.n_splits; s2 += kGMThreads) {
+    const float ms = pb[s2 * pstride + N];
+    const float w = ms == -INFINITY ? 0.0f : exp2f(ms - M);
+    wsp[s2] = w;
+    lloc += w * pb[s2 * pstride + N + 1];
   }
-  if (tid == 0) wsp[0] = l;
-  for (int j = tid; j < N; j += blockDim.x) {
-    float o = 0.0f;
-    for (int s = 0; s < a.n_splits; ++s) {
-      const float ms = pb[s * pstride + N];
-      if (ms != -INFINITY) o += exp2f(ms - M) * pb[s * pstride + j];
+  for (int o = 16; o > 0; o >>= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
+  if ((tid & 31) == 0) red[tid >> 5] = lloc;
+  __syncthreads();
+  if (tid == 0) {
+    float l = 0.0f;
+    for (int w = 0; w < kGMThreads / 32; ++w) l += red[w];
+    s_l = l;
+  }
+  for (int j = tid; j < N; j += kGMThreads) {
+    float o0 = 0.0f, o1 = 0.0f;
+    int s2 = 0;
+    for (; s2 + 1 < a.n_splits; s2 += 2) {
+      o0 = fmaf(wsp[s2], pb[s2 * pstride + j], o0);
+      o1 = fmaf(wsp[s2 + 1], pb[(s2 + 1) * pstride + j], o1);
     }
+    if (s2 < a.n_splits) o0 = fmaf(wsp[s2], pb[s2 * pstride + j], o0);
     const int sl = j / D, c = j % D;
     const int slot = (a.layer * a.n_kv + g * a.gh + sl) * 2 + 1;
-    ohat[j] = o * a.f[slot * D + c];
+    ohat[j] = (o0 + o1) * a.f[slot * D + c];
   }
   __syncthreads();
-  const float inv_l = 1.0f / wsp[0];
+  const int d = tid & (D - 1), part = tid >> 7, span = N / 4;
   const float* u = a.uvt + (static_cast<size_t>(a.layer) * a.n_groups + g) * static_cast<size_t>(N) * N +
-                   static_cast<size_t>(m) * D;
-  for (int d = tid; d < D; d += blockDim.x) {
-    float acc = 0.0f;
-    for (int j = 0; j < N; ++j) acc = fmaf(u[static_cast<size_t>(j) * N + d], ohat[j], acc);
-    a.out[(static_cast<size_t>(b) * a.n_q_heads + g * a.nq + i) * D + d] = acc * inv_l;
+                   static_cast<size_t>(m) * D + d;
+  float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+  for (int j = part * span; j < (part + 1) * span; j += 16) {   // 16 loads in flight per thread
+    float x[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) x[k] = u[static_cast<size_t>(j + k) * N];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) acc[k & 3] = fmaf(x[k], ohat[j + k], acc[k & 3]);
   }
+  psum[part * D + d] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  __syncthreads();
+  if (tid < D)
+    a.out[(static_cast<size_t>(b) * a.n_q_heads + g * a.nq + i) * D + tid] =
+        ((psum[tid] + psum[D + tid]) + (psum[2 * D + tid] + psum[3 * D + tid])) / s_l;
 }
 
 int group_splits(const Plan& plan, int batch, int n_ctx) {
@@ -426,7 +569,12 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   if (gh != 2 && gh != 4) return cudaErrorNotSupported;
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
   const GroupWs wl = group_ws_layout(plan, batch, n_ctx);
-  cudaError_t e = launch_codes(plan, layer, cache, batch, n_ctx, max_tokens, ws, st);
+  if (plan.n_words > 32) return cudaErrorNotSupported;
+  const int n_ctx_pad = (n_ctx + TILE - 1) / TILE * TILE;
+  aatc_group_codes_kernel<<<dim3(n_ctx_pad / TILE, plan.dims.n_kv_heads * 2, batch), TILE, 0, st>>>(
+      static_cast<const uint32_t*>(cache), plan.dev.lay, static_cast<__half*>(ws), layer, plan.dims.n_kv_heads, n_ctx,
+      n_ctx_pad, g.n_tiles, plan.n_words);
+  cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   GroupDecodeArgs a;
   a.codes = static_cast<const __half*>(ws);
@@ -468,8 +616,8 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const size_t msm = static_cast<size_t>(a.n) * 4;
-  aatc_group_merge_kernel<<<dim3(a.nq, a.n_groups, batch), 128, msm, st>>>(a);
+  const size_t msm = (static_cast<size_t>(a.n) + ((a.n_splits + 3) & ~3) + 4 * D) * 4;
+  aatc_group_merge_kernel<<<dim3(a.nq, a.n_groups, batch), kGMThreads, msm, st>>>(a);
   return cudaGetLastError();
 }
 
