@@ -125,3 +125,54 @@ def test_group_plan_refusals(aatc):
     with pytest.raises(aatc.AatcError) as e:
         aatc.decode_attention_noalloc(plan, 0, q, torch.empty((1, 16, 128), device=DEV), cache, 128, 256)
     assert e.value.status == 5
+
+
+def test_group_llama_layer_full_size(aatc):
+    """The Llama-shaped layer with the paper's Llama grouping (two groups of four kv-heads, 512
+    channels per group stream), 32768 tokens: every code of every slice against the oracle's
+    encode of the concatenated kv-heads, and the decode of all 32 query heads."""
+    cfg = W.CONFIGS["llama_layer"]
+    g_h = 4
+    plan, basis, bits, scales = _group_plan(aatc, cfg, g_h)
+    T = cfg.n_ctx
+    kd, vd = W.kv_device(cfg, 0, 1, T, DEV)
+    cache = plan.new_cache(1, T, DEV)
+    aatc.encode(plan, 0, kd, vd, cache, 0, T)
+    u32 = cache.cpu().numpy().view(np.uint32)
+    ng, n = cfg.n_kv_heads // g_h, 128 * g_h
+    mis = tot = 0
+    coeffs = {}
+    for g in range(ng):
+        for kind, x in ((0, kd), (1, vd)):
+            xg = x[0, :, g * g_h:(g + 1) * g_h].float().cpu().numpy().reshape(T, n)
+            b_g = bits[0, g, kind].astype(np.int64)
+            codes_ref, alpha_ref, tq = O.encode_stream(xg, Hn.bf16_round(basis[0, g, kind]).astype(np.float64), b_g,
+                                                       scales[0, g, kind].astype(np.float64))
+            got, alphas, recs = _slice_codes(u32, plan, cfg, g_h, T, 0, g, kind, 0, T, b_g)
+            keep = b_g > 0
+            diff = got - codes_ref
+            thr = np.floor(tq) + 0.5
+            near = np.abs(tq - thr) <= Hn.NEAR_REL * np.abs(thr)
+            bad = (diff != 0) & keep[None, :] & ~((np.abs(diff) == 1) & near)
+            assert not bad.any(), f"group {g} kind {kind}: {int(bad.sum())} codes differ away from a threshold"
+            mis += int(np.count_nonzero(diff[:, keep]))
+            tot += int(keep.sum()) * T
+            assert np.allclose(alphas[0].astype(np.float64), alpha_ref, rtol=2e-5, atol=1e-30)
+            h = np.zeros((T, n), np.float32)
+            for s in range(g_h):
+                assert np.array_equal(alphas[s], alphas[0])
+                bs = b_g[s::g_h]
+                h[:, s::g_h] = O.dequantize_f32(O.unpack_records(recs[s], bs), alphas[s], scales[0, g, kind][s::g_h], bs)
+            coeffs[(g, kind)] = h
+    name = "head groups, Llama layer (2 x 4 kv-heads, 32768 tokens)"
+    Hn.NearThreshold.add(name, mis, tot)
+    Hn.NearThreshold.assert_bound(name)
+    q = W.queries_device(cfg, 0, 1, 1, DEV)[0]
+    out = aatc.decode_attention(plan, 0, q, cache, T, T).cpu().numpy()
+    qh = q.float().cpu().numpy()[0]
+    nq = g_h * cfg.group
+    for g in range(ng):
+        ref = O.decode_attention_head_group(qh[g * nq:(g + 1) * nq], coeffs[(g, 0)], coeffs[(g, 1)],
+                                            basis[0, g, 0], basis[0, g, 1], cfg.group)
+        Hn.check_decode(out[0, g * nq:(g + 1) * nq], ref)
+    assert plan.device_error() == 0
