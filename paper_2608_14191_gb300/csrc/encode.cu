@@ -402,26 +402,20 @@ __device__ __forceinline__ uint32_t bits32(const uint32_t (&U)[N], int i, int pr
 // Writes one token's record words in order.  Keys: word-planar, token lane t of a tile in column
 // t of each record word.  Values: tokens 4Q .. 4Q+3 share slots 4Q .. 4Q+3 of each record word,
 // slot 4Q + (0, 2, 1, 3)[r] holding byte-quarter r of the four tokens' words (token 4Q + i in
-// byte i).  When the lane quad is one whole token quad of this call, a byte transpose across the
-// quad (two shuffles) gives lane i the slot of quarter i, stored as one word; otherwise each token
-// writes its own four bytes.  Every lane of the warp calls it at the same record word.
+// byte i): each token writes its own four bytes.  (Whole slot words through a byte transpose
+// across the lane quad measured slower: the larger inlined flush lengthened the code executed per
+// record word, which a kernel started after other work fetches from memory.)
 struct RecordFlush {
   uint32_t* tile_words;   // record word 0 of the token's tile
   int tt;                 // token lane inside the tile
-  uint32_t s1, s2;        // byte selectors of the two transpose steps (values)
-  int qpos;               // slot of byte-quarter (lane & 3) (values)
-  bool value, quad_ok, ok;
+  bool value, ok;
   int wi;
   __device__ __forceinline__ void operator()(uint32_t w) {
     uint32_t* rw = tile_words + static_cast<size_t>(wi) * TILE;
-    if (!value) {
-      if (ok) rw[tt] = w;
-    } else {
-      const uint32_t y1 = __byte_perm(w, __shfl_xor_sync(0xffffffffu, w, 1), s1);
-      const uint32_t y2 = __byte_perm(y1, __shfl_xor_sync(0xffffffffu, y1, 2), s2);
-      if (quad_ok) {
-        rw[4 * (tt >> 2) + qpos] = y2;
-      } else if (ok) {
+    if (ok) {
+      if (!value) {
+        rw[tt] = w;
+      } else {
         uint8_t* q = reinterpret_cast<uint8_t*>(rw + 4 * (tt >> 2)) + (tt & 3);
         q[0] = static_cast<uint8_t>(w);
         q[8] = static_cast<uint8_t>(w >> 8);
@@ -634,9 +628,6 @@ __global__ void __launch_bounds__(kKThreads, 1)
     const int tl = quad * 32 + lane;                           // token lane inside the tile
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
     const QuantTables tb{sm.inv_s, sm.inv_f, sm.hi, sm.magic};
-    const int t4 = lane & 3;                                   // position in the lane quad
-    const uint32_t s1 = (t4 & 1) ? 0x3715u : 0x6240u, s2 = (t4 & 2) ? 0x3276u : 0x5410u;
-    const int qpos = ((t4 & 1) << 1) | (t4 >> 1);              // slot of byte-quarter t4
     // one instantiation for streams with a channel wider than 8 bits (high bytes kept), one without
     auto drain = [&](auto wide_tag) {
       constexpr bool kWide = decltype(wide_tag)::value;
@@ -663,9 +654,8 @@ __global__ void __launch_bounds__(kKThreads, 1)
           if (!isfinite(amax)) atomicOr(a.err, 1);
           a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
         }
-        // lanes 4Q' .. 4Q'+3 are one token quad of the cache when start is a multiple of 4
         RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
-                      pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
+                      pos_t % TILE, kind == 1, ok, 0};
         pack_token_regs<kWide>(sm.lay, U, UH, f, a.n_words);
       }
     };
@@ -837,9 +827,6 @@ __global__ void __launch_bounds__(kGThreads, 1)
   } else {
     const int eg = warp >> 2, quad = warp & 3, tl = quad * 32 + lane;
     const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
-    const int t4 = lane & 3;
-    const uint32_t s1 = (t4 & 1) ? 0x3715u : 0x6240u, s2 = (t4 & 2) ? 0x3276u : 0x5410u;
-    const int qpos = ((t4 & 1) << 1) | (t4 >> 1);
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     uint32_t uh[8];
 #pragma unroll 1
@@ -880,7 +867,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
         const size_t sidx = (static_cast<size_t>(b) * a.n_kv + grp * GH + sl) * 2 + kind;
         if (ok) a.alpha[sidx * a.n_tiles * TILE + pos_t] = amax;
         RecordFlush f{a.words + sidx * stream_words + static_cast<size_t>(pos_t / TILE) * a.n_words * TILE,
-                      pos_t % TILE, s1, s2, qpos, kind == 1, (a.start & 3) == 0 && (i | 3) < a.n_tokens, ok, 0};
+                      pos_t % TILE, kind == 1, ok, 0};
         pack_token_regs<false>(sm.lay[sl], U[k], uh, f, a.n_words);
       }
     }
