@@ -7,16 +7,15 @@
 // (kv-head block m = j / group) sees the embedded query q~ (q at block m, zeros elsewhere):
 //   score_t = (U_K^T q~) . h_hat_t / sqrt(128) = alpha_t sum_c q'_c f_c code_tc,
 //   out     = rows of block m of U_V applied to sum_t p_t h_hat^V_t.
-// Four launches per call:
-//   codes  every slice's signed codes as f16 (exact for widths <= 8), rebuilt in closed form from
-//          the record layout's run bounds
+// Three launches per call:
 //   query  per (query head, group, sequence): q'' = (U_K^T q~) f log2(e) / sqrt(128) over the n
 //          slice-major channels (thread = channel)
-//   attn   per (split, group, sequence), 8 warps: per 128-token tile the key codes of every slice
-//          (S = q''_hi . code + q''_lo . code, mma.sync m16n8k16 f16, rows = the group's <= 16
-//          query heads, one accumulator over all n channels), online softmax with the exponent of
-//          alpha^V folded into the running maximum (so P' = 2^(s - m) alpha^V stays below 2), then
-//          O_s += P' . code^V for every slice s; row operands from shared memory by ldmatrix
+//   attn   per (split, group, sequence), 8 warps: the slices' record words are the operands of
+//          mma.sync m16n8k16 f16 (a digit or bit masked into a 16-bit half is the subnormal
+//          digit 2^-24), rows = the group's <= 16 query heads: scores summed over every slice
+//          and corrected by the stored-value offsets, online softmax with the exponent of
+//          alpha^V folded into the running maximum (P' = 2^(s - m) alpha^V < 2), value entry sums
+//          per slice, channel sums at the end of the split
 //   merge  per (query head, group, sequence): log-sum-exp over the splits, o_hat = f^V O / l, and
 //          out = U_V[block m rows] o_hat
 #include <cuda_bf16.h>
@@ -33,10 +32,8 @@ namespace {
 constexpr float kGLog2e = 1.4426950408889634f;
 constexpr int kGAThreads = 256;                  // 8 warps
 constexpr int kGRing = 4;                        // code chunks in flight
-constexpr int kGRowHalves = D + 8;               // padded shared-memory row (272 bytes)
 
 struct GroupDecodeArgs {
-  const __half* codes;       // codes workspace [b][n_kv][K|V][n_ctx_pad][128]
   const float* alpha;        // cache alpha region [b][n_kv][K|V][n_tiles * 128]
   const __nv_bfloat16* q;    // [b][H_q][128]
   const float* uk;           // plan: U_K of every (layer, group), [n dim][n channel]
@@ -45,7 +42,12 @@ struct GroupDecodeArgs {
   float* qf;                 // workspace: folded queries [b][n_groups][nq][n]
   float* part;               // workspace: split partials [b][n_groups][nq][n_splits][n + 4]
   float* out;                // [b][H_q][128]
+  const uint32_t* words;     // cache word region (the digit kernel reads the records directly)
+  const short* entry;        // plan: [slot][n_entries] (channel | shift << 8), -1 padded
+  const ChanEnc* enc;        // plan: [slot][128] (offset 2^(b-1) of each stored value)
+  const StreamLayout* lay;   // plan: [slot]
   int layer, n_kv, gh, n_groups, group, nq, n, n_q_heads, n_ctx, n_ctx_pad, n_tiles, n_splits;
+  int n_words, n_entries, ks_max, n_pairs;   // ks_max: k-steps of the widest slice; n_pairs: value tiles
 };
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
@@ -57,12 +59,6 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-// Four 8x8 b16 matrices; lane l gives the address of row l % 8 of matrix l / 8.
-__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))));
 }
 __device__ __forceinline__ void mma16816(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -83,110 +79,6 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t&
   const __half2 l = __floats2half2_rn(x - hf.x, y - hf.y);
   hi = *reinterpret_cast<const uint32_t*>(&h);
   lo = *reinterpret_cast<const uint32_t*>(&l);
-}
-
-// Signed codes of every slot's records as f16 (exact for widths <= 8), in the prefill codes
-// layout ([b][slot][K|V][n_ctx_pad][128]; value tiles transposed to [channel][token]).  Thread =
-// token of one 128-token tile of one slot and kind.  Each stored value is rebuilt in closed form
-// from the stream's run bounds (no entry tables): digit k of channel c (c < l2all[k]) is D2 entry
-// sum_{k' < k} l2[k'] + c when c < l2[k], else the moved pair at D1 bit n_odd + 2 (moved before
-// it); the top bit of a width 2k + 1 channel is D1 bit (odd channels of wider widths) + (c -
-// l2all[k]).  Widths are non-increasing in storage order, which makes every run a prefix.
-__global__ void __launch_bounds__(TILE) aatc_group_codes_kernel(const uint32_t* words, const StreamLayout* lays,
-                                                                __half* codes, int layer, int n_kv, int n_ctx,
-                                                                int n_ctx_pad, int n_tiles, int n_words) {
-  __shared__ uint32_t rec[32][TILE];
-  const int tile = blockIdx.x, hk = blockIdx.y, b = blockIdx.z, t = threadIdx.x;
-  const int head = hk >> 1, kind = hk & 1;
-  const size_t cs = (static_cast<size_t>(b) * n_kv + head) * 2 + kind;
-  const int tok = tile * TILE + t;
-  __half* krow = codes + (cs * n_ctx_pad + tok) * D;
-  __half* vcol = codes + cs * n_ctx_pad * D + static_cast<size_t>(tile) * TILE * D + t;
-  const __half zero = __float2half_rn(0.0f);
-  if (tok >= n_ctx) {                              // padding tokens of the last tile: zero codes
-    if (tok < n_ctx_pad) {
-      if (kind == 1) {
-        for (int c = 0; c < D; ++c) vcol[c * TILE] = zero;
-      } else {
-        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(krow + c) = make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
-    return;
-  }
-  const StreamLayout ly = lays[(layer * n_kv + head) * 2 + kind];
-  const int nw = ly.n2 / 16 + (ly.n1 + 31) / 32;
-  const uint32_t* tw = words + (cs * n_tiles + tile) * static_cast<size_t>(n_words) * TILE;
-  for (int w = 0; w < nw; ++w) {
-    const uint32_t* ww = tw + static_cast<size_t>(w) * TILE;
-    uint32_t x;
-    if (kind == 0) {
-      x = ww[t];
-    } else {                                       // quad-interleaved: quarter r in slot 4Q + (0, 2, 1, 3)[r]
-      const int q4 = 4 * (t >> 2), sh = 8 * (t & 3);
-      x = ((ww[q4] >> sh) & 0xFFu) | (((ww[q4 + 2] >> sh) & 0xFFu) << 8) | (((ww[q4 + 1] >> sh) & 0xFFu) << 16) |
-          (((ww[q4 + 3] >> sh) & 0xFFu) << 24);
-    }
-    rec[w][t] = x;                                 // each thread reads back only its own column
-  }
-  int e0[8], mo[8], od[8];
-  int n_odd = 0;
-  {
-    int e = 0, m = 0;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      e0[k] = e;
-      mo[k] = m;
-      e += ly.l2[k];
-      m += ly.l2all[k] - ly.l2[k];
-    }
-#pragma unroll
-    for (int k = 7; k >= 0; --k) {
-      od[k] = n_odd;
-      n_odd += ly.lodd[k] - ly.l2all[k];
-    }
-  }
-  const int d1w = ly.n2 / 16;
-  auto d1bit = [&](int p) -> uint32_t { return (rec[d1w + (p >> 5)][t] >> (p & 31)) & 1u; };
-  for (int c0 = 0; c0 < D; c0 += 8) {
-    float v[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int c = c0 + i;
-      uint32_t u = 0;
-      int nb = 0;
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        if (c >= ly.lodd[k]) break;                // lodd is non-increasing in k
-        if (c < ly.l2all[k]) {
-          uint32_t dg;
-          if (c < ly.l2[k]) {
-            const int e = e0[k] + c;
-            dg = (rec[e >> 4][t] >> (2 * (e & 15))) & 3u;
-          } else {
-            const int p = n_odd + 2 * (mo[k] + c - ly.l2[k]);
-            dg = d1bit(p) | (d1bit(p + 1) << 1);
-          }
-          u |= dg << (2 * k);
-          nb = 2 * k + 2;
-        } else {
-          u |= d1bit(od[k] + c - ly.l2all[k]) << (2 * k);
-          nb = 2 * k + 1;
-        }
-      }
-      v[i] = nb > 0 ? static_cast<float>(static_cast<int>(u) - (1 << (nb - 1))) : 0.0f;
-    }
-    if (kind == 1) {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) vcol[(c0 + i) * TILE] = __float2half_rn(v[i]);
-    } else {
-      uint4 q;
-      q.x = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[0], v[1]));
-      q.y = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[2], v[3]));
-      q.z = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[4], v[5]));
-      q.w = *reinterpret_cast<const uint32_t*>(&(const __half2&)__floats2half2_rn(v[6], v[7]));
-      *reinterpret_cast<uint4*>(krow + c0) = q;
-    }
-  }
 }
 
 // q'' of one query head over the group's n channels (thread = slice-major channel j' = 128 s + c).
@@ -211,21 +103,54 @@ __global__ void aatc_group_query_kernel(const GroupDecodeArgs a) {
       ((acc[0] + acc[1]) + (acc[2] + acc[3])) * a.f[slot * D + c] * (kGLog2e * 0.08838834764831845f);
 }
 
-template <int GH>
-struct GroupAttnSmem {
-  static constexpr int N = D * GH, NKS = N / 16;
-  uint4 qfrag[NKS][32][2];                        // score A fragments (hi, lo) per k-step and lane
-  uint4 pfrag[TILE / 16][32][2];                  // P' A fragments (hi, lo) of the current tile
-  alignas(128) __half ring[kGRing][TILE][kGRowHalves];
-  float redm[8][16], reds[8][16];
-  float qinv[16], mrow[16], lrow[16], rscale[16];
+// ---------------------------------------------------------------- digit-operand split attention
+// The slices' record words are the tensor-core operands themselves (no unpacked codes): a base-4 digit (or a single bit) masked into the low bits of a 16-bit half
+// is the subnormal f16 digit 2^-24, exact in the product.
+//   scores: per slice and record word, k = the word's 16 D2 fields (or 16 of a D1 word's 32 bits):
+//           A = q''_c 2^shift per entry (rows = queries, hi / lo), B = the 16 tokens' digits of
+//           this warp (b0 = x >> 2t: fields t, t + 8; b1 = x >> 2t + 8: fields t + 4, t + 12);
+//           raw = sum q'' u over all slices, s = alpha^K (raw - C) with C = sum_c q''_c 2^(b_c - 1)
+//   values: per slice and 8 record entries, A = P' (queries x 16 tokens, hi / lo), B = the
+//           entries' digits of those tokens from the quad-interleaved value slots; the entry sums
+//           become channel sums o_c = sum_e 2^shift O_e - 2^(b_c - 1) S' (S' = the represented
+//           sum of P') through shared-memory adds at the end of the split.
+constexpr int kGDMaxPairs = 24;                  // value (slice, 8-entry tile) pairs per warp
+
+struct GroupDigitSmem {
+  int qfrag, pfrag, ring, oc, offs, kent, misc, total, chunk_words, kent_stride;
+  __host__ __device__ GroupDigitSmem(int gh, int ks_max, int n_words, int n_entries) {
+    kent_stride = (n_entries + 7) & ~7;
+    int o = 0;
+    qfrag = o;  o += gh * ks_max * 32 * 32;       // [slice][k-step][lane][hi, lo] uint4
+    pfrag = o;  o += (TILE / 16) * 32 * 32;       // [k-step][lane][hi, lo] uint4
+    chunk_words = n_words * TILE;
+    ring = o;   o += kGRing * chunk_words * 4;    // record words of one slice and kind, one tile
+    oc = o;     o += 16 * D * gh * 4;             // q'' of the queries in the prologue; channel sums at the end
+    offs = o;   o += 2 * D * gh * 4;              // stored-value offsets 2^(b-1), keys then values
+    kent = o;   o += gh * ((n_entries + 7) & ~7) * 2;   // key entry tables of the slices
+    misc = o;   o += 16 * 4 * 20 + 3 * 8 * 16 * 4;
+    total = o;
+  }
 };
 
 template <int GH>
-__global__ void __launch_bounds__(kGAThreads, 1) aatc_group_attn_kernel(const GroupDecodeArgs a) {
-  constexpr int N = D * GH, NKS = N / 16, NCH = 2 * GH;
+__global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const GroupDecodeArgs a) {
+  constexpr int N = D * GH, NCH = 2 * GH;
   extern __shared__ __align__(128) unsigned char smb[];
-  auto& sm = *reinterpret_cast<GroupAttnSmem<GH>*>(smb);
+  const GroupDigitSmem L(GH, a.ks_max, a.n_words, a.n_entries);
+  uint4* qfrag = reinterpret_cast<uint4*>(smb + L.qfrag);
+  uint4* pfrag = reinterpret_cast<uint4*>(smb + L.pfrag);
+  uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
+  float* oc = reinterpret_cast<float*>(smb + L.oc);
+  float* qinv = reinterpret_cast<float*>(smb + L.misc);
+  float* mrow = qinv + 16;
+  float* lrow = mrow + 16;
+  float* srow = lrow + 16;                        // S' of each query
+  float* rscale = srow + 16;
+  float* corr = rscale + 16;                      // C of each query
+  float* redm = corr + 16;                        // [8][16]
+  float* reds = redm + 8 * 16;                    // [8][16]
+  float* redp = reds + 8 * 16;                    // [8][16]
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, gq = lane >> 2, t = lane & 3;
   const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
@@ -235,101 +160,154 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_attn_kernel(const Gr
   const float* kalpha = a.alpha + (slot0 * 2) * a.n_tiles * TILE;
   const float* valpha = a.alpha + (slot0 * 2 + 1) * a.n_tiles * TILE;
   const float* qf = a.qf + (static_cast<size_t>(b) * a.n_groups + g) * a.nq * N;
+  const int pslot0 = (a.layer * a.n_kv + g * GH) * 2;   // plan slot of slice 0, keys (values + 1)
+  const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
 
-  // ---- score A fragments: rows = queries (>= nq zero), scaled by a power of two so the largest
-  // |q''| of a row is below 2^14, split into f16 hi / lo
-  if (tid < 16) {
-    float mx = 0.0f;
-    if (tid < a.nq)
-      for (int j = 0; j < N; ++j) mx = fmaxf(mx, fabsf(qf[tid * N + j]));
-    int ex = 0;
-    if (mx > 0.0f) frexpf(mx, &ex);               // mx < 2^ex
-    sm.qinv[tid] = ldexpf(1.0f, ex - 14);          // the row was scaled by 2^(14 - ex)
-    sm.mrow[tid] = -INFINITY;
-    sm.lrow[tid] = 0.0f;
+  // ---- stage q'' (in the channel-sum buffer), the offsets and the key entry tables
+  float* qs = oc;                                  // [16][N] q'' (rows >= nq zero)
+  float* offk = reinterpret_cast<float*>(smb + L.offs);
+  float* offv = offk + N;
+  short* kent = reinterpret_cast<short*>(smb + L.kent);
+  for (int i = tid; i < 16 * N; i += kGAThreads) qs[i] = i / N < a.nq ? qf[i] : 0.0f;
+  for (int j = tid; j < N; j += kGAThreads) {
+    offk[j] = a.enc[(pslot0 + 2 * (j / D)) * D + j % D].off;
+    offv[j] = a.enc[(pslot0 + 2 * (j / D) + 1) * D + j % D].off;
+  }
+  for (int i = tid; i < GH * L.kent_stride; i += kGAThreads) {
+    const int sl = i / L.kent_stride, e = i % L.kent_stride;
+    kent[i] = e < a.n_entries ? a.entry[static_cast<size_t>(pslot0 + 2 * sl) * a.n_entries + e] : short(-1);
   }
   __syncthreads();
-  for (int idx = tid; idx < NKS * 32; idx += kGAThreads) {
-    const int ks = idx >> 5, ln = idx & 31, r0 = ln >> 2, c0 = ks * 16 + 2 * (ln & 3);
+  // ---- per query (warp w: queries 2w, 2w + 1): scale bound max |q''| 2^(b-1) and C = sum q'' 2^(b-1)
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int r = 2 * warp + h;
+    float mx = 0.0f, c = 0.0f;
+    for (int j = lane; j < N; j += 32) {
+      const float v = qs[r * N + j], off = offk[j];
+      mx = fmaxf(mx, fabsf(v) * off);              // bounds |q'' 2^shift| of every entry (shift <= b - 1)
+      c = fmaf(v, off, c);
+    }
+    for (int o2 = 16; o2 > 0; o2 >>= 1) {
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o2));
+      c += __shfl_xor_sync(0xffffffffu, c, o2);
+    }
+    if (lane == 0) {
+      int ex = 0;
+      if (mx > 0.0f) frexpf(mx, &ex);
+      qinv[r] = ldexpf(1.0f, ex - 14);
+      corr[r] = c;
+      mrow[r] = -INFINITY;
+      lrow[r] = 0.0f;
+      srow[r] = 0.0f;
+    }
+  }
+  __syncthreads();
+  for (int idx = tid; idx < GH * a.ks_max * 32; idx += kGAThreads) {
+    const int sl = idx / (a.ks_max * 32), ks = (idx / 32) % a.ks_max, ln = idx & 31, r0 = ln >> 2, tt = ln & 3;
+    const StreamLayout& ly = a.lay[pslot0 + 2 * sl];
+    const int n2 = ly.n2, ne = ly.n2 + ly.n1, n2w = n2 / 16, nks = n2w + 2 * ((ly.n1 + 31) / 32);
+    int ent[4] = {-1, -1, -1, -1};                // entries in k order 2t, 2t + 1, 2t + 8, 2t + 9
+    if (ks < n2w) {
+      const int e = 16 * ks;
+      ent[0] = e + tt; ent[1] = e + tt + 8; ent[2] = e + tt + 4; ent[3] = e + tt + 12;
+    } else if (ks < nks) {
+      const int u = (ks - n2w) >> 1, s2 = (ks - n2w) & 1, e = n2 + 32 * u + 8 * s2;
+      ent[0] = e + tt; ent[1] = e + tt + 16; ent[2] = e + tt + 4; ent[3] = e + tt + 20;
+    }
+    const short* et = kent + sl * L.kent_stride;
+    const float i0 = 1.0f / qinv[r0], i1 = 1.0f / qinv[r0 + 8];
     float v[8];
-    const int rows[4] = {r0, r0 + 8, r0, r0 + 8};
-    const int cols[4] = {c0, c0, c0 + 8, c0 + 8};
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      const int r = rows[k];
-      const float sc = r < a.nq ? 1.0f / sm.qinv[r] : 0.0f;
-      v[2 * k] = r < a.nq ? qf[r * N + cols[k]] * sc : 0.0f;
-      v[2 * k + 1] = r < a.nq ? qf[r * N + cols[k] + 1] * sc : 0.0f;
+      const int ce = ent[k] >= 0 && ent[k] < ne ? et[ent[k]] : -1;
+      const float w2 = ce >= 0 ? ldexpf(1.0f, (ce >> 8) & 15) : 0.0f;
+      const int j = sl * D + (ce & 0xFF);
+      v[2 * k] = ce >= 0 ? qs[r0 * N + j] * w2 * i0 : 0.0f;
+      v[2 * k + 1] = ce >= 0 ? qs[(r0 + 8) * N + j] * w2 * i1 : 0.0f;
     }
+    // A fragment: a0 = row r0 (k 2t, 2t + 1), a1 = row r0 + 8, a2 = row r0 (k 2t + 8, 2t + 9), a3 = row r0 + 8
     uint4 hi, lo;
-    split2(v[0], v[1], hi.x, lo.x);
-    split2(v[2], v[3], hi.y, lo.y);
-    split2(v[4], v[5], hi.z, lo.z);
-    split2(v[6], v[7], hi.w, lo.w);
-    sm.qfrag[ks][ln][0] = hi;
-    sm.qfrag[ks][ln][1] = lo;
+    split2(v[0], v[2], hi.x, lo.x);
+    split2(v[1], v[3], hi.y, lo.y);
+    split2(v[4], v[6], hi.z, lo.z);
+    split2(v[5], v[7], hi.w, lo.w);
+    qfrag[((sl * a.ks_max + ks) * 32 + ln) * 2] = hi;
+    qfrag[((sl * a.ks_max + ks) * 32 + ln) * 2 + 1] = lo;
   }
+  __syncthreads();
+  for (int i = tid; i < 16 * N; i += kGAThreads) oc[i] = 0.0f;   // q'' no longer needed
 
-  // ---- code chunks: per tile the key codes of slices 0 .. GH-1, then their value codes
+  // ---- record chunks: per tile the key words of slices 0 .. GH-1, then their value words
   const int n_chunks = (tile_hi - tile_lo) * NCH;
+  const int cw = L.chunk_words;
   auto issue = [&](int u) {
     if (u < n_chunks) {
-      const int tile = tile_lo + u / NCH, c = u % NCH, s = c % GH, kind = c / GH;
-      const __half* src = a.codes + ((slot0 + s) * 2 + kind) * static_cast<size_t>(a.n_ctx_pad) * D +
-                          static_cast<size_t>(tile) * TILE * D;
-      __half* dst = &sm.ring[u % kGRing][0][0];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const int p = tid + kGAThreads * k, row = p >> 4, col = (p & 15) * 8;
-        cp_async16(dst + row * kGRowHalves + col, src + row * D + col);
-      }
+      const int tile = tile_lo + u / NCH, c = u % NCH, sl = c % GH, kind = c / GH;
+      const uint32_t* src = a.words + ((slot0 + sl) * 2 + kind) * stream_words + static_cast<size_t>(tile) * cw;
+      uint32_t* dst = ring + (u % kGRing) * cw;
+      for (int p = tid * 4; p < cw; p += kGAThreads * 4) cp_async16(dst + p, src + p);
     }
     cp_async_commit();
   };
   for (int u = 0; u < kGRing - 1; ++u) issue(u);
 
   float sacc[2][4];
-  float oacc[GH][2][4];
+  float oacc[kGDMaxPairs][4];
 #pragma unroll
-  for (int s = 0; s < GH; ++s)
+  for (int pi = 0; pi < kGDMaxPairs; ++pi)
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-      for (int r = 0; r < 4; ++r) oacc[s][nt][r] = 0.0f;
-  const int tw = 16 * warp;                       // score pass: this warp's tokens of the tile
-  const int cw = 16 * warp;                       // value pass: this warp's channels of each slice
-  // ldmatrix row addresses: matrix l / 8 = (rows +8 if l >= 16, columns +8 if l & 8)
-  const int lrow = (lane & 7) + ((lane & 16) ? 8 : 0), lcol = (lane & 8) ? 8 : 0;
+    for (int r = 0; r < 4; ++r) oacc[pi][r] = 0.0f;
+  const int tw = 16 * warp;
+  const uint32_t m2 = 0x00030003u, m1 = 0x00010001u;
 
   for (int u = 0; u < n_chunks; ++u) {
     issue(u + kGRing - 1);
     cp_async_wait<kGRing - 1>();
     __syncthreads();
-    const int tile = tile_lo + u / NCH, c = u % NCH, s = c % GH;
-    const __half* ch = &sm.ring[u % kGRing][0][0];
+    const int tile = tile_lo + u / NCH, c = u % NCH, sl = c % GH;
+    const uint32_t* ch = ring + (u % kGRing) * cw;
+    const StreamLayout ly = a.lay[pslot0 + 2 * sl + (c < GH ? 0 : 1)];
+    const int n2w = ly.n2 / 16, n1w = (ly.n1 + 31) / 32;
     if (c < GH) {
-      // ---- scores of this warp's 16 tokens over slice s
-      if (s == 0)
+      if (sl == 0)
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
           for (int r = 0; r < 4; ++r) sacc[nt][r] = 0.0f;
+      const uint4* qa = qfrag + (sl * a.ks_max) * 32 * 2;
+      for (int w = 0; w < n2w; ++w) {
+        const uint4 ah = qa[(w * 32 + lane) * 2], al = qa[(w * 32 + lane) * 2 + 1];
 #pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        uint32_t bm[4];
-        ldmatrix_x4(bm, ch + (tw + lrow) * kGRowHalves + ks * 16 + lcol);
-        const uint4 ah = sm.qfrag[s * 8 + ks][lane][0], al = sm.qfrag[s * 8 + ks][lane][1];
-        mma16816(sacc[0], ah, bm[0], bm[1]);
-        mma16816(sacc[0], al, bm[0], bm[1]);
-        mma16816(sacc[1], ah, bm[2], bm[3]);
-        mma16816(sacc[1], al, bm[2], bm[3]);
+        for (int nt = 0; nt < 2; ++nt) {
+          const uint32_t x = ch[w * TILE + tw + 8 * nt + gq];
+          const uint32_t b0 = (x >> (2 * t)) & m2, b1 = (x >> (2 * t + 8)) & m2;
+          mma16816(sacc[nt], ah, b0, b1);
+          mma16816(sacc[nt], al, b0, b1);
+        }
       }
-      if (c == GH - 1) {
-        // ---- online softmax of the tile.  Lane (gq, t) holds rows gq, gq + 8 and tokens
-        // tw + 8 nt + 2t + {0, 1}; e = s + floor(log2 alpha^V) keeps P' = 2^(e - m) mant(alpha^V) < 2.
+      for (int w = 0; w < n1w; ++w) {
+#pragma unroll
+        for (int s2 = 0; s2 < 2; ++s2) {
+          const int ks = n2w + 2 * w + s2;
+          const uint4 ah = qa[(ks * 32 + lane) * 2], al = qa[(ks * 32 + lane) * 2 + 1];
+#pragma unroll
+          for (int nt = 0; nt < 2; ++nt) {
+            const uint32_t x = ch[(n2w + w) * TILE + tw + 8 * nt + gq];
+            const uint32_t b0 = (x >> (t + 8 * s2)) & m1, b1 = (x >> (t + 4 + 8 * s2)) & m1;
+            mma16816(sacc[nt], ah, b0, b1);
+            mma16816(sacc[nt], al, b0, b1);
+          }
+        }
+      }
+      if (sl == GH - 1) {
+        // ---- online softmax of the tile, raw = acc 2^24 / scale - C.  Lane (gq, t) holds rows gq,
+        // gq + 8 and tokens tw + 8 nt + 2t + {0, 1}; e = s + floor(log2 alpha^V) keeps
+        // P' = 2^(e - m) mant(alpha^V) < 2.
         float e[2][4], mant[2][4], lav[2][4];
         float mx0 = -INFINITY, mx1 = -INFINITY;
-        const float qi0 = sm.qinv[gq], qi1 = sm.qinv[gq + 8];
+        const float q0 = qinv[gq] * 16777216.0f, q1 = qinv[gq + 8] * 16777216.0f;
+        const float c0 = corr[gq], c1 = corr[gq + 8];
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
@@ -340,12 +318,12 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_attn_kernel(const Gr
             float ev = -INFINITY, mv = 0.0f, lv = 0.0f;
             if (ok) {
               const float ak = kalpha[tok], avv = valpha[tok];
-              const float sv = sacc[nt][r] * (r < 2 ? qi0 : qi1) * ak;
+              const float sv = (r < 2 ? fmaf(sacc[nt][r], q0, -c0) : fmaf(sacc[nt][r], q1, -c1)) * ak;
               int ex = 0;
-              const float fr = frexpf(avv, &ex);        // avv = fr 2^ex, fr in [0.5, 1)
+              const float fr = frexpf(avv, &ex);
               lv = avv > 0.0f ? static_cast<float>(max(ex - 1, -64)) : -64.0f;
               mv = avv > 0.0f ? fr * 2.0f : 0.0f;
-              if (avv > 0.0f && ex - 1 < -64) mv = avv * 18446744073709551616.0f;   // alpha^V / 2^-64
+              if (avv > 0.0f && ex - 1 < -64) mv = avv * 18446744073709551616.0f;
               ev = sv + lv;
             }
             e[nt][r] = ev;
@@ -359,110 +337,163 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_attn_kernel(const Gr
         mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
         mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
         if (t == 0) {
-          sm.redm[warp][gq] = mx0;
-          sm.redm[warp][gq + 8] = mx1;
+          redm[warp * 16 + gq] = mx0;
+          redm[warp * 16 + gq + 8] = mx1;
         }
         __syncthreads();
         if (tid < 16) {
           float mt = -INFINITY;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) mt = fmaxf(mt, sm.redm[w][tid]);
-          const float mo = sm.mrow[tid], mn = fmaxf(mo, mt);
-          sm.rscale[tid] = mo == -INFINITY ? 0.0f : fexp2(mo - mn);
-          sm.mrow[tid] = mn;
+          for (int w = 0; w < 8; ++w) mt = fmaxf(mt, redm[w * 16 + tid]);
+          const float mo = mrow[tid], mn = fmaxf(mo, mt);
+          rscale[tid] = mo == -INFINITY ? 0.0f : fexp2(mo - mn);
+          mrow[tid] = mn;
         }
         __syncthreads();
-        const float m0 = sm.mrow[gq], m1 = sm.mrow[gq + 8];
-        float ls0 = 0.0f, ls1 = 0.0f;
+        const float m0 = mrow[gq], m1r = mrow[gq + 8];
+        float ls0 = 0.0f, ls1 = 0.0f, ps0 = 0.0f, ps1 = 0.0f;
         float p[2][4];
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
           for (int r = 0; r < 4; ++r) {
-            const float mm = r < 2 ? m0 : m1;
-            const float x = e[nt][r] == -INFINITY ? 0.0f : fexp2(e[nt][r] - mm);   // 2^(e - m) <= 1
-            p[nt][r] = x * mant[nt][r];                                           // P' = 2^(s - m) alpha^V
-            const float l = e[nt][r] == -INFINITY ? 0.0f : x * exp2f(-lav[nt][r]);  // 2^(s - m)
+            const float mm = r < 2 ? m0 : m1r;
+            const float x = e[nt][r] == -INFINITY ? 0.0f : fexp2(e[nt][r] - mm);
+            p[nt][r] = x * mant[nt][r];
+            const float l = e[nt][r] == -INFINITY ? 0.0f : x * exp2f(-lav[nt][r]);
             if (r < 2) ls0 += l;
             else ls1 += l;
           }
         uint4 ph, pl;
-        split2(p[0][0], p[0][1], ph.x, pl.x);   // row gq,     tokens 2t, 2t + 1
-        split2(p[0][2], p[0][3], ph.y, pl.y);   // row gq + 8, tokens 2t, 2t + 1
-        split2(p[1][0], p[1][1], ph.z, pl.z);   // row gq,     tokens 2t + 8, 2t + 9
-        split2(p[1][2], p[1][3], ph.w, pl.w);   // row gq + 8, tokens 2t + 8, 2t + 9
-        sm.pfrag[warp][lane][0] = ph;
-        sm.pfrag[warp][lane][1] = pl;
+        split2(p[0][0], p[0][1], ph.x, pl.x);
+        split2(p[0][2], p[0][3], ph.y, pl.y);
+        split2(p[1][0], p[1][1], ph.z, pl.z);
+        split2(p[1][2], p[1][3], ph.w, pl.w);
+        pfrag[(warp * 32 + lane) * 2] = ph;
+        pfrag[(warp * 32 + lane) * 2 + 1] = pl;
+        // S': the represented P' (hi + lo) that the value MMAs add
+        {
+          const __half2* hh = reinterpret_cast<const __half2*>(&ph);
+          const __half2* ll = reinterpret_cast<const __half2*>(&pl);
+          float2 v;
+          v = __half22float2(hh[0]); ps0 += v.x + v.y; v = __half22float2(ll[0]); ps0 += v.x + v.y;
+          v = __half22float2(hh[2]); ps0 += v.x + v.y; v = __half22float2(ll[2]); ps0 += v.x + v.y;
+          v = __half22float2(hh[1]); ps1 += v.x + v.y; v = __half22float2(ll[1]); ps1 += v.x + v.y;
+          v = __half22float2(hh[3]); ps1 += v.x + v.y; v = __half22float2(ll[3]); ps1 += v.x + v.y;
+        }
         ls0 += __shfl_xor_sync(0xffffffffu, ls0, 1);
         ls0 += __shfl_xor_sync(0xffffffffu, ls0, 2);
         ls1 += __shfl_xor_sync(0xffffffffu, ls1, 1);
         ls1 += __shfl_xor_sync(0xffffffffu, ls1, 2);
+        ps0 += __shfl_xor_sync(0xffffffffu, ps0, 1);
+        ps0 += __shfl_xor_sync(0xffffffffu, ps0, 2);
+        ps1 += __shfl_xor_sync(0xffffffffu, ps1, 1);
+        ps1 += __shfl_xor_sync(0xffffffffu, ps1, 2);
         if (t == 0) {
-          sm.reds[warp][gq] = ls0;
-          sm.reds[warp][gq + 8] = ls1;
+          reds[warp * 16 + gq] = ls0;
+          reds[warp * 16 + gq + 8] = ls1;
+          redp[warp * 16 + gq] = ps0;
+          redp[warp * 16 + gq + 8] = ps1;
         }
-        const float r0 = sm.rscale[gq], r1 = sm.rscale[gq + 8];
+        // value accumulators: rows of D are the queries (c0, c1: row gq; c2, c3: row gq + 8)
+        const float r0 = rscale[gq], r1 = rscale[gq + 8];
 #pragma unroll
-        for (int s2 = 0; s2 < GH; ++s2)
-#pragma unroll
-          for (int nt = 0; nt < 2; ++nt) {
-            oacc[s2][nt][0] *= r0;
-            oacc[s2][nt][1] *= r0;
-            oacc[s2][nt][2] *= r1;
-            oacc[s2][nt][3] *= r1;
-          }
+        for (int pi = 0; pi < kGDMaxPairs; ++pi) {
+          oacc[pi][0] *= r0;
+          oacc[pi][1] *= r0;
+          oacc[pi][2] *= r1;
+          oacc[pi][3] *= r1;
+        }
         __syncthreads();
         if (tid < 16) {
-          float lt = 0.0f;
+          float lt = 0.0f, pt = 0.0f;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) lt += sm.reds[w][tid];
-          sm.lrow[tid] = sm.lrow[tid] * sm.rscale[tid] + lt;
+          for (int w = 0; w < 8; ++w) {
+            lt += reds[w * 16 + tid];
+            pt += redp[w * 16 + tid];
+          }
+          lrow[tid] = lrow[tid] * rscale[tid] + lt;
+          srow[tid] = srow[tid] * rscale[tid] + pt;
         }
       }
     } else {
-      // ---- O_s += P' . code^V: this warp's 16 channels of slice s, K = the tile's 128 tokens
+      // ---- O_e += P' . digit_e for this warp's (slice, 8-entry tile) pairs of slice sl
+      const int ne = ly.n2 + ly.n1;
 #pragma unroll
-      for (int kt = 0; kt < TILE / 16; ++kt) {
-        uint32_t bm[4];
-        ldmatrix_x4(bm, ch + (cw + lrow) * kGRowHalves + kt * 16 + lcol);
-        const uint4 ah = sm.pfrag[kt][lane][0], al = sm.pfrag[kt][lane][1];
+      for (int pi = 0; pi < kGDMaxPairs; ++pi) {
+        const int pr = warp + 8 * pi;
+        if (pr >= a.n_pairs) break;
+        // pairs are numbered slice-major: pr = sl' * ntp + nt with ntp n-tiles per slice
+        const int ntp = (a.ks_max * 16 + 7) / 8;
+        const int p_sl = pr / ntp, p_nt = pr % ntp;
+        if (p_sl != sl) continue;
+        const int e = 8 * p_nt + gq;               // this lane's entry (B column gq)
+        uint32_t widx = 0, shb = 0, msk = 0;
+        int qpos = 0;
+        if (e < ly.n2) {
+          const int f = e & 15;
+          widx = e >> 4;
+          qpos = (f >> 2) == 1 ? 2 : (f >> 2) == 2 ? 1 : (f >> 2);
+          shb = 2 * (f & 3);
+          msk = 3u;
+        } else if (e < ne) {
+          const int e1 = e - ly.n2, bb = e1 & 31;
+          widx = n2w + (e1 >> 5);
+          qpos = (bb >> 3) == 1 ? 2 : (bb >> 3) == 2 ? 1 : (bb >> 3);
+          shb = bb & 7;
+          msk = 1u;
+        }
+        const uint32_t mlo = msk, mhi = msk << 16;
+        const uint32_t* wr = ch + widx * TILE + qpos;
+        const int i0 = 2 * (t & 1);
 #pragma unroll
-        for (int s2 = 0; s2 < GH; ++s2)
-          if (s2 == s) {
-            mma16816(oacc[s2][0], ah, bm[0], bm[1]);
-            mma16816(oacc[s2][0], al, bm[0], bm[1]);
-            mma16816(oacc[s2][1], ah, bm[2], bm[3]);
-            mma16816(oacc[s2][1], al, bm[2], bm[3]);
-          }
+        for (int kt = 0; kt < TILE / 16; ++kt) {
+          const uint32_t x0 = wr[4 * (4 * kt + (t >> 1))], x1 = wr[4 * (4 * kt + 2 + (t >> 1))];
+          const uint32_t y0 = x0 >> (8 * i0 + shb), y1 = x1 >> (8 * i0 + shb);
+          const uint32_t b0 = (y0 & mlo) | ((y0 << 8) & mhi), b1 = (y1 & mlo) | ((y1 << 8) & mhi);
+          const uint4 ah = pfrag[(kt * 32 + lane) * 2], al = pfrag[(kt * 32 + lane) * 2 + 1];
+          mma16816(oacc[pi], ah, b0, b1);
+          mma16816(oacc[pi], al, b0, b1);
+        }
       }
     }
-    __syncthreads();                              // the chunk's slot is refilled next
+    __syncthreads();
   }
   cp_async_wait<0>();
 
-  // ---- partials of the split: rows gq, gq + 8; channels 128 s + cw + 8 nt + 2t + {0, 1}
-  const size_t pstride = static_cast<size_t>(N) + 4;
-  float* pb = a.part + ((static_cast<size_t>(b) * a.n_groups + g) * a.nq) * a.n_splits * pstride;
+  // ---- entry sums -> channel sums (shared-memory adds), then the split's partials
+  {
+    const int ntp = (a.ks_max * 16 + 7) / 8;
 #pragma unroll
-  for (int s = 0; s < GH; ++s)
+    for (int pi = 0; pi < kGDMaxPairs; ++pi) {
+      const int pr = warp + 8 * pi;
+      if (pr >= a.n_pairs) break;
+      const int p_sl = pr / ntp, p_nt = pr % ntp;
+      const short* et = a.entry + static_cast<size_t>(pslot0 + 2 * p_sl + 1) * a.n_entries;
+      const StreamLayout ly = a.lay[pslot0 + 2 * p_sl + 1];
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      const int j = s * D + cw + 8 * nt + 2 * t;
-      if (gq < a.nq) {
-        float* d0 = pb + (static_cast<size_t>(gq) * a.n_splits + split) * pstride + j;
-        d0[0] = oacc[s][nt][0];
-        d0[1] = oacc[s][nt][1];
-      }
-      if (gq + 8 < a.nq) {
-        float* d1 = pb + (static_cast<size_t>(gq + 8) * a.n_splits + split) * pstride + j;
-        d1[0] = oacc[s][nt][2];
-        d1[1] = oacc[s][nt][3];
+      for (int k = 0; k < 2; ++k) {
+        const int e = 8 * p_nt + 2 * t + k;        // D column 2t + k
+        const int ce = e < ly.n2 + ly.n1 ? et[e] : -1;
+        if (ce < 0) continue;
+        const float w2 = ldexpf(1.0f, ((ce >> 8) & 15) + 24);   // digits entered as d 2^-24
+        const int j = p_sl * D + (ce & 0xFF);
+        if (gq < a.nq) atomicAdd(&oc[gq * N + j], w2 * oacc[pi][k]);
+        if (gq + 8 < a.nq) atomicAdd(&oc[(gq + 8) * N + j], w2 * oacc[pi][2 + k]);
       }
     }
+  }
+  __syncthreads();
+  const size_t pstride = static_cast<size_t>(N) + 4;
+  float* pb = a.part + ((static_cast<size_t>(b) * a.n_groups + g) * a.nq) * a.n_splits * pstride;
+  for (int idx = tid; idx < a.nq * N; idx += kGAThreads) {
+    const int i = idx / N, j = idx % N;
+    pb[(static_cast<size_t>(i) * a.n_splits + split) * pstride + j] = oc[i * N + j] - offv[j] * srow[i];
+  }
   if (tid < a.nq) {
     float* d = pb + (static_cast<size_t>(tid) * a.n_splits + split) * pstride + N;
-    d[0] = sm.mrow[tid];
-    d[1] = sm.lrow[tid];
+    d[0] = mrow[tid];
+    d[1] = lrow[tid];
   }
 }
 
@@ -545,11 +576,22 @@ int group_splits(const Plan& plan, int batch, int n_ctx) {
 struct GroupWs {
   size_t qf_off, part_off, bytes;
 };
+// k-steps (D2 words + 2 x D1 words) of the widest slice stream of `layer` (keys or values)
+int group_ks_max(const Plan& plan, int layer) {
+  int m = 1;
+  for (int h = 0; h < plan.dims.n_kv_heads; ++h)
+    for (int kind = 0; kind < 2; ++kind) {
+      const StreamLayout& ly = plan.layout[(layer * plan.dims.n_kv_heads + h) * 2 + kind];
+      m = std::max(m, ly.n2 / 16 + 2 * ((ly.n1 + 31) / 32));
+    }
+  return m;
+}
+
 GroupWs group_ws_layout(const Plan& plan, int batch, int n_ctx) {
   const int ng = plan.dims.n_kv_heads / plan.group_heads, n = D * plan.group_heads;
   const int nq = plan.dims.n_q_heads / ng;
   GroupWs w;
-  size_t off = (prefill_workspace(batch, plan.dims.n_kv_heads, n_ctx) + 255) / 256 * 256;
+  size_t off = 0;
   w.qf_off = off;
   off += static_cast<size_t>(batch) * ng * nq * n * 4;
   off = (off + 255) / 256 * 256;
@@ -569,15 +611,7 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   if (gh != 2 && gh != 4) return cudaErrorNotSupported;
   const CacheGeom g = cache_geom(batch, plan.dims.n_kv_heads, max_tokens, plan.n_words);
   const GroupWs wl = group_ws_layout(plan, batch, n_ctx);
-  if (plan.n_words > 32) return cudaErrorNotSupported;
-  const int n_ctx_pad = (n_ctx + TILE - 1) / TILE * TILE;
-  aatc_group_codes_kernel<<<dim3(n_ctx_pad / TILE, plan.dims.n_kv_heads * 2, batch), TILE, 0, st>>>(
-      static_cast<const uint32_t*>(cache), plan.dev.lay, static_cast<__half*>(ws), layer, plan.dims.n_kv_heads, n_ctx,
-      n_ctx_pad, g.n_tiles, plan.n_words);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
   GroupDecodeArgs a;
-  a.codes = static_cast<const __half*>(ws);
   a.alpha = reinterpret_cast<const float*>(static_cast<const uint32_t*>(cache) + g.words_elems);
   a.q = static_cast<const __nv_bfloat16*>(q);
   a.uk = plan.gdev.uk;
@@ -598,22 +632,27 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   a.n_ctx_pad = (n_ctx + TILE - 1) / TILE * TILE;
   a.n_tiles = g.n_tiles;
   a.n_splits = group_splits(plan, batch, n_ctx);
-  if (a.nq > 16) return cudaErrorNotSupported;
+  a.words = static_cast<const uint32_t*>(cache);
+  a.entry = plan.dev.entry;
+  a.enc = plan.dev.enc;
+  a.lay = plan.dev.lay;
+  a.n_words = plan.n_words;
+  a.n_entries = plan.n_entries;
+  a.ks_max = group_ks_max(plan, layer);
+  a.n_pairs = gh * 2 * a.ks_max;                 // (slice, 8-entry tile) pairs of the value records
+  if (a.nq > 16 || a.n_pairs > 8 * kGDMaxPairs) return cudaErrorNotSupported;
   aatc_group_query_kernel<<<dim3(a.nq, a.n_groups, batch), a.n, 0, st>>>(a);
-  e = cudaGetLastError();
+  cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 grid(a.n_splits, a.n_groups, batch);
-  if (gh == 2) {
-    const size_t smem = sizeof(GroupAttnSmem<2>);
-    e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_group_attn_kernel<2>), smem);
-    if (e != cudaSuccess) return e;
-    aatc_group_attn_kernel<2><<<grid, kGAThreads, smem, st>>>(a);
-  } else {
-    const size_t smem = sizeof(GroupAttnSmem<4>);
-    e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_group_attn_kernel<4>), smem);
-    if (e != cudaSuccess) return e;
-    aatc_group_attn_kernel<4><<<grid, kGAThreads, smem, st>>>(a);
-  }
+  const size_t smem = static_cast<size_t>(GroupDigitSmem(gh, a.ks_max, a.n_words, a.n_entries).total);
+  if (smem > 227 * 1024) return cudaErrorNotSupported;
+  const void* kern = gh == 2 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2>)
+                             : reinterpret_cast<const void*>(aatc_group_digit_kernel<4>);
+  e = ensure_smem_optin(kern, smem);
+  if (e != cudaSuccess) return e;
+  if (gh == 2) aatc_group_digit_kernel<2><<<grid, kGAThreads, smem, st>>>(a);
+  else aatc_group_digit_kernel<4><<<grid, kGAThreads, smem, st>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const size_t msm = (static_cast<size_t>(a.n) + ((a.n_splits + 3) & ~3) + 4 * D) * 4;
