@@ -122,7 +122,7 @@ constexpr int kWarps = kThreads / 32;
 //   values:  B = value digits of one record entry for tokens (0, 2) and (1, 3) of a token quad,
 //            from the quad-interleaved value words; A = P' of the same tokens in that order.
 __device__ __forceinline__ void mma_f16(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
       "{%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])

@@ -8,16 +8,18 @@
 //   score_t = (U_K^T q~) . h_hat_t / sqrt(128) = alpha_t sum_c q'_c f_c code_tc,
 //   out     = rows of block m of U_V applied to sum_t p_t h_hat^V_t.
 // Three launches per call:
-//   query  per (query head, group, sequence): q'' = (U_K^T q~) f log2(e) / sqrt(128) over the n
-//          slice-major channels (thread = channel)
+//   query  per (query row < 16, slice, group, sequence): q'' = (U_K^T q~) f log2(e) / sqrt(128)
+//          over the slice's 128 channels, the slice's scale and part of the offset correction, and
+//          the row's words of the slice's score A fragments (entry order of its key records)
 //   attn   per (split, group, sequence), 8 warps: the slices' record words are the operands of
 //          mma.sync m16n8k16 f16 (a digit or bit masked into a 16-bit half is the subnormal
 //          digit 2^-24), rows = the group's <= 16 query heads: scores summed over every slice
 //          and corrected by the stored-value offsets, online softmax with the exponent of
 //          alpha^V folded into the running maximum (P' = 2^(s - m) alpha^V < 2), value entry sums
 //          per slice, channel sums at the end of the split
-//   merge  per (query head, group, sequence): log-sum-exp over the splits, o_hat = f^V O / l, and
-//          out = U_V[block m rows] o_hat
+//   merge  per (query head, slice, group, sequence): log-sum-exp over the splits, o_hat = f^V O
+//          over the slice's channels and its part of U_V[block m rows] o_hat; the last slice to
+//          arrive adds the parts in slice order and divides by l
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -30,8 +32,7 @@ namespace aatc {
 namespace {
 
 constexpr float kGLog2e = 1.4426950408889634f;
-constexpr int kGAThreads = 256;                  // 8 warps
-constexpr int kGRing = 4;                        // code chunks in flight
+constexpr int kGAThreads = 512;                  // 16 warps; warps 0-7 also run the softmax (16 tokens each)
 
 struct GroupDecodeArgs {
   const float* alpha;        // cache alpha region [b][n_kv][K|V][n_tiles * 128]
@@ -39,7 +40,10 @@ struct GroupDecodeArgs {
   const float* uk;           // plan: U_K of every (layer, group), [n dim][n channel]
   const float* uvt;          // plan: U_V^T, [n channel][n dim]
   const float* f;            // plan: [slot][128] f_c
-  float* qf;                 // workspace: folded queries [b][n_groups][nq][n]
+  uint32_t* qfrag;           // workspace: score A fragments [b][n_groups][hi | lo][g_h][ks_max][32][4] (f16 pairs)
+  float* qsc;                // workspace: [b][n_groups][16][g_h][scale, C part] of each query row and slice
+  float* outp;               // workspace: [b][n_groups][16][g_h][128] per-slice output partials
+  int* ticket;               // workspace: [b][n_groups][16] merge arrivals (zeroed by the query kernel)
   float* part;               // workspace: split partials [b][n_groups][nq][n_splits][n + 4]
   float* out;                // [b][H_q][128]
   const uint32_t* words;     // cache word region (the digit kernel reads the records directly)
@@ -47,7 +51,7 @@ struct GroupDecodeArgs {
   const ChanEnc* enc;        // plan: [slot][128] (offset 2^(b-1) of each stored value)
   const StreamLayout* lay;   // plan: [slot]
   int layer, n_kv, gh, n_groups, group, nq, n, n_q_heads, n_ctx, n_ctx_pad, n_tiles, n_splits;
-  int n_words, n_entries, ks_max, n_pairs;   // ks_max: k-steps of the widest slice; n_pairs: value tiles
+  int n_words, n_entries, ks_max, stages;    // ks_max: k-steps of the widest slice; stages: ring depth
 };
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
@@ -61,7 +65,7 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ void mma16816(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
       "{%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
@@ -81,69 +85,155 @@ __device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t&
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
-// q'' of one query head over the group's n channels (thread = slice-major channel j' = 128 s + c).
-__global__ void aatc_group_query_kernel(const GroupDecodeArgs a) {
+// Per (query row i < 16, slice s, group, sequence), 512 threads = 128 channels x 4 quarters of the
+// 128 query dims; slice channel c is slice-major channel j' = 128 s + c:
+//   q''_j' = (U_K^T q~)_j' f_j' log2(e) / sqrt(128)   (zero for rows i >= nq),
+//   scale  = 2^(ceil(log2 max_c |q''| 2^(b - 1)) - 14) so that every A entry q'' 2^shift / scale of
+//            the slice is below 2^14,
+//   C_s    = sum_c q''_j' 2^(b_j' - 1) (the slice's part of the key codes' stored-value offsets),
+// and row i's words of the slice's score A fragments: for k-step ks and lane column t, the f16
+// pairs (k 2t, 2t + 1) and (k 2t + 8, 2t + 9) of q'' 2^shift 2^-p / scale over the k-step's entries
+// (p = 2t for base-4 words, t for bit words: the position at which the digit kernel leaves the
+// lane's fields), hi and lo parts.
+constexpr int kGQThreads = 512;
+__global__ void __launch_bounds__(kGQThreads) aatc_group_query_kernel(const GroupDecodeArgs a) {
   __shared__ float qv[D];
-  const int i = blockIdx.x, g = blockIdx.y, b = blockIdx.z, j = threadIdx.x;
+  __shared__ float part[4][D];
+  __shared__ float qsm[D];
+  __shared__ float redx[4], redc[4];
+  __shared__ float s_scale;
+  const int i = blockIdx.x, s = blockIdx.y % a.gh, g = blockIdx.y / a.gh, b = blockIdx.z, tid = threadIdx.x;
+  const int c = tid & (D - 1), dq = tid >> 7;
+  const bool live = i < a.nq;
   const int m = i / a.group, hq = g * a.nq + i;
-  if (j < D) qv[j] = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q_heads + hq) * D + j]);
+  const size_t bg = static_cast<size_t>(b) * a.n_groups + g;
+  if (s == 0 && tid == 0) a.ticket[bg * 16 + i] = 0;
+  if (live && tid < D) qv[tid] = __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q_heads + hq) * D + tid]);
   __syncthreads();
-  const float* u = a.uk + (static_cast<size_t>(a.layer) * a.n_groups + g) * a.n * a.n + static_cast<size_t>(m) * D * a.n;
-  float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-  for (int d = 0; d < D; d += 16) {                // 16 loads in flight per thread
-    float x[16];
+  const int pslot = (a.layer * a.n_kv + g * a.gh + s) * 2;   // plan slot of the slice's keys
+  if (live) {
+    const float* u = a.uk + (static_cast<size_t>(a.layer) * a.n_groups + g) * a.n * a.n +
+                     static_cast<size_t>(m * D + 32 * dq) * a.n + s * D + c;
+    float x[32];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) x[k] = u[static_cast<size_t>(d + k) * a.n + j];
+    for (int k = 0; k < 32; ++k) x[k] = u[static_cast<size_t>(k) * a.n];   // 32 loads in flight per thread
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-    for (int k = 0; k < 16; ++k) acc[k & 3] = fmaf(x[k], qv[d + k], acc[k & 3]);
+    for (int k = 0; k < 32; ++k) acc[k & 3] = fmaf(x[k], qv[32 * dq + k], acc[k & 3]);
+    part[dq][c] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
   }
-  const int s = j / D, c = j % D;
-  const int slot = (a.layer * a.n_kv + g * a.gh + s) * 2;
-  a.qf[((static_cast<size_t>(b) * a.n_groups + g) * a.nq + i) * a.n + j] =
-      ((acc[0] + acc[1]) + (acc[2] + acc[3])) * a.f[slot * D + c] * (kGLog2e * 0.08838834764831845f);
+  __syncthreads();
+  if (tid < D) {
+    const float qj = live ? ((part[0][c] + part[1][c]) + (part[2][c] + part[3][c])) * a.f[pslot * D + c] *
+                                (kGLog2e * 0.08838834764831845f)
+                          : 0.0f;
+    qsm[c] = qj;
+    const float off = a.enc[pslot * D + c].off;
+    float mx = fabsf(qj) * off, cc = qj * off;
+    for (int o = 16; o > 0; o >>= 1) {
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      cc += __shfl_xor_sync(0xffffffffu, cc, o);
+    }
+    if ((tid & 31) == 0) {
+      redx[tid >> 5] = mx;
+      redc[tid >> 5] = cc;
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    const float mt = fmaxf(fmaxf(redx[0], redx[1]), fmaxf(redx[2], redx[3]));
+    int ex = 0;
+    if (mt > 0.0f) frexpf(mt, &ex);
+    s_scale = ldexpf(1.0f, ex - 14);
+    a.qsc[((bg * 16 + i) * a.gh + s) * 2] = s_scale;
+    a.qsc[((bg * 16 + i) * a.gh + s) * 2 + 1] = (redc[0] + redc[1]) + (redc[2] + redc[3]);
+  }
+  __syncthreads();
+  const float inv = 1.0f / s_scale;
+  const size_t fw = static_cast<size_t>(a.gh) * a.ks_max * 128;   // u32 words of one (hi or lo) table
+  uint32_t* fh = a.qfrag + bg * 2 * fw;
+  uint32_t* fl = fh + fw;
+  const StreamLayout& ly = a.lay[pslot];
+  const int n2 = ly.n2, ne = ly.n2 + ly.n1, n2w = n2 / 16, nks = n2w + 2 * ((ly.n1 + 31) / 32);
+  const short* et = a.entry + static_cast<size_t>(pslot) * a.n_entries;
+  for (int item = tid; item < a.ks_max * 8; item += kGQThreads) {
+    const int ks = item >> 3, tt = (item >> 1) & 3, kp = item & 1;
+    int e0 = -1, e1 = -1;                          // entries at k = 2t + 8 kp and 2t + 8 kp + 1
+    float lsc = 0.0f;
+    if (ks < n2w) {                                // base-4 word: fields t, t + 8 | t + 4, t + 12
+      e0 = 16 * ks + tt + 4 * kp;
+      e1 = e0 + 8;
+      lsc = ldexpf(1.0f, -2 * tt);
+    } else if (ks < nks) {                         // bit word, half s2: bits t, t + 16 | t + 4, t + 20
+      const int uw = (ks - n2w) >> 1, s2 = (ks - n2w) & 1;
+      e0 = n2 + 32 * uw + 8 * s2 + tt + 4 * kp;
+      e1 = e0 + 16;
+      lsc = ldexpf(1.0f, -tt);
+    }
+    const int c0 = e0 >= 0 && e0 < ne ? et[e0] : -1, c1 = e1 >= 0 && e1 < ne ? et[e1] : -1;
+    const float v0 = c0 >= 0 ? qsm[c0 & 0xFF] * ldexpf(lsc, (c0 >> 8) & 15) * inv : 0.0f;
+    const float v1 = c1 >= 0 ? qsm[c1 & 0xFF] * ldexpf(lsc, (c1 >> 8) & 15) * inv : 0.0f;
+    uint32_t hi, lo;
+    split2(v0, v1, hi, lo);
+    // A fragment registers: a0 = row r (k 2t..), a1 = row r + 8, a2 = row r (k 2t + 8..), a3 = row r + 8
+    const size_t idx = ((static_cast<size_t>(s) * a.ks_max + ks) * 32 + (i & 7) * 4 + tt) * 4 + kp * 2 + (i >> 3);
+    fh[idx] = hi;
+    fl[idx] = lo;
+  }
 }
 
 // ---------------------------------------------------------------- digit-operand split attention
-// The slices' record words are the tensor-core operands themselves (no unpacked codes): a base-4 digit (or a single bit) masked into the low bits of a 16-bit half
-// is the subnormal f16 digit 2^-24, exact in the product.
-//   scores: per slice and record word, k = the word's 16 D2 fields (or 16 of a D1 word's 32 bits):
-//           A = q''_c 2^shift per entry (rows = queries, hi / lo), B = the 16 tokens' digits of
-//           this warp (b0 = x >> 2t: fields t, t + 8; b1 = x >> 2t + 8: fields t + 4, t + 12);
-//           raw = sum q'' u over all slices, s = alpha^K (raw - C) with C = sum_c q''_c 2^(b_c - 1)
-//   values: per slice and 8 record entries, A = P' (queries x 16 tokens, hi / lo), B = the
-//           entries' digits of those tokens from the quad-interleaved value slots; the entry sums
-//           become channel sums o_c = sum_e 2^shift O_e - 2^(b_c - 1) S' (S' = the represented
-//           sum of P') through shared-memory adds at the end of the split.
-constexpr int kGDMaxPairs = 24;                  // value (slice, 8-entry tile) pairs per warp
+// The slices' record words are the tensor-core operands themselves (no unpacked codes): a base-4
+// digit (or a single bit) masked into a 16-bit half is the subnormal f16 value d 2^(p - 24), p its
+// bit position in the half; the power 2^p is folded into the other operand's scale.
+//   chunks: per tile, the key words of all g_h slices, then their value words (cp.async ring)
+//   scores: warp (slice sl, part) over its slice's k-steps and 4 (g_h = 4) or 2 (g_h = 2)
+//           token n-tiles: A = q''_c 2^shift per entry (rows = queries, hi / lo, lane t's columns
+//           scaled by 2^-2t for D2 words, 2^-t for D1 words), B = the tokens' fields masked in
+//           place; the slice partials meet in shared memory and are summed per token, then
+//           raw = sum q'' u, s = alpha^K (raw - C) with C = sum_c q''_c 2^(b_c - 1)
+//   values: warp (slice sl, part) owns the 8-entry tiles part, part + 16 / g_h, ... of slice sl:
+//           A = P' (queries x 16 tokens, hi / lo, loaded once per k-step), B = the entries'
+//           fields of those tokens from the quad-interleaved value slots (byte permute + mask);
+//           the entry sums become channel sums o_c = sum_e 2^(shift - p) O_e - 2^(b_c - 1) S'
+//           (S' = the represented sum of P') through shared-memory adds at the end of the split.
+constexpr int kGRS = TILE + 8;                   // padded row stride of the per-slice score partials
 
 struct GroupDigitSmem {
-  int qfrag, pfrag, ring, oc, offs, kent, misc, total, chunk_words, kent_stride;
-  __host__ __device__ GroupDigitSmem(int gh, int ks_max, int n_words, int n_entries) {
-    kent_stride = (n_entries + 7) & ~7;
+  int qfh, qfl, pfh, pfl, ring, red, offs, info, misc, total, chunk_words;
+  __host__ __device__ GroupDigitSmem(int gh, int ks_max, int n_words, int stages) {
+    chunk_words = n_words * TILE;                 // one slice, one kind, one tile
+    const int qf = gh * ks_max * 32 * 16, pf = (TILE / 16) * 32 * 16;
+    const int rw = stages * gh * chunk_words * 4, qc = 16 * D * gh * 4;
     int o = 0;
-    qfrag = o;  o += gh * ks_max * 32 * 32;       // [slice][k-step][lane][hi, lo] uint4
-    pfrag = o;  o += (TILE / 16) * 32 * 32;       // [k-step][lane][hi, lo] uint4
-    chunk_words = n_words * TILE;
-    ring = o;   o += kGRing * chunk_words * 4;    // record words of one slice and kind, one tile
-    oc = o;     o += 16 * D * gh * 4;             // q'' of the queries in the prologue; channel sums at the end
-    offs = o;   o += 2 * D * gh * 4;              // stored-value offsets 2^(b-1), keys then values
-    kent = o;   o += gh * ((n_entries + 7) & ~7) * 2;   // key entry tables of the slices
-    misc = o;   o += 16 * 4 * 20 + 3 * 8 * 16 * 4;
+    qfh = o;   o += qf;                           // [slice][k-step][lane] uint4, hi parts
+    qfl = o;   o += qf;                           //   lo parts
+    pfh = o;   o += pf;                           // [k-step][lane] uint4, hi parts of P'
+    pfl = o;   o += pf;
+    ring = o;  o += rw > qc ? rw : qc;            // record chunks; channel sums at the end
+    red = o;   o += gh * 16 * kGRS * 4;           // [slice][query][token] score partials
+    offs = o;  o += D * gh * 4;                   // stored-value offsets 2^(b-1) of the values
+    info = o;  o += 16 * gh;                      // [slice][K|V] (n2, n1)
+    misc = o;  o += 16 * 4 * (gh + 5) + 3 * 8 * 16 * 4;
     total = o;
   }
 };
 
-template <int GH>
+template <int GH, int NPW>
 __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const GroupDecodeArgs a) {
-  constexpr int N = D * GH, NCH = 2 * GH;
+  constexpr int N = D * GH, WPS = 16 / GH, NTK = TILE / (8 * WPS);   // warps per slice, key n-tiles per warp
   extern __shared__ __align__(128) unsigned char smb[];
-  const GroupDigitSmem L(GH, a.ks_max, a.n_words, a.n_entries);
-  uint4* qfrag = reinterpret_cast<uint4*>(smb + L.qfrag);
-  uint4* pfrag = reinterpret_cast<uint4*>(smb + L.pfrag);
+  const GroupDigitSmem L(GH, a.ks_max, a.n_words, a.stages);
+  uint4* qfh = reinterpret_cast<uint4*>(smb + L.qfh);
+  uint4* qfl = reinterpret_cast<uint4*>(smb + L.qfl);
+  uint4* pfh = reinterpret_cast<uint4*>(smb + L.pfh);
+  uint4* pfl = reinterpret_cast<uint4*>(smb + L.pfl);
   uint32_t* ring = reinterpret_cast<uint32_t*>(smb + L.ring);
-  float* oc = reinterpret_cast<float*>(smb + L.oc);
-  float* qinv = reinterpret_cast<float*>(smb + L.misc);
-  float* mrow = qinv + 16;
+  float* red = reinterpret_cast<float*>(smb + L.red);
+  float* offv = reinterpret_cast<float*>(smb + L.offs);
+  int* info = reinterpret_cast<int*>(smb + L.info);
+  float* qsl = reinterpret_cast<float*>(smb + L.misc);   // [16][g_h] slice scales x 2^24
+  float* mrow = qsl + 16 * GH;
   float* lrow = mrow + 16;
   float* srow = lrow + 16;                        // S' of each query
   float* rscale = srow + 16;
@@ -153,333 +243,326 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
   float* redp = reds + 8 * 16;                    // [8][16]
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, gq = lane >> 2, t = lane & 3;
+  const int ws = warp / WPS, wsub = warp % WPS;   // this warp's slice and its part of the slice
   const int ctx_tiles = (a.n_ctx + TILE - 1) / TILE;
   const int tile_lo = static_cast<int>(static_cast<long>(split) * ctx_tiles / a.n_splits);
   const int tile_hi = static_cast<int>(static_cast<long>(split + 1) * ctx_tiles / a.n_splits);
   const size_t slot0 = static_cast<size_t>(b) * a.n_kv + static_cast<size_t>(g) * GH;   // cache slot of slice 0
   const float* kalpha = a.alpha + (slot0 * 2) * a.n_tiles * TILE;
   const float* valpha = a.alpha + (slot0 * 2 + 1) * a.n_tiles * TILE;
-  const float* qf = a.qf + (static_cast<size_t>(b) * a.n_groups + g) * a.nq * N;
+  const size_t bg = static_cast<size_t>(b) * a.n_groups + g;
   const int pslot0 = (a.layer * a.n_kv + g * GH) * 2;   // plan slot of slice 0, keys (values + 1)
   const size_t stream_words = static_cast<size_t>(a.n_tiles) * a.n_words * TILE;
 
-  // ---- stage q'' (in the channel-sum buffer), the offsets and the key entry tables
-  float* qs = oc;                                  // [16][N] q'' (rows >= nq zero)
-  float* offk = reinterpret_cast<float*>(smb + L.offs);
-  float* offv = offk + N;
-  short* kent = reinterpret_cast<short*>(smb + L.kent);
-  for (int i = tid; i < 16 * N; i += kGAThreads) qs[i] = i / N < a.nq ? qf[i] : 0.0f;
-  for (int j = tid; j < N; j += kGAThreads) {
-    offk[j] = a.enc[(pslot0 + 2 * (j / D)) * D + j % D].off;
-    offv[j] = a.enc[(pslot0 + 2 * (j / D) + 1) * D + j % D].off;
+  // ---- the score A fragments (built by the query kernel) by cp.async, with the first ring chunk;
+  // the value offsets, the slice layouts and the query scales by plain loads
+  {
+    const int fw = GH * a.ks_max * 128;
+    const uint32_t* fsrc = a.qfrag + bg * 2 * fw;
+    uint32_t* fdst = reinterpret_cast<uint32_t*>(qfh);   // hi table, then the lo table (contiguous)
+    for (int p = tid * 4; p < 2 * fw; p += kGAThreads * 4) cp_async16(fdst + p, fsrc + p);
   }
-  for (int i = tid; i < GH * L.kent_stride; i += kGAThreads) {
-    const int sl = i / L.kent_stride, e = i % L.kent_stride;
-    kent[i] = e < a.n_entries ? a.entry[static_cast<size_t>(pslot0 + 2 * sl) * a.n_entries + e] : short(-1);
+  for (int j = tid; j < N; j += kGAThreads) offv[j] = a.enc[(pslot0 + 2 * (j / D) + 1) * D + j % D].off;
+  if (tid < 2 * GH) {
+    info[2 * tid] = a.lay[pslot0 + tid].n2;
+    info[2 * tid + 1] = a.lay[pslot0 + tid].n1;
   }
-  __syncthreads();
-  // ---- per query (warp w: queries 2w, 2w + 1): scale bound max |q''| 2^(b-1) and C = sum q'' 2^(b-1)
+  if (tid < 16 * GH) qsl[tid] = a.qsc[(bg * 16 * GH + tid) * 2] * 16777216.0f;
+  if (tid < 16) {
+    float cs = 0.0f;
 #pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int r = 2 * warp + h;
-    float mx = 0.0f, c = 0.0f;
-    for (int j = lane; j < N; j += 32) {
-      const float v = qs[r * N + j], off = offk[j];
-      mx = fmaxf(mx, fabsf(v) * off);              // bounds |q'' 2^shift| of every entry (shift <= b - 1)
-      c = fmaf(v, off, c);
-    }
-    for (int o2 = 16; o2 > 0; o2 >>= 1) {
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o2));
-      c += __shfl_xor_sync(0xffffffffu, c, o2);
-    }
-    if (lane == 0) {
-      int ex = 0;
-      if (mx > 0.0f) frexpf(mx, &ex);
-      qinv[r] = ldexpf(1.0f, ex - 14);
-      corr[r] = c;
-      mrow[r] = -INFINITY;
-      lrow[r] = 0.0f;
-      srow[r] = 0.0f;
-    }
+    for (int sl = 0; sl < GH; ++sl) cs += a.qsc[((bg * 16 + tid) * GH + sl) * 2 + 1];
+    corr[tid] = cs;
+    mrow[tid] = -INFINITY;
+    lrow[tid] = 0.0f;
+    srow[tid] = 0.0f;
   }
   __syncthreads();
-  for (int idx = tid; idx < GH * a.ks_max * 32; idx += kGAThreads) {
-    const int sl = idx / (a.ks_max * 32), ks = (idx / 32) % a.ks_max, ln = idx & 31, r0 = ln >> 2, tt = ln & 3;
-    const StreamLayout& ly = a.lay[pslot0 + 2 * sl];
-    const int n2 = ly.n2, ne = ly.n2 + ly.n1, n2w = n2 / 16, nks = n2w + 2 * ((ly.n1 + 31) / 32);
-    int ent[4] = {-1, -1, -1, -1};                // entries in k order 2t, 2t + 1, 2t + 8, 2t + 9
-    if (ks < n2w) {
-      const int e = 16 * ks;
-      ent[0] = e + tt; ent[1] = e + tt + 8; ent[2] = e + tt + 4; ent[3] = e + tt + 12;
-    } else if (ks < nks) {
-      const int u = (ks - n2w) >> 1, s2 = (ks - n2w) & 1, e = n2 + 32 * u + 8 * s2;
-      ent[0] = e + tt; ent[1] = e + tt + 16; ent[2] = e + tt + 4; ent[3] = e + tt + 20;
-    }
-    const short* et = kent + sl * L.kent_stride;
-    const float i0 = 1.0f / qinv[r0], i1 = 1.0f / qinv[r0 + 8];
-    float v[8];
+  // ---- this warp's value pairs (8-entry tiles wsub, wsub + WPS, ... of slice ws): word offset of
+  // the lane's entry and the in-place mask of its field (bit position p = the entry's shift in its byte)
+  const int n2v = info[4 * ws + 2], nev = n2v + info[4 * ws + 3], ntpv = (nev + 7) >> 3;
+  const int npv = ntpv > wsub ? min(NPW, (ntpv - wsub + WPS - 1) / WPS) : 0;
+  int poff[NPW];
+  uint32_t pmask[NPW];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int ce = ent[k] >= 0 && ent[k] < ne ? et[ent[k]] : -1;
-      const float w2 = ce >= 0 ? ldexpf(1.0f, (ce >> 8) & 15) : 0.0f;
-      const int j = sl * D + (ce & 0xFF);
-      v[2 * k] = ce >= 0 ? qs[r0 * N + j] * w2 * i0 : 0.0f;
-      v[2 * k + 1] = ce >= 0 ? qs[(r0 + 8) * N + j] * w2 * i1 : 0.0f;
+  for (int j = 0; j < NPW; ++j) {
+    const int e = 8 * (wsub + WPS * j) + gq;
+    int widx = 0, qp = 0, sh = 0;
+    uint32_t mm = 0;
+    if (j < npv && e < n2v) {
+      const int f = e & 15;
+      widx = e >> 4;
+      qp = f >> 2;
+      sh = 2 * (f & 3);
+      mm = 0x00030003u;
+    } else if (j < npv && e < nev) {
+      const int e1 = e - n2v, bb = e1 & 31;
+      widx = (n2v >> 4) + (e1 >> 5);
+      qp = bb >> 3;
+      sh = bb & 7;
+      mm = 0x00010001u;
     }
-    // A fragment: a0 = row r0 (k 2t, 2t + 1), a1 = row r0 + 8, a2 = row r0 (k 2t + 8, 2t + 9), a3 = row r0 + 8
-    uint4 hi, lo;
-    split2(v[0], v[2], hi.x, lo.x);
-    split2(v[1], v[3], hi.y, lo.y);
-    split2(v[4], v[6], hi.z, lo.z);
-    split2(v[5], v[7], hi.w, lo.w);
-    qfrag[((sl * a.ks_max + ks) * 32 + ln) * 2] = hi;
-    qfrag[((sl * a.ks_max + ks) * 32 + ln) * 2 + 1] = lo;
+    qp = qp == 1 ? 2 : qp == 2 ? 1 : qp;          // quarter slot of the byte within the quad
+    poff[j] = widx * TILE + qp + 4 * (t >> 1);
+    pmask[j] = mm << sh;
   }
-  __syncthreads();
-  for (int i = tid; i < 16 * N; i += kGAThreads) oc[i] = 0.0f;   // q'' no longer needed
+  const uint32_t psel = (2 * (t & 1)) | 0x40u | ((2 * (t & 1) + 1) << 8) | 0x4000u;   // bytes i0, i0 + 1 -> halves
 
   // ---- record chunks: per tile the key words of slices 0 .. GH-1, then their value words
-  const int n_chunks = (tile_hi - tile_lo) * NCH;
-  const int cw = L.chunk_words;
+  const int n_chunks = 2 * (tile_hi - tile_lo);
+  const int S = a.stages, cw = L.chunk_words;
   auto issue = [&](int u) {
     if (u < n_chunks) {
-      const int tile = tile_lo + u / NCH, c = u % NCH, sl = c % GH, kind = c / GH;
-      const uint32_t* src = a.words + ((slot0 + sl) * 2 + kind) * stream_words + static_cast<size_t>(tile) * cw;
-      uint32_t* dst = ring + (u % kGRing) * cw;
-      for (int p = tid * 4; p < cw; p += kGAThreads * 4) cp_async16(dst + p, src + p);
+      const int tile = tile_lo + (u >> 1), kind = u & 1;
+      uint32_t* dst = ring + (u % S) * GH * cw;
+#pragma unroll
+      for (int sl = 0; sl < GH; ++sl) {
+        const uint32_t* src = a.words + ((slot0 + sl) * 2 + kind) * stream_words + static_cast<size_t>(tile) * cw;
+        for (int p = tid * 4; p < cw; p += kGAThreads * 4) cp_async16(dst + sl * cw + p, src + p);
+      }
     }
     cp_async_commit();
   };
-  for (int u = 0; u < kGRing - 1; ++u) issue(u);
+  for (int u = 0; u < S - 1; ++u) issue(u);
 
-  float sacc[2][4];
-  float oacc[kGDMaxPairs][4];
+  float oacc[NPW][4];
 #pragma unroll
-  for (int pi = 0; pi < kGDMaxPairs; ++pi)
+  for (int j = 0; j < NPW; ++j)
 #pragma unroll
-    for (int r = 0; r < 4; ++r) oacc[pi][r] = 0.0f;
-  const int tw = 16 * warp;
-  const uint32_t m2 = 0x00030003u, m1 = 0x00010001u;
+    for (int r = 0; r < 4; ++r) oacc[j][r] = 0.0f;
+  const int n2k = info[4 * ws], n2wk = n2k >> 4, n1wk = (info[4 * ws + 1] + 31) >> 5;
+  const uint32_t M2 = 0x00030003u << (2 * t), M1 = 0x00010001u << t;
+  const int tb = wsub * 8 * NTK, tw = 16 * warp;
 
   for (int u = 0; u < n_chunks; ++u) {
-    issue(u + kGRing - 1);
-    cp_async_wait<kGRing - 1>();
+    issue(u + S - 1);
+    if (S == 3) cp_async_wait<2>();
+    else cp_async_wait<1>();
     __syncthreads();
-    const int tile = tile_lo + u / NCH, c = u % NCH, sl = c % GH;
-    const uint32_t* ch = ring + (u % kGRing) * cw;
-    const StreamLayout ly = a.lay[pslot0 + 2 * sl + (c < GH ? 0 : 1)];
-    const int n2w = ly.n2 / 16, n1w = (ly.n1 + 31) / 32;
-    if (c < GH) {
-      if (sl == 0)
+    const int tile = tile_lo + (u >> 1);
+    const uint32_t* cs = ring + (u % S) * GH * cw + ws * cw;   // this warp's slice
+    if ((u & 1) == 0) {
+      // ---- slice partial scores of tokens tb .. tb + 8 NTK
+      float sacc[NTK][4];
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
+      for (int nt = 0; nt < NTK; ++nt)
 #pragma unroll
-          for (int r = 0; r < 4; ++r) sacc[nt][r] = 0.0f;
-      const uint4* qa = qfrag + (sl * a.ks_max) * 32 * 2;
-      for (int w = 0; w < n2w; ++w) {
-        const uint4 ah = qa[(w * 32 + lane) * 2], al = qa[(w * 32 + lane) * 2 + 1];
+        for (int r = 0; r < 4; ++r) sacc[nt][r] = 0.0f;
+      uint32_t bk[NTK][2];
+      const uint4* qh = qfh + ws * a.ks_max * 32 + lane;
+      const uint4* ql = qfl + ws * a.ks_max * 32 + lane;
+      for (int w = 0; w < n2wk; ++w) {
+        const uint4 ah = qh[w * 32], al = ql[w * 32];
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt) {
-          const uint32_t x = ch[w * TILE + tw + 8 * nt + gq];
-          const uint32_t b0 = (x >> (2 * t)) & m2, b1 = (x >> (2 * t + 8)) & m2;
-          mma16816(sacc[nt], ah, b0, b1);
-          mma16816(sacc[nt], al, b0, b1);
+        for (int nt = 0; nt < NTK; ++nt) {
+          const uint32_t x = cs[w * TILE + tb + 8 * nt + gq];
+          bk[nt][0] = x & M2;
+          bk[nt][1] = (x >> 8) & M2;
+          mma16816(sacc[nt], ah, bk[nt][0], bk[nt][1]);
         }
+#pragma unroll
+        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al, bk[nt][0], bk[nt][1]);
       }
-      for (int w = 0; w < n1w; ++w) {
+      for (int w = 0; w < n1wk; ++w) {
+        const int ks = n2wk + 2 * w;
+        const uint4 ah0 = qh[ks * 32], al0 = ql[ks * 32], ah1 = qh[ks * 32 + 32], al1 = ql[ks * 32 + 32];
 #pragma unroll
-        for (int s2 = 0; s2 < 2; ++s2) {
-          const int ks = n2w + 2 * w + s2;
-          const uint4 ah = qa[(ks * 32 + lane) * 2], al = qa[(ks * 32 + lane) * 2 + 1];
-#pragma unroll
-          for (int nt = 0; nt < 2; ++nt) {
-            const uint32_t x = ch[(n2w + w) * TILE + tw + 8 * nt + gq];
-            const uint32_t b0 = (x >> (t + 8 * s2)) & m1, b1 = (x >> (t + 4 + 8 * s2)) & m1;
-            mma16816(sacc[nt], ah, b0, b1);
-            mma16816(sacc[nt], al, b0, b1);
-          }
+        for (int nt = 0; nt < NTK; ++nt) {
+          const uint32_t x = cs[(n2wk + w) * TILE + tb + 8 * nt + gq];
+          bk[nt][0] = x;
+          mma16816(sacc[nt], ah0, x & M1, (x >> 4) & M1);
         }
+#pragma unroll
+        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], ah1, (bk[nt][0] >> 8) & M1, (bk[nt][0] >> 12) & M1);
+#pragma unroll
+        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al0, bk[nt][0] & M1, (bk[nt][0] >> 4) & M1);
+#pragma unroll
+        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al1, (bk[nt][0] >> 8) & M1, (bk[nt][0] >> 12) & M1);
       }
-      if (sl == GH - 1) {
-        // ---- online softmax of the tile, raw = acc 2^24 / scale - C.  Lane (gq, t) holds rows gq,
-        // gq + 8 and tokens tw + 8 nt + 2t + {0, 1}; e = s + floor(log2 alpha^V) keeps
-        // P' = 2^(e - m) mant(alpha^V) < 2.
-        float e[2][4], mant[2][4], lav[2][4];
-        float mx0 = -INFINITY, mx1 = -INFINITY;
-        const float q0 = qinv[gq] * 16777216.0f, q1 = qinv[gq + 8] * 16777216.0f;
-        const float c0 = corr[gq], c1 = corr[gq + 8];
+      float* rs = red + ws * 16 * kGRS;
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
+      for (int nt = 0; nt < NTK; ++nt) {
+        const int col = tb + 8 * nt + 2 * t;
+        *reinterpret_cast<float2*>(&rs[gq * kGRS + col]) = make_float2(sacc[nt][0], sacc[nt][1]);
+        *reinterpret_cast<float2*>(&rs[(gq + 8) * kGRS + col]) = make_float2(sacc[nt][2], sacc[nt][3]);
+      }
+      __syncthreads();
+      // ---- online softmax of the tile (warp w < 8: tokens 16 w ..), raw = sum_s acc_s 2^24 scale_s - C.
+      // Lane (gq, t) holds rows gq, gq + 8 and tokens tw + 8 nt + 2t + {0, 1}; e = s + floor(log2 alpha^V)
+      // keeps P' = 2^(e - m) mant(alpha^V) < 2.
+      float e[2][4], mant[2][4], lav[2][4];
+      if (warp < 8) {
+      float sc[2][4];
 #pragma unroll
-          for (int r = 0; r < 4; ++r) {
-            const int tok = tile * TILE + tw + 8 * nt + 2 * t + (r & 1);
-            const int row = r < 2 ? gq : gq + 8;
-            const bool ok = tok < a.n_ctx && row < a.nq;
-            float ev = -INFINITY, mv = 0.0f, lv = 0.0f;
-            if (ok) {
-              const float ak = kalpha[tok], avv = valpha[tok];
-              const float sv = (r < 2 ? fmaf(sacc[nt][r], q0, -c0) : fmaf(sacc[nt][r], q1, -c1)) * ak;
-              int ex = 0;
-              const float fr = frexpf(avv, &ex);
-              lv = avv > 0.0f ? static_cast<float>(max(ex - 1, -64)) : -64.0f;
-              mv = avv > 0.0f ? fr * 2.0f : 0.0f;
-              if (avv > 0.0f && ex - 1 < -64) mv = avv * 18446744073709551616.0f;
-              ev = sv + lv;
-            }
-            e[nt][r] = ev;
-            mant[nt][r] = mv;
-            lav[nt][r] = lv;
-            if (r < 2) mx0 = fmaxf(mx0, ev);
-            else mx1 = fmaxf(mx1, ev);
+      for (int nt = 0; nt < 2; ++nt) {
+        const int col = tw + 8 * nt + 2 * t;
+        float2 s0 = make_float2(0.0f, 0.0f), s1 = make_float2(0.0f, 0.0f);
+#pragma unroll
+        for (int sl = 0; sl < GH; ++sl) {
+          const float2 v0 = *reinterpret_cast<const float2*>(&red[(sl * 16 + gq) * kGRS + col]);
+          const float2 v1 = *reinterpret_cast<const float2*>(&red[(sl * 16 + gq + 8) * kGRS + col]);
+          const float w0 = qsl[gq * GH + sl], w1 = qsl[(gq + 8) * GH + sl];
+          s0.x = fmaf(v0.x, w0, s0.x); s0.y = fmaf(v0.y, w0, s0.y);
+          s1.x = fmaf(v1.x, w1, s1.x); s1.y = fmaf(v1.y, w1, s1.y);
+        }
+        sc[nt][0] = s0.x; sc[nt][1] = s0.y; sc[nt][2] = s1.x; sc[nt][3] = s1.y;
+      }
+      float mx0 = -INFINITY, mx1 = -INFINITY;
+      const float c0 = corr[gq], c1 = corr[gq + 8];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int tok = tile * TILE + tw + 8 * nt + 2 * t + (r & 1);
+          const int row = r < 2 ? gq : gq + 8;
+          const bool ok = tok < a.n_ctx && row < a.nq;
+          float ev = -INFINITY, mv = 0.0f, lv = 0.0f;
+          if (ok) {
+            const float ak = kalpha[tok], avv = valpha[tok];
+            const float sv = (sc[nt][r] - (r < 2 ? c0 : c1)) * ak;
+            int ex = 0;
+            const float fr = frexpf(avv, &ex);
+            lv = avv > 0.0f ? static_cast<float>(max(ex - 1, -64)) : -64.0f;
+            mv = avv > 0.0f ? fr * 2.0f : 0.0f;
+            if (avv > 0.0f && ex - 1 < -64) mv = avv * 18446744073709551616.0f;
+            ev = sv + lv;
           }
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-        if (t == 0) {
-          redm[warp * 16 + gq] = mx0;
-          redm[warp * 16 + gq + 8] = mx1;
+          e[nt][r] = ev;
+          mant[nt][r] = mv;
+          lav[nt][r] = lv;
+          if (r < 2) mx0 = fmaxf(mx0, ev);
+          else mx1 = fmaxf(mx1, ev);
         }
-        __syncthreads();
-        if (tid < 16) {
-          float mt = -INFINITY;
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      if (t == 0) {
+        redm[warp * 16 + gq] = mx0;
+        redm[warp * 16 + gq + 8] = mx1;
+      }
+      }
+      __syncthreads();
+      if (tid < 16) {
+        float mt = -INFINITY;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) mt = fmaxf(mt, redm[w * 16 + tid]);
-          const float mo = mrow[tid], mn = fmaxf(mo, mt);
-          rscale[tid] = mo == -INFINITY ? 0.0f : fexp2(mo - mn);
-          mrow[tid] = mn;
-        }
-        __syncthreads();
-        const float m0 = mrow[gq], m1r = mrow[gq + 8];
-        float ls0 = 0.0f, ls1 = 0.0f, ps0 = 0.0f, ps1 = 0.0f;
-        float p[2][4];
+        for (int w = 0; w < 8; ++w) mt = fmaxf(mt, redm[w * 16 + tid]);
+        const float mo = mrow[tid], mn = fmaxf(mo, mt);
+        rscale[tid] = mo == -INFINITY ? 0.0f : fexp2(mo - mn);
+        mrow[tid] = mn;
+      }
+      __syncthreads();
+      if (warp < 8) {
+      const float m0 = mrow[gq], m1r = mrow[gq + 8];
+      float ls0 = 0.0f, ls1 = 0.0f, ps0 = 0.0f, ps1 = 0.0f;
+      float p[2][4];
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
+      for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-          for (int r = 0; r < 4; ++r) {
-            const float mm = r < 2 ? m0 : m1r;
-            const float x = e[nt][r] == -INFINITY ? 0.0f : fexp2(e[nt][r] - mm);
-            p[nt][r] = x * mant[nt][r];
-            const float l = e[nt][r] == -INFINITY ? 0.0f : x * exp2f(-lav[nt][r]);
-            if (r < 2) ls0 += l;
-            else ls1 += l;
-          }
-        uint4 ph, pl;
-        split2(p[0][0], p[0][1], ph.x, pl.x);
-        split2(p[0][2], p[0][3], ph.y, pl.y);
-        split2(p[1][0], p[1][1], ph.z, pl.z);
-        split2(p[1][2], p[1][3], ph.w, pl.w);
-        pfrag[(warp * 32 + lane) * 2] = ph;
-        pfrag[(warp * 32 + lane) * 2 + 1] = pl;
-        // S': the represented P' (hi + lo) that the value MMAs add
-        {
-          const __half2* hh = reinterpret_cast<const __half2*>(&ph);
-          const __half2* ll = reinterpret_cast<const __half2*>(&pl);
-          float2 v;
-          v = __half22float2(hh[0]); ps0 += v.x + v.y; v = __half22float2(ll[0]); ps0 += v.x + v.y;
-          v = __half22float2(hh[2]); ps0 += v.x + v.y; v = __half22float2(ll[2]); ps0 += v.x + v.y;
-          v = __half22float2(hh[1]); ps1 += v.x + v.y; v = __half22float2(ll[1]); ps1 += v.x + v.y;
-          v = __half22float2(hh[3]); ps1 += v.x + v.y; v = __half22float2(ll[3]); ps1 += v.x + v.y;
+        for (int r = 0; r < 4; ++r) {
+          const float mm = r < 2 ? m0 : m1r;
+          const float x = e[nt][r] == -INFINITY ? 0.0f : fexp2(e[nt][r] - mm);
+          p[nt][r] = x * mant[nt][r];
+          const float l = e[nt][r] == -INFINITY ? 0.0f : x * exp2f(-lav[nt][r]);
+          if (r < 2) ls0 += l;
+          else ls1 += l;
         }
-        ls0 += __shfl_xor_sync(0xffffffffu, ls0, 1);
-        ls0 += __shfl_xor_sync(0xffffffffu, ls0, 2);
-        ls1 += __shfl_xor_sync(0xffffffffu, ls1, 1);
-        ls1 += __shfl_xor_sync(0xffffffffu, ls1, 2);
-        ps0 += __shfl_xor_sync(0xffffffffu, ps0, 1);
-        ps0 += __shfl_xor_sync(0xffffffffu, ps0, 2);
-        ps1 += __shfl_xor_sync(0xffffffffu, ps1, 1);
-        ps1 += __shfl_xor_sync(0xffffffffu, ps1, 2);
-        if (t == 0) {
-          reds[warp * 16 + gq] = ls0;
-          reds[warp * 16 + gq + 8] = ls1;
-          redp[warp * 16 + gq] = ps0;
-          redp[warp * 16 + gq + 8] = ps1;
-        }
-        // value accumulators: rows of D are the queries (c0, c1: row gq; c2, c3: row gq + 8)
-        const float r0 = rscale[gq], r1 = rscale[gq + 8];
+      uint4 ph, pl;
+      split2(p[0][0], p[0][1], ph.x, pl.x);
+      split2(p[0][2], p[0][3], ph.y, pl.y);
+      split2(p[1][0], p[1][1], ph.z, pl.z);
+      split2(p[1][2], p[1][3], ph.w, pl.w);
+      pfh[warp * 32 + lane] = ph;
+      pfl[warp * 32 + lane] = pl;
+      // S': the represented P' (hi + lo) that the value MMAs add
+      {
+        const __half2* hh = reinterpret_cast<const __half2*>(&ph);
+        const __half2* ll = reinterpret_cast<const __half2*>(&pl);
+        float2 v;
+        v = __half22float2(hh[0]); ps0 += v.x + v.y; v = __half22float2(ll[0]); ps0 += v.x + v.y;
+        v = __half22float2(hh[2]); ps0 += v.x + v.y; v = __half22float2(ll[2]); ps0 += v.x + v.y;
+        v = __half22float2(hh[1]); ps1 += v.x + v.y; v = __half22float2(ll[1]); ps1 += v.x + v.y;
+        v = __half22float2(hh[3]); ps1 += v.x + v.y; v = __half22float2(ll[3]); ps1 += v.x + v.y;
+      }
+      ls0 += __shfl_xor_sync(0xffffffffu, ls0, 1);
+      ls0 += __shfl_xor_sync(0xffffffffu, ls0, 2);
+      ls1 += __shfl_xor_sync(0xffffffffu, ls1, 1);
+      ls1 += __shfl_xor_sync(0xffffffffu, ls1, 2);
+      ps0 += __shfl_xor_sync(0xffffffffu, ps0, 1);
+      ps0 += __shfl_xor_sync(0xffffffffu, ps0, 2);
+      ps1 += __shfl_xor_sync(0xffffffffu, ps1, 1);
+      ps1 += __shfl_xor_sync(0xffffffffu, ps1, 2);
+      if (t == 0) {
+        reds[warp * 16 + gq] = ls0;
+        reds[warp * 16 + gq + 8] = ls1;
+        redp[warp * 16 + gq] = ps0;
+        redp[warp * 16 + gq + 8] = ps1;
+      }
+      }
+      // value accumulators: rows of D are the queries (c0, c1: row gq; c2, c3: row gq + 8)
+      const float r0 = rscale[gq], r1 = rscale[gq + 8];
 #pragma unroll
-        for (int pi = 0; pi < kGDMaxPairs; ++pi) {
-          oacc[pi][0] *= r0;
-          oacc[pi][1] *= r0;
-          oacc[pi][2] *= r1;
-          oacc[pi][3] *= r1;
-        }
-        __syncthreads();
-        if (tid < 16) {
-          float lt = 0.0f, pt = 0.0f;
+      for (int j = 0; j < NPW; ++j) {
+        oacc[j][0] *= r0;
+        oacc[j][1] *= r0;
+        oacc[j][2] *= r1;
+        oacc[j][3] *= r1;
+      }
+      __syncthreads();
+      if (tid < 16) {
+        float lt = 0.0f, pt = 0.0f;
 #pragma unroll
-          for (int w = 0; w < 8; ++w) {
-            lt += reds[w * 16 + tid];
-            pt += redp[w * 16 + tid];
-          }
-          lrow[tid] = lrow[tid] * rscale[tid] + lt;
-          srow[tid] = srow[tid] * rscale[tid] + pt;
+        for (int w = 0; w < 8; ++w) {
+          lt += reds[w * 16 + tid];
+          pt += redp[w * 16 + tid];
         }
+        lrow[tid] = lrow[tid] * rscale[tid] + lt;
+        srow[tid] = srow[tid] * rscale[tid] + pt;
       }
     } else {
-      // ---- O_e += P' . digit_e for this warp's (slice, 8-entry tile) pairs of slice sl
-      const int ne = ly.n2 + ly.n1;
+      // ---- O_e += P' . field_e 2^p over this warp's pairs, P' loaded once per k-step
+      uint32_t bv[NPW][2];
 #pragma unroll
-      for (int pi = 0; pi < kGDMaxPairs; ++pi) {
-        const int pr = warp + 8 * pi;
-        if (pr >= a.n_pairs) break;
-        // pairs are numbered slice-major: pr = sl' * ntp + nt with ntp n-tiles per slice
-        const int ntp = (a.ks_max * 16 + 7) / 8;
-        const int p_sl = pr / ntp, p_nt = pr % ntp;
-        if (p_sl != sl) continue;
-        const int e = 8 * p_nt + gq;               // this lane's entry (B column gq)
-        uint32_t widx = 0, shb = 0, msk = 0;
-        int qpos = 0;
-        if (e < ly.n2) {
-          const int f = e & 15;
-          widx = e >> 4;
-          qpos = (f >> 2) == 1 ? 2 : (f >> 2) == 2 ? 1 : (f >> 2);
-          shb = 2 * (f & 3);
-          msk = 3u;
-        } else if (e < ne) {
-          const int e1 = e - ly.n2, bb = e1 & 31;
-          widx = n2w + (e1 >> 5);
-          qpos = (bb >> 3) == 1 ? 2 : (bb >> 3) == 2 ? 1 : (bb >> 3);
-          shb = bb & 7;
-          msk = 1u;
-        }
-        const uint32_t mlo = msk, mhi = msk << 16;
-        const uint32_t* wr = ch + widx * TILE + qpos;
-        const int i0 = 2 * (t & 1);
+      for (int kt = 0; kt < TILE / 16; ++kt) {
+        const uint4 ah = pfh[kt * 32 + lane], al = pfl[kt * 32 + lane];
 #pragma unroll
-        for (int kt = 0; kt < TILE / 16; ++kt) {
-          const uint32_t x0 = wr[4 * (4 * kt + (t >> 1))], x1 = wr[4 * (4 * kt + 2 + (t >> 1))];
-          const uint32_t y0 = x0 >> (8 * i0 + shb), y1 = x1 >> (8 * i0 + shb);
-          const uint32_t b0 = (y0 & mlo) | ((y0 << 8) & mhi), b1 = (y1 & mlo) | ((y1 << 8) & mhi);
-          const uint4 ah = pfrag[(kt * 32 + lane) * 2], al = pfrag[(kt * 32 + lane) * 2 + 1];
-          mma16816(oacc[pi], ah, b0, b1);
-          mma16816(oacc[pi], al, b0, b1);
+        for (int j = 0; j < NPW; ++j) {
+          if (j < npv) {
+            const uint32_t x0 = cs[poff[j] + 16 * kt], x1 = cs[poff[j] + 16 * kt + 8];
+            bv[j][0] = __byte_perm(x0, 0u, psel) & pmask[j];
+            bv[j][1] = __byte_perm(x1, 0u, psel) & pmask[j];
+            mma16816(oacc[j], ah, bv[j][0], bv[j][1]);
+          }
         }
+#pragma unroll
+        for (int j = 0; j < NPW; ++j)
+          if (j < npv) mma16816(oacc[j], al, bv[j][0], bv[j][1]);
       }
     }
     __syncthreads();
   }
   cp_async_wait<0>();
+  __syncthreads();
 
   // ---- entry sums -> channel sums (shared-memory adds), then the split's partials
+  float* oc = reinterpret_cast<float*>(ring);     // [16][N]
+  for (int i = tid; i < 16 * N; i += kGAThreads) oc[i] = 0.0f;
+  __syncthreads();
   {
-    const int ntp = (a.ks_max * 16 + 7) / 8;
+    const short* et = a.entry + static_cast<size_t>(pslot0 + 2 * ws + 1) * a.n_entries;
 #pragma unroll
-    for (int pi = 0; pi < kGDMaxPairs; ++pi) {
-      const int pr = warp + 8 * pi;
-      if (pr >= a.n_pairs) break;
-      const int p_sl = pr / ntp, p_nt = pr % ntp;
-      const short* et = a.entry + static_cast<size_t>(pslot0 + 2 * p_sl + 1) * a.n_entries;
-      const StreamLayout ly = a.lay[pslot0 + 2 * p_sl + 1];
+    for (int j = 0; j < NPW; ++j) {
+      if (j >= npv) break;
 #pragma unroll
       for (int k = 0; k < 2; ++k) {
-        const int e = 8 * p_nt + 2 * t + k;        // D column 2t + k
-        const int ce = e < ly.n2 + ly.n1 ? et[e] : -1;
+        const int e = 8 * (wsub + WPS * j) + 2 * t + k;   // D column 2t + k
+        const int ce = e < nev ? et[e] : -1;
         if (ce < 0) continue;
-        const float w2 = ldexpf(1.0f, ((ce >> 8) & 15) + 24);   // digits entered as d 2^-24
-        const int j = p_sl * D + (ce & 0xFF);
-        if (gq < a.nq) atomicAdd(&oc[gq * N + j], w2 * oacc[pi][k]);
-        if (gq + 8 < a.nq) atomicAdd(&oc[(gq + 8) * N + j], w2 * oacc[pi][2 + k]);
+        const int p = e < n2v ? 2 * (e & 3) : (e - n2v) & 7;   // the field's bit position in its byte
+        const float w2 = ldexpf(1.0f, ((ce >> 8) & 15) + 24 - p);   // fields entered as d 2^(p - 24)
+        const int jj = ws * D + (ce & 0xFF);
+        if (gq < a.nq) atomicAdd(&oc[gq * N + jj], w2 * oacc[j][k]);
+        if (gq + 8 < a.nq) atomicAdd(&oc[(gq + 8) * N + jj], w2 * oacc[j][2 + k]);
       }
     }
   }
@@ -497,21 +580,24 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
   }
 }
 
-// Per (query head, group, sequence), 512 threads: combine the splits (weights 2^(m_s - M)),
-// o_hat_j = f^V_j O_j / l (thread = channel), then out = U_V[block rows] o_hat with four threads
-// per output dim, each over a quarter of the channels.
+// Per (query head i, slice s, group, sequence), 512 threads: combine the splits (weights
+// 2^(m_s - M), l = sum w_s l_s), o_hat_j' = f^V_j' sum_s w_s O_s,j' over the slice's 128 channels
+// (4 quarters of the splits), then the slice's part of U_V[block m rows] o_hat (4 quarters of the
+// channels).  The CTA that arrives last for (i, group, sequence) adds the g_h parts in slice order
+// and divides by l, so the result does not depend on the arrival order.
 constexpr int kGMThreads = 512;
 __global__ void __launch_bounds__(kGMThreads) aatc_group_merge_kernel(const GroupDecodeArgs a) {
-  extern __shared__ float msm[];                  // ohat [n], w [n_splits], part [4][128]
-  float* ohat = msm;
-  float* wsp = msm + a.n;
-  float* psum = wsp + ((a.n_splits + 3) & ~3);
+  extern __shared__ float wsp[];                  // w [n_splits]
   __shared__ float red[kGMThreads / 32];
+  __shared__ float part[4][D];
+  __shared__ float ohat[D];
   __shared__ float s_l;
-  const int i = blockIdx.x, g = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
-  const int N = a.n, m = i / a.group;
+  __shared__ int s_last;
+  const int i = blockIdx.x, s = blockIdx.y % a.gh, g = blockIdx.y / a.gh, b = blockIdx.z, tid = threadIdx.x;
+  const int N = a.n, m = i / a.group, c = tid & (D - 1), q4 = tid >> 7;
+  const size_t bg = static_cast<size_t>(b) * a.n_groups + g;
   const size_t pstride = static_cast<size_t>(N) + 4;
-  const float* pb = a.part + (((static_cast<size_t>(b) * a.n_groups + g) * a.nq + i) * a.n_splits) * pstride;
+  const float* pb = a.part + ((bg * a.nq + i) * a.n_splits) * pstride;
   // M = max_s m_s (block reduction), then w_s and l = sum_s w_s l_s
   float mloc = -INFINITY;
   for (int s2 = tid; s2 < a.n_splits; s2 += kGMThreads) mloc = fmaxf(mloc, pb[s2 * pstride + N]);
@@ -536,35 +622,52 @@ __global__ void __launch_bounds__(kGMThreads) aatc_group_merge_kernel(const Grou
     for (int w = 0; w < kGMThreads / 32; ++w) l += red[w];
     s_l = l;
   }
-  for (int j = tid; j < N; j += kGMThreads) {
-    float o0 = 0.0f, o1 = 0.0f;
-    int s2 = 0;
-    for (; s2 + 1 < a.n_splits; s2 += 2) {
-      o0 = fmaf(wsp[s2], pb[s2 * pstride + j], o0);
-      o1 = fmaf(wsp[s2 + 1], pb[(s2 + 1) * pstride + j], o1);
+  // o_hat over the slice's channels: quarter q4 takes splits q4, q4 + 4, ...
+  {
+    const float* pc = pb + s * D + c;
+    float o[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int s0 = q4; s0 < a.n_splits; s0 += 4 * 24) {   // 24 loads in flight per thread
+      float x[24];
+#pragma unroll
+      for (int k = 0; k < 24; ++k) x[k] = s0 + 4 * k < a.n_splits ? pc[static_cast<size_t>(s0 + 4 * k) * pstride] : 0.0f;
+#pragma unroll
+      for (int k = 0; k < 24; ++k)
+        if (s0 + 4 * k < a.n_splits) o[k & 3] = fmaf(wsp[s0 + 4 * k], x[k], o[k & 3]);
     }
-    if (s2 < a.n_splits) o0 = fmaf(wsp[s2], pb[s2 * pstride + j], o0);
-    const int sl = j / D, c = j % D;
-    const int slot = (a.layer * a.n_kv + g * a.gh + sl) * 2 + 1;
-    ohat[j] = (o0 + o1) * a.f[slot * D + c];
+    part[q4][c] = (o[0] + o[1]) + (o[2] + o[3]);
   }
   __syncthreads();
-  const int d = tid & (D - 1), part = tid >> 7, span = N / 4;
-  const float* u = a.uvt + (static_cast<size_t>(a.layer) * a.n_groups + g) * static_cast<size_t>(N) * N +
-                   static_cast<size_t>(m) * D + d;
-  float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-  for (int j = part * span; j < (part + 1) * span; j += 16) {   // 16 loads in flight per thread
-    float x[16];
-#pragma unroll
-    for (int k = 0; k < 16; ++k) x[k] = u[static_cast<size_t>(j + k) * N];
-#pragma unroll
-    for (int k = 0; k < 16; ++k) acc[k & 3] = fmaf(x[k], ohat[j + k], acc[k & 3]);
+  if (tid < D) {
+    const int slot = (a.layer * a.n_kv + g * a.gh + s) * 2 + 1;
+    ohat[c] = ((part[0][c] + part[1][c]) + (part[2][c] + part[3][c])) * a.f[slot * D + c];
   }
-  psum[part * D + d] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
   __syncthreads();
-  if (tid < D)
-    a.out[(static_cast<size_t>(b) * a.n_q_heads + g * a.nq + i) * D + tid] =
-        ((psum[tid] + psum[D + tid]) + (psum[2 * D + tid] + psum[3 * D + tid])) / s_l;
+  // the slice's part of U_V[block m rows] o_hat: quarter q4 takes channels 32 q4 .. 32 q4 + 31
+  {
+    const float* u = a.uvt + (static_cast<size_t>(a.layer) * a.n_groups + g) * static_cast<size_t>(N) * N +
+                     static_cast<size_t>(s * D + 32 * q4) * N + static_cast<size_t>(m) * D + c;
+    float x[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) x[k] = u[static_cast<size_t>(k) * N];   // 32 loads in flight per thread
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+    for (int k = 0; k < 32; ++k) acc[k & 3] = fmaf(x[k], ohat[32 * q4 + k], acc[k & 3]);
+    part[q4][c] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  }
+  __syncthreads();
+  float* op = a.outp + (bg * 16 + i) * a.gh * D;
+  if (tid < D) op[s * D + c] = (part[0][c] + part[1][c]) + (part[2][c] + part[3][c]);
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(&a.ticket[bg * 16 + i], 1) == a.gh - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (tid < D) {
+    float o = 0.0f;
+    for (int s2 = 0; s2 < a.gh; ++s2) o += __ldcg(&op[s2 * D + c]);
+    a.out[(static_cast<size_t>(b) * a.n_q_heads + g * a.nq + i) * D + c] = o / s_l;
+  }
 }
 
 int group_splits(const Plan& plan, int batch, int n_ctx) {
@@ -574,7 +677,7 @@ int group_splits(const Plan& plan, int batch, int n_ctx) {
 }
 
 struct GroupWs {
-  size_t qf_off, part_off, bytes;
+  size_t frag_off, qsc_off, outp_off, ticket_off, part_off, bytes;
 };
 // k-steps (D2 words + 2 x D1 words) of the widest slice stream of `layer` (keys or values)
 int group_ks_max(const Plan& plan, int layer) {
@@ -590,10 +693,18 @@ int group_ks_max(const Plan& plan, int layer) {
 GroupWs group_ws_layout(const Plan& plan, int batch, int n_ctx) {
   const int ng = plan.dims.n_kv_heads / plan.group_heads, n = D * plan.group_heads;
   const int nq = plan.dims.n_q_heads / ng;
+  int ks = 1;                                     // the widest layer's k-steps size the fragment tables
+  for (int l = 0; l < plan.dims.n_layers; ++l) ks = std::max(ks, group_ks_max(plan, l));
   GroupWs w;
   size_t off = 0;
-  w.qf_off = off;
-  off += static_cast<size_t>(batch) * ng * nq * n * 4;
+  w.frag_off = off;
+  off += static_cast<size_t>(batch) * ng * 2 * plan.group_heads * ks * 128 * 4;
+  w.qsc_off = off;
+  off += static_cast<size_t>(batch) * ng * 16 * plan.group_heads * 2 * 4;
+  w.outp_off = off;
+  off += static_cast<size_t>(batch) * ng * 16 * plan.group_heads * D * 4;
+  w.ticket_off = off;
+  off += static_cast<size_t>(batch) * ng * 16 * 4;
   off = (off + 255) / 256 * 256;
   w.part_off = off;
   off += static_cast<size_t>(batch) * ng * nq * group_splits(plan, batch, n_ctx) * (n + 4) * 4;
@@ -617,7 +728,10 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   a.uk = plan.gdev.uk;
   a.uvt = plan.gdev.uvt;
   a.f = plan.dev.f;
-  a.qf = reinterpret_cast<float*>(static_cast<char*>(ws) + wl.qf_off);
+  a.qfrag = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + wl.frag_off);
+  a.qsc = reinterpret_cast<float*>(static_cast<char*>(ws) + wl.qsc_off);
+  a.outp = reinterpret_cast<float*>(static_cast<char*>(ws) + wl.outp_off);
+  a.ticket = reinterpret_cast<int*>(static_cast<char*>(ws) + wl.ticket_off);
   a.part = reinterpret_cast<float*>(static_cast<char*>(ws) + wl.part_off);
   a.out = out;
   a.layer = layer;
@@ -639,24 +753,35 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   a.n_words = plan.n_words;
   a.n_entries = plan.n_entries;
   a.ks_max = group_ks_max(plan, layer);
-  a.n_pairs = gh * 2 * a.ks_max;                 // (slice, 8-entry tile) pairs of the value records
-  if (a.nq > 16 || a.n_pairs > 8 * kGDMaxPairs) return cudaErrorNotSupported;
-  aatc_group_query_kernel<<<dim3(a.nq, a.n_groups, batch), a.n, 0, st>>>(a);
+  // value pairs per warp: 8-entry tiles of the widest value slice over the 8 / g_h warps of a slice
+  int ntp = 1;
+  for (int h = 0; h < a.n_kv; ++h) {
+    const StreamLayout& ly = plan.layout[(layer * a.n_kv + h) * 2 + 1];
+    ntp = std::max(ntp, (ly.n2 + ly.n1 + 7) / 8);
+  }
+  const int npw = (ntp + 16 / gh - 1) / (16 / gh);
+  a.stages = 3;
+  if (GroupDigitSmem(gh, a.ks_max, a.n_words, 3).total > 227 * 1024) a.stages = 2;
+  const size_t smem = static_cast<size_t>(GroupDigitSmem(gh, a.ks_max, a.n_words, a.stages).total);
+  if (a.nq > 16 || npw > 12 || smem > 227 * 1024) return cudaErrorNotSupported;
+  aatc_group_query_kernel<<<dim3(16, a.n_groups * gh, batch), kGQThreads, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 grid(a.n_splits, a.n_groups, batch);
-  const size_t smem = static_cast<size_t>(GroupDigitSmem(gh, a.ks_max, a.n_words, a.n_entries).total);
-  if (smem > 227 * 1024) return cudaErrorNotSupported;
-  const void* kern = gh == 2 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2>)
-                             : reinterpret_cast<const void*>(aatc_group_digit_kernel<4>);
+  const void* kern = gh == 2 ? (npw <= 6 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 6>)
+                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 12>))
+                             : (npw <= 6 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 6>)
+                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 12>));
   e = ensure_smem_optin(kern, smem);
   if (e != cudaSuccess) return e;
-  if (gh == 2) aatc_group_digit_kernel<2><<<grid, kGAThreads, smem, st>>>(a);
-  else aatc_group_digit_kernel<4><<<grid, kGAThreads, smem, st>>>(a);
+  if (gh == 2 && npw <= 6) aatc_group_digit_kernel<2, 6><<<grid, kGAThreads, smem, st>>>(a);
+  else if (gh == 2) aatc_group_digit_kernel<2, 12><<<grid, kGAThreads, smem, st>>>(a);
+  else if (npw <= 6) aatc_group_digit_kernel<4, 6><<<grid, kGAThreads, smem, st>>>(a);
+  else aatc_group_digit_kernel<4, 12><<<grid, kGAThreads, smem, st>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const size_t msm = (static_cast<size_t>(a.n) + ((a.n_splits + 3) & ~3) + 4 * D) * 4;
-  aatc_group_merge_kernel<<<dim3(a.nq, a.n_groups, batch), kGMThreads, msm, st>>>(a);
+  const size_t msm = static_cast<size_t>(a.n_splits) * 4;
+  aatc_group_merge_kernel<<<dim3(a.nq, a.n_groups * gh, batch), kGMThreads, msm, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -52,10 +52,12 @@ def _slice_codes(u32, plan, cfg, g_h, max_tokens, b, g, kind, t0, n, bits):
     return codes, alphas, recs
 
 
-@pytest.mark.parametrize("g_h,n_kv,n_q", [(4, 8, 32), (2, 4, 16)])
-def test_group_encode_decode_matches_oracle(aatc, g_h, n_kv, n_q):
-    cfg = W.Config(8, "groups", 1, n_kv, n_q, 1, 700, (2.75,), 1, "head-group plan")
-    plan, basis, bits, scales = _group_plan(aatc, cfg, g_h)
+@pytest.mark.parametrize("g_h,n_kv,n_q,avg_bits", [(4, 8, 32, 2.75), (2, 4, 16, 2.75), (4, 4, 16, 5.0), (2, 2, 8, 7.0)])
+def test_group_encode_decode_matches_oracle(aatc, g_h, n_kv, n_q, avg_bits):
+    """2.75 bits: the common decode variant; 5 and 7 bits: more value entries per slice than one
+    pair set per warp holds (the wider variant) and longer records."""
+    cfg = W.Config(8, "groups", 1, n_kv, n_q, 1, 700, (avg_bits,), 1, "head-group plan")
+    plan, basis, bits, scales = _group_plan(aatc, cfg, g_h, avg_bits)
     T, max_tokens = 653, 700
     k, v = W.kv_host(cfg, 0, 1, T)
     kd = torch.from_numpy(k).to(DEV).to(torch.bfloat16)
@@ -96,7 +98,7 @@ def test_group_encode_decode_matches_oracle(aatc, g_h, n_kv, n_q):
                 bs = b_g[s::g_h]
                 h[:, s::g_h] = O.dequantize_f32(O.unpack_records(recs[s], bs), alphas[s], scales[0, g, kind][s::g_h], bs)
             coeffs[(g, kind)] = h
-    name = f"head groups (g_h {g_h}, {n_kv} kv-heads, {T} tokens)"
+    name = f"head groups (g_h {g_h}, {n_kv} kv-heads, {T} tokens, {avg_bits} bits)"
     Hn.NearThreshold.add(name, mis, tot)
     Hn.NearThreshold.assert_bound(name)
     for peaky in (1.0, 8.0):
