@@ -721,6 +721,9 @@ __global__ void __launch_bounds__(kThreads)
 //    values first.  m is only a reference point: o = sum P' code and l = sum p share it, and the
 //    merge rescales both alike.
 __host__ __device__ constexpr int fused_stage_bytes(int wu) { return 2 * wu * TILE * 4 + 2 * TILE * 4; }
+// row pitch of the per-query entry sums in the epilogue: = 8 (mod 16), so the four queries of a
+// lane quad (rows t = 0..3) fall in distinct banks
+__host__ __device__ constexpr int fused_entry_pitch(int n_entries) { return ((n_entries + 7) / 8 * 8) | 8; }
 constexpr float kPScale = 32.0f;            // P' < 2^9 times 2^5: f16 operands below 2^14
 
 struct FusedSmem {
@@ -731,7 +734,7 @@ struct FusedSmem {
     bars = o;  o = align16(o + 8 * wg * n_stages);
     cnt = o;   o = align16(o + 4 * wg * n_stages);
     qf = o;    o += nks * np * 32 * 8;                        // query B fragments [ks][p][lane]
-    qc = o;    o += 2 * MAX_GROUP * 4;                        // C_g, score scales
+    qc = o;    o += 2 * MAX_GROUP * 4 + D * 4;                // C_g, score scales; value offsets 2^(b_c - 1)
     pf = o;    o += warps * 2 * np * 32 * 8;                  // P' B fragments [warp][ks][p][lane]
     cetab = o; o += D * 8 * 2;                                // value channel -> record entries
     etab = o;  o = align16(o + n_entries * 2);                // value entry table
@@ -740,8 +743,10 @@ struct FusedSmem {
     o = (o + 127) & ~127;
     ring = o;
     const int rings = wg * n_stages * fused_stage_bytes(wu);
-    // after the loop the rings hold each warp's (m, l, S', entry sums) per query
-    const int epi = warps * (3 * MAX_GROUP + gmax * n_entries) * 4;
+    // after the loop the rings hold each warp's (m, l, S', entry sums) per query, the warps'
+    // factors 2^(m_w - M), the totals (M, l, S') and the entry sums over the warps
+    const int nep = fused_entry_pitch(n_entries);
+    const int epi = (warps * (3 * MAX_GROUP + gmax * nep) + warps * gmax + 3 * gmax + gmax * nep) * 4;
     total = ring + (rings > epi ? rings : epi);
   }
 };
@@ -834,6 +839,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   for (int k = 0; k < RR; ++k) u0[k] = __ldg(uk + k * D);
   const float fk = a.f[sk * D + c];
   const float offk = a.enc[sk * D + c].off;                     // 2^(b_c - 1), 0 if b_c = 0
+  if (tid < D) reinterpret_cast<float*>(smb + L.qc)[2 * MAX_GROUP + tid] = a.enc[sv * D + tid].off;
   const StreamLayout lk = a.lay[sk];
   if (tid < WG * NS) reinterpret_cast<int*>(smb + L.cnt)[tid] = 0;
   // everything below may read what the preceding grid in the stream wrote (cache, q, workspace)
@@ -952,10 +958,12 @@ __global__ void __launch_bounds__(128 * WG, 1)
     }
   }
   const float* qc = reinterpret_cast<const float*>(smb + L.qc);
-  if (leader)
-    for (int j = 1; j < min(NS, n_j); ++j) issue(j, j);
   ptx::grid_launch_dependents();
   __syncthreads();
+  // the rest of each group's ring: lane 0 of the group's last warp, which starts its first tile
+  // after the other three (they need only the tile issued before the fold)
+  if ((tid & 127) == 96)
+    for (int j = 1; j < min(NS, n_j); ++j) issue(j, j);
 
   // masks: scores (lane t's fields of a k-step), values (lane row g's fields of an M-tile)
   const uint32_t km2 = 0x00030003u << (2 * t);
@@ -1158,9 +1166,10 @@ __global__ void __launch_bounds__(128 * WG, 1)
   }
   // ---- per-warp (m, l, S') and entry sums into the drained rings
   float* epi = reinterpret_cast<float*>(smb + L.ring);
-  const int NE = a.n_entries;
-  constexpr int kEpiStride = 3 * MAX_GROUP;                  // + GMAX * NE floats per warp
-  float* wm = epi + warp * (kEpiStride + GMAX * NE);         // [m, l, S'][MAX_GROUP], then E[GMAX][NE]
+  const int NE = a.n_entries, NEP = fused_entry_pitch(NE);
+  constexpr int kEpiStride = 3 * MAX_GROUP;                  // + GMAX * NEP floats per warp
+  const int wstride = kEpiStride + GMAX * NEP;               // per-warp block: (m, l, S'), then E
+  float* wm = epi + warp * wstride;                          // [m, l, S'][MAX_GROUP], then E[GMAX][NEP]
   float* wE = wm + kEpiStride;
 #pragma unroll
   for (int p = 0; p < NP; ++p) {
@@ -1193,46 +1202,84 @@ __global__ void __launch_bounds__(128 * WG, 1)
       }
 #pragma unroll
       for (int p = 0; p < NP; ++p) {
-        float* dst = wE + (4 * p + t) * NE;
+        float* dst = wE + (4 * p + t) * NEP;
         if (e < NE) dst[e] = (vacc[jj][p][0] + vacc[jj][p][1]) * sc;
         if (e + 8 < NE) dst[e + 8] = (vacc[jj][p][2] + vacc[jj][p][3]) * sc;
       }
     }
   }
   __syncthreads();
+  // ---- the CTA maximum M per query, each warp's factor 2^(m_w - M) and the totals l and S'
+  // (warp q, lane w = warp w's values), then the entry sums over the warps (each warp's sums
+  // scaled once, in a fixed order)
+  float* ff = epi + NW * wstride;                            // [NW][GMAX]
+  float* tot = ff + NW * GMAX;                               // [M, l, S'][GMAX]
+  float* etot = tot + 3 * GMAX;                              // [GMAX][NEP]
+  if (warp < GMAX) {
+    const float* ww = epi + (lane < NW ? lane : 0) * wstride;
+    const float mw = lane < NW ? ww[warp] : -INFINITY;
+    float M = mw;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float f = mw > -INFINITY ? fast_exp2(mw - M) : 0.0f;
+    float l = lane < NW ? f * ww[MAX_GROUP + warp] : 0.0f;
+    float sp = lane < NW ? f * ww[2 * MAX_GROUP + warp] : 0.0f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      l += __shfl_xor_sync(0xffffffffu, l, o);
+      sp += __shfl_xor_sync(0xffffffffu, sp, o);
+    }
+    if (lane < NW) ff[lane * GMAX + warp] = f;
+    if (lane == 0) {
+      tot[warp] = M;
+      tot[GMAX + warp] = l;
+      tot[2 * GMAX + warp] = sp;
+    }
+  }
+  __syncthreads();
+  for (int i4 = tid; i4 < GMAX * NEP / 4; i4 += NT) {         // four entries of one query row
+    const int idx = 4 * i4, q = idx / NEP;
+    float4 ev[NW];
+    float fw[NW];
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {                           // all loads first, then the sums
+      ev[w] = *reinterpret_cast<const float4*>(epi + w * wstride + kEpiStride + idx);
+      fw[w] = ff[w * GMAX + q];
+    }
+    float4 e0 = make_float4(0.0f, 0.0f, 0.0f, 0.0f), e1 = e0;
+#pragma unroll
+    for (int w = 0; w < NW; w += 2) {
+      e0.x = fmaf(fw[w], ev[w].x, e0.x); e0.y = fmaf(fw[w], ev[w].y, e0.y);
+      e0.z = fmaf(fw[w], ev[w].z, e0.z); e0.w = fmaf(fw[w], ev[w].w, e0.w);
+      e1.x = fmaf(fw[w + 1], ev[w + 1].x, e1.x); e1.y = fmaf(fw[w + 1], ev[w + 1].y, e1.y);
+      e1.z = fmaf(fw[w + 1], ev[w + 1].z, e1.z); e1.w = fmaf(fw[w + 1], ev[w + 1].w, e1.w);
+    }
+    *reinterpret_cast<float4*>(etot + idx) = make_float4(e0.x + e1.x, e0.y + e1.y, e0.z + e1.z, e0.w + e1.w);
+  }
+  __syncthreads();
   // ---- the split's partial per query: thread = (value channel c, query parity part)
   const size_t pbase = (static_cast<size_t>(b) * a.n_q + head * G) * a.n_splits;
   {
     const uint4 cev = *reinterpret_cast<const uint4*>(cetab + c * 8);
-    const short* ce = reinterpret_cast<const short*>(&cev);
+    const uint32_t cw4[4] = {cev.x, cev.y, cev.z, cev.w};
     float w8[8];
     int e8[8];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      e8[k] = min(max(static_cast<int>(ce[k]), 0), NE - 1);
-      w8[k] = ce[k] >= 0 ? pow2i((etab[e8[k]] >> 8) & 15) : 0.0f;
+    for (int k = 0; k < 8; ++k) {                            // entry k of channel c: short k of the row
+      const int ce = static_cast<short>(cw4[k >> 1] >> (16 * (k & 1)));
+      e8[k] = min(max(ce, 0), NE - 1);
+      w8[k] = ce >= 0 ? pow2i((etab[e8[k]] >> 8) & 15) : 0.0f;
     }
-    const float off = a.enc[sv * D + c].off;
+    const float off = reinterpret_cast<const float*>(smb + L.qc)[2 * MAX_GROUP + c];
     for (int q = part; q < G; q += WG) {
-      float M = -INFINITY;
+      float o = -off * tot[2 * GMAX + q];
 #pragma unroll
-      for (int w = 0; w < NW; ++w) M = fmaxf(M, epi[w * (kEpiStride + GMAX * NE) + q]);
-      float o = 0.0f, l = 0.0f;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) {
-        const float* ww = epi + w * (kEpiStride + GMAX * NE);
-        const float f = ww[q] > -INFINITY ? fast_exp2(ww[q] - M) : 0.0f;
-        float ow = -off * ww[2 * MAX_GROUP + q];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) ow = fmaf(w8[k], ww[kEpiStride + q * NE + e8[k]], ow);
-        o = fmaf(f, ow, o);
-        l = fmaf(f, ww[MAX_GROUP + q], l);
-      }
+      for (int k = 0; k < 8; ++k) o = fmaf(w8[k], etot[q * NEP + e8[k]], o);
       float* dst = a.ws + (pbase + static_cast<size_t>(q) * a.n_splits + split) * a.pstride;
       dst[c] = o;
       if (c == 0) {
-        dst[D] = M;
-        dst[D + 1] = l;
+        dst[D] = tot[q];
+        dst[D + 1] = tot[GMAX + q];
       }
     }
   }
