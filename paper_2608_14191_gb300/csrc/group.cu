@@ -32,7 +32,7 @@ namespace aatc {
 namespace {
 
 constexpr float kGLog2e = 1.4426950408889634f;
-constexpr int kGAThreads = 512;                  // 16 warps; warps 0-7 also run the softmax (16 tokens each)
+constexpr int kGAThreads = 256;                  // 8 warps; each also runs the softmax of 16 tokens
 
 struct GroupDecodeArgs {
   const float* alpha;        // cache alpha region [b][n_kv][K|V][n_tiles * 128]
@@ -65,7 +65,7 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ void mma16816(float (&c)[4], const uint4& a, uint32_t b0, uint32_t b1) {
-  asm(
+  asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
       "{%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
@@ -187,12 +187,12 @@ __global__ void __launch_bounds__(kGQThreads) aatc_group_query_kernel(const Grou
 // digit (or a single bit) masked into a 16-bit half is the subnormal f16 value d 2^(p - 24), p its
 // bit position in the half; the power 2^p is folded into the other operand's scale.
 //   chunks: per tile, the key words of all g_h slices, then their value words (cp.async ring)
-//   scores: warp (slice sl, part) over its slice's k-steps and 4 (g_h = 4) or 2 (g_h = 2)
+//   scores: warp (slice sl, part) over its slice's k-steps and 8 (g_h = 4) or 4 (g_h = 2)
 //           token n-tiles: A = q''_c 2^shift per entry (rows = queries, hi / lo, lane t's columns
 //           scaled by 2^-2t for D2 words, 2^-t for D1 words), B = the tokens' fields masked in
 //           place; the slice partials meet in shared memory and are summed per token, then
 //           raw = sum q'' u, s = alpha^K (raw - C) with C = sum_c q''_c 2^(b_c - 1)
-//   values: warp (slice sl, part) owns the 8-entry tiles part, part + 16 / g_h, ... of slice sl:
+//   values: warp (slice sl, part) owns the 8-entry tiles part, part + 8 / g_h, ... of slice sl:
 //           A = P' (queries x 16 tokens, hi / lo, loaded once per k-step), B = the entries'
 //           fields of those tokens from the quad-interleaved value slots (byte permute + mask);
 //           the entry sums become channel sums o_c = sum_e 2^(shift - p) O_e - 2^(b_c - 1) S'
@@ -221,7 +221,7 @@ struct GroupDigitSmem {
 
 template <int GH, int NPW>
 __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const GroupDecodeArgs a) {
-  constexpr int N = D * GH, WPS = 16 / GH, NTK = TILE / (8 * WPS);   // warps per slice, key n-tiles per warp
+  constexpr int N = D * GH, WPS = 8 / GH, NTK = TILE / (8 * WPS);   // warps per slice, key n-tiles per warp
   extern __shared__ __align__(128) unsigned char smb[];
   const GroupDigitSmem L(GH, a.ks_max, a.n_words, a.stages);
   uint4* qfh = reinterpret_cast<uint4*>(smb + L.qfh);
@@ -348,7 +348,6 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
       for (int nt = 0; nt < NTK; ++nt)
 #pragma unroll
         for (int r = 0; r < 4; ++r) sacc[nt][r] = 0.0f;
-      uint32_t bk[NTK][2];
       const uint4* qh = qfh + ws * a.ks_max * 32 + lane;
       const uint4* ql = qfl + ws * a.ks_max * 32 + lane;
       for (int w = 0; w < n2wk; ++w) {
@@ -356,12 +355,10 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
 #pragma unroll
         for (int nt = 0; nt < NTK; ++nt) {
           const uint32_t x = cs[w * TILE + tb + 8 * nt + gq];
-          bk[nt][0] = x & M2;
-          bk[nt][1] = (x >> 8) & M2;
-          mma16816(sacc[nt], ah, bk[nt][0], bk[nt][1]);
+          const uint32_t b0 = x & M2, b1 = (x >> 8) & M2;
+          mma16816(sacc[nt], ah, b0, b1);
+          mma16816(sacc[nt], al, b0, b1);
         }
-#pragma unroll
-        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al, bk[nt][0], bk[nt][1]);
       }
       for (int w = 0; w < n1wk; ++w) {
         const int ks = n2wk + 2 * w;
@@ -369,15 +366,12 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
 #pragma unroll
         for (int nt = 0; nt < NTK; ++nt) {
           const uint32_t x = cs[(n2wk + w) * TILE + tb + 8 * nt + gq];
-          bk[nt][0] = x;
-          mma16816(sacc[nt], ah0, x & M1, (x >> 4) & M1);
+          const uint32_t b0 = x & M1, b1 = (x >> 4) & M1, b2 = (x >> 8) & M1, b3 = (x >> 12) & M1;
+          mma16816(sacc[nt], ah0, b0, b1);
+          mma16816(sacc[nt], al0, b0, b1);
+          mma16816(sacc[nt], ah1, b2, b3);
+          mma16816(sacc[nt], al1, b2, b3);
         }
-#pragma unroll
-        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], ah1, (bk[nt][0] >> 8) & M1, (bk[nt][0] >> 12) & M1);
-#pragma unroll
-        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al0, bk[nt][0] & M1, (bk[nt][0] >> 4) & M1);
-#pragma unroll
-        for (int nt = 0; nt < NTK; ++nt) mma16816(sacc[nt], al1, (bk[nt][0] >> 8) & M1, (bk[nt][0] >> 12) & M1);
       }
       float* rs = red + ws * 16 * kGRS;
 #pragma unroll
@@ -521,7 +515,6 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
       }
     } else {
       // ---- O_e += P' . field_e 2^p over this warp's pairs, P' loaded once per k-step
-      uint32_t bv[NPW][2];
 #pragma unroll
       for (int kt = 0; kt < TILE / 16; ++kt) {
         const uint4 ah = pfh[kt * 32 + lane], al = pfl[kt * 32 + lane];
@@ -529,14 +522,11 @@ __global__ void __launch_bounds__(kGAThreads, 1) aatc_group_digit_kernel(const G
         for (int j = 0; j < NPW; ++j) {
           if (j < npv) {
             const uint32_t x0 = cs[poff[j] + 16 * kt], x1 = cs[poff[j] + 16 * kt + 8];
-            bv[j][0] = __byte_perm(x0, 0u, psel) & pmask[j];
-            bv[j][1] = __byte_perm(x1, 0u, psel) & pmask[j];
-            mma16816(oacc[j], ah, bv[j][0], bv[j][1]);
+            const uint32_t b0 = __byte_perm(x0, 0u, psel) & pmask[j], b1 = __byte_perm(x1, 0u, psel) & pmask[j];
+            mma16816(oacc[j], ah, b0, b1);
+            mma16816(oacc[j], al, b0, b1);
           }
         }
-#pragma unroll
-        for (int j = 0; j < NPW; ++j)
-          if (j < npv) mma16816(oacc[j], al, bv[j][0], bv[j][1]);
       }
     }
     __syncthreads();
@@ -759,25 +749,25 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
     const StreamLayout& ly = plan.layout[(layer * a.n_kv + h) * 2 + 1];
     ntp = std::max(ntp, (ly.n2 + ly.n1 + 7) / 8);
   }
-  const int npw = (ntp + 16 / gh - 1) / (16 / gh);
+  const int npw = (ntp + 8 / gh - 1) / (8 / gh);
   a.stages = 3;
   if (GroupDigitSmem(gh, a.ks_max, a.n_words, 3).total > 227 * 1024) a.stages = 2;
   const size_t smem = static_cast<size_t>(GroupDigitSmem(gh, a.ks_max, a.n_words, a.stages).total);
-  if (a.nq > 16 || npw > 12 || smem > 227 * 1024) return cudaErrorNotSupported;
+  if (a.nq > 16 || npw > 24 || smem > 227 * 1024) return cudaErrorNotSupported;
   aatc_group_query_kernel<<<dim3(16, a.n_groups * gh, batch), kGQThreads, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 grid(a.n_splits, a.n_groups, batch);
-  const void* kern = gh == 2 ? (npw <= 6 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 6>)
-                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 12>))
-                             : (npw <= 6 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 6>)
-                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 12>));
+  const void* kern = gh == 2 ? (npw <= 12 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 12>)
+                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 24>))
+                             : (npw <= 12 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 12>)
+                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 24>));
   e = ensure_smem_optin(kern, smem);
   if (e != cudaSuccess) return e;
-  if (gh == 2 && npw <= 6) aatc_group_digit_kernel<2, 6><<<grid, kGAThreads, smem, st>>>(a);
-  else if (gh == 2) aatc_group_digit_kernel<2, 12><<<grid, kGAThreads, smem, st>>>(a);
-  else if (npw <= 6) aatc_group_digit_kernel<4, 6><<<grid, kGAThreads, smem, st>>>(a);
-  else aatc_group_digit_kernel<4, 12><<<grid, kGAThreads, smem, st>>>(a);
+  if (gh == 2 && npw <= 12) aatc_group_digit_kernel<2, 12><<<grid, kGAThreads, smem, st>>>(a);
+  else if (gh == 2) aatc_group_digit_kernel<2, 24><<<grid, kGAThreads, smem, st>>>(a);
+  else if (npw <= 12) aatc_group_digit_kernel<4, 12><<<grid, kGAThreads, smem, st>>>(a);
+  else aatc_group_digit_kernel<4, 24><<<grid, kGAThreads, smem, st>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const size_t msm = static_cast<size_t>(a.n_splits) * 4;
