@@ -537,8 +537,8 @@ def group_timing(aatc, device, g_h=4, n_calls=64, reps=3, enc_iters=6, n_copies=
                       "frac_of_measured_hbm": round(dec_gbs / peak, 4),
                       "workspace_bytes": plan.workspace_bytes(B, T)},
            "roofline": {"bound": "hbm", "achieved": round(dec_gbs, 2), "peak": peak, "unit": "GB/s",
-                        "frac": round(dec_gbs / peak, 4), "traffic": None,
-                        "kernel": "one group decode call (codes + query + attention + merge kernels)",
+                        "frac": round(dec_gbs / peak, 4), "traffic": _traffic("decode_groups"),
+                        "kernel": "one group decode call (query + digit attention + merge kernels)",
                         "peak_source": f"{kind} hbm_gbs (MEASURED_PEAKS.json)"},
            "planner_seconds": round(plan_s, 2),
            "timing": f"encode: {enc_iters} calls rotating over {n_copies} caches; decode: {n_calls}-call CUDA graph "
@@ -1221,6 +1221,29 @@ def run_profile_once(args):
     print(json.dumps({"profile_once": cfg.name, "decode_bytes": decode_bytes(plan, cfg, B, T)}))
 
 
+def run_profile_groups():
+    """Minimal launch sequence of the head-group path for ncu captures: the Llama-shaped layer
+    with two groups of four kv-heads, one encode and two decodes."""
+    import torch
+    import paper_2608_14191_gb300 as aatc
+    from paper_2608_14191_gb300 import build as bld
+    bld.build()
+    aatc.load()
+    dev = torch.device("cuda", 0)
+    cfg = W.CONFIGS["llama_layer"]
+    plan, _ = group_plan_for(aatc, cfg, 4)
+    T = cfg.n_ctx
+    kd, vd = W.kv_device(cfg, 0, 1, T, dev)
+    qs = W.queries_device(cfg, 0, 1, 2, dev)
+    cache = plan.new_cache(1, T, dev)
+    aatc.encode(plan, 0, kd, vd, cache, 0, T)
+    for i in range(2):
+        aatc.decode_attention(plan, 0, qs[i], cache, T, T)
+    torch.cuda.synchronize()
+    assert plan.device_error() == 0
+    print(json.dumps({"profile_groups": "llama layer, 2 groups x 4 kv-heads, 32768 tokens"}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -1234,6 +1257,7 @@ def main():
     ap.add_argument("--profile-once", action="store_true", help="one encode + two decodes, for ncu")
     ap.add_argument("--profile-hidden", action="store_true", help="one encode from hidden states, for ncu")
     ap.add_argument("--profile-prefill", action="store_true", help="one Qwen-shaped prefill at batch 2, for ncu")
+    ap.add_argument("--profile-groups", action="store_true", help="one head-group encode + two decodes, for ncu")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -1247,6 +1271,8 @@ def main():
         aatc.load()
         hidden_encode_timing(aatc, torch.device("cuda", 0), iters=0, warmup=1)
         print(json.dumps({"profile_hidden": "llama layer input, d_model 4096, 32768 tokens"}))
+    elif args.profile_groups:
+        run_profile_groups()
     elif args.profile_prefill:
         import torch
         import paper_2608_14191_gb300 as aatc

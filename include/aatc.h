@@ -337,7 +337,12 @@ aatc_status_t aatc_decode_workspace_bytes(aatc_plan_t plan, int32_t batch, int32
  *   out       : device fp32 [batch][n_q_heads][128]
  *   workspace : device, >= aatc_decode_workspace_bytes(batch, n_ctx), contents ignored
  * Errors: AATC_ERR_INVALID_ARG (n_ctx < 1 ...), AATC_ERR_CAPACITY (n_ctx > max_tokens),
- * AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (group > 8), AATC_ERR_CUDA.
+ * AATC_ERR_WORKSPACE, AATC_ERR_UNSUPPORTED (group > 8; or a layer whose record tables exceed what
+ * the kernels hold: more than 2048 record entries per stream, per-kv-head tables beyond one SM's
+ * 227 KB of shared memory, and for head-group plans more than 24 value tiles of 8 entries per
+ * warp -- 48 per value slice at g_h = 4, 96 at g_h = 2 -- or score fragments plus a two-stage
+ * record ring beyond 227 KB, about 5 bits on average at g_h = 4; all refused before any launch),
+ * AATC_ERR_CUDA.
  */
 aatc_status_t aatc_decode_attention(aatc_plan_t plan, int32_t layer, const void* q,
                                     const void* cache, int32_t batch, int32_t n_ctx,

@@ -19,7 +19,9 @@ thread_local int32_t g_last_cuda_error = 0;
 aatc_status_t cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return AATC_OK;
   g_last_cuda_error = static_cast<int32_t>(e);
-  return AATC_ERR_CUDA;
+  // the launchers answer cudaErrorNotSupported, before any launch, for a shape their kernels do
+  // not implement (record tables beyond one SM's shared memory, more value tiles than a warp holds)
+  return e == cudaErrorNotSupported ? AATC_ERR_UNSUPPORTED : AATC_ERR_CUDA;
 }
 
 aatc::Plan* as_plan(aatc_plan_t p) {

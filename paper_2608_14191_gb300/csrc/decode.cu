@@ -1827,6 +1827,9 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
   a.qfrag = reinterpret_cast<uint4*>(static_cast<char*>(ws) + wsl.qfrag_off);
   a.qcorr = reinterpret_cast<float*>(static_cast<char*>(ws) + wsl.qcorr_off);
   if (plan.n_entries > kMaxEntries) return cudaErrorNotSupported;
+  // every shape refusal comes before the first launch of the call
+  const size_t msm = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
+  if (msm > 227 * 1024) return cudaErrorNotSupported;
   cudaError_t e = cudaSuccess;
   if (fk) {
     const int wu = n2w + n1w, nks = n2w + 2 * n1w;
@@ -1843,8 +1846,6 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     const unsigned n_cta = static_cast<unsigned>(static_cast<long>(sp.n_splits) * a.n_kv * batch);
     e = launch_pdl(fk, dim3(n_cta), dim3(128 * wg), smem, st, a);
     if (e != cudaSuccess) return e;
-    const size_t msm = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
-    if (msm > 227 * 1024) return cudaErrorNotSupported;
     e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msm);
     if (e != cudaSuccess) return e;
     return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msm, st, a);
@@ -1857,21 +1858,19 @@ cudaError_t launch_decode(const Plan& plan, int layer, const void* q, const void
     n_ks = std::max(n_ks, lk.n2 / 16 + 2 * ((lk.n1 + 31) / 32));
     n_jobs_v = std::max(n_jobs_v, lv.n2 / 16 + 2 * ((lv.n1 + 31) / 32));
   }
+  const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
+  const size_t smem = static_cast<size_t>(L.total);
+  const int jpw = (n_jobs_v + kWarps - 1) / kWarps;            // value M-tiles per warp
+  if (a.n_splits > 0 && (jpw > 12 || smem > 227 * 1024)) return cudaErrorNotSupported;
   if (a.n_splits > 0) {
     e = launch_pdl(aatc_decode_query_kernel, dim3(a.n_kv, batch, MAX_GROUP), dim3(kQThreads), 0, st, a);
     if (e != cudaSuccess) return e;
-    const SplitSmem L(n_ks, np, sp.split_len, plan.n_words, plan.n_entries);
-    const size_t smem = static_cast<size_t>(L.total);
-    const int jpw = (n_jobs_v + kWarps - 1) / kWarps;          // value M-tiles per warp
-    if (jpw > 12 || smem > 227 * 1024) return cudaErrorNotSupported;
     e = np == 1 ? launch_split_g<1>(a, batch, jpw, smem, st) : launch_split_g<2>(a, batch, jpw, smem, st);
     if (e != cudaSuccess) return e;
   }
-  const size_t msmem = 4 * (static_cast<size_t>(D) * D + kMWarps * D + D + static_cast<size_t>((a.n_full + 3) & ~3));
-  if (msmem > 227 * 1024) return cudaErrorNotSupported;
-  e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msmem);
+  e = ensure_smem_optin(reinterpret_cast<const void*>(aatc_decode_merge_kernel), msm);
   if (e != cudaSuccess) return e;
-  return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msmem, st, a);
+  return launch_pdl(aatc_decode_merge_kernel, dim3(a.n_q, batch), dim3(kMThreads), msm, st, a);
 }
 
 cudaError_t launch_dequant(const Plan& plan, int layer, const void* cache, int batch, int t0, int n, int max_tokens,
