@@ -727,7 +727,7 @@ __host__ __device__ constexpr int fused_entry_pitch(int n_entries) { return ((n_
 constexpr float kPScale = 32.0f;            // P' < 2^9 times 2^5: f16 operands below 2^14
 
 struct FusedSmem {
-  int bars, cnt, qf, qc, pf, cetab, etab, ketab, fold, ring, total;
+  int bars, cnt, qf, qc, pf, cetab, cw8, ketab, fold, ring, total;
   __host__ __device__ FusedSmem(int wu, int nks, int np, int wg, int n_entries, int n_stages) {
     const int gmax = 4 * np, warps = 4 * wg;
     int o = 0;
@@ -736,8 +736,8 @@ struct FusedSmem {
     qf = o;    o += nks * np * 32 * 8;                        // query B fragments [ks][p][lane]
     qc = o;    o += 2 * MAX_GROUP * 4 + D * 4;                // C_g, score scales; value offsets 2^(b_c - 1)
     pf = o;    o += warps * 2 * np * 32 * 8;                  // P' B fragments [warp][ks][p][lane]
-    cetab = o; o += D * 8 * 2;                                // value channel -> record entries
-    etab = o;  o = align16(o + n_entries * 2);                // value entry table
+    cetab = o; o += D * 8 * 2;                                // value channel -> its record entries (clamped)
+    cw8 = o;   o += D * 8 * 4;                                // 2^shift of those entries (0: none)
     ketab = o; o = align16(o + n_entries * 2);                // key entry table
     fold = o;  o += ((2 + wg) * gmax * D + 2 * warps * gmax) * 4;   // q, q', partial q' [wg]; reductions
     o = (o + 127) & ~127;
@@ -779,7 +779,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
   const uint2* qf = reinterpret_cast<const uint2*>(smb + L.qf);
   unsigned char* pfw = smb + L.pf + warp * (2 * NP * 32 * 8);
   const short* cetab = reinterpret_cast<const short*>(smb + L.cetab);
-  const short* etab = reinterpret_cast<const short*>(smb + L.etab);
+  const float* cw8 = reinterpret_cast<const float*>(smb + L.cw8);
   const short* ketab = reinterpret_cast<const short*>(smb + L.ketab);
   unsigned char* ring = smb + L.ring + wg * NS * kStage;
 
@@ -824,12 +824,15 @@ __global__ void __launch_bounds__(128 * WG, 1)
   // plan constants (never written by a kernel): the streams' entry tables, key channel constants
   // (the first 8 entries of each channel: all of them for widths up to 8, the only plans this
   // kernel is launched for)
-  for (int i = tid; i < D * 8; i += NT)
-    reinterpret_cast<short*>(smb + L.cetab)[i] = a.chan_ent[(static_cast<size_t>(sv) * D + (i >> 3)) * kChanEnt + (i & 7)];
-  for (int i = tid; i < a.n_entries; i += NT) {
-    reinterpret_cast<short*>(smb + L.etab)[i] = a.entry[static_cast<size_t>(sv) * a.n_entries + i];
-    reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
+  for (int i = tid; i < D * 8; i += NT) {
+    const int ce = a.chan_ent[(static_cast<size_t>(sv) * D + (i >> 3)) * kChanEnt + (i & 7)];
+    const int e = min(max(ce, 0), a.n_entries - 1);
+    reinterpret_cast<short*>(smb + L.cetab)[i] = static_cast<short>(e);
+    reinterpret_cast<float*>(smb + L.cw8)[i] =
+        ce >= 0 ? pow2i((a.entry[static_cast<size_t>(sv) * a.n_entries + e] >> 8) & 15) : 0.0f;
   }
+  for (int i = tid; i < a.n_entries; i += NT)
+    reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
   const int c = tid & (D - 1), part = tid >> 7;                 // channel, part of the fold (WG parts)
   // U_K rows of this thread's part of the fold: plan constants, requested before the wait
   constexpr int DR = D / WG, RR = DR < 64 ? DR : 64;
@@ -907,20 +910,16 @@ __global__ void __launch_bounds__(128 * WG, 1)
   __syncthreads();
   {
     float* qcw = reinterpret_cast<float*>(smb + L.qc);
-    float inv[GMAX];
-#pragma unroll
-    for (int q = 0; q < GMAX; ++q) {
+    if (tid < GMAX) {
+      const int q = tid;
       float cs = 0.0f, m = 0.0f;
 #pragma unroll
       for (int w = 0; w < 4; ++w) {                               // the four warps of part 0
         cs += fred[w * GMAX + q];
         m = fmaxf(m, fred[(NW + w) * GMAX + q]);
       }
-      inv[q] = m > 0.0f ? kOpMax / m : 0.0f;
-      if (tid == q) {
-        qcw[q] = q < G ? cs : 0.0f;
-        qcw[MAX_GROUP + q] = q < G && m > 0.0f ? m * (kDigitScale / kOpMax) : 0.0f;   // raw sum -> sum q' u
-      }
+      qcw[q] = q < G ? cs : 0.0f;
+      qcw[MAX_GROUP + q] = q < G && m > 0.0f ? m * (kDigitScale / kOpMax) : 0.0f;   // raw sum -> sum q' u
     }
     // lane t of k-step ks holds fields (k 2t, 2t+1, 2t+8, 2t+9) = D2 (t, t+8, t+4, t+12) of word
     // ks, or D1 bits (t, t+16, t+4, t+20) + 8 hs of word u for k-step ks = N2W + 2u + hs; the
@@ -928,6 +927,10 @@ __global__ void __launch_bounds__(128 * WG, 1)
     uint2* qfw = reinterpret_cast<uint2*>(smb + L.qf);
     for (int i = tid; i < NKS * 4 * GMAX; i += NT) {
       const int q = i % GMAX, tt = (i / GMAX) & 3, ks = i / (4 * GMAX);
+      float mq = 0.0f;                                            // largest |coefficient| of query q
+#pragma unroll
+      for (int w = 0; w < 4; ++w) mq = fmaxf(mq, fred[(NW + w) * GMAX + q]);
+      const float invq = mq > 0.0f ? kOpMax / mq : 0.0f;
       int f[4], base, lim;
       float s01, s89;
       if (ks < N2W) {
@@ -947,7 +950,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const int ce = f[k] < lim && q < G ? ketab[base + f[k]] : 0;
-        v[k] = f[k] < lim && q < G ? xq[q * D + (ce & 0xFF)] * inv[q] * pow2i(ce >> 8) * (k < 2 ? s01 : s89) : 0.0f;
+        v[k] = f[k] < lim && q < G ? xq[q * D + (ce & 0xFF)] * invq * pow2i(ce >> 8) * (k < 2 ? s01 : s89) : 0.0f;
       }
       uint32_t h01, l01, h89, l89;
       f16_split2(v[0], v[1], h01, l01);
@@ -1262,14 +1265,11 @@ __global__ void __launch_bounds__(128 * WG, 1)
   {
     const uint4 cev = *reinterpret_cast<const uint4*>(cetab + c * 8);
     const uint32_t cw4[4] = {cev.x, cev.y, cev.z, cev.w};
-    float w8[8];
+    const float4 wa = *reinterpret_cast<const float4*>(cw8 + c * 8), wb = *reinterpret_cast<const float4*>(cw8 + c * 8 + 4);
+    const float w8[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
     int e8[8];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {                            // entry k of channel c: short k of the row
-      const int ce = static_cast<short>(cw4[k >> 1] >> (16 * (k & 1)));
-      e8[k] = min(max(ce, 0), NE - 1);
-      w8[k] = ce >= 0 ? pow2i((etab[e8[k]] >> 8) & 15) : 0.0f;
-    }
+    for (int k = 0; k < 8; ++k) e8[k] = static_cast<int>(cw4[k >> 1] >> (16 * (k & 1))) & 0xFFFF;   // entry k of c
     const float off = reinterpret_cast<const float*>(smb + L.qc)[2 * MAX_GROUP + c];
     for (int q = part; q < G; q += WG) {
       float o = -off * tot[2 * GMAX + q];
@@ -1349,7 +1349,7 @@ __global__ void __launch_bounds__(kMThreads)
     for (int w = 1; w < kMWarps; ++w) m_f = fmaxf(m_f, red[0][w]);
     float lp = 0.0f;
     for (int t = tid; t < a.n_full; t += kMThreads) {
-      const float pw = exp2f(sf[t] - m_f);
+      const float pw = fast_exp2(sf[t] - m_f);
       sf[t] = pw;
       lp += pw;
     }
@@ -1398,12 +1398,12 @@ __global__ void __launch_bounds__(kMThreads)
 #pragma unroll
       for (int u = 0; u < 8; ++u) mc = fmaxf(mc, ml[u].x);
       if (mc > -INFINITY) {                          // else nothing attended so far: sums stay 0
-        const float r = exp2f(mw - mc);              // mw = -inf -> 0
+        const float r = fast_exp2(mw - mc);              // mw = -inf -> 0
         lw *= r;
         acc.x *= r; acc.y *= r; acc.z *= r; acc.w *= r;
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-          const float w = exp2f(ml[u].x - mc);
+          const float w = fast_exp2(ml[u].x - mc);
           lw = fmaf(w, ml[u].y, lw);
           acc.x = fmaf(w, v[u].x, acc.x);
           acc.y = fmaf(w, v[u].y, acc.y);
@@ -1423,18 +1423,18 @@ __global__ void __launch_bounds__(kMThreads)
     for (int w = 0; w < kMWarps; ++w) M = fmaxf(M, red[0][w]);
     if (M > -INFINITY)
 #pragma unroll
-      for (int w = 0; w < kMWarps; ++w) L = fmaf(exp2f(red[0][w] - M), red[1][w], L);
+      for (int w = 0; w < kMWarps; ++w) L = fmaf(fast_exp2(red[0][w] - M), red[1][w], L);
   }
   // ---- log-sum-exp merge of the two parts: out = (U_V (f o) a_p + o_f a_f) / (L a_p + l_f a_f)
   const float Mt = fmaxf(M, m_f);
-  const float ap = a.n_splits > 0 ? exp2f(M - Mt) : 0.0f;
-  const float af = a.n_full > 0 ? exp2f(m_f - Mt) : 0.0f;
+  const float ap = a.n_splits > 0 ? fast_exp2(M - Mt) : 0.0f;
+  const float af = a.n_full > 0 ? fast_exp2(m_f - Mt) : 0.0f;
   const float inv_den = 1.0f / fmaf(L, ap, l_f * af);
   if (tid < D) {
     float o = 0.0f;
     if (a.n_splits > 0 && M > -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < kMWarps; ++w) o = fmaf(exp2f(red[0][w] - M), osum[w * D + tid], o);
+      for (int w = 0; w < kMWarps; ++w) o = fmaf(fast_exp2(red[0][w] - M), osum[w * D + tid], o);
     }
     ohat[tid] = o * fv * ap;
   }
@@ -1443,10 +1443,10 @@ __global__ void __launch_bounds__(kMThreads)
   // out[d] = sum_c U_V[d][c] o_hat[c]: four threads per dimension, quarters of c
   {
     const int d = tid & (D - 1), qtr = tid >> 7;
-    float r = 0.0f;
-#pragma unroll 16
-    for (int c = qtr * 32; c < qtr * 32 + 32; ++c) r = fmaf(ut_s[c * D + d], ohat[c], r);
-    osum[qtr * D + d] = r;
+    float r4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+    for (int c = 0; c < 32; ++c) r4[c & 3] = fmaf(ut_s[(qtr * 32 + c) * D + d], ohat[qtr * 32 + c], r4[c & 3]);
+    osum[qtr * D + d] = (r4[0] + r4[1]) + (r4[2] + r4[3]);
   }
   __syncthreads();
   if (tid < D)
