@@ -758,15 +758,18 @@ cudaError_t launch_group_decode(const Plan& plan, int layer, const void* q, cons
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 grid(a.n_splits, a.n_groups, batch);
+  // pairs per warp: 12, 16 (g_h = 4 at ~2.75 bits: up to 32 value tiles per slice) or 24
   const void* kern = gh == 2 ? (npw <= 12 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 12>)
-                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 24>))
+                                          : reinterpret_cast<const void*>(aatc_group_digit_kernel<2, 24>))
                              : (npw <= 12 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 12>)
-                                         : reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 24>));
+                                : npw <= 16 ? reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 16>)
+                                            : reinterpret_cast<const void*>(aatc_group_digit_kernel<4, 24>));
   e = ensure_smem_optin(kern, smem);
   if (e != cudaSuccess) return e;
   if (gh == 2 && npw <= 12) aatc_group_digit_kernel<2, 12><<<grid, kGAThreads, smem, st>>>(a);
   else if (gh == 2) aatc_group_digit_kernel<2, 24><<<grid, kGAThreads, smem, st>>>(a);
   else if (npw <= 12) aatc_group_digit_kernel<4, 12><<<grid, kGAThreads, smem, st>>>(a);
+  else if (npw <= 16) aatc_group_digit_kernel<4, 16><<<grid, kGAThreads, smem, st>>>(a);
   else aatc_group_digit_kernel<4, 24><<<grid, kGAThreads, smem, st>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
