@@ -129,6 +129,29 @@ def test_group_plan_refusals(aatc):
     assert e.value.status == 5
 
 
+def test_group_decode_refuses_oversized_records(aatc):
+    """A group plan whose slices need more value tiles per warp than the decode holds (7 bits on
+    every channel of a g_h = 4 group: 3 base-4 digits and one bit per channel, 512 record entries
+    per slice, 32 value tiles per warp) is refused with AATC_ERR_UNSUPPORTED before any launch;
+    the output keeps its contents."""
+    g_h, n_kv, n_q, T = 4, 4, 16, 256
+    n = 128 * g_h
+    basis = np.broadcast_to(np.eye(n, dtype=np.float32), (1, 1, 2, n, n)).copy()
+    bits = np.full((1, 1, 2, n), 7, np.uint8)
+    scales = np.ones((1, 1, 2, n), np.float32)
+    plan = aatc.GroupPlan(aatc.dims(1, n_kv, n_q), g_h, basis, bits, scales)
+    cache = plan.new_cache(1, T, DEV)
+    cache.zero_()
+    q = torch.zeros((1, n_q, 128), dtype=torch.bfloat16, device=DEV)
+    out = torch.full((1, n_q, 128), 3.0, dtype=torch.float32, device=DEV)
+    with pytest.raises(aatc.AatcError) as e:
+        aatc.decode_attention(plan, 0, q, cache, T, T, out=out)
+    assert e.value.status == 5
+    torch.cuda.synchronize()
+    assert bool(torch.all(out == 3.0))
+    assert plan.device_error() == 0
+
+
 def test_group_llama_layer_full_size(aatc):
     """The Llama-shaped layer with the paper's Llama grouping (two groups of four kv-heads, 512
     channels per group stream), 32768 tokens: every code of every slice against the oracle's
