@@ -739,7 +739,7 @@ struct FusedSmem {
     cetab = o; o += D * 8 * 2;                                // value channel -> its record entries (clamped)
     cw8 = o;   o += D * 8 * 4;                                // 2^shift of those entries (0: none)
     ketab = o; o = align16(o + n_entries * 2);                // key entry table
-    fold = o;  o += (gmax * (D + 4 * wg) + gmax * D + 2 * warps * gmax) * 4;   // q (padded parts), q'; reductions
+    fold = o;  o += ((2 + wg) * gmax * D + 2 * warps * gmax) * 4;   // q, q', partial q' [wg]; reductions
     o = (o + 127) & ~127;
     ring = o;
     const int rings = wg * n_stages * fused_stage_bytes(wu);
@@ -833,70 +833,71 @@ __global__ void __launch_bounds__(128 * WG, 1)
   }
   for (int i = tid; i < a.n_entries; i += NT)
     reinterpret_cast<short*>(smb + L.ketab)[i] = a.entry[static_cast<size_t>(sk) * a.n_entries + i];
-  const int c = tid & (D - 1), part = tid >> 7;                 // epilogue: value channel, query parity
-  // fold: warp w owns the CPW channels CPW w .. CPW w + CPW - 1; lane = (channel, part of the 128
-  // dims), so a channel's dot products finish with shuffles inside the warp.  U_K rows of the
-  // lane's part: plan constants, requested before the wait.
-  constexpr int CPW = D / NW, DR = D / WG, QP = WG * (DR + 4);  // qv rows: parts padded by 4 floats
-  static_assert(CPW * WG == 32 && DR <= 64 && (GMAX * D) % NT == 0, "fold lane mapping");
-  const int fch = CPW * warp + (lane % CPW), fpart = lane / CPW;
-  const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(fpart * DR) * D + fch;
-  float u0[DR];
+  const int c = tid & (D - 1), part = tid >> 7;                 // channel, part of the fold (WG parts)
+  // U_K rows of this thread's part of the fold: plan constants, requested before the wait
+  constexpr int DR = D / WG, RR = DR < 64 ? DR : 64;
+  const float* uk = a.u32 + static_cast<size_t>(sk) * D * D + static_cast<size_t>(part * DR) * D + c;
+  float u0[RR];
 #pragma unroll
-  for (int k = 0; k < DR; ++k) u0[k] = __ldg(uk + k * D);
-  const float fk = a.f[sk * D + fch];
-  const float offk = a.enc[sk * D + fch].off;                   // 2^(b_c - 1), 0 if b_c = 0
+  for (int k = 0; k < RR; ++k) u0[k] = __ldg(uk + k * D);
+  const float fk = a.f[sk * D + c];
+  const float offk = a.enc[sk * D + c].off;                     // 2^(b_c - 1), 0 if b_c = 0
   if (tid < D) reinterpret_cast<float*>(smb + L.qc)[2 * MAX_GROUP + tid] = a.enc[sv * D + tid].off;
   const StreamLayout lk = a.lay[sk];
   if (tid < WG * NS) reinterpret_cast<int*>(smb + L.cnt)[tid] = 0;
   // everything below may read what the preceding grid in the stream wrote (cache, q, workspace)
   ptx::grid_dependency_wait();
-  constexpr int QPT = GMAX * D / NT;             // query values per thread
-  float qr[QPT];
-#pragma unroll
-  for (int j = 0; j < QPT; ++j) {                // the query loads go out before the first tile's copies
-    const int i = tid + j * NT, gq = i >> 7;
-    qr[j] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + (i & (D - 1))]) : 0.0f;
-  }
   if (leader && n_j > 0) issue(0, 0);          // first tile now, the rest of the ring after the fold
 
   // ---- query rotation and fold, while the first tiles are in flight:
   //   q'_{g,c} = (U_K^T q_g)_c f^K_c log2(e) / sqrt(128),  C_g = sum_c q'_{g,c} 2^(b_c - 1),
   // and the score B fragments: q'_{g,c(e)} 2^shift(e) per record entry e, scaled so the largest
   // is 2^14, as f16 hi / lo; columns 2 gs (hi) and 2 gs + 1 (lo) of query group p for query 4p + gs
-  float* qv = reinterpret_cast<float*>(smb + L.fold);           // [GMAX][WG][DR + 4] q
-  float* xq = qv + GMAX * QP;                                   // [GMAX][128] q'
-  float* fred = xq + GMAX * D;                                  // [2][NW][GMAX]
-#pragma unroll
-  for (int j = 0; j < QPT; ++j) {
-    const int i = tid + j * NT, d = i & (D - 1);
-    qv[(i >> 7) * QP + (d / DR) * (DR + 4) + d % DR] = qr[j];
+  float* qv = reinterpret_cast<float*>(smb + L.fold);           // [GMAX][128] q
+  float* xq = qv + GMAX * D;                                    // [GMAX][128] q'
+  float* xpart = xq + GMAX * D;                                 // [WG][GMAX][128] partial U_K^T q
+  float* fred = xpart + WG * GMAX * D;                          // [2][NW][GMAX]
+  for (int i = tid; i < GMAX * D; i += NT) {
+    const int gq = i >> 7;
+    qv[i] = gq < G ? __bfloat162float(a.q[(static_cast<size_t>(b) * a.n_q + head * G + gq) * D + (i & (D - 1))]) : 0.0f;
   }
   __syncthreads();
   {
-    // lane (channel fch, part fpart) sums dimensions [fpart DR, (fpart + 1) DR) of every query
+    // part p of the thread sums dimensions [p D / WG, (p + 1) D / WG), RR rows of U_K in flight
     float acc[GMAX];
 #pragma unroll
     for (int q = 0; q < GMAX; ++q) acc[q] = 0.0f;
+#pragma unroll 1
+    for (int r = 0; r < DR / RR; ++r) {
+      float u[RR];
 #pragma unroll
-    for (int k4 = 0; k4 < DR / 4; ++k4)
+      for (int k = 0; k < RR; ++k) u[k] = r == 0 ? u0[k] : __ldg(uk + (RR * r + k) * D);
 #pragma unroll
-      for (int q = 0; q < GMAX; ++q) {
-        const float4 qq = *reinterpret_cast<const float4*>(qv + q * QP + fpart * (DR + 4) + 4 * k4);
-        acc[q] = fmaf(u0[4 * k4], qq.x, acc[q]);
-        acc[q] = fmaf(u0[4 * k4 + 1], qq.y, acc[q]);
-        acc[q] = fmaf(u0[4 * k4 + 2], qq.z, acc[q]);
-        acc[q] = fmaf(u0[4 * k4 + 3], qq.w, acc[q]);
-      }
+      for (int k4 = 0; k4 < RR / 4; ++k4)
+#pragma unroll
+        for (int q = 0; q < GMAX; ++q) {
+          const float4 qq = *reinterpret_cast<const float4*>(qv + q * D + part * DR + RR * r + 4 * k4);
+          acc[q] = fmaf(u[4 * k4], qq.x, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 1], qq.y, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 2], qq.z, acc[q]);
+          acc[q] = fmaf(u[4 * k4 + 3], qq.w, acc[q]);
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < GMAX; ++q) xpart[(part * GMAX + q) * D + c] = acc[q];
+  }
+  __syncthreads();
+  if (part == 0) {
 #pragma unroll
     for (int q = 0; q < GMAX; ++q) {
+      float sum = 0.0f;
 #pragma unroll
-      for (int o = CPW; o < 32; o <<= 1) acc[q] += __shfl_xor_sync(0xffffffffu, acc[q], o);   // over the parts
-      const float x = acc[q] * fk * (kLog2e * 0.08838834764831845f);
-      if (fpart == 0) xq[q * D + fch] = x;
-      float cr = x * offk, mx = fabsf(x) * offk;                  // largest |coefficient| of the channel
+      for (int p2 = 0; p2 < WG; ++p2) sum += xpart[(p2 * GMAX + q) * D + c];
+      const float x = sum * fk * (kLog2e * 0.08838834764831845f);
+      xq[q * D + c] = x;
+      float cr = x * offk, mx = fabsf(x) * offk;                  // largest |coefficient| of c
 #pragma unroll
-      for (int o = 1; o < CPW; o <<= 1) {                         // over the warp's channels
+      for (int o = 16; o > 0; o >>= 1) {
         cr += __shfl_xor_sync(0xffffffffu, cr, o);
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
       }
@@ -913,7 +914,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
       const int q = tid;
       float cs = 0.0f, m = 0.0f;
 #pragma unroll
-      for (int w = 0; w < NW; ++w) {                              // the warps' channel groups
+      for (int w = 0; w < 4; ++w) {                               // the four warps of part 0
         cs += fred[w * GMAX + q];
         m = fmaxf(m, fred[(NW + w) * GMAX + q]);
       }
@@ -928,7 +929,7 @@ __global__ void __launch_bounds__(128 * WG, 1)
       const int q = i % GMAX, tt = (i / GMAX) & 3, ks = i / (4 * GMAX);
       float mq = 0.0f;                                            // largest |coefficient| of query q
 #pragma unroll
-      for (int w = 0; w < NW; ++w) mq = fmaxf(mq, fred[(NW + w) * GMAX + q]);
+      for (int w = 0; w < 4; ++w) mq = fmaxf(mq, fred[(NW + w) * GMAX + q]);
       const float invq = mq > 0.0f ? kOpMax / mq : 0.0f;
       int f[4], base, lim;
       float s01, s89;
